@@ -1,0 +1,180 @@
+"""Seeded synthetic inputs shaped like the SENSE workloads.
+
+This module only draws random inputs; it holds no step of the method.  Both
+the CUDA path and the CPU oracle receive the same tensors from here.
+
+Recipes (all seeded; per-chunk seeds make large stores reproducible chunk by
+chunk, independent of the device that draws them):
+
+* keys: ``n_clusters`` centroids uniform on the unit sphere; each key picks a
+  centroid uniformly and adds Gaussian noise, then is put back on the unit
+  sphere and stored as bf16.  Noise reading "A" draws N(0, sigma^2/d) per
+  coordinate (noise vector norm ~ sigma); reading "B" draws N(0, sigma^2)
+  per coordinate.
+* queries: a uniformly chosen key plus Gaussian noise (same readings), back
+  on the unit sphere, as bf16; the source key index is returned.
+* lattice keys/queries: entries from {-3..3} * 2^-6 (exact in bf16, and all
+  dot products are exact in fp32), used to make ties frequent.
+* spans: int32 token ids, uniform in [0, vocab) or Zipf(s) by rank
+  (P(r) proportional to (r+1)^-s), drawn by inverse CDF.
+* gate inputs: fp32 logits N(0, std^2) per tree node row, bf16 hidden states
+  N(0, 1); ``plant_gate_rows`` raises chosen child tokens in their parent's
+  row so that exact-match and top-k paths are exercised.
+"""
+from __future__ import annotations
+
+import torch
+
+CHUNK_ROWS = 65536
+
+
+def _gen(device, seed: int) -> torch.Generator:
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed) & ((1 << 63) - 1))
+    return g
+
+
+def _sub_seed(seed: int, stream: int, chunk: int = 0) -> int:
+    return (int(seed) * 1000003 + stream * 7919 + chunk * 104729) & ((1 << 62) - 1)
+
+
+def _unit_rows(x: torch.Tensor) -> torch.Tensor:
+    # Put draws on the unit sphere (this shapes the input distribution).
+    return x / x.norm(dim=1, keepdim=True).clamp_min(1e-30)
+
+
+def centroids(n_clusters: int, d: int, seed: int = 0, device="cpu") -> torch.Tensor:
+    g = _gen(device, _sub_seed(seed, 1))
+    c = torch.randn(n_clusters, d, generator=g, device=device, dtype=torch.float32)
+    return _unit_rows(c)
+
+
+def clustered_unit_keys(n: int, d: int, n_clusters: int, sigma: float = 0.3,
+                        seed: int = 0, device="cpu", reading: str = "A",
+                        out: torch.Tensor | None = None) -> torch.Tensor:
+    """bf16 [n, d] keys drawn around ``n_clusters`` unit centroids."""
+    c = centroids(n_clusters, d, seed, device)
+    scale = sigma / (d ** 0.5) if reading == "A" else sigma
+    if out is None:
+        out = torch.empty(n, d, dtype=torch.bfloat16, device=device)
+    for ci, lo in enumerate(range(0, n, CHUNK_ROWS)):
+        hi = min(n, lo + CHUNK_ROWS)
+        g = _gen(device, _sub_seed(seed, 2, ci))
+        a = torch.randint(0, n_clusters, (hi - lo,), generator=g, device=device)
+        e = torch.randn(hi - lo, d, generator=g, device=device, dtype=torch.float32)
+        x = c[a] + scale * e
+        out[lo:hi] = _unit_rows(x).to(torch.bfloat16)
+        del e, x
+    return out
+
+
+def noisy_queries(keys: torch.Tensor, q: int, noise: float = 0.05, seed: int = 0,
+                  reading: str = "A"):
+    """(bf16 [q, d] queries, int64 [q] source key index)."""
+    n, d = keys.shape
+    dev = keys.device
+    g = _gen(dev, _sub_seed(seed, 3))
+    src = torch.randint(0, n, (q,), generator=g, device=dev)
+    scale = noise / (d ** 0.5) if reading == "A" else noise
+    e = torch.randn(q, d, generator=g, device=dev, dtype=torch.float32)
+    x = keys[src].float() + scale * e
+    return _unit_rows(x).to(torch.bfloat16), src
+
+
+def lattice_rows(n: int, d: int, seed: int = 0, device="cpu") -> torch.Tensor:
+    """bf16 [n, d] with entries in {-3..3} * 2^-6 (exact in bf16)."""
+    out = torch.empty(n, d, dtype=torch.bfloat16, device=device)
+    for ci, lo in enumerate(range(0, n, CHUNK_ROWS)):
+        hi = min(n, lo + CHUNK_ROWS)
+        g = _gen(device, _sub_seed(seed, 4, ci))
+        v = torch.randint(-3, 4, (hi - lo, d), generator=g, device=device)
+        out[lo:hi] = (v.float() * (2.0 ** -6)).to(torch.bfloat16)
+    return out
+
+
+def gaussian_rows_f32(n: int, d: int, seed: int = 0, device="cpu",
+                      std: float = 1.0) -> torch.Tensor:
+    g = _gen(device, _sub_seed(seed, 5))
+    return std * torch.randn(n, d, generator=g, device=device, dtype=torch.float32)
+
+
+def spans_uniform(n: int, m: int, vocab: int, seed: int = 0, device="cpu") -> torch.Tensor:
+    out = torch.empty(n, m, dtype=torch.int32, device=device)
+    for ci, lo in enumerate(range(0, n, CHUNK_ROWS * 16)):
+        hi = min(n, lo + CHUNK_ROWS * 16)
+        g = _gen(device, _sub_seed(seed, 6, ci))
+        out[lo:hi] = torch.randint(0, vocab, (hi - lo, m), generator=g, device=device,
+                                   dtype=torch.int32)
+    return out
+
+
+def zipf_cdf(vocab: int, s: float = 1.1, device="cpu") -> torch.Tensor:
+    r = torch.arange(1, vocab + 1, dtype=torch.float64, device=device)
+    w = r.pow(-s)
+    c = torch.cumsum(w, 0)
+    return c / c[-1]
+
+
+def spans_zipf(n: int, m: int, vocab: int, s: float = 1.1, seed: int = 0,
+               device="cpu") -> torch.Tensor:
+    """int32 [n, m] token ids; token id = frequency rank, P(r) ~ (r+1)^-s."""
+    cdf = zipf_cdf(vocab, s, device)
+    out = torch.empty(n, m, dtype=torch.int32, device=device)
+    for ci, lo in enumerate(range(0, n, CHUNK_ROWS * 16)):
+        hi = min(n, lo + CHUNK_ROWS * 16)
+        g = _gen(device, _sub_seed(seed, 7, ci))
+        u = torch.rand(hi - lo, m, generator=g, device=device, dtype=torch.float64)
+        t = torch.searchsorted(cdf, u.reshape(-1), right=True).clamp_max(vocab - 1)
+        out[lo:hi] = t.reshape(hi - lo, m).to(torch.int32)
+    return out
+
+
+def gate_logits(q: int, rows: int, vocab: int, std: float = 3.0, seed: int = 0,
+                device="cpu", out: torch.Tensor | None = None) -> torch.Tensor:
+    """fp32 [q, rows, vocab] i.i.d. N(0, std^2)."""
+    if out is None:
+        out = torch.empty(q, rows, vocab, dtype=torch.float32, device=device)
+    for qi in range(q):
+        g = _gen(device, _sub_seed(seed, 8, qi))
+        out[qi].normal_(0.0, std, generator=g)
+    return out
+
+
+def gate_hidden(q: int, rows: int, d: int, seed: int = 0, device="cpu") -> torch.Tensor:
+    g = _gen(device, _sub_seed(seed, 9))
+    return torch.randn(q, rows, d, generator=g, device=device,
+                       dtype=torch.float32).to(torch.bfloat16)
+
+
+def plant_gate_rows(root_logits: torch.Tensor, node_logits: torch.Tensor,
+                    tokens: torch.Tensor, parent: torch.Tensor,
+                    num_nodes: torch.Tensor, seed: int = 0,
+                    p_top: float = 0.6, p_near: float = 0.15,
+                    p_sharp: float = 0.2) -> None:
+    """In-place structure for gate tests (CPU tensors).
+
+    For each tree node n, the row that predicts it is its parent's row (the
+    root row for depth 0).  A seeded fraction ``p_top`` of nodes gets +20 on
+    its token in that row (usually the argmax afterwards), ``p_near`` gets
+    its token set just below the row maximum (a near-top alternative), and a
+    fraction ``p_sharp`` of all rows is multiplied by 10 (low entropy).
+    """
+    g = _gen("cpu", _sub_seed(seed, 10))
+    qn, cap, _ = node_logits.shape
+    for q in range(qn):
+        nn = int(num_nodes[q])
+        u = torch.rand(nn, generator=g, dtype=torch.float64)
+        for n in range(nn):
+            p = int(parent[q, n])
+            row = root_logits[q] if p < 0 else node_logits[q, p]
+            t = int(tokens[q, n])
+            if u[n] < p_top:
+                row[t] += 20.0
+            elif u[n] < p_top + p_near:
+                row[t] = row.max() - 0.05 - 0.5 * float(torch.rand(1, generator=g))
+        sharp = torch.rand(cap + 1, generator=g) < p_sharp
+        if sharp[0]:
+            root_logits[q] *= 10.0
+        for n in range(nn):
+            if sharp[n + 1]:
+                node_logits[q, n] *= 10.0
