@@ -1,0 +1,405 @@
+"""Benchmark of the SENSE drafting hot path on GB300.
+
+One step = one pass of the whole path for one batch of queries on a seeded
+synthetic workload resident in HBM: exact top-k retrieval over the bf16
+datastore, span gather, loose-trie draft tree and soft-gated evaluation.
+
+Default workload (LLaMA-7B-shaped store): n = 1,048,576 keys, d = 4096 bf16
+(8.6 GB), 1 query per step (512 distinct queries, each a perturbed key),
+k = 32, spans of 16 Zipf(1.1) tokens over a 32,000-token vocabulary, tree
+capped at 64 nodes, gate on fp32 N(0, 3^2) logits for every tree node with the
+paper's defaults (gamma 0.05, top-3, window 6).
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle
+on bounded samples of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+WORKLOADS = {
+    # name: n, d, q, k, m, vocab, cap, clusters, zipf
+    "llama7b_1m": dict(n=1048576, d=4096, q=1, k=32, m=16, vocab=32000, cap=64,
+                       clusters=1024, zipf=True, distinct=512),
+    "tiny_4k": dict(n=4096, d=4096, q=8, k=8, m=8, vocab=32000, cap=64, clusters=64,
+                    zipf=False, distinct=8),
+    "qwen7b_4m": dict(n=4194304, d=3584, q=16, k=64, m=16, vocab=152064, cap=128,
+                      clusters=4096, zipf=True, distinct=64),
+    "llama70b_8m": dict(n=8388608, d=8192, q=1, k=64, m=16, vocab=128256, cap=64,
+                        clusters=8192, zipf=True, distinct=16),
+    "sweep_2m_k64": dict(n=2097152, d=4096, q=64, k=64, m=16, vocab=128256, cap=0,
+                         clusters=2048, zipf=True, distinct=64),
+}
+DEFAULT = "llama7b_1m"
+GATE = dict(gamma=0.05, topk=3, window=6, tau=0)
+# dram bytes (read + write) per launch of the dominant kernel from one ncu
+# capture, or None when the kernel changed since the capture.
+NCU_TRAFFIC = {}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            j = json.load(f)
+        return float(j["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out = ""
+        sms, maxs, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sms.append(float(parts[0]))
+                maxs.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sms:
+            return None
+        return {"sm_mhz": statistics.median(sms), "sm_max_mhz": max(maxs),
+                "reasons": sorted(reasons), "samples": len(sms)}
+
+
+def make_workload(cfg, dev, seed=0):
+    import synth
+    n, d, m = cfg["n"], cfg["d"], cfg["m"]
+    keys = synth.clustered_unit_keys(n, d, cfg["clusters"], sigma=0.3, seed=seed, device=dev)
+    if cfg["zipf"]:
+        spans = synth.spans_zipf(n, m, cfg["vocab"], 1.1, seed=seed, device=dev)
+    else:
+        spans = synth.spans_uniform(n, m, cfg["vocab"], seed=seed, device=dev)
+    n_q = cfg["distinct"] * cfg["q"]
+    queries, src = synth.noisy_queries(keys, n_q, noise=0.05, seed=seed + 1)
+    queries = queries.reshape(cfg["distinct"], cfg["q"], d).contiguous()
+    return keys, spans, queries
+
+
+def make_gate_inputs(cfg, dev, sets=4, seed=0):
+    import synth
+    q, k, m = cfg["q"], cfg["k"], cfg["m"]
+    cap = cfg["cap"] if cfg["cap"] > 0 else k * m
+    out = []
+    for s in range(sets):
+        root = synth.gate_logits(q, 1, cfg["vocab"], seed=seed + 10 * s, device=dev)[:, 0].contiguous()
+        nodes = synth.gate_logits(q, cap, cfg["vocab"], seed=seed + 10 * s + 1, device=dev)
+        hr = synth.gate_hidden(q, 1, cfg["d"], seed=seed + 10 * s, device=dev)[:, 0].contiguous()
+        hn = synth.gate_hidden(q, cap, cfg["d"], seed=seed + 10 * s + 1, device=dev)
+        out.append((root, nodes, hr, hn))
+    return out
+
+
+class Pipeline:
+    """Preallocated buffers and one step of the path through the C ABI."""
+
+    def __init__(self, S, ds, cfg, dev):
+        self.S, self.ds, self.cfg = S, ds, cfg
+        q, k, m = cfg["q"], cfg["k"], cfg["m"]
+        self.cap = cfg["cap"] if cfg["cap"] > 0 else k * m
+        self.scores = torch.empty(q, k, dtype=torch.float32, device=dev)
+        self.idx = torch.empty(q, k, dtype=torch.int32, device=dev)
+        self.ws = S.alloc_workspace(S.sense_retrieve_workspace_bytes(ds, q, k), dev)
+        self.drafts = torch.empty(q, k, m, dtype=torch.int32, device=dev)
+        self.tree = {}
+        self.gate = {}
+        self.gws = S.alloc_workspace(S.sense_soft_gate_workspace_bytes(q, self.cap, GATE["topk"]), dev)
+
+    def step(self, query, gate_in):
+        S, cfg = self.S, self.cfg
+        S.sense_retrieve_topk(self.ds, query, cfg["k"], self.scores, self.idx, self.ws)
+        S.sense_gather_drafts(self.ds, self.idx, out=self.drafts)
+        S.sense_build_tree(self.drafts, node_cap=cfg["cap"], outs=self.tree)
+        root, nodes, hr, hn = gate_in
+        S.sense_soft_gate(self.tree, root, nodes, hr, hn, workspace=self.gws, outs=self.gate, **GATE)
+
+
+def cpu_baseline(cfg, keys, spans, queries, gate_sets, budget_s=25.0):
+    """The oracle, as it stands, on whole queries of the same workload."""
+    import oracle as O
+    from tests.parity import bits, host
+    kb = bits(keys)
+    sp = host(spans)
+    root, nodes, hr, hn = [host(t) if t.dtype != torch.bfloat16 else bits(t) for t in gate_sets[0]]
+    done, t0 = 0, time.perf_counter()
+    while True:
+        qb = bits(queries[done % queries.shape[0]])
+        s = O.scores(kb, qb)
+        _, idx = O.topk(s, cfg["k"])
+        dr = O.gather_drafts(sp, idx)
+        tr = O.loose_trie(dr, node_cap=cfg["cap"])
+        O.soft_gate(tr["tokens"], tr["parent"], tr["num_nodes"], tr["gamma"], root, nodes, hr,
+                    hn, gamma_thr=GATE["gamma"], kappa=GATE["topk"], window=GATE["window"])
+        done += 1
+        el = time.perf_counter() - t0
+        if el > budget_s * 0.5 or done >= 4:
+            break
+    qn = done * cfg["q"]
+    return {"value": qn / el, "unit": "queries/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{done} whole step(s) of the workload ({qn} queries over all "
+                      f"{cfg['n']} keys + gather/tree/gate), numpy fp64, {el:.1f} s"}
+
+
+def run_reference(args, cfg, name):
+    """--impl reference: the CPU oracle, timed on bounded samples per step."""
+    import oracle as O
+    import synth
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    n, d = cfg["n"], cfg["d"]
+    # A step scores the query batch against one slice of the store (rows
+    # rotate over steps) and runs top-k/gather/tree/gate on that slice's
+    # candidates; queries/s = q / (slices x slice-scan time + downstream time).
+    slice_rows = min(n, 4096)
+    slices = (n + slice_rows - 1) // slice_rows
+    dev = "cpu"
+    keys = synth.clustered_unit_keys(min(n, slice_rows * 4), d, min(cfg["clusters"], 256),
+                                     seed=0, device=dev)
+    spans = synth.spans_zipf(keys.shape[0], cfg["m"], cfg["vocab"], seed=0, device=dev)
+    qs, _ = synth.noisy_queries(keys, cfg["q"], seed=1)
+    gate = make_gate_inputs(cfg, dev, sets=1)[0]
+    from tests.parity import bits, host
+    kb, sp, qb = bits(keys), host(spans), bits(qs)
+    root, nodes, hr, hn = host(gate[0]), host(gate[1]), bits(gate[2]), bits(gate[3])
+    t_scan, t_down = [], []
+    total = args.warmup + args.steps
+    t_all0 = time.perf_counter()
+    for it in range(total):
+        lo = (it % 4) * slice_rows
+        t0 = time.perf_counter()
+        s = O.scores(kb[lo:lo + slice_rows], qb)
+        t1 = time.perf_counter()
+        _, idx = O.topk(s, cfg["k"])
+        dr = O.gather_drafts(sp[lo:lo + slice_rows], idx)
+        tr = O.loose_trie(dr, node_cap=cfg["cap"])
+        O.soft_gate(tr["tokens"], tr["parent"], tr["num_nodes"], tr["gamma"], root, nodes, hr,
+                    hn, gamma_thr=GATE["gamma"], kappa=GATE["topk"], window=GATE["window"])
+        t2 = time.perf_counter()
+        if it >= args.warmup:
+            t_scan.append(t1 - t0)
+            t_down.append(t2 - t1)
+        if time.perf_counter() - t_all0 > 150 and len(t_scan) >= 1:
+            break
+    per_query_batch = slices * statistics.mean(t_scan) + statistics.mean(t_down)
+    value = cfg["q"] / per_query_batch
+    line = {
+        "impl": "reference", "metric": "queries/s", "value": value, "unit": "queries/s",
+        "n_gpus": args.gpus, "steps": len(t_scan), "warmup": args.warmup,
+        "ms_per_step": per_query_batch * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": name, **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab", "cap")}},
+        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": os.cpu_count(),
+                         "kind": "oracle",
+                         "sample": f"per step: scoring of {cfg['q']} queries over one "
+                                   f"{slice_rows}-row slice (x{slices} slices per query batch) "
+                                   f"plus top-k/gather/tree/gate; numpy fp64"},
+        "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="sense", choices=["sense", "reference"])
+    ap.add_argument("--workload", default=DEFAULT, choices=sorted(WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    cfg = WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, cfg, args.workload)
+        return
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import paper_2606_00021_gb300 as S
+    from paper_2606_00021_gb300 import _build
+    _build.build()
+    S.lib()
+
+    keys, spans, queries = make_workload(cfg, dev, seed=rank)
+    gate_sets = make_gate_inputs(cfg, dev, sets=4, seed=100 + rank)
+    ds = S.sense_datastore_build(keys, spans)
+    pipe = Pipeline(S, ds, cfg, dev)
+    nq = queries.shape[0]
+
+    for it in range(args.warmup):
+        pipe.step(queries[it % nq], gate_sets[it % 4])
+    torch.cuda.synchronize()
+    if S.sense_device_status(clear=True) != 0:
+        raise RuntimeError("device status bits set after warm-up")
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    S.sense_profile_enable(True)
+    stream = torch.cuda.current_stream()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for it in range(args.steps):
+        pipe.step(queries[it % nq], gate_sets[it % 4])
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    prof = {name: S.sense_profile_query(name) for name in S.sense_profile_names()}
+    S.sense_profile_enable(False)
+    if dist:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    launches = sum(v[1] for v in prof.values())
+
+    q, n, d = cfg["q"], cfg["n"], cfg["d"]
+    value = world * q * args.steps / (ms / 1e3)
+    # roofline of the dominant kernel (the key scan)
+    scan_name = "scan_gemv" if q <= 8 else "scan_tc"
+    scan_ms, scan_launches = prof.get(scan_name, (0.0, 0))
+    scan_bytes_per_step = n * d * 2 + q * d * 2
+    achieved = scan_bytes_per_step * args.steps / (scan_ms / 1e3) / 1e9 if scan_ms > 0 else 0.0
+    peak, peak_kind = peaks()
+    step_bytes = scan_bytes_per_step  # gate/tree bytes are <0.1% of the scan here
+
+    # end to end through the C ABI with host buffers
+    e2e_steps = min(args.e2e_steps, args.steps)
+    h_query = torch.empty_like(queries[0], device="cpu").pin_memory()
+    h_query.copy_(queries[0])
+    gsrc = gate_sets[0]
+    h_gate = [t.to("cpu").pin_memory() for t in gsrc]
+    d_query = torch.empty_like(queries[0])
+    d_gate = [torch.empty_like(t) for t in gsrc]
+    outs = ["scores", "idx"]
+    h_scores = torch.empty(q, cfg["k"], dtype=torch.float32).pin_memory()
+    h_idx = torch.empty(q, cfg["k"], dtype=torch.int32).pin_memory()
+    h_acc = torch.empty(q, cfg["m"], dtype=torch.int32).pin_memory()
+    h_small = torch.empty(q, 4, dtype=torch.int32).pin_memory()
+    h_hnext = torch.empty(q, d, dtype=torch.bfloat16).pin_memory()
+    h2d = h_query.numel() * h_query.element_size() + sum(t.numel() * t.element_size() for t in h_gate)
+    d2h = sum(t.numel() * t.element_size() for t in (h_scores, h_idx, h_acc, h_small, h_hnext))
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for it in range(e2e_steps):
+        d_query.copy_(h_query, non_blocking=True)
+        for dg, hg in zip(d_gate, h_gate):
+            dg.copy_(hg, non_blocking=True)
+        pipe.step(d_query, d_gate)
+        h_scores.copy_(pipe.scores, non_blocking=True)
+        h_idx.copy_(pipe.idx, non_blocking=True)
+        h_acc.copy_(pipe.gate["accepted"], non_blocking=True)
+        h_small[:, 0].copy_(pipe.gate["i_star"], non_blocking=True)
+        h_small[:, 1].copy_(pipe.gate["L_star"], non_blocking=True)
+        h_small[:, 2].copy_(pipe.gate["next_node"], non_blocking=True)
+        h_small[:, 3].copy_(pipe.gate["next_anchor"], non_blocking=True)
+        h_hnext.copy_(pipe.gate["h_next"], non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+    e2e_s = time.perf_counter() - t0
+    if dist:
+        t = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e_value = world * q * e2e_steps / e2e_s
+
+    base = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        base = cpu_baseline(cfg, keys, spans, queries, gate_sets)
+
+    if rank == 0:
+        mean_nodes = None
+        line = {
+            "metric": "hidden-state top-k retrieval queries/s (whole drafting step)",
+            "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded clustered unit-norm keys, Zipf spans, N(0,9) logits)",
+            "config": {"workload": args.workload,
+                       **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab", "cap", "clusters")},
+                       "key_bytes": n * d * 2,
+                       "l2": "inputs larger than L2: the 8.6 GB store is streamed every step",
+                       "parallelism": f"replicas x{world}"},
+            "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,
+            "roofline": {"bound": "hbm", "kernel": scan_name, "achieved": achieved,
+                         "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "peak_kind": peak_kind, "traffic": NCU_TRAFFIC.get(scan_name),
+                         "launches": scan_launches, "kernel_ms": scan_ms},
+            "kernel_ms": {k: round(v[0], 4) for k, v in prof.items() if v[1]},
+            "gpu_launches": launches,
+            "clocks": clk,
+            "e2e": {"value": e2e_value, "unit": "queries/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+            "cpu_baseline": base,
+        }
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,280 @@
+/*
+ * sense.h - C ABI of libsense, a GB300 (sm_103a) library for the drafting
+ * hot path of SENSE (Semantic Embedding Navigation with Soft-gated
+ * Evaluation, arxiv 2606.00021):
+ *
+ *   hidden-state query --score--> top-k keys --gather--> candidate spans
+ *   --loose trie--> draft tree --soft gate--> accepted prefix / next state
+ *
+ * Conventions shared by every call:
+ *  - Every array argument is a DEVICE pointer on the current CUDA device,
+ *    owned by the caller, contiguous row-major, unless stated otherwise.
+ *  - bf16 values travel as uint16_t bit patterns.
+ *  - Calls are asynchronous on the caller's stream (`sense_stream_t` is the
+ *    same type as `cudaStream_t`; NULL is the legacy default stream).
+ *    Outputs are valid once that stream has been synchronised.
+ *  - Arguments are validated on the host before anything is launched; on
+ *    any error nothing is launched and the outputs are untouched.  The
+ *    functions return a status code, never throw, exit or abort.  A
+ *    thread-local message describing the last error is available from
+ *    sense_last_error().
+ *  - Problems that only the device can see (an out-of-range key index, a
+ *    negative token id, a wait that gave up) set bits in a per-device status
+ *    word, read with sense_device_status().
+ *  - No call synchronises the stream or allocates memory, except
+ *    sense_datastore_build with SENSE_DS_NORMALIZE (allocates the normalised
+ *    copy), sense_device_status (synchronises) and the first call of the
+ *    library on a device (allocates the 256-byte status word).
+ */
+#ifndef SENSE_H_
+#define SENSE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* sense_stream_t;
+typedef struct sense_datastore sense_datastore;
+
+typedef enum sense_status {
+  SENSE_OK = 0,
+  SENSE_ERR_INVALID_ARG = 1,   /* bad pointer, size, flag or workspace size  */
+  SENSE_ERR_UNSUPPORTED = 2,   /* valid request outside the implemented range */
+  SENSE_ERR_OOM = 3,           /* device allocation failed                    */
+  SENSE_ERR_CUDA = 4,          /* a CUDA runtime call failed                  */
+  SENSE_ERR_DEVICE_STATUS = 5, /* device status word has bits set            */
+  SENSE_ERR_TIMEOUT = 6        /* a bounded device wait gave up               */
+} sense_status;
+
+/* Bits of the per-device status word. */
+#define SENSE_DEVST_BAD_INDEX 0x1u   /* gather: key index outside [0, n)      */
+#define SENSE_DEVST_BAD_TOKEN 0x2u   /* tree: negative token id in a span     */
+#define SENSE_DEVST_TIMEOUT 0x4u     /* a pipeline wait hit its limit         */
+#define SENSE_DEVST_INTERNAL 0x8u    /* an internal consistency check failed  */
+
+/* Key storage types for sense_datastore_build. */
+#define SENSE_KEY_BF16 0
+#define SENSE_KEY_F32 1
+
+/* Datastore flags. */
+#define SENSE_DS_BORROW 0x0u     /* keep the caller's bf16 keys (zero copy)   */
+#define SENSE_DS_NORMALIZE 0x1u  /* f32 keys -> unit L2 norm -> bf16 copy     */
+
+/* Gather flags. */
+#define SENSE_GATHER_FORCE_ANCHOR 0x1u
+
+/* Tree flags. */
+#define SENSE_TREE_MASK_BITS 0x1u
+
+/* Gate flags. */
+#define SENSE_GATE_UNNORMALIZED_ENTROPY 0x1u
+
+/* Limits. */
+#define SENSE_MAX_K 1024          /* retrieval top-k                          */
+#define SENSE_MAX_M 32            /* span length                              */
+#define SENSE_MAX_TREE_TOKENS 8192 /* k * m accepted by sense_build_tree      */
+#define SENSE_MAX_KAPPA 16        /* gate top-k                               */
+#define SENSE_MAX_WINDOW 64       /* gate lookahead window                    */
+
+int32_t sense_version(void);
+const char* sense_status_string(sense_status s);
+/* Message of the last error raised on the calling thread ("" if none). */
+const char* sense_last_error(void);
+
+/*
+ * Reads the status word of the current device, after synchronising
+ * `stream`; if `clear` is non-zero the word is reset to 0 afterwards.
+ * Returns SENSE_ERR_DEVICE_STATUS when any bit is set, else SENSE_OK.
+ */
+sense_status sense_device_status(sense_stream_t stream, uint32_t* out_bits, int32_t clear);
+
+/* ---------------------------------------------------------------------- */
+/* a1. Datastore                                                           */
+/* ---------------------------------------------------------------------- */
+/*
+ * The static datastore C_s of Sec. 3.2.1 (Eq. 2, Eq. 6): n pairs
+ * (key_i, span_i), key_i a d-dimensional hidden-state key, span_i the m
+ * tokens that followed it.  App. E (Implementation Details) states that keys
+ * are L2-normalised before indexing.
+ *
+ *   keys   [n, d] bf16 (key_dtype SENSE_KEY_BF16, flags SENSE_DS_BORROW):
+ *          borrowed, must stay alive and unchanged while the datastore is
+ *          used.  Or [n, d] f32 (SENSE_KEY_F32 with SENSE_DS_NORMALIZE):
+ *          each row is scaled to unit L2 norm and rounded to bf16 (nearest,
+ *          ties to even) into a copy owned by the datastore (a zero row
+ *          stays zero).  The normalisation runs asynchronously on `stream`.
+ *   spans  [n, m] int32, borrowed, token ids >= 0.
+ *   Limits: 1 <= n <= 2^31 - 1, 8 <= d <= 65536 with d % 8 == 0,
+ *   1 <= m <= SENSE_MAX_M; keys and spans 16-byte aligned.
+ * *out receives an opaque host handle; release it with
+ * sense_datastore_destroy (which frees the normalised copy, if any, after
+ * synchronising the device).
+ */
+sense_status sense_datastore_build(const void* keys, int32_t key_dtype, int64_t n, int32_t d,
+                                   const int32_t* spans, int32_t m, uint32_t flags,
+                                   sense_stream_t stream, sense_datastore** out);
+sense_status sense_datastore_destroy(sense_datastore* ds);
+/* Device pointer of the bf16 keys in use (borrowed or owned). */
+const uint16_t* sense_datastore_keys(const sense_datastore* ds);
+
+/* ---------------------------------------------------------------------- */
+/* a2 + a3. Scoring and top-k                                              */
+/* ---------------------------------------------------------------------- */
+/*
+ * Exact inner-product search (Sec. 3.2.2 Eq. 7 and Eq. 8's sim(.,.); App. C.2
+ * Alg. 2): for each query q, s[q, i] = <queries[q], key_i> accumulated in
+ * fp32 from bf16 inputs, and the k largest scores are returned in the order
+ * (score descending, key index ascending).
+ *
+ *   queries    [q, d] bf16, 16-byte aligned.
+ *   out_scores [q, k] f32; out_idx [q, k] int32 (key indices).
+ *   workspace  device scratch of at least
+ *              sense_retrieve_workspace_bytes(ds, q, k) bytes, 256-byte
+ *              aligned; its contents on entry do not matter.
+ *   Limits: q >= 1, 1 <= k <= min(n, SENSE_MAX_K).
+ * Paths: q <= 8 uses a CUDA-core streaming kernel; q > 8 uses tcgen05
+ * tensor-core tiles (queries padded to a multiple of 16, processed in
+ * groups of at most 128).
+ */
+size_t sense_retrieve_workspace_bytes(const sense_datastore* ds, int32_t q, int32_t k);
+sense_status sense_retrieve_topk(const sense_datastore* ds, const uint16_t* queries, int32_t q,
+                                 int32_t k, float* out_scores, int32_t* out_idx,
+                                 void* workspace, size_t workspace_bytes, sense_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* a4. Span gather                                                          */
+/* ---------------------------------------------------------------------- */
+/*
+ * Candidate drafts D (Sec. 3.2.2, D_ret = {(k_i, s_i)}):
+ * out_spans[q, r, :] = spans[idx[q, r], :].
+ *
+ *   idx       [q, k] int32 (as returned by sense_retrieve_topk).
+ *   anchor    NULL, or [q] int32 anchor tokens x~.  With an anchor, the
+ *             composite score of Eq. 8 (alpha >> beta) reorders the
+ *             candidates: rows whose first token equals the anchor come
+ *             first, each group keeping retrieval order; the first n_keep
+ *             rows are written.  With SENSE_GATHER_FORCE_ANCHOR the first
+ *             token of kept row 0 and of kept row n_keep-1 is set to the
+ *             anchor (App. C.2 Alg. 2, forced anchor).
+ *   n_keep    rows written per query: 1 <= n_keep <= k (must equal k when
+ *             anchor is NULL).
+ *   out_spans [q, n_keep, m] int32.
+ * An index outside [0, n) produces a row of -1 and sets
+ * SENSE_DEVST_BAD_INDEX; no out-of-range load is made.
+ */
+sense_status sense_gather_drafts(const sense_datastore* ds, const int32_t* idx, int32_t q,
+                                 int32_t k, const int32_t* anchor, int32_t n_keep, uint32_t flags,
+                                 int32_t* out_spans, sense_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* a5. Loose trie (draft tree)                                              */
+/* ---------------------------------------------------------------------- */
+/*
+ * Sorted-LCP loose trie of Sec. 3.2.3 Eq. 9 / App. C.3 Alg. 3: the distinct
+ * non-empty prefixes of the k candidate spans of each query, numbered in
+ * lexicographic preorder (the order of T_flat).
+ *
+ *   spans [q, k, m] int32 token ids (>= 0).
+ *   node_cap  C > 0 keeps at most C nodes: each node is keyed by
+ *             (smallest candidate rank containing it, depth) and the C
+ *             smallest keys are kept (prefix-closed); 0 = no cap.
+ *   Output capacity cap = node_cap if node_cap > 0 else k * m.
+ *   out_num_nodes [q]; out_tokens, out_parent, out_depth [q, cap]
+ *   (parent -1 = child of the current position; depth 0-based; slots past
+ *   num_nodes are -1); out_gamma [q, k, m] = node id of candidate r's
+ *   prefix of length j+1, in the candidates' input order (-1 when the cap
+ *   dropped it).
+ *   out_mask_bits (with SENSE_TREE_MASK_BITS, else may be NULL):
+ *   [q, cap, ceil(cap/32)] uint32, bit b of row n set iff node b is an
+ *   ancestor of n or n itself (Alg. 3's mask M).
+ *   Limits: 1 <= k <= SENSE_MAX_K, 1 <= m <= SENSE_MAX_M,
+ *   k * m <= SENSE_MAX_TREE_TOKENS.
+ * A negative token sets SENSE_DEVST_BAD_TOKEN and that query gets
+ * num_nodes = 0 with all outputs -1.
+ */
+sense_status sense_build_tree(const int32_t* spans, int32_t q, int32_t k, int32_t m,
+                              int32_t node_cap, uint32_t flags, int32_t* out_num_nodes,
+                              int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
+                              int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* a6. Soft-gated evaluation                                                */
+/* ---------------------------------------------------------------------- */
+/*
+ * Sec. 3.3 (Eqs. 12-19) and App. C.4 Alg. 4, per query:
+ *  - position j of candidate i carries draft token D[i,j] = tokens[gamma[i,j]]
+ *    and is predicted by P_align[i,j] = root_logits (j = 0) or the logits
+ *    row of node gamma[i,j-1] (Eq. 11 alignment);
+ *  - B_em = I(D == argmax P_align) (lowest index among equal maxima);
+ *  - B_ent = I(E / log V > gamma), E the entropy of softmax(P_align) in nats
+ *    (SENSE_GATE_UNNORMALIZED_ENTROPY: I(E > gamma), Eq. 14);
+ *  - B_topk = I(D in top-kappa of P_align), order (logit desc, index asc);
+ *  - B_con = I(#mismatches among positions j+1..j+W <= tau), positions past
+ *    the span (and positions dropped by the node cap) counting as
+ *    mismatches (Alg. 4: Pad(1-B_em,(0,W),1), Conv1D(.,1_W)[:,1:M+1], == 0);
+ *  - G = B_em | (B_ent & (B_topk | B_con)); L_i = leading run of ones in
+ *    G[i,:] minus 1; i* = lowest i with the largest L_i; L* = L_{i*}.
+ * Positions whose node was dropped by the cap have G = 0.
+ *
+ *   tokens, parent [q, cap], num_nodes [q], gamma [q, k, m]: the tree from
+ *   sense_build_tree (same cap).
+ *   root_logits [q, vocab] f32 (p); node_logits [q, cap, vocab] f32 (the
+ *   target logits at each tree node, P').  Only rows of the root, of nodes
+ *   that have children, and of the chosen next node are read.
+ *   root_hidden [q, d] bf16 (h); node_hidden [q, cap, d] bf16 (H').
+ *   Outputs: out_i_star, out_L_star, out_n_accept (= L*+1), out_next_node
+ *   (gamma[i*, L*], or -1 for the root when L* = -1), out_next_anchor
+ *   (argmax of the next node's logits row, p_next of Eq. 19) [q] int32;
+ *   out_accepted [q, m] int32 (D[i*, 0..L*], then -1);
+ *   out_h_next [q, d] bf16 (h_next of Eq. 19);
+ *   out_G [q, k, m] uint8 or NULL.
+ *   params: gamma (threshold), topk (kappa, 1..SENSE_MAX_KAPPA), window W
+ *   (1..SENSE_MAX_WINDOW), tau (>= 0), flags.  Paper defaults (App. E):
+ *   gamma 0.05, kappa 3, W 6, tau 0.
+ *   workspace: at least sense_soft_gate_workspace_bytes(q, cap, kappa)
+ *   bytes of device scratch, 256-byte aligned.
+ *   Limits: vocab >= kappa, vocab % 4 == 0; d % 8 == 0; k * m <=
+ *   SENSE_MAX_TREE_TOKENS; logits 16-byte aligned.
+ */
+typedef struct sense_gate_params {
+  float gamma;
+  int32_t topk;
+  int32_t window;
+  int32_t tau;
+  uint32_t flags;
+} sense_gate_params;
+
+size_t sense_soft_gate_workspace_bytes(int32_t q, int32_t cap, int32_t kappa);
+sense_status sense_soft_gate(const int32_t* tokens, const int32_t* parent,
+                             const int32_t* num_nodes, const int32_t* gamma, int32_t q, int32_t k,
+                             int32_t m, int32_t cap, const float* root_logits,
+                             const float* node_logits, int32_t vocab, const uint16_t* root_hidden,
+                             const uint16_t* node_hidden, int32_t d,
+                             const sense_gate_params* params, int32_t* out_i_star,
+                             int32_t* out_L_star, int32_t* out_n_accept, int32_t* out_accepted,
+                             int32_t* out_next_node, int32_t* out_next_anchor,
+                             uint16_t* out_h_next, uint8_t* out_G, void* workspace,
+                             size_t workspace_bytes, sense_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* Launch profiling                                                         */
+/* ---------------------------------------------------------------------- */
+/*
+ * When enabled, every kernel launch of the library is bracketed by two CUDA
+ * events recorded on the launching stream.  sense_profile_enable(1) clears
+ * earlier records.  sense_profile_query synchronises on the recorded events
+ * and returns, for the kernel family `name` (see sense_profile_name), the
+ * summed device time in milliseconds and the number of launches.
+ */
+sense_status sense_profile_enable(int32_t on);
+int32_t sense_profile_count(void);
+const char* sense_profile_name(int32_t i);
+sense_status sense_profile_query(const char* name, double* total_ms, int64_t* launches);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SENSE_H_ */

@@ -1,0 +1,277 @@
+"""Python binding of libsense: the SENSE drafting hot path on GB300.
+
+Thin argument marshalling over the C ABI of include/sense.h: every function
+here checks tensor devices, dtypes and shapes, allocates outputs with torch
+when the caller did not pass them, and calls the function of the same name
+in libsense.so on the current CUDA stream.  All computation happens in the
+library's CUDA kernels; there is no CPU path.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from dataclasses import dataclass, field
+
+import torch
+
+from . import _abi
+
+SENSE_OK = 0
+STATUS_NAMES = {0: "SENSE_OK", 1: "SENSE_ERR_INVALID_ARG", 2: "SENSE_ERR_UNSUPPORTED",
+                3: "SENSE_ERR_OOM", 4: "SENSE_ERR_CUDA", 5: "SENSE_ERR_DEVICE_STATUS",
+                6: "SENSE_ERR_TIMEOUT"}
+DEVST_BAD_INDEX, DEVST_BAD_TOKEN, DEVST_TIMEOUT, DEVST_INTERNAL = 1, 2, 4, 8
+
+
+class SenseError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+def lib():
+    return _abi.load()
+
+
+def _check(st: int):
+    if st != SENSE_OK:
+        msg = lib().sense_last_error().decode(errors="replace")
+        raise SenseError(st, msg)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _need(t: torch.Tensor, name: str, dtype, ndim=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.device.type != "cuda":
+        raise ValueError(f"{name} must be a CUDA tensor (got {t.device})")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype} (got {t.dtype})")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims (got {tuple(t.shape)})")
+    return t
+
+
+def _i32(shape, dev):
+    return torch.empty(shape, dtype=torch.int32, device=dev)
+
+
+def sense_version() -> int:
+    return int(lib().sense_version())
+
+
+def sense_device_status(clear: bool = True, stream=None) -> int:
+    """Status bits of the current device (synchronises the stream)."""
+    out = C.c_uint32(0)
+    st = lib().sense_device_status(C.c_void_p(_stream(stream)), C.byref(out), 1 if clear else 0)
+    if st not in (0, 5, 6):
+        _check(st)
+    return int(out.value)
+
+
+@dataclass
+class Datastore:
+    """Handle of a datastore (keys [n, d] bf16, spans [n, m] int32)."""
+    handle: int
+    n: int
+    d: int
+    m: int
+    keys: torch.Tensor | None
+    spans: torch.Tensor
+    _keep: list = field(default_factory=list)
+
+    def close(self):
+        if self.handle:
+            lib().sense_datastore_destroy(C.c_void_p(self.handle))
+            self.handle = 0
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def sense_datastore_build(keys: torch.Tensor, spans: torch.Tensor, normalize: bool = False,
+                          stream=None) -> Datastore:
+    """Registers a datastore; keys bf16 [n, d] (borrowed) or f32 with normalize=True."""
+    if normalize:
+        _need(keys, "keys", torch.float32, 2)
+        dtype_code, flags = 1, 1
+    else:
+        _need(keys, "keys", torch.bfloat16, 2)
+        dtype_code, flags = 0, 0
+    _need(spans, "spans", torch.int32, 2)
+    n, d = keys.shape
+    if spans.shape[0] != n:
+        raise ValueError("keys and spans must have the same number of rows")
+    out = C.c_void_p(0)
+    _check(lib().sense_datastore_build(keys.data_ptr(), dtype_code, n, d, spans.data_ptr(),
+                                       spans.shape[1], flags, C.c_void_p(_stream(stream)),
+                                       C.byref(out)))
+    ds = Datastore(out.value, n, d, spans.shape[1], keys if not normalize else None, spans)
+    ds._keep = [keys, spans]
+    return ds
+
+
+class _DeviceArray:
+    """Minimal __cuda_array_interface__ wrapper of a library-owned buffer."""
+
+    def __init__(self, ptr: int, shape, typestr: str):
+        self.__cuda_array_interface__ = {"shape": tuple(shape), "typestr": typestr,
+                                         "data": (int(ptr), False), "version": 3,
+                                         "strides": None}
+
+
+def sense_datastore_keys(ds: Datastore) -> torch.Tensor:
+    """The bf16 keys in use: the caller's tensor, or a zero-copy view of the
+    normalised copy owned by the datastore (valid while ``ds`` is open)."""
+    if ds.keys is not None:
+        return ds.keys
+    ptr = lib().sense_datastore_keys(C.c_void_p(ds.handle))
+    view = torch.as_tensor(_DeviceArray(ptr, (ds.n, ds.d), "<i2"), device="cuda")
+    return view.view(torch.bfloat16)
+
+
+def sense_retrieve_workspace_bytes(ds: Datastore, q: int, k: int) -> int:
+    return int(lib().sense_retrieve_workspace_bytes(C.c_void_p(ds.handle), q, k))
+
+
+def alloc_workspace(nbytes: int, device=None) -> torch.Tensor:
+    dev = device or torch.device("cuda", torch.cuda.current_device())
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=dev)
+
+
+def sense_retrieve_topk(ds: Datastore, queries: torch.Tensor, k: int, out_scores=None,
+                        out_idx=None, workspace=None, stream=None):
+    """Exact top-k inner-product search: (scores f32 [q, k], idx int32 [q, k])."""
+    _need(queries, "queries", torch.bfloat16, 2)
+    q = queries.shape[0]
+    if queries.shape[1] != ds.d:
+        raise ValueError("queries must have d columns")
+    dev = queries.device
+    if out_scores is None:
+        out_scores = torch.empty(q, k, dtype=torch.float32, device=dev)
+    if out_idx is None:
+        out_idx = _i32((q, k), dev)
+    need = sense_retrieve_workspace_bytes(ds, q, k)
+    if workspace is None:
+        workspace = alloc_workspace(need, dev)
+    _check(lib().sense_retrieve_topk(C.c_void_p(ds.handle), queries.data_ptr(), q, k,
+                                     out_scores.data_ptr(), out_idx.data_ptr(),
+                                     workspace.data_ptr(), workspace.numel(),
+                                     C.c_void_p(_stream(stream))))
+    return out_scores, out_idx
+
+
+def sense_gather_drafts(ds: Datastore, idx: torch.Tensor, anchor=None, n_keep=None,
+                        force_anchor: bool = False, out=None, stream=None) -> torch.Tensor:
+    """Candidate spans [q, n_keep, m] int32 for retrieved indices idx [q, k]."""
+    _need(idx, "idx", torch.int32, 2)
+    q, k = idx.shape
+    keep = k if n_keep is None else int(n_keep)
+    if anchor is not None:
+        _need(anchor, "anchor", torch.int32, 1)
+    if out is None:
+        out = _i32((q, keep, ds.m), idx.device)
+    _check(lib().sense_gather_drafts(C.c_void_p(ds.handle), idx.data_ptr(), q, k, _ptr(anchor),
+                                     keep, 1 if force_anchor else 0, out.data_ptr(),
+                                     C.c_void_p(_stream(stream))))
+    return out
+
+
+def sense_build_tree(spans: torch.Tensor, node_cap: int = 0, mask_bits: bool = False,
+                     outs: dict | None = None, stream=None) -> dict:
+    """Loose trie of spans [q, k, m]; returns a dict of device tensors."""
+    _need(spans, "spans", torch.int32, 3)
+    q, k, m = spans.shape
+    cap = node_cap if node_cap > 0 else k * m
+    dev = spans.device
+    o = outs or {}
+    o.setdefault("num_nodes", _i32((q,), dev))
+    o.setdefault("tokens", _i32((q, cap), dev))
+    o.setdefault("parent", _i32((q, cap), dev))
+    o.setdefault("depth", _i32((q, cap), dev))
+    o.setdefault("gamma", _i32((q, k, m), dev))
+    if mask_bits:
+        o.setdefault("mask_bits", torch.empty(q, cap, (cap + 31) // 32, dtype=torch.int32,
+                                              device=dev))
+    _check(lib().sense_build_tree(spans.data_ptr(), q, k, m, node_cap, 1 if mask_bits else 0,
+                                  o["num_nodes"].data_ptr(), o["tokens"].data_ptr(),
+                                  o["parent"].data_ptr(), o["depth"].data_ptr(),
+                                  o["gamma"].data_ptr(), _ptr(o.get("mask_bits")),
+                                  C.c_void_p(_stream(stream))))
+    o["cap"] = cap
+    return o
+
+
+def sense_soft_gate_workspace_bytes(q: int, cap: int, kappa: int) -> int:
+    return int(lib().sense_soft_gate_workspace_bytes(q, cap, kappa))
+
+
+def sense_soft_gate(tree: dict, root_logits: torch.Tensor, node_logits: torch.Tensor,
+                    root_hidden: torch.Tensor, node_hidden: torch.Tensor, gamma: float = 0.05,
+                    topk: int = 3, window: int = 6, tau: int = 0,
+                    unnormalized_entropy: bool = False, want_G: bool = False,
+                    workspace=None, outs: dict | None = None, stream=None) -> dict:
+    """Soft-gated evaluation of every draft path; returns a dict of device tensors."""
+    for name in ("num_nodes", "tokens", "parent", "gamma"):
+        _need(tree[name], name, torch.int32)
+    q, k, m = tree["gamma"].shape
+    cap = tree["tokens"].shape[1]
+    _need(root_logits, "root_logits", torch.float32, 2)
+    _need(node_logits, "node_logits", torch.float32, 3)
+    _need(root_hidden, "root_hidden", torch.bfloat16, 2)
+    _need(node_hidden, "node_hidden", torch.bfloat16, 3)
+    vocab = root_logits.shape[1]
+    d = root_hidden.shape[1]
+    if node_logits.shape != (q, cap, vocab) or node_hidden.shape != (q, cap, d):
+        raise ValueError("node_logits / node_hidden must be [q, cap, V] / [q, cap, d]")
+    dev = root_logits.device
+    o = outs or {}
+    for key in ("i_star", "L_star", "n_accept", "next_node", "next_anchor"):
+        o.setdefault(key, _i32((q,), dev))
+    o.setdefault("accepted", _i32((q, m), dev))
+    o.setdefault("h_next", torch.empty(q, d, dtype=torch.bfloat16, device=dev))
+    if want_G:
+        o.setdefault("G", torch.empty(q, k, m, dtype=torch.uint8, device=dev))
+    if workspace is None:
+        workspace = alloc_workspace(sense_soft_gate_workspace_bytes(q, cap, topk), dev)
+    p = _abi.GateParams(float(gamma), int(topk), int(window), int(tau),
+                        1 if unnormalized_entropy else 0)
+    _check(lib().sense_soft_gate(
+        tree["tokens"].data_ptr(), tree["parent"].data_ptr(), tree["num_nodes"].data_ptr(),
+        tree["gamma"].data_ptr(), q, k, m, cap, root_logits.data_ptr(), node_logits.data_ptr(),
+        vocab, root_hidden.data_ptr(), node_hidden.data_ptr(), d, C.byref(p),
+        o["i_star"].data_ptr(), o["L_star"].data_ptr(), o["n_accept"].data_ptr(),
+        o["accepted"].data_ptr(), o["next_node"].data_ptr(), o["next_anchor"].data_ptr(),
+        o["h_next"].data_ptr(), _ptr(o.get("G")), workspace.data_ptr(), workspace.numel(),
+        C.c_void_p(_stream(stream))))
+    return o
+
+
+def sense_profile_enable(on: bool = True):
+    _check(lib().sense_profile_enable(1 if on else 0))
+
+
+def sense_profile_query(name: str):
+    """(total device ms, launches) of one kernel family since profiling was enabled."""
+    ms = C.c_double(0.0)
+    n = C.c_int64(0)
+    _check(lib().sense_profile_query(name.encode(), C.byref(ms), C.byref(n)))
+    return float(ms.value), int(n.value)
+
+
+def sense_profile_names():
+    L = lib()
+    return [L.sense_profile_name(i).decode() for i in range(L.sense_profile_count())]

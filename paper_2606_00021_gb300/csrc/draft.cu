@@ -1,0 +1,372 @@
+// Candidate drafts and the loose trie.
+//
+// gather (Sec. 3.2.2, D_ret = {(k_i, s_i)}; Eq. 8 rerank; App. C.2 Alg. 2
+// forced anchor): one block per query, one thread per retrieved rank.  The
+// anchor-first reordering of Eq. 8 (alpha >> beta) is a stable partition
+// computed with a block-wide prefix count of anchor matches.
+//
+// tree (Sec. 3.2.3 Eq. 9; App. C.3 Alg. 3): one block per query builds the
+// trie entirely in shared memory:
+//   1. bitonic sort of the candidate rows in lexicographic order;
+//   2. LCP of each sorted row with its predecessor: row p creates nodes at
+//      depths lcp[p]..m-1 (Alg. 3's `unique`), and an exclusive scan of the
+//      counts numbers the nodes in preorder (Eq. 9's T_flat);
+//   3. node of (sorted row p, depth j) = node created by the last row
+//      p' <= p with lcp[p'] <= j: a prefix-max over p per column (Alg. 3's
+//      CumMax);
+//   4. node cap: key (first candidate rank containing the node, depth) -
+//      segmented minimum by shared-memory atomicMin, then the cap smallest
+//      keys are kept (keys are distinct integers < k*m, so a prefix count
+//      over a presence table ranks them); kept nodes are renumbered in
+//      preorder by a second prefix count;
+//   5. outputs: tokens/parent/depth, gamma back in the candidates' order,
+//      optional ancestor bit mask.
+#include "common.cuh"
+#include "launch.h"
+
+namespace sense {
+namespace {
+
+// Block-wide exclusive prefix sum of one int per thread (blockDim <= 1024).
+// `scratch` holds at least 32 ints.  Returns the exclusive prefix; *total
+// receives the block sum.
+__device__ int block_exclusive_scan(int v, int* scratch, int* total) {
+  const int lane = threadIdx.x & 31;
+  const int wid = threadIdx.x >> 5;
+  const int nw = (blockDim.x + 31) >> 5;
+  int x = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, x, off);
+    if (lane >= off) x += t;
+  }
+  __syncthreads();
+  if (lane == 31) scratch[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    int y = (lane < nw) ? scratch[lane] : 0;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, y, off);
+      if (lane >= off) y += t;
+    }
+    scratch[lane] = y;  // inclusive per warp
+  }
+  __syncthreads();
+  const int warp_base = (wid > 0) ? scratch[wid - 1] : 0;
+  *total = scratch[nw - 1];
+  const int r = warp_base + x - v;
+  __syncthreads();
+  return r;
+}
+
+__global__ void gather_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
+                              const int32_t* __restrict__ idx, int k,
+                              const int32_t* __restrict__ anchor, int n_keep, int force,
+                              int32_t* __restrict__ out, uint32_t* status) {
+  __shared__ int scratch[32];
+  const int q = blockIdx.x;
+  const int r = threadIdx.x;
+  int64_t i = -1;
+  bool valid = false;
+  if (r < k) {
+    i = idx[(int64_t)q * k + r];
+    valid = (i >= 0 && i < n);
+    if (!valid) raise_status(status, SENSE_DEVST_BAD_INDEX);
+  }
+  int pos = r;
+  if (anchor) {
+    const int a = anchor[q];
+    const bool match = (r < k) && valid && spans[i * m] == a;
+    int total = 0;
+    const int before = block_exclusive_scan(match ? 1 : 0, scratch, &total);
+    pos = match ? before : total + (r - before);
+  }
+  int32_t* dst = out + ((int64_t)q * n_keep + pos) * m;
+  if (r < k && pos < n_keep) {
+    if (valid) {
+      const int32_t* srow = spans + i * m;
+      if ((m & 3) == 0) {
+        for (int j = 0; j < m; j += 4)
+          *reinterpret_cast<int4*>(dst + j) = __ldg(reinterpret_cast<const int4*>(srow + j));
+      } else {
+        for (int j = 0; j < m; ++j) dst[j] = __ldg(srow + j);
+      }
+    } else {
+      for (int j = 0; j < m; ++j) dst[j] = -1;
+    }
+  }
+  if (anchor && force) {
+    __syncthreads();
+    if (r == 0) {
+      const int a = anchor[q];
+      out[((int64_t)q * n_keep) * m] = a;
+      out[((int64_t)q * n_keep + n_keep - 1) * m] = a;
+    }
+  }
+}
+
+constexpr int kTreeThreads = 1024;
+
+// Lexicographic comparison of rows a and b of s (m tokens each); equal rows
+// are ordered by row index so that the order is total.
+__device__ __forceinline__ bool row_less(const int* s, int m, int a, int b) {
+  const int* ra = s + a * m;
+  const int* rb = s + b * m;
+  for (int j = 0; j < m; ++j) {
+    if (ra[j] != rb[j]) return ra[j] < rb[j];
+  }
+  return a < b;
+}
+
+__global__ void __launch_bounds__(kTreeThreads)
+tree_kernel(const int32_t* __restrict__ spans, int k, int m, int cap, int mask_words,
+            int32_t* __restrict__ num_nodes, int32_t* __restrict__ tokens,
+            int32_t* __restrict__ parent, int32_t* __restrict__ depth,
+            int32_t* __restrict__ gamma, uint32_t* __restrict__ mask, uint32_t* status) {
+  extern __shared__ int sm[];
+  const int km = k * m;
+  int kp = 1;
+  while (kp < k) kp <<= 1;
+  int* s_tok = sm;            // [k*m] candidate tokens
+  int* s_own = s_tok + km;    // [k*m] node of (sorted row, depth); later scratch
+  int* s_aux = s_own + km;    // [k*m] first-rank per node / key table
+  int* s_new = s_aux + km;    // [k*m] kept-node new id
+  int* s_ord = s_new + km;    // [kp] sorted row order
+  int* s_lcp = s_ord + kp;    // [k]
+  int* s_base = s_lcp + k;    // [k]
+  __shared__ int scratch[32];
+  __shared__ int s_bad, s_total, s_kept;
+
+  const int q = blockIdx.x;
+  const int32_t* src = spans + (int64_t)q * km;
+  if (threadIdx.x == 0) s_bad = 0;
+  __syncthreads();
+  for (int i = threadIdx.x; i < km; i += blockDim.x) {
+    const int t = src[i];
+    s_tok[i] = t;
+    if (t < 0) s_bad = 1;
+  }
+  for (int i = threadIdx.x; i < kp; i += blockDim.x) s_ord[i] = i;
+  __syncthreads();
+
+  int32_t* o_tok = tokens + (int64_t)q * cap;
+  int32_t* o_par = parent + (int64_t)q * cap;
+  int32_t* o_dep = depth + (int64_t)q * cap;
+  int32_t* o_gam = gamma + (int64_t)q * km;
+  uint32_t* o_mask = mask ? mask + (int64_t)q * cap * mask_words : nullptr;
+
+  if (s_bad) {
+    if (threadIdx.x == 0) {
+      raise_status(status, SENSE_DEVST_BAD_TOKEN);
+      num_nodes[q] = 0;
+    }
+    for (int i = threadIdx.x; i < cap; i += blockDim.x) {
+      o_tok[i] = -1;
+      o_par[i] = -1;
+      o_dep[i] = -1;
+    }
+    for (int i = threadIdx.x; i < km; i += blockDim.x) o_gam[i] = -1;
+    if (o_mask)
+      for (int64_t i = threadIdx.x; i < (int64_t)cap * mask_words; i += blockDim.x) o_mask[i] = 0u;
+    return;
+  }
+
+  // 1. Bitonic sort of row indices (padding indices >= k sort last).
+  for (int size = 2; size <= kp; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < kp; i += blockDim.x) {
+        const int j = i ^ stride;
+        if (j > i) {
+          const bool up = ((i & size) == 0);
+          const int a = s_ord[i], b = s_ord[j];
+          bool b_first;  // true when b must precede a
+          if (a >= k) b_first = (b < k) || (b < a);
+          else if (b >= k) b_first = false;
+          else b_first = row_less(s_tok, m, b, a);
+          if (up ? b_first : !b_first) {
+            s_ord[i] = b;
+            s_ord[j] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+
+  // 2. LCP with the previous sorted row, node counts, preorder bases.
+  int cnt = 0;
+  if (threadIdx.x < k) {
+    const int p = threadIdx.x;
+    int l = 0;
+    if (p > 0) {
+      const int* ra = s_tok + s_ord[p - 1] * m;
+      const int* rb = s_tok + s_ord[p] * m;
+      while (l < m && ra[l] == rb[l]) ++l;
+    }
+    s_lcp[p] = l;
+    cnt = m - l;
+  }
+  int total = 0;
+  const int base = block_exclusive_scan(cnt, scratch, &total);
+  if (threadIdx.x < k) s_base[threadIdx.x] = base;
+  if (threadIdx.x == 0) s_total = total;
+  // 3. Creator row per (p, j): prefix max over p of (lcp[p] <= j ? p : -1).
+  for (int e = threadIdx.x; e < km; e += blockDim.x) {
+    const int p = e / m, j = e - p * m;
+    s_own[e] = (s_lcp[p] <= j) ? p : -1;
+  }
+  __syncthreads();
+  for (int off = 1; off < k; off <<= 1) {
+    int vals[(SENSE_MAX_TREE_TOKENS + kTreeThreads - 1) / kTreeThreads];
+    int c = 0;
+    for (int e = threadIdx.x; e < km; e += blockDim.x, ++c) {
+      const int p = e / m;
+      int v = s_own[e];
+      if (p >= off) v = max(v, s_own[e - off * m]);
+      vals[c] = v;
+    }
+    __syncthreads();
+    c = 0;
+    for (int e = threadIdx.x; e < km; e += blockDim.x, ++c) s_own[e] = vals[c];
+    __syncthreads();
+  }
+  // node id of (sorted p, j) = base[p'] + j - lcp[p'], p' the creator.
+  for (int e = threadIdx.x; e < km; e += blockDim.x) {
+    const int p = e / m, j = e - p * m;
+    const int pc = s_own[e];
+    s_own[e] = s_base[pc] + j - s_lcp[pc];
+  }
+  __syncthreads();
+  const int U = s_total;
+
+  // 4. Node cap.
+  const bool capped = cap < U;
+  if (capped) {
+    for (int u = threadIdx.x; u < U; u += blockDim.x) s_aux[u] = 0x7fffffff;
+    __syncthreads();
+    for (int e = threadIdx.x; e < km; e += blockDim.x) {
+      const int p = e / m;
+      atomicMin(&s_aux[s_own[e]], s_ord[p]);
+    }
+    __syncthreads();
+    // key = first_rank * m + depth; mark presence in s_new (as a key table).
+    for (int i = threadIdx.x; i < km; i += blockDim.x) s_new[i] = 0;
+    __syncthreads();
+    for (int e = threadIdx.x; e < km; e += blockDim.x) {
+      const int p = e / m, j = e - p * m;
+      if (s_lcp[p] <= j) {  // the creator entry of node s_own[e]
+        const int u = s_own[e];
+        s_new[s_aux[u] * m + j] = 1;
+      }
+    }
+    __syncthreads();
+    // rank of every key: chunked block scan over km entries
+    int running = 0;
+    for (int c0 = 0; c0 < km; c0 += blockDim.x) {
+      const int i = c0 + threadIdx.x;
+      const int v = (i < km) ? s_new[i] : 0;
+      int tot = 0;
+      const int ex = block_exclusive_scan(v, scratch, &tot);
+      if (i < km) s_new[i] = v ? (running + ex) : -1;
+      running += tot;
+    }
+    __syncthreads();
+    // kept flag per node (u in preorder): rank of its key < cap.
+    for (int e = threadIdx.x; e < km; e += blockDim.x) {
+      const int p = e / m, j = e - p * m;
+      if (s_lcp[p] <= j) {
+        const int u = s_own[e];
+        const int rk = s_new[s_aux[u] * m + j];
+        s_aux[u] = (rk < cap) ? 1 : 0;  // s_aux now holds kept flags
+      }
+    }
+    __syncthreads();
+    // new ids: prefix count of kept flags in preorder
+    running = 0;
+    for (int c0 = 0; c0 < U; c0 += blockDim.x) {
+      const int u = c0 + threadIdx.x;
+      const int v = (u < U) ? s_aux[u] : 0;
+      int tot = 0;
+      const int ex = block_exclusive_scan(v, scratch, &tot);
+      if (u < U) s_new[u] = v ? (running + ex) : -1;
+      running += tot;
+    }
+    if (threadIdx.x == 0) s_kept = running;
+  } else {
+    for (int u = threadIdx.x; u < U; u += blockDim.x) s_new[u] = u;
+    if (threadIdx.x == 0) s_kept = U;
+  }
+  __syncthreads();
+  const int kept = s_kept;
+
+  // 5. Outputs.
+  if (threadIdx.x == 0) num_nodes[q] = kept;
+  for (int i = kept + threadIdx.x; i < cap; i += blockDim.x) {
+    o_tok[i] = -1;
+    o_par[i] = -1;
+    o_dep[i] = -1;
+  }
+  for (int e = threadIdx.x; e < km; e += blockDim.x) {
+    const int p = e / m, j = e - p * m;
+    const int u = s_own[e];
+    const int nid = s_new[u];
+    o_gam[s_ord[p] * m + j] = nid;
+    if (s_lcp[p] <= j && nid >= 0) {
+      o_tok[nid] = s_tok[s_ord[p] * m + j];
+      o_dep[nid] = j;
+      o_par[nid] = (j > 0) ? s_new[s_own[e - 1]] : -1;
+    }
+  }
+  if (o_mask) {
+    for (int64_t i = threadIdx.x; i < (int64_t)cap * mask_words; i += blockDim.x) o_mask[i] = 0u;
+    __syncthreads();
+    for (int e = threadIdx.x; e < km; e += blockDim.x) {
+      const int p = e / m, j = e - p * m;
+      if (s_lcp[p] <= j) {
+        const int nid = s_new[s_own[e]];
+        if (nid >= 0) {
+          uint32_t* row = o_mask + (int64_t)nid * mask_words;
+          for (int jj = 0; jj <= j; ++jj) {
+            const int b = s_new[s_own[p * m + jj]];
+            atomicOr(&row[b >> 5], 1u << (b & 31));
+          }
+        }
+      }
+    }
+  }
+}
+
+}  // namespace
+
+sense_status launch_gather(const int32_t* spans, int64_t n, int m, const int32_t* idx, int q,
+                           int k, const int32_t* anchor, int n_keep, int force,
+                           int32_t* out_spans, uint32_t* status, cudaStream_t s) {
+  const int threads = ((k + 31) / 32) * 32;
+  LaunchScope ls(K_GATHER, s);
+  gather_kernel<<<q, threads, 0, s>>>(spans, n, m, idx, k, anchor, n_keep, force, out_spans,
+                                      status);
+  return cuda_check(cudaGetLastError(), "launch gather");
+}
+
+size_t tree_smem_bytes(int k, int m) {
+  int kp = 1;
+  while (kp < k) kp <<= 1;
+  return sizeof(int) * ((size_t)4 * k * m + kp + 2 * (size_t)k);
+}
+
+sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int mask_bits,
+                         int32_t* num_nodes, int32_t* tokens, int32_t* parent, int32_t* depth,
+                         int32_t* gamma, uint32_t* mask, uint32_t* status, cudaStream_t s) {
+  const size_t smem = tree_smem_bytes(k, m);
+  cudaError_t e = cudaFuncSetAttribute(tree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(tree)");
+  const int words = (cap + 31) / 32;
+  LaunchScope ls(K_TREE, s);
+  tree_kernel<<<q, kTreeThreads, smem, s>>>(spans, k, m, cap, words, num_nodes, tokens, parent,
+                                            depth, gamma, mask_bits ? mask : nullptr, status);
+  return cuda_check(cudaGetLastError(), "launch tree");
+}
+
+}  // namespace sense

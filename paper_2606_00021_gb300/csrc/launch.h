@@ -1,0 +1,91 @@
+// Internal launch interface between the C-ABI layer and the kernel files.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "sense.h"
+
+namespace sense {
+
+// The key scan visits rows in tiles of kTileRows.  Every kSampleStride-th
+// tile forms the sample from which a per-query score threshold is taken;
+// the remaining tiles are scanned against that threshold.
+constexpr int kTileRows = 128;
+constexpr int kSampleStride = 16;
+
+enum ScanMode { SCAN_ALL = 0, SCAN_SAMPLE = 1, SCAN_REST = 2 };
+
+// Number of sample rows / rest rows for n keys (including the padding rows
+// of a partial last tile).
+inline int64_t num_tiles(int64_t n) { return (n + kTileRows - 1) / kTileRows; }
+inline int64_t sample_tiles(int64_t n) { return (num_tiles(n) + kSampleStride - 1) / kSampleStride; }
+inline int64_t rest_tiles(int64_t n) { return num_tiles(n) - sample_tiles(n); }
+
+// Scan `n_work` work rows (mapped to key rows by `mode`) for q <= 8 queries.
+// SCAN_SAMPLE writes every candidate key to out[qi * n_work + w];
+// SCAN_ALL / SCAN_REST append keys >= thresh[qi] (0 if thresh is null) to
+// out[qi * pool_cap + counts[qi]++].
+sense_status launch_scan_gemv(const uint16_t* keys, int64_t n, int d, const uint16_t* queries,
+                              int q, int mode, int64_t n_work, const uint64_t* thresh,
+                              uint64_t* out, uint32_t* counts, int64_t pool_cap,
+                              uint32_t* status, cudaStream_t s);
+
+// Same contract for 8 < q <= 128 queries on tcgen05 tensor cores.
+sense_status launch_scan_tc(const uint16_t* keys, int64_t n, int d, const uint16_t* queries,
+                            int q, int mode, int64_t n_work, const uint64_t* thresh,
+                            uint64_t* out, uint32_t* counts, int64_t pool_cap, uint32_t* status,
+                            cudaStream_t s);
+size_t scan_tc_smem_bytes(int d, int q);
+
+// Per query: exact k-th largest score code among the s_len sample keys ->
+// thresh[qi] = code << 32; sample keys at or above it are appended to the pool.
+sense_status launch_threshold(const uint64_t* sample, int64_t s_len, int q, int k,
+                              uint64_t* thresh, uint64_t* pool, uint32_t* counts,
+                              int64_t pool_cap, uint32_t* status, cudaStream_t s);
+
+// Per query: the k largest pool keys, sorted descending -> scores, indices.
+sense_status launch_merge(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap, int q,
+                          int k, float* out_scores, int32_t* out_idx, uint32_t* status,
+                          cudaStream_t s);
+
+sense_status launch_normalize(const float* src, int64_t n, int d, uint16_t* dst, cudaStream_t s);
+
+sense_status launch_gather(const int32_t* spans, int64_t n, int m, const int32_t* idx, int q,
+                           int k, const int32_t* anchor, int n_keep, int force,
+                           int32_t* out_spans, uint32_t* status, cudaStream_t s);
+
+sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int mask_bits,
+                         int32_t* num_nodes, int32_t* tokens, int32_t* parent, int32_t* depth,
+                         int32_t* gamma, uint32_t* mask, uint32_t* status, cudaStream_t s);
+
+struct GateArgs {
+  const int32_t* tokens;
+  const int32_t* parent;
+  const int32_t* num_nodes;
+  const int32_t* gamma;
+  int q, k, m, cap;
+  const float* root_logits;
+  const float* node_logits;
+  int vocab;
+  const uint16_t* root_hidden;
+  const uint16_t* node_hidden;
+  int d;
+  float thr;
+  int kappa, window, tau;
+  int unnormalized;
+  int32_t* i_star;
+  int32_t* L_star;
+  int32_t* n_accept;
+  int32_t* accepted;
+  int32_t* next_node;
+  int32_t* next_anchor;
+  uint16_t* h_next;
+  uint8_t* G;
+  void* workspace;
+  uint32_t* status;
+};
+size_t gate_workspace_bytes(int q, int cap, int kappa);
+sense_status launch_gate(const GateArgs& a, cudaStream_t s);
+
+}  // namespace sense

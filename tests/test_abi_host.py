@@ -1,0 +1,82 @@
+"""Host-side checks of the C ABI: the library builds and loads without a GPU,
+exports every function declared in include/sense.h, and rejects invalid
+arguments before touching the device."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_00021_gb300 import _abi, _build
+    _build.build()
+    return _abi.load()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "sense.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(sense_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert len(names) >= 15
+    for n in names:
+        assert hasattr(lib, n), n
+    from paper_2606_00021_gb300 import _abi
+    assert set(names) == set(_abi.SIGNATURES), "binding and header disagree"
+
+
+def test_status_strings(lib):
+    assert lib.sense_status_string(0) == b"SENSE_OK"
+    assert lib.sense_status_string(1) == b"SENSE_ERR_INVALID_ARG"
+    assert lib.sense_status_string(6) == b"SENSE_ERR_TIMEOUT"
+    assert lib.sense_version() >= 10000
+
+
+def test_invalid_arguments_rejected_on_host(lib):
+    p = C.c_void_p(16 * 1024)  # never dereferenced: validation fails first
+    out = C.c_void_p(0)
+    # datastore: bad n, d, m, alignment, flags
+    assert lib.sense_datastore_build(p, 0, 0, 64, p, 4, 0, None, C.byref(out)) == 1
+    assert lib.sense_datastore_build(p, 0, 10, 60, p, 4, 0, None, C.byref(out)) == 1
+    assert lib.sense_datastore_build(p, 0, 10, 64, p, 33, 0, None, C.byref(out)) == 1
+    assert lib.sense_datastore_build(C.c_void_p(16 * 1024 + 2), 0, 10, 64, p, 4, 0, None,
+                                     C.byref(out)) == 1
+    assert lib.sense_datastore_build(p, 0, 10, 64, p, 4, 0x80, None, C.byref(out)) == 1
+    assert lib.sense_datastore_build(p, 0, 10, 64, p, 4, 1, None, C.byref(out)) == 1
+    assert b"SENSE_DS_NORMALIZE" in lib.sense_last_error()
+    # retrieve / gather on a NULL handle
+    assert lib.sense_retrieve_topk(None, p, 1, 1, p, p, p, 1 << 20, None) == 1
+    assert lib.sense_gather_drafts(None, p, 1, 1, None, 1, 0, p, None) == 1
+    # tree: k, m, k*m, cap, flags
+    args = (p, p, p, p, p, None, None)
+    assert lib.sense_build_tree(p, 1, 0, 4, 0, 0, *args) == 1
+    assert lib.sense_build_tree(p, 1, 4, 33, 0, 0, *args) == 1
+    assert lib.sense_build_tree(p, 1, 1024, 16, 0, 0, *args) == 1
+    assert lib.sense_build_tree(p, 1, 4, 4, -1, 0, *args) == 1
+    assert lib.sense_build_tree(p, 1, 4, 4, 0, 1, *args) == 1  # mask bits without buffer
+    # gate parameters
+    from paper_2606_00021_gb300._abi import GateParams
+    gp = GateParams(0.05, 0, 6, 0, 0)
+    ptrs = [p] * 4
+    call = lambda g, v=128, d=64: lib.sense_soft_gate(*ptrs, 1, 4, 4, 16, p, p, v, p, p, d,
+                                                      C.byref(g), *([p] * 7), None, p,
+                                                      1 << 20, None)
+    assert call(gp) == 1
+    assert call(GateParams(0.05, 3, 0, 0, 0)) == 1
+    assert call(GateParams(0.05, 3, 6, -1, 0)) == 1
+    assert call(GateParams(0.05, 3, 6, 0, 0), v=130) == 1
+    assert call(GateParams(0.05, 3, 6, 0, 0), d=60) == 1
+    assert call(GateParams(float("nan"), 3, 6, 0, 0)) == 1
+
+
+def test_workspace_sizes(lib):
+    assert lib.sense_retrieve_workspace_bytes(None, 1, 1) == 0
+    assert lib.sense_soft_gate_workspace_bytes(2, 64, 3) >= 2 * 65 * 4
+    assert lib.sense_soft_gate_workspace_bytes(2, 64, 3) % 256 == 0
