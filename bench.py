@@ -257,9 +257,14 @@ def main():
     ap.add_argument("--workload", default=DEFAULT, choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--n-keys", type=int, default=0,
+                    help="override the store size (small cases for profiler captures)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
-    cfg = WORKLOADS[args.workload]
+    cfg = dict(WORKLOADS[args.workload])
+    if args.n_keys > 0:
+        cfg["n"] = args.n_keys
+        args.workload = f"{args.workload}@n={args.n_keys}"
     if args.impl == "reference":
         run_reference(args, cfg, args.workload)
         return
@@ -328,6 +333,13 @@ def main():
     peak, peak_kind = peaks()
     step_bytes = scan_bytes_per_step  # gate/tree bytes are <0.1% of the scan here
 
+    # draft tree size (nodes per query) over a few steps, for draft tokens/s
+    nodes = []
+    for it in range(16):
+        pipe.step(queries[it % nq], gate_sets[it % 4])
+        nodes.append(pipe.tree["num_nodes"].float().mean().item())
+    mean_nodes = float(np.mean(nodes))
+
     # end to end through the C ABI with host buffers
     e2e_steps = min(args.e2e_steps, args.steps)
     h_query = torch.empty_like(queries[0], device="cpu").pin_memory()
@@ -336,7 +348,6 @@ def main():
     h_gate = [t.to("cpu").pin_memory() for t in gsrc]
     d_query = torch.empty_like(queries[0])
     d_gate = [torch.empty_like(t) for t in gsrc]
-    outs = ["scores", "idx"]
     h_scores = torch.empty(q, cfg["k"], dtype=torch.float32).pin_memory()
     h_idx = torch.empty(q, cfg["k"], dtype=torch.int32).pin_memory()
     h_acc = torch.empty(q, cfg["m"], dtype=torch.int32).pin_memory()
@@ -372,7 +383,6 @@ def main():
         base = cpu_baseline(cfg, keys, spans, queries, gate_sets)
 
     if rank == 0:
-        mean_nodes = None
         line = {
             "metric": "hidden-state top-k retrieval queries/s (whole drafting step)",
             "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
@@ -385,6 +395,8 @@ def main():
                        "l2": "inputs larger than L2: the 8.6 GB store is streamed every step",
                        "parallelism": f"replicas x{world}"},
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,
+            "draft_tokens_per_s": value * mean_nodes,
+            "mean_tree_nodes": mean_nodes,
             "roofline": {"bound": "hbm", "kernel": scan_name, "achieved": achieved,
                          "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                          "peak_kind": peak_kind, "traffic": NCU_TRAFFIC.get(scan_name),

@@ -197,7 +197,7 @@ def sense_build_tree(spans: torch.Tensor, node_cap: int = 0, mask_bits: bool = F
     q, k, m = spans.shape
     cap = node_cap if node_cap > 0 else k * m
     dev = spans.device
-    o = outs or {}
+    o = outs if outs is not None else {}
     o.setdefault("num_nodes", _i32((q,), dev))
     o.setdefault("tokens", _i32((q, cap), dev))
     o.setdefault("parent", _i32((q, cap), dev))
@@ -238,7 +238,7 @@ def sense_soft_gate(tree: dict, root_logits: torch.Tensor, node_logits: torch.Te
     if node_logits.shape != (q, cap, vocab) or node_hidden.shape != (q, cap, d):
         raise ValueError("node_logits / node_hidden must be [q, cap, V] / [q, cap, d]")
     dev = root_logits.device
-    o = outs or {}
+    o = outs if outs is not None else {}
     for key in ("i_star", "L_star", "n_accept", "next_node", "next_anchor"):
         o.setdefault(key, _i32((q,), dev))
     o.setdefault("accepted", _i32((q, m), dev))
