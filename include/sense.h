@@ -144,6 +144,33 @@ sense_status sense_retrieve_topk(const sense_datastore* ds, const uint16_t* quer
                                  int32_t k, float* out_scores, int32_t* out_idx,
                                  void* workspace, size_t workspace_bytes, sense_stream_t stream);
 
+/*
+ * Same search as sense_retrieve_topk, for callers that cannot allocate
+ * device memory and have no workspace to pass: for example a serving
+ * process whose device memory is all handed out in advance by another
+ * allocator, or a plug-in whose host application exposes no device
+ * allocator and forbids cudaMalloc (it can synchronise the device and fail
+ * mid-request).  The paper has no counterpart to this entry point.
+ *
+ * Scratch comes from one file-scope device array of
+ * SENSE_NOALLOC_SCRATCH_BYTES bytes, held by every GPU that loads the
+ * library until the process exits.  This function calls no cudaMalloc,
+ * cudaFree or other allocating routine.  Its first call on a device looks
+ * up the array's device address (cudaGetSymbolAddress) with that device
+ * current; make that first call before any stream capture.  A request whose
+ * workspace (sense_retrieve_workspace_bytes) exceeds the array minus 256
+ * bytes is rejected with SENSE_ERR_UNSUPPORTED.  All calls share the array,
+ * which keeps the last call's contents (the counters that must start at zero
+ * are cleared by every call); calls that overlap on the GPU race on it, so
+ * order them on one stream.  Device-side checks of this function record
+ * into a status word inside the array, not the one sense_device_status reads.
+ * Arguments, outputs and results are those of sense_retrieve_topk.
+ */
+#define SENSE_NOALLOC_SCRATCH_BYTES (32u << 20)
+sense_status sense_retrieve_topk_noalloc(const sense_datastore* ds, const uint16_t* queries,
+                                         int32_t q, int32_t k, float* out_scores,
+                                         int32_t* out_idx, sense_stream_t stream);
+
 /* ---------------------------------------------------------------------- */
 /* a4. Span gather                                                          */
 /* ---------------------------------------------------------------------- */

@@ -174,6 +174,28 @@ def sense_retrieve_topk(ds: Datastore, queries: torch.Tensor, k: int, out_scores
     return out_scores, out_idx
 
 
+def sense_retrieve_topk_noalloc(ds: Datastore, queries: torch.Tensor, k: int, out_scores=None,
+                                out_idx=None, stream=None):
+    """Top-k search whose scratch is the library's fixed static device array.
+
+    For callers that cannot allocate device memory or pass a workspace; the
+    C entry point allocates nothing (only the outputs are allocated here when
+    not given).  Requests larger than the static scratch raise SenseError."""
+    _need(queries, "queries", torch.bfloat16, 2)
+    q = queries.shape[0]
+    if queries.shape[1] != ds.d:
+        raise ValueError("queries must have d columns")
+    dev = queries.device
+    if out_scores is None:
+        out_scores = torch.empty(q, k, dtype=torch.float32, device=dev)
+    if out_idx is None:
+        out_idx = _i32((q, k), dev)
+    _check(lib().sense_retrieve_topk_noalloc(C.c_void_p(ds.handle), queries.data_ptr(), q, k,
+                                             out_scores.data_ptr(), out_idx.data_ptr(),
+                                             C.c_void_p(_stream(stream))))
+    return out_scores, out_idx
+
+
 def sense_gather_drafts(ds: Datastore, idx: torch.Tensor, anchor=None, n_keep=None,
                         force_anchor: bool = False, out=None, stream=None) -> torch.Tensor:
     """Candidate spans [q, n_keep, m] int32 for retrieved indices idx [q, k]."""

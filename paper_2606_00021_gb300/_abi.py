@@ -26,6 +26,7 @@ SIGNATURES = {
     "sense_datastore_keys": (c_p, [c_p]),
     "sense_retrieve_workspace_bytes": (c_size, [c_p, c_i32, c_i32]),
     "sense_retrieve_topk": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_p, c_p, c_size, c_p]),
+    "sense_retrieve_topk_noalloc": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_p, c_p]),
     "sense_gather_drafts": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_i32, c_u32, c_p, c_p]),
     "sense_build_tree": (c_i32, [c_p, c_i32, c_i32, c_i32, c_i32, c_u32, c_p, c_p, c_p, c_p,
                                  c_p, c_p, c_p]),

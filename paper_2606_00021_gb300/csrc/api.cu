@@ -12,16 +12,6 @@
 #include "common.cuh"
 #include "launch.h"
 
-struct sense_datastore {
-  const uint16_t* keys;  // bf16 [n, d] in use
-  uint16_t* owned;       // normalised copy owned by the handle, or null
-  const int32_t* spans;  // [n, m]
-  int64_t n;
-  int32_t d;
-  int32_t m;
-  int device;
-};
-
 namespace sense {
 
 namespace {
@@ -158,17 +148,8 @@ sense_status launch_normalize(const float* src, int64_t n, int d, uint16_t* dst,
 // Retrieval plan
 // ---------------------------------------------------------------------------
 namespace {
-struct RetrievePlan {
-  bool tc;          // tensor-core scan
-  int group;        // queries per pass over the keys
-  bool sampling;    // sample-threshold pass enabled
-  int64_t s_rows;   // sample work rows
-  int64_t r_rows;   // rest work rows
-  int64_t pool_cap; // pool slots per query
-  size_t off_counts, off_thresh, off_sample, off_pool, total;
-};
-
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+}  // namespace
 
 RetrievePlan make_plan(const sense_datastore* ds, int q, int k) {
   RetrievePlan p{};
@@ -193,6 +174,7 @@ RetrievePlan make_plan(const sense_datastore* ds, int q, int k) {
   return p;
 }
 
+namespace {
 sense_status check_ds(const sense_datastore* ds) {
   if (!ds) return fail(SENSE_ERR_INVALID_ARG, "datastore handle is NULL");
   if (ds->device != current_device())

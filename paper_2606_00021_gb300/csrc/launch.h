@@ -6,6 +6,17 @@
 
 #include "sense.h"
 
+// Datastore handle (opaque to callers of the C ABI).
+struct sense_datastore {
+  const uint16_t* keys;  // bf16 [n, d] in use
+  uint16_t* owned;       // normalised copy owned by the handle, or null
+  const int32_t* spans;  // [n, m]
+  int64_t n;
+  int32_t d;
+  int32_t m;
+  int device;
+};
+
 namespace sense {
 
 // The key scan visits rows in tiles of kTileRows.  Every kSampleStride-th
@@ -21,6 +32,18 @@ enum ScanMode { SCAN_ALL = 0, SCAN_SAMPLE = 1, SCAN_REST = 2 };
 inline int64_t num_tiles(int64_t n) { return (n + kTileRows - 1) / kTileRows; }
 inline int64_t sample_tiles(int64_t n) { return (num_tiles(n) + kSampleStride - 1) / kSampleStride; }
 inline int64_t rest_tiles(int64_t n) { return num_tiles(n) - sample_tiles(n); }
+
+// How one retrieval call splits its work and its workspace.
+struct RetrievePlan {
+  bool tc;           // tensor-core scan
+  int group;         // queries per pass over the keys
+  bool sampling;     // sample-threshold pass enabled
+  int64_t s_rows;    // sample work rows
+  int64_t r_rows;    // rest work rows
+  int64_t pool_cap;  // pool slots per query
+  size_t off_counts, off_thresh, off_sample, off_pool, total;
+};
+RetrievePlan make_plan(const sense_datastore* ds, int q, int k);
 
 // Scan `n_work` work rows (mapped to key rows by `mode`) for q <= 8 queries.
 // SCAN_SAMPLE writes every candidate key to out[qi * n_work + w];
