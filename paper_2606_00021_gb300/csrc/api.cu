@@ -30,7 +30,7 @@ std::vector<ProfRec> g_prof;
 std::vector<cudaEvent_t> g_ev_pool;
 const char* const kKernelNames[K_COUNT] = {
     "normalize", "scan_gemv", "scan_tc", "threshold", "merge",
-    "gather",    "tree",      "gate_rows", "gate_decide"};
+    "gather",    "tree",      "gate_rows", "gate_decide", "pad_queries"};
 
 cudaEvent_t take_event() {
   if (!g_ev_pool.empty()) {
@@ -155,7 +155,6 @@ RetrievePlan make_plan(const sense_datastore* ds, int q, int k) {
   RetrievePlan p{};
   p.tc = q > 8;
   p.group = p.tc ? (q < 128 ? q : 128) : q;
-  if (p.tc) p.group = 8;  // interim: tensor path not wired yet
   p.s_rows = sample_tiles(ds->n) * (int64_t)kTileRows;
   p.r_rows = rest_tiles(ds->n) * (int64_t)kTileRows;
   p.sampling = sample_tiles(ds->n) >= 4 && p.s_rows >= 4LL * k && p.s_rows >= 2048;
@@ -170,8 +169,61 @@ RetrievePlan make_plan(const sense_datastore* ds, int q, int k) {
   if (p.sampling) off = align256(off + sizeof(uint64_t) * g * (size_t)p.s_rows);
   p.off_pool = off;
   off = align256(off + sizeof(uint64_t) * g * (size_t)p.pool_cap);
+  p.off_qpad = off;
+  if (p.tc) off = align256(off + sizeof(uint16_t) * (size_t)((g + 15) / 16 * 16) * ds->d);
   p.total = off;
   return p;
+}
+
+sense_status run_retrieve(const RetrievePlan& p, const sense_datastore* ds,
+                          const uint16_t* queries, int q, int k, float* out_scores,
+                          int32_t* out_idx, char* ws, uint32_t* status, cudaStream_t stream) {
+  uint32_t* counts = reinterpret_cast<uint32_t*>(ws + p.off_counts);
+  uint64_t* thresh = reinterpret_cast<uint64_t*>(ws + p.off_thresh);
+  uint64_t* sample = reinterpret_cast<uint64_t*>(ws + p.off_sample);
+  uint64_t* pool = reinterpret_cast<uint64_t*>(ws + p.off_pool);
+  uint16_t* qpad = reinterpret_cast<uint16_t*>(ws + p.off_qpad);
+  const int64_t n = ds->n;
+  const int d = ds->d;
+  sense_status st = SENSE_OK;
+  for (int g0 = 0; g0 < q; g0 += p.group) {
+    const int gq = (q - g0 < p.group) ? (q - g0) : p.group;
+    const int nq = (gq + 15) / 16 * 16;
+    const uint16_t* qg = queries + (int64_t)g0 * d;
+    st = cuda_check(cudaMemsetAsync(counts, 0, sizeof(uint32_t) * gq, stream), "clear pool counts");
+    if (st != SENSE_OK) return st;
+    if (p.tc) {
+      st = launch_pad_queries(qg, gq, d, qpad, nq, stream);
+      if (st != SENSE_OK) return st;
+    }
+    // scan(mode): the work set of `mode` against `thr`, into `out`
+    auto scan = [&](int mode, const uint64_t* thr, uint64_t* out, int64_t cap) -> sense_status {
+      const int64_t halves = (mode == SCAN_SAMPLE) ? sample_tiles(n)
+                           : (mode == SCAN_REST)   ? rest_tiles(n)
+                                                   : num_tiles(n);
+      if (p.tc)
+        return launch_scan_tc(ds->keys, n, d, qpad, gq, nq, mode, halves, thr, out, counts, cap,
+                              status, stream);
+      const int64_t rows = (mode == SCAN_ALL) ? n : halves * kTileRows;
+      return launch_scan_gemv(ds->keys, n, d, qg, gq, mode, rows, thr, out, counts, cap, status,
+                              stream);
+    };
+    if (p.sampling) {
+      st = scan(SCAN_SAMPLE, nullptr, sample, 0);
+      if (st != SENSE_OK) return st;
+      st = launch_threshold(sample, p.s_rows, gq, k, thresh, pool, counts, p.pool_cap, status,
+                            stream);
+      if (st != SENSE_OK) return st;
+      st = scan(SCAN_REST, thresh, pool, p.pool_cap);
+    } else {
+      st = scan(SCAN_ALL, nullptr, pool, p.pool_cap);
+    }
+    if (st != SENSE_OK) return st;
+    st = launch_merge(pool, counts, p.pool_cap, gq, k, out_scores + (int64_t)g0 * k,
+                      out_idx + (int64_t)g0 * k, status, stream);
+    if (st != SENSE_OK) return st;
+  }
+  return SENSE_OK;
 }
 
 namespace {
@@ -303,40 +355,16 @@ sense_status sense_retrieve_topk(const sense_datastore* ds, const uint16_t* quer
   if (k < 1 || k > SENSE_MAX_K || (int64_t)k > ds->n)
     return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, min(n=%lld, %d)]", k, (long long)ds->n, SENSE_MAX_K);
   if (!aligned(queries, 16)) return fail(SENSE_ERR_INVALID_ARG, "queries must be 16-byte aligned");
+  if (q > 8 && ds->n > 2147483647LL - 1024)
+    return fail(SENSE_ERR_UNSUPPORTED, "batched (q > 8) retrieval supports n <= 2^31 - 1025");
   if (!aligned(workspace, 256)) return fail(SENSE_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
   const RetrievePlan p = make_plan(ds, q, k);
   if (workspace_bytes < p.total)
     return fail(SENSE_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", workspace_bytes, p.total);
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
-  char* ws = static_cast<char*>(workspace);
-  uint32_t* counts = reinterpret_cast<uint32_t*>(ws + p.off_counts);
-  uint64_t* thresh = reinterpret_cast<uint64_t*>(ws + p.off_thresh);
-  uint64_t* sample = reinterpret_cast<uint64_t*>(ws + p.off_sample);
-  uint64_t* pool = reinterpret_cast<uint64_t*>(ws + p.off_pool);
-  for (int g0 = 0; g0 < q; g0 += p.group) {
-    const int gq = (q - g0 < p.group) ? (q - g0) : p.group;
-    const uint16_t* qg = queries + (int64_t)g0 * ds->d;
-    st = cuda_check(cudaMemsetAsync(counts, 0, sizeof(uint32_t) * gq, stream), "clear pool counts");
-    if (st != SENSE_OK) return st;
-    if (p.sampling) {
-      st = launch_scan_gemv(ds->keys, ds->n, ds->d, qg, gq, SCAN_SAMPLE, p.s_rows, nullptr,
-                            sample, counts, 0, status, stream);
-      if (st != SENSE_OK) return st;
-      st = launch_threshold(sample, p.s_rows, gq, k, thresh, pool, counts, p.pool_cap, status, stream);
-      if (st != SENSE_OK) return st;
-      st = launch_scan_gemv(ds->keys, ds->n, ds->d, qg, gq, SCAN_REST, p.r_rows, thresh, pool,
-                            counts, p.pool_cap, status, stream);
-    } else {
-      st = launch_scan_gemv(ds->keys, ds->n, ds->d, qg, gq, SCAN_ALL, ds->n, nullptr, pool,
-                            counts, p.pool_cap, status, stream);
-    }
-    if (st != SENSE_OK) return st;
-    st = launch_merge(pool, counts, p.pool_cap, gq, k, out_scores + (int64_t)g0 * k,
-                      out_idx + (int64_t)g0 * k, status, stream);
-    if (st != SENSE_OK) return st;
-  }
-  return SENSE_OK;
+  return run_retrieve(p, ds, queries, q, k, out_scores, out_idx, static_cast<char*>(workspace),
+                      status, stream);
 }
 
 sense_status sense_gather_drafts(const sense_datastore* ds, const int32_t* idx, int32_t q,

@@ -33,6 +33,7 @@ enum KernelId {
   K_TREE,
   K_GATE_ROWS,
   K_GATE_DECIDE,
+  K_PAD_QUERIES,
   K_COUNT
 };
 

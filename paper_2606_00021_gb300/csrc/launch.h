@@ -41,9 +41,14 @@ struct RetrievePlan {
   int64_t s_rows;    // sample work rows
   int64_t r_rows;    // rest work rows
   int64_t pool_cap;  // pool slots per query
-  size_t off_counts, off_thresh, off_sample, off_pool, total;
+  size_t off_counts, off_thresh, off_sample, off_pool, off_qpad, total;
 };
 RetrievePlan make_plan(const sense_datastore* ds, int q, int k);
+
+// Runs one retrieval call with its workspace at `ws` (laid out by `p`).
+sense_status run_retrieve(const RetrievePlan& p, const sense_datastore* ds,
+                          const uint16_t* queries, int q, int k, float* out_scores,
+                          int32_t* out_idx, char* ws, uint32_t* status, cudaStream_t s);
 
 // Scan `n_work` work rows (mapped to key rows by `mode`) for q <= 8 queries.
 // SCAN_SAMPLE writes every candidate key to out[qi * n_work + w];
@@ -54,12 +59,16 @@ sense_status launch_scan_gemv(const uint16_t* keys, int64_t n, int d, const uint
                               uint64_t* out, uint32_t* counts, int64_t pool_cap,
                               uint32_t* status, cudaStream_t s);
 
-// Same contract for 8 < q <= 128 queries on tcgen05 tensor cores.
-sense_status launch_scan_tc(const uint16_t* keys, int64_t n, int d, const uint16_t* queries,
-                            int q, int mode, int64_t n_work, const uint64_t* thresh,
+// Same contract on tcgen05 tensor cores for qg <= nq <= 128 queries held in
+// `qpad` ([nq, d] bf16, rows >= qg zero); the work set is n_half 128-row
+// tiles selected by `mode`.
+sense_status launch_scan_tc(const uint16_t* keys, int64_t n, int d, const uint16_t* qpad, int qg,
+                            int nq, int mode, int64_t n_half, const uint64_t* thresh,
                             uint64_t* out, uint32_t* counts, int64_t pool_cap, uint32_t* status,
                             cudaStream_t s);
-size_t scan_tc_smem_bytes(int d, int q);
+sense_status launch_pad_queries(const uint16_t* src, int qg, int d, uint16_t* dst, int nq,
+                                cudaStream_t s);
+size_t scan_tc_smem_bytes(int d, int nq);
 
 // Per query: exact k-th largest score code among the s_len sample keys ->
 // thresh[qi] = code << 32; sample keys at or above it are appended to the pool.

@@ -76,6 +76,8 @@ extern "C" sense_status sense_retrieve_topk_noalloc(const sense_datastore* ds,
     return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, min(n=%lld, %d)]", k,
                 (long long)ds->n, SENSE_MAX_K);
   if (!is_aligned(queries, 16)) return fail(SENSE_ERR_INVALID_ARG, "queries must be 16-byte aligned");
+  if (q > 8 && ds->n > 2147483647LL - 1024)
+    return fail(SENSE_ERR_UNSUPPORTED, "batched (q > 8) retrieval supports n <= 2^31 - 1025");
   const RetrievePlan p = make_plan(ds, q, k);
   if (p.total > kNoallocScratchBytes - kStatusBytes)
     return fail(SENSE_ERR_UNSUPPORTED,
@@ -86,35 +88,8 @@ extern "C" sense_status sense_retrieve_topk_noalloc(const sense_datastore* ds,
   st = scratch_address(&base);
   if (st != SENSE_OK) return st;
   uint32_t* status = reinterpret_cast<uint32_t*>(base);
-  char* ws = base + kStatusBytes;
-  uint32_t* counts = reinterpret_cast<uint32_t*>(ws + p.off_counts);
-  uint64_t* thresh = reinterpret_cast<uint64_t*>(ws + p.off_thresh);
-  uint64_t* sample = reinterpret_cast<uint64_t*>(ws + p.off_sample);
-  uint64_t* pool = reinterpret_cast<uint64_t*>(ws + p.off_pool);
   st = cuda_check(cudaMemsetAsync(status, 0, sizeof(uint32_t), stream), "clear status word");
   if (st != SENSE_OK) return st;
-  for (int g0 = 0; g0 < q; g0 += p.group) {
-    const int gq = (q - g0 < p.group) ? (q - g0) : p.group;
-    const uint16_t* qg = queries + (int64_t)g0 * ds->d;
-    st = cuda_check(cudaMemsetAsync(counts, 0, sizeof(uint32_t) * gq, stream), "clear pool counts");
-    if (st != SENSE_OK) return st;
-    if (p.sampling) {
-      st = launch_scan_gemv(ds->keys, ds->n, ds->d, qg, gq, SCAN_SAMPLE, p.s_rows, nullptr,
-                            sample, counts, 0, status, stream);
-      if (st != SENSE_OK) return st;
-      st = launch_threshold(sample, p.s_rows, gq, k, thresh, pool, counts, p.pool_cap, status,
-                            stream);
-      if (st != SENSE_OK) return st;
-      st = launch_scan_gemv(ds->keys, ds->n, ds->d, qg, gq, SCAN_REST, p.r_rows, thresh, pool,
-                            counts, p.pool_cap, status, stream);
-    } else {
-      st = launch_scan_gemv(ds->keys, ds->n, ds->d, qg, gq, SCAN_ALL, ds->n, nullptr, pool,
-                            counts, p.pool_cap, status, stream);
-    }
-    if (st != SENSE_OK) return st;
-    st = launch_merge(pool, counts, p.pool_cap, gq, k, out_scores + (int64_t)g0 * k,
-                      out_idx + (int64_t)g0 * k, status, stream);
-    if (st != SENSE_OK) return st;
-  }
-  return SENSE_OK;
+  return run_retrieve(p, ds, queries, q, k, out_scores, out_idx, base + kStatusBytes, status,
+                      stream);
 }

@@ -53,8 +53,33 @@ def test_retrieve_matches_oracle(S, n, d, q, k, clusters):
 
 
 @cuda
+@pytest.mark.parametrize("n,d,q,k,clusters", [
+    (4096, 4096, 16, 8, 64),        # tensor path, one pass, no sampling
+    (5000, 512, 9, 17, 16),         # q padded 9 -> 16, ragged tile
+    (131072 + 77, 512, 33, 32, 256),  # sampled, nq = 48
+    (200003, 256, 64, 64, 512),     # sampled, q = 64
+    (70000, 1024, 128, 5, 64),      # full 128-query group
+    (66000, 320, 130, 16, 64),      # two groups (128 + 2), d not a multiple of 64
+])
+def test_retrieve_tensor_path_matches_oracle(S, n, d, q, k, clusters):
+    dev = torch.device("cuda")
+    keys = synth.clustered_unit_keys(n, d, clusters, seed=n % 89, device=dev)
+    spans = synth.spans_uniform(n, 4, 32000, seed=1, device=dev)
+    qs, _ = synth.noisy_queries(keys, q, seed=n % 11)
+    ds = S.sense_datastore_build(keys, spans)
+    sc, ix = S.sense_retrieve_topk(ds, qs, k)
+    torch.cuda.synchronize()
+    assert _clear(S) == 0
+    full = O.scores(bits(keys), bits(qs))
+    for qi in range(q):
+        check_topk(host(sc[qi]), host(ix[qi]), full[qi], k)
+
+
+@cuda
 @pytest.mark.parametrize("n,d,q,k", [(20000, 256, 1, 64), (20000, 256, 8, 17),
-                                     (150000, 128, 3, 100), (4096, 64, 2, 4096 // 4)])
+                                     (150000, 128, 3, 100), (4096, 64, 2, 4096 // 4),
+                                     (20000, 256, 16, 64), (150000, 192, 40, 100),
+                                     (9000, 64, 129, 33)])
 def test_retrieve_lattice_bit_exact(S, n, d, q, k):
     """Lattice entries make every fp32 sum exact: scores, order and ties
     (lower index first) must equal the oracle bit for bit."""
