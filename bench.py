@@ -30,19 +30,8 @@ if ROOT not in sys.path:
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-WORKLOADS = {
-    # name: n, d, q, k, m, vocab, cap, clusters, zipf
-    "llama7b_1m": dict(n=1048576, d=4096, q=1, k=32, m=16, vocab=32000, cap=64,
-                       clusters=1024, zipf=True, distinct=512),
-    "tiny_4k": dict(n=4096, d=4096, q=8, k=8, m=8, vocab=32000, cap=64, clusters=64,
-                    zipf=False, distinct=8),
-    "qwen7b_4m": dict(n=4194304, d=3584, q=16, k=64, m=16, vocab=152064, cap=128,
-                      clusters=4096, zipf=True, distinct=64),
-    "llama70b_8m": dict(n=8388608, d=8192, q=1, k=64, m=16, vocab=128256, cap=64,
-                        clusters=8192, zipf=True, distinct=16),
-    "sweep_2m_k64": dict(n=2097152, d=4096, q=64, k=64, m=16, vocab=128256, cap=0,
-                         clusters=2048, zipf=True, distinct=64),
-}
+from synth.workloads import WORKLOADS  # noqa: E402
+
 DEFAULT = "llama7b_1m"
 GATE = dict(gamma=0.05, topk=3, window=6, tau=0)
 # dram bytes (read + write) per launch of the dominant kernel from one ncu
@@ -285,13 +274,16 @@ def main():
     S.lib()
 
     keys, spans, queries = make_workload(cfg, dev, seed=rank)
-    gate_sets = make_gate_inputs(cfg, dev, sets=4, seed=100 + rank)
+    cap = cfg["cap"] if cfg["cap"] > 0 else cfg["k"] * cfg["m"]
+    gate_bytes = cfg["q"] * (cap + 1) * cfg["vocab"] * 4
+    n_sets = 4 if gate_bytes < (2 << 30) else 1
+    gate_sets = make_gate_inputs(cfg, dev, sets=n_sets, seed=100 + rank)
     ds = S.sense_datastore_build(keys, spans)
     pipe = Pipeline(S, ds, cfg, dev)
     nq = queries.shape[0]
 
     for it in range(args.warmup):
-        pipe.step(queries[it % nq], gate_sets[it % 4])
+        pipe.step(queries[it % nq], gate_sets[it % n_sets])
     torch.cuda.synchronize()
     if S.sense_device_status(clear=True) != 0:
         raise RuntimeError("device status bits set after warm-up")
@@ -308,7 +300,7 @@ def main():
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for it in range(args.steps):
-        pipe.step(queries[it % nq], gate_sets[it % 4])
+        pipe.step(queries[it % nq], gate_sets[it % n_sets])
     e1.record(stream)
     torch.cuda.synchronize()
     if dist:
@@ -336,12 +328,14 @@ def main():
     # draft tree size (nodes per query) over a few steps, for draft tokens/s
     nodes = []
     for it in range(16):
-        pipe.step(queries[it % nq], gate_sets[it % 4])
+        pipe.step(queries[it % nq], gate_sets[it % n_sets])
         nodes.append(pipe.tree["num_nodes"].float().mean().item())
     mean_nodes = float(np.mean(nodes))
 
     # end to end through the C ABI with host buffers
     e2e_steps = min(args.e2e_steps, args.steps)
+    if gate_bytes > (1 << 30):
+        e2e_steps = min(e2e_steps, 10)
     h_query = torch.empty_like(queries[0], device="cpu").pin_memory()
     h_query.copy_(queries[0])
     gsrc = gate_sets[0]

@@ -167,6 +167,8 @@ RetrievePlan make_plan(const sense_datastore* ds, int q, int k) {
   off = align256(off + sizeof(uint64_t) * g);
   p.off_sample = off;
   if (p.sampling) off = align256(off + sizeof(uint64_t) * g * (size_t)p.s_rows);
+  p.off_cand = off;
+  if (p.sampling) off = align256(off + sizeof(uint64_t) * g * (size_t)chunk_count(p.s_rows) * k);
   p.off_pool = off;
   off = align256(off + sizeof(uint64_t) * g * (size_t)p.pool_cap);
   p.off_qpad = off;
@@ -181,6 +183,7 @@ sense_status run_retrieve(const RetrievePlan& p, const sense_datastore* ds,
   uint32_t* counts = reinterpret_cast<uint32_t*>(ws + p.off_counts);
   uint64_t* thresh = reinterpret_cast<uint64_t*>(ws + p.off_thresh);
   uint64_t* sample = reinterpret_cast<uint64_t*>(ws + p.off_sample);
+  uint64_t* cand = reinterpret_cast<uint64_t*>(ws + p.off_cand);
   uint64_t* pool = reinterpret_cast<uint64_t*>(ws + p.off_pool);
   uint16_t* qpad = reinterpret_cast<uint16_t*>(ws + p.off_qpad);
   const int64_t n = ds->n;
@@ -211,8 +214,8 @@ sense_status run_retrieve(const RetrievePlan& p, const sense_datastore* ds,
     if (p.sampling) {
       st = scan(SCAN_SAMPLE, nullptr, sample, 0);
       if (st != SENSE_OK) return st;
-      st = launch_threshold(sample, p.s_rows, gq, k, thresh, pool, counts, p.pool_cap, status,
-                            stream);
+      st = launch_threshold(sample, p.s_rows, gq, k, cand, thresh, pool, counts, p.pool_cap,
+                            status, stream);
       if (st != SENSE_OK) return st;
       st = scan(SCAN_REST, thresh, pool, p.pool_cap);
     } else {

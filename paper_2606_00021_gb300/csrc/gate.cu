@@ -5,12 +5,17 @@
 // predicted by the row of node gamma[i, j-1] (the root row for j = 0), so the
 // distinct rows are the root and the tree's inner nodes.  The gate therefore
 // runs in two kernels:
-//  1. gate_rows: one block per needed row streams its V fp32 logits once
-//     (128-bit loads) and produces argmax (lowest index among maxima), the
-//     entropy of softmax (online max / sum-exp / sum (x-max) exp, combined
-//     across threads in fp64: H = log Z - S / Z) and the top-kappa list
-//     under the order (logit desc, index asc).  A node is an inner node iff
-//     the next node in preorder is its child, so the test is O(1).
+//  1. gate_rows: each needed row is cut into `segs` segments, one block per
+//     segment.  A block streams its V/segs fp32 logits once (eight 128-bit
+//     loads in flight per thread) and keeps, per thread, the running max,
+//     sum exp(x - max) and sum (x - max) exp(x - max) (entropy H = log Z -
+//     S / Z), the argmax (lowest index among maxima) and a top-kappa list
+//     under (logit desc, index asc); the maximum of each 32-value chunk gates
+//     the rare updates of the argmax and the list.  The block combines its
+//     threads (fp64), writes a partial, and the last block of a row to
+//     finish (an atomic counter per row) merges the segments into the row's
+//     statistics.  A node is an inner node iff the next node in preorder is
+//     its child, so the test is O(1).
 //  2. gate_decide: one block per query evaluates B_em, B_ent, B_topk, the
 //     lookahead B_con, G, the accepted prefix lengths L_i, i*, and writes
 //     the accepted tokens, the next node, its argmax (streaming that row if
@@ -24,7 +29,9 @@ namespace sense {
 namespace {
 
 constexpr int kRowThreads = 256;
+constexpr int kVec = 8;                          // float4 loads per thread per step
 constexpr int kStatsInts = 2 + SENSE_MAX_KAPPA;  // argmax, ent flag, top list
+constexpr int kMaxSegs = 16;
 
 struct ArgMax {
   float v;
@@ -33,6 +40,17 @@ struct ArgMax {
 __device__ __forceinline__ bool better(float va, int ia, float vb, int ib) {
   return va > vb || (va == vb && ia < ib);
 }
+
+// Statistics of one segment of a row (workspace).
+struct Partial {
+  double z, s;  // relative to m
+  float m;
+  float bv;
+  int bi;
+  int pad;
+  float tv[SENSE_MAX_KAPPA];
+  int ti[SENSE_MAX_KAPPA];
+};
 
 template <int KM>
 struct TopList {
@@ -66,190 +84,213 @@ struct TopList {
   }
 };
 
-struct Online {
-  float m, z, s;  // running max, sum exp(x-m), sum (x-m) exp(x-m)
-};
-__device__ __forceinline__ void online_add(Online& o, float x) {
-  if (x > o.m) {
-    const float sc = __expf(o.m - x);
-    o.s = sc * (o.s + (o.m - x) * o.z);
-    o.z = sc * o.z + 1.0f;
-    o.m = x;
-  } else {
-    const float e = __expf(x - o.m);
-    o.z += e;
-    o.s = fmaf(x - o.m, e, o.s);
-  }
-}
-
 template <int KM>
-__device__ void row_stats(const float* __restrict__ row, int vocab, int kappa, float thr,
-                          int unnormalized, int32_t* __restrict__ out) {
-  __shared__ float s_m[kRowThreads];
-  __shared__ double s_z[kRowThreads], s_s[kRowThreads];
-  __shared__ ArgMax s_w[32];
-  __shared__ int s_pick;
-
-  Online o;
-  o.m = -FLT_MAX;
-  o.z = 0.0f;
-  o.s = 0.0f;
-  float bv = -FLT_MAX;
+struct RowAcc {
+  float m = -FLT_MAX;  // running max
+  float z = 0.0f;      // sum exp(x - m)
+  float s = 0.0f;      // sum (x - m) exp(x - m)
+  float bv = -FLT_MAX; // argmax value / index (lowest index among maxima)
   int bi = 0x7fffffff;
   TopList<KM> tl;
-  tl.init();
 
-  const int n4 = vocab >> 2;
-  const float4* r4 = reinterpret_cast<const float4*>(row);
-  int c = threadIdx.x;
-  for (; c + 3 * kRowThreads < n4; c += 4 * kRowThreads) {
-    float4 x[4];
+  // Folds kVec float4 (element indices idx[u] * 4 + e, increasing) into the
+  // state.  Padding slots hold -FLT_MAX and contribute nothing.
+  __device__ __forceinline__ void add(const float4 (&x)[kVec], const int (&idx)[kVec]) {
+    float cm = -FLT_MAX;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) x[u] = __ldcs(r4 + c + u * kRowThreads);
+    for (int u = 0; u < kVec; ++u)
+      cm = fmaxf(cm, fmaxf(fmaxf(x[u].x, x[u].y), fmaxf(x[u].z, x[u].w)));
+    if (cm > m) {
+      const float sc = __expf(m - cm);
+      s = sc * (s + (m - cm) * z);
+      z = sc * z;
+      m = cm;
+    }
+    if (cm > bv) {
+      bv = cm;
+      bool found = false;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int base = (c + u * kRowThreads) * 4;
+      for (int u = 0; u < kVec; ++u) {
+        const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          if (!found && xs[e] == cm) {
+            bi = idx[u] * 4 + e;
+            found = true;
+          }
+        }
+      }
+    }
+    if (cm > tl.v[KM - 1]) {
+#pragma unroll
+      for (int u = 0; u < kVec; ++u) {
+        const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) tl.push(xs[e], idx[u] * 4 + e);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
       const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        online_add(o, xs[e]);
-        if (xs[e] > bv) {
-          bv = xs[e];
-          bi = base + e;
-        }
-        tl.push(xs[e], base + e);
+        const float t = fmaxf(xs[e] - m, -200.0f);  // exp underflows to 0 below
+        const float ex = __expf(t);
+        z += ex;
+        s = fmaf(t, ex, s);
       }
     }
   }
-  for (; c < n4; c += kRowThreads) {
-    const float4 x = __ldcs(r4 + c);
-    const float xs[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      online_add(o, xs[e]);
-      if (xs[e] > bv) {
-        bv = xs[e];
-        bi = c * 4 + e;
-      }
-      tl.push(xs[e], c * 4 + e);
-    }
-  }
+};
 
-  // Entropy: combine (m, z, s) across the block in fp64.
-  s_m[threadIdx.x] = o.m;
+__device__ __forceinline__ ArgMax warp_best(ArgMax a) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, a.v, off);
+    const int oi = __shfl_xor_sync(0xffffffffu, a.i, off);
+    if (better(ov, oi, a.v, a.i)) {
+      a.v = ov;
+      a.i = oi;
+    }
+  }
+  return a;
+}
+
+// Reduces one segment [lo4, hi4) of a row (float4 indices) over the block
+// and writes the block's partial to *out (thread 0 writes scalars).
+template <int KM>
+__device__ void segment_stats(const float* __restrict__ row, int lo4, int hi4, int kappa,
+                              Partial* out) {
+  __shared__ float s_m[kRowThreads / 32];
+  __shared__ double s_z[kRowThreads / 32], s_s[kRowThreads / 32];
+  __shared__ ArgMax s_w[kRowThreads / 32];
+  __shared__ ArgMax s_pick;
+
+  RowAcc<KM> acc;
+  acc.tl.init();
+  const float4* r4 = reinterpret_cast<const float4*>(row);
+  const float4 pad = make_float4(-FLT_MAX, -FLT_MAX, -FLT_MAX, -FLT_MAX);
+  for (int c = lo4 + threadIdx.x; c < hi4; c += kVec * kRowThreads) {
+    float4 x[kVec];
+    int idx[kVec];
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
+      idx[u] = c + u * kRowThreads;
+      x[u] = (idx[u] < hi4) ? __ldcs(r4 + idx[u]) : pad;
+    }
+    acc.add(x, idx);
+  }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  constexpr int NW = kRowThreads / 32;
+  // block max
+  float mm = acc.m;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, off));
+  if (lane == 0) s_m[wid] = mm;
   __syncthreads();
-  if (threadIdx.x < 32) {
-    float mm = -FLT_MAX;
-    for (int t = threadIdx.x; t < kRowThreads; t += 32) mm = fmaxf(mm, s_m[t]);
+  float M = s_m[0];
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, off));
-    if (threadIdx.x == 0) s_m[0] = mm;  // safe: all lanes read s_m before
+  for (int w = 1; w < NW; ++w) M = fmaxf(M, s_m[w]);
+  // rescale (z, s) to M in fp64 and sum
+  double z = 0.0, s = 0.0;
+  if (acc.z > 0.0f) {
+    const double d = (double)acc.m - (double)M;
+    const double sc = exp(d);
+    z = (double)acc.z * sc;
+    s = sc * ((double)acc.s + d * (double)acc.z);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    z += __shfl_xor_sync(0xffffffffu, z, off);
+    s += __shfl_xor_sync(0xffffffffu, s, off);
+  }
+  ArgMax a = warp_best(ArgMax{acc.bv, acc.bi});
+  if (lane == 0) {
+    s_z[wid] = z;
+    s_s[wid] = s;
+    s_w[wid] = a;
   }
   __syncthreads();
-  const double M = (double)s_m[0];
-  {
-    double z = 0.0, s = 0.0;
-    if (o.z > 0.0f) {
-      const double sc = exp((double)o.m - M);
-      z = (double)o.z * sc;
-      s = sc * ((double)o.s + ((double)o.m - M) * (double)o.z);
+  if (threadIdx.x == 0) {
+    double Z = 0.0, Sx = 0.0;
+    ArgMax b = s_w[0];
+    for (int w = 0; w < NW; ++w) {
+      Z += s_z[w];
+      Sx += s_s[w];
+      if (better(s_w[w].v, s_w[w].i, b.v, b.i)) b = s_w[w];
     }
-    s_z[threadIdx.x] = z;
-    s_s[threadIdx.x] = s;
+    out->z = Z;
+    out->s = Sx;
+    out->m = M;
+    out->bv = b.v;
+    out->bi = b.i;
   }
-  // Argmax: warp reduce then block reduce.
-  {
-    float v = bv;
-    int i = bi;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, v, off);
-      const int oi = __shfl_xor_sync(0xffffffffu, i, off);
-      if (better(ov, oi, v, i)) {
-        v = ov;
-        i = oi;
-      }
-    }
-    if ((threadIdx.x & 31) == 0) s_w[threadIdx.x >> 5] = ArgMax{v, i};
-  }
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    double z = 0.0, s = 0.0;
-    for (int t = threadIdx.x; t < kRowThreads; t += 32) {
-      z += s_z[t];
-      s += s_s[t];
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      z += __shfl_xor_sync(0xffffffffu, z, off);
-      s += __shfl_xor_sync(0xffffffffu, s, off);
-    }
-    ArgMax a = (threadIdx.x < kRowThreads / 32) ? s_w[threadIdx.x] : ArgMax{-FLT_MAX, 0x7fffffff};
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, a.v, off);
-      const int oi = __shfl_xor_sync(0xffffffffu, a.i, off);
-      if (better(ov, oi, a.v, a.i)) {
-        a.v = ov;
-        a.i = oi;
-      }
-    }
-    if (threadIdx.x == 0) {
-      const double H = log(z) - s / z;
-      const double score = unnormalized ? H : H / log((double)vocab);
-      out[0] = a.i;
-      out[1] = (score > (double)thr) ? 1 : 0;
-    }
-  }
-  // Top-kappa: kappa rounds of a block-wide best over the thread heads.
-  int head = 0;
+  // top-kappa of the segment: kappa rounds of a block-wide best over heads
   for (int r = 0; r < kappa; ++r) {
-    float v = (head < KM) ? tl.v[0] : -FLT_MAX;
-    int i = (head < KM) ? tl.i[0] : 0x7fffffff;
-    // (tl is kept shifted so that slot 0 is the current head)
-    float wv = v;
-    int wi = i;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, wv, off);
-      const int oi = __shfl_xor_sync(0xffffffffu, wi, off);
-      if (better(ov, oi, wv, wi)) {
-        wv = ov;
-        wi = oi;
-      }
+    ArgMax h = warp_best(ArgMax{acc.tl.v[0], acc.tl.i[0]});
+    __syncthreads();
+    if (lane == 0) s_w[wid] = h;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      ArgMax b = s_w[0];
+      for (int w = 1; w < NW; ++w)
+        if (better(s_w[w].v, s_w[w].i, b.v, b.i)) b = s_w[w];
+      s_pick = b;
+      out->tv[r] = b.v;
+      out->ti[r] = b.i;
     }
     __syncthreads();
-    if ((threadIdx.x & 31) == 0) s_w[threadIdx.x >> 5] = ArgMax{wv, wi};
-    __syncthreads();
-    if (threadIdx.x < 32) {
-      ArgMax a = (threadIdx.x < kRowThreads / 32) ? s_w[threadIdx.x] : ArgMax{-FLT_MAX, 0x7fffffff};
+    if (acc.tl.i[0] == s_pick.i && acc.tl.v[0] == s_pick.v) {
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, a.v, off);
-        const int oi = __shfl_xor_sync(0xffffffffu, a.i, off);
-        if (better(ov, oi, a.v, a.i)) {
-          a.v = ov;
-          a.i = oi;
-        }
+      for (int t = 0; t < KM - 1; ++t) {
+        acc.tl.v[t] = acc.tl.v[t + 1];
+        acc.tl.i[t] = acc.tl.i[t + 1];
       }
-      if (threadIdx.x == 0) {
-        s_pick = a.i;
-        out[2 + r] = a.i;
-      }
-    }
-    __syncthreads();
-    if (head < KM && tl.i[0] == s_pick) {
-#pragma unroll
-      for (int s = 0; s < KM - 1; ++s) {
-        tl.v[s] = tl.v[s + 1];
-        tl.i[s] = tl.i[s + 1];
-      }
-      tl.v[KM - 1] = -FLT_MAX;
-      tl.i[KM - 1] = 0x7fffffff;
-      ++head;
+      acc.tl.v[KM - 1] = -FLT_MAX;
+      acc.tl.i[KM - 1] = 0x7fffffff;
     }
   }
-  for (int r = kappa + threadIdx.x; r < SENSE_MAX_KAPPA; r += kRowThreads) out[2 + r] = -1;
+}
+
+// Merges the segment partials of one row into its statistics (one thread).
+__device__ void finish_row(const Partial* parts, int segs, int vocab, int kappa, float thr,
+                           int unnormalized, int32_t* __restrict__ out) {
+  float M = -FLT_MAX;
+  for (int g = 0; g < segs; ++g) M = fmaxf(M, parts[g].m);
+  double Z = 0.0, Sx = 0.0;
+  ArgMax b{-FLT_MAX, 0x7fffffff};
+  for (int g = 0; g < segs; ++g) {
+    const Partial& p = parts[g];
+    if (p.z > 0.0) {
+      const double d = (double)p.m - (double)M;
+      const double sc = exp(d);
+      Z += p.z * sc;
+      Sx += sc * (p.s + d * p.z);
+    }
+    if (better(p.bv, p.bi, b.v, b.i)) b = ArgMax{p.bv, p.bi};
+  }
+  const double H = log(Z) - Sx / Z;
+  const double score = unnormalized ? H : H / log((double)vocab);
+  out[0] = b.i;
+  out[1] = (score > (double)thr) ? 1 : 0;
+  int head[kMaxSegs];
+  for (int g = 0; g < segs; ++g) head[g] = 0;
+  for (int r = 0; r < kappa; ++r) {
+    int bg = -1;
+    ArgMax bb{-FLT_MAX, 0x7fffffff};
+    for (int g = 0; g < segs; ++g) {
+      if (head[g] >= kappa) continue;
+      const float v = parts[g].tv[head[g]];
+      const int ix = parts[g].ti[head[g]];
+      if (bg < 0 || better(v, ix, bb.v, bb.i)) {
+        bb = ArgMax{v, ix};
+        bg = g;
+      }
+    }
+    out[2 + r] = bb.i;
+    if (bg >= 0) ++head[bg];
+  }
+  for (int r = kappa; r < SENSE_MAX_KAPPA; ++r) out[2 + r] = -1;
 }
 
 template <int KM>
@@ -257,8 +298,11 @@ __global__ void __launch_bounds__(kRowThreads)
 gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ num_nodes,
                  int cap, const float* __restrict__ root_logits,
                  const float* __restrict__ node_logits, int vocab, int kappa, float thr,
-                 int unnormalized, int32_t* __restrict__ stats) {
-  const int slot = blockIdx.x;  // 0 = root, 1 + n = node n
+                 int unnormalized, int segs, int seg4, Partial* __restrict__ parts,
+                 unsigned* __restrict__ done, int32_t* __restrict__ stats) {
+  __shared__ int s_last;
+  const int slot = blockIdx.x / segs;  // 0 = root, 1 + n = node n
+  const int seg = blockIdx.x - slot * segs;
   const int q = blockIdx.y;
   const float* row;
   if (slot == 0) {
@@ -270,8 +314,28 @@ gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__
     if (!inner) return;
     row = node_logits + ((int64_t)q * cap + n) * vocab;
   }
-  row_stats<KM>(row, vocab, kappa, thr, unnormalized,
-                stats + ((int64_t)q * (cap + 1) + slot) * kStatsInts);
+  const int n4 = vocab >> 2;
+  const int lo4 = seg * seg4;
+  const int hi4 = min(n4, lo4 + seg4);
+  const int64_t rid = (int64_t)q * (cap + 1) + slot;
+  Partial* rp = parts + rid * segs;
+  segment_stats<KM>(row, lo4, hi4, kappa, rp + seg);
+  if (segs == 1) {
+    __syncthreads();
+    if (threadIdx.x == 0) finish_row(rp, 1, vocab, kappa, thr, unnormalized, stats + rid * kStatsInts);
+    return;
+  }
+  // last block of the row to finish merges the segments
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(&done[rid], 1u) == (unsigned)segs - 1u);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (threadIdx.x == 0) {
+    finish_row(rp, segs, vocab, kappa, thr, unnormalized, stats + rid * kStatsInts);
+    done[rid] = 0u;
+  }
 }
 
 constexpr int kDecideThreads = 1024;
@@ -440,27 +504,57 @@ gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats) {
   }
 }
 
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+int gate_segments(int q, int cap, int vocab) {
+  const int64_t rows = (int64_t)q * (cap + 1);
+  const int n4 = vocab >> 2;
+  int64_t segs = (4LL * sm_count() + rows - 1) / rows;
+  const int64_t by_len = n4 / 512;  // at least 8 KB of logits per segment
+  if (segs > by_len) segs = by_len;
+  if (segs > kMaxSegs) segs = kMaxSegs;
+  if (segs < 1) segs = 1;
+  return (int)segs;
+}
+
 }  // namespace
 
 size_t gate_workspace_bytes(int q, int cap, int kappa) {
   (void)kappa;
-  const size_t b = (size_t)q * (cap + 1) * kStatsInts * sizeof(int32_t);
-  return (b + 255) & ~(size_t)255;
+  const size_t rows = (size_t)q * (cap + 1);
+  size_t b = align256(rows * kStatsInts * sizeof(int32_t));
+  b += align256(rows * kMaxSegs * sizeof(Partial));
+  b += align256(rows * sizeof(unsigned));
+  return b;
 }
 
 sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
-  int32_t* stats = static_cast<int32_t*>(a.workspace);
+  const size_t rows = (size_t)a.q * (a.cap + 1);
+  char* ws = static_cast<char*>(a.workspace);
+  int32_t* stats = reinterpret_cast<int32_t*>(ws);
+  ws += align256(rows * kStatsInts * sizeof(int32_t));
+  Partial* parts = reinterpret_cast<Partial*>(ws);
+  ws += align256(rows * kMaxSegs * sizeof(Partial));
+  unsigned* done = reinterpret_cast<unsigned*>(ws);
+  const int segs = gate_segments(a.q, a.cap, a.vocab);
+  const int n4 = a.vocab >> 2;
+  const int seg4 = (n4 + segs - 1) / segs;
+  if (segs > 1) {
+    sense_status st = cuda_check(cudaMemsetAsync(done, 0, rows * sizeof(unsigned), s),
+                                 "clear gate counters");
+    if (st != SENSE_OK) return st;
+  }
   {
-    dim3 grid(a.cap + 1, a.q);
+    dim3 grid((unsigned)((a.cap + 1) * segs), a.q);
     LaunchScope ls(K_GATE_ROWS, s);
     if (a.kappa <= 4) {
-      gate_rows_kernel<4><<<grid, kRowThreads, 0, s>>>(a.parent, a.num_nodes, a.cap, a.root_logits,
-                                                       a.node_logits, a.vocab, a.kappa, a.thr,
-                                                       a.unnormalized, stats);
+      gate_rows_kernel<4><<<grid, kRowThreads, 0, s>>>(
+          a.parent, a.num_nodes, a.cap, a.root_logits, a.node_logits, a.vocab, a.kappa, a.thr,
+          a.unnormalized, segs, seg4, parts, done, stats);
     } else {
       gate_rows_kernel<SENSE_MAX_KAPPA><<<grid, kRowThreads, 0, s>>>(
           a.parent, a.num_nodes, a.cap, a.root_logits, a.node_logits, a.vocab, a.kappa, a.thr,
-          a.unnormalized, stats);
+          a.unnormalized, segs, seg4, parts, done, stats);
     }
     sense_status st = cuda_check(cudaGetLastError(), "launch gate_rows");
     if (st != SENSE_OK) return st;

@@ -41,7 +41,7 @@ struct RetrievePlan {
   int64_t s_rows;    // sample work rows
   int64_t r_rows;    // rest work rows
   int64_t pool_cap;  // pool slots per query
-  size_t off_counts, off_thresh, off_sample, off_pool, off_qpad, total;
+  size_t off_counts, off_thresh, off_sample, off_cand, off_pool, off_qpad, total;
 };
 RetrievePlan make_plan(const sense_datastore* ds, int q, int k);
 
@@ -71,9 +71,11 @@ sense_status launch_pad_queries(const uint16_t* src, int qg, int d, uint16_t* ds
 size_t scan_tc_smem_bytes(int d, int nq);
 
 // Per query: exact k-th largest score code among the s_len sample keys ->
-// thresh[qi] = code << 32; sample keys at or above it are appended to the pool.
+// thresh[qi] = code << 32; sample keys at or above it are appended to the
+// pool.  `cand` holds q * chunk_count(s_len) * k keys of scratch.
+int64_t chunk_count(int64_t s_len);
 sense_status launch_threshold(const uint64_t* sample, int64_t s_len, int q, int k,
-                              uint64_t* thresh, uint64_t* pool, uint32_t* counts,
+                              uint64_t* cand, uint64_t* thresh, uint64_t* pool, uint32_t* counts,
                               int64_t pool_cap, uint32_t* status, cudaStream_t s);
 
 // Per query: the k largest pool keys, sorted descending -> scores, indices.

@@ -2,15 +2,23 @@
 // similarity; ties to the lower key index).
 //
 // A candidate key packs (score code, ~index) into 64 bits so that the total
-// order (score desc, index asc) is plain unsigned order.  Both kernels run
-// one 1024-thread block per query and select by MSD radix: a 256-bin
-// shared-memory histogram per 8-bit digit (warp-aggregated with
-// __match_any_sync, since candidates share their high digits), a warp scan
-// to find the digit holding the k-th largest key, and early exit once that
-// digit's bin holds exactly the keys still needed.
-//  - threshold: k-th largest score code of the sample -> per-query threshold;
-//    sample keys at or above it are copied into the query's pool;
-//  - merge: the k largest keys of the pool, bitonic-sorted in shared memory.
+// order (score desc, index asc) is plain unsigned order.  Selection is an
+// MSD radix select: a 256-bin shared-memory histogram per 8-bit digit
+// (warp-aggregated with __match_any_sync, since candidates share their high
+// digits), a warp scan to find the digit holding the k-th largest key, and
+// early exit once that digit's bin holds exactly the keys still needed.
+// Keys are read from shared memory when they fit, else from global memory.
+//  - chunk_topk: sample keys are cut into chunks of kChunk; one block per
+//    (chunk, query) keeps the chunk's k largest keys.  The k largest of the
+//    whole sample are among the union of these lists, and a key left out of
+//    its chunk's list has k larger keys beside it, so it can be neither in
+//    the final top-k nor needed by the threshold below;
+//  - threshold: per query, the k-th largest score code of the lists gives
+//    the per-query threshold (a lower bound of the final k-th score: the
+//    sample is a subset of the keys); list keys at or above it enter the
+//    query's pool;
+//  - merge: per query, the k largest pool keys, bitonic-sorted in shared
+//    memory, become the output scores and indices.
 #include "common.cuh"
 #include "launch.h"
 
@@ -18,6 +26,8 @@ namespace sense {
 namespace {
 
 constexpr int kSelThreads = 1024;
+constexpr int kChunk = 8192;          // keys per first-level block (64 KB)
+constexpr int kSmemKeys = 12288;      // keys staged in shared memory (96 KB)
 
 struct Digit {
   int bucket;
@@ -67,50 +77,110 @@ __device__ void find_digit(const unsigned* hist, int remaining, Digit* out) {
   }
 }
 
-__global__ void __launch_bounds__(kSelThreads)
-threshold_kernel(const uint64_t* __restrict__ sample, int64_t s_len, int k,
+// Radix select over keys get(0..cnt): finds the digits of the k-th largest
+// key from bit 63 down to bit `low`.  On return the keys whose masked bits
+// are >= prefix are the ones to keep: exactly k of them when the search
+// stopped early or went down to bit 0 (keys distinct), at least k otherwise.
+// Returns false if fewer than k keys exist.  All threads must call it.
+template <class Get>
+__device__ bool radix_select(Get get, int64_t cnt, int k, int low, unsigned* hist, Digit* dig,
+                             uint64_t* out_prefix, uint64_t* out_mask) {
+  uint64_t prefix = 0, pmask = 0;
+  int remaining = k;
+  for (int shift = 56; shift >= low; shift -= 8) {
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+    if (threadIdx.x == 0) dig->bucket = -1;
+    __syncthreads();
+    for (int64_t i0 = 0; i0 < cnt; i0 += blockDim.x) {
+      const int64_t i = i0 + threadIdx.x;
+      const uint64_t c = (i < cnt) ? get(i) : 0ull;
+      const bool act = (i < cnt) && ((c & pmask) == prefix);
+      hist_add(hist, act, (unsigned)(c >> shift) & 255u);
+    }
+    __syncthreads();
+    find_digit(hist, remaining, dig);
+    __syncthreads();
+    if (dig->bucket < 0) {
+      *out_prefix = prefix;
+      *out_mask = pmask;
+      return false;
+    }
+    remaining -= dig->above;
+    prefix |= (uint64_t)dig->bucket << shift;
+    pmask |= 255ull << shift;
+    const bool exact = (int)hist[dig->bucket] == remaining;
+    __syncthreads();
+    if (exact) break;
+  }
+  *out_prefix = prefix;
+  *out_mask = pmask;
+  return true;
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1)
+chunk_topk_kernel(const uint64_t* __restrict__ sample, int64_t s_len, int k, int n_chunks,
+                  uint64_t* __restrict__ cand, uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];
+  __shared__ unsigned hist[256];
+  __shared__ Digit dig;
+  __shared__ unsigned n_sel;
+  const int c = blockIdx.x, q = blockIdx.y;
+  const int64_t lo = (int64_t)c * kChunk;
+  const int cnt = (int)min((int64_t)kChunk, s_len - lo);
+  const uint64_t* src = sample + (int64_t)q * s_len + lo;
+  uint64_t* dst = cand + ((int64_t)q * n_chunks + c) * k;
+  if (cnt <= k) {
+    for (int i = threadIdx.x; i < k; i += blockDim.x) dst[i] = (i < cnt) ? src[i] : 0ull;
+    return;
+  }
+  for (int i = threadIdx.x; i < cnt; i += blockDim.x) s_keys[i] = src[i];
+  __syncthreads();
+  uint64_t prefix, pmask;
+  const bool ok = radix_select([&](int64_t i) { return s_keys[i]; }, cnt, k, 0, hist, &dig,
+                               &prefix, &pmask);
+  if (!ok) {
+    if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_INTERNAL);
+    return;
+  }
+  if (threadIdx.x == 0) n_sel = 0;
+  __syncthreads();
+  for (int i = threadIdx.x; i < cnt; i += blockDim.x) {
+    const uint64_t key = s_keys[i];
+    if ((key & pmask) >= prefix) {
+      const unsigned p = atomicAdd(&n_sel, 1u);
+      if (p < (unsigned)k) dst[p] = key;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1)
+threshold_kernel(const uint64_t* __restrict__ lists, int64_t len, int k,
                  uint64_t* __restrict__ thresh, uint64_t* __restrict__ pool,
                  uint32_t* __restrict__ counts, int64_t pool_cap, uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];
   __shared__ unsigned hist[256];
   __shared__ Digit dig;
   const int q = blockIdx.x;
-  const uint64_t* src = sample + (int64_t)q * s_len;
-  uint32_t prefix = 0, pmask = 0;
-  int remaining = k;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
-    if (threadIdx.x == 0) dig.bucket = -1;
+  const uint64_t* src = lists + (int64_t)q * len;
+  const bool staged = len <= kSmemKeys;
+  if (staged) {
+    for (int64_t i = threadIdx.x; i < len; i += blockDim.x) s_keys[i] = src[i];
     __syncthreads();
-    for (int64_t i0 = 0; i0 < s_len; i0 += blockDim.x) {
-      const int64_t i = i0 + threadIdx.x;
-      const uint32_t hi = (i < s_len) ? (uint32_t)(src[i] >> 32) : 0u;
-      const bool act = (i < s_len) && ((hi & pmask) == prefix);
-      hist_add(hist, act, (hi >> shift) & 255u);
-    }
-    __syncthreads();
-    find_digit(hist, remaining, &dig);
-    __syncthreads();
-    if (dig.bucket < 0) {  // fewer than k sample keys: cannot happen when s_len >= k
-      if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_INTERNAL);
-      prefix = 0;
-      pmask = 0;
-      break;
-    }
-    remaining -= dig.above;
-    prefix |= (uint32_t)dig.bucket << shift;
-    pmask |= 255u << shift;
-    const bool exact = (int)hist[dig.bucket] == remaining;
-    __syncthreads();
-    if (exact) break;  // every key with this prefix is needed: prefix is a valid bound
   }
-  // Keys whose high word matches the prefix (or exceeds it) number >= k.
-  const uint64_t t0 = (uint64_t)prefix << 32;
+  auto get = [&](int64_t i) { return staged ? s_keys[i] : src[i]; };
+  uint64_t prefix, pmask;
+  // Score codes only (bits 63..32): the threshold needs no index order.
+  const bool ok = radix_select(get, len, k, 32, hist, &dig, &prefix, &pmask);
+  if (!ok && threadIdx.x == 0) raise_status(status, SENSE_DEVST_INTERNAL);
+  // Keys whose masked high word is >= the prefix number at least k; the
+  // threshold keeps them all (prefix's unselected low bits are zero).
+  const uint64_t t0 = ok ? prefix : 0ull;
   if (threadIdx.x == 0) thresh[q] = t0;
   uint64_t* dst = pool + (int64_t)q * pool_cap;
-  for (int64_t i0 = 0; i0 < s_len; i0 += blockDim.x) {
+  for (int64_t i0 = 0; i0 < len; i0 += blockDim.x) {
     const int64_t i = i0 + threadIdx.x;
-    const uint64_t c = (i < s_len) ? src[i] : 0ull;
-    const bool want = (i < s_len) && (c >= t0);
+    const uint64_t c = (i < len) ? get(i) : 0ull;
+    const bool want = (i < len) && c != 0ull && (c >= t0);
     const uint32_t pos = warp_append(&counts[q], want);
     if (want) {
       if ((int64_t)pos < pool_cap) dst[pos] = c;
@@ -119,10 +189,11 @@ threshold_kernel(const uint64_t* __restrict__ sample, int64_t s_len, int k,
   }
 }
 
-__global__ void __launch_bounds__(kSelThreads)
+__global__ void __launch_bounds__(kSelThreads, 1)
 merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
              int64_t pool_cap, int k, float* __restrict__ out_scores,
              int32_t* __restrict__ out_idx, uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];
   __shared__ unsigned hist[256];
   __shared__ Digit dig;
   __shared__ unsigned n_sel;
@@ -131,34 +202,14 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
   const uint64_t* src = pool + (int64_t)q * pool_cap;
   int64_t cnt = counts[q];
   if (cnt > pool_cap) cnt = pool_cap;
-
-  uint64_t prefix = 0, pmask = 0;
-  int remaining = k;
-  bool ok = true;
-  for (int shift = 56; shift >= 0; shift -= 8) {
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
-    if (threadIdx.x == 0) dig.bucket = -1;
+  const bool staged = cnt <= kSmemKeys;
+  if (staged) {
+    for (int64_t i = threadIdx.x; i < cnt; i += blockDim.x) s_keys[i] = src[i];
     __syncthreads();
-    for (int64_t i0 = 0; i0 < cnt; i0 += blockDim.x) {
-      const int64_t i = i0 + threadIdx.x;
-      const uint64_t c = (i < cnt) ? src[i] : 0ull;
-      const bool act = (i < cnt) && ((c & pmask) == prefix);
-      hist_add(hist, act, (unsigned)(c >> shift) & 255u);
-    }
-    __syncthreads();
-    find_digit(hist, remaining, &dig);
-    __syncthreads();
-    if (dig.bucket < 0) {
-      ok = false;
-      break;
-    }
-    remaining -= dig.above;
-    prefix |= (uint64_t)dig.bucket << shift;
-    pmask |= 255ull << shift;
-    const bool exact = (int)hist[dig.bucket] == remaining;
-    __syncthreads();
-    if (exact) break;
   }
+  auto get = [&](int64_t i) { return staged ? s_keys[i] : src[i]; };
+  uint64_t prefix, pmask;
+  const bool ok = radix_select(get, cnt, k, 0, hist, &dig, &prefix, &pmask);
   if (!ok) {  // fewer than k candidates: internal error, outputs marked
     if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_INTERNAL);
     for (int r = threadIdx.x; r < k; r += blockDim.x) {
@@ -171,7 +222,7 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
   if (threadIdx.x == 0) n_sel = 0;
   __syncthreads();
   for (int64_t i = threadIdx.x; i < cnt; i += blockDim.x) {
-    const uint64_t c = src[i];
+    const uint64_t c = get(i);
     if ((c & pmask) >= prefix) {
       const unsigned p = atomicAdd(&n_sel, 1u);
       if (p < (unsigned)k) sel[p] = c;
@@ -208,22 +259,49 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
   }
 }
 
+template <class K>
+sense_status set_smem(K kern, size_t bytes) {
+  return cuda_check(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)bytes),
+                    "cudaFuncSetAttribute(select)");
+}
+
 }  // namespace
 
+int64_t chunk_count(int64_t s_len) { return (s_len + kChunk - 1) / kChunk; }
+
 sense_status launch_threshold(const uint64_t* sample, int64_t s_len, int q, int k,
-                              uint64_t* thresh, uint64_t* pool, uint32_t* counts,
+                              uint64_t* cand, uint64_t* thresh, uint64_t* pool, uint32_t* counts,
                               int64_t pool_cap, uint32_t* status, cudaStream_t s) {
+  const int64_t nch = chunk_count(s_len);
+  const size_t chunk_smem = kChunk * sizeof(uint64_t);
+  sense_status st = set_smem(chunk_topk_kernel, chunk_smem);
+  if (st != SENSE_OK) return st;
+  {
+    LaunchScope ls(K_THRESHOLD, s);
+    chunk_topk_kernel<<<dim3((unsigned)nch, q), kSelThreads, chunk_smem, s>>>(
+        sample, s_len, k, (int)nch, cand, status);
+    st = cuda_check(cudaGetLastError(), "launch chunk_topk");
+    if (st != SENSE_OK) return st;
+  }
+  const int64_t len = nch * k;
+  const size_t smem = (len <= kSmemKeys) ? (size_t)len * sizeof(uint64_t) : 0;
+  st = set_smem(threshold_kernel, kSmemKeys * sizeof(uint64_t));
+  if (st != SENSE_OK) return st;
   LaunchScope ls(K_THRESHOLD, s);
-  threshold_kernel<<<q, kSelThreads, 0, s>>>(sample, s_len, k, thresh, pool, counts, pool_cap,
-                                             status);
+  threshold_kernel<<<q, kSelThreads, smem, s>>>(cand, len, k, thresh, pool, counts, pool_cap,
+                                                status);
   return cuda_check(cudaGetLastError(), "launch threshold");
 }
 
 sense_status launch_merge(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap, int q,
                           int k, float* out_scores, int32_t* out_idx, uint32_t* status,
                           cudaStream_t s) {
+  sense_status st = set_smem(merge_kernel, kSmemKeys * sizeof(uint64_t));
+  if (st != SENSE_OK) return st;
   LaunchScope ls(K_MERGE, s);
-  merge_kernel<<<q, kSelThreads, 0, s>>>(pool, counts, pool_cap, k, out_scores, out_idx, status);
+  merge_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(pool, counts, pool_cap, k,
+                                                                   out_scores, out_idx, status);
   return cuda_check(cudaGetLastError(), "launch merge");
 }
 

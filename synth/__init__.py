@@ -51,12 +51,14 @@ def centroids(n_clusters: int, d: int, seed: int = 0, device="cpu") -> torch.Ten
 
 def clustered_unit_keys(n: int, d: int, n_clusters: int, sigma: float = 0.3,
                         seed: int = 0, device="cpu", reading: str = "A",
-                        out: torch.Tensor | None = None) -> torch.Tensor:
-    """bf16 [n, d] keys drawn around ``n_clusters`` unit centroids."""
+                        out: torch.Tensor | None = None, return_assign: bool = False):
+    """bf16 [n, d] keys drawn around ``n_clusters`` unit centroids (and, with
+    ``return_assign``, the int32 [n] cluster of each key)."""
     c = centroids(n_clusters, d, seed, device)
     scale = sigma / (d ** 0.5) if reading == "A" else sigma
     if out is None:
         out = torch.empty(n, d, dtype=torch.bfloat16, device=device)
+    assign = torch.empty(n, dtype=torch.int32, device=device) if return_assign else None
     for ci, lo in enumerate(range(0, n, CHUNK_ROWS)):
         hi = min(n, lo + CHUNK_ROWS)
         g = _gen(device, _sub_seed(seed, 2, ci))
@@ -64,8 +66,10 @@ def clustered_unit_keys(n: int, d: int, n_clusters: int, sigma: float = 0.3,
         e = torch.randn(hi - lo, d, generator=g, device=device, dtype=torch.float32)
         x = c[a] + scale * e
         out[lo:hi] = _unit_rows(x).to(torch.bfloat16)
+        if assign is not None:
+            assign[lo:hi] = a.to(torch.int32)
         del e, x
-    return out
+    return (out, assign) if return_assign else out
 
 
 def noisy_queries(keys: torch.Tensor, q: int, noise: float = 0.05, seed: int = 0,
