@@ -6,16 +6,20 @@
 // distinct rows are the root and the tree's inner nodes.  The gate therefore
 // runs in two kernels:
 //  1. gate_rows: each needed row is cut into `segs` segments, one block per
-//     segment.  A block streams its V/segs fp32 logits once (eight 128-bit
-//     loads in flight per thread) and keeps, per thread, the running max,
-//     sum exp(x - max) and sum (x - max) exp(x - max) (entropy H = log Z -
-//     S / Z), the argmax (lowest index among maxima) and a top-kappa list
-//     under (logit desc, index asc); the maximum of each 32-value chunk gates
-//     the rare updates of the argmax and the list.  The block combines its
-//     threads (fp64), writes a partial, and the last block of a row to
-//     finish (an atomic counter per row) merges the segments into the row's
-//     statistics.  A node is an inner node iff the next node in preorder is
-//     its child, so the test is O(1).
+//     segment.  Thread 0 streams the segment through a 4-stage shared-memory
+//     ring with 1-D bulk copies (cp.async.bulk, 16 KB per stage, completion
+//     on an mbarrier; every wait is bounded by clock64 and a timeout sets
+//     SENSE_DEVST_TIMEOUT).  From shared memory each thread keeps the running
+//     max, sum exp(x - max) and sum (x - max) exp(x - max) (entropy
+//     H = log Z - S / Z, accumulated with ex2 in base-2 units), the argmax
+//     (lowest index among maxima) and a top-kappa list under (logit desc,
+//     index asc); after the first stage the block's kappa-th largest value
+//     bounds the row's kappa-th largest from below, and warp votes keep list
+//     updates off the common path.  The block combines its threads (fp64),
+//     writes a partial, and the last block of a row to finish (an atomic
+//     counter per row) merges the segments into the row's statistics.  A
+//     node is an inner node iff the next node in preorder is its child, so
+//     the test is O(1).
 //  2. gate_decide: one block per query evaluates B_em, B_ent, B_topk, the
 //     lookahead B_con, G, the accepted prefix lengths L_i, i*, and writes
 //     the accepted tokens, the next node, its argmax (streaming that row if
@@ -24,14 +28,19 @@
 
 #include "common.cuh"
 #include "launch.h"
+#include "tc_ptx.cuh"
 
 namespace sense {
 namespace {
 
 constexpr int kRowThreads = 256;
-constexpr int kVec = 8;                          // float4 loads per thread per step
-constexpr int kStatsInts = 2 + SENSE_MAX_KAPPA;  // argmax, ent flag, top list
+constexpr int kStageBytes = 16384;                 // one ring stage
+constexpr int kStageF4 = kStageBytes / 16;         // float4 per stage
+constexpr int kStages = 4;
+constexpr int kVec = kStageF4 / kRowThreads;       // float4 per thread per stage
+constexpr int kStatsInts = 2 + SENSE_MAX_KAPPA;    // argmax, ent flag, top list
 constexpr int kMaxSegs = 16;
+constexpr long long kWaitCycles = 4000000000LL;
 
 struct ArgMax {
   float v;
@@ -84,60 +93,78 @@ struct TopList {
   }
 };
 
+// 2^x (one MUFU op; results below the normal range flush to 0).
+__device__ __forceinline__ float exp2_ftz(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+constexpr float kLog2e = 1.4426950408889634f;  // log2(e)
+
 template <int KM>
 struct RowAcc {
-  float m = -FLT_MAX;  // running max
-  float z = 0.0f;      // sum exp(x - m)
-  float s = 0.0f;      // sum (x - m) exp(x - m)
-  float bv = -FLT_MAX; // argmax value / index (lowest index among maxima)
-  int bi = 0x7fffffff;
+  float m = -FLT_MAX;  // running max (also the argmax value)
+  float z0 = 0.0f, z1 = 0.0f;    // sum exp(x - m), two chains
+  float s0 = 0.0f, s1 = 0.0f;    // sum ((x - m) log2 e) exp(x - m), two chains
+  int mstage = -1;     // stage holding this thread's first maximum
+  float lb = -FLT_MAX; // lower bound of the row's kappa-th largest value
   TopList<KM> tl;
 
-  // Folds kVec float4 (element indices idx[u] * 4 + e, increasing) into the
-  // state.  Padding slots hold -FLT_MAX and contribute nothing.
-  __device__ __forceinline__ void add(const float4 (&x)[kVec], const int (&idx)[kVec]) {
+  // Folds kVec float4 (element indices idx[u] * 4 + e, increasing) of stage
+  // `st` into the state.  Padding slots hold -FLT_MAX and contribute
+  // nothing.  Called by all 32 lanes of a warp together (it votes).
+  __device__ __forceinline__ void add(const float4 (&x)[kVec], const int (&idx)[kVec], int st) {
     float cm = -FLT_MAX;
 #pragma unroll
     for (int u = 0; u < kVec; ++u)
       cm = fmaxf(cm, fmaxf(fmaxf(x[u].x, x[u].y), fmaxf(x[u].z, x[u].w)));
-    if (cm > m) {
-      const float sc = __expf(m - cm);
-      s = sc * (s + (m - cm) * z);
-      z = sc * z;
+    const bool live = cm > -FLT_MAX;  // false past the end of the segment
+    if (live && cm > m) {
+      if (m > -FLT_MAX) {
+        const float d2 = (m - cm) * kLog2e;
+        const float sc = exp2_ftz(d2);
+        s0 = sc * (s0 + d2 * z0);
+        s1 = sc * (s1 + d2 * z1);
+        z0 *= sc;
+        z1 *= sc;
+      }
       m = cm;
+      mstage = st;
     }
-    if (cm > bv) {
-      bv = cm;
-      bool found = false;
+    float thr = fmaxf(tl.v[KM - 1], lb);
+    if (__any_sync(0xffffffffu, live && cm >= thr)) {
 #pragma unroll
       for (int u = 0; u < kVec; ++u) {
         const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          if (!found && xs[e] == cm) {
-            bi = idx[u] * 4 + e;
-            found = true;
+          const bool want = live && xs[e] >= thr;
+          if (__any_sync(0xffffffffu, want)) {
+            if (want) {
+              tl.push(xs[e], idx[u] * 4 + e);
+              thr = fmaxf(tl.v[KM - 1], lb);
+            }
           }
         }
       }
     }
-    if (cm > tl.v[KM - 1]) {
+    if (live) {
+      const float mb = m * kLog2e;
 #pragma unroll
       for (int u = 0; u < kVec; ++u) {
         const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) tl.push(xs[e], idx[u] * 4 + e);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kVec; ++u) {
-      const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float t = fmaxf(xs[e] - m, -200.0f);  // exp underflows to 0 below
-        const float ex = __expf(t);
-        z += ex;
-        s = fmaf(t, ex, s);
+        for (int e = 0; e < 4; e += 2) {
+          const float ta = fmaxf(fmaf(xs[e], kLog2e, -mb), -250.0f);
+          const float tb = fmaxf(fmaf(xs[e + 1], kLog2e, -mb), -250.0f);
+          const float ea = exp2_ftz(ta);
+          const float eb = exp2_ftz(tb);
+          z0 += ea;
+          z1 += eb;
+          s0 = fmaf(ta, ea, s0);
+          s1 = fmaf(tb, eb, s1);
+        }
       }
     }
   }
@@ -156,33 +183,137 @@ __device__ __forceinline__ ArgMax warp_best(ArgMax a) {
   return a;
 }
 
+// Bounded wait on an mbarrier phase; false after ~2 s.
+__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity) {
+  if (ptx::mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!ptx::mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > kWaitCycles) return false;
+  }
+  return true;
+}
+
 // Reduces one segment [lo4, hi4) of a row (float4 indices) over the block
-// and writes the block's partial to *out (thread 0 writes scalars).
+// and writes the block's partial to *out.  Returns false (uniformly) if a
+// stage never arrived.
 template <int KM>
-__device__ void segment_stats(const float* __restrict__ row, int lo4, int hi4, int kappa,
-                              Partial* out) {
+__device__ bool segment_stats(const float* __restrict__ row, int lo4, int hi4, int kappa,
+                              Partial* out, float4* ring, uint64_t* full) {
   __shared__ float s_m[kRowThreads / 32];
   __shared__ double s_z[kRowThreads / 32], s_s[kRowThreads / 32];
   __shared__ ArgMax s_w[kRowThreads / 32];
   __shared__ ArgMax s_pick;
+  __shared__ float s_top[(kRowThreads / 32) * SENSE_MAX_KAPPA];
+
+  const int tid = threadIdx.x;
+  const float4* row4 = reinterpret_cast<const float4*>(row);
+  const int n_st = (hi4 - lo4 + kStageF4 - 1) / kStageF4;
+  uint64_t pol = 0;
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) ptx::mbar_init(ptx::smem_u32(full + s), 1);
+    ptx::fence_barrier_init();
+    pol = ptx::policy_evict_first();
+  }
+  __syncthreads();
+  auto issue = [&](int i) {
+    const int f0 = lo4 + i * kStageF4;
+    const int nf = min(kStageF4, hi4 - f0);
+    const uint32_t bar = ptx::smem_u32(full + (i % kStages));
+    ptx::mbar_arrive_expect_tx(bar, (uint32_t)nf * 16u);
+    ptx::bulk_load(ptx::smem_u32(ring + (size_t)(i % kStages) * kStageF4), row4 + f0,
+                   (uint32_t)nf * 16u, bar, pol);
+  };
+  if (tid == 0)
+    for (int i = 0; i < kStages - 1 && i < n_st; ++i) issue(i);
 
   RowAcc<KM> acc;
   acc.tl.init();
-  const float4* r4 = reinterpret_cast<const float4*>(row);
   const float4 pad = make_float4(-FLT_MAX, -FLT_MAX, -FLT_MAX, -FLT_MAX);
-  for (int c = lo4 + threadIdx.x; c < hi4; c += kVec * kRowThreads) {
+  bool ok = true;
+  for (int i = 0; i < n_st; ++i) {
+    const bool got = wait_phase(ptx::smem_u32(full + (i % kStages)), (uint32_t)((i / kStages) & 1));
+    if (__syncthreads_or(!got)) {  // uniform: every thread leaves together
+      ok = false;
+      if (tid == 0) {  // let the copies in flight land before the block exits
+        for (int j = i; j < i + kStages - 1 && j < n_st; ++j)
+          wait_phase(ptx::smem_u32(full + (j % kStages)), (uint32_t)((j / kStages) & 1));
+      }
+      break;
+    }
+    // every thread is past stage i-1, so its buffer may be refilled
+    if (tid == 0 && i + kStages - 1 < n_st) issue(i + kStages - 1);
+    const float4* st = ring + (size_t)(i % kStages) * kStageF4;
+    const int f0 = lo4 + i * kStageF4;
+    const int nf = min(kStageF4, hi4 - f0);
     float4 x[kVec];
     int idx[kVec];
 #pragma unroll
     for (int u = 0; u < kVec; ++u) {
-      idx[u] = c + u * kRowThreads;
-      x[u] = (idx[u] < hi4) ? __ldcs(r4 + idx[u]) : pad;
+      const int j = tid + u * kRowThreads;
+      idx[u] = f0 + j;
+      x[u] = (j < nf) ? st[j] : pad;
     }
-    acc.add(x, idx);
+    acc.add(x, idx, i);
+    if (i == 0 && n_st > 1) {
+      // The block's kappa-th largest value so far bounds the row's kappa-th
+      // largest from below: later values under it cannot enter.
+      float hv[KM];
+      int hx[KM];
+#pragma unroll
+      for (int t = 0; t < KM; ++t) {
+        hv[t] = acc.tl.v[t];
+        hx[t] = acc.tl.i[t];
+      }
+      for (int r = 0; r < kappa; ++r) {
+        const ArgMax w = warp_best(ArgMax{hv[0], hx[0]});
+        if ((tid & 31) == 0) s_top[(tid >> 5) * SENSE_MAX_KAPPA + r] = w.v;
+        if (hx[0] == w.i && hv[0] == w.v) {
+#pragma unroll
+          for (int t = 0; t < KM - 1; ++t) {
+            hv[t] = hv[t + 1];
+            hx[t] = hx[t + 1];
+          }
+          hv[KM - 1] = -FLT_MAX;
+          hx[KM - 1] = 0x7fffffff;
+        }
+      }
+      __syncthreads();
+      float best[SENSE_MAX_KAPPA];
+      for (int r = 0; r < kappa; ++r) best[r] = -FLT_MAX;
+      for (int w = 0; w < kRowThreads / 32; ++w) {
+        for (int r = 0; r < kappa; ++r) {
+          float v = s_top[w * SENSE_MAX_KAPPA + r];
+          for (int t = 0; t < kappa; ++t) {
+            if (v > best[t]) {
+              const float tmp = best[t];
+              best[t] = v;
+              v = tmp;
+            }
+          }
+        }
+      }
+      acc.lb = best[kappa - 1];
+    }
   }
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  if (!ok) return false;
+  // argmax index: the first element equal to the maximum in its stage
+  int bi = 0x7fffffff;
+  if (acc.mstage >= 0) {
+    const int f0 = lo4 + acc.mstage * kStageF4;
+    for (int u = 0; u < kVec && bi == 0x7fffffff; ++u) {
+      const int j = f0 + tid + u * kRowThreads;
+      if (j >= hi4) break;
+      const float4 v = row4[j];
+      if (v.x == acc.m) bi = j * 4;
+      else if (v.y == acc.m) bi = j * 4 + 1;
+      else if (v.z == acc.m) bi = j * 4 + 2;
+      else if (v.w == acc.m) bi = j * 4 + 3;
+    }
+  }
+  const float acc_z = acc.z0 + acc.z1;
+  const float acc_s = (acc.s0 + acc.s1) * (1.0f / kLog2e);  // natural-log units
+  const int lane = tid & 31, wid = tid >> 5;
   constexpr int NW = kRowThreads / 32;
-  // block max
   float mm = acc.m;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, off));
@@ -191,27 +322,26 @@ __device__ void segment_stats(const float* __restrict__ row, int lo4, int hi4, i
   float M = s_m[0];
 #pragma unroll
   for (int w = 1; w < NW; ++w) M = fmaxf(M, s_m[w]);
-  // rescale (z, s) to M in fp64 and sum
   double z = 0.0, s = 0.0;
-  if (acc.z > 0.0f) {
+  if (acc_z > 0.0f) {
     const double d = (double)acc.m - (double)M;
     const double sc = exp(d);
-    z = (double)acc.z * sc;
-    s = sc * ((double)acc.s + d * (double)acc.z);
+    z = (double)acc_z * sc;
+    s = sc * ((double)acc_s + d * (double)acc_z);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     z += __shfl_xor_sync(0xffffffffu, z, off);
     s += __shfl_xor_sync(0xffffffffu, s, off);
   }
-  ArgMax a = warp_best(ArgMax{acc.bv, acc.bi});
+  ArgMax a = warp_best(ArgMax{acc.m, bi});
   if (lane == 0) {
     s_z[wid] = z;
     s_s[wid] = s;
     s_w[wid] = a;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (tid == 0) {
     double Z = 0.0, Sx = 0.0;
     ArgMax b = s_w[0];
     for (int w = 0; w < NW; ++w) {
@@ -231,7 +361,7 @@ __device__ void segment_stats(const float* __restrict__ row, int lo4, int hi4, i
     __syncthreads();
     if (lane == 0) s_w[wid] = h;
     __syncthreads();
-    if (threadIdx.x == 0) {
+    if (tid == 0) {
       ArgMax b = s_w[0];
       for (int w = 1; w < NW; ++w)
         if (better(s_w[w].v, s_w[w].i, b.v, b.i)) b = s_w[w];
@@ -250,6 +380,7 @@ __device__ void segment_stats(const float* __restrict__ row, int lo4, int hi4, i
       acc.tl.i[KM - 1] = 0x7fffffff;
     }
   }
+  return true;
 }
 
 // Merges the segment partials of one row into its statistics (one thread).
@@ -299,7 +430,9 @@ gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__
                  int cap, const float* __restrict__ root_logits,
                  const float* __restrict__ node_logits, int vocab, int kappa, float thr,
                  int unnormalized, int segs, int seg4, Partial* __restrict__ parts,
-                 unsigned* __restrict__ done, int32_t* __restrict__ stats) {
+                 unsigned* __restrict__ done, int32_t* __restrict__ stats, uint32_t* status) {
+  extern __shared__ __align__(128) float4 ring[];
+  __shared__ __align__(8) uint64_t full[kStages];
   __shared__ int s_last;
   const int slot = blockIdx.x / segs;  // 0 = root, 1 + n = node n
   const int seg = blockIdx.x - slot * segs;
@@ -319,7 +452,10 @@ gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__
   const int hi4 = min(n4, lo4 + seg4);
   const int64_t rid = (int64_t)q * (cap + 1) + slot;
   Partial* rp = parts + rid * segs;
-  segment_stats<KM>(row, lo4, hi4, kappa, rp + seg);
+  if (!segment_stats<KM>(row, lo4, hi4, kappa, rp + seg, ring, full)) {
+    if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_TIMEOUT);
+    return;
+  }
   if (segs == 1) {
     __syncthreads();
     if (threadIdx.x == 0) finish_row(rp, 1, vocab, kappa, thr, unnormalized, stats + rid * kStatsInts);
@@ -509,8 +645,8 @@ size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 int gate_segments(int q, int cap, int vocab) {
   const int64_t rows = (int64_t)q * (cap + 1);
   const int n4 = vocab >> 2;
-  int64_t segs = (4LL * sm_count() + rows - 1) / rows;
-  const int64_t by_len = n4 / 512;  // at least 8 KB of logits per segment
+  int64_t segs = (2LL * sm_count() + rows - 1) / rows;
+  const int64_t by_len = n4 / (2 * kStageF4);  // at least two stages per segment
   if (segs > by_len) segs = by_len;
   if (segs > kMaxSegs) segs = kMaxSegs;
   if (segs < 1) segs = 1;
@@ -546,17 +682,19 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
   }
   {
     dim3 grid((unsigned)((a.cap + 1) * segs), a.q);
+    const size_t ring = (size_t)kStages * kStageBytes;
+    auto k4 = gate_rows_kernel<4>;
+    auto k16 = gate_rows_kernel<SENSE_MAX_KAPPA>;
+    auto kern = (a.kappa <= 4) ? k4 : k16;
+    sense_status st = cuda_check(
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ring),
+        "cudaFuncSetAttribute(gate_rows)");
+    if (st != SENSE_OK) return st;
     LaunchScope ls(K_GATE_ROWS, s);
-    if (a.kappa <= 4) {
-      gate_rows_kernel<4><<<grid, kRowThreads, 0, s>>>(
-          a.parent, a.num_nodes, a.cap, a.root_logits, a.node_logits, a.vocab, a.kappa, a.thr,
-          a.unnormalized, segs, seg4, parts, done, stats);
-    } else {
-      gate_rows_kernel<SENSE_MAX_KAPPA><<<grid, kRowThreads, 0, s>>>(
-          a.parent, a.num_nodes, a.cap, a.root_logits, a.node_logits, a.vocab, a.kappa, a.thr,
-          a.unnormalized, segs, seg4, parts, done, stats);
-    }
-    sense_status st = cuda_check(cudaGetLastError(), "launch gate_rows");
+    kern<<<grid, kRowThreads, ring, s>>>(a.parent, a.num_nodes, a.cap, a.root_logits,
+                                         a.node_logits, a.vocab, a.kappa, a.thr, a.unnormalized,
+                                         segs, seg4, parts, done, stats, a.status);
+    st = cuda_check(cudaGetLastError(), "launch gate_rows");
     if (st != SENSE_OK) return st;
   }
   const size_t smem = (size_t)a.k * a.m;
