@@ -33,6 +33,7 @@ import torch  # noqa: E402
 from synth.workloads import WORKLOADS  # noqa: E402
 
 DEFAULT = "llama7b_1m"
+METRIC = "hidden-state top-k retrieval queries/s (whole drafting step)"
 GATE = dict(gamma=0.05, topk=3, window=6, tau=0)
 # dram bytes (read + write) per launch of the dominant kernel from one ncu
 # capture, or None when the kernel changed since the capture.
@@ -97,6 +98,20 @@ class ClockSampler:
             return None
         return {"sm_mhz": statistics.median(sms), "sm_max_mhz": max(maxs),
                 "reasons": sorted(reasons), "samples": len(sms)}
+
+
+def max_over_ranks(x: float, dist=None, device="cpu") -> float:
+    """The largest of every rank's value (timings are taken as the slowest)."""
+    if dist is None:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: int, world: int, seconds: float) -> float:
+    """Whole-job units per second: every rank processed units_per_rank."""
+    return world * units_per_rank / seconds
 
 
 def make_workload(cfg, dev, seed=0):
@@ -221,7 +236,7 @@ def run_reference(args, cfg, name):
     per_query_batch = slices * statistics.mean(t_scan) + statistics.mean(t_down)
     value = cfg["q"] / per_query_batch
     line = {
-        "impl": "reference", "metric": "queries/s", "value": value, "unit": "queries/s",
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "queries/s",
         "n_gpus": args.gpus, "steps": len(t_scan), "warmup": args.warmup,
         "ms_per_step": per_query_batch * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -309,14 +324,11 @@ def main():
     ms = e0.elapsed_time(e1)
     prof = {name: S.sense_profile_query(name) for name in S.sense_profile_names()}
     S.sense_profile_enable(False)
-    if dist:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, dist, dev)
     launches = sum(v[1] for v in prof.values())
 
     q, n, d = cfg["q"], cfg["n"], cfg["d"]
-    value = world * q * args.steps / (ms / 1e3)
+    value = job_throughput(q * args.steps, world, ms / 1e3)
     # roofline of the dominant kernel (the key scan)
     scan_name = "scan_gemv" if q <= 8 else "scan_tc"
     scan_ms, scan_launches = prof.get(scan_name, (0.0, 0))
@@ -365,12 +377,8 @@ def main():
         h_small[:, 3].copy_(pipe.gate["next_anchor"], non_blocking=True)
         h_hnext.copy_(pipe.gate["h_next"], non_blocking=True)
         torch.cuda.current_stream().synchronize()
-    e2e_s = time.perf_counter() - t0
-    if dist:
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
-    e2e_value = world * q * e2e_steps / e2e_s
+    e2e_s = max_over_ranks(time.perf_counter() - t0, dist, dev)
+    e2e_value = job_throughput(q * e2e_steps, world, e2e_s)
 
     base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -378,7 +386,7 @@ def main():
 
     if rank == 0:
         line = {
-            "metric": "hidden-state top-k retrieval queries/s (whole drafting step)",
+            "metric": METRIC,
             "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",

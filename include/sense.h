@@ -287,6 +287,19 @@ sense_status sense_soft_gate(const int32_t* tokens, const int32_t* parent,
                              size_t workspace_bytes, sense_stream_t stream);
 
 /* ---------------------------------------------------------------------- */
+/* Diagnostics                                                              */
+/* ---------------------------------------------------------------------- */
+/*
+ * Failure-detection self test (the paper has no counterpart): one block
+ * waits on a shared-memory barrier that nothing arrives on, through the same
+ * bounded wait the tensor-core pipeline uses, with a limit of limit_cycles
+ * SM clocks (1 .. 2^34).  The wait gives up, sets SENSE_DEVST_TIMEOUT in the
+ * device status word and the kernel returns; the context stays usable.
+ * Read the result with sense_device_status.
+ */
+sense_status sense_selftest_timeout(sense_stream_t stream, int64_t limit_cycles);
+
+/* ---------------------------------------------------------------------- */
 /* Launch profiling                                                         */
 /* ---------------------------------------------------------------------- */
 /*

@@ -282,6 +282,13 @@ def sense_soft_gate(tree: dict, root_logits: torch.Tensor, node_logits: torch.Te
     return o
 
 
+def sense_selftest_timeout(limit_cycles: int = 200_000_000, stream=None) -> int:
+    """Runs the bounded-wait self test and returns the device status bits
+    it left (SENSE_DEVST_TIMEOUT expected); clears them afterwards."""
+    _check(lib().sense_selftest_timeout(C.c_void_p(_stream(stream)), int(limit_cycles)))
+    return sense_device_status(clear=True, stream=stream)
+
+
 def sense_profile_enable(on: bool = True):
     _check(lib().sense_profile_enable(1 if on else 0))
 

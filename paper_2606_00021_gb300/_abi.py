@@ -34,6 +34,7 @@ SIGNATURES = {
     "sense_soft_gate": (c_i32, [c_p, c_p, c_p, c_p, c_i32, c_i32, c_i32, c_i32, c_p, c_p, c_i32,
                                 c_p, c_p, c_i32, C.POINTER(GateParams), c_p, c_p, c_p, c_p, c_p,
                                 c_p, c_p, c_p, c_p, c_size, c_p]),
+    "sense_selftest_timeout": (c_i32, [c_p, c_i64]),
     "sense_profile_enable": (c_i32, [c_i32]),
     "sense_profile_count": (c_i32, []),
     "sense_profile_name": (C.c_char_p, [c_i32]),

@@ -484,6 +484,14 @@ sense_status sense_soft_gate(const int32_t* tokens, const int32_t* parent,
   return launch_gate(a, stream);
 }
 
+sense_status sense_selftest_timeout(sense_stream_t stream, int64_t limit_cycles) {
+  if (limit_cycles < 1 || limit_cycles > (1LL << 34))
+    return fail(SENSE_ERR_INVALID_ARG, "limit_cycles=%lld outside [1, 2^34]", (long long)limit_cycles);
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  return launch_selftest_wait(limit_cycles, status, stream);
+}
+
 sense_status sense_profile_enable(int32_t on) {
   std::lock_guard<std::mutex> lk(g_mu);
   for (auto& r : g_prof) {

@@ -66,6 +66,7 @@ sense_status launch_scan_tc(const uint16_t* keys, int64_t n, int d, const uint16
                             int nq, int mode, int64_t n_half, const uint64_t* thresh,
                             uint64_t* out, uint32_t* counts, int64_t pool_cap, uint32_t* status,
                             cudaStream_t s);
+sense_status launch_selftest_wait(long long limit, uint32_t* status, cudaStream_t s);
 sense_status launch_pad_queries(const uint16_t* src, int qg, int d, uint16_t* dst, int nq,
                                 cudaStream_t s);
 size_t scan_tc_smem_bytes(int d, int nq);

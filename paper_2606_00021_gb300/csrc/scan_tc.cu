@@ -70,13 +70,13 @@ struct Shared {
 
 // Bounded wait: false if the abort flag is raised or the wait times out.
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort,
-                                         uint32_t* status) {
+                                         uint32_t* status, long long limit = kWaitCycles) {
   if (ptx::mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (ptx::mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > limit) {
       *abort = 1;
       raise_status(status, SENSE_DEVST_TIMEOUT);
       return false;
@@ -267,6 +267,21 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tm_keys,
   }
 }
 
+// One block waits, through the same bounded wait as the scan's pipeline,
+// on a barrier nothing arrives on: the wait gives up after `limit` cycles
+// and reports SENSE_DEVST_TIMEOUT.
+__global__ void selftest_wait_kernel(long long limit, uint32_t* status) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort;
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(ptx::smem_u32(&bar), 1);
+    abort = 0;
+    ptx::fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) wait_bar(ptx::smem_u32(&bar), 0, &abort, status, limit);
+}
+
 __global__ void pad_queries_kernel(const uint16_t* __restrict__ src, int qg, int d,
                                    uint16_t* __restrict__ dst, int nq) {
   const int64_t total = (int64_t)nq * d;
@@ -324,6 +339,11 @@ size_t scan_tc_smem_bytes(int d, int nq) {
   const int S = stages_for(nq);
   const size_t stage = 2 * kTileBytes + (size_t)nq * kBlockK * 2;
   return 1024 + S * stage + (2 * S + 5) * 8 + sizeof(Shared) + 8 * 128;
+}
+
+sense_status launch_selftest_wait(long long limit, uint32_t* status, cudaStream_t s) {
+  selftest_wait_kernel<<<1, 32, 0, s>>>(limit, status);
+  return cuda_check(cudaGetLastError(), "launch selftest_wait");
 }
 
 sense_status launch_pad_queries(const uint16_t* src, int qg, int d, uint16_t* dst, int nq,

@@ -304,3 +304,27 @@ def test_gate_golden_fixture(S):
         assert int(got["next_anchor"][0]) == case["next_anchor"]
         assert host(got["accepted"])[0][:case["L_star"] + 1].tolist() == case["accepted"]
         assert torch.equal(got["h_next"][0], hn[0, case["next_node"]])
+
+
+# ---------------------------------------------------------------- failure detection
+
+@cuda
+def test_bounded_wait_reports_timeout_and_context_survives(S):
+    """A pipeline wait that nothing satisfies gives up, reports
+    SENSE_DEVST_TIMEOUT, and the device keeps working afterwards."""
+    assert S.sense_device_status(clear=True) == 0
+    t0 = __import__("time").perf_counter()
+    bits_ = S.sense_selftest_timeout(100_000_000)  # ~50 ms of SM clocks
+    assert bits_ & S.DEVST_TIMEOUT
+    assert __import__("time").perf_counter() - t0 < 30
+    dev = torch.device("cuda")
+    keys = synth.clustered_unit_keys(2048, 128, 8, seed=1, device=dev)
+    spans = synth.spans_uniform(2048, 4, 10, seed=1, device=dev)
+    ds = S.sense_datastore_build(keys, spans)
+    qs, _ = synth.noisy_queries(keys, 16, seed=1)
+    sc, ix = S.sense_retrieve_topk(ds, qs, 8)
+    torch.cuda.synchronize()
+    assert S.sense_device_status(clear=True) == 0
+    full = O.scores(bits(keys), bits(qs))
+    for qi in range(16):
+        check_topk(host(sc[qi]), host(ix[qi]), full[qi], 8)
