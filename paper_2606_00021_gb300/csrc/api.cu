@@ -155,10 +155,14 @@ RetrievePlan make_plan(const sense_datastore* ds, int q, int k) {
   RetrievePlan p{};
   p.tc = q > 8;
   p.group = p.tc ? (q < 128 ? q : 128) : q;
+  p.fused = !p.tc && q <= kFusedMaxQ && k <= kFusedMaxK &&
+            fused_smem_bytes(q, ds->d, k) <= 110 * 1024;  // two blocks per SM
+  p.fused_blocks = p.fused ? fused_blocks() : 0;
   p.s_rows = sample_tiles(ds->n) * (int64_t)kTileRows;
   p.r_rows = rest_tiles(ds->n) * (int64_t)kTileRows;
   p.sampling = sample_tiles(ds->n) >= 4 && p.s_rows >= 4LL * k && p.s_rows >= 2048;
-  p.pool_cap = ds->n;
+  p.pool_cap = p.fused ? (int64_t)p.fused_blocks * k : ds->n;
+  if (p.fused) p.sampling = false;
   const int g = p.group;
   size_t off = 0;
   p.off_counts = off;
@@ -189,6 +193,11 @@ sense_status run_retrieve(const RetrievePlan& p, const sense_datastore* ds,
   const int64_t n = ds->n;
   const int d = ds->d;
   sense_status st = SENSE_OK;
+  if (p.fused) {
+    st = launch_scan_gemv_topk(ds->keys, n, d, queries, q, k, p.fused_blocks, pool, stream);
+    if (st != SENSE_OK) return st;
+    return launch_merge_lists(pool, p.fused_blocks, q, k, out_scores, out_idx, status, stream);
+  }
   for (int g0 = 0; g0 < q; g0 += p.group) {
     const int gq = (q - g0 < p.group) ? (q - g0) : p.group;
     const int nq = (gq + 15) / 16 * 16;

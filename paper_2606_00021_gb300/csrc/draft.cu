@@ -60,6 +60,26 @@ __device__ int block_exclusive_scan(int v, int* scratch, int* total) {
   return r;
 }
 
+// Rank of the set entries of flag[0..len): flag[i] != 0 becomes the number
+// of set entries before i, flag[i] == 0 becomes -1; returns the set count.
+// Each thread scans a contiguous run, then one block scan joins the runs.
+__device__ int block_rank_flags(int* flag, int len, int* scratch) {
+  const int per = (len + blockDim.x - 1) / blockDim.x;
+  const int lo = min(len, (int)threadIdx.x * per);
+  const int hi = min(len, lo + per);
+  int cnt = 0;
+  for (int i = lo; i < hi; ++i) cnt += flag[i] != 0;
+  int total = 0;
+  int run = block_exclusive_scan(cnt, scratch, &total);
+  for (int i = lo; i < hi; ++i) {
+    const int f = flag[i];
+    flag[i] = f ? run : -1;
+    run += f != 0;
+  }
+  __syncthreads();
+  return total;
+}
+
 __global__ void gather_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
                               const int32_t* __restrict__ idx, int k,
                               const int32_t* __restrict__ anchor, int n_keep, int force,
@@ -217,24 +237,25 @@ tree_kernel(const int32_t* __restrict__ spans, int k, int m, int cap, int mask_w
     s_own[e] = (s_lcp[p] <= j) ? p : -1;
   }
   __syncthreads();
+  // Hillis-Steele prefix max over p, ping-ponging between s_own and s_aux.
+  int* pm_in = s_own;
+  int* pm_out = s_aux;
   for (int off = 1; off < k; off <<= 1) {
-    int vals[(SENSE_MAX_TREE_TOKENS + kTreeThreads - 1) / kTreeThreads];
-    int c = 0;
-    for (int e = threadIdx.x; e < km; e += blockDim.x, ++c) {
+    for (int e = threadIdx.x; e < km; e += blockDim.x) {
       const int p = e / m;
-      int v = s_own[e];
-      if (p >= off) v = max(v, s_own[e - off * m]);
-      vals[c] = v;
+      int v = pm_in[e];
+      if (p >= off) v = max(v, pm_in[e - off * m]);
+      pm_out[e] = v;
     }
     __syncthreads();
-    c = 0;
-    for (int e = threadIdx.x; e < km; e += blockDim.x, ++c) s_own[e] = vals[c];
-    __syncthreads();
+    int* t = pm_in;
+    pm_in = pm_out;
+    pm_out = t;
   }
   // node id of (sorted p, j) = base[p'] + j - lcp[p'], p' the creator.
   for (int e = threadIdx.x; e < km; e += blockDim.x) {
     const int p = e / m, j = e - p * m;
-    const int pc = s_own[e];
+    const int pc = pm_in[e];
     s_own[e] = s_base[pc] + j - s_lcp[pc];
   }
   __syncthreads();
@@ -261,17 +282,8 @@ tree_kernel(const int32_t* __restrict__ spans, int k, int m, int cap, int mask_w
       }
     }
     __syncthreads();
-    // rank of every key: chunked block scan over km entries
-    int running = 0;
-    for (int c0 = 0; c0 < km; c0 += blockDim.x) {
-      const int i = c0 + threadIdx.x;
-      const int v = (i < km) ? s_new[i] : 0;
-      int tot = 0;
-      const int ex = block_exclusive_scan(v, scratch, &tot);
-      if (i < km) s_new[i] = v ? (running + ex) : -1;
-      running += tot;
-    }
-    __syncthreads();
+    // rank of every present key
+    block_rank_flags(s_new, km, scratch);
     // kept flag per node (u in preorder): rank of its key < cap.
     for (int e = threadIdx.x; e < km; e += blockDim.x) {
       const int p = e / m, j = e - p * m;
@@ -283,16 +295,10 @@ tree_kernel(const int32_t* __restrict__ spans, int k, int m, int cap, int mask_w
     }
     __syncthreads();
     // new ids: prefix count of kept flags in preorder
-    running = 0;
-    for (int c0 = 0; c0 < U; c0 += blockDim.x) {
-      const int u = c0 + threadIdx.x;
-      const int v = (u < U) ? s_aux[u] : 0;
-      int tot = 0;
-      const int ex = block_exclusive_scan(v, scratch, &tot);
-      if (u < U) s_new[u] = v ? (running + ex) : -1;
-      running += tot;
-    }
-    if (threadIdx.x == 0) s_kept = running;
+    for (int u = threadIdx.x; u < U; u += blockDim.x) s_new[u] = s_aux[u];
+    __syncthreads();
+    const int nk = block_rank_flags(s_new, U, scratch);
+    if (threadIdx.x == 0) s_kept = nk;
   } else {
     for (int u = threadIdx.x; u < U; u += blockDim.x) s_new[u] = u;
     if (threadIdx.x == 0) s_kept = U;
@@ -364,7 +370,11 @@ sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int
   if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(tree)");
   const int words = (cap + 31) / 32;
   LaunchScope ls(K_TREE, s);
-  tree_kernel<<<q, kTreeThreads, smem, s>>>(spans, k, m, cap, words, num_nodes, tokens, parent,
+  // one thread per candidate row at least; fewer threads make the many
+  // block barriers of a small tree cheaper
+  int threads = 128;
+  while (threads < k) threads <<= 1;
+  tree_kernel<<<q, threads, smem, s>>>(spans, k, m, cap, words, num_nodes, tokens, parent,
                                             depth, gamma, mask_bits ? mask : nullptr, status);
   return cuda_check(cudaGetLastError(), "launch tree");
 }

@@ -323,11 +323,11 @@ __device__ bool segment_stats(const float* __restrict__ row, int lo4, int hi4, i
 #pragma unroll
   for (int w = 1; w < NW; ++w) M = fmaxf(M, s_m[w]);
   double z = 0.0, s = 0.0;
-  if (acc_z > 0.0f) {
-    const double d = (double)acc.m - (double)M;
-    const double sc = exp(d);
-    z = (double)acc_z * sc;
-    s = sc * ((double)acc_s + d * (double)acc_z);
+  if (acc_z > 0.0f) {  // rescale this thread's sums to the block max (fp32)
+    const float d = acc.m - M;
+    const float sc = exp2_ftz(d * kLog2e);
+    z = (double)(acc_z * sc);
+    s = (double)(sc * (acc_s + d * acc_z));
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -393,17 +393,17 @@ __device__ void finish_row(const Partial* parts, int segs, int vocab, int kappa,
   for (int g = 0; g < segs; ++g) {
     const Partial& p = parts[g];
     if (p.z > 0.0) {
-      const double d = (double)p.m - (double)M;
-      const double sc = exp(d);
+      const float d = p.m - M;
+      const double sc = (double)exp2_ftz(d * kLog2e);
       Z += p.z * sc;
-      Sx += sc * (p.s + d * p.z);
+      Sx += sc * (p.s + (double)d * p.z);
     }
     if (better(p.bv, p.bi, b.v, b.i)) b = ArgMax{p.bv, p.bi};
   }
-  const double H = log(Z) - Sx / Z;
-  const double score = unnormalized ? H : H / log((double)vocab);
+  const float H = logf((float)Z) - (float)(Sx / Z);
+  const float score = unnormalized ? H : H / logf((float)vocab);
   out[0] = b.i;
-  out[1] = (score > (double)thr) ? 1 : 0;
+  out[1] = (score > thr) ? 1 : 0;
   int head[kMaxSegs];
   for (int g = 0; g < segs; ++g) head[g] = 0;
   for (int r = 0; r < kappa; ++r) {
@@ -515,10 +515,10 @@ gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats) {
   __syncthreads();
   // B_con over the strictly-future window j+1..j+W; positions past the span
   // and dropped positions count as mismatches.  Then G.
-  uint8_t g_val[(SENSE_MAX_TREE_TOKENS + kDecideThreads - 1) / kDecideThreads];
   {
-    int c = 0;
-    for (int e = threadIdx.x; e < km; e += blockDim.x, ++c) {
+    // bit 4 (G) of a position is written in place: readers of other
+    // positions only use bits 0-1, which no thread changes here
+    for (int e = threadIdx.x; e < km; e += blockDim.x) {
       const int i = e / m, j = e - i * m;
       const uint8_t f = s_flags[e];
       int mism = 0;
@@ -532,11 +532,8 @@ gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats) {
       }
       const bool con = mism <= a.tau;
       const bool valid = f & 1, em = f & 2, ent = f & 4, tk = f & 8;
-      g_val[c] = (valid && (em || (ent && (tk || con)))) ? 1 : 0;
+      if (valid && (em || (ent && (tk || con)))) s_flags[e] = f | 16;
     }
-    __syncthreads();
-    c = 0;
-    for (int e = threadIdx.x; e < km; e += blockDim.x, ++c) s_flags[e] |= g_val[c] << 4;
     __syncthreads();
   }
   if (a.G) {
@@ -699,7 +696,8 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
   }
   const size_t smem = (size_t)a.k * a.m;
   LaunchScope ls(K_GATE_DECIDE, s);
-  gate_decide_kernel<<<a.q, kDecideThreads, smem, s>>>(a, stats);
+  const int threads = (a.k * a.m <= 4096) ? 256 : kDecideThreads;
+  gate_decide_kernel<<<a.q, threads, smem, s>>>(a, stats);
   return cuda_check(cudaGetLastError(), "launch gate_decide");
 }
 

@@ -37,6 +37,8 @@ inline int64_t rest_tiles(int64_t n) { return num_tiles(n) - sample_tiles(n); }
 struct RetrievePlan {
   bool tc;           // tensor-core scan
   int group;         // queries per pass over the keys
+  bool fused;        // single-pass scan with in-register top-k lists
+  int fused_blocks;  // its grid size
   bool sampling;     // sample-threshold pass enabled
   int64_t s_rows;    // sample work rows
   int64_t r_rows;    // rest work rows
@@ -59,6 +61,22 @@ sense_status launch_scan_gemv(const uint16_t* keys, int64_t n, int d, const uint
                               uint64_t* out, uint32_t* counts, int64_t pool_cap,
                               uint32_t* status, cudaStream_t s);
 
+// Single-pass scan for q <= kFusedMaxQ queries and k <= kFusedMaxK: every
+// warp keeps a sorted top-k list per query in registers, every block merges
+// its warps' lists and writes its k best keys per query to
+// cand[(qi * blocks + block) * k + r].  `blocks` must be the grid size the
+// workspace was planned with (fused_blocks()).
+constexpr int kFusedMaxQ = 4;
+constexpr int kFusedMaxK = 128;
+int fused_blocks();
+inline size_t fused_smem_bytes(int q, int d, int k) {
+  const int kpl = k <= 32 ? 1 : (k <= 64 ? 2 : 4);
+  return (size_t)q * d * 2 + (size_t)q * 8 * kpl * 32 * sizeof(uint64_t);
+}
+sense_status launch_scan_gemv_topk(const uint16_t* keys, int64_t n, int d,
+                                   const uint16_t* queries, int q, int k, int blocks,
+                                   uint64_t* cand, cudaStream_t s);
+
 // Same contract on tcgen05 tensor cores for qg <= nq <= 128 queries held in
 // `qpad` ([nq, d] bf16, rows >= qg zero); the work set is n_half 128-row
 // tiles selected by `mode`.
@@ -79,7 +97,14 @@ sense_status launch_threshold(const uint64_t* sample, int64_t s_len, int q, int 
                               uint64_t* cand, uint64_t* thresh, uint64_t* pool, uint32_t* counts,
                               int64_t pool_cap, uint32_t* status, cudaStream_t s);
 
+// Per query: the k largest keys of `nlists` descending-sorted lists of k
+// keys ([q][nlists][k]), sorted descending -> scores, indices.
+sense_status launch_merge_lists(const uint64_t* lists, int nlists, int q, int k,
+                                float* out_scores, int32_t* out_idx, uint32_t* status,
+                                cudaStream_t s);
+
 // Per query: the k largest pool keys, sorted descending -> scores, indices.
+// With counts == nullptr every one of the pool_cap slots is a candidate.
 sense_status launch_merge(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap, int q,
                           int k, float* out_scores, int32_t* out_idx, uint32_t* status,
                           cudaStream_t s);

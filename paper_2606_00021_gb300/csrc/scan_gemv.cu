@@ -115,6 +115,144 @@ scan_gemv_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
   }
 }
 
+// Sorted list of KPL * 32 candidate keys spread over a warp: position
+// r = s * 32 + lane lives in v[s] of that lane, larger keys first.
+template <int KPL>
+__device__ __forceinline__ void list_insert(uint64_t (&v)[KPL], uint64_t c, int lane) {
+  int p = 0;  // keys ahead of c (all keys are distinct)
+#pragma unroll
+  for (int s = 0; s < KPL; ++s) p += __popc(__ballot_sync(0xffffffffu, v[s] > c));
+  uint64_t up[KPL], last[KPL];
+#pragma unroll
+  for (int s = 0; s < KPL; ++s) {
+    up[s] = __shfl_up_sync(0xffffffffu, v[s], 1);
+    last[s] = __shfl_sync(0xffffffffu, v[s], 31);
+  }
+#pragma unroll
+  for (int s = 0; s < KPL; ++s) {
+    const int r = s * 32 + lane;
+    const uint64_t prev = (lane == 0) ? (s > 0 ? last[s > 0 ? s - 1 : 0] : 0ull) : up[s];
+    v[s] = (r < p) ? v[s] : (r == p ? c : prev);
+  }
+}
+
+// Single pass: the GEMV scan of scan_gemv_kernel with the top-k kept in
+// per-warp register lists instead of a threshold filter.  Scores are
+// warp-uniform after the reduction, so list updates never diverge.  At the
+// end the block sorts its warps' lists (bitonic, shared memory) and writes
+// its k best keys per query.
+template <int Q, int KPL, int UNROLL>
+__global__ void __launch_bounds__(256, 2)
+scan_gemv_topk_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
+                      const uint16_t* __restrict__ queries, int k,
+                      uint64_t* __restrict__ cand) {
+  constexpr int K = KPL * 32;   // list length per warp
+  constexpr int L = 8 * K;      // entries per query per block (8 warps)
+  extern __shared__ uint4 s_q[];  // [Q][C] bf16 chunks, then the lists
+  const int C = d >> 3;
+  const uint4* qsrc = reinterpret_cast<const uint4*>(queries);
+  for (int i = threadIdx.x; i < Q * C; i += blockDim.x) s_q[i] = qsrc[i];
+  uint64_t* s_list = reinterpret_cast<uint64_t*>(s_q + Q * C);  // [Q][L]
+  __syncthreads();
+
+  const int lane = threadIdx.x & 31;
+  const int wid = threadIdx.x >> 5;
+  const int64_t warp0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  uint64_t v[Q][KPL];
+  uint64_t lmin[Q];
+#pragma unroll
+  for (int qi = 0; qi < Q; ++qi) {
+    lmin[qi] = 0ull;
+#pragma unroll
+    for (int s = 0; s < KPL; ++s) v[qi][s] = 0ull;
+  }
+
+  for (int64_t row = warp0; row < n; row += nwarps) {
+    float acc[Q];
+#pragma unroll
+    for (int qi = 0; qi < Q; ++qi) acc[qi] = 0.0f;
+    const uint4* kr = reinterpret_cast<const uint4*>(keys + row * (int64_t)d);
+    for (int c0 = 0; c0 < C; c0 += 32 * UNROLL) {
+      uint4 kv[UNROLL];
+#pragma unroll
+      for (int u = 0; u < UNROLL; ++u) {
+        const int c = c0 + u * 32 + lane;
+        kv[u] = (c < C) ? ld_stream_v4(kr + c) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < UNROLL; ++u) {
+        const int c = c0 + u * 32 + lane;
+        if (c < C) {
+#pragma unroll
+          for (int qi = 0; qi < Q; ++qi) acc[qi] = dot8(kv[u], s_q[qi * C + c], acc[qi]);
+        }
+      }
+    }
+#pragma unroll
+    for (int qi = 0; qi < Q; ++qi) {
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) acc[qi] += __shfl_xor_sync(0xffffffffu, acc[qi], off);
+      const uint64_t c = cand_key(acc[qi], (uint32_t)row);
+      if (c > lmin[qi]) {  // warp-uniform
+        list_insert<KPL>(v[qi], c, lane);
+        lmin[qi] = __shfl_sync(0xffffffffu, v[qi][KPL - 1], 31);
+      }
+    }
+  }
+  // block merge: lists of all warps per query, sorted descending
+#pragma unroll
+  for (int qi = 0; qi < Q; ++qi) {
+#pragma unroll
+    for (int s = 0; s < KPL; ++s) s_list[qi * L + wid * K + s * 32 + lane] = v[qi][s];
+  }
+  __syncthreads();
+  for (int size = 2; size <= L; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int t = threadIdx.x; t < Q * L; t += blockDim.x) {
+        const int i = t % L, base = t - i;
+        const int j = i ^ stride;
+        if (j > i) {
+          const bool desc = ((i & size) == 0);
+          const uint64_t a = s_list[base + i], b = s_list[base + j];
+          if (desc ? (a < b) : (a > b)) {
+            s_list[base + i] = b;
+            s_list[base + j] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  for (int t = threadIdx.x; t < Q * k; t += blockDim.x) {
+    const int qi = t / k, r = t - qi * k;
+    cand[((int64_t)qi * gridDim.x + blockIdx.x) * k + r] = s_list[qi * L + r];
+  }
+}
+
+template <int Q, int KPL>
+sense_status launch_topk_q(const uint16_t* keys, int64_t n, int d, const uint16_t* queries, int k,
+                           int blocks, uint64_t* cand, cudaStream_t s) {
+  constexpr int UNROLL = (Q <= 2) ? 16 : 8;
+  auto kern = scan_gemv_topk_kernel<Q, KPL, UNROLL>;
+  const size_t smem = fused_smem_bytes(Q, d, KPL * 32);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(scan_gemv_topk)");
+  }
+  LaunchScope ls(K_SCAN_GEMV, s);
+  kern<<<blocks, 256, smem, s>>>(keys, n, d, queries, k, cand);
+  return cuda_check(cudaGetLastError(), "launch scan_gemv_topk");
+}
+
+template <int Q>
+sense_status launch_topk_kpl(const uint16_t* keys, int64_t n, int d, const uint16_t* queries,
+                             int k, int blocks, uint64_t* cand, cudaStream_t s) {
+  if (k <= 32) return launch_topk_q<Q, 1>(keys, n, d, queries, k, blocks, cand, s);
+  if (k <= 64) return launch_topk_q<Q, 2>(keys, n, d, queries, k, blocks, cand, s);
+  return launch_topk_q<Q, 4>(keys, n, d, queries, k, blocks, cand, s);
+}
+
 template <int Q, int MODE>
 sense_status launch_q_mode(const uint16_t* keys, int64_t n, int d, const uint16_t* queries,
                            int64_t n_work, const uint64_t* thresh, uint64_t* out, uint32_t* counts,
@@ -157,6 +295,21 @@ sense_status launch_q(const uint16_t* keys, int64_t n, int d, const uint16_t* qu
 }
 
 }  // namespace
+
+int fused_blocks() { return 2 * sm_count(); }
+
+sense_status launch_scan_gemv_topk(const uint16_t* keys, int64_t n, int d,
+                                   const uint16_t* queries, int q, int k, int blocks,
+                                   uint64_t* cand, cudaStream_t s) {
+  if (k < 1 || k > kFusedMaxK) return fail(SENSE_ERR_UNSUPPORTED, "fused scan needs k <= %d", kFusedMaxK);
+  switch (q) {
+    case 1: return launch_topk_kpl<1>(keys, n, d, queries, k, blocks, cand, s);
+    case 2: return launch_topk_kpl<2>(keys, n, d, queries, k, blocks, cand, s);
+    case 3: return launch_topk_kpl<3>(keys, n, d, queries, k, blocks, cand, s);
+    case 4: return launch_topk_kpl<4>(keys, n, d, queries, k, blocks, cand, s);
+    default: return fail(SENSE_ERR_UNSUPPORTED, "fused scan supports 1..%d queries", kFusedMaxQ);
+  }
+}
 
 sense_status launch_scan_gemv(const uint16_t* keys, int64_t n, int d, const uint16_t* queries,
                               int q, int mode, int64_t n_work, const uint64_t* thresh,

@@ -27,7 +27,7 @@ namespace {
 
 constexpr int kSelThreads = 1024;
 constexpr int kChunk = 8192;          // keys per first-level block (64 KB)
-constexpr int kSmemKeys = 12288;      // keys staged in shared memory (96 KB)
+constexpr int kSmemKeys = 24576;      // keys staged in shared memory (192 KB)
 
 struct Digit {
   int bucket;
@@ -200,7 +200,7 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
   __shared__ uint64_t sel[SENSE_MAX_K];
   const int q = blockIdx.x;
   const uint64_t* src = pool + (int64_t)q * pool_cap;
-  int64_t cnt = counts[q];
+  int64_t cnt = counts ? (int64_t)counts[q] : pool_cap;  // no counts: every slot is used
   if (cnt > pool_cap) cnt = pool_cap;
   const bool staged = cnt <= kSmemKeys;
   if (staged) {
@@ -259,6 +259,103 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
   }
 }
 
+// Exact top-k of `nlists` lists of k keys per query, each list sorted in
+// descending order (the per-block output of the single-pass scan).  The
+// k-th largest list head is a lower bound T of the k-th largest key (k lists
+// each hold a key >= T), so only list prefixes >= T are candidates; they are
+// gathered into shared memory, selected and sorted.  If the gathered set
+// would not fit, every key of every list is used instead.
+constexpr int kGather = 4096;
+
+__global__ void __launch_bounds__(kSelThreads, 1)
+merge_lists_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
+                   float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
+                   uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];  // [kSmemKeys]
+  __shared__ unsigned hist[256];
+  __shared__ Digit dig;
+  __shared__ unsigned n_sel, n_got;
+  __shared__ uint64_t sel[SENSE_MAX_K];
+  const int q = blockIdx.x;
+  const uint64_t* src = lists + (int64_t)q * nlists * k;
+  // 1. lower bound from the list heads
+  for (int b = threadIdx.x; b < nlists; b += blockDim.x) s_keys[b] = src[(int64_t)b * k];
+  __syncthreads();
+  uint64_t t = 0ull;
+  if (nlists >= k) {
+    uint64_t prefix, pmask;
+    if (radix_select([&](int64_t i) { return s_keys[i]; }, nlists, k, 0, hist, &dig, &prefix,
+                     &pmask))
+      t = prefix;
+  }
+  // 2. gather list prefixes >= t
+  if (threadIdx.x == 0) n_got = 0;
+  __syncthreads();
+  for (int b = threadIdx.x; b < nlists; b += blockDim.x) {
+    const uint64_t* lb = src + (int64_t)b * k;
+    for (int r = 0; r < k; ++r) {
+      const uint64_t c = lb[r];
+      if (c < t || c == 0ull) break;
+      const unsigned p = atomicAdd(&n_got, 1u);
+      if (p < (unsigned)kGather) s_keys[p] = c;
+    }
+  }
+  __syncthreads();
+  const bool small = n_got <= (unsigned)kGather;
+  const int64_t cnt = small ? (int64_t)n_got : (int64_t)nlists * k;
+  if (!small) {  // too many ties near the bound: use every key
+    for (int64_t i = threadIdx.x; i < cnt && i < kSmemKeys; i += blockDim.x) s_keys[i] = src[i];
+    __syncthreads();
+  }
+  auto get = [&](int64_t i) { return (i < kSmemKeys) ? s_keys[i] : src[i]; };
+  uint64_t prefix, pmask;
+  const bool ok = radix_select(get, cnt, k, 0, hist, &dig, &prefix, &pmask);
+  if (!ok) {
+    if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_INTERNAL);
+    for (int r = threadIdx.x; r < k; r += blockDim.x) {
+      out_scores[(int64_t)q * k + r] = 0.0f;
+      out_idx[(int64_t)q * k + r] = -1;
+    }
+    return;
+  }
+  if (threadIdx.x == 0) n_sel = 0;
+  __syncthreads();
+  for (int64_t i = threadIdx.x; i < cnt; i += blockDim.x) {
+    const uint64_t c = get(i);
+    if ((c & pmask) >= prefix) {
+      const unsigned p = atomicAdd(&n_sel, 1u);
+      if (p < (unsigned)k) sel[p] = c;
+    }
+  }
+  __syncthreads();
+  int kp = 1;
+  while (kp < k) kp <<= 1;
+  for (int i = threadIdx.x; i < kp; i += blockDim.x)
+    if (i >= k) sel[i] = 0ull;
+  __syncthreads();
+  for (int size = 2; size <= kp; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < kp; i += blockDim.x) {
+        const int j = i ^ stride;
+        if (j > i) {
+          const bool desc = ((i & size) == 0);
+          const uint64_t a = sel[i], b = sel[j];
+          if (desc ? (a < b) : (a > b)) {
+            sel[i] = b;
+            sel[j] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  for (int r = threadIdx.x; r < k; r += blockDim.x) {
+    const uint64_t c = sel[r];
+    out_scores[(int64_t)q * k + r] = code_score((uint32_t)(c >> 32));
+    out_idx[(int64_t)q * k + r] = (int32_t)cand_index(c);
+  }
+}
+
 template <class K>
 sense_status set_smem(K kern, size_t bytes) {
   return cuda_check(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -292,6 +389,17 @@ sense_status launch_threshold(const uint64_t* sample, int64_t s_len, int q, int 
   threshold_kernel<<<q, kSelThreads, smem, s>>>(cand, len, k, thresh, pool, counts, pool_cap,
                                                 status);
   return cuda_check(cudaGetLastError(), "launch threshold");
+}
+
+sense_status launch_merge_lists(const uint64_t* lists, int nlists, int q, int k,
+                                float* out_scores, int32_t* out_idx, uint32_t* status,
+                                cudaStream_t s) {
+  sense_status st = set_smem(merge_lists_kernel, kSmemKeys * sizeof(uint64_t));
+  if (st != SENSE_OK) return st;
+  LaunchScope ls(K_MERGE, s);
+  merge_lists_kernel<<<q, 256, kSmemKeys * sizeof(uint64_t), s>>>(
+      lists, nlists, k, out_scores, out_idx, status);
+  return cuda_check(cudaGetLastError(), "launch merge_lists");
 }
 
 sense_status launch_merge(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap, int q,
