@@ -5,21 +5,21 @@
 // predicted by the row of node gamma[i, j-1] (the root row for j = 0), so the
 // distinct rows are the root and the tree's inner nodes.  The gate therefore
 // runs in two kernels:
-//  1. gate_rows: each needed row is cut into `segs` segments, one block per
-//     segment.  Thread 0 streams the segment through a 4-stage shared-memory
-//     ring with 1-D bulk copies (cp.async.bulk, 16 KB per stage, completion
-//     on an mbarrier; every wait is bounded by clock64 and a timeout sets
-//     SENSE_DEVST_TIMEOUT).  From shared memory each thread keeps the running
-//     max, sum exp(x - max) and sum (x - max) exp(x - max) (entropy
-//     H = log Z - S / Z, accumulated with ex2 in base-2 units), the argmax
-//     (lowest index among maxima) and a top-kappa list under (logit desc,
-//     index asc); after the first stage the block's kappa-th largest value
-//     bounds the row's kappa-th largest from below, and warp votes keep list
-//     updates off the common path.  The block combines its threads (fp64),
-//     writes a partial, and the last block of a row to finish (an atomic
-//     counter per row) merges the segments into the row's statistics.  A
-//     node is an inner node iff the next node in preorder is its child, so
-//     the test is O(1).
+//  1. gate_rows: a persistent grid of warps; each warp takes whole rows
+//     (root or inner-node logits) from an atomic counter and streams a row
+//     through its own 6-stage shared-memory ring with 1-D bulk copies
+//     (cp.async.bulk, 4 KB per stage, completion on an mbarrier; every wait
+//     is bounded by clock64 and a timeout sets SENSE_DEVST_TIMEOUT).  Each
+//     lane keeps the running max, the sums exp(x - max) and (x - max)
+//     exp(x - max) in packed fp32 pairs (entropy H = log Z - S / Z, with
+//     ex2 in base-2 units), the stage holding its first maximum (the argmax
+//     index is read back once at the end: lowest index among maxima) and a
+//     top-kappa list under (logit desc, index asc).  A lower bound of the
+//     row's kappa-th largest value, seeded from the lane maxima of the
+//     first stage and refreshed from the lists after stages 1, 3, 7, 15, 31,
+//     keeps list updates (warp-voted) off the common path.  All combining is
+//     done with warp shuffles: no block barriers.  A node is an inner node
+//     iff the next node in preorder is its child, so the test is O(1).
 //  2. gate_decide: one block per query evaluates B_em, B_ent, B_topk, the
 //     lookahead B_con, G, the accepted prefix lengths L_i, i*, and writes
 //     the accepted tokens, the next node, its argmax (streaming that row if
@@ -34,10 +34,11 @@ namespace sense {
 namespace {
 
 constexpr int kRowThreads = 256;
-constexpr int kStageBytes = 16384;                 // one ring stage
-constexpr int kStageF4 = kStageBytes / 16;         // float4 per stage
-constexpr int kStages = 4;
-constexpr int kVec = kStageF4 / kRowThreads;       // float4 per thread per stage
+constexpr int kWarps = kRowThreads / 32;
+constexpr int kWStageF4 = 256;                     // float4 per warp stage (4 KB)
+constexpr int kWStages = 6;                        // ring depth per warp
+constexpr int kLaneF4 = kWStageF4 / 32;            // float4 per lane per stage
+constexpr size_t kRingBytes = (size_t)kWarps * kWStages * kWStageF4 * 16;
 constexpr int kStatsInts = 2 + SENSE_MAX_KAPPA;    // argmax, ent flag, top list
 constexpr int kMaxSegs = 16;
 constexpr long long kWaitCycles = 4000000000LL;
@@ -49,17 +50,6 @@ struct ArgMax {
 __device__ __forceinline__ bool better(float va, int ia, float vb, int ib) {
   return va > vb || (va == vb && ia < ib);
 }
-
-// Statistics of one segment of a row (workspace).
-struct Partial {
-  double z, s;  // relative to m
-  float m;
-  float bv;
-  int bi;
-  int pad;
-  float tv[SENSE_MAX_KAPPA];
-  int ti[SENSE_MAX_KAPPA];
-};
 
 template <int KM>
 struct TopList {
@@ -100,42 +90,67 @@ __device__ __forceinline__ float exp2_ftz(float x) {
   return y;
 }
 
+// Two fp32 lanes in one 64-bit register: packed Blackwell FMA / ADD.
+__device__ __forceinline__ uint64_t pk(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void upk(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 constexpr float kLog2e = 1.4426950408889634f;  // log2(e)
 
 template <int KM>
 struct RowAcc {
-  float m = -FLT_MAX;  // running max (also the argmax value)
-  float z0 = 0.0f, z1 = 0.0f;    // sum exp(x - m), two chains
-  float s0 = 0.0f, s1 = 0.0f;    // sum ((x - m) log2 e) exp(x - m), two chains
-  int mstage = -1;     // stage holding this thread's first maximum
-  float lb = -FLT_MAX; // lower bound of the row's kappa-th largest value
+  float m = -FLT_MAX;       // running max (also the argmax value)
+  uint64_t z = 0, s = 0;    // packed pairs: sum exp(x - m), sum ((x - m) log2 e) exp(x - m)
+  int mstage = -1;          // stage holding this thread's first maximum
+  float lb = -FLT_MAX;      // lower bound of the row's kappa-th largest value
   TopList<KM> tl;
 
-  // Folds kVec float4 (element indices idx[u] * 4 + e, increasing) of stage
-  // `st` into the state.  Padding slots hold -FLT_MAX and contribute
-  // nothing.  Called by all 32 lanes of a warp together (it votes).
-  __device__ __forceinline__ void add(const float4 (&x)[kVec], const int (&idx)[kVec], int st) {
+  __device__ __forceinline__ void rescale(float cm) {
+    if (m > -FLT_MAX) {
+      const float d2 = (m - cm) * kLog2e;
+      const float sc = exp2_ftz(d2);
+      float z0, z1, s0, s1;
+      upk(z, z0, z1);
+      upk(s, s0, s1);
+      s = pk(sc * (s0 + d2 * z0), sc * (s1 + d2 * z1));
+      z = pk(sc * z0, sc * z1);
+    }
+    m = cm;
+  }
+
+  // Folds one stage: kLaneF4 float4 of this lane (element indices
+  // idx[u] * 4 + e, increasing).  Padding slots hold -FLT_MAX.  Called by
+  // all 32 lanes of a warp together (it votes).
+  __device__ __forceinline__ void add(const float4 (&x)[kLaneF4], const int (&idx)[kLaneF4],
+                                      int st) {
     float cm = -FLT_MAX;
 #pragma unroll
-    for (int u = 0; u < kVec; ++u)
+    for (int u = 0; u < kLaneF4; ++u)
       cm = fmaxf(cm, fmaxf(fmaxf(x[u].x, x[u].y), fmaxf(x[u].z, x[u].w)));
-    const bool live = cm > -FLT_MAX;  // false past the end of the segment
+    const bool live = cm > -FLT_MAX;  // false past the end of the range
     if (live && cm > m) {
-      if (m > -FLT_MAX) {
-        const float d2 = (m - cm) * kLog2e;
-        const float sc = exp2_ftz(d2);
-        s0 = sc * (s0 + d2 * z0);
-        s1 = sc * (s1 + d2 * z1);
-        z0 *= sc;
-        z1 *= sc;
-      }
-      m = cm;
+      rescale(cm);
       mstage = st;
     }
     float thr = fmaxf(tl.v[KM - 1], lb);
     if (__any_sync(0xffffffffu, live && cm >= thr)) {
 #pragma unroll
-      for (int u = 0; u < kVec; ++u) {
+      for (int u = 0; u < kLaneF4; ++u) {
         const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -150,22 +165,27 @@ struct RowAcc {
       }
     }
     if (live) {
-      const float mb = m * kLog2e;
+      const uint64_t l2 = pk(kLog2e, kLog2e);
+      const uint64_t nmb = pk(-m * kLog2e, -m * kLog2e);
+      uint64_t z2 = 0, s2 = 0;  // second chain
 #pragma unroll
-      for (int u = 0; u < kVec; ++u) {
-        const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
-#pragma unroll
-        for (int e = 0; e < 4; e += 2) {
-          const float ta = fmaxf(fmaf(xs[e], kLog2e, -mb), -250.0f);
-          const float tb = fmaxf(fmaf(xs[e + 1], kLog2e, -mb), -250.0f);
-          const float ea = exp2_ftz(ta);
-          const float eb = exp2_ftz(tb);
-          z0 += ea;
-          z1 += eb;
-          s0 = fmaf(ta, ea, s0);
-          s1 = fmaf(tb, eb, s1);
-        }
+      for (int u = 0; u < kLaneF4; ++u) {
+        float t0, t1, t2, t3;
+        upk(fma2(pk(x[u].x, x[u].y), l2, nmb), t0, t1);
+        upk(fma2(pk(x[u].z, x[u].w), l2, nmb), t2, t3);
+        t0 = fmaxf(t0, -250.0f);  // exp underflows to 0 below
+        t1 = fmaxf(t1, -250.0f);
+        t2 = fmaxf(t2, -250.0f);
+        t3 = fmaxf(t3, -250.0f);
+        const uint64_t ea = pk(exp2_ftz(t0), exp2_ftz(t1));
+        const uint64_t eb = pk(exp2_ftz(t2), exp2_ftz(t3));
+        z = add2(z, ea);
+        s = fma2(pk(t0, t1), ea, s);
+        z2 = add2(z2, eb);
+        s2 = fma2(pk(t2, t3), eb, s2);
       }
+      z = add2(z, z2);
+      s = add2(s, s2);
     }
   }
 };
@@ -193,184 +213,243 @@ __device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity) {
   return true;
 }
 
-// Reduces one segment [lo4, hi4) of a row (float4 indices) over the block
-// and writes the block's partial to *out.  Returns false (uniformly) if a
-// stage never arrived.
+// kappa-th largest value of the warp's lists (each lane's list sorted):
+// kappa rounds of a warp-wide best over the list heads.
 template <int KM>
-__device__ bool segment_stats(const float* __restrict__ row, int lo4, int hi4, int kappa,
-                              Partial* out, float4* ring, uint64_t* full) {
-  __shared__ float s_m[kRowThreads / 32];
-  __shared__ double s_z[kRowThreads / 32], s_s[kRowThreads / 32];
-  __shared__ ArgMax s_w[kRowThreads / 32];
-  __shared__ ArgMax s_pick;
-  __shared__ float s_top[(kRowThreads / 32) * SENSE_MAX_KAPPA];
-
-  const int tid = threadIdx.x;
-  const float4* row4 = reinterpret_cast<const float4*>(row);
-  const int n_st = (hi4 - lo4 + kStageF4 - 1) / kStageF4;
-  uint64_t pol = 0;
-  if (tid == 0) {
-    for (int s = 0; s < kStages; ++s) ptx::mbar_init(ptx::smem_u32(full + s), 1);
-    ptx::fence_barrier_init();
-    pol = ptx::policy_evict_first();
+__device__ __forceinline__ float warp_kth(const TopList<KM>& tl, int kappa) {
+  float hv[KM];
+  int hx[KM];
+#pragma unroll
+  for (int t = 0; t < KM; ++t) {
+    hv[t] = tl.v[t];
+    hx[t] = tl.i[t];
   }
-  __syncthreads();
-  auto issue = [&](int i) {
-    const int f0 = lo4 + i * kStageF4;
-    const int nf = min(kStageF4, hi4 - f0);
-    const uint32_t bar = ptx::smem_u32(full + (i % kStages));
+  float kth = -FLT_MAX;
+  for (int r = 0; r < kappa; ++r) {
+    const ArgMax w = warp_best(ArgMax{hv[0], hx[0]});
+    kth = w.v;
+    if (hx[0] == w.i && hv[0] == w.v) {
+#pragma unroll
+      for (int t = 0; t < KM - 1; ++t) {
+        hv[t] = hv[t + 1];
+        hx[t] = hx[t + 1];
+      }
+      hv[KM - 1] = -FLT_MAX;
+      hx[KM - 1] = 0x7fffffff;
+    }
+  }
+  return kth;
+}
+
+// Statistics of one segment of a row, merged by the row's last warp.
+struct Partial {
+  double z, s;  // relative to m
+  float m;
+  float bv;
+  int bi;
+  int pad;
+  float tv[SENSE_MAX_KAPPA];
+  int ti[SENSE_MAX_KAPPA];
+};
+
+// Row statistics from its segment partials, written to out.  Called by a
+// whole warp: lane g holds partial g (segs <= 32), then warp reductions.
+__device__ void finish_row(const Partial* parts, int segs, int vocab, int kappa, float thr,
+                           int unnormalized, int32_t* __restrict__ out) {
+  const int lane = threadIdx.x & 31;
+  const bool has = lane < segs;
+  float m = -FLT_MAX, bv = -FLT_MAX;
+  double pz = 0.0, ps = 0.0;
+  int bi = 0x7fffffff;
+  float tv[SENSE_MAX_KAPPA];
+  int ti[SENSE_MAX_KAPPA];
+  if (has) {
+    const Partial& p = parts[lane];
+    m = p.m;
+    pz = p.z;
+    ps = p.s;
+    bv = p.bv;
+    bi = p.bi;
+  }
+#pragma unroll
+  for (int r = 0; r < SENSE_MAX_KAPPA; ++r) {
+    tv[r] = (has && r < kappa) ? parts[lane].tv[r] : -FLT_MAX;
+    ti[r] = (has && r < kappa) ? parts[lane].ti[r] : 0x7fffffff;
+  }
+  float M = m;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+  double Z = 0.0, Sx = 0.0;
+  if (has && pz > 0.0) {
+    const float d = m - M;
+    const double sc = (double)exp2_ftz(d * kLog2e);
+    Z = pz * sc;
+    Sx = sc * (ps + (double)d * pz);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    Z += __shfl_xor_sync(0xffffffffu, Z, off);
+    Sx += __shfl_xor_sync(0xffffffffu, Sx, off);
+  }
+  const ArgMax b = warp_best(ArgMax{bv, bi});
+  int head = 0;
+  for (int r = 0; r < kappa; ++r) {
+    float hv = -FLT_MAX;
+    int hx = 0x7fffffff;
+#pragma unroll
+    for (int t = 0; t < SENSE_MAX_KAPPA; ++t)
+      if (t == head) {
+        hv = tv[t];
+        hx = ti[t];
+      }
+    const ArgMax w = warp_best(ArgMax{hv, hx});
+    if (lane == 0) out[2 + r] = w.i;
+    if (hx == w.i && hv == w.v) ++head;
+  }
+  if (lane == 0) {
+    const float H = logf((float)Z) - (float)(Sx / Z);
+    const float score = unnormalized ? H : H / logf((float)vocab);
+    out[0] = b.i;
+    out[1] = (score > thr) ? 1 : 0;
+    for (int r = kappa; r < SENSE_MAX_KAPPA; ++r) out[2 + r] = -1;
+  }
+}
+
+// One segment [lo4, hi4) of a row (float4 indices), streamed by one warp
+// through its ring.  `seq` counts the warp's stages across tasks (it fixes
+// buffer and phase of every stage).  Lane 0 receives the partial; returns
+// false (whole warp) if a stage never arrived.
+template <int KM>
+__device__ bool warp_segment(const float* __restrict__ row, int lo4, int hi4, int kappa,
+                             float4* ring, uint64_t* bars, uint32_t& seq, uint64_t pol,
+                             Partial* out) {
+  const int lane = threadIdx.x & 31;
+  const float4* row4 = reinterpret_cast<const float4*>(row) + lo4;
+  const int n4 = hi4 - lo4;
+  const int n = (n4 + kWStageF4 - 1) / kWStageF4;
+  auto issue = [&](int j) {  // lane 0: stage j of this row
+    const uint32_t g = seq + (uint32_t)j;
+    const int f0 = j * kWStageF4;
+    const int nf = min(kWStageF4, n4 - f0);
+    const uint32_t bar = ptx::smem_u32(bars + (g % kWStages));
     ptx::mbar_arrive_expect_tx(bar, (uint32_t)nf * 16u);
-    ptx::bulk_load(ptx::smem_u32(ring + (size_t)(i % kStages) * kStageF4), row4 + f0,
+    ptx::bulk_load(ptx::smem_u32(ring + (size_t)(g % kWStages) * kWStageF4), row4 + f0,
                    (uint32_t)nf * 16u, bar, pol);
   };
-  if (tid == 0)
-    for (int i = 0; i < kStages - 1 && i < n_st; ++i) issue(i);
+  int next = min(kWStages - 1, n);  // stages issued (same value in every lane)
+  if (lane == 0)
+    for (int j = 0; j < next; ++j) issue(j);
 
   RowAcc<KM> acc;
   acc.tl.init();
   const float4 pad = make_float4(-FLT_MAX, -FLT_MAX, -FLT_MAX, -FLT_MAX);
   bool ok = true;
-  for (int i = 0; i < n_st; ++i) {
-    const bool got = wait_phase(ptx::smem_u32(full + (i % kStages)), (uint32_t)((i / kStages) & 1));
-    if (__syncthreads_or(!got)) {  // uniform: every thread leaves together
+  for (int i = 0; i < n; ++i) {
+    const uint32_t g = seq + (uint32_t)i;
+    const bool got = wait_phase(ptx::smem_u32(bars + (g % kWStages)), (g / kWStages) & 1u);
+    if (!__all_sync(0xffffffffu, got)) {
+      if (lane == 0)  // let the copies in flight land before giving up
+        for (int j = i; j < next; ++j) {
+          const uint32_t gj = seq + (uint32_t)j;
+          wait_phase(ptx::smem_u32(bars + (gj % kWStages)), (gj / kWStages) & 1u);
+        }
       ok = false;
-      if (tid == 0) {  // let the copies in flight land before the block exits
-        for (int j = i; j < i + kStages - 1 && j < n_st; ++j)
-          wait_phase(ptx::smem_u32(full + (j % kStages)), (uint32_t)((j / kStages) & 1));
-      }
       break;
     }
-    // every thread is past stage i-1, so its buffer may be refilled
-    if (tid == 0 && i + kStages - 1 < n_st) issue(i + kStages - 1);
-    const float4* st = ring + (size_t)(i % kStages) * kStageF4;
-    const int f0 = lo4 + i * kStageF4;
-    const int nf = min(kStageF4, hi4 - f0);
-    float4 x[kVec];
-    int idx[kVec];
+    if (next < n) {  // every lane is past stage i-1: refill its buffer
+      if (lane == 0) issue(next);
+      ++next;
+    }
+    const float4* st = ring + (size_t)(g % kWStages) * kWStageF4;
+    const int f0 = i * kWStageF4;
+    const int nf = min(kWStageF4, n4 - f0);
+    float4 x[kLaneF4];
+    int idx[kLaneF4];
+    if (nf == kWStageF4) {
 #pragma unroll
-    for (int u = 0; u < kVec; ++u) {
-      const int j = tid + u * kRowThreads;
-      idx[u] = f0 + j;
-      x[u] = (j < nf) ? st[j] : pad;
+      for (int u = 0; u < kLaneF4; ++u) {
+        x[u] = st[lane + 32 * u];
+        idx[u] = lo4 + f0 + lane + 32 * u;
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < kLaneF4; ++u) {
+        const int j = lane + 32 * u;
+        x[u] = (j < nf) ? st[j] : pad;
+        idx[u] = lo4 + f0 + j;
+      }
+    }
+    if (i == 0) {
+      // seed the bound: the kappa-th largest lane maximum of the first stage
+      float cm = -FLT_MAX;
+#pragma unroll
+      for (int u = 0; u < kLaneF4; ++u)
+        cm = fmaxf(cm, fmaxf(fmaxf(x[u].x, x[u].y), fmaxf(x[u].z, x[u].w)));
+      float b = -FLT_MAX;
+      for (int r = 0; r < kappa; ++r) {
+        const ArgMax w = warp_best(ArgMax{cm, lane});
+        b = w.v;
+        if (lane == w.i) cm = -FLT_MAX;
+      }
+      acc.lb = b;
     }
     acc.add(x, idx, i);
-    if (i == 0 && n_st > 1) {
-      // The block's kappa-th largest value so far bounds the row's kappa-th
-      // largest from below: later values under it cannot enter.
-      float hv[KM];
-      int hx[KM];
-#pragma unroll
-      for (int t = 0; t < KM; ++t) {
-        hv[t] = acc.tl.v[t];
-        hx[t] = acc.tl.i[t];
-      }
-      for (int r = 0; r < kappa; ++r) {
-        const ArgMax w = warp_best(ArgMax{hv[0], hx[0]});
-        if ((tid & 31) == 0) s_top[(tid >> 5) * SENSE_MAX_KAPPA + r] = w.v;
-        if (hx[0] == w.i && hv[0] == w.v) {
-#pragma unroll
-          for (int t = 0; t < KM - 1; ++t) {
-            hv[t] = hv[t + 1];
-            hx[t] = hx[t + 1];
-          }
-          hv[KM - 1] = -FLT_MAX;
-          hx[KM - 1] = 0x7fffffff;
-        }
-      }
-      __syncthreads();
-      float best[SENSE_MAX_KAPPA];
-      for (int r = 0; r < kappa; ++r) best[r] = -FLT_MAX;
-      for (int w = 0; w < kRowThreads / 32; ++w) {
-        for (int r = 0; r < kappa; ++r) {
-          float v = s_top[w * SENSE_MAX_KAPPA + r];
-          for (int t = 0; t < kappa; ++t) {
-            if (v > best[t]) {
-              const float tmp = best[t];
-              best[t] = v;
-              v = tmp;
-            }
-          }
-        }
-      }
-      acc.lb = best[kappa - 1];
-    }
+    if (((i + 2) & (i + 1)) == 0 && i < 32)  // after stages 1, 3, 7, 15, 31
+      acc.lb = fmaxf(acc.lb, warp_kth<KM>(acc.tl, kappa));
   }
+  seq += (uint32_t)n;
   if (!ok) return false;
-  // argmax index: the first element equal to the maximum in its stage
+  // argmax: this lane's first maximum, read back from its stage
   int bi = 0x7fffffff;
   if (acc.mstage >= 0) {
-    const int f0 = lo4 + acc.mstage * kStageF4;
-    for (int u = 0; u < kVec && bi == 0x7fffffff; ++u) {
-      const int j = f0 + tid + u * kRowThreads;
-      if (j >= hi4) break;
+    const int f0 = acc.mstage * kWStageF4;
+    for (int u = 0; u < kLaneF4 && bi == 0x7fffffff; ++u) {
+      const int j = f0 + lane + 32 * u;
+      if (j >= n4) break;
       const float4 v = row4[j];
-      if (v.x == acc.m) bi = j * 4;
-      else if (v.y == acc.m) bi = j * 4 + 1;
-      else if (v.z == acc.m) bi = j * 4 + 2;
-      else if (v.w == acc.m) bi = j * 4 + 3;
+      const int e = (lo4 + j) * 4;
+      if (v.x == acc.m) bi = e;
+      else if (v.y == acc.m) bi = e + 1;
+      else if (v.z == acc.m) bi = e + 2;
+      else if (v.w == acc.m) bi = e + 3;
     }
   }
-  const float acc_z = acc.z0 + acc.z1;
-  const float acc_s = (acc.s0 + acc.s1) * (1.0f / kLog2e);  // natural-log units
-  const int lane = tid & 31, wid = tid >> 5;
-  constexpr int NW = kRowThreads / 32;
-  float mm = acc.m;
+  float z0, z1, s0, s1;
+  upk(acc.z, z0, z1);
+  upk(acc.s, s0, s1);
+  const float lz = z0 + z1;
+  const float ls = (s0 + s1) * (1.0f / kLog2e);  // natural-log units
+  float M = acc.m;
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, off));
-  if (lane == 0) s_m[wid] = mm;
-  __syncthreads();
-  float M = s_m[0];
-#pragma unroll
-  for (int w = 1; w < NW; ++w) M = fmaxf(M, s_m[w]);
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
   double z = 0.0, s = 0.0;
-  if (acc_z > 0.0f) {  // rescale this thread's sums to the block max (fp32)
+  if (lz > 0.0f) {  // rescale this lane's sums to the row max
     const float d = acc.m - M;
     const float sc = exp2_ftz(d * kLog2e);
-    z = (double)(acc_z * sc);
-    s = (double)(sc * (acc_s + d * acc_z));
+    z = (double)(lz * sc);
+    s = (double)(sc * (ls + d * lz));
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     z += __shfl_xor_sync(0xffffffffu, z, off);
     s += __shfl_xor_sync(0xffffffffu, s, off);
   }
-  ArgMax a = warp_best(ArgMax{acc.m, bi});
+  const ArgMax am = warp_best(ArgMax{acc.m, bi});
   if (lane == 0) {
-    s_z[wid] = z;
-    s_s[wid] = s;
-    s_w[wid] = a;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    double Z = 0.0, Sx = 0.0;
-    ArgMax b = s_w[0];
-    for (int w = 0; w < NW; ++w) {
-      Z += s_z[w];
-      Sx += s_s[w];
-      if (better(s_w[w].v, s_w[w].i, b.v, b.i)) b = s_w[w];
-    }
-    out->z = Z;
-    out->s = Sx;
+    out->z = z;
+    out->s = s;
     out->m = M;
-    out->bv = b.v;
-    out->bi = b.i;
+    out->bv = am.v;
+    out->bi = am.i;
   }
-  // top-kappa of the segment: kappa rounds of a block-wide best over heads
+  // top-kappa: kappa rounds of a warp-wide best over the list heads
   for (int r = 0; r < kappa; ++r) {
-    ArgMax h = warp_best(ArgMax{acc.tl.v[0], acc.tl.i[0]});
-    __syncthreads();
-    if (lane == 0) s_w[wid] = h;
-    __syncthreads();
-    if (tid == 0) {
-      ArgMax b = s_w[0];
-      for (int w = 1; w < NW; ++w)
-        if (better(s_w[w].v, s_w[w].i, b.v, b.i)) b = s_w[w];
-      s_pick = b;
-      out->tv[r] = b.v;
-      out->ti[r] = b.i;
+    const ArgMax w = warp_best(ArgMax{acc.tl.v[0], acc.tl.i[0]});
+    if (lane == 0) {
+      out->tv[r] = w.v;
+      out->ti[r] = w.i;
     }
-    __syncthreads();
-    if (acc.tl.i[0] == s_pick.i && acc.tl.v[0] == s_pick.v) {
+    if (acc.tl.i[0] == w.i && acc.tl.v[0] == w.v) {
 #pragma unroll
       for (int t = 0; t < KM - 1; ++t) {
         acc.tl.v[t] = acc.tl.v[t + 1];
@@ -380,97 +459,78 @@ __device__ bool segment_stats(const float* __restrict__ row, int lo4, int hi4, i
       acc.tl.i[KM - 1] = 0x7fffffff;
     }
   }
+  __syncwarp();
   return true;
 }
 
-// Merges the segment partials of one row into its statistics (one thread).
-__device__ void finish_row(const Partial* parts, int segs, int vocab, int kappa, float thr,
-                           int unnormalized, int32_t* __restrict__ out) {
-  float M = -FLT_MAX;
-  for (int g = 0; g < segs; ++g) M = fmaxf(M, parts[g].m);
-  double Z = 0.0, Sx = 0.0;
-  ArgMax b{-FLT_MAX, 0x7fffffff};
-  for (int g = 0; g < segs; ++g) {
-    const Partial& p = parts[g];
-    if (p.z > 0.0) {
-      const float d = p.m - M;
-      const double sc = (double)exp2_ftz(d * kLog2e);
-      Z += p.z * sc;
-      Sx += sc * (p.s + (double)d * p.z);
-    }
-    if (better(p.bv, p.bi, b.v, b.i)) b = ArgMax{p.bv, p.bi};
+template <int KM>
+__global__ void __launch_bounds__(kRowThreads, 1)
+gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ num_nodes,
+                 int q_count, int cap, const float* __restrict__ root_logits,
+                 const float* __restrict__ node_logits, int vocab, int kappa, float thr,
+                 int unnormalized, int segs, int seg4, unsigned* __restrict__ next_task,
+                 Partial* __restrict__ parts, unsigned* __restrict__ done,
+                 int32_t* __restrict__ stats, uint32_t* status) {
+  extern __shared__ __align__(128) float4 ring_all[];
+  __shared__ __align__(8) uint64_t bars_all[kWarps * kWStages];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    for (int b = 0; b < kWarps * kWStages; ++b) ptx::mbar_init(ptx::smem_u32(bars_all + b), 1);
+    ptx::fence_barrier_init();
   }
-  const float H = logf((float)Z) - (float)(Sx / Z);
-  const float score = unnormalized ? H : H / logf((float)vocab);
-  out[0] = b.i;
-  out[1] = (score > thr) ? 1 : 0;
-  int head[kMaxSegs];
-  for (int g = 0; g < segs; ++g) head[g] = 0;
-  for (int r = 0; r < kappa; ++r) {
-    int bg = -1;
-    ArgMax bb{-FLT_MAX, 0x7fffffff};
-    for (int g = 0; g < segs; ++g) {
-      if (head[g] >= kappa) continue;
-      const float v = parts[g].tv[head[g]];
-      const int ix = parts[g].ti[head[g]];
-      if (bg < 0 || better(v, ix, bb.v, bb.i)) {
-        bb = ArgMax{v, ix};
-        bg = g;
+  __syncthreads();
+  float4* ring = ring_all + (size_t)wid * kWStages * kWStageF4;
+  uint64_t* bars = bars_all + wid * kWStages;
+  const uint64_t pol = (lane == 0) ? ptx::policy_evict_first() : 0ull;
+  __shared__ Partial s_part[kWarps];  // the partial of a one-piece row
+  const unsigned n_tasks = (unsigned)q_count * (unsigned)(cap + 1) * (unsigned)segs;
+  const int n4 = vocab >> 2;
+  uint32_t seq = 0;
+  while (true) {
+    unsigned t = 0;
+    if (lane == 0) t = atomicAdd(next_task, 1u);
+    t = __shfl_sync(0xffffffffu, t, 0);
+    if (t >= n_tasks) break;
+    const unsigned rid = t / (unsigned)segs;  // row task: q * (cap + 1) + slot
+    const int seg = (int)(t - rid * (unsigned)segs);
+    const int q = (int)(rid / (unsigned)(cap + 1));
+    const int slot = (int)(rid - (unsigned)q * (unsigned)(cap + 1));  // 0 = root, 1 + n = node n
+    const float* row;
+    if (slot == 0) {
+      row = root_logits + (int64_t)q * vocab;
+    } else {
+      const int nd = slot - 1;
+      const int nn = min(num_nodes[q], cap);
+      const bool inner = (nd + 1 < nn) && parent[(int64_t)q * cap + nd + 1] == nd;
+      if (!inner) continue;
+      row = node_logits + ((int64_t)q * cap + nd) * vocab;
+    }
+    const int lo4 = seg * seg4;
+    const int hi4 = min(n4, lo4 + seg4);
+    Partial* slot_out = (segs == 1) ? &s_part[wid] : parts + (int64_t)rid * segs + seg;
+    if (!warp_segment<KM>(row, lo4, hi4, kappa, ring, bars, seq, pol, slot_out)) {
+      if (lane == 0) raise_status(status, SENSE_DEVST_TIMEOUT);
+      break;
+    }
+    int32_t* out = stats + (int64_t)rid * kStatsInts;
+    if (segs == 1) {
+      __syncwarp();
+      finish_row(&s_part[wid], 1, vocab, kappa, thr, unnormalized, out);
+    } else {
+      // the row's last segment to finish merges the partials
+      unsigned last = 0;
+      if (lane == 0) {
+        __threadfence();
+        last = atomicAdd(&done[rid], 1u) == (unsigned)segs - 1u;
+      }
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (last) {
+        __threadfence();
+        finish_row(parts + (int64_t)rid * segs, segs, vocab, kappa, thr, unnormalized, out);
+        if (lane == 0) done[rid] = 0u;
       }
     }
-    out[2 + r] = bb.i;
-    if (bg >= 0) ++head[bg];
-  }
-  for (int r = kappa; r < SENSE_MAX_KAPPA; ++r) out[2 + r] = -1;
-}
-
-template <int KM>
-__global__ void __launch_bounds__(kRowThreads)
-gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ num_nodes,
-                 int cap, const float* __restrict__ root_logits,
-                 const float* __restrict__ node_logits, int vocab, int kappa, float thr,
-                 int unnormalized, int segs, int seg4, Partial* __restrict__ parts,
-                 unsigned* __restrict__ done, int32_t* __restrict__ stats, uint32_t* status) {
-  extern __shared__ __align__(128) float4 ring[];
-  __shared__ __align__(8) uint64_t full[kStages];
-  __shared__ int s_last;
-  const int slot = blockIdx.x / segs;  // 0 = root, 1 + n = node n
-  const int seg = blockIdx.x - slot * segs;
-  const int q = blockIdx.y;
-  const float* row;
-  if (slot == 0) {
-    row = root_logits + (int64_t)q * vocab;
-  } else {
-    const int n = slot - 1;
-    const int nn = min(num_nodes[q], cap);
-    const bool inner = (n + 1 < nn) && parent[(int64_t)q * cap + n + 1] == n;
-    if (!inner) return;
-    row = node_logits + ((int64_t)q * cap + n) * vocab;
-  }
-  const int n4 = vocab >> 2;
-  const int lo4 = seg * seg4;
-  const int hi4 = min(n4, lo4 + seg4);
-  const int64_t rid = (int64_t)q * (cap + 1) + slot;
-  Partial* rp = parts + rid * segs;
-  if (!segment_stats<KM>(row, lo4, hi4, kappa, rp + seg, ring, full)) {
-    if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_TIMEOUT);
-    return;
-  }
-  if (segs == 1) {
-    __syncthreads();
-    if (threadIdx.x == 0) finish_row(rp, 1, vocab, kappa, thr, unnormalized, stats + rid * kStatsInts);
-    return;
-  }
-  // last block of the row to finish merges the segments
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(&done[rid], 1u) == (unsigned)segs - 1u);
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  if (threadIdx.x == 0) {
-    finish_row(rp, segs, vocab, kappa, thr, unnormalized, stats + rid * kStatsInts);
-    done[rid] = 0u;
+    __syncwarp();
   }
 }
 
@@ -639,25 +699,28 @@ gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats) {
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+}  // namespace
+
+// Segments per row: enough row pieces for every streaming warp of the
+// grid, each piece at least two stages long.
 int gate_segments(int q, int cap, int vocab) {
   const int64_t rows = (int64_t)q * (cap + 1);
-  const int n4 = vocab >> 2;
-  int64_t segs = (2LL * sm_count() + rows - 1) / rows;
-  const int64_t by_len = n4 / (2 * kStageF4);  // at least two stages per segment
+  const int64_t warps = (int64_t)sm_count() * kWarps;
+  int64_t segs = (warps + rows - 1) / rows;
+  const int64_t by_len = (vocab >> 2) / (2 * kWStageF4);
   if (segs > by_len) segs = by_len;
   if (segs > kMaxSegs) segs = kMaxSegs;
   if (segs < 1) segs = 1;
   return (int)segs;
 }
 
-}  // namespace
-
 size_t gate_workspace_bytes(int q, int cap, int kappa) {
   (void)kappa;
   const size_t rows = (size_t)q * (cap + 1);
+  const int segs = gate_segments(q, cap, 1 << 30);  // upper bound over vocabularies
   size_t b = align256(rows * kStatsInts * sizeof(int32_t));
-  b += align256(rows * kMaxSegs * sizeof(Partial));
-  b += align256(rows * sizeof(unsigned));
+  b += 256;  // task counter
+  if (segs > 1) b += align256(rows * segs * sizeof(Partial)) + align256(rows * sizeof(unsigned));
   return b;
 }
 
@@ -666,31 +729,37 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
   char* ws = static_cast<char*>(a.workspace);
   int32_t* stats = reinterpret_cast<int32_t*>(ws);
   ws += align256(rows * kStatsInts * sizeof(int32_t));
-  Partial* parts = reinterpret_cast<Partial*>(ws);
-  ws += align256(rows * kMaxSegs * sizeof(Partial));
-  unsigned* done = reinterpret_cast<unsigned*>(ws);
+  unsigned* next_task = reinterpret_cast<unsigned*>(ws);
+  ws += 256;
   const int segs = gate_segments(a.q, a.cap, a.vocab);
   const int n4 = a.vocab >> 2;
   const int seg4 = (n4 + segs - 1) / segs;
+  Partial* parts = reinterpret_cast<Partial*>(ws);
+  unsigned* done = nullptr;
+  if (segs > 1) done = reinterpret_cast<unsigned*>(ws + align256(rows * segs * sizeof(Partial)));
+  sense_status st = cuda_check(cudaMemsetAsync(next_task, 0, sizeof(unsigned), s),
+                               "clear gate task counter");
+  if (st != SENSE_OK) return st;
   if (segs > 1) {
-    sense_status st = cuda_check(cudaMemsetAsync(done, 0, rows * sizeof(unsigned), s),
-                                 "clear gate counters");
+    st = cuda_check(cudaMemsetAsync(done, 0, rows * sizeof(unsigned), s), "clear gate counters");
     if (st != SENSE_OK) return st;
   }
   {
-    dim3 grid((unsigned)((a.cap + 1) * segs), a.q);
-    const size_t ring = (size_t)kStages * kStageBytes;
     auto k4 = gate_rows_kernel<4>;
     auto k16 = gate_rows_kernel<SENSE_MAX_KAPPA>;
     auto kern = (a.kappa <= 4) ? k4 : k16;
-    sense_status st = cuda_check(
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ring),
+    st = cuda_check(
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kRingBytes),
         "cudaFuncSetAttribute(gate_rows)");
     if (st != SENSE_OK) return st;
+    // persistent: one block of kWarps row-streaming warps per SM; with few
+    // row pieces, spread them over as many SMs as there are pieces
+    int64_t blocks = sm_count();
+    if (blocks > (int64_t)rows * segs) blocks = (int64_t)rows * segs;
     LaunchScope ls(K_GATE_ROWS, s);
-    kern<<<grid, kRowThreads, ring, s>>>(a.parent, a.num_nodes, a.cap, a.root_logits,
-                                         a.node_logits, a.vocab, a.kappa, a.thr, a.unnormalized,
-                                         segs, seg4, parts, done, stats, a.status);
+    kern<<<(unsigned)blocks, kRowThreads, kRingBytes, s>>>(
+        a.parent, a.num_nodes, a.q, a.cap, a.root_logits, a.node_logits, a.vocab, a.kappa, a.thr,
+        a.unnormalized, segs, seg4, next_task, parts, done, stats, a.status);
     st = cuda_check(cudaGetLastError(), "launch gate_rows");
     if (st != SENSE_OK) return st;
   }
