@@ -35,9 +35,12 @@ from synth.workloads import WORKLOADS  # noqa: E402
 DEFAULT = "llama7b_1m"
 METRIC = "hidden-state top-k retrieval queries/s (whole drafting step)"
 GATE = dict(gamma=0.05, topk=3, window=6, tau=0)
-# dram bytes (read + write) per launch of the dominant kernel from one ncu
-# capture, or None when the kernel changed since the capture.
-NCU_TRAFFIC = {}
+# DRAM bytes (read + write) per launch of the dominant kernel on the default
+# workload, from one ncu capture (profiles/scan_gemv_llama7b_1m.md): the
+# 262,144-key case read 2.14776 GB and wrote 2.92 MB; traffic grows with the
+# rows scanned, so x4 for the 1,048,576-key store.  None once the kernel
+# changes after the capture.
+NCU_TRAFFIC = {("scan_gemv", "llama7b_1m"): (2.147761e9 + 2.923264e6) * 4}
 
 
 def peaks():
@@ -348,12 +351,14 @@ def main():
     e2e_steps = min(args.e2e_steps, args.steps)
     if gate_bytes > (1 << 30):
         e2e_steps = min(e2e_steps, 10)
+    if gate_bytes > (4 << 30):
+        e2e_steps = 0  # per-step inputs beyond host staging (reported as skipped)
     h_query = torch.empty_like(queries[0], device="cpu").pin_memory()
     h_query.copy_(queries[0])
     gsrc = gate_sets[0]
-    h_gate = [t.to("cpu").pin_memory() for t in gsrc]
+    h_gate = [t.to("cpu").pin_memory() for t in gsrc] if gate_bytes <= (4 << 30) else []
     d_query = torch.empty_like(queries[0])
-    d_gate = [torch.empty_like(t) for t in gsrc]
+    d_gate = [torch.empty_like(t) for t in gsrc] if h_gate else []
     h_scores = torch.empty(q, cfg["k"], dtype=torch.float32).pin_memory()
     h_idx = torch.empty(q, cfg["k"], dtype=torch.int32).pin_memory()
     h_acc = torch.empty(q, cfg["m"], dtype=torch.int32).pin_memory()
@@ -361,6 +366,8 @@ def main():
     h_hnext = torch.empty(q, d, dtype=torch.bfloat16).pin_memory()
     h2d = h_query.numel() * h_query.element_size() + sum(t.numel() * t.element_size() for t in h_gate)
     d2h = sum(t.numel() * t.element_size() for t in (h_scores, h_idx, h_acc, h_small, h_hnext))
+    if e2e_steps == 0:
+        h_gate = []
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for it in range(e2e_steps):
@@ -378,7 +385,7 @@ def main():
         h_hnext.copy_(pipe.gate["h_next"], non_blocking=True)
         torch.cuda.current_stream().synchronize()
     e2e_s = max_over_ranks(time.perf_counter() - t0, dist, dev)
-    e2e_value = job_throughput(q * e2e_steps, world, e2e_s)
+    e2e_value = job_throughput(q * e2e_steps, world, e2e_s) if e2e_steps else None
 
     base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -394,20 +401,23 @@ def main():
             "config": {"workload": args.workload,
                        **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab", "cap", "clusters")},
                        "key_bytes": n * d * 2,
-                       "l2": "inputs larger than L2: the 8.6 GB store is streamed every step",
+                       "l2": f"inputs larger than L2: the {n * d * 2 / 1e9:.1f} GB store is "
+                             "streamed every step",
                        "parallelism": f"replicas x{world}"},
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,
             "draft_tokens_per_s": value * mean_nodes,
             "mean_tree_nodes": mean_nodes,
             "roofline": {"bound": "hbm", "kernel": scan_name, "achieved": achieved,
                          "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                         "peak_kind": peak_kind, "traffic": NCU_TRAFFIC.get(scan_name),
+                         "peak_kind": peak_kind,
+                         "traffic": NCU_TRAFFIC.get((scan_name, args.workload)),
                          "launches": scan_launches, "kernel_ms": scan_ms},
             "kernel_ms": {k: round(v[0], 4) for k, v in prof.items() if v[1]},
             "gpu_launches": launches,
             "clocks": clk,
-            "e2e": {"value": e2e_value, "unit": "queries/s", "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+            "e2e": ({"value": e2e_value, "unit": "queries/s", "h2d_bytes_per_step": h2d,
+                     "d2h_bytes_per_step": d2h, "steps": e2e_steps} if e2e_steps else
+                    {"value": None, "skipped": "per-step gate inputs exceed 4 GB of host staging"}),
             "cpu_baseline": base,
         }
         print(json.dumps(line), flush=True)
