@@ -266,12 +266,17 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=200)
     ap.add_argument("--n-keys", type=int, default=0,
                     help="override the store size (small cases for profiler captures)")
+    ap.add_argument("--queries", type=int, default=0,
+                    help="override the queries per step (small cases for profiler captures)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     cfg = dict(WORKLOADS[args.workload])
     if args.n_keys > 0:
         cfg["n"] = args.n_keys
         args.workload = f"{args.workload}@n={args.n_keys}"
+    if args.queries > 0:
+        cfg["q"] = args.queries
+        args.workload = f"{args.workload}@q={args.queries}"
     if args.impl == "reference":
         run_reference(args, cfg, args.workload)
         return
