@@ -9,8 +9,10 @@ from .sense_oracle import (  # noqa: F401
     gather_drafts,
     loose_trie,
     loose_trie_alg3,
+    mask_from_bits,
     normalize_keys_bf16,
     scores,
     soft_gate,
     topk,
+    tree_mask_full,
 )

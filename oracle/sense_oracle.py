@@ -19,6 +19,8 @@ for floating point, following the step order and notation of the paper:
                         Alg. 2 forced anchor
   loose_trie           §3.2.3 Eq. 9 (sorted-LCP trie), node-capped
   loose_trie_alg3      App. C.3 Alg. 3 restated step by step (uncapped)
+  mask_from_bits,      App. C.6 Eq. 20 (additive tree attention mask over a
+  tree_mask_full        static KV cache) from Alg. 3's mask M
   soft_gate            §3.3 Eqs. 11-19 and App. C.4 Alg. 4
 
 Readings where the paper is silent or ambiguous are stated at each function.
@@ -314,6 +316,53 @@ def loose_trie_alg3(d_sorted_or_not: np.ndarray):
     for i in range(n):
         mask[gam[i, ii], gam[i, jj]] = 1
     return t_flat, gam, mask, pi
+
+
+# ----------------------------------------------------------------------------
+# tree attention mask over a static KV cache (App. C.6 Eq. 20)
+# ----------------------------------------------------------------------------
+
+
+def mask_from_bits(bits_rows: np.ndarray, num_nodes: int) -> np.ndarray:
+    """Alg. 3's 0/1 draft mask M (L x L) from ancestor bit rows.
+
+    ``bits_rows[n, w]`` holds bits 32w..32w+31 of row n (the layout of
+    ``loose_trie(..., mask_bits=True)``): M[n, b] = bit b of row n.
+    """
+    b = np.asarray(bits_rows)
+    big_l = int(num_nodes)
+    out = np.zeros((big_l, big_l), dtype=np.int64)
+    for n in range(big_l):
+        for c in range(big_l):
+            out[n, c] = (int(b[n, c // 32]) >> (c % 32)) & 1
+    return out
+
+
+def tree_mask_full(M: np.ndarray, m: int, cache_len: int, rows=None) -> np.ndarray:
+    """Additive attention mask M_full of App. C.6 Eq. 20, fp64.
+
+    The L draft tokens sit at cache positions m..m+L-1 behind m committed
+    tokens, in a static cache of cache_len positions.  Row i (draft token i)
+    gets 0 at column j when j < m (every committed token is visible) or when
+    m <= j < m+L and M[i, j-m] = 1 (an ancestor-or-self tree token), and
+    -inf everywhere else.
+
+    Reading: ``rows`` >= L pads the output for a fixed node capacity; a
+    padding row has no tree entries, so the same rule gives it 0 on the
+    committed columns and -inf elsewhere.  m + L must fit in the cache.
+    """
+    big_m = np.asarray(M)
+    big_l = big_m.shape[0]
+    rows = big_l if rows is None else int(rows)
+    if m < 0 or m + big_l > cache_len or rows < big_l:
+        raise ValueError("need 0 <= m, m + L <= cache_len and rows >= L")
+    out = np.full((rows, cache_len), -np.inf)
+    out[:, :m] = 0.0
+    for i in range(big_l):
+        for c in range(big_l):
+            if big_m[i, c] == 1:
+                out[i, m + c] = 0.0
+    return out
 
 
 # ----------------------------------------------------------------------------

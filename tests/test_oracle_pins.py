@@ -438,3 +438,71 @@ def test_gate_cap_truncation():
                       np.zeros((1, 1)), np.zeros((1, 5, 1)), gamma_thr=-1.0, kappa=v)
     assert out["G"][0].tolist() == [[1, 1, 1, 1], [1, 0, 0, 0]]
     assert out["i_star"][0] == 0 and out["L_star"][0] == 3
+
+
+# --------------------------------------------------------------------------
+# tree attention mask over a static KV cache (App. C.6 Eq. 20)
+# --------------------------------------------------------------------------
+
+def test_tree_mask_full_chain_is_shifted_causal():
+    # one span -> a chain: every draft token sees the committed tokens and
+    # the draft tokens up to itself, i.e. the textbook causal mask
+    m, cache, depth = 5, 16, 7
+    tr = O.loose_trie(np.array([[3, 1, 4, 1, 5, 9, 2]]), mask_bits=True)
+    M = O.mask_from_bits(tr["mask_bits"][0], tr["num_nodes"][0])
+    np.testing.assert_array_equal(M, np.tril(np.ones((depth, depth), dtype=np.int64)))
+    full = O.tree_mask_full(M, m, cache)
+    causal = np.triu(np.full((m + depth, m + depth), -np.inf), k=1)[m:]
+    want = np.full((depth, cache), -np.inf)
+    want[:, :m + depth] = causal
+    np.testing.assert_array_equal(full, want)
+
+
+def test_tree_mask_full_golden():
+    g = json.load(open(os.path.join(GOLDEN, "trie_small.json")))
+    u = g["uncapped"]
+    words = np.array(u["mask_words"], dtype=np.uint32)[:, None]
+    M = O.mask_from_bits(words, u["num_nodes"])
+    _, _, mask_alg3, _ = O.loose_trie_alg3(np.array(g["spans"]))
+    np.testing.assert_array_equal(M, mask_alg3)
+    full = O.tree_mask_full(M, 2, 14, rows=12)
+    # node 5 is the path (5, 4, 0) = nodes 0, 4, 5: committed columns 0, 1
+    # plus cache positions 2 + {0, 4, 5}
+    assert np.nonzero(full[5] == 0)[0].tolist() == [0, 1, 2, 6, 7]
+    # every row sees m + depth + 1 columns; padding rows see the m committed
+    assert (full[:9] == 0).sum(axis=1).tolist() == [2 + d + 1 for d in u["depth"]]
+    assert (full[9:] == 0).sum(axis=1).tolist() == [2, 2, 2]
+    assert np.all(full[9:, :2] == 0)
+    with pytest.raises(ValueError):
+        O.tree_mask_full(M, 6, 14)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_tree_mask_full_attention_equals_per_path_causal(seed):
+    # Tree attention with M_full over the cache gives each draft token the
+    # same output as causal attention over its own sequence (committed
+    # tokens, then its root path), computed here by torch's reference SDPA.
+    rng = np.random.default_rng(300 + seed)
+    spans = _rand_spans(rng, 6, 4, 3)
+    tr = O.loose_trie(spans, mask_bits=True)
+    L = int(tr["num_nodes"][0])
+    M = O.mask_from_bits(tr["mask_bits"][0], L)
+    m, cache, hd = 5, 5 + L + 3, 8
+    g = torch.Generator().manual_seed(seed)
+    q = torch.randn(L, hd, generator=g, dtype=torch.float64)
+    kc = torch.randn(cache, hd, generator=g, dtype=torch.float64)
+    vc = torch.randn(cache, hd, generator=g, dtype=torch.float64)
+    full = torch.from_numpy(O.tree_mask_full(M, m, cache))
+    tree_out = torch.softmax(q @ kc.T / math.sqrt(hd) + full, dim=-1) @ vc
+    par = tr["parent"][0]
+    for i in range(L):
+        path, p = [], i
+        while p >= 0:
+            path.append(p)
+            p = par[p]
+        cols = list(range(m)) + [m + n for n in reversed(path)]
+        qs = torch.zeros(len(cols), hd, dtype=torch.float64)
+        qs[-1] = q[i]
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            qs[None], kc[cols][None], vc[cols][None], is_causal=True)[0, -1]
+        torch.testing.assert_close(tree_out[i], ref, rtol=1e-12, atol=1e-12)
