@@ -30,6 +30,7 @@ if ROOT not in sys.path:
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
+import synth  # noqa: E402
 from synth.workloads import WORKLOADS  # noqa: E402
 
 DEFAULT = "llama7b_1m"
@@ -120,7 +121,8 @@ def job_throughput(units_per_rank: int, world: int, seconds: float) -> float:
 def make_workload(cfg, dev, seed=0):
     import synth
     n, d, m = cfg["n"], cfg["d"], cfg["m"]
-    keys = synth.clustered_unit_keys(n, d, cfg["clusters"], sigma=0.3, seed=seed, device=dev)
+    keys, assign = synth.clustered_unit_keys(n, d, cfg["clusters"], sigma=0.3, seed=seed,
+                                             device=dev, return_assign=True)
     if cfg["zipf"]:
         spans = synth.spans_zipf(n, m, cfg["vocab"], 1.1, seed=seed, device=dev)
     else:
@@ -128,7 +130,7 @@ def make_workload(cfg, dev, seed=0):
     n_q = cfg["distinct"] * cfg["q"]
     queries, src = synth.noisy_queries(keys, n_q, noise=0.05, seed=seed + 1)
     queries = queries.reshape(cfg["distinct"], cfg["q"], d).contiguous()
-    return keys, spans, queries
+    return keys, spans, queries, assign
 
 
 def make_gate_inputs(cfg, dev, sets=4, seed=0):
@@ -296,7 +298,7 @@ def main():
     _build.build()
     S.lib()
 
-    keys, spans, queries = make_workload(cfg, dev, seed=rank)
+    keys, spans, queries, assign = make_workload(cfg, dev, seed=rank)
     cap = cfg["cap"] if cfg["cap"] > 0 else cfg["k"] * cfg["m"]
     gate_bytes = cfg["q"] * (cap + 1) * cfg["vocab"] * 4
     n_sets = 4 if gate_bytes < (2 << 30) else 1
@@ -346,11 +348,34 @@ def main():
     step_bytes = scan_bytes_per_step  # gate/tree bytes are <0.1% of the scan here
 
     # draft tree size (nodes per query) over a few steps, for draft tokens/s
-    nodes = []
+    # and the loose trie's compression of the k*m candidate tokens (Sec. 4.3
+    # "Loose Trie Compression"): distinct prefixes of the uncapped trie, on
+    # the workload's spans and on spans that share prefixes within a key
+    # cluster (the same retrieved indices)
+    nodes, distinct, distinct_t = [], [], []
+    tspans = synth.spans_cluster_template(assign, cfg["clusters"], cfg["m"], cfg["vocab"],
+                                          seed=rank)
+    tds = S.sense_datastore_build(keys, tspans)
+    tdrafts = torch.empty_like(pipe.drafts)
     for it in range(16):
         pipe.step(queries[it % nq], gate_sets[it % n_sets])
         nodes.append(pipe.tree["num_nodes"].float().mean().item())
+        full = S.sense_build_tree(pipe.drafts, node_cap=0)
+        distinct.append(full["num_nodes"].float().mean().item())
+        S.sense_gather_drafts(tds, pipe.idx, out=tdrafts)
+        full = S.sense_build_tree(tdrafts, node_cap=0)
+        distinct_t.append(full["num_nodes"].float().mean().item())
+    del tds, tspans, tdrafts, full
     mean_nodes = float(np.mean(nodes))
+    km = cfg["k"] * cfg["m"]
+
+    def compression(dist):
+        return {"distinct_prefixes": float(np.mean(dist)),
+                "nodes_over_tokens": float(np.mean(dist)) / km,
+                "compression": 1.0 - float(np.mean(dist)) / km}
+    trie = {"candidate_tokens": km, "workload_spans": compression(distinct),
+            "cluster_template_spans": compression(distinct_t),
+            "capped_nodes": mean_nodes, "cap": pipe.cap}
 
     # end to end through the C ABI with host buffers
     e2e_steps = min(args.e2e_steps, args.steps)
@@ -412,6 +437,7 @@ def main():
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,
             "draft_tokens_per_s": value * mean_nodes,
             "mean_tree_nodes": mean_nodes,
+            "trie_compression": trie,
             "roofline": {"bound": "hbm", "kernel": scan_name, "achieved": achieved,
                          "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                          "peak_kind": peak_kind,

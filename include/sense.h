@@ -54,6 +54,8 @@ typedef enum sense_status {
 #define SENSE_DEVST_BAD_TOKEN 0x2u   /* tree: negative token id in a span     */
 #define SENSE_DEVST_TIMEOUT 0x4u     /* a pipeline wait hit its limit         */
 #define SENSE_DEVST_INTERNAL 0x8u    /* an internal consistency check failed  */
+#define SENSE_DEVST_BAD_LENGTH 0x10u /* tree mask: committed length + nodes
+                                        outside [0, cache_len]               */
 
 /* Key storage types for sense_datastore_build. */
 #define SENSE_KEY_BF16 0
@@ -226,6 +228,35 @@ sense_status sense_build_tree(const int32_t* spans, int32_t q, int32_t k, int32_
                               int32_t node_cap, uint32_t flags, int32_t* out_num_nodes,
                               int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
                               int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* Tree attention mask over a static KV cache                               */
+/* ---------------------------------------------------------------------- */
+/*
+ * App. C.6 Eq. 20: the additive mask M_full with which the target model
+ * verifies all L = num_nodes draft tokens in one forward pass over a static
+ * KV cache.  The draft tokens occupy cache positions m .. m+L-1 behind the
+ * m committed tokens.  For draft token i and cache position j:
+ *   M_full[i, j] = 0     if j < m,
+ *                = 0     if m <= j < m+L and node j-m is an ancestor of i
+ *                        or i itself (Alg. 3's M, from sense_build_tree's
+ *                        SENSE_TREE_MASK_BITS output),
+ *                = -inf  otherwise.
+ * Rows i >= L pad the fixed capacity: they get 0 on the m committed
+ * columns and -inf elsewhere.
+ *
+ *   mask_bits [q, cap, ceil(cap/32)] uint32 (bit b of row n: M[n, b]);
+ *   num_nodes [q] int32 (L); prefix_len [q] int32 (m);
+ *   out [q, cap, cache_len] f32.
+ *   Limits: q >= 1, 1 <= cap <= SENSE_MAX_TREE_TOKENS, cache_len >= 1;
+ *   arrays 4-byte aligned (16-byte aligned out with cache_len % 4 == 0
+ *   takes the vector store path).
+ * A query with m < 0 or m + L > cache_len (or L outside [0, cap]) sets
+ * SENSE_DEVST_BAD_LENGTH and gets rows of -inf.
+ */
+sense_status sense_tree_mask_full(const uint32_t* mask_bits, const int32_t* num_nodes, int32_t q,
+                                  int32_t cap, const int32_t* prefix_len, int32_t cache_len,
+                                  float* out, sense_stream_t stream);
 
 /* ---------------------------------------------------------------------- */
 /* a6. Soft-gated evaluation                                                */

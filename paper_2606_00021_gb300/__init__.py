@@ -19,7 +19,7 @@ SENSE_OK = 0
 STATUS_NAMES = {0: "SENSE_OK", 1: "SENSE_ERR_INVALID_ARG", 2: "SENSE_ERR_UNSUPPORTED",
                 3: "SENSE_ERR_OOM", 4: "SENSE_ERR_CUDA", 5: "SENSE_ERR_DEVICE_STATUS",
                 6: "SENSE_ERR_TIMEOUT"}
-DEVST_BAD_INDEX, DEVST_BAD_TOKEN, DEVST_TIMEOUT, DEVST_INTERNAL = 1, 2, 4, 8
+DEVST_BAD_INDEX, DEVST_BAD_TOKEN, DEVST_TIMEOUT, DEVST_INTERNAL, DEVST_BAD_LENGTH = 1, 2, 4, 8, 16
 
 
 class SenseError(RuntimeError):
@@ -235,6 +235,24 @@ def sense_build_tree(spans: torch.Tensor, node_cap: int = 0, mask_bits: bool = F
                                   C.c_void_p(_stream(stream))))
     o["cap"] = cap
     return o
+
+
+def sense_tree_mask_full(tree: dict, prefix_len: torch.Tensor, cache_len: int,
+                         out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Additive static-KV attention mask [q, cap, cache_len] f32 of a tree
+    built with mask_bits=True; prefix_len [q] int32 committed lengths."""
+    bits = tree["mask_bits"]
+    _need(bits, "mask_bits", torch.int32, 3)
+    _need(tree["num_nodes"], "num_nodes", torch.int32, 1)
+    _need(prefix_len, "prefix_len", torch.int32, 1)
+    q, cap, _ = bits.shape
+    if out is None:
+        out = torch.empty(q, cap, cache_len, dtype=torch.float32, device=bits.device)
+    _need(out, "out", torch.float32, 3)
+    _check(lib().sense_tree_mask_full(bits.data_ptr(), tree["num_nodes"].data_ptr(), q, cap,
+                                      prefix_len.data_ptr(), cache_len, out.data_ptr(),
+                                      C.c_void_p(_stream(stream))))
+    return out
 
 
 def sense_soft_gate_workspace_bytes(q: int, cap: int, kappa: int) -> int:

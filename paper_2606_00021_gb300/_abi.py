@@ -30,6 +30,7 @@ SIGNATURES = {
     "sense_gather_drafts": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_i32, c_u32, c_p, c_p]),
     "sense_build_tree": (c_i32, [c_p, c_i32, c_i32, c_i32, c_i32, c_u32, c_p, c_p, c_p, c_p,
                                  c_p, c_p, c_p]),
+    "sense_tree_mask_full": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_i32, c_p, c_p]),
     "sense_soft_gate_workspace_bytes": (c_size, [c_i32, c_i32, c_i32]),
     "sense_soft_gate": (c_i32, [c_p, c_p, c_p, c_p, c_i32, c_i32, c_i32, c_i32, c_p, c_p, c_i32,
                                 c_p, c_p, c_i32, C.POINTER(GateParams), c_p, c_p, c_p, c_p, c_p,

@@ -30,7 +30,8 @@ std::vector<ProfRec> g_prof;
 std::vector<cudaEvent_t> g_ev_pool;
 const char* const kKernelNames[K_COUNT] = {
     "normalize", "scan_gemv", "scan_tc", "threshold", "merge",
-    "gather",    "tree",      "gate_rows", "gate_decide", "pad_queries"};
+    "gather",    "tree",      "gate_rows", "gate_decide", "pad_queries",
+    "tree_mask"};
 
 cudaEvent_t take_event() {
   if (!g_ev_pool.empty()) {
@@ -417,6 +418,23 @@ sense_status sense_build_tree(const int32_t* spans, int32_t q, int32_t k, int32_
   if (!status) return SENSE_ERR_OOM;
   return launch_tree(spans, q, k, m, cap, bits ? 1 : 0, out_num_nodes, out_tokens, out_parent,
                      out_depth, out_gamma, out_mask_bits, status, stream);
+}
+
+sense_status sense_tree_mask_full(const uint32_t* mask_bits, const int32_t* num_nodes, int32_t q,
+                                  int32_t cap, const int32_t* prefix_len, int32_t cache_len,
+                                  float* out, sense_stream_t stream) {
+  if (!mask_bits || !num_nodes || !prefix_len || !out)
+    return fail(SENSE_ERR_INVALID_ARG, "mask_bits, num_nodes, prefix_len and out must be non-NULL");
+  if (q < 1) return fail(SENSE_ERR_INVALID_ARG, "q=%d must be >= 1", q);
+  if (cap < 1 || cap > SENSE_MAX_TREE_TOKENS)
+    return fail(SENSE_ERR_INVALID_ARG, "cap=%d outside [1, %d]", cap, SENSE_MAX_TREE_TOKENS);
+  if (cache_len < 1) return fail(SENSE_ERR_INVALID_ARG, "cache_len=%d must be >= 1", cache_len);
+  if (!aligned(mask_bits, 4) || !aligned(num_nodes, 4) || !aligned(prefix_len, 4) || !aligned(out, 4))
+    return fail(SENSE_ERR_INVALID_ARG, "arrays must be 4-byte aligned");
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  return launch_tree_mask_full(mask_bits, num_nodes, prefix_len, q, cap, cache_len, out, status,
+                               stream);
 }
 
 size_t sense_soft_gate_workspace_bytes(int32_t q, int32_t cap, int32_t kappa) {

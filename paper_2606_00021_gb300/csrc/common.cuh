@@ -34,6 +34,7 @@ enum KernelId {
   K_GATE_ROWS,
   K_GATE_DECIDE,
   K_PAD_QUERIES,
+  K_TREE_MASK,
   K_COUNT
 };
 

@@ -21,6 +21,13 @@
 //      preorder by a second prefix count;
 //   5. outputs: tokens/parent/depth, gamma back in the candidates' order,
 //      optional ancestor bit mask.
+//
+// tree mask (App. C.6 Eq. 20): the additive attention mask of the draft
+// tokens over a static KV cache, written from the ancestor bit rows.  One
+// block per output row (grid-stride); the row's mask words are staged in
+// shared memory and the row is written with 16-byte stores.
+#include <algorithm>
+
 #include "common.cuh"
 #include "launch.h"
 
@@ -343,6 +350,47 @@ tree_kernel(const int32_t* __restrict__ spans, int k, int m, int cap, int mask_w
   }
 }
 
+
+// Row r = (query qi, draft token i) of the [q, cap, cache_len] mask.
+template <bool VEC>
+__global__ void __launch_bounds__(256)
+tree_mask_full_kernel(const uint32_t* __restrict__ mask_bits, const int32_t* __restrict__ num_nodes,
+                      const int32_t* __restrict__ prefix_len, int q, int cap, int words,
+                      int cache_len, float* __restrict__ out, uint32_t* status) {
+  __shared__ uint32_t s_w[SENSE_MAX_TREE_TOKENS / 32];
+  const float NEG = -__int_as_float(0x7f800000);
+  const int64_t rows = (int64_t)q * cap;
+  for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
+    const int qi = (int)(r / cap), i = (int)(r - (int64_t)qi * cap);
+    const int L = num_nodes[qi], m = prefix_len[qi];
+    const bool bad = m < 0 || L < 0 || L > cap || (int64_t)m + L > cache_len;
+    if (bad && i == 0 && threadIdx.x == 0) raise_status(status, SENSE_DEVST_BAD_LENGTH);
+    const bool tree_row = !bad && i < L;
+    __syncthreads();  // s_w of the previous row is no longer read
+    if (tree_row)
+      for (int w = threadIdx.x; w < words; w += blockDim.x)
+        s_w[w] = mask_bits[r * words + w];
+    __syncthreads();
+    const int lo = bad ? 0 : m;          // columns [0, lo) are 0
+    const int hi = tree_row ? m + L : 0;  // tree columns [lo, hi) follow the bits
+    auto val = [&](int c) -> float {
+      if (c < lo) return 0.0f;
+      if (c < hi) {
+        const int b = c - m;
+        return ((s_w[b >> 5] >> (b & 31)) & 1u) ? 0.0f : NEG;
+      }
+      return NEG;
+    };
+    float* row = out + r * cache_len;
+    if (VEC) {
+      for (int c = 4 * threadIdx.x; c < cache_len; c += 4 * blockDim.x)
+        *reinterpret_cast<float4*>(row + c) = make_float4(val(c), val(c + 1), val(c + 2), val(c + 3));
+    } else {
+      for (int c = threadIdx.x; c < cache_len; c += blockDim.x) row[c] = val(c);
+    }
+  }
+}
+
 }  // namespace
 
 sense_status launch_gather(const int32_t* spans, int64_t n, int m, const int32_t* idx, int q,
@@ -377,6 +425,23 @@ sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int
   tree_kernel<<<q, threads, smem, s>>>(spans, k, m, cap, words, num_nodes, tokens, parent,
                                             depth, gamma, mask_bits ? mask : nullptr, status);
   return cuda_check(cudaGetLastError(), "launch tree");
+}
+
+sense_status launch_tree_mask_full(const uint32_t* mask_bits, const int32_t* num_nodes,
+                                   const int32_t* prefix_len, int q, int cap, int cache_len,
+                                   float* out, uint32_t* status, cudaStream_t s) {
+  const int words = (cap + 31) / 32;
+  const int64_t rows = (int64_t)q * cap;
+  const int grid = (int)std::min<int64_t>(rows, (int64_t)sm_count() * 16);
+  const bool vec = (cache_len % 4 == 0) && (reinterpret_cast<uintptr_t>(out) % 16 == 0);
+  LaunchScope ls(K_TREE_MASK, s);
+  if (vec)
+    tree_mask_full_kernel<true><<<grid, 256, 0, s>>>(mask_bits, num_nodes, prefix_len, q, cap,
+                                                     words, cache_len, out, status);
+  else
+    tree_mask_full_kernel<false><<<grid, 256, 0, s>>>(mask_bits, num_nodes, prefix_len, q, cap,
+                                                      words, cache_len, out, status);
+  return cuda_check(cudaGetLastError(), "launch tree mask");
 }
 
 }  // namespace sense

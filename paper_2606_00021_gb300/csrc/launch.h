@@ -119,6 +119,13 @@ sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int
                          int32_t* num_nodes, int32_t* tokens, int32_t* parent, int32_t* depth,
                          int32_t* gamma, uint32_t* mask, uint32_t* status, cudaStream_t s);
 
+// Additive mask of App. C.6 Eq. 20 for q trees of capacity cap:
+// out[q, cap, cache_len] f32 from the ancestor bit rows mask_bits
+// [q, cap, ceil(cap/32)], the node counts and the committed lengths.
+sense_status launch_tree_mask_full(const uint32_t* mask_bits, const int32_t* num_nodes,
+                                   const int32_t* prefix_len, int q, int cap, int cache_len,
+                                   float* out, uint32_t* status, cudaStream_t s);
+
 struct GateArgs {
   const int32_t* tokens;
   const int32_t* parent;

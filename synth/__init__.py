@@ -133,6 +133,28 @@ def spans_zipf(n: int, m: int, vocab: int, s: float = 1.1, seed: int = 0,
     return out
 
 
+
+def spans_cluster_template(assign: torch.Tensor, n_clusters: int, m: int, vocab: int,
+                           s: float = 1.1, seed: int = 0) -> torch.Tensor:
+    """int32 [n, m] spans that share prefixes within a key cluster.
+
+    Each cluster owns one Zipf(s) template span; a key of that cluster keeps
+    the template's first l tokens, l uniform on {0..m}, and draws the rest
+    from Zipf(s) (nearby hidden states tend to continue alike)."""
+    dev = assign.device
+    n = assign.shape[0]
+    tmpl = spans_zipf(n_clusters, m, vocab, s, seed=_sub_seed(seed, 10), device=dev)
+    fresh = spans_zipf(n, m, vocab, s, seed=_sub_seed(seed, 11), device=dev)
+    out = torch.empty(n, m, dtype=torch.int32, device=dev)
+    col = torch.arange(m, device=dev)
+    for ci, lo in enumerate(range(0, n, CHUNK_ROWS * 16)):
+        hi = min(n, lo + CHUNK_ROWS * 16)
+        g = _gen(dev, _sub_seed(seed, 12, ci))
+        keep = torch.randint(0, m + 1, (hi - lo, 1), generator=g, device=dev)
+        a = assign[lo:hi].long()
+        out[lo:hi] = torch.where(col[None, :] < keep, tmpl[a], fresh[lo:hi])
+    return out
+
 def gate_logits(q: int, rows: int, vocab: int, std: float = 3.0, seed: int = 0,
                 device="cpu", out: torch.Tensor | None = None) -> torch.Tensor:
     """fp32 [q, rows, vocab] i.i.d. N(0, std^2)."""

@@ -61,6 +61,12 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert lib.sense_build_tree(p, 1, 1024, 16, 0, 0, *args) == 1
     assert lib.sense_build_tree(p, 1, 4, 4, -1, 0, *args) == 1
     assert lib.sense_build_tree(p, 1, 4, 4, 0, 1, *args) == 1  # mask bits without buffer
+    # tree mask: q, cap, cache_len, NULL output
+    assert lib.sense_tree_mask_full(p, p, 0, 8, p, 16, p, None) == 1
+    assert lib.sense_tree_mask_full(p, p, 1, 0, p, 16, p, None) == 1
+    assert lib.sense_tree_mask_full(p, p, 1, 8193, p, 16, p, None) == 1
+    assert lib.sense_tree_mask_full(p, p, 1, 8, p, 0, p, None) == 1
+    assert lib.sense_tree_mask_full(p, p, 1, 8, p, 16, None, None) == 1
     # gate parameters
     from paper_2606_00021_gb300._abi import GateParams
     gp = GateParams(0.05, 0, 6, 0, 0)

@@ -230,6 +230,60 @@ def test_tree_special_cases_and_bad_token(S):
     np.testing.assert_array_equal(host(got["tokens"][0]), want0["tokens"][0])
 
 
+# ---------------------------------------------------------------- tree mask (Eq. 20)
+
+def _mask_want(sp, cap, prefix, cache_len):
+    tr = O.loose_trie(sp, node_cap=cap, mask_bits=True)
+    rows = tr["tokens"].shape[1]
+    out = np.empty((sp.shape[0], rows, cache_len))
+    for qi in range(sp.shape[0]):
+        nn = int(tr["num_nodes"][qi])
+        M = O.mask_from_bits(tr["mask_bits"][qi], nn)
+        out[qi] = O.tree_mask_full(M, int(prefix[qi]), cache_len, rows=rows)
+    return out
+
+
+@cuda
+@pytest.mark.parametrize("q,k,m,vocab,cap,cache_len", [
+    (3, 8, 8, 5, 64, 256), (2, 32, 16, 3, 128, 1027), (2, 64, 8, 4, 0, 600),
+    (1, 1, 5, 3, 0, 5), (4, 16, 4, 2, 33, 97),
+])
+def test_tree_mask_full_matches_oracle(S, q, k, m, vocab, cap, cache_len):
+    dev = torch.device("cuda")
+    sp = _tree_spans(q, k, m, vocab, seed=q * 31 + k + cache_len)
+    tree = S.sense_build_tree(torch.from_numpy(sp).to(dev), node_cap=cap, mask_bits=True)
+    nn = host(tree["num_nodes"])
+    rng = np.random.default_rng(cache_len)
+    # committed lengths from 0 up to the largest that fits (m + L == cache_len)
+    prefix = np.array([int(rng.integers(0, cache_len - nn[qi] + 1)) for qi in range(q)],
+                      dtype=np.int32)
+    prefix[0] = cache_len - nn[0]
+    if q > 1:
+        prefix[1] = 0
+    got = S.sense_tree_mask_full(tree, torch.from_numpy(prefix).to(dev), cache_len)
+    torch.cuda.synchronize()
+    assert _clear(S) == 0
+    want = _mask_want(sp, cap, prefix, cache_len).astype(np.float32)
+    np.testing.assert_array_equal(host(got), want)
+
+
+@cuda
+def test_tree_mask_full_flags_bad_length(S):
+    dev = torch.device("cuda")
+    sp = _tree_spans(3, 8, 6, 4, seed=5)
+    tree = S.sense_build_tree(torch.from_numpy(sp).to(dev), node_cap=40, mask_bits=True)
+    nn = host(tree["num_nodes"])
+    cache_len = 64
+    prefix = np.array([3, cache_len - nn[1] + 1, -1], dtype=np.int32)
+    _clear(S)
+    got = host(S.sense_tree_mask_full(tree, torch.from_numpy(prefix).to(dev), cache_len))
+    st = S.sense_device_status(clear=True)
+    assert st == S.DEVST_BAD_LENGTH
+    assert np.all(got[1:] == -np.inf)
+    want = _mask_want(sp[:1], 40, prefix[:1], cache_len).astype(np.float32)
+    np.testing.assert_array_equal(got[:1], want)
+
+
 # ---------------------------------------------------------------- gate
 
 def _gate_case(q, k, m, v, d, cap, seed, plant=True):
