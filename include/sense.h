@@ -38,6 +38,7 @@ extern "C" {
 
 typedef struct CUstream_st* sense_stream_t;
 typedef struct sense_datastore sense_datastore;
+typedef struct sense_ivf sense_ivf;
 
 typedef enum sense_status {
   SENSE_OK = 0,
@@ -71,6 +72,10 @@ typedef enum sense_status {
 /* Tree flags. */
 #define SENSE_TREE_MASK_BITS 0x1u
 
+/* Projection / k-means flags. */
+#define SENSE_PROJECT_NORMALIZE 0x1u /* unit L2 norm of every projected row   */
+#define SENSE_KMEANS_SPHERICAL 0x1u  /* inner-product assignment, unit centroids */
+
 /* Gate flags. */
 #define SENSE_GATE_UNNORMALIZED_ENTROPY 0x1u
 
@@ -80,6 +85,7 @@ typedef enum sense_status {
 #define SENSE_MAX_TREE_TOKENS 8192 /* k * m accepted by sense_build_tree      */
 #define SENSE_MAX_KAPPA 16        /* gate top-k                               */
 #define SENSE_MAX_WINDOW 64       /* gate lookahead window                    */
+#define SENSE_MAX_PROJ_DIM 128    /* projected key dimension                  */
 
 int32_t sense_version(void);
 const char* sense_status_string(sense_status s);
@@ -172,6 +178,110 @@ sense_status sense_retrieve_topk(const sense_datastore* ds, const uint16_t* quer
 sense_status sense_retrieve_topk_noalloc(const sense_datastore* ds, const uint16_t* queries,
                                          int32_t q, int32_t k, float* out_scores,
                                          int32_t* out_idx, sense_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* Approximate retrieval: PCA projection and an IVF / IVF-PQ index          */
+/* ---------------------------------------------------------------------- */
+/*
+ * Sec. 3.2.2 Eq. 7 retrieves with ANN(k_t, C_db, N'); App. E builds it from
+ * final-layer hidden states projected by PCA to 64 dimensions and
+ * L2-normalised (Alg. 2: k = L2Norm(PCA(h))), indexed by FAISS IVF-PQ with
+ * nlist = 4096 cells, nprobe = 32 and pq_m = 16 sub-quantizers.
+ *
+ * Arithmetic: fp32 without fused multiply-add, in a fixed order, so that
+ * every decision (cell, code, probe, top-k index) is reproducible:
+ * projected-space dot products and squared distances are summed term by
+ * term in index order; the projection's length-d dot products are summed as
+ * 32 interleaved partial sums (partial l takes the 4-column groups g with
+ * g mod 32 = l, ascending) combined by an xor butterfly (16, 8, 4, 2, 1).
+ */
+
+/*
+ * y = (x - mean) W^T for bf16 rows x [n, d] and a basis W [v, d] f32 (rows =
+ * principal axes); mean [d] f32 or NULL.  With SENSE_PROJECT_NORMALIZE each
+ * row is then divided by its L2 norm (zero rows stay zero).  out [n, v] f32.
+ * Limits: d % 8 == 0, 1 <= v <= SENSE_MAX_PROJ_DIM; x, basis, mean 16-byte
+ * aligned.  The PCA basis itself is fitted offline by the caller.
+ */
+sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float* basis, int32_t v,
+                           const float* mean, uint32_t flags, float* out, sense_stream_t stream);
+
+/*
+ * Lloyd's k-means (training of the coarse quantizer and of the PQ
+ * codebooks): `iters` rounds of assignment (SENSE_KMEANS_SPHERICAL: largest
+ * inner product, else smallest squared L2 distance; ties to the lowest
+ * centroid) and update (member means accumulated as 2^-31 fixed-point
+ * integers, divided in fp64, rounded to fp32; an empty cluster keeps its
+ * centroid; spherical: then unit norm; spherical seeds are normalised
+ * first).  x [n, dim] f32 with row stride ld floats (dim in {4, 8, 16, 32,
+ * 64, 128}); init [k, dim] seeds; centroids [k, dim] out; out_assign [n]
+ * (last round's assignment) or NULL.  workspace: at least
+ * sense_kmeans_workspace_bytes(n, dim, k) bytes, 256-byte aligned.
+ * Limits: 1 <= n < 2^31, 1 <= k <= 65536, iters >= 0.
+ */
+size_t sense_kmeans_workspace_bytes(int64_t n, int32_t dim, int32_t k);
+sense_status sense_kmeans(const float* x, int64_t n, int32_t dim, int32_t ld, int32_t k,
+                          int32_t iters, uint32_t flags, const float* init, float* centroids,
+                          int32_t* out_assign, void* workspace, size_t workspace_bytes,
+                          sense_stream_t stream);
+
+/*
+ * Cell of each vector (largest inner product with a centroid, ties to the
+ * lowest cell) and its residual r = x - c_cell, for training PQ codebooks.
+ * vecs [n, v] f32, centroids [nlist, v]; out_cell [n] int32,
+ * out_residuals [n, v] f32.  v in {16, 32, 64, 128}, nlist <= 16384.
+ */
+sense_status sense_ivf_residuals(const float* vecs, int64_t n, int32_t v, const float* centroids,
+                                 int32_t nlist, int32_t* out_cell, float* out_residuals,
+                                 sense_stream_t stream);
+
+/*
+ * Builds an inverted-file index over unit vectors vecs [n, v] f32 (copied;
+ * the index owns its memory, allocated here, freed by sense_ivf_destroy).
+ *  - cell of x = arg max_c <x, c> over centroids [nlist, v] (unit centroids:
+ *    the nearest one);
+ *  - lists in cell order, members in ascending key index;
+ *  - codebooks NULL (pq_m = 0): the lists hold the vectors (IVF-flat);
+ *    codebooks [pq_m, 256, v / pq_m] f32: the lists hold 8-bit codes of
+ *    the residual x - c_cell, sub-vector m coded as its nearest codeword
+ *    (squared L2, ties to the lowest index), as FAISS IVF-PQ encodes.
+ * Synchronises `stream` (it reads the longest list length back).
+ * Limits: n < 2^31, v in {16, 32, 64, 128}, nlist <= 16384, v / pq_m <= 16.
+ */
+sense_status sense_ivf_build(const float* vecs, int64_t n, int32_t v, const float* centroids,
+                             int32_t nlist, const float* codebooks, int32_t pq_m,
+                             sense_stream_t stream, sense_ivf** out);
+sense_status sense_ivf_destroy(sense_ivf* ix);
+
+/*
+ * Read-only view of an index: out_info [5] = {n, v, nlist, pq_m, longest
+ * list}; device pointers to the list offsets [nlist + 1] int64, the key
+ * index of each slot [n] int32 and the payload (flat: vectors [n, v] f32;
+ * PQ: codes [n, pq_m] uint8), in list order.  Any output may be NULL.
+ */
+sense_status sense_ivf_arrays(const sense_ivf* ix, int64_t* out_info, const int64_t** out_offsets,
+                              const int32_t** out_ids, const void** out_payload);
+
+/*
+ * Top-k of the approximate scores over the nprobe best cells, per query:
+ *  - coarse score <q, c> for every cell; the nprobe largest are probed
+ *    (ties to the lower cell); out_probes [q, nprobe] int32 or NULL;
+ *  - IVF-flat: score = <q, x>; IVF-PQ: score = <q, c_cell> +
+ *    sum_m <q_m, B_m[code_m]> (m ascending), the inner product decomposed
+ *    over the residual;
+ *  - out_scores [q, k] f32 / out_idx [q, k] int32 key indices, order (score
+ *    desc, index asc); slots past the number of candidates in the probed
+ *    lists get -inf / -1.
+ * queries [q, v] f32 (projected, e.g. by sense_project).  workspace: at
+ * least sense_ivf_search_workspace_bytes(ix, q, k, nprobe) bytes, 256-byte
+ * aligned.  Limits: 1 <= q <= 65535, 1 <= k <= SENSE_MAX_K,
+ * 1 <= nprobe <= min(nlist, SENSE_MAX_K).
+ */
+size_t sense_ivf_search_workspace_bytes(const sense_ivf* ix, int32_t q, int32_t k, int32_t nprobe);
+sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t q, int32_t k,
+                              int32_t nprobe, float* out_scores, int32_t* out_idx,
+                              int32_t* out_probes, void* workspace, size_t workspace_bytes,
+                              sense_stream_t stream);
 
 /* ---------------------------------------------------------------------- */
 /* a4. Span gather                                                          */

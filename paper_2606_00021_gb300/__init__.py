@@ -255,6 +255,148 @@ def sense_tree_mask_full(tree: dict, prefix_len: torch.Tensor, cache_len: int,
     return out
 
 
+# ---------------------------------------------------------------- approximate retrieval
+
+def sense_project(x: torch.Tensor, basis: torch.Tensor, mean: torch.Tensor | None = None,
+                  normalize: bool = True, out: torch.Tensor | None = None,
+                  stream=None) -> torch.Tensor:
+    """(x - mean) basis^T [n, v] f32 for bf16 rows x [n, d] (unit rows with
+    ``normalize``): the query / key construction k = L2Norm(PCA(h))."""
+    _need(x, "x", torch.bfloat16, 2)
+    _need(basis, "basis", torch.float32, 2)
+    n, d = x.shape
+    v = basis.shape[0]
+    if basis.shape[1] != d:
+        raise ValueError("basis must be [v, d]")
+    if mean is not None:
+        _need(mean, "mean", torch.float32, 1)
+    if out is None:
+        out = torch.empty(n, v, dtype=torch.float32, device=x.device)
+    _need(out, "out", torch.float32, 2)
+    _check(lib().sense_project(x.data_ptr(), n, d, basis.data_ptr(), v, _ptr(mean),
+                               1 if normalize else 0, out.data_ptr(),
+                               C.c_void_p(_stream(stream))))
+    return out
+
+
+def sense_kmeans(x: torch.Tensor, init: torch.Tensor, iters: int, spherical: bool,
+                 want_assign: bool = False, stream=None):
+    """Lloyd's k-means on the rows of x [n, dim] f32 (rows may be strided, e.g.
+    a column slice of a wider matrix) from seeds init [k, dim]; returns
+    centroids (and the last round's assignment with ``want_assign``)."""
+    if not isinstance(x, torch.Tensor) or x.dtype != torch.float32 or x.dim() != 2 \
+            or x.device.type != "cuda" or x.stride(1) != 1:
+        raise ValueError("x must be a CUDA float32 [n, dim] tensor with unit column stride")
+    _need(init, "init", torch.float32, 2)
+    n, dim = x.shape
+    ld = x.stride(0) if n > 1 else dim
+    k = init.shape[0]
+    if init.shape[1] != dim:
+        raise ValueError("init must be [k, dim]")
+    cent = torch.empty(k, dim, dtype=torch.float32, device=x.device)
+    assign = _i32((n,), x.device) if want_assign else None
+    ws = alloc_workspace(lib().sense_kmeans_workspace_bytes(n, dim, k), x.device)
+    _check(lib().sense_kmeans(x.data_ptr(), n, dim, ld, k, iters, 1 if spherical else 0,
+                              init.data_ptr(), cent.data_ptr(), _ptr(assign), ws.data_ptr(),
+                              ws.numel(), C.c_void_p(_stream(stream))))
+    return (cent, assign) if want_assign else cent
+
+
+def sense_ivf_residuals(vecs: torch.Tensor, centroids: torch.Tensor, stream=None):
+    """(cell int32 [n], residual f32 [n, v]) of each vector."""
+    _need(vecs, "vecs", torch.float32, 2)
+    _need(centroids, "centroids", torch.float32, 2)
+    n, v = vecs.shape
+    cell = _i32((n,), vecs.device)
+    res = torch.empty_like(vecs)
+    _check(lib().sense_ivf_residuals(vecs.data_ptr(), n, v, centroids.data_ptr(),
+                                     centroids.shape[0], cell.data_ptr(), res.data_ptr(),
+                                     C.c_void_p(_stream(stream))))
+    return cell, res
+
+
+@dataclass
+class IvfIndex:
+    """Handle of an IVF-flat / IVF-PQ index (library-owned device memory)."""
+    handle: int
+    n: int
+    v: int
+    nlist: int
+    pq_m: int
+    max_list: int
+
+    def close(self):
+        if self.handle:
+            lib().sense_ivf_destroy(C.c_void_p(self.handle))
+            self.handle = 0
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def arrays(self) -> dict:
+        """Zero-copy views of the lists (valid while the index is open)."""
+        off, ids, pay = C.c_void_p(0), C.c_void_p(0), C.c_void_p(0)
+        info = (C.c_int64 * 5)()
+        _check(lib().sense_ivf_arrays(C.c_void_p(self.handle), info, C.byref(off), C.byref(ids),
+                                      C.byref(pay)))
+        view = lambda p, shape, ts: torch.as_tensor(_DeviceArray(p.value, shape, ts), device="cuda")
+        out = {"offsets": view(off, (self.nlist + 1,), "<i8"), "ids": view(ids, (self.n,), "<i4")}
+        if self.pq_m:
+            out["codes"] = view(pay, (self.n, self.pq_m), "|u1")
+        else:
+            out["vectors"] = view(pay, (self.n, self.v), "<f4")
+        return out
+
+
+def sense_ivf_build(vecs: torch.Tensor, centroids: torch.Tensor,
+                    codebooks: torch.Tensor | None = None, stream=None) -> IvfIndex:
+    """IVF-flat (codebooks None) or IVF-PQ (codebooks [pq_m, 256, v/pq_m]) index."""
+    _need(vecs, "vecs", torch.float32, 2)
+    _need(centroids, "centroids", torch.float32, 2)
+    n, v = vecs.shape
+    pq_m = 0
+    if codebooks is not None:
+        _need(codebooks, "codebooks", torch.float32, 3)
+        pq_m = codebooks.shape[0]
+    out = C.c_void_p(0)
+    _check(lib().sense_ivf_build(vecs.data_ptr(), n, v, centroids.data_ptr(), centroids.shape[0],
+                                 _ptr(codebooks), pq_m, C.c_void_p(_stream(stream)),
+                                 C.byref(out)))
+    info = (C.c_int64 * 5)()
+    _check(lib().sense_ivf_arrays(out, info, None, None, None))
+    return IvfIndex(out.value, n, v, centroids.shape[0], pq_m, int(info[4]))
+
+
+def sense_ivf_search_workspace_bytes(ix: IvfIndex, q: int, k: int, nprobe: int) -> int:
+    return int(lib().sense_ivf_search_workspace_bytes(C.c_void_p(ix.handle), q, k, nprobe))
+
+
+def sense_ivf_search(ix: IvfIndex, queries: torch.Tensor, k: int, nprobe: int,
+                     out_scores=None, out_idx=None, want_probes: bool = False, workspace=None,
+                     stream=None):
+    """Approximate top-k: (scores f32 [q, k], idx int32 [q, k][, probes int32 [q, nprobe]])."""
+    _need(queries, "queries", torch.float32, 2)
+    q = queries.shape[0]
+    if queries.shape[1] != ix.v:
+        raise ValueError(f"queries must have {ix.v} columns")
+    dev = queries.device
+    if out_scores is None:
+        out_scores = torch.empty(q, k, dtype=torch.float32, device=dev)
+    if out_idx is None:
+        out_idx = _i32((q, k), dev)
+    probes = _i32((q, nprobe), dev) if want_probes else None
+    if workspace is None:
+        workspace = alloc_workspace(sense_ivf_search_workspace_bytes(ix, q, k, nprobe), dev)
+    _check(lib().sense_ivf_search(C.c_void_p(ix.handle), queries.data_ptr(), q, k, nprobe,
+                                  out_scores.data_ptr(), out_idx.data_ptr(), _ptr(probes),
+                                  workspace.data_ptr(), workspace.numel(),
+                                  C.c_void_p(_stream(stream))))
+    return (out_scores, out_idx, probes) if want_probes else (out_scores, out_idx)
+
+
 def sense_soft_gate_workspace_bytes(q: int, cap: int, kappa: int) -> int:
     return int(lib().sense_soft_gate_workspace_bytes(q, cap, kappa))
 

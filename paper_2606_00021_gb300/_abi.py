@@ -31,6 +31,17 @@ SIGNATURES = {
     "sense_build_tree": (c_i32, [c_p, c_i32, c_i32, c_i32, c_i32, c_u32, c_p, c_p, c_p, c_p,
                                  c_p, c_p, c_p]),
     "sense_tree_mask_full": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_i32, c_p, c_p]),
+    "sense_project": (c_i32, [c_p, c_i64, c_i32, c_p, c_i32, c_p, c_u32, c_p, c_p]),
+    "sense_kmeans_workspace_bytes": (c_size, [c_i64, c_i32, c_i32]),
+    "sense_kmeans": (c_i32, [c_p, c_i64, c_i32, c_i32, c_i32, c_i32, c_u32, c_p, c_p, c_p, c_p,
+                             c_size, c_p]),
+    "sense_ivf_residuals": (c_i32, [c_p, c_i64, c_i32, c_p, c_i32, c_p, c_p, c_p]),
+    "sense_ivf_build": (c_i32, [c_p, c_i64, c_i32, c_p, c_i32, c_p, c_i32, c_p, C.POINTER(c_p)]),
+    "sense_ivf_destroy": (c_i32, [c_p]),
+    "sense_ivf_arrays": (c_i32, [c_p, C.POINTER(c_i64), C.POINTER(c_p), C.POINTER(c_p),
+                                 C.POINTER(c_p)]),
+    "sense_ivf_search_workspace_bytes": (c_size, [c_p, c_i32, c_i32, c_i32]),
+    "sense_ivf_search": (c_i32, [c_p, c_p, c_i32, c_i32, c_i32, c_p, c_p, c_p, c_p, c_size, c_p]),
     "sense_soft_gate_workspace_bytes": (c_size, [c_i32, c_i32, c_i32]),
     "sense_soft_gate": (c_i32, [c_p, c_p, c_p, c_p, c_i32, c_i32, c_i32, c_i32, c_p, c_p, c_i32,
                                 c_p, c_p, c_i32, C.POINTER(GateParams), c_p, c_p, c_p, c_p, c_p,

@@ -35,6 +35,11 @@ enum KernelId {
   K_GATE_DECIDE,
   K_PAD_QUERIES,
   K_TREE_MASK,
+  K_PROJECT,
+  K_KMEANS,
+  K_IVF_BUILD,
+  K_IVF_COARSE,
+  K_IVF_SCAN,
   K_COUNT
 };
 

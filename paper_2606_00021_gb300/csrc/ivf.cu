@@ -1,0 +1,927 @@
+// Approximate retrieval over projected keys: PCA projection, k-means, and an
+// inverted-file index with flat vectors or product-quantised residuals.
+//
+// Sec. 3.2.2 Eq. 7 retrieves the top-N' by ANN(k_t, C_db, N'); App. E sets it
+// up: hidden states projected by PCA to 64 dimensions and L2-normalised
+// (Alg. 2, k = L2Norm(PCA(h))), a FAISS IVF-PQ index with nlist = 4096,
+// nprobe = 32 and pq_m = 16.  Every step here ends in an integer decision (a
+// cell, a code, a probe, a top-k index), so the arithmetic follows one fixed
+// fp32 evaluation order, with no fused multiply-add (__fmul_rn / __fadd_rn):
+//  - projected-space dot products and squared distances (dimension <= 128)
+//    are summed term by term, index ascending, by one thread;
+//  - the projection's long dot products (dimension d) are summed by the 32
+//    lanes of a warp: lane l owns the 4-column groups g with g mod 32 = l,
+//    in ascending order, and the lane sums are combined by an xor butterfly
+//    (offsets 16, 8, 4, 2, 1);
+//  - k-means sums are 2^-31 fixed-point integers (order-free atomics),
+//    divided in fp64.
+// Kernels:
+//  project_rows_kernel   one warp per (row, output): query batches
+//  project_tile_kernel   16 rows x 32 outputs per block, 16 warps, each lane
+//                        holding 4 x 8 partial sums: key stores
+//  normalize_rows_kernel one thread per row
+//  assign_kernel<D,MODE> one thread per vector, centroids staged in shared
+//                        memory: k-means and cell assignment (arg max inner
+//                        product or arg min L2) and the coarse scores of a
+//                        search (thread per cell, queries staged)
+//  kmeans_accum / kmeans_finish: fixed-point member sums, new centroids
+//  list kernels          stable counting sort of the cells (per-block
+//                        histograms, a column scan, one warp placing each
+//                        block's ids in order)
+//  pq_encode_kernel      residual sub-vector -> nearest of 256 codewords
+//  ivf_scan_kernel       one block per (probe, query): flat dot products or
+//                        LUT sums, candidates appended to the query's pool;
+//                        the exact top-k of the pool is the existing merge.
+#include <algorithm>
+#include <vector>
+
+#include "common.cuh"
+#include "launch.h"
+
+struct sense_ivf {
+  int64_t n;
+  int32_t v;
+  int32_t nlist;
+  int32_t pq_m;  // 0: flat
+  int32_t dsub;
+  int64_t max_list;
+  int device;
+  float* centroids;  // [nlist, v]
+  float* codebooks;  // [pq_m, 256, dsub] or null
+  int64_t* offsets;  // [nlist + 1]
+  int32_t* ids;      // [n] key index of each list slot
+  float* vectors;    // flat: [n, v] in list order
+  uint8_t* codes;    // pq: [n, pq_m] in list order
+};
+
+namespace sense {
+namespace {
+
+constexpr int kIdBlock = 4096;   // ids per block of the stable counting sort
+constexpr int kMaxList = 16384;  // nlist limit (per-block histogram in shared memory)
+constexpr float kFix = 2147483648.0f;  // 2^31
+
+enum AssignMode { ARGMAX_IP = 0, ARGMIN_L2 = 1, ALL_IP = 2 };
+
+// ---------------------------------------------------------------------------
+// projection
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ float madd(float acc, float a, float b) {
+  return __fadd_rn(acc, __fmul_rn(a, b));
+}
+
+__device__ __forceinline__ float butterfly(float v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, off));
+  return v;
+}
+
+// Four bf16 columns j..j+3 of a row, centred (x - mu, rounded to fp32).
+__device__ __forceinline__ float4 load_x4(const uint16_t* xr, const float* mu, int j) {
+  const uint2 w = *reinterpret_cast<const uint2*>(xr + j);
+  float4 x = make_float4(bf_lo(w.x), bf_hi(w.x), bf_lo(w.y), bf_hi(w.y));
+  if (mu) {
+    const float4 m = *reinterpret_cast<const float4*>(mu + j);
+    x = make_float4(__fsub_rn(x.x, m.x), __fsub_rn(x.y, m.y), __fsub_rn(x.z, m.z),
+                    __fsub_rn(x.w, m.w));
+  }
+  return x;
+}
+
+__global__ void __launch_bounds__(256)
+project_rows_kernel(const uint16_t* __restrict__ x, int64_t n, int d,
+                    const float* __restrict__ w, int v, const float* __restrict__ mu,
+                    float* __restrict__ out) {
+  const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (gw >= n * v) return;  // warp-uniform
+  const int64_t row = gw / v;
+  const int o = (int)(gw - row * v);
+  const uint16_t* xr = x + row * d;
+  const float* wr = w + (int64_t)o * d;
+  float acc = 0.0f;
+  for (int j = 4 * lane; j < d; j += 128) {
+    const float4 xv = load_x4(xr, mu, j);
+    const float4 wv = *reinterpret_cast<const float4*>(wr + j);
+    acc = madd(acc, xv.x, wv.x);
+    acc = madd(acc, xv.y, wv.y);
+    acc = madd(acc, xv.z, wv.z);
+    acc = madd(acc, xv.w, wv.w);
+  }
+  acc = butterfly(acc);
+  if (lane == 0) out[row * v + o] = acc;
+}
+
+// Block: 16 rows x 32 outputs, 16 warps.  Warp w takes rows 4*(w & 3) .. +3
+// and outputs 8*(w >> 2) .. +7 of the block's 32; lane l keeps the 32
+// partial sums of its column groups.  Columns are staged 128 at a time.
+constexpr int kPtRows = 16, kPtOuts = 32, kPtCols = 128;
+
+__global__ void __launch_bounds__(512)
+project_tile_kernel(const uint16_t* __restrict__ x, int64_t n, int d,
+                    const float* __restrict__ w, int v, const float* __restrict__ mu,
+                    float* __restrict__ out) {
+  __shared__ __align__(16) float xs[kPtRows][kPtCols];
+  __shared__ __align__(16) float ws[kPtOuts][kPtCols];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t row0 = (int64_t)blockIdx.x * kPtRows;
+  const int out0 = blockIdx.y * kPtOuts;
+  const int rg = 4 * (warp & 3), og = 8 * (warp >> 2);
+  float acc[4][8];
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int o = 0; o < 8; ++o) acc[r][o] = 0.0f;
+  for (int c0 = 0; c0 < d; c0 += kPtCols) {
+    __syncthreads();
+    // stage x: 16 rows x 128 columns as 4-column groups (512 groups)
+    {
+      const int r = threadIdx.x >> 5, g = threadIdx.x & 31;
+      const int64_t row = row0 + r;
+      float4 xv = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (row < n && c0 + 4 * g < d) xv = load_x4(x + row * d, mu, c0 + 4 * g);
+      *reinterpret_cast<float4*>(&xs[r][4 * g]) = xv;
+    }
+    // stage w: 32 outputs x 128 columns (1024 float4, 2 per thread)
+    for (int e = threadIdx.x; e < kPtOuts * 32; e += blockDim.x) {
+      const int o = e >> 5, g = e & 31;
+      float4 wv = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (out0 + o < v && c0 + 4 * g < d)
+        wv = *reinterpret_cast<const float4*>(w + (int64_t)(out0 + o) * d + c0 + 4 * g);
+      *reinterpret_cast<float4*>(&ws[o][4 * g]) = wv;
+    }
+    __syncthreads();
+    if (c0 + 4 * lane < d) {
+      float4 xv[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) xv[r] = *reinterpret_cast<const float4*>(&xs[rg + r][4 * lane]);
+#pragma unroll
+      for (int o = 0; o < 8; ++o) {
+        const float4 wv = *reinterpret_cast<const float4*>(&ws[og + o][4 * lane]);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          float a = acc[r][o];
+          a = madd(a, xv[r].x, wv.x);
+          a = madd(a, xv[r].y, wv.y);
+          a = madd(a, xv[r].z, wv.z);
+          a = madd(a, xv[r].w, wv.w);
+          acc[r][o] = a;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int o = 0; o < 8; ++o) acc[r][o] = butterfly(acc[r][o]);
+  // every lane holds the 32 sums; lane l writes (r, o) = (l / 8, l % 8)
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+#pragma unroll
+    for (int o = 0; o < 8; ++o) {
+      if (lane == 8 * r + o) {
+        const int64_t row = row0 + rg + r;
+        const int oo = out0 + og + o;
+        if (row < n && oo < v) out[row * v + oo] = acc[r][o];
+      }
+    }
+  }
+}
+
+__global__ void normalize_rows_kernel(float* __restrict__ y, int64_t n, int v) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  float* r = y + i * v;
+  float s = 0.0f;
+  for (int o = 0; o < v; ++o) s = madd(s, r[o], r[o]);
+  const float nrm = __fsqrt_rn(s);
+  for (int o = 0; o < v; ++o) r[o] = nrm > 0.0f ? __fdiv_rn(r[o], nrm) : 0.0f;
+}
+
+// ---------------------------------------------------------------------------
+// assignment / coarse scores
+// ---------------------------------------------------------------------------
+
+// One thread per row of x ([n, D], row stride ld floats); the rows of c
+// ([k, D], contiguous) are staged in shared memory tiles.
+//  ARGMAX_IP: out_assign[i] = arg max_c <x_i, c> (first maximum)
+//  ARGMIN_L2: out_assign[i] = arg min_c ||x_i - c||^2 (first minimum)
+//  ALL_IP:    x = cells, c = queries: pool[c * n + i] = key(<x_i, c>, i)
+template <int D, int MODE>
+__global__ void __launch_bounds__(128)
+assign_kernel(const float* __restrict__ x, int64_t n, int ld, const float* __restrict__ c,
+              int k, int32_t* __restrict__ out_assign, uint64_t* __restrict__ pool) {
+  constexpr int kTile = (D <= 16) ? 256 : (8192 / D);
+  __shared__ __align__(16) float cs[kTile * D];
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const bool live = i < n;
+  float xr[D];
+#pragma unroll
+  for (int j = 0; j < D; ++j) xr[j] = live ? x[i * ld + j] : 0.0f;
+  float best = (MODE == ARGMIN_L2) ? __int_as_float(0x7f800000) : -__int_as_float(0x7f800000);
+  int arg = 0;
+  for (int t0 = 0; t0 < k; t0 += kTile) {
+    const int tn = min(kTile, k - t0);
+    __syncthreads();
+    for (int e = threadIdx.x; e < tn * D; e += blockDim.x) cs[e] = c[(int64_t)t0 * D + e];
+    __syncthreads();
+    if (!live) continue;
+    for (int t = 0; t < tn; ++t) {
+      const float* cr = cs + t * D;
+      float s = 0.0f;
+      if (MODE == ARGMIN_L2) {
+#pragma unroll
+        for (int j = 0; j < D; ++j) {
+          const float u = __fsub_rn(xr[j], cr[j]);
+          s = madd(s, u, u);
+        }
+        if (s < best || (t0 + t == 0)) {
+          best = s;
+          arg = t0 + t;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < D; ++j) s = madd(s, xr[j], cr[j]);
+        if (MODE == ALL_IP) {
+          pool[(int64_t)(t0 + t) * n + i] = cand_key(s, (uint32_t)i);
+        } else if (s > best || (t0 + t == 0)) {
+          best = s;
+          arg = t0 + t;
+        }
+      }
+    }
+  }
+  if (MODE != ALL_IP && live) out_assign[i] = arg;
+}
+
+template <int MODE>
+sense_status launch_assign_mode(const float* x, int64_t n, int dim, int ld, const float* c, int k,
+                                int32_t* out_assign, uint64_t* pool, cudaStream_t s) {
+  const dim3 grid((unsigned)((n + 127) / 128));
+#define SENSE_ASSIGN_CASE(DD)                                                               \
+  case DD:                                                                                  \
+    assign_kernel<DD, MODE><<<grid, 128, 0, s>>>(x, n, ld, c, k, out_assign, pool);         \
+    break;
+  switch (dim) {
+    SENSE_ASSIGN_CASE(4)
+    SENSE_ASSIGN_CASE(8)
+    SENSE_ASSIGN_CASE(16)
+    SENSE_ASSIGN_CASE(32)
+    SENSE_ASSIGN_CASE(64)
+    SENSE_ASSIGN_CASE(128)
+    default:
+      return fail(SENSE_ERR_UNSUPPORTED, "dimension %d not in {4, 8, 16, 32, 64, 128}", dim);
+  }
+#undef SENSE_ASSIGN_CASE
+  return cuda_check(cudaGetLastError(), "launch assign");
+}
+
+// ---------------------------------------------------------------------------
+// k-means update
+// ---------------------------------------------------------------------------
+
+__global__ void kmeans_accum_kernel(const float* __restrict__ x, int64_t n, int dim, int ld,
+                                    const int32_t* __restrict__ assign,
+                                    unsigned long long* __restrict__ sums,
+                                    unsigned* __restrict__ cnt) {
+  const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= n * dim) return;
+  const int64_t i = e / dim;
+  const int j = (int)(e - i * dim);
+  const int a = assign[i];
+  const long long f = __float2ll_rn(__fmul_rn(x[i * ld + j], kFix));  // exact scaling
+  atomicAdd(&sums[(int64_t)a * dim + j], (unsigned long long)f);
+  if (j == 0) atomicAdd(&cnt[a], 1u);
+}
+
+// One thread per centroid: member mean (previous centroid if empty), then
+// unit norm for spherical k-means; clears the sums for the next round.
+__global__ void kmeans_finish_kernel(float* __restrict__ c, int k, int dim,
+                                     unsigned long long* __restrict__ sums,
+                                     unsigned* __restrict__ cnt, int spherical) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= k) return;
+  float* cr = c + (int64_t)t * dim;
+  const unsigned m = cnt[t];
+  for (int j = 0; j < dim; ++j) {
+    unsigned long long* sp = &sums[(int64_t)t * dim + j];
+    if (m > 0) {
+      const double mean = __ddiv_rn(__ll2double_rn((long long)*sp), (double)m);
+      cr[j] = __double2float_rn(mean * (1.0 / 2147483648.0));
+    }
+    *sp = 0ull;
+  }
+  cnt[t] = 0u;
+  if (spherical) {
+    float s = 0.0f;
+    for (int j = 0; j < dim; ++j) s = madd(s, cr[j], cr[j]);
+    const float nrm = __fsqrt_rn(s);
+    for (int j = 0; j < dim; ++j) cr[j] = nrm > 0.0f ? __fdiv_rn(cr[j], nrm) : 0.0f;
+  }
+}
+
+// Unit norm of every centroid (spherical k-means starts from unit seeds).
+__global__ void normalize_centroids_kernel(float* __restrict__ c, int k, int dim) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= k) return;
+  float* cr = c + (int64_t)t * dim;
+  float s = 0.0f;
+  for (int j = 0; j < dim; ++j) s = madd(s, cr[j], cr[j]);
+  const float nrm = __fsqrt_rn(s);
+  for (int j = 0; j < dim; ++j) cr[j] = nrm > 0.0f ? __fdiv_rn(cr[j], nrm) : 0.0f;
+}
+
+// ---------------------------------------------------------------------------
+// inverted lists: stable counting sort of the cells
+// ---------------------------------------------------------------------------
+
+__global__ void cell_hist_kernel(const int32_t* __restrict__ cell, int64_t n, int nlist,
+                                 unsigned* __restrict__ hist) {
+  extern __shared__ unsigned sh[];
+  for (int c = threadIdx.x; c < nlist; c += blockDim.x) sh[c] = 0u;
+  __syncthreads();
+  const int64_t lo = (int64_t)blockIdx.x * kIdBlock;
+  const int64_t hi = min(n, lo + kIdBlock);
+  for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) atomicAdd(&sh[cell[i]], 1u);
+  __syncthreads();
+  unsigned* row = hist + (int64_t)blockIdx.x * nlist;
+  for (int c = threadIdx.x; c < nlist; c += blockDim.x) row[c] = sh[c];
+}
+
+// One thread per cell: total over the id blocks, and each block's base
+// (count of this cell's members in earlier blocks).
+__global__ void cell_totals_kernel(const unsigned* __restrict__ hist, int nb, int nlist,
+                                   unsigned* __restrict__ base, int64_t* __restrict__ totals) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= nlist) return;
+  unsigned run = 0;
+  for (int b = 0; b < nb; ++b) {
+    base[(int64_t)b * nlist + c] = run;
+    run += hist[(int64_t)b * nlist + c];
+  }
+  totals[c] = run;
+}
+
+// One block: offsets[c] = sum of totals[0..c), offsets[nlist] = n (in place
+// over totals[0..nlist] -> offsets), and the longest list.
+__global__ void __launch_bounds__(1024)
+cell_offsets_kernel(int64_t* __restrict__ off, int nlist, int64_t* __restrict__ max_list) {
+  __shared__ int64_t part[1024];
+  __shared__ int64_t mx[1024];
+  const int per = (nlist + blockDim.x - 1) / blockDim.x;
+  const int lo = threadIdx.x * per, hi = min(nlist, lo + per);
+  int64_t s = 0, m = 0;
+  for (int c = lo; c < hi; ++c) {
+    s += off[c];
+    m = max(m, off[c]);
+  }
+  part[threadIdx.x] = s;
+  mx[threadIdx.x] = m;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int64_t run = 0, mm = 0;
+    for (int t = 0; t < (int)blockDim.x; ++t) {
+      const int64_t v = part[t];
+      part[t] = run;
+      run += v;
+      mm = max(mm, mx[t]);
+    }
+    off[nlist] = run;
+    *max_list = mm;
+  }
+  __syncthreads();
+  int64_t run = part[threadIdx.x];
+  for (int c = lo; c < hi; ++c) {
+    const int64_t v = off[c];
+    off[c] = run;
+    run += v;
+  }
+}
+
+// One warp per id block: walks the ids in ascending order, 32 at a time, and
+// gives each the next slot of its cell (stable).
+__global__ void __launch_bounds__(32)
+cell_place_kernel(const int32_t* __restrict__ cell, int64_t n, int nlist,
+                  const int64_t* __restrict__ off, const unsigned* __restrict__ base,
+                  int32_t* __restrict__ pos, int32_t* __restrict__ ids) {
+  extern __shared__ int64_t next[];
+  const int lane = threadIdx.x;
+  for (int c = lane; c < nlist; c += 32) next[c] = off[c] + base[(int64_t)blockIdx.x * nlist + c];
+  __syncwarp();
+  const int64_t lo = (int64_t)blockIdx.x * kIdBlock;
+  const int64_t hi = min(n, lo + kIdBlock);
+  for (int64_t i0 = lo; i0 < hi; i0 += 32) {
+    const int64_t i = i0 + lane;
+    const bool live = i < hi;
+    const unsigned act = __ballot_sync(0xffffffffu, live);
+    if (live) {
+      const int c = cell[i];
+      const unsigned peers = __match_any_sync(act, c);
+      const int rank = __popc(peers & ((1u << lane) - 1u));
+      const int64_t p = next[c] + rank;
+      pos[i] = (int32_t)p;
+      ids[p] = (int32_t)i;
+      __syncwarp(act);
+      if (rank == 0) next[c] += __popc(peers);
+    }
+    __syncwarp();
+  }
+}
+
+// Flat lists: one warp per vector copies it to its slot.
+__global__ void scatter_vectors_kernel(const float* __restrict__ x, int64_t n, int v,
+                                       const int32_t* __restrict__ pos, float* __restrict__ out) {
+  const int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (i >= n) return;
+  const float* src = x + i * v;
+  float* dst = out + (int64_t)pos[i] * v;
+  for (int j = lane; j < v; j += 32) dst[j] = src[j];
+}
+
+// PQ codes: a block covers 32 vectors (lanes) x all sub-quantizers (warps
+// stride over them); the codebooks sit in shared memory.  Residual
+// r = x - c_cell, code_m = arg min_b ||r_m - B_m[b]||^2 (first minimum).
+__global__ void __launch_bounds__(256)
+pq_encode_kernel(const float* __restrict__ x, int64_t n, int v, const float* __restrict__ cent,
+                 const int32_t* __restrict__ cell, const float* __restrict__ cb, int pq_m,
+                 int dsub, const int32_t* __restrict__ pos, uint8_t* __restrict__ codes) {
+  extern __shared__ float scb[];  // [pq_m][256][dsub]
+  const int total = pq_m * 256 * dsub;
+  for (int e = threadIdx.x; e < total; e += blockDim.x) scb[e] = cb[e];
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t i = (int64_t)blockIdx.x * 32 + lane;
+  if (i >= n) return;
+  const float* xr = x + i * v;
+  const float* cr = cent + (int64_t)cell[i] * v;
+  uint8_t* out = codes + (int64_t)pos[i] * pq_m;
+  float r[16];
+  for (int m = warp; m < pq_m; m += blockDim.x >> 5) {
+    for (int j = 0; j < dsub; ++j) r[j] = __fsub_rn(xr[m * dsub + j], cr[m * dsub + j]);
+    const float* bm = scb + m * 256 * dsub;
+    float best = 0.0f;
+    int arg = 0;
+    for (int b = 0; b < 256; ++b) {
+      float s = 0.0f;
+      for (int j = 0; j < dsub; ++j) {
+        const float u = __fsub_rn(r[j], bm[b * dsub + j]);
+        s = madd(s, u, u);
+      }
+      if (b == 0 || s < best) {
+        best = s;
+        arg = b;
+      }
+    }
+    out[m] = (uint8_t)arg;
+  }
+}
+
+// Residuals r = x - c_cell (for training PQ codebooks).
+__global__ void residual_kernel(const float* __restrict__ x, int64_t n, int v,
+                                const float* __restrict__ cent, const int32_t* __restrict__ cell,
+                                float* __restrict__ out) {
+  const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= n * v) return;
+  const int64_t i = e / v;
+  const int j = (int)(e - i * v);
+  out[e] = __fsub_rn(x[e], cent[(int64_t)cell[i] * v + j]);
+}
+
+// ---------------------------------------------------------------------------
+// search: list scan
+// ---------------------------------------------------------------------------
+
+constexpr int kScanThreads = 256;
+constexpr int kFlatStride = 132;  // padded row stride (floats) of staged vectors, v <= 128
+
+// One block per (probe p, query qi).  Flat: each thread scores one staged
+// vector (<q, x> in index order).  PQ: the block builds the query's lookup
+// table LUT[m][b] = <q_m, B_m[b]> in shared memory; each thread reads one
+// code row and sums coarse + LUT[0][c_0] + ... + LUT[pq_m-1][c_{pq_m-1}].
+// Candidates go to the query's pool (warp-aggregated append).
+__global__ void __launch_bounds__(kScanThreads)
+ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries, int nprobe,
+                const float* __restrict__ probe_score, const int32_t* __restrict__ probe_cell,
+                uint64_t* __restrict__ pool, uint32_t* __restrict__ counts, int64_t pool_cap,
+                uint32_t* status) {
+  extern __shared__ __align__(16) float sm[];
+  const int p = blockIdx.x, qi = blockIdx.y;
+  const int v = ix.v;
+  float* sq = sm;                  // [v]
+  float* stage = sm + 128;         // flat: [kScanThreads][kFlatStride]; pq: LUT [pq_m][256]
+  const float* q = queries + (int64_t)qi * v;
+  for (int j = threadIdx.x; j < v; j += blockDim.x) sq[j] = q[j];
+  const int cell = probe_cell[(int64_t)qi * nprobe + p];
+  const float coarse = probe_score[(int64_t)qi * nprobe + p];
+  if (cell < 0 || cell >= ix.nlist) {
+    if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_INTERNAL);
+    return;
+  }
+  __syncthreads();
+  const int64_t lo = ix.offsets[cell], hi = ix.offsets[cell + 1];
+  uint64_t* dst = pool + (int64_t)qi * pool_cap;
+  if (ix.pq_m > 0) {
+    const int dsub = ix.dsub;
+    for (int e = threadIdx.x; e < ix.pq_m * 256; e += blockDim.x) {
+      const int m = e >> 8;
+      const float* bb = ix.codebooks + (int64_t)e * dsub;
+      float s = 0.0f;
+      for (int j = 0; j < dsub; ++j) s = madd(s, sq[m * dsub + j], bb[j]);
+      stage[e] = s;
+    }
+    __syncthreads();
+    for (int64_t s0 = lo; s0 < hi; s0 += blockDim.x) {
+      const int64_t slot = s0 + threadIdx.x;
+      const bool live = slot < hi;
+      float s = coarse;
+      if (live) {
+        const uint8_t* cr = ix.codes + slot * ix.pq_m;
+        for (int m = 0; m < ix.pq_m; ++m) s = __fadd_rn(s, stage[(m << 8) + cr[m]]);
+      }
+      const uint32_t at = warp_append(&counts[qi], live);
+      if (live) {
+        if ((int64_t)at < pool_cap) dst[at] = cand_key(s, (uint32_t)ix.ids[slot]);
+        else raise_status(status, SENSE_DEVST_INTERNAL);
+      }
+    }
+  } else {
+    for (int64_t s0 = lo; s0 < hi; s0 += blockDim.x) {
+      const int rows = (int)min((int64_t)blockDim.x, hi - s0);
+      __syncthreads();
+      // stage `rows` vectors (v floats each) with 16-byte loads
+      const int vq = v >> 2;
+      for (int e = threadIdx.x; e < rows * vq; e += blockDim.x) {
+        const int r = e / vq, g = e - r * vq;
+        *reinterpret_cast<float4*>(stage + r * kFlatStride + 4 * g) =
+            *reinterpret_cast<const float4*>(ix.vectors + (s0 + r) * v + 4 * g);
+      }
+      __syncthreads();
+      const bool live = threadIdx.x < rows;
+      float s = 0.0f;
+      if (live) {
+        const float* xr = stage + threadIdx.x * kFlatStride;
+        for (int g = 0; g < vq; ++g) {
+          const float4 xv = *reinterpret_cast<const float4*>(xr + 4 * g);
+          s = madd(s, sq[4 * g], xv.x);
+          s = madd(s, sq[4 * g + 1], xv.y);
+          s = madd(s, sq[4 * g + 2], xv.z);
+          s = madd(s, sq[4 * g + 3], xv.w);
+        }
+      }
+      const uint32_t at = warp_append(&counts[qi], live);
+      if (live) {
+        const int64_t slot = s0 + threadIdx.x;
+        if ((int64_t)at < pool_cap) dst[at] = cand_key(s, (uint32_t)ix.ids[slot]);
+        else raise_status(status, SENSE_DEVST_INTERNAL);
+      }
+    }
+  }
+}
+
+size_t scan_smem_bytes(const sense_ivf* ix) {
+  const size_t stage = ix->pq_m > 0 ? (size_t)ix->pq_m * 256 : (size_t)kScanThreads * kFlatStride;
+  return (128 + stage) * sizeof(float);
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct SearchPlan {
+  size_t off_coarse, off_pscore, off_pcell, off_counts, off_pool, total;
+  int64_t pool_cap;
+};
+
+SearchPlan search_plan(const sense_ivf* ix, int q, int nprobe) {
+  SearchPlan p{};
+  size_t o = 0;
+  p.off_coarse = o;
+  o = align256(o + (size_t)q * ix->nlist * 8);
+  p.off_pscore = o;
+  o = align256(o + (size_t)q * nprobe * 4);
+  p.off_pcell = o;
+  o = align256(o + (size_t)q * nprobe * 4);
+  p.off_counts = o;
+  o = align256(o + (size_t)q * 4);
+  p.pool_cap = std::max<int64_t>(1, (int64_t)nprobe * ix->max_list);
+  p.off_pool = o;
+  o = align256(o + (size_t)q * p.pool_cap * 8);
+  p.total = o;
+  return p;
+}
+
+int current_device() {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  return dev;
+}
+
+bool aligned(const void* ptr, size_t a) { return (reinterpret_cast<uintptr_t>(ptr) % a) == 0; }
+
+bool dim_ok(int dim) {
+  return dim == 4 || dim == 8 || dim == 16 || dim == 32 || dim == 64 || dim == 128;
+}
+
+void free_ivf(sense_ivf* ix) {
+  if (!ix) return;
+  cudaFree(ix->centroids);
+  cudaFree(ix->codebooks);
+  cudaFree(ix->offsets);
+  cudaFree(ix->ids);
+  cudaFree(ix->vectors);
+  cudaFree(ix->codes);
+  delete ix;
+}
+
+}  // namespace
+}  // namespace sense
+
+using namespace sense;
+
+extern "C" {
+
+sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float* basis, int32_t v,
+                           const float* mean, uint32_t flags, float* out, sense_stream_t stream) {
+  if (!x || !basis || !out) return fail(SENSE_ERR_INVALID_ARG, "x, basis and out must be non-NULL");
+  if (n < 1) return fail(SENSE_ERR_INVALID_ARG, "n=%lld must be >= 1", (long long)n);
+  if (d < 8 || d % 8) return fail(SENSE_ERR_INVALID_ARG, "d=%d must be a positive multiple of 8", d);
+  if (v < 1 || v > SENSE_MAX_PROJ_DIM)
+    return fail(SENSE_ERR_INVALID_ARG, "v=%d outside [1, %d]", v, SENSE_MAX_PROJ_DIM);
+  if (flags & ~SENSE_PROJECT_NORMALIZE) return fail(SENSE_ERR_INVALID_ARG, "unknown flags 0x%x", flags);
+  if (!aligned(x, 16) || !aligned(basis, 16) || (mean && !aligned(mean, 16)) || !aligned(out, 4))
+    return fail(SENSE_ERR_INVALID_ARG, "x, basis and mean must be 16-byte aligned");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  {
+    LaunchScope ls(K_PROJECT, s);
+    if (n * v <= 16384) {
+      const int64_t threads = n * v * 32;
+      project_rows_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(x, n, d, basis, v, mean,
+                                                                            out);
+    } else {
+      const dim3 grid((unsigned)((n + kPtRows - 1) / kPtRows), (unsigned)((v + kPtOuts - 1) / kPtOuts));
+      project_tile_kernel<<<grid, 512, 0, s>>>(x, n, d, basis, v, mean, out);
+    }
+    sense_status st = cuda_check(cudaGetLastError(), "launch project");
+    if (st != SENSE_OK) return st;
+  }
+  if (flags & SENSE_PROJECT_NORMALIZE) {
+    LaunchScope ls(K_PROJECT, s);
+    normalize_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(out, n, v);
+    return cuda_check(cudaGetLastError(), "launch normalize rows");
+  }
+  return SENSE_OK;
+}
+
+size_t sense_kmeans_workspace_bytes(int64_t n, int32_t dim, int32_t k) {
+  if (n < 1 || dim < 1 || k < 1) return 0;
+  return align256((size_t)n * 4) + align256((size_t)k * dim * 8) + align256((size_t)k * 4);
+}
+
+sense_status sense_kmeans(const float* x, int64_t n, int32_t dim, int32_t ld, int32_t k,
+                          int32_t iters, uint32_t flags, const float* init, float* centroids,
+                          int32_t* out_assign, void* workspace, size_t workspace_bytes,
+                          sense_stream_t stream) {
+  if (!x || !init || !centroids || !workspace)
+    return fail(SENSE_ERR_INVALID_ARG, "x, init, centroids and workspace must be non-NULL");
+  if (n < 1 || n > INT32_MAX) return fail(SENSE_ERR_INVALID_ARG, "n=%lld outside [1, 2^31)", (long long)n);
+  if (!dim_ok(dim)) return fail(SENSE_ERR_INVALID_ARG, "dim=%d not in {4, 8, 16, 32, 64, 128}", dim);
+  if (ld < dim) return fail(SENSE_ERR_INVALID_ARG, "ld=%d < dim=%d", ld, dim);
+  if (k < 1 || k > 65536) return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, 65536]", k);
+  if (iters < 0) return fail(SENSE_ERR_INVALID_ARG, "iters=%d must be >= 0", iters);
+  if (flags & ~SENSE_KMEANS_SPHERICAL) return fail(SENSE_ERR_INVALID_ARG, "unknown flags 0x%x", flags);
+  if (workspace_bytes < sense_kmeans_workspace_bytes(n, dim, k))
+    return fail(SENSE_ERR_INVALID_ARG, "workspace of %zu bytes < %zu", workspace_bytes,
+                sense_kmeans_workspace_bytes(n, dim, k));
+  if (!aligned(workspace, 256)) return fail(SENSE_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  int32_t* assign = reinterpret_cast<int32_t*>(ws);
+  auto* sums = reinterpret_cast<unsigned long long*>(ws + align256((size_t)n * 4));
+  auto* cnt = reinterpret_cast<unsigned*>(ws + align256((size_t)n * 4) + align256((size_t)k * dim * 8));
+  const bool sph = (flags & SENSE_KMEANS_SPHERICAL) != 0;
+  sense_status st = cuda_check(cudaMemcpyAsync(centroids, init, (size_t)k * dim * 4,
+                                               cudaMemcpyDeviceToDevice, s), "copy init");
+  if (st != SENSE_OK) return st;
+  st = cuda_check(cudaMemsetAsync(sums, 0, (size_t)k * dim * 8, s), "clear sums");
+  if (st != SENSE_OK) return st;
+  st = cuda_check(cudaMemsetAsync(cnt, 0, (size_t)k * 4, s), "clear counts");
+  if (st != SENSE_OK) return st;
+  LaunchScope ls(K_KMEANS, s);
+  if (sph) normalize_centroids_kernel<<<(k + 127) / 128, 128, 0, s>>>(centroids, k, dim);
+  for (int it = 0; it < iters; ++it) {
+    st = sph ? launch_assign_mode<ARGMAX_IP>(x, n, dim, ld, centroids, k, assign, nullptr, s)
+             : launch_assign_mode<ARGMIN_L2>(x, n, dim, ld, centroids, k, assign, nullptr, s);
+    if (st != SENSE_OK) return st;
+    const int64_t e = n * dim;
+    kmeans_accum_kernel<<<(unsigned)((e + 255) / 256), 256, 0, s>>>(x, n, dim, ld, assign, sums, cnt);
+    kmeans_finish_kernel<<<(k + 127) / 128, 128, 0, s>>>(centroids, k, dim, sums, cnt, sph ? 1 : 0);
+  }
+  if (out_assign && iters > 0) {
+    st = cuda_check(cudaMemcpyAsync(out_assign, assign, (size_t)n * 4, cudaMemcpyDeviceToDevice, s),
+                    "copy assignment");
+    if (st != SENSE_OK) return st;
+  }
+  return cuda_check(cudaGetLastError(), "launch kmeans");
+}
+
+sense_status sense_ivf_residuals(const float* vecs, int64_t n, int32_t v, const float* centroids,
+                                 int32_t nlist, int32_t* out_cell, float* out_residuals,
+                                 sense_stream_t stream) {
+  if (!vecs || !centroids || !out_cell || !out_residuals)
+    return fail(SENSE_ERR_INVALID_ARG, "arrays must be non-NULL");
+  if (n < 1 || n > INT32_MAX) return fail(SENSE_ERR_INVALID_ARG, "n=%lld outside [1, 2^31)", (long long)n);
+  if (!dim_ok(v) || v < 16) return fail(SENSE_ERR_INVALID_ARG, "v=%d not in {16, 32, 64, 128}", v);
+  if (nlist < 1 || nlist > kMaxList) return fail(SENSE_ERR_INVALID_ARG, "nlist=%d outside [1, %d]", nlist, kMaxList);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  LaunchScope ls(K_IVF_BUILD, s);
+  sense_status st = launch_assign_mode<ARGMAX_IP>(vecs, n, v, v, centroids, nlist, out_cell, nullptr, s);
+  if (st != SENSE_OK) return st;
+  residual_kernel<<<(unsigned)((n * v + 255) / 256), 256, 0, s>>>(vecs, n, v, centroids, out_cell,
+                                                                  out_residuals);
+  return cuda_check(cudaGetLastError(), "launch residuals");
+}
+
+sense_status sense_ivf_build(const float* vecs, int64_t n, int32_t v, const float* centroids,
+                             int32_t nlist, const float* codebooks, int32_t pq_m,
+                             sense_stream_t stream, sense_ivf** out) {
+  if (!out) return fail(SENSE_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (!vecs || !centroids) return fail(SENSE_ERR_INVALID_ARG, "vecs and centroids must be non-NULL");
+  if (n < 1 || n > INT32_MAX) return fail(SENSE_ERR_INVALID_ARG, "n=%lld outside [1, 2^31)", (long long)n);
+  if (!dim_ok(v) || v < 16) return fail(SENSE_ERR_INVALID_ARG, "v=%d not in {16, 32, 64, 128}", v);
+  if (nlist < 1 || nlist > kMaxList) return fail(SENSE_ERR_INVALID_ARG, "nlist=%d outside [1, %d]", nlist, kMaxList);
+  if (codebooks) {
+    if (pq_m < 1 || v % pq_m || v / pq_m > 16)
+      return fail(SENSE_ERR_INVALID_ARG, "pq_m=%d must divide v=%d with v/pq_m <= 16", pq_m, v);
+  } else if (pq_m != 0) {
+    return fail(SENSE_ERR_INVALID_ARG, "pq_m=%d needs codebooks", pq_m);
+  }
+  if (!aligned(vecs, 16) || !aligned(centroids, 16)) return fail(SENSE_ERR_INVALID_ARG, "vecs and centroids must be 16-byte aligned");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  auto* ix = new sense_ivf{};
+  ix->n = n;
+  ix->v = v;
+  ix->nlist = nlist;
+  ix->pq_m = codebooks ? pq_m : 0;
+  ix->dsub = codebooks ? v / pq_m : 0;
+  ix->device = current_device();
+  const int nb = (int)((n + kIdBlock - 1) / kIdBlock);
+  int32_t* cell = nullptr;
+  int32_t* pos = nullptr;
+  unsigned* hist = nullptr;
+  unsigned* base = nullptr;
+  int64_t* dmax = nullptr;
+  auto cleanup = [&](sense_status st) {
+    cudaFree(cell);
+    cudaFree(pos);
+    cudaFree(hist);
+    cudaFree(base);
+    cudaFree(dmax);
+    if (st != SENSE_OK) free_ivf(ix);
+    return st;
+  };
+  auto alloc = [&](void** p, size_t bytes) {
+    return cudaMalloc(p, bytes) == cudaSuccess;
+  };
+  bool ok = alloc((void**)&ix->centroids, (size_t)nlist * v * 4) &&
+            alloc((void**)&ix->offsets, (size_t)(nlist + 1) * 8) &&
+            alloc((void**)&ix->ids, (size_t)n * 4) && alloc((void**)&cell, (size_t)n * 4) &&
+            alloc((void**)&pos, (size_t)n * 4) && alloc((void**)&hist, (size_t)nb * nlist * 4) &&
+            alloc((void**)&base, (size_t)nb * nlist * 4) && alloc((void**)&dmax, 8);
+  if (ok && codebooks)
+    ok = alloc((void**)&ix->codebooks, (size_t)pq_m * 256 * ix->dsub * 4) &&
+         alloc((void**)&ix->codes, (size_t)n * pq_m);
+  if (ok && !codebooks) ok = alloc((void**)&ix->vectors, (size_t)n * v * 4);
+  if (!ok) {
+    cudaGetLastError();
+    return cleanup(fail(SENSE_ERR_OOM, "index allocation failed"));
+  }
+  sense_status st = cuda_check(cudaMemcpyAsync(ix->centroids, centroids, (size_t)nlist * v * 4,
+                                               cudaMemcpyDeviceToDevice, s), "copy centroids");
+  if (st == SENSE_OK && codebooks)
+    st = cuda_check(cudaMemcpyAsync(ix->codebooks, codebooks, (size_t)pq_m * 256 * ix->dsub * 4,
+                                    cudaMemcpyDeviceToDevice, s), "copy codebooks");
+  if (st != SENSE_OK) return cleanup(st);
+  {
+    LaunchScope ls(K_IVF_BUILD, s);
+    st = launch_assign_mode<ARGMAX_IP>(vecs, n, v, v, ix->centroids, nlist, cell, nullptr, s);
+    if (st != SENSE_OK) return cleanup(st);
+    const size_t hsm = (size_t)nlist * 4;
+    if (hsm > 48 * 1024) {
+      st = cuda_check(cudaFuncSetAttribute(cell_hist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)hsm), "smem attribute");
+      if (st != SENSE_OK) return cleanup(st);
+    }
+    cell_hist_kernel<<<nb, 256, hsm, s>>>(cell, n, nlist, hist);
+    cell_totals_kernel<<<(nlist + 127) / 128, 128, 0, s>>>(hist, nb, nlist, base, ix->offsets);
+    cell_offsets_kernel<<<1, 1024, 0, s>>>(ix->offsets, nlist, dmax);
+    const size_t psm = (size_t)nlist * 8;
+    if (psm > 48 * 1024) {
+      st = cuda_check(cudaFuncSetAttribute(cell_place_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)psm), "smem attribute");
+      if (st != SENSE_OK) return cleanup(st);
+    }
+    cell_place_kernel<<<nb, 32, psm, s>>>(cell, n, nlist, ix->offsets, base, pos, ix->ids);
+    if (codebooks) {
+      const size_t csm = (size_t)pq_m * 256 * ix->dsub * 4;
+      if (csm > 48 * 1024) {
+        st = cuda_check(cudaFuncSetAttribute(pq_encode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)csm), "smem attribute");
+        if (st != SENSE_OK) return cleanup(st);
+      }
+      pq_encode_kernel<<<(unsigned)((n + 31) / 32), 256, csm, s>>>(vecs, n, v, ix->centroids, cell,
+                                                                  ix->codebooks, pq_m, ix->dsub, pos,
+                                                                  ix->codes);
+    } else {
+      scatter_vectors_kernel<<<(unsigned)((n * 32 + 255) / 256), 256, 0, s>>>(vecs, n, v, pos,
+                                                                            ix->vectors);
+    }
+    st = cuda_check(cudaGetLastError(), "launch ivf build");
+    if (st != SENSE_OK) return cleanup(st);
+  }
+  st = cuda_check(cudaMemcpyAsync(&ix->max_list, dmax, 8, cudaMemcpyDeviceToHost, s), "read max list");
+  if (st == SENSE_OK) st = cuda_check(cudaStreamSynchronize(s), "ivf build");
+  if (st != SENSE_OK) return cleanup(st);
+  *out = ix;
+  return cleanup(SENSE_OK);
+}
+
+sense_status sense_ivf_destroy(sense_ivf* ix) {
+  free_ivf(ix);
+  return SENSE_OK;
+}
+
+sense_status sense_ivf_arrays(const sense_ivf* ix, int64_t* out_info, const int64_t** out_offsets,
+                              const int32_t** out_ids, const void** out_payload) {
+  if (!ix) return fail(SENSE_ERR_INVALID_ARG, "ix is NULL");
+  if (out_info) {
+    out_info[0] = ix->n;
+    out_info[1] = ix->v;
+    out_info[2] = ix->nlist;
+    out_info[3] = ix->pq_m;
+    out_info[4] = ix->max_list;
+  }
+  if (out_offsets) *out_offsets = ix->offsets;
+  if (out_ids) *out_ids = ix->ids;
+  if (out_payload) *out_payload = ix->pq_m ? (const void*)ix->codes : (const void*)ix->vectors;
+  return SENSE_OK;
+}
+
+size_t sense_ivf_search_workspace_bytes(const sense_ivf* ix, int32_t q, int32_t k, int32_t nprobe) {
+  if (!ix || q < 1 || k < 1 || nprobe < 1) return 0;
+  return search_plan(ix, q, nprobe).total;
+}
+
+sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t q, int32_t k,
+                              int32_t nprobe, float* out_scores, int32_t* out_idx,
+                              int32_t* out_probes, void* workspace, size_t workspace_bytes,
+                              sense_stream_t stream) {
+  if (!ix) return fail(SENSE_ERR_INVALID_ARG, "ix is NULL");
+  if (!queries || !out_scores || !out_idx || !workspace)
+    return fail(SENSE_ERR_INVALID_ARG, "queries, outputs and workspace must be non-NULL");
+  if (q < 1 || q > 65535) return fail(SENSE_ERR_INVALID_ARG, "q=%d outside [1, 65535]", q);
+  if (k < 1 || k > SENSE_MAX_K) return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, %d]", k, SENSE_MAX_K);
+  if (nprobe < 1 || nprobe > ix->nlist || nprobe > SENSE_MAX_K)
+    return fail(SENSE_ERR_INVALID_ARG, "nprobe=%d outside [1, min(nlist=%d, %d)]", nprobe, ix->nlist,
+                SENSE_MAX_K);
+  if (!aligned(queries, 16)) return fail(SENSE_ERR_INVALID_ARG, "queries must be 16-byte aligned");
+  if (!aligned(workspace, 256)) return fail(SENSE_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  const SearchPlan p = search_plan(ix, q, nprobe);
+  if (workspace_bytes < p.total)
+    return fail(SENSE_ERR_INVALID_ARG, "workspace of %zu bytes < %zu", workspace_bytes, p.total);
+  if (current_device() != ix->device) return fail(SENSE_ERR_INVALID_ARG, "index lives on device %d", ix->device);
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  auto* coarse = reinterpret_cast<uint64_t*>(ws + p.off_coarse);
+  auto* pscore = reinterpret_cast<float*>(ws + p.off_pscore);
+  auto* pcell = out_probes ? out_probes : reinterpret_cast<int32_t*>(ws + p.off_pcell);
+  auto* counts = reinterpret_cast<uint32_t*>(ws + p.off_counts);
+  auto* pool = reinterpret_cast<uint64_t*>(ws + p.off_pool);
+  sense_status st = cuda_check(cudaMemsetAsync(counts, 0, (size_t)q * 4, s), "clear counts");
+  if (st != SENSE_OK) return st;
+  {
+    LaunchScope ls(K_IVF_COARSE, s);
+    // cells as rows, queries staged: pool row qi holds key(<q_qi, c>, c)
+    st = launch_assign_mode<ALL_IP>(ix->centroids, ix->nlist, ix->v, ix->v, queries, q, nullptr,
+                                    coarse, s);
+    if (st != SENSE_OK) return st;
+  }
+  st = launch_merge(coarse, nullptr, ix->nlist, q, nprobe, pscore, pcell, status, s);
+  if (st != SENSE_OK) return st;
+  {
+    const size_t smem = scan_smem_bytes(ix);
+    st = cuda_check(cudaFuncSetAttribute(ivf_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem), "smem attribute");
+    if (st != SENSE_OK) return st;
+    LaunchScope ls(K_IVF_SCAN, s);
+    ivf_scan_kernel<<<dim3(nprobe, q), kScanThreads, smem, s>>>(*ix, queries, nprobe, pscore, pcell,
+                                                                pool, counts, p.pool_cap, status);
+    st = cuda_check(cudaGetLastError(), "launch ivf scan");
+    if (st != SENSE_OK) return st;
+  }
+  return launch_merge_short(pool, counts, p.pool_cap, q, k, out_scores, out_idx, status, s);
+}
+
+}  // extern "C"

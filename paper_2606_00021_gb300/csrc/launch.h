@@ -109,6 +109,12 @@ sense_status launch_merge(const uint64_t* pool, const uint32_t* counts, int64_t 
                           int k, float* out_scores, int32_t* out_idx, uint32_t* status,
                           cudaStream_t s);
 
+// Same, but a query whose pool holds fewer than k keys is not an error: its
+// remaining output slots get score -inf and index -1.
+sense_status launch_merge_short(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap,
+                                int q, int k, float* out_scores, int32_t* out_idx,
+                                uint32_t* status, cudaStream_t s);
+
 sense_status launch_normalize(const float* src, int64_t n, int d, uint16_t* dst, cudaStream_t s);
 
 sense_status launch_gather(const int32_t* spans, int64_t n, int m, const int32_t* idx, int q,

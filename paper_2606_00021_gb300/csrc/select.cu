@@ -192,7 +192,7 @@ threshold_kernel(const uint64_t* __restrict__ lists, int64_t len, int k,
 __global__ void __launch_bounds__(kSelThreads, 1)
 merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
              int64_t pool_cap, int k, float* __restrict__ out_scores,
-             int32_t* __restrict__ out_idx, uint32_t* status) {
+             int32_t* __restrict__ out_idx, uint32_t* status, int pad_short) {
   extern __shared__ uint64_t s_keys[];
   __shared__ unsigned hist[256];
   __shared__ Digit dig;
@@ -209,7 +209,12 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
   }
   auto get = [&](int64_t i) { return staged ? s_keys[i] : src[i]; };
   uint64_t prefix, pmask;
-  const bool ok = radix_select(get, cnt, k, 0, hist, &dig, &prefix, &pmask);
+  bool ok = radix_select(get, cnt, k, 0, hist, &dig, &prefix, &pmask);
+  if (!ok && pad_short) {  // fewer than k candidates allowed: keep them all
+    prefix = 0ull;
+    pmask = 0ull;
+    ok = true;
+  }
   if (!ok) {  // fewer than k candidates: internal error, outputs marked
     if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_INTERNAL);
     for (int r = threadIdx.x; r < k; r += blockDim.x) {
@@ -231,8 +236,9 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
   __syncthreads();
   int kp = 1;
   while (kp < k) kp <<= 1;
+  const int got = min((int)n_sel, k);  // k, or the whole pool when it is short
   for (int i = threadIdx.x; i < kp; i += blockDim.x) {
-    if (i >= k) sel[i] = 0ull;
+    if (i >= got) sel[i] = 0ull;
   }
   __syncthreads();
   // Bitonic sort, descending.
@@ -254,8 +260,9 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
   }
   for (int r = threadIdx.x; r < k; r += blockDim.x) {
     const uint64_t c = sel[r];
-    out_scores[(int64_t)q * k + r] = code_score((uint32_t)(c >> 32));
-    out_idx[(int64_t)q * k + r] = (int32_t)cand_index(c);
+    const bool real = r < got;  // slots past a short pool: -inf, -1
+    out_scores[(int64_t)q * k + r] = real ? code_score((uint32_t)(c >> 32)) : -__int_as_float(0x7f800000);
+    out_idx[(int64_t)q * k + r] = real ? (int32_t)cand_index(c) : -1;
   }
 }
 
@@ -409,7 +416,18 @@ sense_status launch_merge(const uint64_t* pool, const uint32_t* counts, int64_t 
   if (st != SENSE_OK) return st;
   LaunchScope ls(K_MERGE, s);
   merge_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(pool, counts, pool_cap, k,
-                                                                   out_scores, out_idx, status);
+                                                                   out_scores, out_idx, status, 0);
+  return cuda_check(cudaGetLastError(), "launch merge");
+}
+
+sense_status launch_merge_short(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap,
+                                int q, int k, float* out_scores, int32_t* out_idx,
+                                uint32_t* status, cudaStream_t s) {
+  sense_status st = set_smem(merge_kernel, kSmemKeys * sizeof(uint64_t));
+  if (st != SENSE_OK) return st;
+  LaunchScope ls(K_MERGE, s);
+  merge_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(pool, counts, pool_cap, k,
+                                                                   out_scores, out_idx, status, 1);
   return cuda_check(cudaGetLastError(), "launch merge");
 }
 

@@ -1,0 +1,220 @@
+"""GPU-vs-oracle parity of the approximate retrieval path (PCA projection,
+k-means, IVF-flat / IVF-PQ build and search), through the C ABI.
+
+Every step ends in an integer decision taken in fp32 in the same stated
+order on both sides, so every output is compared bit for bit: projected
+vectors, centroids, assignments, lists, codes, probes, scores and indices.
+Inputs come from seeded generators; expected values only from ``oracle``.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import ivf_oracle as I
+from tests.parity import bits, host
+
+pytestmark = pytest.mark.gpu
+cuda = pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+@pytest.fixture(scope="module")
+def S():
+    import paper_2606_00021_gb300 as S
+    S.lib()
+    return S
+
+
+def _unit(rng, n, d):
+    x = rng.standard_normal((n, d))
+    return (x / np.linalg.norm(x, axis=1, keepdims=True)).astype(np.float32)
+
+
+def _clustered(rng, n, v, nclust, spread=0.25):
+    c = _unit(rng, nclust, v)
+    x = c[rng.integers(0, nclust, n)] + spread / np.sqrt(v) * rng.standard_normal((n, v))
+    return (x / np.linalg.norm(x, axis=1, keepdims=True)).astype(np.float32)
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+# ---------------------------------------------------------------- projection
+
+@cuda
+@pytest.mark.parametrize("n,d,v,centre,norm", [
+    (1, 4096, 64, True, True), (5, 1000, 16, False, True), (300, 4096, 64, True, True),
+    (333, 1000, 48, True, False), (40, 512, 128, False, True), (2000, 256, 20, True, True),
+])
+def test_project_matches_oracle(S, n, d, v, centre, norm):
+    rng = np.random.default_rng(n + d + v)
+    x = synth.gaussian_rows_f32(n, d, seed=n).to(torch.bfloat16)
+    w = (rng.standard_normal((v, d)) / np.sqrt(d)).astype(np.float32)
+    mu = (0.1 * rng.standard_normal(d)).astype(np.float32) if centre else None
+    got = S.sense_project(x.cuda(), _dev(w), None if mu is None else _dev(mu), normalize=norm)
+    torch.cuda.synchronize()
+    want = I.project(bits(x), w, mu, normalize=norm)
+    np.testing.assert_array_equal(host(got), want)
+
+
+# ---------------------------------------------------------------- k-means
+
+@cuda
+@pytest.mark.parametrize("n,dim,ld,k,iters,sph", [
+    (2000, 64, 64, 16, 3, True), (3000, 16, 16, 256, 2, False), (1500, 4, 64, 256, 3, False),
+    (500, 32, 32, 7, 0, True), (4100, 128, 128, 40, 2, True),
+])
+def test_kmeans_matches_oracle(S, n, dim, ld, k, iters, sph):
+    rng = np.random.default_rng(n + k)
+    x = _clustered(rng, n, ld, 12) if ld >= 16 else rng.standard_normal((n, ld)).astype(np.float32)
+    init = x[rng.choice(n, size=k, replace=False), :dim].copy()
+    cent, assign = S.sense_kmeans(_dev(x)[:, :dim], _dev(init), iters, sph, want_assign=True)
+    torch.cuda.synchronize()
+    want_c, want_a = I.kmeans(x[:, :dim], init, iters, sph)
+    np.testing.assert_array_equal(host(cent), want_c)
+    if iters:
+        np.testing.assert_array_equal(host(assign), want_a)
+
+
+# ---------------------------------------------------------------- index build
+
+def _index_inputs(seed, n, v, nlist, pq_m):
+    rng = np.random.default_rng(seed)
+    x = _clustered(rng, n, v, max(4, nlist // 2))
+    cent = _unit(rng, nlist, v)
+    cb = None
+    if pq_m:
+        dsub = v // pq_m
+        cb = (0.3 / np.sqrt(v) * rng.standard_normal((pq_m, 256, dsub))).astype(np.float32)
+    return rng, x, cent, cb
+
+
+@cuda
+@pytest.mark.parametrize("n,v,nlist,pq_m", [
+    (5000, 64, 64, 0), (5000, 64, 64, 16), (9000, 16, 300, 4), (1, 32, 8, 8), (700, 128, 9, 8),
+])
+def test_ivf_build_matches_oracle(S, n, v, nlist, pq_m):
+    _, x, cent, cb = _index_inputs(n + nlist, n, v, nlist, pq_m)
+    ix = S.sense_ivf_build(_dev(x), _dev(cent), None if cb is None else _dev(cb))
+    arr = ix.arrays()
+    torch.cuda.synchronize()
+    want = I.ivf_build(x, cent, cb)
+    np.testing.assert_array_equal(host(arr["offsets"]), want["offsets"])
+    np.testing.assert_array_equal(host(arr["ids"]), want["ids"])
+    assert ix.max_list == int(np.diff(want["offsets"]).max())
+    if pq_m:
+        np.testing.assert_array_equal(host(arr["codes"]), want["codes"])
+    else:
+        np.testing.assert_array_equal(host(arr["vectors"]), want["vectors"])
+    cell, res = S.sense_ivf_residuals(_dev(x), _dev(cent))
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(host(cell), want["cell"])
+    np.testing.assert_array_equal(host(res), x - cent[want["cell"]])
+    ix.close()
+
+
+# ---------------------------------------------------------------- search
+
+@cuda
+@pytest.mark.parametrize("n,v,nlist,pq_m,q,k,nprobe", [
+    (6000, 64, 64, 0, 1, 32, 8), (6000, 64, 64, 16, 7, 100, 8), (6000, 64, 64, 16, 64, 16, 64),
+    (9000, 16, 300, 4, 5, 64, 1), (3000, 32, 40, 0, 33, 256, 3), (2000, 64, 16, 16, 3, 500, 2),
+])
+def test_ivf_search_matches_oracle(S, n, v, nlist, pq_m, q, k, nprobe):
+    rng, x, cent, cb = _index_inputs(7 * n + q, n, v, nlist, pq_m)
+    qs = _clustered(rng, q, v, 8)
+    ix = S.sense_ivf_build(_dev(x), _dev(cent), None if cb is None else _dev(cb))
+    sc, idx, probes = S.sense_ivf_search(ix, _dev(qs), k, nprobe, want_probes=True)
+    torch.cuda.synchronize()
+    assert S.sense_device_status(clear=True) == 0
+    index = I.ivf_build(x, cent, cb)
+    ws, wi, wp = I.ivf_search(index, cent, qs, nprobe, k, codebooks=cb)
+    np.testing.assert_array_equal(host(probes), wp)
+    np.testing.assert_array_equal(host(idx), wi)
+    np.testing.assert_array_equal(host(sc), ws)
+    ix.close()
+
+
+@cuda
+def test_ivf_golden_on_gpu(S):
+    """The hand-worked index, embedded in 16 dimensions: the extra
+    coordinates are zero, their codebooks code zero first, and the golden
+    codebooks fill codewords 0..3 of sub-quantizers 0 and 1 (the rest lie
+    far away)."""
+    g = json.load(open(os.path.join(GOLDEN, "ivf_small.json")))
+    v, pq_m = 16, 16
+    x = np.zeros((5, v), np.float32)
+    x[:, :2] = g["vectors"]
+    c = np.zeros((2, v), np.float32)
+    c[:, :2] = g["centroids"]
+    cb = np.full((pq_m, 256, 1), 1000.0, np.float32)
+    cb[2:, 0, 0] = 0.0
+    for m in range(2):
+        cb[m, :4, 0] = np.array(g["codebooks"][m])[:, 0]
+    ixf = S.sense_ivf_build(_dev(x), _dev(c))
+    ixp = S.sense_ivf_build(_dev(x), _dev(c), _dev(cb))
+    qv = np.zeros((1, v), np.float32)
+    qv[0, :2] = g["query"]
+    arr = ixp.arrays()
+    assert host(arr["ids"]).tolist() == g["ids"]
+    assert host(arr["codes"])[:, :2].tolist() == g["codes_list_order"]
+    s, i = S.sense_ivf_search(ixf, _dev(qv), 3, 2)
+    assert host(i)[0].tolist() == g["flat_nprobe2_k3"]["idx"]
+    assert host(s)[0].tolist() == g["flat_nprobe2_k3"]["scores"]
+    s, i = S.sense_ivf_search(ixf, _dev(qv), 4, 1)
+    assert host(i)[0].tolist() == g["flat_nprobe1_k4"]["idx"]
+    assert host(s)[0, 3] == -np.inf
+    s, i = S.sense_ivf_search(ixp, _dev(qv), 4, 2)
+    assert host(i)[0].tolist() == g["pq_nprobe2_k4"]["idx"]
+    assert host(s)[0].tolist() == g["pq_nprobe2_k4"]["scores"]
+    assert S.sense_device_status(clear=True) == 0
+
+
+@cuda
+def test_projected_pipeline_and_recall(S):
+    """Hidden states -> PCA-64 keys -> k-means cells -> IVF-PQ, all on the
+    GPU, equal to the oracle's chain (the k-means seeds are rows of the
+    oracle's own projections and residuals); recall@k of IVF-flat against the
+    exact search in the projected space is high when most cells are probed."""
+    rng = np.random.default_rng(99)
+    n, d, v, nlist, pq_m, q, k = 6000, 1024, 64, 32, 16, 6, 20
+    keys = synth.clustered_unit_keys(n, d, 24, seed=3)
+    qh, _ = synth.noisy_queries(keys, q, seed=4)
+    w = np.linalg.qr(rng.standard_normal((d, v)))[0].T.astype(np.float32).copy()
+    # oracle chain
+    kp_w = I.project(bits(keys), w)
+    qp_w = I.project(bits(qh), w)
+    init = kp_w[rng.choice(n, nlist, replace=False)].copy()
+    cent_w = I.kmeans(kp_w, init, 4, True)[0]
+    res_w = kp_w - cent_w[I.assign_ip(kp_w, cent_w)]
+    cb_init = np.stack([res_w[:256, m * 4:(m + 1) * 4] for m in range(pq_m)])
+    cb_w = np.stack([I.kmeans(res_w[:, m * 4:(m + 1) * 4], cb_init[m], 3, False)[0]
+                     for m in range(pq_m)])
+    ws, wi, _ = I.ivf_search(I.ivf_build(kp_w, cent_w, cb_w), cent_w, qp_w, 8, k, codebooks=cb_w)
+    # GPU chain from the same inputs
+    kp = S.sense_project(keys.cuda(), _dev(w))
+    qp = S.sense_project(qh.cuda(), _dev(w))
+    cent = S.sense_kmeans(kp, _dev(init), 4, True)
+    cell, res = S.sense_ivf_residuals(kp, cent)
+    # sub-quantizer m trains on columns 4m..4m+3 of the residuals (row stride v)
+    cbs = [S.sense_kmeans(res[:, 4 * m:4 * m + 4], _dev(cb_init[m]), 3, False)
+           for m in range(pq_m)]
+    ix = S.sense_ivf_build(kp, cent, torch.stack(cbs))
+    sc, idx = S.sense_ivf_search(ix, qp, k, 8)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(host(kp), kp_w)
+    np.testing.assert_array_equal(host(qp), qp_w)
+    np.testing.assert_array_equal(host(cent), cent_w)
+    np.testing.assert_array_equal(host(res), res_w)
+    np.testing.assert_array_equal(host(torch.stack(cbs)), cb_w)
+    np.testing.assert_array_equal(host(idx), wi)
+    np.testing.assert_array_equal(host(sc), ws)
+    flat = S.sense_ivf_build(kp, cent)
+    _, fi = S.sense_ivf_search(flat, qp, k, 24)
+    exact = np.argsort(-(qp_w.astype(np.float64) @ kp_w.astype(np.float64).T), axis=1)[:, :k]
+    assert I.recall_at_k(host(fi), exact) > 0.9

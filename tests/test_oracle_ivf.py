@@ -52,6 +52,23 @@ def test_dot_exact_on_dyadic_values_and_order_matters():
     assert I.dot_seq(x[:, ::-1].copy(), np.ones_like(x))[0] == 2.0 ** -23
 
 
+def test_dot_lanes_order_and_bound():
+    rng = np.random.default_rng(12)
+    a = rng.standard_normal((30, 1000)).astype(np.float32)
+    b = rng.standard_normal((30, 1000)).astype(np.float32)
+    ex = np.sum(a.astype(np.float64) * b, axis=1)
+    bound = 1000 * U * np.sum(np.abs(a.astype(np.float64) * b), axis=1)
+    assert np.all(np.abs(I.dot_lanes(a, b) - ex) <= bound)
+    # lane partials: column 128 joins lane 0 (with columns 0..3), column 4
+    # starts lane 1; the butterfly then adds lane 1 to lane 0 last
+    x = np.zeros((1, 256), np.float32)
+    x[0, 0], x[0, 128], x[0, 4] = 1.0, 2.0 ** -24, 2.0 ** -24
+    # lane 0: 1 + 2^-24 -> 1 (ties to even); lane 1: 2^-24; final 1 + 2^-24 -> 1
+    assert I.dot_lanes(x, np.ones_like(x))[0] == 1.0
+    x[0, 132] = 2.0 ** -24  # lane 1 now holds 2^-23: 1 + 2^-23 is exact
+    assert I.dot_lanes(x, np.ones_like(x))[0] == 1.0 + 2.0 ** -23
+
+
 # ---------------------------------------------------------------- projection
 
 def test_project_matches_fp64_and_is_unit():
