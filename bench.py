@@ -160,15 +160,77 @@ class Pipeline:
         self.drafts = torch.empty(q, k, m, dtype=torch.int32, device=dev)
         self.tree = {}
         self.gate = {}
+        self.ann = None
         self.gws = S.alloc_workspace(S.sense_soft_gate_workspace_bytes(q, self.cap, GATE["topk"]), dev)
+
+    def use_ann(self, ann, dev):
+        """Retrieve through the projected IVF index instead of the exact scan."""
+        q, k = self.cfg["q"], self.cfg["k"]
+        self.ann = ann
+        self.qproj = torch.empty(q, ann["index"].v, dtype=torch.float32, device=dev)
+        self.ws = self.S.alloc_workspace(
+            self.S.sense_ivf_search_workspace_bytes(ann["index"], q, k, ann["nprobe"]), dev)
+
+    def retrieve(self, query):
+        S, cfg = self.S, self.cfg
+        if self.ann is None:
+            S.sense_retrieve_topk(self.ds, query, cfg["k"], self.scores, self.idx, self.ws)
+        else:
+            a = self.ann
+            S.sense_project(query, a["basis"], a["mean"], out=self.qproj)
+            S.sense_ivf_search(a["index"], self.qproj, cfg["k"], a["nprobe"], self.scores,
+                               self.idx, workspace=self.ws)
 
     def step(self, query, gate_in):
         S, cfg = self.S, self.cfg
-        S.sense_retrieve_topk(self.ds, query, cfg["k"], self.scores, self.idx, self.ws)
+        self.retrieve(query)
         S.sense_gather_drafts(self.ds, self.idx, out=self.drafts)
         S.sense_build_tree(self.drafts, node_cap=cfg["cap"], outs=self.tree)
         root, nodes, hr, hn = gate_in
         S.sense_soft_gate(self.tree, root, nodes, hr, hn, workspace=self.gws, outs=self.gate, **GATE)
+
+
+def build_ann(S, keys, kind, nlist, nprobe, pq_m, v, dev, seed=0):
+    """Index construction for the approximate path (outside the timed region):
+    the PCA basis is fitted offline on a 65,536-key sample (eigenvectors of
+    its covariance, as the paper's setup fits PCA with a library); keys are
+    projected and normalised, the coarse quantizer is trained by spherical
+    k-means (10 rounds on 64 x nlist keys), PQ codebooks by k-means on the
+    residual sub-vectors (10 rounds), and the index is built - all but the
+    PCA fit in the library's kernels."""
+    n, d = keys.shape
+    g = torch.Generator(device=dev).manual_seed(seed + 7)
+    sample = keys[torch.randint(0, n, (min(n, 65536),), generator=g, device=dev)].float()
+    mean = sample.mean(0)
+    xc = sample - mean
+    evals, evecs = torch.linalg.eigh((xc.T @ xc / xc.shape[0]).double())
+    basis = evecs[:, -v:].flip(1).T.float().contiguous()
+    mean = mean.contiguous()
+    del sample, xc, evecs
+    t0 = time.perf_counter()
+    kp = torch.empty(n, v, dtype=torch.float32, device=dev)
+    for lo in range(0, n, 1 << 20):
+        hi = min(n, lo + (1 << 20))
+        S.sense_project(keys[lo:hi], basis, mean, out=kp[lo:hi])
+    train = kp[torch.randperm(n, generator=g, device=dev)[:min(n, 64 * nlist)]].contiguous()
+    cent = S.sense_kmeans(train, train[:nlist].clone(), 10, True)
+    cbs = None
+    if kind == "ivfpq":
+        _, res = S.sense_ivf_residuals(train, cent)
+        dsub = v // pq_m
+        cbs = torch.stack([S.sense_kmeans(res[:, m * dsub:(m + 1) * dsub],
+                                          res[:256, m * dsub:(m + 1) * dsub].contiguous(), 10,
+                                          False) for m in range(pq_m)])
+        del res
+    ix = S.sense_ivf_build(kp, cent, cbs)
+    torch.cuda.synchronize()
+    build_s = time.perf_counter() - t0
+    sizes = (ix.arrays()["offsets"][1:] - ix.arrays()["offsets"][:-1]).float()
+    del train
+    return {"index": ix, "basis": basis, "mean": mean, "nprobe": nprobe, "kind": kind,
+            "keys_proj": kp,
+            "nlist": nlist, "pq_m": pq_m if kind == "ivfpq" else 0, "v": v,
+            "build_s": build_s, "mean_list": float(sizes.mean()), "max_list": ix.max_list}
 
 
 def cpu_baseline(cfg, keys, spans, queries, gate_sets, budget_s=25.0):
@@ -270,6 +332,12 @@ def main():
                     help="override the store size (small cases for profiler captures)")
     ap.add_argument("--queries", type=int, default=0,
                     help="override the queries per step (small cases for profiler captures)")
+    ap.add_argument("--retrieval", default="exact", choices=["exact", "ivfpq", "ivfflat"],
+                    help="exact scan of the full keys, or the PCA + IVF index of App. E")
+    ap.add_argument("--nlist", type=int, default=4096)
+    ap.add_argument("--nprobe", type=int, default=32)
+    ap.add_argument("--pq-m", type=int, default=16)
+    ap.add_argument("--proj-dim", type=int, default=64)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     cfg = dict(WORKLOADS[args.workload])
@@ -306,6 +374,11 @@ def main():
     ds = S.sense_datastore_build(keys, spans)
     pipe = Pipeline(S, ds, cfg, dev)
     nq = queries.shape[0]
+    ann = None
+    if args.retrieval != "exact":
+        ann = build_ann(S, keys, args.retrieval, args.nlist, args.nprobe, args.pq_m,
+                        args.proj_dim, dev, seed=rank)
+        pipe.use_ann(ann, dev)
 
     for it in range(args.warmup):
         pipe.step(queries[it % nq], gate_sets[it % n_sets])
@@ -339,13 +412,59 @@ def main():
 
     q, n, d = cfg["q"], cfg["n"], cfg["d"]
     value = job_throughput(q * args.steps, world, ms / 1e3)
-    # roofline of the dominant kernel (the key scan)
-    scan_name = "scan_gemv" if q <= 8 else "scan_tc"
-    scan_ms, scan_launches = prof.get(scan_name, (0.0, 0))
-    scan_bytes_per_step = n * d * 2 + q * d * 2
-    achieved = scan_bytes_per_step * args.steps / (scan_ms / 1e3) / 1e9 if scan_ms > 0 else 0.0
     peak, peak_kind = peaks()
-    step_bytes = scan_bytes_per_step  # gate/tree bytes are <0.1% of the scan here
+    retrieval = {"kind": "exact"}
+    if ann is None:
+        # roofline of the dominant kernel (the key scan)
+        scan_name = "scan_gemv" if q <= 8 else "scan_tc"
+        scan_bytes_per_step = n * d * 2 + q * d * 2
+        step_bytes = scan_bytes_per_step  # gate/tree bytes are <0.1% of the scan here
+        traffic = NCU_TRAFFIC.get((scan_name, args.workload))
+    else:
+        # entries scanned per query (probed list sizes, over the distinct batches)
+        off = ann["index"].arrays()["offsets"]
+        sizes = off[1:] - off[:-1]
+        scanned = []
+        for b in range(min(nq, 64)):
+            pipe.S.sense_project(queries[b], ann["basis"], ann["mean"], out=pipe.qproj)
+            _, _, pr = S.sense_ivf_search(ann["index"], pipe.qproj, cfg["k"], ann["nprobe"],
+                                          want_probes=True)
+            scanned.append(sizes[pr.long()].sum(dim=1).float().mean().item())
+        per_q = float(np.mean(scanned))
+        v_, nl, pq_m = ann["v"], ann["nlist"], ann["pq_m"]
+        entry = (pq_m if pq_m else 4 * v_) + 4 + 8  # payload + key index + pool write
+        kb = {"project": v_ * d * 4 + q * d * 2 + q * v_ * 4,
+              "ivf_coarse": nl * v_ * 4 + q * nl * 8,
+              "ivf_scan": q * per_q * entry}
+        scan_name = max(kb, key=lambda name: prof.get(name, (0.0, 0))[0])
+        scan_bytes_per_step = kb[scan_name]
+        step_bytes = sum(kb.values())
+        traffic = None
+        # recall@k of the approximate top-k against (a) the exact top-k of the
+        # full keys and (b) the exact top-k of the projected keys (a one-cell
+        # flat index scans every projected key: the index's own loss)
+        ex_ws = S.alloc_workspace(S.sense_retrieve_workspace_bytes(ds, q, cfg["k"]), dev)
+        one = S.sense_ivf_build(ann["keys_proj"], ann["keys_proj"][:1].clone())
+        hits, hits_p = [], []
+        for b in range(min(nq, 64)):
+            _, ex_i = S.sense_retrieve_topk(ds, queries[b], cfg["k"], workspace=ex_ws)
+            pipe.retrieve(queries[b])
+            _, px_i = S.sense_ivf_search(one, pipe.qproj, cfg["k"], 1)
+            for a_row, e_row, p_row in zip(pipe.idx.cpu().tolist(), ex_i.cpu().tolist(),
+                                           px_i.cpu().tolist()):
+                hits.append(len(set(a_row) & set(e_row)) / len(e_row))
+                hits_p.append(len(set(a_row) & set(p_row)) / len(p_row))
+        del ex_ws, one
+        ann.pop("keys_proj")
+        retrieval = {"kind": ann["kind"], "proj_dim": v_, "nlist": nl, "nprobe": ann["nprobe"],
+                     "pq_m": pq_m, "build_s": round(ann["build_s"], 3),
+                     "mean_list": ann["mean_list"], "max_list": ann["max_list"],
+                     "entries_scanned_per_query": per_q,
+                     "recall_at_k_vs_exact": float(np.mean(hits)),
+                     "recall_at_k_vs_exact_projected": float(np.mean(hits_p)),
+                     "recall_queries": len(hits)}
+    scan_ms, scan_launches = prof.get(scan_name, (0.0, 0))
+    achieved = scan_bytes_per_step * args.steps / (scan_ms / 1e3) / 1e9 if scan_ms > 0 else 0.0
 
     # draft tree size (nodes per query) over a few steps, for draft tokens/s
     # and the loose trie's compression of the k*m candidate tokens (Sec. 4.3
@@ -419,7 +538,11 @@ def main():
 
     base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        base = cpu_baseline(cfg, keys, spans, queries, gate_sets)
+        if ann is None:
+            base = cpu_baseline(cfg, keys, spans, queries, gate_sets)
+        else:
+            base = {"value": None, "skipped": "the oracle's index build over the full store "
+                    "(fp32 loops in numpy) does not fit a bounded CPU sample"}
 
     if rank == 0:
         line = {
@@ -428,12 +551,13 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded clustered unit-norm keys, Zipf spans, N(0,9) logits)",
-            "config": {"workload": args.workload,
+            "config": {"workload": args.workload, "retrieval": args.retrieval,
                        **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab", "cap", "clusters")},
                        "key_bytes": n * d * 2,
                        "l2": f"inputs larger than L2: the {n * d * 2 / 1e9:.1f} GB store is "
                              "streamed every step",
                        "parallelism": f"replicas x{world}"},
+            "retrieval": retrieval,
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,
             "draft_tokens_per_s": value * mean_nodes,
             "mean_tree_nodes": mean_nodes,
@@ -441,7 +565,7 @@ def main():
             "roofline": {"bound": "hbm", "kernel": scan_name, "achieved": achieved,
                          "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                          "peak_kind": peak_kind,
-                         "traffic": NCU_TRAFFIC.get((scan_name, args.workload)),
+                         "traffic": traffic,
                          "launches": scan_launches, "kernel_ms": scan_ms},
             "kernel_ms": {k: round(v[0], 4) for k, v in prof.items() if v[1]},
             "gpu_launches": launches,

@@ -101,13 +101,27 @@ project_rows_kernel(const uint16_t* __restrict__ x, int64_t n, int d,
   const uint16_t* xr = x + row * d;
   const float* wr = w + (int64_t)o * d;
   float acc = 0.0f;
-  for (int j = 4 * lane; j < d; j += 128) {
-    const float4 xv = load_x4(xr, mu, j);
-    const float4 wv = *reinterpret_cast<const float4*>(wr + j);
-    acc = madd(acc, xv.x, wv.x);
-    acc = madd(acc, xv.y, wv.y);
-    acc = madd(acc, xv.z, wv.z);
-    acc = madd(acc, xv.w, wv.w);
+  // 8 column groups in flight per lane, consumed in ascending order
+  constexpr int U = 8;
+  for (int j0 = 4 * lane; j0 < d; j0 += 128 * U) {
+    float4 xv[U], wv[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int j = j0 + 128 * u;
+      if (j < d) {
+        xv[u] = load_x4(xr, mu, j);
+        wv[u] = *reinterpret_cast<const float4*>(wr + j);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (j0 + 128 * u < d) {
+        acc = madd(acc, xv[u].x, wv[u].x);
+        acc = madd(acc, xv[u].y, wv[u].y);
+        acc = madd(acc, xv[u].z, wv[u].z);
+        acc = madd(acc, xv[u].w, wv[u].w);
+      }
+    }
   }
   acc = butterfly(acc);
   if (lane == 0) out[row * v + o] = acc;
@@ -208,7 +222,7 @@ __global__ void normalize_rows_kernel(float* __restrict__ y, int64_t n, int v) {
 //  ARGMAX_IP: out_assign[i] = arg max_c <x_i, c> (first maximum)
 //  ARGMIN_L2: out_assign[i] = arg min_c ||x_i - c||^2 (first minimum)
 //  ALL_IP:    x = cells, c = queries: pool[c * n + i] = key(<x_i, c>, i)
-template <int D, int MODE>
+template <int D, int MODE, bool VEC>
 __global__ void __launch_bounds__(128)
 assign_kernel(const float* __restrict__ x, int64_t n, int ld, const float* __restrict__ c,
               int k, int32_t* __restrict__ out_assign, uint64_t* __restrict__ pool) {
@@ -217,8 +231,20 @@ assign_kernel(const float* __restrict__ x, int64_t n, int ld, const float* __res
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const bool live = i < n;
   float xr[D];
+  if (VEC) {  // 16-byte row loads (x 16-byte aligned, ld % 4 == 0)
 #pragma unroll
-  for (int j = 0; j < D; ++j) xr[j] = live ? x[i * ld + j] : 0.0f;
+    for (int j = 0; j < D; j += 4) {
+      float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (live) t = *reinterpret_cast<const float4*>(x + i * ld + j);
+      xr[j] = t.x;
+      xr[j + 1] = t.y;
+      xr[j + 2] = t.z;
+      xr[j + 3] = t.w;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < D; ++j) xr[j] = live ? x[i * ld + j] : 0.0f;
+  }
   float best = (MODE == ARGMIN_L2) ? __int_as_float(0x7f800000) : -__int_as_float(0x7f800000);
   int arg = 0;
   for (int t0 = 0; t0 < k; t0 += kTile) {
@@ -259,9 +285,13 @@ template <int MODE>
 sense_status launch_assign_mode(const float* x, int64_t n, int dim, int ld, const float* c, int k,
                                 int32_t* out_assign, uint64_t* pool, cudaStream_t s) {
   const dim3 grid((unsigned)((n + 127) / 128));
+  const bool vec = (reinterpret_cast<uintptr_t>(x) % 16 == 0) && (ld % 4 == 0);
 #define SENSE_ASSIGN_CASE(DD)                                                               \
   case DD:                                                                                  \
-    assign_kernel<DD, MODE><<<grid, 128, 0, s>>>(x, n, ld, c, k, out_assign, pool);         \
+    if (vec)                                                                                \
+      assign_kernel<DD, MODE, true><<<grid, 128, 0, s>>>(x, n, ld, c, k, out_assign, pool); \
+    else                                                                                    \
+      assign_kernel<DD, MODE, false><<<grid, 128, 0, s>>>(x, n, ld, c, k, out_assign, pool); \
     break;
   switch (dim) {
     SENSE_ASSIGN_CASE(4)
