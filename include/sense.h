@@ -39,6 +39,7 @@ extern "C" {
 typedef struct CUstream_st* sense_stream_t;
 typedef struct sense_datastore sense_datastore;
 typedef struct sense_ivf sense_ivf;
+typedef struct sense_ctx sense_ctx;
 
 typedef enum sense_status {
   SENSE_OK = 0,
@@ -306,6 +307,79 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
  */
 sense_status sense_gather_drafts(const sense_datastore* ds, const int32_t* idx, int32_t q,
                                  int32_t k, const int32_t* anchor, int32_t n_keep, uint32_t flags,
+                                 int32_t* out_spans, sense_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* Dynamic context buffer and hybrid candidates                             */
+/* ---------------------------------------------------------------------- */
+/*
+ * Sec. 3.2.1 Eq. 6: C_db = C_s u C_d, where the dynamic buffer C_d is filled
+ * from the generation itself.  Alg. 1 appends (hidden state, token it
+ * predicted) pairs with R.Update after prefill and after every accepted
+ * step; Alg. 2 searches C_d with DynSearch, adds a boost delta to its scores
+ * (s = [s_s; s_d + delta]) and reranks the union with Eq. 8.
+ * Readings (the paper does not define DynSearch or a buffer size): an entry
+ * is a position p with key L2Norm(h_p) stored as bf16 and span y_{p+1} ..
+ * y_{p+M} (the tokens predicted by h_p .. h_{p+M-1}); it is searchable once
+ * those M tokens have been appended; the buffer keeps the `capacity` most
+ * recent positions as a ring; DynSearch is the exact inner-product top-k
+ * (ties to the older position).
+ */
+
+/* Creates an empty buffer (allocates capacity * (2 d + 4) bytes on the
+ * current device).  Limits: 1 <= m <= SENSE_MAX_M, m <= capacity <= 2^24,
+ * d % 8 == 0. */
+sense_status sense_ctx_create(int32_t capacity, int32_t d, int32_t m, sense_ctx** out);
+sense_status sense_ctx_destroy(sense_ctx* ctx);
+/* Forgets every entry (no device work). */
+sense_status sense_ctx_reset(sense_ctx* ctx);
+/* Positions appended since creation or the last reset (-1 for NULL). */
+int64_t sense_ctx_count(const sense_ctx* ctx);
+
+/*
+ * R.Update: appends t positions.  hidden [t, d] bf16 (16-byte aligned):
+ * the hidden state at each position; tokens [t] int32: the token that state
+ * predicted (Alg. 1 passes H_align[i*, 0:L*+1] with the accepted tokens a).
+ * When t > capacity only the last `capacity` rows are kept.  Asynchronous
+ * on `stream`; later searches on the same stream see the new entries.
+ */
+sense_status sense_ctx_append(sense_ctx* ctx, const uint16_t* hidden, const int32_t* tokens,
+                              int32_t t, sense_stream_t stream);
+
+/*
+ * DynSearch: per query (queries [q, d] bf16, 16-byte aligned), the k
+ * searchable entries with the largest <q, key> (fp32 accumulation), order
+ * (score desc, position asc).  out_scores [q, k] f32 = score + delta;
+ * out_pos [q, k] int32 positions; out_spans [q, k, m] int32.  Slots past the
+ * number of searchable entries get -inf, -1 and a span of -1.  workspace:
+ * sense_ctx_search_workspace_bytes(ctx, q, k) bytes, 256-byte aligned.
+ * Limits: 1 <= q <= 65535, 1 <= k <= SENSE_MAX_K, delta finite.
+ */
+size_t sense_ctx_search_workspace_bytes(const sense_ctx* ctx, int32_t q, int32_t k);
+sense_status sense_ctx_search(const sense_ctx* ctx, const uint16_t* queries, int32_t q, int32_t k,
+                              float delta, float* out_scores, int32_t* out_pos,
+                              int32_t* out_spans, void* workspace, size_t workspace_bytes,
+                              sense_stream_t stream);
+
+/*
+ * Hybrid candidate drafts (Alg. 2, D_all = D_s u D_d and Eq. 8): per query,
+ * the static results (static_scores [q, ks] f32 and static_idx [q, ks] key
+ * indices of `ds`, e.g. from sense_retrieve_topk) and the dynamic results
+ * (dyn_scores [q, kd] f32 already boosted, -inf = empty slot, dyn_spans
+ * [q, kd, m] from sense_ctx_search) are ordered by score (desc; ties keep
+ * static before dynamic and rank order within each).  With an anchor x~ per
+ * query (anchor [q] or NULL) the candidates starting with x~ move first
+ * (stable), the first n_keep rows are kept, and SENSE_GATHER_FORCE_ANCHOR
+ * sets the first token of the first and of the last kept row to x~.  Rows
+ * past the number of live candidates are -1.  out_spans [q, n_keep, m].
+ * Limits: 1 <= ks + kd <= 2048, 1 <= n_keep <= ks + kd, m = the datastore's
+ * span length.  A static index outside [0, n) sets SENSE_DEVST_BAD_INDEX and
+ * that candidate is dropped.
+ */
+sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_scores,
+                                 const int32_t* static_idx, int32_t ks, const float* dyn_scores,
+                                 const int32_t* dyn_spans, int32_t kd, int32_t q,
+                                 const int32_t* anchor, int32_t n_keep, uint32_t flags,
                                  int32_t* out_spans, sense_stream_t stream);
 
 /* ---------------------------------------------------------------------- */

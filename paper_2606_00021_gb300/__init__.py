@@ -397,6 +397,94 @@ def sense_ivf_search(ix: IvfIndex, queries: torch.Tensor, k: int, nprobe: int,
     return (out_scores, out_idx, probes) if want_probes else (out_scores, out_idx)
 
 
+# ---------------------------------------------------------------- dynamic context buffer
+
+@dataclass
+class ContextBuffer:
+    """Handle of a dynamic context buffer C_d (library-owned device ring)."""
+    handle: int
+    capacity: int
+    d: int
+    m: int
+
+    def close(self):
+        if self.handle:
+            lib().sense_ctx_destroy(C.c_void_p(self.handle))
+            self.handle = 0
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @property
+    def count(self) -> int:
+        return int(lib().sense_ctx_count(C.c_void_p(self.handle)))
+
+    def reset(self):
+        _check(lib().sense_ctx_reset(C.c_void_p(self.handle)))
+
+
+def sense_ctx_create(capacity: int, d: int, m: int) -> ContextBuffer:
+    out = C.c_void_p(0)
+    _check(lib().sense_ctx_create(capacity, d, m, C.byref(out)))
+    return ContextBuffer(out.value, capacity, d, m)
+
+
+def sense_ctx_append(ctx: ContextBuffer, hidden: torch.Tensor, tokens: torch.Tensor, stream=None):
+    """R.Update: hidden [t, d] bf16 states and the tokens [t] int32 they predicted."""
+    _need(hidden, "hidden", torch.bfloat16, 2)
+    _need(tokens, "tokens", torch.int32, 1)
+    if hidden.shape[0] != tokens.shape[0] or hidden.shape[1] != ctx.d:
+        raise ValueError("hidden must be [t, d] and tokens [t]")
+    _check(lib().sense_ctx_append(C.c_void_p(ctx.handle), hidden.data_ptr(), tokens.data_ptr(),
+                                  hidden.shape[0], C.c_void_p(_stream(stream))))
+
+
+def sense_ctx_search(ctx: ContextBuffer, queries: torch.Tensor, k: int, delta: float = 0.0,
+                     outs: dict | None = None, workspace=None, stream=None) -> dict:
+    """DynSearch: dict of scores [q, k] (boosted), pos [q, k], spans [q, k, m]."""
+    _need(queries, "queries", torch.bfloat16, 2)
+    q = queries.shape[0]
+    dev = queries.device
+    o = outs if outs is not None else {}
+    o.setdefault("scores", torch.empty(q, k, dtype=torch.float32, device=dev))
+    o.setdefault("pos", _i32((q, k), dev))
+    o.setdefault("spans", _i32((q, k, ctx.m), dev))
+    if workspace is None:
+        workspace = alloc_workspace(lib().sense_ctx_search_workspace_bytes(
+            C.c_void_p(ctx.handle), q, k), dev)
+    _check(lib().sense_ctx_search(C.c_void_p(ctx.handle), queries.data_ptr(), q, k,
+                                  C.c_float(delta), o["scores"].data_ptr(), o["pos"].data_ptr(),
+                                  o["spans"].data_ptr(), workspace.data_ptr(), workspace.numel(),
+                                  C.c_void_p(_stream(stream))))
+    return o
+
+
+def sense_hybrid_drafts(ds: Datastore, static_scores: torch.Tensor, static_idx: torch.Tensor,
+                        dyn: dict | None, anchor: torch.Tensor | None = None,
+                        n_keep: int | None = None, force_anchor: bool = False, out=None,
+                        stream=None) -> torch.Tensor:
+    """Candidate drafts [q, n_keep, m] from static results and DynSearch results."""
+    _need(static_scores, "static_scores", torch.float32, 2)
+    _need(static_idx, "static_idx", torch.int32, 2)
+    q, ks = static_idx.shape
+    kd = 0 if dyn is None else dyn["scores"].shape[1]
+    keep = ks + kd if n_keep is None else n_keep
+    if anchor is not None:
+        _need(anchor, "anchor", torch.int32, 1)
+    if out is None:
+        out = _i32((q, keep, ds.m), static_idx.device)
+    _check(lib().sense_hybrid_drafts(C.c_void_p(ds.handle), static_scores.data_ptr(),
+                                     static_idx.data_ptr(), ks,
+                                     None if dyn is None else dyn["scores"].data_ptr(),
+                                     None if dyn is None else dyn["spans"].data_ptr(), kd, q,
+                                     _ptr(anchor), keep, 1 if force_anchor else 0,
+                                     out.data_ptr(), C.c_void_p(_stream(stream))))
+    return out
+
+
 def sense_soft_gate_workspace_bytes(q: int, cap: int, kappa: int) -> int:
     return int(lib().sense_soft_gate_workspace_bytes(q, cap, kappa))
 

@@ -40,6 +40,7 @@ enum KernelId {
   K_IVF_BUILD,
   K_IVF_COARSE,
   K_IVF_SCAN,
+  K_CTX,
   K_COUNT
 };
 

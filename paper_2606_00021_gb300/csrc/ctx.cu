@@ -1,0 +1,364 @@
+// Dynamic context buffer C_d and the hybrid static + dynamic candidate list.
+//
+// Sec. 3.2.1 Eq. 6 joins a static corpus C_s and a dynamic buffer C_d filled
+// from the generation itself: Alg. 1 calls R.Update(h, y) after prefill and
+// R.Update(H_align[i*, 0:L*+1], a) after each accepted step, i.e. it appends
+// (hidden state, the token that state predicted) pairs.  Alg. 2 searches the
+// buffer with DynSearch, boosts its scores by delta and reranks the union
+// with Eq. 8.  Readings (the paper leaves DynSearch and the buffer size
+// open): an entry is a position p with key L2Norm(h_p) (bf16, like the
+// static keys) and span y_{p+1} .. y_{p+M}; it is searchable once its M
+// continuation tokens exist; the buffer is a ring over the C most recent
+// positions; DynSearch is the exact inner-product top-k (ties to the older
+// position).
+//  - ctx_append_kernel: one warp per appended row: fp64 norm, bf16 key into
+//    ring slot p mod C, token into the token ring;
+//  - ctx_score_kernel: one warp per (entry, query): fp32 dot product of the
+//    bf16 key and query + delta -> candidate key in the query's pool;
+//  - the exact top-k of the pool is the shared merge; ctx_spans_kernel
+//    turns the winners into positions and spans;
+//  - hybrid_kernel: one block per query sorts the union of static and
+//    dynamic candidates by (score desc, union index asc), applies the
+//    anchor-first stable partition and the forced anchor, and copies the
+//    kept spans.
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+#include "launch.h"
+
+struct sense_ctx {
+  int32_t cap;
+  int32_t d;
+  int32_t m;
+  int64_t count;     // positions appended so far (host side, stream-ordered)
+  int device;
+  uint16_t* keys;    // [cap, d] bf16 ring
+  int32_t* tokens;   // [cap] ring: tokens[p mod cap] = y_{p+1}
+};
+
+namespace sense {
+namespace {
+
+constexpr int kHybridMax = 2048;  // static + dynamic candidates per query
+
+__global__ void __launch_bounds__(256)
+ctx_append_kernel(const uint16_t* __restrict__ hidden, const int32_t* __restrict__ tok, int t,
+                  int first, int64_t count, int cap, int d, uint16_t* __restrict__ keys,
+                  int32_t* __restrict__ ring) {
+  const int lane = threadIdx.x & 31;
+  const int i = first + (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  if (i >= t) return;  // warp-uniform
+  const int64_t slot = (count + i) % cap;
+  const uint16_t* x = hidden + (int64_t)i * d;
+  double ss = 0.0;
+  for (int j = lane; j < d; j += 32) {
+    const double v = (double)__uint_as_float((uint32_t)x[j] << 16);
+    ss = fma(v, v, ss);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+  const double nrm = sqrt(ss);
+  __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(keys + slot * d);
+  for (int j = lane; j < d; j += 32) {
+    const double v = (double)__uint_as_float((uint32_t)x[j] << 16);
+    y[j] = nrm > 0.0 ? __double2bfloat16(v / nrm) : __double2bfloat16(0.0);
+  }
+  if (lane == 0) ring[slot] = tok[i];
+}
+
+__global__ void __launch_bounds__(256)
+ctx_score_kernel(const uint16_t* __restrict__ keys, const uint16_t* __restrict__ queries, int q,
+                 int d, int cap, int64_t lo, int n_valid, float delta,
+                 uint64_t* __restrict__ pool) {
+  const int lane = threadIdx.x & 31;
+  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (w >= (int64_t)n_valid * q) return;  // warp-uniform
+  const int qi = (int)(w / n_valid);
+  const int e = (int)(w - (int64_t)qi * n_valid);
+  const uint16_t* kr = keys + ((lo + e) % cap) * d;
+  const uint16_t* qr = queries + (int64_t)qi * d;
+  float acc = 0.0f;
+  for (int j = 8 * lane; j < d; j += 256) {
+    const uint4 a = *reinterpret_cast<const uint4*>(kr + j);
+    const uint4 b = *reinterpret_cast<const uint4*>(qr + j);
+    acc = fmaf(bf_lo(a.x), bf_lo(b.x), acc);
+    acc = fmaf(bf_hi(a.x), bf_hi(b.x), acc);
+    acc = fmaf(bf_lo(a.y), bf_lo(b.y), acc);
+    acc = fmaf(bf_hi(a.y), bf_hi(b.y), acc);
+    acc = fmaf(bf_lo(a.z), bf_lo(b.z), acc);
+    acc = fmaf(bf_hi(a.z), bf_hi(b.z), acc);
+    acc = fmaf(bf_lo(a.w), bf_lo(b.w), acc);
+    acc = fmaf(bf_hi(a.w), bf_hi(b.w), acc);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if (lane == 0) pool[(int64_t)qi * n_valid + e] = cand_key(acc + delta, (uint32_t)e);
+}
+
+__global__ void ctx_spans_kernel(const int32_t* __restrict__ rel, int q, int k, int64_t lo,
+                                 int cap, int m, const int32_t* __restrict__ ring,
+                                 int32_t* __restrict__ out_pos, int32_t* __restrict__ out_spans) {
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= (int64_t)q * k) return;
+  const int e = rel[t];
+  int32_t* sp = out_spans + t * m;
+  if (e < 0) {
+    out_pos[t] = -1;
+    for (int j = 0; j < m; ++j) sp[j] = -1;
+    return;
+  }
+  const int64_t p = lo + e;
+  out_pos[t] = (int32_t)p;
+  for (int j = 0; j < m; ++j) sp[j] = ring[(p + j) % cap];
+}
+
+// One block (1024 threads) per query.  Union index u < ks: static rank u;
+// u >= ks: dynamic rank u - ks.
+__global__ void __launch_bounds__(1024)
+hybrid_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
+              const float* __restrict__ s_scores, const int32_t* __restrict__ s_idx, int ks,
+              const float* __restrict__ d_scores, const int32_t* __restrict__ d_spans, int kd,
+              const int32_t* __restrict__ anchor, int n_keep, int force,
+              int32_t* __restrict__ out, uint32_t* status) {
+  __shared__ uint64_t key[kHybridMax];
+  __shared__ int dest[kHybridMax];
+  __shared__ int n_live;
+  const int qi = blockIdx.x;
+  const int tot = ks + kd;
+  int pw = 1;
+  while (pw < tot) pw <<= 1;
+  const bool has_anchor = anchor != nullptr;
+  const int a = has_anchor ? anchor[qi] : 0;
+  if (threadIdx.x == 0) n_live = 0;
+  __syncthreads();
+  for (int u = threadIdx.x; u < pw; u += blockDim.x) {
+    uint64_t kk = 0ull;
+    if (u < ks) {
+      const int idx = s_idx[(int64_t)qi * ks + u];
+      if (idx >= 0 && idx < n) kk = cand_key(s_scores[(int64_t)qi * ks + u], (uint32_t)u);
+      else raise_status(status, SENSE_DEVST_BAD_INDEX);
+    } else if (u < tot) {
+      const float s = d_scores[(int64_t)qi * kd + (u - ks)];
+      if (s > -__int_as_float(0x7f800000)) kk = cand_key(s, (uint32_t)u);
+    }
+    if (kk) atomicAdd(&n_live, 1);
+    key[u] = kk;
+  }
+  __syncthreads();
+  // bitonic sort, descending: (score desc, union index asc); empty keys last
+  for (int size = 2; size <= pw; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < pw; i += blockDim.x) {
+        const int j = i ^ stride;
+        if (j > i) {
+          const bool desc = (i & size) == 0;
+          const uint64_t x = key[i], y = key[j];
+          if (desc ? (x < y) : (x > y)) {
+            key[i] = y;
+            key[j] = x;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  const int live = n_live;
+  auto first_token = [&](int u) -> int {
+    if (u < ks) return spans[(int64_t)s_idx[(int64_t)qi * ks + u] * m];
+    return d_spans[((int64_t)qi * kd + (u - ks)) * m];
+  };
+  // stable partition (anchor matches first), one warp, 32 candidates a step
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    int base = 0;
+    for (int pass = 0; pass < (has_anchor ? 2 : 1); ++pass) {
+      for (int r0 = 0; r0 < live; r0 += 32) {
+        const int r = r0 + lane;
+        bool take = false;
+        int u = 0;
+        if (r < live) {
+          u = (int)cand_index(key[r]);
+          const bool match = has_anchor && first_token(u) == a;
+          take = has_anchor ? (pass == 0 ? match : !match) : true;
+        }
+        const unsigned b = __ballot_sync(0xffffffffu, take);
+        if (take) dest[base + __popc(b & ((1u << lane) - 1u))] = u;
+        base += __popc(b);
+      }
+    }
+  }
+  __syncthreads();
+  const int64_t obase = (int64_t)qi * n_keep * m;
+  for (int e = threadIdx.x; e < n_keep * m; e += blockDim.x) {
+    const int o = e / m, j = e - o * m;
+    int v = -1;
+    if (o < live) {
+      const int u = dest[o];
+      v = (u < ks) ? spans[(int64_t)s_idx[(int64_t)qi * ks + u] * m + j]
+                   : d_spans[((int64_t)qi * kd + (u - ks)) * m + j];
+    }
+    if (force && has_anchor && j == 0 && (o == 0 || o == n_keep - 1)) v = a;
+    out[obase + e] = v;
+  }
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+int current_device() {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  return dev;
+}
+
+bool aligned(const void* ptr, size_t a) { return (reinterpret_cast<uintptr_t>(ptr) % a) == 0; }
+
+// Searchable positions [lo, lo + n_valid) after `count` appended positions.
+void ctx_range(const sense_ctx* c, int64_t* lo, int* n_valid) {
+  const int64_t l = c->count > c->cap ? c->count - c->cap : 0;
+  const int64_t hi = c->count - c->m + 1;  // exclusive
+  *lo = l;
+  *n_valid = hi > l ? (int)(hi - l) : 0;
+}
+
+}  // namespace
+}  // namespace sense
+
+using namespace sense;
+
+extern "C" {
+
+sense_status sense_ctx_create(int32_t capacity, int32_t d, int32_t m, sense_ctx** out) {
+  if (!out) return fail(SENSE_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (m < 1 || m > SENSE_MAX_M) return fail(SENSE_ERR_INVALID_ARG, "m=%d outside [1, %d]", m, SENSE_MAX_M);
+  if (capacity < m || capacity > (1 << 24))
+    return fail(SENSE_ERR_INVALID_ARG, "capacity=%d outside [m, 2^24]", capacity);
+  if (d < 8 || d % 8) return fail(SENSE_ERR_INVALID_ARG, "d=%d must be a positive multiple of 8", d);
+  auto* c = new sense_ctx{};
+  c->cap = capacity;
+  c->d = d;
+  c->m = m;
+  c->device = current_device();
+  if (cudaMalloc(&c->keys, (size_t)capacity * d * 2) != cudaSuccess ||
+      cudaMalloc(&c->tokens, (size_t)capacity * 4) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(c->keys);
+    cudaFree(c->tokens);
+    delete c;
+    return fail(SENSE_ERR_OOM, "context buffer allocation failed");
+  }
+  *out = c;
+  return SENSE_OK;
+}
+
+sense_status sense_ctx_destroy(sense_ctx* c) {
+  if (!c) return SENSE_OK;
+  cudaFree(c->keys);
+  cudaFree(c->tokens);
+  delete c;
+  return SENSE_OK;
+}
+
+sense_status sense_ctx_reset(sense_ctx* c) {
+  if (!c) return fail(SENSE_ERR_INVALID_ARG, "ctx is NULL");
+  c->count = 0;
+  return SENSE_OK;
+}
+
+int64_t sense_ctx_count(const sense_ctx* c) { return c ? c->count : -1; }
+
+sense_status sense_ctx_append(sense_ctx* c, const uint16_t* hidden, const int32_t* tokens, int32_t t,
+                              sense_stream_t stream) {
+  if (!c) return fail(SENSE_ERR_INVALID_ARG, "ctx is NULL");
+  if (t < 0) return fail(SENSE_ERR_INVALID_ARG, "t=%d must be >= 0", t);
+  if (t == 0) return SENSE_OK;
+  if (!hidden || !tokens) return fail(SENSE_ERR_INVALID_ARG, "hidden and tokens must be non-NULL");
+  if (!aligned(hidden, 16) || !aligned(tokens, 4)) return fail(SENSE_ERR_INVALID_ARG, "hidden must be 16-byte aligned");
+  if (c->count + t >= INT32_MAX) return fail(SENSE_ERR_UNSUPPORTED, "more than 2^31 positions");
+  if (current_device() != c->device) return fail(SENSE_ERR_INVALID_ARG, "ctx lives on device %d", c->device);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int first = t > c->cap ? t - c->cap : 0;  // earlier rows would be overwritten
+  const int64_t warps = t - first;
+  {
+    LaunchScope ls(K_CTX, s);
+    ctx_append_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(
+        hidden, tokens, t, first, c->count, c->cap, c->d, c->keys, c->tokens);
+    sense_status st = cuda_check(cudaGetLastError(), "launch ctx append");
+    if (st != SENSE_OK) return st;
+  }
+  c->count += t;
+  return SENSE_OK;
+}
+
+size_t sense_ctx_search_workspace_bytes(const sense_ctx* c, int32_t q, int32_t k) {
+  if (!c || q < 1 || k < 1) return 0;
+  return align256((size_t)q * c->cap * 8) + align256((size_t)q * k * 4);
+}
+
+sense_status sense_ctx_search(const sense_ctx* c, const uint16_t* queries, int32_t q, int32_t k,
+                              float delta, float* out_scores, int32_t* out_pos, int32_t* out_spans,
+                              void* workspace, size_t workspace_bytes, sense_stream_t stream) {
+  if (!c) return fail(SENSE_ERR_INVALID_ARG, "ctx is NULL");
+  if (!queries || !out_scores || !out_pos || !out_spans || !workspace)
+    return fail(SENSE_ERR_INVALID_ARG, "queries, outputs and workspace must be non-NULL");
+  if (q < 1 || q > 65535) return fail(SENSE_ERR_INVALID_ARG, "q=%d outside [1, 65535]", q);
+  if (k < 1 || k > SENSE_MAX_K) return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, %d]", k, SENSE_MAX_K);
+  if (!(delta == delta) || delta > 1e30f || delta < -1e30f) return fail(SENSE_ERR_INVALID_ARG, "delta must be finite");
+  if (!aligned(queries, 16)) return fail(SENSE_ERR_INVALID_ARG, "queries must be 16-byte aligned");
+  if (!aligned(workspace, 256)) return fail(SENSE_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  if (workspace_bytes < sense_ctx_search_workspace_bytes(c, q, k))
+    return fail(SENSE_ERR_INVALID_ARG, "workspace of %zu bytes < %zu", workspace_bytes,
+                sense_ctx_search_workspace_bytes(c, q, k));
+  if (current_device() != c->device) return fail(SENSE_ERR_INVALID_ARG, "ctx lives on device %d", c->device);
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int64_t lo;
+  int n_valid;
+  ctx_range(c, &lo, &n_valid);
+  char* ws = static_cast<char*>(workspace);
+  auto* pool = reinterpret_cast<uint64_t*>(ws);
+  auto* rel = reinterpret_cast<int32_t*>(ws + align256((size_t)q * c->cap * 8));
+  if (n_valid > 0) {
+    LaunchScope ls(K_CTX, s);
+    const int64_t threads = (int64_t)n_valid * q * 32;
+    ctx_score_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(
+        c->keys, queries, q, c->d, c->cap, lo, n_valid, delta, pool);
+    sense_status st = cuda_check(cudaGetLastError(), "launch ctx score");
+    if (st != SENSE_OK) return st;
+  }
+  sense_status st = launch_merge_short(pool, nullptr, n_valid, q, k, out_scores, rel, status, s);
+  if (st != SENSE_OK) return st;
+  LaunchScope ls(K_CTX, s);
+  ctx_spans_kernel<<<(unsigned)(((int64_t)q * k + 255) / 256), 256, 0, s>>>(
+      rel, q, k, lo, c->cap, c->m, c->tokens, out_pos, out_spans);
+  return cuda_check(cudaGetLastError(), "launch ctx spans");
+}
+
+sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_scores,
+                                 const int32_t* static_idx, int32_t ks, const float* dyn_scores,
+                                 const int32_t* dyn_spans, int32_t kd, int32_t q,
+                                 const int32_t* anchor, int32_t n_keep, uint32_t flags,
+                                 int32_t* out_spans, sense_stream_t stream) {
+  if (!ds) return fail(SENSE_ERR_INVALID_ARG, "ds is NULL");
+  if (q < 1 || q > 65535) return fail(SENSE_ERR_INVALID_ARG, "q=%d outside [1, 65535]", q);
+  if (ks < 0 || kd < 0 || ks + kd < 1 || ks + kd > kHybridMax)
+    return fail(SENSE_ERR_INVALID_ARG, "ks=%d, kd=%d: need 1 <= ks + kd <= %d", ks, kd, kHybridMax);
+  if ((ks && (!static_scores || !static_idx)) || (kd && (!dyn_scores || !dyn_spans)) || !out_spans)
+    return fail(SENSE_ERR_INVALID_ARG, "candidate arrays and out_spans must be non-NULL");
+  if (n_keep < 1 || n_keep > ks + kd)
+    return fail(SENSE_ERR_INVALID_ARG, "n_keep=%d outside [1, ks + kd]", n_keep);
+  if (flags & ~SENSE_GATHER_FORCE_ANCHOR) return fail(SENSE_ERR_INVALID_ARG, "unknown flags 0x%x", flags);
+  if ((flags & SENSE_GATHER_FORCE_ANCHOR) && !anchor)
+    return fail(SENSE_ERR_INVALID_ARG, "SENSE_GATHER_FORCE_ANCHOR needs anchor");
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  LaunchScope ls(K_CTX, s);
+  hybrid_kernel<<<q, 1024, 0, s>>>(ds->spans, ds->n, ds->m, static_scores, static_idx, ks,
+                                   dyn_scores, dyn_spans, kd, anchor, n_keep,
+                                   (flags & SENSE_GATHER_FORCE_ANCHOR) ? 1 : 0, out_spans, status);
+  return cuda_check(cudaGetLastError(), "launch hybrid drafts");
+}
+
+}  // extern "C"
