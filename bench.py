@@ -190,6 +190,27 @@ class Pipeline:
         S.sense_soft_gate(self.tree, root, nodes, hr, hn, workspace=self.gws, outs=self.gate, **GATE)
 
 
+class GraphStep:
+    """The whole drafting step captured as one CUDA graph per gate-input set.
+    The graphs read the query from a fixed staging buffer; a step copies the
+    next query into it (device to device) and replays one graph."""
+
+    def __init__(self, pipe, query0, gate_sets):
+        self.d_query = torch.empty_like(query0)
+        self.d_query.copy_(query0)
+        self.graphs = []
+        for gset in gate_sets:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                pipe.step(self.d_query, gset)
+            self.graphs.append(g)
+        torch.cuda.synchronize()
+
+    def step(self, query, gi):
+        self.d_query.copy_(query, non_blocking=True)
+        self.graphs[gi].replay()
+
+
 def build_ann(S, keys, kind, nlist, nprobe, pq_m, v, dev, seed=0):
     """Index construction for the approximate path (outside the timed region):
     the PCA basis is fitted offline on a 65,536-key sample (eigenvectors of
@@ -338,6 +359,8 @@ def main():
     ap.add_argument("--nprobe", type=int, default=32)
     ap.add_argument("--pq-m", type=int, default=16)
     ap.add_argument("--proj-dim", type=int, default=64)
+    ap.add_argument("--graph", action="store_true",
+                    help="time CUDA graph replays of the whole step")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     cfg = dict(WORKLOADS[args.workload])
@@ -385,6 +408,19 @@ def main():
     torch.cuda.synchronize()
     if S.sense_device_status(clear=True) != 0:
         raise RuntimeError("device status bits set after warm-up")
+    graph, graph_error = None, None
+    if args.graph:
+        try:
+            graph = GraphStep(pipe, queries[0], gate_sets)
+        except Exception as e:  # capture refused: time eager launches and say why
+            graph_error = f"graph capture failed ({type(e).__name__}: {e}); eager launches timed"
+            torch.cuda.synchronize()
+    if graph is not None:
+        for it in range(args.warmup):
+            graph.step(queries[it % nq], it % n_sets)
+        torch.cuda.synchronize()
+        if S.sense_device_status(clear=True) != 0:
+            raise RuntimeError("device status bits set after graph warm-up")
 
     clocks = ClockSampler(local)
     clocks.start()
@@ -392,19 +428,42 @@ def main():
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    S.sense_profile_enable(True)
     stream = torch.cuda.current_stream()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for it in range(args.steps):
-        pipe.step(queries[it % nq], gate_sets[it % n_sets])
-    e1.record(stream)
-    torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
-    clk = clocks.stop()
-    ms = e0.elapsed_time(e1)
+    graph_note = graph_error
+    if graph is not None:
+        # timed region: per step, copy the query into the staging buffer and
+        # replay the captured step of this gate-input set
+        e0.record(stream)
+        for it in range(args.steps):
+            graph.step(queries[it % nq], it % n_sets)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        clk = clocks.stop()
+        ms = e0.elapsed_time(e1)
+        # CUDA events cannot time single kernels inside a replay: the
+        # per-kernel times (roofline) come from an eager pass over the same
+        # steps right after
+        S.sense_profile_enable(True)
+        for it in range(args.steps):
+            pipe.step(queries[it % nq], gate_sets[it % n_sets])
+        torch.cuda.synchronize()
+        graph_note = (f"timed region: {args.steps} CUDA graph replays; kernel times from an "
+                      f"eager pass of the same {args.steps} steps")
+    else:
+        S.sense_profile_enable(True)
+        e0.record(stream)
+        for it in range(args.steps):
+            pipe.step(queries[it % nq], gate_sets[it % n_sets])
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        clk = clocks.stop()
+        ms = e0.elapsed_time(e1)
     prof = {name: S.sense_profile_query(name) for name in S.sense_profile_names()}
     S.sense_profile_enable(False)
     ms = max_over_ranks(ms, dist, dev)
@@ -558,6 +617,8 @@ def main():
                              "streamed every step",
                        "parallelism": f"replicas x{world}"},
             "retrieval": retrieval,
+            "launch": "cuda_graph" if graph is not None else "eager",
+            "launch_note": graph_note,
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,
             "draft_tokens_per_s": value * mean_nodes,
             "mean_tree_nodes": mean_nodes,
