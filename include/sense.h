@@ -331,10 +331,13 @@ sense_status sense_gather_drafts(const sense_datastore* ds, const int32_t* idx, 
  * d % 8 == 0. */
 sense_status sense_ctx_create(int32_t capacity, int32_t d, int32_t m, sense_ctx** out);
 sense_status sense_ctx_destroy(sense_ctx* ctx);
-/* Forgets every entry (no device work). */
-sense_status sense_ctx_reset(sense_ctx* ctx);
-/* Positions appended since creation or the last reset (-1 for NULL). */
-int64_t sense_ctx_count(const sense_ctx* ctx);
+/* The buffer's position counter lives on the device, so that appends whose
+ * length is only known there (sense_ctx_append_path) need no host round
+ * trip.  sense_ctx_reset forgets every entry (asynchronous on `stream`);
+ * sense_ctx_count synchronises `stream` and reads the number of positions
+ * appended since creation or the last reset. */
+sense_status sense_ctx_reset(sense_ctx* ctx, sense_stream_t stream);
+sense_status sense_ctx_count(const sense_ctx* ctx, sense_stream_t stream, int64_t* out);
 
 /*
  * R.Update: appends t positions.  hidden [t, d] bf16 (16-byte aligned):
@@ -347,17 +350,33 @@ sense_status sense_ctx_append(sense_ctx* ctx, const uint16_t* hidden, const int3
                               int32_t t, sense_stream_t stream);
 
 /*
+ * R.Update after a verified step (Alg. 1): appends the accepted path
+ * H_align[i*, 0:L*+1] with the accepted tokens a, entirely on the device.
+ * Position j < n_accept gets the hidden state root_hidden [d] (j = 0) or
+ * node_hidden[gamma[i*, j-1]] (node_hidden [n_nodes, d] bf16; gamma [k, m]
+ * of this query's tree) and the token accepted[j]; i_star, n_accept and
+ * accepted are device pointers (the outputs of sense_soft_gate for one
+ * query).  An i* or a node outside its range sets SENSE_DEVST_BAD_INDEX and
+ * that position is skipped.
+ */
+sense_status sense_ctx_append_path(sense_ctx* ctx, const uint16_t* root_hidden,
+                                   const uint16_t* node_hidden, int32_t n_nodes,
+                                   const int32_t* gamma, int32_t k, const int32_t* i_star,
+                                   const int32_t* n_accept, const int32_t* accepted,
+                                   sense_stream_t stream);
+
+/*
  * DynSearch: per query (queries [q, d] bf16, 16-byte aligned), the k
  * searchable entries with the largest <q, key> (fp32 accumulation), order
  * (score desc, position asc).  out_scores [q, k] f32 = score + delta;
- * out_pos [q, k] int32 positions; out_spans [q, k, m] int32.  Slots past the
+ * out_pos [q, k] int64 positions; out_spans [q, k, m] int32.  Slots past the
  * number of searchable entries get -inf, -1 and a span of -1.  workspace:
  * sense_ctx_search_workspace_bytes(ctx, q, k) bytes, 256-byte aligned.
  * Limits: 1 <= q <= 65535, 1 <= k <= SENSE_MAX_K, delta finite.
  */
 size_t sense_ctx_search_workspace_bytes(const sense_ctx* ctx, int32_t q, int32_t k);
 sense_status sense_ctx_search(const sense_ctx* ctx, const uint16_t* queries, int32_t q, int32_t k,
-                              float delta, float* out_scores, int32_t* out_pos,
+                              float delta, float* out_scores, int64_t* out_pos,
                               int32_t* out_spans, void* workspace, size_t workspace_bytes,
                               sense_stream_t stream);
 

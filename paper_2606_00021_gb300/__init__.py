@@ -420,10 +420,14 @@ class ContextBuffer:
 
     @property
     def count(self) -> int:
-        return int(lib().sense_ctx_count(C.c_void_p(self.handle)))
+        """Positions appended so far (synchronises the current stream)."""
+        out = C.c_int64(0)
+        _check(lib().sense_ctx_count(C.c_void_p(self.handle), C.c_void_p(_stream(None)),
+                                     C.byref(out)))
+        return int(out.value)
 
-    def reset(self):
-        _check(lib().sense_ctx_reset(C.c_void_p(self.handle)))
+    def reset(self, stream=None):
+        _check(lib().sense_ctx_reset(C.c_void_p(self.handle), C.c_void_p(_stream(stream))))
 
 
 def sense_ctx_create(capacity: int, d: int, m: int) -> ContextBuffer:
@@ -442,6 +446,24 @@ def sense_ctx_append(ctx: ContextBuffer, hidden: torch.Tensor, tokens: torch.Ten
                                   hidden.shape[0], C.c_void_p(_stream(stream))))
 
 
+def sense_ctx_append_path(ctx: ContextBuffer, root_hidden: torch.Tensor,
+                          node_hidden: torch.Tensor, gamma: torch.Tensor, i_star: torch.Tensor,
+                          n_accept: torch.Tensor, accepted: torch.Tensor, stream=None):
+    """R.Update of one verified step, on the device: root_hidden [d] and
+    node_hidden [n_nodes, d] bf16, gamma [k, m], i_star / n_accept [1] and
+    accepted [m] int32 (one query's tree and gate outputs)."""
+    _need(root_hidden, "root_hidden", torch.bfloat16, 1)
+    _need(node_hidden, "node_hidden", torch.bfloat16, 2)
+    _need(gamma, "gamma", torch.int32, 2)
+    for t, name in ((i_star, "i_star"), (n_accept, "n_accept"), (accepted, "accepted")):
+        _need(t, name, torch.int32, 1)
+    _check(lib().sense_ctx_append_path(C.c_void_p(ctx.handle), root_hidden.data_ptr(),
+                                       node_hidden.data_ptr(), node_hidden.shape[0],
+                                       gamma.data_ptr(), gamma.shape[0], i_star.data_ptr(),
+                                       n_accept.data_ptr(), accepted.data_ptr(),
+                                       C.c_void_p(_stream(stream))))
+
+
 def sense_ctx_search(ctx: ContextBuffer, queries: torch.Tensor, k: int, delta: float = 0.0,
                      outs: dict | None = None, workspace=None, stream=None) -> dict:
     """DynSearch: dict of scores [q, k] (boosted), pos [q, k], spans [q, k, m]."""
@@ -450,7 +472,7 @@ def sense_ctx_search(ctx: ContextBuffer, queries: torch.Tensor, k: int, delta: f
     dev = queries.device
     o = outs if outs is not None else {}
     o.setdefault("scores", torch.empty(q, k, dtype=torch.float32, device=dev))
-    o.setdefault("pos", _i32((q, k), dev))
+    o.setdefault("pos", torch.empty(q, k, dtype=torch.int64, device=dev))
     o.setdefault("spans", _i32((q, k, ctx.m), dev))
     if workspace is None:
         workspace = alloc_workspace(lib().sense_ctx_search_workspace_bytes(

@@ -44,9 +44,10 @@ SIGNATURES = {
     "sense_ivf_search": (c_i32, [c_p, c_p, c_i32, c_i32, c_i32, c_p, c_p, c_p, c_p, c_size, c_p]),
     "sense_ctx_create": (c_i32, [c_i32, c_i32, c_i32, C.POINTER(c_p)]),
     "sense_ctx_destroy": (c_i32, [c_p]),
-    "sense_ctx_reset": (c_i32, [c_p]),
-    "sense_ctx_count": (c_i64, [c_p]),
+    "sense_ctx_reset": (c_i32, [c_p, c_p]),
+    "sense_ctx_count": (c_i32, [c_p, c_p, C.POINTER(c_i64)]),
     "sense_ctx_append": (c_i32, [c_p, c_p, c_p, c_i32, c_p]),
+    "sense_ctx_append_path": (c_i32, [c_p, c_p, c_p, c_i32, c_p, c_i32, c_p, c_p, c_p, c_p]),
     "sense_ctx_search_workspace_bytes": (c_size, [c_p, c_i32, c_i32]),
     "sense_ctx_search": (c_i32, [c_p, c_p, c_i32, c_i32, C.c_float, c_p, c_p, c_p, c_p, c_size,
                                  c_p]),

@@ -11,8 +11,13 @@
 // continuation tokens exist; the buffer is a ring over the C most recent
 // positions; DynSearch is the exact inner-product top-k (ties to the older
 // position).
+// The position counter lives in device memory, so that appends whose length
+// is only known on the device (the accepted prefix of a step) need no host
+// round trip and a whole decode step can be captured in a CUDA graph.
 //  - ctx_append_kernel: one warp per appended row: fp64 norm, bf16 key into
-//    ring slot p mod C, token into the token ring;
+//    ring slot p mod C, token into the token ring (rows: a host-given block,
+//    or the accepted path H_align[i*, 0:L*+1] read through Gamma);
+//  - ctx_bump_kernel: advances the counter after the rows are written;
 //  - ctx_score_kernel: one warp per (entry, query): fp32 dot product of the
 //    bf16 key and query + delta -> candidate key in the query's pool;
 //  - the exact top-k of the pool is the shared merge; ctx_spans_kernel
@@ -23,6 +28,8 @@
 //    kept spans.
 #include <cuda_bf16.h>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "launch.h"
 
@@ -30,10 +37,10 @@ struct sense_ctx {
   int32_t cap;
   int32_t d;
   int32_t m;
-  int64_t count;     // positions appended so far (host side, stream-ordered)
   int device;
   uint16_t* keys;    // [cap, d] bf16 ring
   int32_t* tokens;   // [cap] ring: tokens[p mod cap] = y_{p+1}
+  int64_t* count;    // device: positions appended so far (stream-ordered)
 };
 
 namespace sense {
@@ -41,15 +48,10 @@ namespace {
 
 constexpr int kHybridMax = 2048;  // static + dynamic candidates per query
 
-__global__ void __launch_bounds__(256)
-ctx_append_kernel(const uint16_t* __restrict__ hidden, const int32_t* __restrict__ tok, int t,
-                  int first, int64_t count, int cap, int d, uint16_t* __restrict__ keys,
-                  int32_t* __restrict__ ring) {
+// Writes the key and token of one position; `x` is its bf16 hidden state.
+__device__ void append_row(const uint16_t* __restrict__ x, int32_t token, int64_t slot, int d,
+                           uint16_t* __restrict__ keys, int32_t* __restrict__ ring) {
   const int lane = threadIdx.x & 31;
-  const int i = first + (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
-  if (i >= t) return;  // warp-uniform
-  const int64_t slot = (count + i) % cap;
-  const uint16_t* x = hidden + (int64_t)i * d;
   double ss = 0.0;
   for (int j = lane; j < d; j += 32) {
     const double v = (double)__uint_as_float((uint32_t)x[j] << 16);
@@ -63,43 +65,112 @@ ctx_append_kernel(const uint16_t* __restrict__ hidden, const int32_t* __restrict
     const double v = (double)__uint_as_float((uint32_t)x[j] << 16);
     y[j] = nrm > 0.0 ? __double2bfloat16(v / nrm) : __double2bfloat16(0.0);
   }
-  if (lane == 0) ring[slot] = tok[i];
+  if (lane == 0) ring[slot] = token;
 }
 
+// Host-given rows: one warp per row i in [first, t).
+__global__ void __launch_bounds__(256)
+ctx_append_kernel(const uint16_t* __restrict__ hidden, const int32_t* __restrict__ tok, int t,
+                  int first, const int64_t* __restrict__ count, int cap, int d,
+                  uint16_t* __restrict__ keys, int32_t* __restrict__ ring) {
+  const int i = first + (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  if (i >= t) return;  // warp-uniform
+  append_row(hidden + (int64_t)i * d, tok[i], (*count + i) % cap, d, keys, ring);
+}
+
+// Accepted path of one step: warp j < n_accept appends H_align[i*, j] (the
+// root state for j = 0, else the state of node Gamma[i*, j-1]) with the
+// accepted token a_j.
+__global__ void __launch_bounds__(256)
+ctx_append_path_kernel(const uint16_t* __restrict__ root, const uint16_t* __restrict__ nodes,
+                       int n_nodes, const int32_t* __restrict__ gamma, int k, int m,
+                       const int32_t* __restrict__ i_star, const int32_t* __restrict__ n_accept,
+                       const int32_t* __restrict__ accepted, const int64_t* __restrict__ count,
+                       int cap, int d, uint16_t* __restrict__ keys, int32_t* __restrict__ ring,
+                       uint32_t* status) {
+  const int j = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const int na = *n_accept, is = *i_star;
+  if (j >= na || j >= m) return;  // warp-uniform
+  if (is < 0 || is >= k || na > m) {
+    if ((threadIdx.x & 31) == 0) raise_status(status, SENSE_DEVST_BAD_INDEX);
+    return;
+  }
+  const uint16_t* x = root;
+  if (j > 0) {
+    const int node = gamma[(int64_t)is * m + j - 1];
+    if (node < 0 || node >= n_nodes) {
+      if ((threadIdx.x & 31) == 0) raise_status(status, SENSE_DEVST_BAD_INDEX);
+      return;
+    }
+    x = nodes + (int64_t)node * d;
+  }
+  append_row(x, accepted[j], (*count + j) % cap, d, keys, ring);
+}
+
+// count += t (host value) or += *t_dev (clamped to [0, m_max]).
+__global__ void ctx_bump_kernel(int64_t* count, int64_t t, const int32_t* t_dev, int m_max) {
+  if (t_dev) {
+    int v = *t_dev;
+    t = v < 0 ? 0 : (v > m_max ? m_max : v);
+  }
+  *count += t;
+}
+
+// Searchable positions [lo, lo + n_valid) after `count` appended positions.
+__device__ __forceinline__ void ctx_range_dev(int64_t count, int cap, int m, int64_t* lo,
+                                              int* n_valid) {
+  const int64_t l = count > cap ? count - cap : 0;
+  const int64_t hi = count - m + 1;  // exclusive
+  *lo = l;
+  *n_valid = hi > l ? (int)(hi - l) : 0;
+}
+
+// Grid-stride over (query, entry) pairs, one warp each; also records the
+// number of searchable entries as every query's pool count.
 __global__ void __launch_bounds__(256)
 ctx_score_kernel(const uint16_t* __restrict__ keys, const uint16_t* __restrict__ queries, int q,
-                 int d, int cap, int64_t lo, int n_valid, float delta,
-                 uint64_t* __restrict__ pool) {
+                 int d, int cap, int m, const int64_t* __restrict__ count, float delta,
+                 uint64_t* __restrict__ pool, uint32_t* __restrict__ counts) {
   const int lane = threadIdx.x & 31;
-  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  if (w >= (int64_t)n_valid * q) return;  // warp-uniform
-  const int qi = (int)(w / n_valid);
-  const int e = (int)(w - (int64_t)qi * n_valid);
-  const uint16_t* kr = keys + ((lo + e) % cap) * d;
-  const uint16_t* qr = queries + (int64_t)qi * d;
-  float acc = 0.0f;
-  for (int j = 8 * lane; j < d; j += 256) {
-    const uint4 a = *reinterpret_cast<const uint4*>(kr + j);
-    const uint4 b = *reinterpret_cast<const uint4*>(qr + j);
-    acc = fmaf(bf_lo(a.x), bf_lo(b.x), acc);
-    acc = fmaf(bf_hi(a.x), bf_hi(b.x), acc);
-    acc = fmaf(bf_lo(a.y), bf_lo(b.y), acc);
-    acc = fmaf(bf_hi(a.y), bf_hi(b.y), acc);
-    acc = fmaf(bf_lo(a.z), bf_lo(b.z), acc);
-    acc = fmaf(bf_hi(a.z), bf_hi(b.z), acc);
-    acc = fmaf(bf_lo(a.w), bf_lo(b.w), acc);
-    acc = fmaf(bf_hi(a.w), bf_hi(b.w), acc);
-  }
+  int64_t lo;
+  int n_valid;
+  ctx_range_dev(*count, cap, m, &lo, &n_valid);
+  const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  if (gw < q && lane == 0) counts[gw] = (uint32_t)n_valid;
+  for (int64_t w = gw; w < (int64_t)n_valid * q; w += nw) {
+    const int qi = (int)(w / n_valid);
+    const int e = (int)(w - (int64_t)qi * n_valid);
+    const uint16_t* kr = keys + ((lo + e) % cap) * d;
+    const uint16_t* qr = queries + (int64_t)qi * d;
+    float acc = 0.0f;
+    for (int j = 8 * lane; j < d; j += 256) {
+      const uint4 a = *reinterpret_cast<const uint4*>(kr + j);
+      const uint4 b = *reinterpret_cast<const uint4*>(qr + j);
+      acc = fmaf(bf_lo(a.x), bf_lo(b.x), acc);
+      acc = fmaf(bf_hi(a.x), bf_hi(b.x), acc);
+      acc = fmaf(bf_lo(a.y), bf_lo(b.y), acc);
+      acc = fmaf(bf_hi(a.y), bf_hi(b.y), acc);
+      acc = fmaf(bf_lo(a.z), bf_lo(b.z), acc);
+      acc = fmaf(bf_hi(a.z), bf_hi(b.z), acc);
+      acc = fmaf(bf_lo(a.w), bf_lo(b.w), acc);
+      acc = fmaf(bf_hi(a.w), bf_hi(b.w), acc);
+    }
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-  if (lane == 0) pool[(int64_t)qi * n_valid + e] = cand_key(acc + delta, (uint32_t)e);
+    for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    if (lane == 0) pool[(int64_t)qi * cap + e] = cand_key(acc + delta, (uint32_t)e);
+  }
 }
 
-__global__ void ctx_spans_kernel(const int32_t* __restrict__ rel, int q, int k, int64_t lo,
-                                 int cap, int m, const int32_t* __restrict__ ring,
-                                 int32_t* __restrict__ out_pos, int32_t* __restrict__ out_spans) {
+__global__ void ctx_spans_kernel(const int32_t* __restrict__ rel, int q, int k,
+                                 const int64_t* __restrict__ count, int cap, int m,
+                                 const int32_t* __restrict__ ring, int64_t* __restrict__ out_pos,
+                                 int32_t* __restrict__ out_spans) {
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= (int64_t)q * k) return;
+  int64_t lo;
+  int n_valid;
+  ctx_range_dev(*count, cap, m, &lo, &n_valid);
   const int e = rel[t];
   int32_t* sp = out_spans + t * m;
   if (e < 0) {
@@ -108,7 +179,7 @@ __global__ void ctx_spans_kernel(const int32_t* __restrict__ rel, int q, int k, 
     return;
   }
   const int64_t p = lo + e;
-  out_pos[t] = (int32_t)p;
+  out_pos[t] = p;
   for (int j = 0; j < m; ++j) sp[j] = ring[(p + j) % cap];
 }
 
@@ -212,14 +283,6 @@ int current_device() {
 
 bool aligned(const void* ptr, size_t a) { return (reinterpret_cast<uintptr_t>(ptr) % a) == 0; }
 
-// Searchable positions [lo, lo + n_valid) after `count` appended positions.
-void ctx_range(const sense_ctx* c, int64_t* lo, int* n_valid) {
-  const int64_t l = c->count > c->cap ? c->count - c->cap : 0;
-  const int64_t hi = c->count - c->m + 1;  // exclusive
-  *lo = l;
-  *n_valid = hi > l ? (int)(hi - l) : 0;
-}
-
 }  // namespace
 }  // namespace sense
 
@@ -240,10 +303,13 @@ sense_status sense_ctx_create(int32_t capacity, int32_t d, int32_t m, sense_ctx*
   c->m = m;
   c->device = current_device();
   if (cudaMalloc(&c->keys, (size_t)capacity * d * 2) != cudaSuccess ||
-      cudaMalloc(&c->tokens, (size_t)capacity * 4) != cudaSuccess) {
+      cudaMalloc(&c->tokens, (size_t)capacity * 4) != cudaSuccess ||
+      cudaMalloc(&c->count, sizeof(int64_t)) != cudaSuccess ||
+      cudaMemset(c->count, 0, sizeof(int64_t)) != cudaSuccess) {
     cudaGetLastError();
     cudaFree(c->keys);
     cudaFree(c->tokens);
+    cudaFree(c->count);
     delete c;
     return fail(SENSE_ERR_OOM, "context buffer allocation failed");
   }
@@ -255,17 +321,24 @@ sense_status sense_ctx_destroy(sense_ctx* c) {
   if (!c) return SENSE_OK;
   cudaFree(c->keys);
   cudaFree(c->tokens);
+  cudaFree(c->count);
   delete c;
   return SENSE_OK;
 }
 
-sense_status sense_ctx_reset(sense_ctx* c) {
+sense_status sense_ctx_reset(sense_ctx* c, sense_stream_t stream) {
   if (!c) return fail(SENSE_ERR_INVALID_ARG, "ctx is NULL");
-  c->count = 0;
-  return SENSE_OK;
+  return cuda_check(cudaMemsetAsync(c->count, 0, sizeof(int64_t),
+                                    reinterpret_cast<cudaStream_t>(stream)), "reset ctx");
 }
 
-int64_t sense_ctx_count(const sense_ctx* c) { return c ? c->count : -1; }
+sense_status sense_ctx_count(const sense_ctx* c, sense_stream_t stream, int64_t* out) {
+  if (!c || !out) return fail(SENSE_ERR_INVALID_ARG, "ctx and out must be non-NULL");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  sense_status st = cuda_check(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+  if (st != SENSE_OK) return st;
+  return cuda_check(cudaMemcpy(out, c->count, sizeof(int64_t), cudaMemcpyDeviceToHost), "read count");
+}
 
 sense_status sense_ctx_append(sense_ctx* c, const uint16_t* hidden, const int32_t* tokens, int32_t t,
                               sense_stream_t stream) {
@@ -274,29 +347,47 @@ sense_status sense_ctx_append(sense_ctx* c, const uint16_t* hidden, const int32_
   if (t == 0) return SENSE_OK;
   if (!hidden || !tokens) return fail(SENSE_ERR_INVALID_ARG, "hidden and tokens must be non-NULL");
   if (!aligned(hidden, 16) || !aligned(tokens, 4)) return fail(SENSE_ERR_INVALID_ARG, "hidden must be 16-byte aligned");
-  if (c->count + t >= INT32_MAX) return fail(SENSE_ERR_UNSUPPORTED, "more than 2^31 positions");
   if (current_device() != c->device) return fail(SENSE_ERR_INVALID_ARG, "ctx lives on device %d", c->device);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int first = t > c->cap ? t - c->cap : 0;  // earlier rows would be overwritten
   const int64_t warps = t - first;
-  {
-    LaunchScope ls(K_CTX, s);
-    ctx_append_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(
-        hidden, tokens, t, first, c->count, c->cap, c->d, c->keys, c->tokens);
-    sense_status st = cuda_check(cudaGetLastError(), "launch ctx append");
-    if (st != SENSE_OK) return st;
-  }
-  c->count += t;
-  return SENSE_OK;
+  LaunchScope ls(K_CTX, s);
+  ctx_append_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(
+      hidden, tokens, t, first, c->count, c->cap, c->d, c->keys, c->tokens);
+  ctx_bump_kernel<<<1, 1, 0, s>>>(c->count, t, nullptr, 0);
+  return cuda_check(cudaGetLastError(), "launch ctx append");
+}
+
+sense_status sense_ctx_append_path(sense_ctx* c, const uint16_t* root_hidden,
+                                   const uint16_t* node_hidden, int32_t n_nodes,
+                                   const int32_t* gamma, int32_t k, const int32_t* i_star,
+                                   const int32_t* n_accept, const int32_t* accepted,
+                                   sense_stream_t stream) {
+  if (!c) return fail(SENSE_ERR_INVALID_ARG, "ctx is NULL");
+  if (!root_hidden || !node_hidden || !gamma || !i_star || !n_accept || !accepted)
+    return fail(SENSE_ERR_INVALID_ARG, "arrays must be non-NULL");
+  if (k < 1 || n_nodes < 1) return fail(SENSE_ERR_INVALID_ARG, "k=%d and n_nodes=%d must be >= 1", k, n_nodes);
+  if (!aligned(root_hidden, 16) || !aligned(node_hidden, 16))
+    return fail(SENSE_ERR_INVALID_ARG, "hidden states must be 16-byte aligned");
+  if (current_device() != c->device) return fail(SENSE_ERR_INVALID_ARG, "ctx lives on device %d", c->device);
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  LaunchScope ls(K_CTX, s);
+  ctx_append_path_kernel<<<(unsigned)((c->m * 32 + 255) / 256), 256, 0, s>>>(
+      root_hidden, node_hidden, n_nodes, gamma, k, c->m, i_star, n_accept, accepted, c->count,
+      c->cap, c->d, c->keys, c->tokens, status);
+  ctx_bump_kernel<<<1, 1, 0, s>>>(c->count, 0, n_accept, c->m);
+  return cuda_check(cudaGetLastError(), "launch ctx append path");
 }
 
 size_t sense_ctx_search_workspace_bytes(const sense_ctx* c, int32_t q, int32_t k) {
   if (!c || q < 1 || k < 1) return 0;
-  return align256((size_t)q * c->cap * 8) + align256((size_t)q * k * 4);
+  return align256((size_t)q * c->cap * 8) + align256((size_t)q * 4) + align256((size_t)q * k * 4);
 }
 
 sense_status sense_ctx_search(const sense_ctx* c, const uint16_t* queries, int32_t q, int32_t k,
-                              float delta, float* out_scores, int32_t* out_pos, int32_t* out_spans,
+                              float delta, float* out_scores, int64_t* out_pos, int32_t* out_spans,
                               void* workspace, size_t workspace_bytes, sense_stream_t stream) {
   if (!c) return fail(SENSE_ERR_INVALID_ARG, "ctx is NULL");
   if (!queries || !out_scores || !out_pos || !out_spans || !workspace)
@@ -313,25 +404,25 @@ sense_status sense_ctx_search(const sense_ctx* c, const uint16_t* queries, int32
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int64_t lo;
-  int n_valid;
-  ctx_range(c, &lo, &n_valid);
   char* ws = static_cast<char*>(workspace);
   auto* pool = reinterpret_cast<uint64_t*>(ws);
-  auto* rel = reinterpret_cast<int32_t*>(ws + align256((size_t)q * c->cap * 8));
-  if (n_valid > 0) {
+  auto* counts = reinterpret_cast<uint32_t*>(ws + align256((size_t)q * c->cap * 8));
+  auto* rel = reinterpret_cast<int32_t*>(ws + align256((size_t)q * c->cap * 8) + align256((size_t)q * 4));
+  {
     LaunchScope ls(K_CTX, s);
-    const int64_t threads = (int64_t)n_valid * q * 32;
-    ctx_score_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(
-        c->keys, queries, q, c->d, c->cap, lo, n_valid, delta, pool);
+    const int64_t want = ((int64_t)q * c->cap * 32 + 255) / 256;
+    const int64_t floor_q = ((int64_t)q * 32 + 255) / 256;  // at least one warp per query
+    const int64_t blocks = std::max(floor_q, std::min<int64_t>(want, (int64_t)sm_count() * 16));
+    ctx_score_kernel<<<(unsigned)blocks, 256, 0, s>>>(c->keys, queries, q, c->d, c->cap, c->m,
+                                                      c->count, delta, pool, counts);
     sense_status st = cuda_check(cudaGetLastError(), "launch ctx score");
     if (st != SENSE_OK) return st;
   }
-  sense_status st = launch_merge_short(pool, nullptr, n_valid, q, k, out_scores, rel, status, s);
+  sense_status st = launch_merge_short(pool, counts, c->cap, q, k, out_scores, rel, status, s);
   if (st != SENSE_OK) return st;
   LaunchScope ls(K_CTX, s);
   ctx_spans_kernel<<<(unsigned)(((int64_t)q * k + 255) / 256), 256, 0, s>>>(
-      rel, q, k, lo, c->cap, c->m, c->tokens, out_pos, out_spans);
+      rel, q, k, c->count, c->cap, c->m, c->tokens, out_pos, out_spans);
   return cuda_check(cudaGetLastError(), "launch ctx spans");
 }
 

@@ -128,3 +128,79 @@ def test_hybrid_drafts_match_oracle(S, q, ks, kd, keep, anchored, force):
     want = X.hybrid_drafts(s_sc, sp_h[s_idx], d_sc if kd else np.zeros((q, 0)),
                            d_sp if kd else np.zeros((q, 0, m), np.int32), anchor, keep, force)
     np.testing.assert_array_equal(host(got), want)
+
+
+def _path_case(rng, d, n_nodes, k, m):
+    root = synth.gaussian_rows_f32(1, d, seed=int(rng.integers(1 << 30))).to(torch.bfloat16)[0]
+    nodes = synth.gaussian_rows_f32(n_nodes, d, seed=int(rng.integers(1 << 30))).to(torch.bfloat16)
+    gamma = rng.integers(0, n_nodes, (k, m)).astype(np.int32)
+    accepted = rng.integers(0, 300, m).astype(np.int32)
+    return root, nodes, gamma, accepted
+
+
+@cuda
+def test_ctx_append_path_matches_oracle(S):
+    """R.Update of verified steps on the device: the appended history is the
+    root state, then the states of the accepted path's nodes (through
+    Gamma), with the accepted tokens; n_accept = 0 appends nothing."""
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(21)
+    d, m, cap, k, n_nodes = 256, 5, 64, 4, 20
+    pre_h = synth.gaussian_rows_f32(10, d, seed=77).to(torch.bfloat16)
+    pre_t = rng.integers(0, 300, 10).astype(np.int32)
+    ctx = S.sense_ctx_create(cap, d, m)
+    S.sense_ctx_append(ctx, pre_h.to(dev), torch.from_numpy(pre_t).to(dev))
+    hist_h, hist_t = [bits(pre_h)], [pre_t]
+    qs = synth.gaussian_rows_f32(2, d, seed=78).to(torch.bfloat16)
+    for step, (i_star, n_acc) in enumerate([(2, 3), (0, 0), (3, 5), (1, 1), (2, 5)] * 4):
+        root, nodes, gamma, acc = _path_case(rng, d, n_nodes, k, m)
+        S.sense_ctx_append_path(ctx, root.to(dev), nodes.to(dev), torch.from_numpy(gamma).to(dev),
+                                torch.tensor([i_star], dtype=torch.int32, device=dev),
+                                torch.tensor([n_acc], dtype=torch.int32, device=dev),
+                                torch.from_numpy(acc).to(dev))
+        rows = [bits(root[None])[0]] + [bits(nodes[gamma[i_star, j - 1]][None])[0]
+                                        for j in range(1, n_acc)]
+        if n_acc:
+            hist_h.append(np.stack(rows))
+            hist_t.append(acc[:n_acc])
+        got = S.sense_ctx_search(ctx, qs.to(dev), 12, delta=0.1)
+        torch.cuda.synchronize()
+        assert S.sense_device_status(clear=True) == 0
+        hh, ht = np.concatenate(hist_h), np.concatenate(hist_t)
+        assert ctx.count == len(ht)
+        _check_search(got, hh, ht, cap, m, bits(qs), 12, 0.1)
+    ctx.close()
+
+
+@cuda
+def test_ctx_step_replays_as_cuda_graph(S):
+    """The device-side counter lets (append path, search) be captured once
+    and replayed: each replay appends the accepted path again."""
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(5)
+    d, m, cap, k, n_nodes = 128, 4, 32, 3, 12
+    root, nodes, gamma, acc = _path_case(rng, d, n_nodes, k, m)
+    args = (root.to(dev), nodes.to(dev), torch.from_numpy(gamma).to(dev),
+            torch.tensor([1], dtype=torch.int32, device=dev),
+            torch.tensor([4], dtype=torch.int32, device=dev), torch.from_numpy(acc).to(dev))
+    qs = synth.gaussian_rows_f32(2, d, seed=9).to(torch.bfloat16).to(dev)
+    ctx = S.sense_ctx_create(cap, d, m)
+    out = S.sense_ctx_search(ctx, qs, 6)  # outputs and workspace allocated before capture
+    ws = S.alloc_workspace(S.lib().sense_ctx_search_workspace_bytes(
+        __import__("ctypes").c_void_p(ctx.handle), 2, 6))
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        S.sense_ctx_append_path(ctx, *args)
+        S.sense_ctx_search(ctx, qs, 6, outs=out, workspace=ws)
+    ctx.reset()
+    rows = np.stack([bits(root[None])[0]] + [bits(nodes[gamma[1, j - 1]][None])[0]
+                                             for j in range(1, 4)])
+    for rep in range(1, 4):
+        g.replay()
+        torch.cuda.synchronize()
+        assert ctx.count == 4 * rep
+        hh = np.concatenate([rows] * rep)
+        ht = np.concatenate([acc[:4]] * rep)
+        _check_search(out, hh, ht, cap, m, bits(qs.cpu()), 6, 0.0)
+    ctx.close()
