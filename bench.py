@@ -181,13 +181,35 @@ class Pipeline:
             S.sense_ivf_search(a["index"], self.qproj, cfg["k"], a["nprobe"], self.scores,
                                self.idx, workspace=self.ws)
 
+    def use_dynamic(self, ctx, kd, delta, dev):
+        """Hybrid retrieval (Alg. 2): the dynamic buffer is searched beside the
+        static store, the union is reranked with the previous step's anchor,
+        and the accepted path is appended after the gate (Alg. 1 R.Update)."""
+        q = self.cfg["q"]
+        self.dyn = {"ctx": ctx, "kd": kd, "delta": delta, "outs": {},
+                    "ws": self.S.alloc_workspace(self.S.lib().sense_ctx_search_workspace_bytes(
+                        __import__("ctypes").c_void_p(ctx.handle), q, kd), dev),
+                    "anchor": torch.zeros(q, dtype=torch.int32, device=dev)}
+
     def step(self, query, gate_in):
         S, cfg = self.S, self.cfg
         self.retrieve(query)
-        S.sense_gather_drafts(self.ds, self.idx, out=self.drafts)
+        dyn = getattr(self, "dyn", None)
+        if dyn is None:
+            S.sense_gather_drafts(self.ds, self.idx, out=self.drafts)
+        else:
+            S.sense_ctx_search(dyn["ctx"], query, dyn["kd"], dyn["delta"], outs=dyn["outs"],
+                               workspace=dyn["ws"])
+            S.sense_hybrid_drafts(self.ds, self.scores, self.idx, dyn["outs"], dyn["anchor"],
+                                  cfg["k"], True, out=self.drafts)
         S.sense_build_tree(self.drafts, node_cap=cfg["cap"], outs=self.tree)
         root, nodes, hr, hn = gate_in
         S.sense_soft_gate(self.tree, root, nodes, hr, hn, workspace=self.gws, outs=self.gate, **GATE)
+        if dyn is not None:
+            g = self.gate
+            S.sense_ctx_append_path(dyn["ctx"], hr[0], hn[0], self.tree["gamma"][0],
+                                    g["i_star"][:1], g["n_accept"][:1], g["accepted"][0])
+            dyn["anchor"].copy_(g["next_anchor"])  # x~ of the next step
 
 
 class GraphStep:
@@ -361,6 +383,10 @@ def main():
     ap.add_argument("--proj-dim", type=int, default=64)
     ap.add_argument("--graph", action="store_true",
                     help="time CUDA graph replays of the whole step")
+    ap.add_argument("--dynamic", type=int, default=0, metavar="CAPACITY",
+                    help="add the dynamic context buffer of this many positions (q = 1)")
+    ap.add_argument("--dyn-k", type=int, default=16)
+    ap.add_argument("--delta", type=float, default=0.05)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     cfg = dict(WORKLOADS[args.workload])
@@ -402,6 +428,23 @@ def main():
         ann = build_ann(S, keys, args.retrieval, args.nlist, args.nprobe, args.pq_m,
                         args.proj_dim, dev, seed=rank)
         pipe.use_ann(ann, dev)
+    dyn_info = None
+    if args.dynamic:
+        if cfg["q"] != 1:
+            raise SystemExit("--dynamic models one sequence: use a workload with q = 1")
+        # prefill: the buffer starts full of the sequence's own states (store
+        # keys of random clusters stand in for them) and Zipf tokens
+        ctx = S.sense_ctx_create(args.dynamic, cfg["d"], cfg["m"])
+        g = torch.Generator(device=dev).manual_seed(rank + 11)
+        pre = keys[torch.randint(0, cfg["n"], (args.dynamic,), generator=g, device=dev)]
+        pre_tok = synth.spans_zipf(args.dynamic, 1, cfg["vocab"], 1.1, seed=rank + 12,
+                                   device=dev)[:, 0].contiguous()
+        S.sense_ctx_append(ctx, pre.contiguous(), pre_tok)
+        del pre
+        pipe.use_dynamic(ctx, args.dyn_k, args.delta, dev)
+        dyn_info = {"capacity": args.dynamic, "prefill": args.dynamic, "k_dynamic": args.dyn_k,
+                    "delta": args.delta, "n_keep": cfg["k"], "anchor": "previous step's x~",
+                    "update": "accepted path appended every step (device-side count)"}
 
     for it in range(args.warmup):
         pipe.step(queries[it % nq], gate_sets[it % n_sets])
@@ -597,8 +640,10 @@ def main():
 
     base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        if ann is None:
+        if ann is None and not args.dynamic:
             base = cpu_baseline(cfg, keys, spans, queries, gate_sets)
+        elif args.dynamic:
+            base = {"value": None, "skipped": "the oracle baseline times the static path only"}
         else:
             base = {"value": None, "skipped": "the oracle's index build over the full store "
                     "(fp32 loops in numpy) does not fit a bounded CPU sample"}
@@ -611,12 +656,14 @@ def main():
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded clustered unit-norm keys, Zipf spans, N(0,9) logits)",
             "config": {"workload": args.workload, "retrieval": args.retrieval,
+                       "dynamic_capacity": args.dynamic,
                        **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab", "cap", "clusters")},
                        "key_bytes": n * d * 2,
                        "l2": f"inputs larger than L2: the {n * d * 2 / 1e9:.1f} GB store is "
                              "streamed every step",
                        "parallelism": f"replicas x{world}"},
             "retrieval": retrieval,
+            "dynamic": dyn_info,
             "launch": "cuda_graph" if graph is not None else "eager",
             "launch_note": graph_note,
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,

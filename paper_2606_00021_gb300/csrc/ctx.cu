@@ -351,9 +351,12 @@ sense_status sense_ctx_append(sense_ctx* c, const uint16_t* hidden, const int32_
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int first = t > c->cap ? t - c->cap : 0;  // earlier rows would be overwritten
   const int64_t warps = t - first;
+  {
+    LaunchScope ls(K_CTX, s);
+    ctx_append_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(
+        hidden, tokens, t, first, c->count, c->cap, c->d, c->keys, c->tokens);
+  }
   LaunchScope ls(K_CTX, s);
-  ctx_append_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(
-      hidden, tokens, t, first, c->count, c->cap, c->d, c->keys, c->tokens);
   ctx_bump_kernel<<<1, 1, 0, s>>>(c->count, t, nullptr, 0);
   return cuda_check(cudaGetLastError(), "launch ctx append");
 }
@@ -373,10 +376,13 @@ sense_status sense_ctx_append_path(sense_ctx* c, const uint16_t* root_hidden,
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  {
+    LaunchScope ls(K_CTX, s);
+    ctx_append_path_kernel<<<(unsigned)((c->m * 32 + 255) / 256), 256, 0, s>>>(
+        root_hidden, node_hidden, n_nodes, gamma, k, c->m, i_star, n_accept, accepted, c->count,
+        c->cap, c->d, c->keys, c->tokens, status);
+  }
   LaunchScope ls(K_CTX, s);
-  ctx_append_path_kernel<<<(unsigned)((c->m * 32 + 255) / 256), 256, 0, s>>>(
-      root_hidden, node_hidden, n_nodes, gamma, k, c->m, i_star, n_accept, accepted, c->count,
-      c->cap, c->d, c->keys, c->tokens, status);
   ctx_bump_kernel<<<1, 1, 0, s>>>(c->count, 0, n_accept, c->m);
   return cuda_check(cudaGetLastError(), "launch ctx append path");
 }
