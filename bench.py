@@ -235,8 +235,9 @@ class GraphStep:
 
 def build_ann(S, keys, kind, nlist, nprobe, pq_m, v, dev, seed=0):
     """Index construction for the approximate path (outside the timed region):
-    the PCA basis is fitted offline on a 65,536-key sample (eigenvectors of
-    its covariance, as the paper's setup fits PCA with a library); keys are
+    the PCA basis is fitted offline on a 65,536-key sample (top eigenvectors
+    of its covariance, by scipy on the host, as the paper's setup fits PCA
+    with a library); keys are
     projected and normalised, the coarse quantizer is trained by spherical
     k-means (10 rounds on 64 x nlist keys), PQ codebooks by k-means on the
     residual sub-vectors (10 rounds), and the index is built - all but the
@@ -246,10 +247,13 @@ def build_ann(S, keys, kind, nlist, nprobe, pq_m, v, dev, seed=0):
     sample = keys[torch.randint(0, n, (min(n, 65536),), generator=g, device=dev)].float()
     mean = sample.mean(0)
     xc = sample - mean
-    evals, evecs = torch.linalg.eigh((xc.T @ xc / xc.shape[0]).double())
-    basis = evecs[:, -v:].flip(1).T.float().contiguous()
+    cov = (xc.T @ xc / xc.shape[0]).double().cpu().numpy()
+    del sample, xc
+    import scipy.linalg
+    _, evecs = scipy.linalg.eigh(cov, subset_by_index=[d - v, d - 1])
+    basis = torch.from_numpy(np.ascontiguousarray(evecs[:, ::-1].T)).float().to(dev).contiguous()
     mean = mean.contiguous()
-    del sample, xc, evecs
+    del cov, evecs
     t0 = time.perf_counter()
     kp = torch.empty(n, v, dtype=torch.float32, device=dev)
     for lo in range(0, n, 1 << 20):

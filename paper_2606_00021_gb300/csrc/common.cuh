@@ -104,4 +104,27 @@ __device__ __forceinline__ uint32_t warp_append(uint32_t* counter, bool want) {
   return base + __popc(m & ((1u << lane) - 1u));
 }
 
+// Sorted list of KPL * 32 candidate keys spread over a warp: position
+// r = s * 32 + lane lives in v[s] of that lane, larger keys first.  Inserts
+// the warp-uniform key c (distinct from every key in the list); the last
+// entry drops out.
+template <int KPL>
+__device__ __forceinline__ void list_insert(uint64_t (&v)[KPL], uint64_t c, int lane) {
+  int p = 0;  // keys ahead of c (all keys are distinct)
+#pragma unroll
+  for (int s = 0; s < KPL; ++s) p += __popc(__ballot_sync(0xffffffffu, v[s] > c));
+  uint64_t up[KPL], last[KPL];
+#pragma unroll
+  for (int s = 0; s < KPL; ++s) {
+    up[s] = __shfl_up_sync(0xffffffffu, v[s], 1);
+    last[s] = __shfl_sync(0xffffffffu, v[s], 31);
+  }
+#pragma unroll
+  for (int s = 0; s < KPL; ++s) {
+    const int r = s * 32 + lane;
+    const uint64_t prev = (lane == 0) ? (s > 0 ? last[s > 0 ? s - 1 : 0] : 0ull) : up[s];
+    v[s] = (r < p) ? v[s] : (r == p ? c : prev);
+  }
+}
+
 }  // namespace sense

@@ -162,25 +162,22 @@ ctx_score_kernel(const uint16_t* __restrict__ keys, const uint16_t* __restrict__
   }
 }
 
+// One thread per (slot, span token).
 __global__ void ctx_spans_kernel(const int32_t* __restrict__ rel, int q, int k,
                                  const int64_t* __restrict__ count, int cap, int m,
                                  const int32_t* __restrict__ ring, int64_t* __restrict__ out_pos,
                                  int32_t* __restrict__ out_spans) {
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= (int64_t)q * k) return;
+  if (t >= (int64_t)q * k * m) return;
+  const int64_t slot = t / m;
+  const int j = (int)(t - slot * m);
   int64_t lo;
   int n_valid;
   ctx_range_dev(*count, cap, m, &lo, &n_valid);
-  const int e = rel[t];
-  int32_t* sp = out_spans + t * m;
-  if (e < 0) {
-    out_pos[t] = -1;
-    for (int j = 0; j < m; ++j) sp[j] = -1;
-    return;
-  }
+  const int e = rel[slot];
   const int64_t p = lo + e;
-  out_pos[t] = p;
-  for (int j = 0; j < m; ++j) sp[j] = ring[(p + j) % cap];
+  if (j == 0) out_pos[slot] = e < 0 ? -1 : p;
+  out_spans[t] = e < 0 ? -1 : ring[(p + j) % cap];
 }
 
 // One block (1024 threads) per query.  Union index u < ks: static rank u;
@@ -427,7 +424,7 @@ sense_status sense_ctx_search(const sense_ctx* c, const uint16_t* queries, int32
   sense_status st = launch_merge_short(pool, counts, c->cap, q, k, out_scores, rel, status, s);
   if (st != SENSE_OK) return st;
   LaunchScope ls(K_CTX, s);
-  ctx_spans_kernel<<<(unsigned)(((int64_t)q * k + 255) / 256), 256, 0, s>>>(
+  ctx_spans_kernel<<<(unsigned)(((int64_t)q * k * c->m + 255) / 256), 256, 0, s>>>(
       rel, q, k, c->count, c->cap, c->m, c->tokens, out_pos, out_spans);
   return cuda_check(cudaGetLastError(), "launch ctx spans");
 }

@@ -16,7 +16,8 @@
 //  - k-means sums are 2^-31 fixed-point integers (order-free atomics),
 //    divided in fp64.
 // Kernels:
-//  project_rows_kernel   one warp per (row, output): query batches
+//  project_rows_kernel   row staged in shared memory, one warp per output:
+//                        query batches
 //  project_tile_kernel   16 rows x 32 outputs per block, 16 warps, each lane
 //                        holding 4 x 8 partial sums: key stores
 //  normalize_rows_kernel one thread per row
@@ -89,39 +90,47 @@ __device__ __forceinline__ float4 load_x4(const uint16_t* xr, const float* mu, i
   return x;
 }
 
+// Block (output group, row): the centred row is staged in shared memory once;
+// warp w computes output 8 * blockIdx.x + w, streaming its row of W.
 __global__ void __launch_bounds__(256)
 project_rows_kernel(const uint16_t* __restrict__ x, int64_t n, int d,
                     const float* __restrict__ w, int v, const float* __restrict__ mu,
                     float* __restrict__ out) {
-  const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  extern __shared__ __align__(16) float sx[];  // [d]
+  const int64_t row = blockIdx.y;
   const int lane = threadIdx.x & 31;
-  if (gw >= n * v) return;  // warp-uniform
-  const int64_t row = gw / v;
-  const int o = (int)(gw - row * v);
   const uint16_t* xr = x + row * d;
+  for (int j = 4 * threadIdx.x; j < d; j += 4 * blockDim.x)
+    *reinterpret_cast<float4*>(sx + j) = load_x4(xr, mu, j);
+  __syncthreads();
+  const int o = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (o >= v) return;  // warp-uniform
   const float* wr = w + (int64_t)o * d;
   float acc = 0.0f;
-  // 8 column groups in flight per lane, consumed in ascending order
+  // full rounds of 8 column groups per lane (W loads issued together, then
+  // consumed in ascending order), then the remaining groups one by one
   constexpr int U = 8;
-  for (int j0 = 4 * lane; j0 < d; j0 += 128 * U) {
-    float4 xv[U], wv[U];
+  int j0 = 4 * lane;
+  for (; j0 + 128 * (U - 1) < d; j0 += 128 * U) {
+    float4 wv[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) wv[u] = *reinterpret_cast<const float4*>(wr + j0 + 128 * u);
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int j = j0 + 128 * u;
-      if (j < d) {
-        xv[u] = load_x4(xr, mu, j);
-        wv[u] = *reinterpret_cast<const float4*>(wr + j);
-      }
+      const float4 xv = *reinterpret_cast<const float4*>(sx + j0 + 128 * u);
+      acc = madd(acc, xv.x, wv[u].x);
+      acc = madd(acc, xv.y, wv[u].y);
+      acc = madd(acc, xv.z, wv[u].z);
+      acc = madd(acc, xv.w, wv[u].w);
     }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (j0 + 128 * u < d) {
-        acc = madd(acc, xv[u].x, wv[u].x);
-        acc = madd(acc, xv[u].y, wv[u].y);
-        acc = madd(acc, xv[u].z, wv[u].z);
-        acc = madd(acc, xv[u].w, wv[u].w);
-      }
-    }
+  }
+  for (; j0 < d; j0 += 128) {
+    const float4 xv = *reinterpret_cast<const float4*>(sx + j0);
+    const float4 wv = *reinterpret_cast<const float4*>(wr + j0);
+    acc = madd(acc, xv.x, wv.x);
+    acc = madd(acc, xv.y, wv.y);
+    acc = madd(acc, xv.z, wv.z);
+    acc = madd(acc, xv.w, wv.w);
   }
   acc = butterfly(acc);
   if (lane == 0) out[row * v + o] = acc;
@@ -203,14 +212,29 @@ project_tile_kernel(const uint16_t* __restrict__ x, int64_t n, int d,
   }
 }
 
-__global__ void normalize_rows_kernel(float* __restrict__ y, int64_t n, int v) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n) return;
+// One warp per row (v <= 128): the lanes load the row, every lane forms the
+// sum of squares in index order from shuffled values, then scales its part.
+__global__ void __launch_bounds__(256)
+normalize_rows_kernel(float* __restrict__ y, int64_t n, int v) {
+  const int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (i >= n) return;  // warp-uniform
   float* r = y + i * v;
+  float part[4];
+#pragma unroll
+  for (int t = 0; t < 4; ++t) part[t] = (32 * t + lane < v) ? r[32 * t + lane] : 0.0f;
   float s = 0.0f;
-  for (int o = 0; o < v; ++o) s = madd(s, r[o], r[o]);
+#pragma unroll
+  for (int t = 0; t < 4; ++t) {
+    for (int l = 0; l < 32 && 32 * t + l < v; ++l) {
+      const float e = __shfl_sync(0xffffffffu, part[t], l);
+      s = madd(s, e, e);
+    }
+  }
   const float nrm = __fsqrt_rn(s);
-  for (int o = 0; o < v; ++o) r[o] = nrm > 0.0f ? __fdiv_rn(r[o], nrm) : 0.0f;
+#pragma unroll
+  for (int t = 0; t < 4; ++t)
+    if (32 * t + lane < v) r[32 * t + lane] = nrm > 0.0f ? __fdiv_rn(part[t], nrm) : 0.0f;
 }
 
 // ---------------------------------------------------------------------------
@@ -520,19 +544,39 @@ __global__ void residual_kernel(const float* __restrict__ x, int64_t n, int v,
 }
 
 // ---------------------------------------------------------------------------
-// search: list scan
+// search: lookup tables and list scan
 // ---------------------------------------------------------------------------
+
+// PQ lookup table of each query: lut[qi][m][b] = <q_m, B_m[b]> (dsub terms in
+// index order).  One block per query; shared by all of its probe blocks.
+__global__ void __launch_bounds__(256)
+pq_lut_kernel(const float* __restrict__ queries, int v, const float* __restrict__ cb, int pq_m,
+              int dsub, float* __restrict__ lut) {
+  __shared__ float sq[128];
+  const int qi = blockIdx.x;
+  for (int j = threadIdx.x; j < v; j += blockDim.x) sq[j] = queries[(int64_t)qi * v + j];
+  __syncthreads();
+  float* out = lut + (int64_t)qi * pq_m * 256;
+  for (int e = threadIdx.x; e < pq_m * 256; e += blockDim.x) {
+    const int m = e >> 8;
+    const float* bb = cb + (int64_t)e * dsub;
+    float s = 0.0f;
+    for (int j = 0; j < dsub; ++j) s = madd(s, sq[m * dsub + j], bb[j]);
+    out[e] = s;
+  }
+}
 
 constexpr int kScanThreads = 256;
 constexpr int kFlatStride = 132;  // padded row stride (floats) of staged vectors, v <= 128
 
 // One block per (probe p, query qi).  Flat: each thread scores one staged
-// vector (<q, x> in index order).  PQ: the block builds the query's lookup
-// table LUT[m][b] = <q_m, B_m[b]> in shared memory; each thread reads one
-// code row and sums coarse + LUT[0][c_0] + ... + LUT[pq_m-1][c_{pq_m-1}].
+// vector (<q, x> in index order).  PQ: the block stages the query's lookup
+// table in shared memory; each thread reads one code row and sums
+// coarse + LUT[0][c_0] + ... + LUT[pq_m-1][c_{pq_m-1}].
 // Candidates go to the query's pool (warp-aggregated append).
 __global__ void __launch_bounds__(kScanThreads)
-ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries, int nprobe,
+ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries,
+                const float* __restrict__ lut, int nprobe,
                 const float* __restrict__ probe_score, const int32_t* __restrict__ probe_cell,
                 uint64_t* __restrict__ pool, uint32_t* __restrict__ counts, int64_t pool_cap,
                 uint32_t* status) {
@@ -553,14 +597,9 @@ ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries, int nprob
   const int64_t lo = ix.offsets[cell], hi = ix.offsets[cell + 1];
   uint64_t* dst = pool + (int64_t)qi * pool_cap;
   if (ix.pq_m > 0) {
-    const int dsub = ix.dsub;
-    for (int e = threadIdx.x; e < ix.pq_m * 256; e += blockDim.x) {
-      const int m = e >> 8;
-      const float* bb = ix.codebooks + (int64_t)e * dsub;
-      float s = 0.0f;
-      for (int j = 0; j < dsub; ++j) s = madd(s, sq[m * dsub + j], bb[j]);
-      stage[e] = s;
-    }
+    const float4* src = reinterpret_cast<const float4*>(lut + (int64_t)qi * ix.pq_m * 256);
+    for (int e = threadIdx.x; e < ix.pq_m * 64; e += blockDim.x)
+      reinterpret_cast<float4*>(stage)[e] = src[e];
     __syncthreads();
     for (int64_t s0 = lo; s0 < hi; s0 += blockDim.x) {
       const int64_t slot = s0 + threadIdx.x;
@@ -618,7 +657,7 @@ size_t scan_smem_bytes(const sense_ivf* ix) {
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct SearchPlan {
-  size_t off_coarse, off_pscore, off_pcell, off_counts, off_pool, total;
+  size_t off_coarse, off_pscore, off_pcell, off_counts, off_lut, off_pool, total;
   int64_t pool_cap;
 };
 
@@ -633,6 +672,8 @@ SearchPlan search_plan(const sense_ivf* ix, int q, int nprobe) {
   o = align256(o + (size_t)q * nprobe * 4);
   p.off_counts = o;
   o = align256(o + (size_t)q * 4);
+  p.off_lut = o;
+  o = align256(o + (size_t)q * ix->pq_m * 256 * 4);
   p.pool_cap = std::max<int64_t>(1, (int64_t)nprobe * ix->max_list);
   p.off_pool = o;
   o = align256(o + (size_t)q * p.pool_cap * 8);
@@ -683,10 +724,9 @@ sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float*
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   {
     LaunchScope ls(K_PROJECT, s);
-    if (n * v <= 16384) {
-      const int64_t threads = n * v * 32;
-      project_rows_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(x, n, d, basis, v, mean,
-                                                                            out);
+    if (n * v <= 16384 && n <= 65535 && d <= 12288) {
+      const dim3 grid((unsigned)((v + 7) / 8), (unsigned)n);
+      project_rows_kernel<<<grid, 256, (size_t)d * 4, s>>>(x, n, d, basis, v, mean, out);
     } else {
       const dim3 grid((unsigned)((n + kPtRows - 1) / kPtRows), (unsigned)((v + kPtOuts - 1) / kPtOuts));
       project_tile_kernel<<<grid, 512, 0, s>>>(x, n, d, basis, v, mean, out);
@@ -696,7 +736,7 @@ sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float*
   }
   if (flags & SENSE_PROJECT_NORMALIZE) {
     LaunchScope ls(K_PROJECT, s);
-    normalize_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(out, n, v);
+    normalize_rows_kernel<<<(unsigned)((n * 32 + 255) / 256), 256, 0, s>>>(out, n, v);
     return cuda_check(cudaGetLastError(), "launch normalize rows");
   }
   return SENSE_OK;
@@ -929,6 +969,7 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
   auto* pcell = out_probes ? out_probes : reinterpret_cast<int32_t*>(ws + p.off_pcell);
   auto* counts = reinterpret_cast<uint32_t*>(ws + p.off_counts);
   auto* pool = reinterpret_cast<uint64_t*>(ws + p.off_pool);
+  auto* lut = reinterpret_cast<float*>(ws + p.off_lut);
   sense_status st = cuda_check(cudaMemsetAsync(counts, 0, (size_t)q * 4, s), "clear counts");
   if (st != SENSE_OK) return st;
   {
@@ -936,6 +977,12 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
     // cells as rows, queries staged: pool row qi holds key(<q_qi, c>, c)
     st = launch_assign_mode<ALL_IP>(ix->centroids, ix->nlist, ix->v, ix->v, queries, q, nullptr,
                                     coarse, s);
+    if (st != SENSE_OK) return st;
+  }
+  if (ix->pq_m > 0) {
+    LaunchScope ls(K_IVF_COARSE, s);
+    pq_lut_kernel<<<q, 256, 0, s>>>(queries, ix->v, ix->codebooks, ix->pq_m, ix->dsub, lut);
+    st = cuda_check(cudaGetLastError(), "launch pq lut");
     if (st != SENSE_OK) return st;
   }
   st = launch_merge(coarse, nullptr, ix->nlist, q, nprobe, pscore, pcell, status, s);
@@ -946,8 +993,9 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
                                          (int)smem), "smem attribute");
     if (st != SENSE_OK) return st;
     LaunchScope ls(K_IVF_SCAN, s);
-    ivf_scan_kernel<<<dim3(nprobe, q), kScanThreads, smem, s>>>(*ix, queries, nprobe, pscore, pcell,
-                                                                pool, counts, p.pool_cap, status);
+    ivf_scan_kernel<<<dim3(nprobe, q), kScanThreads, smem, s>>>(*ix, queries, lut, nprobe, pscore,
+                                                                pcell, pool, counts, p.pool_cap,
+                                                                status);
     st = cuda_check(cudaGetLastError(), "launch ivf scan");
     if (st != SENSE_OK) return st;
   }

@@ -115,27 +115,6 @@ scan_gemv_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
   }
 }
 
-// Sorted list of KPL * 32 candidate keys spread over a warp: position
-// r = s * 32 + lane lives in v[s] of that lane, larger keys first.
-template <int KPL>
-__device__ __forceinline__ void list_insert(uint64_t (&v)[KPL], uint64_t c, int lane) {
-  int p = 0;  // keys ahead of c (all keys are distinct)
-#pragma unroll
-  for (int s = 0; s < KPL; ++s) p += __popc(__ballot_sync(0xffffffffu, v[s] > c));
-  uint64_t up[KPL], last[KPL];
-#pragma unroll
-  for (int s = 0; s < KPL; ++s) {
-    up[s] = __shfl_up_sync(0xffffffffu, v[s], 1);
-    last[s] = __shfl_sync(0xffffffffu, v[s], 31);
-  }
-#pragma unroll
-  for (int s = 0; s < KPL; ++s) {
-    const int r = s * 32 + lane;
-    const uint64_t prev = (lane == 0) ? (s > 0 ? last[s > 0 ? s - 1 : 0] : 0ull) : up[s];
-    v[s] = (r < p) ? v[s] : (r == p ? c : prev);
-  }
-}
-
 // Single pass: the GEMV scan of scan_gemv_kernel with the top-k kept in
 // per-warp register lists instead of a threshold filter.  Scores are
 // warp-uniform after the reduction, so list updates never diverge.  At the
