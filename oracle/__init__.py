@@ -14,5 +14,6 @@ from .sense_oracle import (  # noqa: F401
     scores,
     soft_gate,
     topk,
+    tree_attention,
     tree_mask_full,
 )

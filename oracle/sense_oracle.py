@@ -21,6 +21,8 @@ for floating point, following the step order and notation of the paper:
   loose_trie_alg3      App. C.3 Alg. 3 restated step by step (uncapped)
   mask_from_bits,      App. C.6 Eq. 20 (additive tree attention mask over a
   tree_mask_full        static KV cache) from Alg. 3's mask M
+  tree_attention       the masked attention of the verify forward (Alg. 1)
+                        under that mask
   soft_gate            §3.3 Eqs. 11-19 and App. C.4 Alg. 4
 
 Readings where the paper is silent or ambiguous are stated at each function.
@@ -362,6 +364,32 @@ def tree_mask_full(M: np.ndarray, m: int, cache_len: int, rows=None) -> np.ndarr
         for c in range(big_l):
             if big_m[i, c] == 1:
                 out[i, m + c] = 0.0
+    return out
+
+
+def tree_attention(q_bits: np.ndarray, k_bits: np.ndarray, v_bits: np.ndarray, m: int,
+                   M: np.ndarray, scale: float) -> np.ndarray:
+    """Tree-masked attention of the L draft tokens over a static KV cache, fp64.
+
+    The verify forward of Alg. 1 (Forward(T, M_full, K)) scores every draft
+    token against the cache under the additive mask M_full of Eq. 20:
+    O[h] = softmax(scale * Q[h] K[h]^T + M_full) V[h] over the first m + L
+    cache positions.  q_bits [H, L, D], k_bits / v_bits [H, >= m + L, D]
+    (bf16 bits); M [L, L] is Alg. 3's 0/1 mask.  Returns [H, L, D].
+    """
+    qf = bf16_bits_to_f64(np.asarray(q_bits))
+    kf = bf16_bits_to_f64(np.asarray(k_bits))
+    vf = bf16_bits_to_f64(np.asarray(v_bits))
+    big_l = qf.shape[1]
+    n = m + big_l
+    full = tree_mask_full(M, m, n)
+    out = np.empty_like(qf)
+    for h in range(qf.shape[0]):
+        s = scale * (qf[h] @ kf[h, :n].T) + full
+        s = s - s.max(axis=1, keepdims=True)
+        p = np.exp(s)
+        p /= p.sum(axis=1, keepdims=True)
+        out[h] = p @ vf[h, :n]
     return out
 
 

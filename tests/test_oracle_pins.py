@@ -506,3 +506,40 @@ def test_tree_mask_full_attention_equals_per_path_causal(seed):
         ref = torch.nn.functional.scaled_dot_product_attention(
             qs[None], kc[cols][None], vc[cols][None], is_causal=True)[0, -1]
         torch.testing.assert_close(tree_out[i], ref, rtol=1e-12, atol=1e-12)
+
+
+def _bf(x):
+    return _bits(torch.from_numpy(np.asarray(x, np.float32)).to(torch.bfloat16))
+
+
+def test_tree_attention_matches_sdpa_with_float_mask():
+    rng = np.random.default_rng(31)
+    spans = _rand_spans(rng, 8, 5, 3)
+    tr = O.loose_trie(spans, mask_bits=True)
+    L = int(tr["num_nodes"][0])
+    M = O.mask_from_bits(tr["mask_bits"][0], L)
+    H, D, m = 3, 16, 7
+    q = _bf(rng.standard_normal((H, L, D)))
+    k = _bf(rng.standard_normal((H, m + L + 5, D)))
+    v = _bf(rng.standard_normal((H, m + L + 5, D)))
+    got = O.tree_attention(q, k, v, m, M, 0.25)
+    qt, kt, vt = (torch.from_numpy(O.bf16_bits_to_f64(a)) for a in (q, k, v))
+    full = torch.from_numpy(O.tree_mask_full(M, m, m + L))
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        qt, kt[:, :m + L], vt[:, :m + L], attn_mask=full, scale=0.25)
+    np.testing.assert_allclose(got, ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_tree_attention_chain_is_causal_attention():
+    rng = np.random.default_rng(32)
+    L, m, H, D = 6, 4, 2, 8
+    M = np.tril(np.ones((L, L), dtype=np.int64))
+    q = _bf(rng.standard_normal((H, L, D)))
+    k = _bf(rng.standard_normal((H, m + L, D)))
+    v = _bf(rng.standard_normal((H, m + L, D)))
+    got = O.tree_attention(q, k, v, m, M, 1 / np.sqrt(D))
+    qt, kt, vt = (torch.from_numpy(O.bf16_bits_to_f64(a)) for a in (q, k, v))
+    # causal attention over the whole sequence; the last L rows are the tree
+    qfull = torch.cat([torch.zeros(H, m, D, dtype=torch.float64), qt], dim=1)
+    ref = torch.nn.functional.scaled_dot_product_attention(qfull, kt, vt, is_causal=True)[:, m:]
+    np.testing.assert_allclose(got, ref.numpy(), rtol=1e-12, atol=1e-12)
