@@ -461,6 +461,36 @@ sense_status sense_tree_mask_full(const uint32_t* mask_bits, const int32_t* num_
                                   int32_t cap, const int32_t* prefix_len, int32_t cache_len,
                                   float* out, sense_stream_t stream);
 
+/*
+ * Tree-masked attention of the verify forward (Alg. 1: Forward(T, M_full,
+ * K)) for one sequence, on tcgen05 tensor cores: per head h,
+ *   out[h] = softmax(scale * Q[h] K[h]^T + M_full) V[h]
+ * over the first prefix_len + L cache positions, where the L draft tokens
+ * sit at positions prefix_len .. prefix_len + L - 1 and M_full is the mask
+ * of Eq. 20 built on the fly from Alg. 3's ancestor bits (see
+ * sense_tree_mask_full).
+ *   q [heads, L, 128] bf16 (the draft tokens' queries);
+ *   k_cache [heads, capacity, 128] bf16; vt_cache [heads, 128, capacity]
+ *   bf16 (V stored transposed per head, so that both products read K-major
+ *   tiles); positions past prefix_len + L are never used;
+ *   mask_bits: L rows of mask_words uint32 (row n, bit b: node b is an
+ *   ancestor of n or n itself), e.g. one query's rows of sense_build_tree's
+ *   SENSE_TREE_MASK_BITS output;
+ *   out [heads, L, 128] f32.  Probabilities are rounded to bf16 before the
+ *   product with V (fp32 accumulation throughout).
+ *   workspace: sense_tree_attention_workspace_bytes(heads, L, prefix_len)
+ *   bytes, 256-byte aligned.
+ * Limits: d_head == 128, 1 <= L <= 128, capacity % 128 == 0, prefix_len +
+ * L <= capacity, scale > 0; q, caches and out 16-byte aligned.
+ */
+size_t sense_tree_attention_workspace_bytes(int32_t heads, int32_t L, int32_t prefix_len);
+sense_status sense_tree_attention(const uint16_t* q, const uint16_t* k_cache,
+                                  const uint16_t* vt_cache, int32_t heads, int32_t L,
+                                  int32_t d_head, int32_t capacity, int32_t prefix_len,
+                                  const uint32_t* mask_bits, int32_t mask_words, float scale,
+                                  float* out, void* workspace, size_t workspace_bytes,
+                                  sense_stream_t stream);
+
 /* ---------------------------------------------------------------------- */
 /* a6. Soft-gated evaluation                                                */
 /* ---------------------------------------------------------------------- */

@@ -507,6 +507,32 @@ def sense_hybrid_drafts(ds: Datastore, static_scores: torch.Tensor, static_idx: 
     return out
 
 
+def sense_tree_attention(q: torch.Tensor, k_cache: torch.Tensor, vt_cache: torch.Tensor,
+                         prefix_len: int, mask_bits: torch.Tensor, scale: float,
+                         out: torch.Tensor | None = None, workspace=None,
+                         stream=None) -> torch.Tensor:
+    """Tree-masked attention of the verify forward: q [H, L, 128] bf16,
+    k_cache [H, C, 128] and vt_cache [H, 128, C] bf16, mask_bits [>= L, words]
+    int32 ancestor rows of one tree; returns out [H, L, 128] f32."""
+    _need(q, "q", torch.bfloat16, 3)
+    _need(k_cache, "k_cache", torch.bfloat16, 3)
+    _need(vt_cache, "vt_cache", torch.bfloat16, 3)
+    _need(mask_bits, "mask_bits", torch.int32, 2)
+    heads, L, dh = q.shape
+    cap = k_cache.shape[1]
+    if out is None:
+        out = torch.empty(heads, L, dh, dtype=torch.float32, device=q.device)
+    if workspace is None:
+        workspace = alloc_workspace(
+            lib().sense_tree_attention_workspace_bytes(heads, L, prefix_len), q.device)
+    _check(lib().sense_tree_attention(q.data_ptr(), k_cache.data_ptr(), vt_cache.data_ptr(), heads,
+                                      L, dh, cap, prefix_len, mask_bits.data_ptr(),
+                                      mask_bits.shape[1], C.c_float(scale), out.data_ptr(),
+                                      workspace.data_ptr(), workspace.numel(),
+                                      C.c_void_p(_stream(stream))))
+    return out
+
+
 def sense_soft_gate_workspace_bytes(q: int, cap: int, kappa: int) -> int:
     return int(lib().sense_soft_gate_workspace_bytes(q, cap, kappa))
 

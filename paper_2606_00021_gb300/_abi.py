@@ -53,6 +53,9 @@ SIGNATURES = {
                                  c_p]),
     "sense_hybrid_drafts": (c_i32, [c_p, c_p, c_p, c_i32, c_p, c_p, c_i32, c_i32, c_p, c_i32,
                                     c_u32, c_p, c_p]),
+    "sense_tree_attention_workspace_bytes": (c_size, [c_i32, c_i32, c_i32]),
+    "sense_tree_attention": (c_i32, [c_p, c_p, c_p, c_i32, c_i32, c_i32, c_i32, c_i32, c_p, c_i32,
+                                     C.c_float, c_p, c_p, c_size, c_p]),
     "sense_soft_gate_workspace_bytes": (c_size, [c_i32, c_i32, c_i32]),
     "sense_soft_gate": (c_i32, [c_p, c_p, c_p, c_p, c_i32, c_i32, c_i32, c_i32, c_p, c_p, c_i32,
                                 c_p, c_p, c_i32, C.POINTER(GateParams), c_p, c_p, c_p, c_p, c_p,

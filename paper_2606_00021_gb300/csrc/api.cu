@@ -32,7 +32,7 @@ const char* const kKernelNames[K_COUNT] = {
     "normalize", "scan_gemv", "scan_tc", "threshold", "merge",
     "gather",    "tree",      "gate_rows", "gate_decide", "pad_queries",
     "tree_mask", "project",  "kmeans",    "ivf_build", "ivf_coarse",
-    "ivf_scan",  "ctx"};
+    "ivf_scan",  "ctx",       "tree_attn"};
 
 cudaEvent_t take_event() {
   if (!g_ev_pool.empty()) {

@@ -1,0 +1,496 @@
+// Tree-masked attention of the draft tokens over a static KV cache, on
+// tcgen05 tensor cores (the attention of Alg. 1's verify forward,
+// Forward(T, M_full, K), under the mask M_full of App. C.6 Eq. 20).
+//
+// For one head, the L <= 128 draft tokens attend to the n = m + L cache
+// positions: position j is visible to token i if j < m (committed tokens)
+// or if m <= j < m + L and node j - m is an ancestor of i or i itself
+// (Alg. 3's mask, given as ancestor bit rows).  O = softmax(scale Q K^T +
+// M_full) V.
+//
+// Design (flash-attention over 128-key blocks; one CTA per (head, key split)):
+//  - warp 0 (one lane) loads Q [128 x 128] once and, per block, the K tile
+//    [128 keys x 128] and the V^T tile [128 x 128 keys] with 3-D TMA loads
+//    (128-byte swizzle; keys past n are zero-filled) into a 2-stage ring;
+//  - warp 1 (one lane) issues S = Q K^T into one of two fp32 TMEM buffers
+//    (M = 128 tokens, N = 128 keys, K = 128), then O += P V into a third
+//    TMEM buffer once the softmax warps have written P;
+//  - warps 2-5 own one token row each: they read S with tcgen05.ld, apply
+//    the scale and the mask, keep a running reference maximum (log2 domain;
+//    O and the row sum are rescaled only when the block maximum exceeds the
+//    reference by more than 2^8), write P = 2^(s - ref) as bf16 into shared
+//    memory in the 128-byte-swizzled K-major layout the MMA reads, and sum
+//    the bf16 values of P into the row sum;
+//  - each split writes its unnormalised O, reference maximum and row sum;
+//    a combine kernel rescales the splits to a common maximum and divides.
+// The key range is split so that heads x splits fill the SMs: the cache
+// (2 x n x 128 x 2 bytes per head) is streamed once.
+// Every mbarrier wait gives up after ~2 s of clock64 time: it sets
+// SENSE_DEVST_TIMEOUT and an abort flag that releases the other roles; the
+// producer then waits (bounded) for its copies in flight, the MMA thread for
+// its MMAs, and the CTA frees its TMEM before returning.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "launch.h"
+#include "tc_ptx.cuh"
+
+namespace sense {
+namespace {
+
+constexpr int kAttnThreads = 192;
+constexpr int kHd = 128;                  // head dimension
+constexpr int kBN = 128;                  // keys per block
+constexpr int kSlab = 128 * 64 * 2;       // 128 rows x 64 bf16 (one 128-byte swizzle slab)
+constexpr int kTile = 2 * kSlab;          // 128 x 128 bf16
+constexpr int kStages = 2;
+constexpr int kStageBytes = 2 * kTile;    // K tile + V^T tile
+constexpr long long kWaitCycles = 4000000000LL;
+constexpr float kRescale = 8.0f;          // log2 growth that triggers a rescale of O
+
+struct AttnArgs {
+  int L, m, n, nb, splits, bps;
+  float scale_log2;
+  const uint32_t* mask;
+  int mask_words;
+  float* part_o;   // [H, splits, 128, 128]
+  float* part_ml;  // [H, splits, 128, 2]: reference maximum (log2), row sum
+  uint32_t* status;
+};
+
+struct AttnShared {
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort,
+                                         uint32_t* status) {
+  if (ptx::mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (ptx::mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *abort = 1;
+      raise_status(status, SENSE_DEVST_TIMEOUT);
+      return false;
+    }
+  }
+}
+__device__ __forceinline__ void drain_bar(uint32_t bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!ptx::mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > kWaitCycles) return;
+  }
+}
+
+// Bit t (0 <= t < 128) of the four mask words, without indexing a register array.
+__device__ __forceinline__ bool tree_bit(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3, int t) {
+  const uint32_t w = t < 64 ? (t < 32 ? w0 : w1) : (t < 96 ? w2 : w3);
+  return (w >> (t & 31)) & 1u;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(a));
+  const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(b));
+  return lo | (hi << 16);
+}
+
+__global__ void __launch_bounds__(kAttnThreads, 1)
+tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                 const __grid_constant__ CUtensorMap tm_vt, const AttnArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* s_q = smem;                       // Q tile
+  uint8_t* s_p = smem + kTile;               // P tile
+  uint8_t* s_kv = smem + 2 * kTile;          // stages: K tile, V^T tile
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_kv + kStages * kStageBytes);
+  // bars: q_full, kv_full[S], kv_empty[S], s_full[2], s_empty[2], p_full, o_done, mma_done
+  const int Q_FULL = 0, KV_FULL = 1, KV_EMPTY = 1 + kStages, S_FULL = 1 + 2 * kStages,
+            S_EMPTY = 3 + 2 * kStages, P_FULL = 5 + 2 * kStages, O_DONE = 6 + 2 * kStages,
+            MMA_DONE = 7 + 2 * kStages, NBARS = 8 + 2 * kStages;
+  AttnShared* sh = reinterpret_cast<AttnShared*>(bars + NBARS);
+  volatile int* abort = &sh->abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x, sp = blockIdx.y;
+  const int j0 = sp * a.bps;
+  const int j1 = min(a.nb, j0 + a.bps);
+  const int nbl = max(0, j1 - j0);
+  auto bar = [&](int i) { return ptx::smem_u32(bars + i); };
+
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(bar(Q_FULL), 1);
+    for (int s = 0; s < kStages; ++s) {
+      ptx::mbar_init(bar(KV_FULL + s), 1);
+      ptx::mbar_init(bar(KV_EMPTY + s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      ptx::mbar_init(bar(S_FULL + b), 1);
+      ptx::mbar_init(bar(S_EMPTY + b), 4);
+    }
+    ptx::mbar_init(bar(P_FULL), 4);
+    ptx::mbar_init(bar(O_DONE), 1);
+    ptx::mbar_init(bar(MMA_DONE), 1);
+    sh->abort = 0;
+    ptx::fence_barrier_init();
+    ptx::prefetch_tensormap(&tm_q);
+    ptx::prefetch_tensormap(&tm_k);
+    ptx::prefetch_tensormap(&tm_vt);
+  }
+  if (warp == 1) ptx::tmem_alloc(ptx::smem_u32(&sh->tmem_base), 512);
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = sh->tmem_base;  // S buffers at columns 0 and 128, O at 256
+
+  if (warp == 0 && lane == 0 && nbl > 0) {
+    // ------------------------------------------------ TMA producer
+    const uint64_t pol_stream = ptx::policy_evict_first();
+    const uint64_t pol_keep = ptx::policy_evict_last();
+    ptx::mbar_arrive_expect_tx(bar(Q_FULL), kTile);
+    ptx::tma_load_3d(ptx::smem_u32(s_q), &tm_q, bar(Q_FULL), 0, 0, h, pol_keep);
+    ptx::tma_load_3d(ptx::smem_u32(s_q + kSlab), &tm_q, bar(Q_FULL), 64, 0, h, pol_keep);
+    int issued = 0;
+    bool ok = true;
+    for (int jj = 0; jj < nbl && ok; ++jj) {
+      const int s = jj % kStages;
+      const uint32_t ph = (uint32_t)((jj / kStages) & 1);
+      if (!wait_bar(bar(KV_EMPTY + s), ph ^ 1u, abort, a.status)) {
+        ok = false;
+        break;
+      }
+      uint8_t* st = s_kv + s * kStageBytes;
+      const int key0 = (j0 + jj) * kBN;
+      ptx::mbar_arrive_expect_tx(bar(KV_FULL + s), kStageBytes);
+      ptx::tma_load_3d(ptx::smem_u32(st), &tm_k, bar(KV_FULL + s), 0, key0, h, pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(st + kSlab), &tm_k, bar(KV_FULL + s), 64, key0, h, pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(st + kTile), &tm_vt, bar(KV_FULL + s), key0, 0, h, pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(st + kTile + kSlab), &tm_vt, bar(KV_FULL + s), key0 + 64, 0, h,
+                       pol_stream);
+      ++issued;
+    }
+    drain_bar(bar(Q_FULL), 0);
+    if (!ok) {  // wait (bounded) for the copies that may still be in flight
+      for (int jj = max(0, issued - kStages); jj < issued; ++jj)
+        drain_bar(bar(KV_FULL + jj % kStages), (uint32_t)((jj / kStages) & 1));
+    }
+  } else if (warp == 1 && lane == 0 && nbl > 0) {
+    // ------------------------------------------------ MMA issuer
+    const uint32_t idesc = ptx::idesc_bf16_f32(128, 128);
+    const uint32_t q_addr = ptx::smem_u32(s_q), p_addr = ptx::smem_u32(s_p);
+    bool ok = wait_bar(bar(Q_FULL), 0, abort, a.status);
+    auto pv = [&](int i) -> bool {
+      if (!wait_bar(bar(P_FULL), (uint32_t)(i & 1), abort, a.status)) return false;
+      ptx::tc_fence_after();
+      const uint32_t vt = ptx::smem_u32(s_kv + (i % kStages) * kStageBytes + kTile);
+#pragma unroll
+      for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          ptx::mma_bf16(tmem + 256, ptx::desc_sw128(p_addr + kc * kSlab + t * 32),
+                        ptx::desc_sw128(vt + kc * kSlab + t * 32), idesc,
+                        (i > 0 || kc > 0 || t > 0) ? 1u : 0u);
+      ptx::mma_commit(bar(O_DONE));
+      ptx::mma_commit(bar(KV_EMPTY + i % kStages));
+      return true;
+    };
+    for (int jj = 0; jj < nbl && ok; ++jj) {
+      const int s = jj % kStages, b = jj & 1;
+      if (!wait_bar(bar(KV_FULL + s), (uint32_t)((jj / kStages) & 1), abort, a.status) ||
+          !wait_bar(bar(S_EMPTY + b), (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      const uint32_t kt = ptx::smem_u32(s_kv + s * kStageBytes);
+#pragma unroll
+      for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          ptx::mma_bf16(tmem + 128 * b, ptx::desc_sw128(q_addr + kc * kSlab + t * 32),
+                        ptx::desc_sw128(kt + kc * kSlab + t * 32), idesc,
+                        (kc > 0 || t > 0) ? 1u : 0u);
+      ptx::mma_commit(bar(S_FULL + b));
+      if (jj > 0 && !pv(jj - 1)) ok = false;
+    }
+    if (ok) pv(nbl - 1);
+    ptx::mma_commit(bar(MMA_DONE));
+    drain_bar(bar(MMA_DONE), 0);
+  } else if (warp >= 2) {
+    // ------------------------------------------------ softmax / epilogue
+    const int q4 = warp & 3;  // TMEM lane quarter this warp may access
+    const int r = q4 * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(q4 * 32) << 16);
+    uint32_t mw0 = 0u, mw1 = 0u, mw2 = 0u, mw3 = 0u;
+    if (r < a.L) {
+      const uint32_t* mr = a.mask + (int64_t)r * a.mask_words;
+      mw0 = mr[0];
+      if (a.mask_words > 1) mw1 = mr[1];
+      if (a.mask_words > 2) mw2 = mr[2];
+      if (a.mask_words > 3) mw3 = mr[3];
+    }
+    const float NEG = -__int_as_float(0x7f800000);
+    float ref = NEG, rowsum = 0.0f;
+    bool ok = true;
+    uint8_t* prow = s_p + r * 128;
+    const int sw = r & 7;
+    for (int jj = 0; jj < nbl && ok; ++jj) {
+      const int b = jj & 1;
+      if (!wait_bar(bar(S_FULL + b), (uint32_t)((jj >> 1) & 1), abort, a.status)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      float sv[kBN];
+#pragma unroll
+      for (int c = 0; c < kBN / 16; ++c) {
+        uint32_t rr[16];
+        ptx::tmem_ld16(lane_base + 128 * b + 16 * c, rr);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) sv[16 * c + e] = __uint_as_float(rr[e]);
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(bar(S_EMPTY + b));
+      // scale (log2 domain) and mask
+      const int key0 = (j0 + jj) * kBN;
+      float bmax = NEG;
+#pragma unroll
+      for (int c = 0; c < kBN; ++c) {
+        const int col = key0 + c;
+        bool vis = col < a.m;
+        if (!vis && r < a.L && col < a.m + a.L) vis = tree_bit(mw0, mw1, mw2, mw3, col - a.m);
+        sv[c] = vis ? sv[c] * a.scale_log2 : NEG;
+        bmax = fmaxf(bmax, sv[c]);
+      }
+      float factor = 1.0f;
+      bool rescale = false;
+      if (ref == NEG) {
+        ref = bmax;  // O is still zero for this row: nothing to rescale
+      } else if (bmax > ref + kRescale) {
+        factor = exp2f(ref - bmax);
+        ref = bmax;
+        rescale = true;
+      }
+      if (jj > 0) {  // O += P V of the previous block must be done (O and P reused)
+        if (!wait_bar(bar(O_DONE), (uint32_t)((jj - 1) & 1), abort, a.status)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        if (rescale) {
+#pragma unroll 1
+          for (int c = 0; c < kHd / 16; ++c) {
+            uint32_t rr[16];
+            ptx::tmem_ld16(lane_base + 256 + 16 * c, rr);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * factor);
+            ptx::tmem_st16(lane_base + 256 + 16 * c, rr);
+          }
+          rowsum *= factor;
+        }
+      }
+      // P = 2^(s - ref) as bf16, stored in the swizzled K-major layout
+#pragma unroll
+      for (int g = 0; g < kBN / 8; ++g) {
+        float pv[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float x = sv[8 * g + e];
+          const float pe = (x == NEG || ref == NEG) ? 0.0f : exp2f(x - ref);
+          pv[e] = __bfloat162float(__float2bfloat16_rn(pe));
+          rowsum += pv[e];
+        }
+        const uint4 w4 = make_uint4(pack_bf16(pv[0], pv[1]), pack_bf16(pv[2], pv[3]),
+                                    pack_bf16(pv[4], pv[5]), pack_bf16(pv[6], pv[7]));
+        const int slab = g >> 3, chunk = g & 7;
+        *reinterpret_cast<uint4*>(prow + slab * kSlab + ((chunk ^ sw) << 4)) = w4;
+      }
+      ptx::fence_proxy_async_smem();
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(bar(P_FULL));
+    }
+    // partial output of this split
+    const int64_t pbase = ((int64_t)h * a.splits + sp) * 128 + r;
+    float* po = a.part_o + pbase * kHd;
+    if (ok && nbl > 0 && wait_bar(bar(O_DONE), (uint32_t)((nbl - 1) & 1), abort, a.status)) {
+      ptx::tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < kHd / 16; ++c) {
+        uint32_t rr[16];
+        ptx::tmem_ld16(lane_base + 256 + 16 * c, rr);
+#pragma unroll
+        for (int e = 0; e < 16; e += 4)
+          *reinterpret_cast<float4*>(po + 16 * c + e) =
+              make_float4(__uint_as_float(rr[e]), __uint_as_float(rr[e + 1]),
+                          __uint_as_float(rr[e + 2]), __uint_as_float(rr[e + 3]));
+      }
+      a.part_ml[pbase * 2] = ref;
+      a.part_ml[pbase * 2 + 1] = rowsum;
+    } else {
+      a.part_ml[pbase * 2] = NEG;
+      a.part_ml[pbase * 2 + 1] = 0.0f;
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, 512);
+  }
+}
+
+// out[h, r, :] = sum_s 2^(ref_s - M) O_s / sum_s 2^(ref_s - M) l_s, one warp
+// per (head, row).
+__global__ void __launch_bounds__(256)
+tree_attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_ml,
+                         int heads, int splits, int L, float* __restrict__ out) {
+  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (w >= (int64_t)heads * L) return;
+  const int h = (int)(w / L), r = (int)(w - (int64_t)h * L);
+  const float NEG = -__int_as_float(0x7f800000);
+  float mx = NEG;
+  for (int s = 0; s < splits; ++s) {
+    const int64_t pb = ((int64_t)h * splits + s) * 128 + r;
+    if (part_ml[pb * 2 + 1] > 0.0f) mx = fmaxf(mx, part_ml[pb * 2]);
+  }
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  float den = 0.0f;
+  for (int s = 0; s < splits; ++s) {
+    const int64_t pb = ((int64_t)h * splits + s) * 128 + r;
+    const float l = part_ml[pb * 2 + 1];
+    if (!(l > 0.0f)) continue;
+    const float f = exp2f(part_ml[pb * 2] - mx);
+    den += f * l;
+    const float4 o = *reinterpret_cast<const float4*>(part_o + pb * kHd + 4 * lane);
+    acc.x += f * o.x;
+    acc.y += f * o.y;
+    acc.z += f * o.z;
+    acc.w += f * o.w;
+  }
+  const float inv = den > 0.0f ? 1.0f / den : 0.0f;
+  *reinterpret_cast<float4*>(out + ((int64_t)h * L + r) * kHd + 4 * lane) =
+      make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+}
+
+sense_status make_map3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                       uint64_t stride1, uint64_t stride2) {
+  void* fn = nullptr;
+  sense_status st = tensor_map_encoder(&fn);
+  if (st != SENSE_OK) return st;
+  auto enc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  const cuuint64_t dims[3] = {d0, d1, d2};
+  const cuuint64_t strides[2] = {stride1, stride2};
+  const cuuint32_t box[3] = {64, 128, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(SENSE_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+  return SENSE_OK;
+}
+
+size_t attn_smem_bytes() {
+  return 1024 + 2 * kTile + kStages * kStageBytes + (8 + 2 * kStages) * 8 + sizeof(AttnShared);
+}
+
+int attn_splits(int heads, int nb) {
+  const int per = std::max(1, sm_count() / heads);
+  return std::max(1, std::min(nb, per));
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+}  // namespace
+}  // namespace sense
+
+using namespace sense;
+
+extern "C" {
+
+size_t sense_tree_attention_workspace_bytes(int32_t heads, int32_t L, int32_t prefix_len) {
+  if (heads < 1 || L < 1 || prefix_len < 0) return 0;
+  const int nb = (prefix_len + L + kBN - 1) / kBN;
+  const int splits = attn_splits(heads, nb);
+  return align256((size_t)heads * splits * 128 * kHd * 4) + align256((size_t)heads * splits * 128 * 8);
+}
+
+sense_status sense_tree_attention(const uint16_t* q, const uint16_t* k_cache,
+                                  const uint16_t* vt_cache, int32_t heads, int32_t L,
+                                  int32_t d_head, int32_t capacity, int32_t prefix_len,
+                                  const uint32_t* mask_bits, int32_t mask_words, float scale,
+                                  float* out, void* workspace, size_t workspace_bytes,
+                                  sense_stream_t stream) {
+  if (!q || !k_cache || !vt_cache || !mask_bits || !out || !workspace)
+    return fail(SENSE_ERR_INVALID_ARG, "arrays and workspace must be non-NULL");
+  if (d_head != kHd) return fail(SENSE_ERR_UNSUPPORTED, "d_head=%d: only 128 is implemented", d_head);
+  if (heads < 1 || heads > 65535) return fail(SENSE_ERR_INVALID_ARG, "heads=%d outside [1, 65535]", heads);
+  if (L < 1 || L > 128) return fail(SENSE_ERR_INVALID_ARG, "L=%d outside [1, 128]", L);
+  if (capacity < 128 || capacity % 128)
+    return fail(SENSE_ERR_INVALID_ARG, "capacity=%d must be a positive multiple of 128", capacity);
+  if (prefix_len < 0 || (int64_t)prefix_len + L > capacity)
+    return fail(SENSE_ERR_INVALID_ARG, "prefix_len=%d + L=%d exceeds capacity=%d", prefix_len, L, capacity);
+  if (mask_words < (L + 31) / 32) return fail(SENSE_ERR_INVALID_ARG, "mask_words=%d < ceil(L/32)", mask_words);
+  if (!(scale > 0.0f) || scale > 1e30f) return fail(SENSE_ERR_INVALID_ARG, "scale must be positive and finite");
+  if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(vt_cache, 16) || !aligned(out, 16))
+    return fail(SENSE_ERR_INVALID_ARG, "q, caches and out must be 16-byte aligned");
+  if (!aligned(workspace, 256)) return fail(SENSE_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  if (workspace_bytes < sense_tree_attention_workspace_bytes(heads, L, prefix_len))
+    return fail(SENSE_ERR_INVALID_ARG, "workspace of %zu bytes < %zu", workspace_bytes,
+                sense_tree_attention_workspace_bytes(heads, L, prefix_len));
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int n = prefix_len + L;
+  const int nb = (n + kBN - 1) / kBN;
+  const int splits = attn_splits(heads, nb);
+  alignas(64) CUtensorMap tm_q, tm_k, tm_vt;
+  // Q [H, L, 128]; K [H, capacity, 128] seen up to n keys; V^T [H, 128, capacity] up to n keys
+  sense_status st = make_map3(&tm_q, q, kHd, L, heads, (uint64_t)kHd * 2, (uint64_t)L * kHd * 2);
+  if (st == SENSE_OK)
+    st = make_map3(&tm_k, k_cache, kHd, n, heads, (uint64_t)kHd * 2, (uint64_t)capacity * kHd * 2);
+  if (st == SENSE_OK)
+    st = make_map3(&tm_vt, vt_cache, n, kHd, heads, (uint64_t)capacity * 2,
+                   (uint64_t)kHd * capacity * 2);
+  if (st != SENSE_OK) return st;
+  AttnArgs a{};
+  a.L = L;
+  a.m = prefix_len;
+  a.n = n;
+  a.nb = nb;
+  a.splits = splits;
+  a.bps = (nb + splits - 1) / splits;
+  a.scale_log2 = scale * 1.4426950408889634f;
+  a.mask = mask_bits;
+  a.mask_words = mask_words;
+  char* ws = static_cast<char*>(workspace);
+  a.part_o = reinterpret_cast<float*>(ws);
+  a.part_ml = reinterpret_cast<float*>(ws + align256((size_t)heads * splits * 128 * kHd * 4));
+  a.status = status;
+  const size_t smem = attn_smem_bytes();
+  st = cuda_check(cudaFuncSetAttribute(tree_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem), "cudaFuncSetAttribute(tree_attn)");
+  if (st != SENSE_OK) return st;
+  {
+    LaunchScope ls(K_TREE_ATTN, s);
+    tree_attn_kernel<<<dim3(heads, splits), kAttnThreads, smem, s>>>(tm_q, tm_k, tm_vt, a);
+    st = cuda_check(cudaGetLastError(), "launch tree attention");
+    if (st != SENSE_OK) return st;
+  }
+  LaunchScope ls(K_TREE_ATTN, s);
+  const int64_t threads = (int64_t)heads * L * 32;
+  tree_attn_combine_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(
+      a.part_o, a.part_ml, heads, splits, L, out);
+  return cuda_check(cudaGetLastError(), "launch tree attention combine");
+}
+
+}  // extern "C"

@@ -41,6 +41,7 @@ enum KernelId {
   K_IVF_COARSE,
   K_IVF_SCAN,
   K_CTX,
+  K_TREE_ATTN,
   K_COUNT
 };
 

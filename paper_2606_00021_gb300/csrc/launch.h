@@ -88,6 +88,8 @@ sense_status launch_selftest_wait(long long limit, uint32_t* status, cudaStream_
 sense_status launch_pad_queries(const uint16_t* src, int qg, int d, uint16_t* dst, int nq,
                                 cudaStream_t s);
 size_t scan_tc_smem_bytes(int d, int nq);
+// The driver's cuTensorMapEncodeTiled (as a PFN_cuTensorMapEncodeTiled_v12000).
+sense_status tensor_map_encoder(void** fn);
 
 // Per query: exact k-th largest score code among the s_len sample keys ->
 // thresh[qi] = code << 32; sample keys at or above it are appended to the

@@ -310,6 +310,17 @@ sense_status get_encode(PFN_cuTensorMapEncodeTiled_v12000* fn) {
   return SENSE_OK;
 }
 
+}  // namespace
+
+sense_status tensor_map_encoder(void** fn) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = nullptr;
+  sense_status st = get_encode(&enc);
+  *fn = reinterpret_cast<void*>(enc);
+  return st;
+}
+
+namespace {
+
 sense_status make_map(CUtensorMap* m, const void* base, int64_t rows, int d, int box_rows) {
   PFN_cuTensorMapEncodeTiled_v12000 enc = nullptr;
   sense_status st = get_encode(&enc);
