@@ -191,6 +191,22 @@ class Pipeline:
                         __import__("ctypes").c_void_p(ctx.handle), q, kd), dev),
                     "anchor": torch.zeros(q, dtype=torch.int32, device=dev)}
 
+    def use_verify(self, heads, prefix, dev, seed=0):
+        """Adds the tree-masked attention of the verify forward (Alg. 1) on a
+        synthetic KV cache: heads x 128-dim, `prefix` committed positions,
+        the tree's cap rows as draft tokens."""
+        L = self.cap
+        capacity = ((prefix + L + 127) // 128) * 128
+        g = torch.Generator(device=dev).manual_seed(seed + 21)
+        mk = lambda *shape: torch.randn(*shape, generator=g, device=dev).to(torch.bfloat16)
+        self.verify = {"q": mk(heads, L, 128), "k": mk(heads, capacity, 128),
+                       "vt": mk(heads, 128, capacity), "prefix": prefix,
+                       "scale": 1.0 / 128 ** 0.5,
+                       "out": torch.empty(heads, L, 128, dtype=torch.float32, device=dev),
+                       "ws": self.S.alloc_workspace(self.S.lib().sense_tree_attention_workspace_bytes(
+                           heads, L, prefix), dev),
+                       "heads": heads, "L": L, "capacity": capacity}
+
     def step(self, query, gate_in):
         S, cfg = self.S, self.cfg
         self.retrieve(query)
@@ -202,7 +218,13 @@ class Pipeline:
                                workspace=dyn["ws"])
             S.sense_hybrid_drafts(self.ds, self.scores, self.idx, dyn["outs"], dyn["anchor"],
                                   cfg["k"], True, out=self.drafts)
-        S.sense_build_tree(self.drafts, node_cap=cfg["cap"], outs=self.tree)
+        ver = getattr(self, "verify", None)
+        S.sense_build_tree(self.drafts, node_cap=cfg["cap"], mask_bits=ver is not None,
+                           outs=self.tree)
+        if ver is not None:
+            S.sense_tree_attention(ver["q"], ver["k"], ver["vt"], ver["prefix"],
+                                   self.tree["mask_bits"][0], ver["scale"], out=ver["out"],
+                                   workspace=ver["ws"])
         root, nodes, hr, hn = gate_in
         S.sense_soft_gate(self.tree, root, nodes, hr, hn, workspace=self.gws, outs=self.gate, **GATE)
         if dyn is not None:
@@ -389,6 +411,9 @@ def main():
                     help="time CUDA graph replays of the whole step")
     ap.add_argument("--dynamic", type=int, default=0, metavar="CAPACITY",
                     help="add the dynamic context buffer of this many positions (q = 1)")
+    ap.add_argument("--verify", type=int, default=0, metavar="HEADS",
+                    help="add the tree-masked verify attention on a synthetic KV cache (q = 1)")
+    ap.add_argument("--verify-prefix", type=int, default=4096)
     ap.add_argument("--dyn-k", type=int, default=16)
     ap.add_argument("--delta", type=float, default=0.05)
     args = ap.parse_args()
@@ -432,6 +457,10 @@ def main():
         ann = build_ann(S, keys, args.retrieval, args.nlist, args.nprobe, args.pq_m,
                         args.proj_dim, dev, seed=rank)
         pipe.use_ann(ann, dev)
+    if args.verify:
+        if cfg["q"] != 1 or pipe.cap > 128:
+            raise SystemExit("--verify models one sequence with at most 128 tree nodes")
+        pipe.use_verify(args.verify, args.verify_prefix, dev, seed=rank)
     dyn_info = None
     if args.dynamic:
         if cfg["q"] != 1:
@@ -609,6 +638,21 @@ def main():
         scan_bytes_per_step, traffic = gate_bytes_step, None
         achieved = scan_bytes_per_step * args.steps / (scan_ms / 1e3) / 1e9
 
+    verify_info = None
+    if args.verify:
+        v = pipe.verify
+        n_keys = v["prefix"] + v["L"]
+        vbytes = 2 * v["heads"] * n_keys * 128 * 2 + v["heads"] * v["L"] * 128 * (2 + 4)
+        vflops = 4 * v["heads"] * v["L"] * n_keys * 128
+        t_ms, t_launches = prof.get("tree_attn", (0.0, 0))
+        per = t_ms / max(1, t_launches // 2) / 1e3  # main kernel + combine per step
+        verify_info = {"heads": v["heads"], "head_dim": 128, "draft_tokens": v["L"],
+                       "prefix": v["prefix"], "cache_capacity": v["capacity"],
+                       "us_per_step": per * 1e6,
+                       "algorithmic_bytes": vbytes, "gbs": vbytes / per / 1e9 if per else None,
+                       "frac_of_hbm": (vbytes / per / 1e9) / peak if per else None,
+                       "tflops": vflops / per / 1e12 if per else None}
+
     def compression(dist):
         return {"distinct_prefixes": float(np.mean(dist)),
                 "nodes_over_tokens": float(np.mean(dist)) / km,
@@ -659,9 +703,9 @@ def main():
 
     base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        if ann is None and not args.dynamic:
+        if ann is None and not args.dynamic and not args.verify:
             base = cpu_baseline(cfg, keys, spans, queries, gate_sets)
-        elif args.dynamic:
+        elif args.dynamic or args.verify:
             base = {"value": None, "skipped": "the oracle baseline times the static path only"}
         else:
             base = {"value": None, "skipped": "the oracle's index build over the full store "
@@ -675,7 +719,7 @@ def main():
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded clustered unit-norm keys, Zipf spans, N(0,9) logits)",
             "config": {"workload": args.workload, "retrieval": args.retrieval,
-                       "dynamic_capacity": args.dynamic,
+                       "dynamic_capacity": args.dynamic, "verify_heads": args.verify,
                        **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab", "cap", "clusters")},
                        "key_bytes": n * d * 2,
                        "l2": f"inputs larger than L2: the {n * d * 2 / 1e9:.1f} GB store is "
@@ -683,6 +727,7 @@ def main():
                        "parallelism": f"replicas x{world}"},
             "retrieval": retrieval,
             "dynamic": dyn_info,
+            "verify": verify_info,
             "launch": "cuda_graph" if graph is not None else "eager",
             "launch_note": graph_note,
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,

@@ -14,13 +14,16 @@
 //    (128-byte swizzle; keys past n are zero-filled) into a 2-stage ring;
 //  - warp 1 (one lane) issues S = Q K^T into one of two fp32 TMEM buffers
 //    (M = 128 tokens, N = 128 keys, K = 128), then O += P V into a third
-//    TMEM buffer once the softmax warps have written P;
+//    TMEM buffer once the softmax warps have written P (two P buffers, so
+//    the softmax of block j overlaps the product of block j - 1);
 //  - warps 2-5 own one token row each: they read S with tcgen05.ld, apply
-//    the scale and the mask, keep a running reference maximum (log2 domain;
-//    O and the row sum are rescaled only when the block maximum exceeds the
-//    reference by more than 2^8), write P = 2^(s - ref) as bf16 into shared
-//    memory in the 128-byte-swizzled K-major layout the MMA reads, and sum
-//    the bf16 values of P into the row sum;
+//    the scale and the mask (blocks wholly inside the committed prefix need
+//    none), keep a running reference maximum (log2 domain; O and the row sum
+//    are rescaled only when the block maximum exceeds the reference by more
+//    than 2^8, and only then wait for the previous product), write
+//    P = 2^(s - ref) (ex2.approx) as bf16 into shared memory in the
+//    128-byte-swizzled K-major layout the MMA reads, and sum the bf16
+//    values of P into the row sum;
 //  - each split writes its unnormalised O, reference maximum and row sum;
 //    a combine kernel rescales the splits to a common maximum and divides.
 // The key range is split so that heads x splits fill the SMs: the cache
@@ -94,6 +97,12 @@ __device__ __forceinline__ bool tree_bit(uint32_t w0, uint32_t w1, uint32_t w2, 
   return (w >> (t & 31)) & 1u;
 }
 
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(a));
   const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(b));
@@ -107,13 +116,14 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* s_q = smem;                       // Q tile
-  uint8_t* s_p = smem + kTile;               // P tile
-  uint8_t* s_kv = smem + 2 * kTile;          // stages: K tile, V^T tile
+  uint8_t* s_p = smem + kTile;               // two P tiles
+  uint8_t* s_kv = smem + 3 * kTile;          // stages: K tile, V^T tile
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_kv + kStages * kStageBytes);
-  // bars: q_full, kv_full[S], kv_empty[S], s_full[2], s_empty[2], p_full, o_done, mma_done
+  // bars: q_full, kv_full[S], kv_empty[S], s_full[2], s_empty[2], p_full[2],
+  // p_empty[2], o_done, mma_done
   const int Q_FULL = 0, KV_FULL = 1, KV_EMPTY = 1 + kStages, S_FULL = 1 + 2 * kStages,
-            S_EMPTY = 3 + 2 * kStages, P_FULL = 5 + 2 * kStages, O_DONE = 6 + 2 * kStages,
-            MMA_DONE = 7 + 2 * kStages, NBARS = 8 + 2 * kStages;
+            S_EMPTY = 3 + 2 * kStages, P_FULL = 5 + 2 * kStages, P_EMPTY = 7 + 2 * kStages,
+            O_DONE = 9 + 2 * kStages, MMA_DONE = 10 + 2 * kStages, NBARS = 11 + 2 * kStages;
   AttnShared* sh = reinterpret_cast<AttnShared*>(bars + NBARS);
   volatile int* abort = &sh->abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -132,8 +142,9 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     for (int b = 0; b < 2; ++b) {
       ptx::mbar_init(bar(S_FULL + b), 1);
       ptx::mbar_init(bar(S_EMPTY + b), 4);
+      ptx::mbar_init(bar(P_FULL + b), 4);
+      ptx::mbar_init(bar(P_EMPTY + b), 1);
     }
-    ptx::mbar_init(bar(P_FULL), 4);
     ptx::mbar_init(bar(O_DONE), 1);
     ptx::mbar_init(bar(MMA_DONE), 1);
     sh->abort = 0;
@@ -185,17 +196,20 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     const uint32_t q_addr = ptx::smem_u32(s_q), p_addr = ptx::smem_u32(s_p);
     bool ok = wait_bar(bar(Q_FULL), 0, abort, a.status);
     auto pv = [&](int i) -> bool {
-      if (!wait_bar(bar(P_FULL), (uint32_t)(i & 1), abort, a.status)) return false;
+      const int pb = i & 1;
+      if (!wait_bar(bar(P_FULL + pb), (uint32_t)((i >> 1) & 1), abort, a.status)) return false;
       ptx::tc_fence_after();
       const uint32_t vt = ptx::smem_u32(s_kv + (i % kStages) * kStageBytes + kTile);
+      const uint32_t pa = p_addr + pb * kTile;
 #pragma unroll
       for (int kc = 0; kc < 2; ++kc)
 #pragma unroll
         for (int t = 0; t < 4; ++t)
-          ptx::mma_bf16(tmem + 256, ptx::desc_sw128(p_addr + kc * kSlab + t * 32),
+          ptx::mma_bf16(tmem + 256, ptx::desc_sw128(pa + kc * kSlab + t * 32),
                         ptx::desc_sw128(vt + kc * kSlab + t * 32), idesc,
                         (i > 0 || kc > 0 || t > 0) ? 1u : 0u);
       ptx::mma_commit(bar(O_DONE));
+      ptx::mma_commit(bar(P_EMPTY + pb));
       ptx::mma_commit(bar(KV_EMPTY + i % kStages));
       return true;
     };
@@ -237,7 +251,6 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     const float NEG = -__int_as_float(0x7f800000);
     float ref = NEG, rowsum = 0.0f;
     bool ok = true;
-    uint8_t* prow = s_p + r * 128;
     const int sw = r & 7;
     for (int jj = 0; jj < nbl && ok; ++jj) {
       const int b = jj & 1;
@@ -247,79 +260,100 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
       }
       ptx::tc_fence_after();
       float sv[kBN];
+      {
+        uint32_t rr[kBN / 16][16];
 #pragma unroll
-      for (int c = 0; c < kBN / 16; ++c) {
-        uint32_t rr[16];
-        ptx::tmem_ld16(lane_base + 128 * b + 16 * c, rr);
+        for (int c = 0; c < kBN / 16; ++c) ptx::tmem_ld16_nowait(lane_base + 128 * b + 16 * c, rr[c]);
+        ptx::tmem_ld_wait();
 #pragma unroll
-        for (int e = 0; e < 16; ++e) sv[16 * c + e] = __uint_as_float(rr[e]);
+        for (int c = 0; c < kBN / 16; ++c)
+#pragma unroll
+          for (int e = 0; e < 16; ++e) sv[16 * c + e] = __uint_as_float(rr[c][e]);
       }
       ptx::tc_fence_before();
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(bar(S_EMPTY + b));
-      // scale (log2 domain) and mask
+      // scale (log2 domain) and mask; blocks inside the prefix are all visible
       const int key0 = (j0 + jj) * kBN;
-      float bmax = NEG;
+      float bm[8];
 #pragma unroll
-      for (int c = 0; c < kBN; ++c) {
-        const int col = key0 + c;
-        bool vis = col < a.m;
-        if (!vis && r < a.L && col < a.m + a.L) vis = tree_bit(mw0, mw1, mw2, mw3, col - a.m);
-        sv[c] = vis ? sv[c] * a.scale_log2 : NEG;
-        bmax = fmaxf(bmax, sv[c]);
+      for (int e = 0; e < 8; ++e) bm[e] = NEG;
+      if (key0 + kBN <= a.m) {
+#pragma unroll
+        for (int c = 0; c < kBN; ++c) {
+          sv[c] *= a.scale_log2;
+          bm[c & 7] = fmaxf(bm[c & 7], sv[c]);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < kBN; ++c) {
+          const int col = key0 + c;
+          bool vis = col < a.m;
+          if (!vis && r < a.L && col < a.m + a.L) vis = tree_bit(mw0, mw1, mw2, mw3, col - a.m);
+          sv[c] = vis ? sv[c] * a.scale_log2 : NEG;
+          bm[c & 7] = fmaxf(bm[c & 7], sv[c]);
+        }
       }
+      const float bmax = fmaxf(fmaxf(fmaxf(bm[0], bm[1]), fmaxf(bm[2], bm[3])),
+                               fmaxf(fmaxf(bm[4], bm[5]), fmaxf(bm[6], bm[7])));
       float factor = 1.0f;
       bool rescale = false;
       if (ref == NEG) {
         ref = bmax;  // O is still zero for this row: nothing to rescale
       } else if (bmax > ref + kRescale) {
-        factor = exp2f(ref - bmax);
+        factor = ex2(ref - bmax);
         ref = bmax;
         rescale = true;
       }
-      if (jj > 0) {  // O += P V of the previous block must be done (O and P reused)
+      // P buffer b is free once the product of block jj - 2 is done
+      if (!wait_bar(bar(P_EMPTY + b), (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status)) {
+        ok = false;
+        break;
+      }
+      if (rescale) {  // O must hold the product of block jj - 1 before it is scaled
         if (!wait_bar(bar(O_DONE), (uint32_t)((jj - 1) & 1), abort, a.status)) {
           ok = false;
           break;
         }
         ptx::tc_fence_after();
-        if (rescale) {
 #pragma unroll 1
-          for (int c = 0; c < kHd / 16; ++c) {
-            uint32_t rr[16];
-            ptx::tmem_ld16(lane_base + 256 + 16 * c, rr);
+        for (int c = 0; c < kHd / 16; ++c) {
+          uint32_t rr[16];
+          ptx::tmem_ld16(lane_base + 256 + 16 * c, rr);
 #pragma unroll
-            for (int e = 0; e < 16; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * factor);
-            ptx::tmem_st16(lane_base + 256 + 16 * c, rr);
-          }
-          rowsum *= factor;
+          for (int e = 0; e < 16; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * factor);
+          ptx::tmem_st16(lane_base + 256 + 16 * c, rr);
         }
+        rowsum *= factor;
       }
       // P = 2^(s - ref) as bf16, stored in the swizzled K-major layout
+      uint8_t* prow = s_p + b * kTile + r * 128;
+      float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int g = 0; g < kBN / 8; ++g) {
         float pv[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const float x = sv[8 * g + e];
-          const float pe = (x == NEG || ref == NEG) ? 0.0f : exp2f(x - ref);
+          const float pe = (x == NEG || ref == NEG) ? 0.0f : ex2(x - ref);
           pv[e] = __bfloat162float(__float2bfloat16_rn(pe));
-          rowsum += pv[e];
+          ps[e] += pv[e];
         }
         const uint4 w4 = make_uint4(pack_bf16(pv[0], pv[1]), pack_bf16(pv[2], pv[3]),
                                     pack_bf16(pv[4], pv[5]), pack_bf16(pv[6], pv[7]));
         const int slab = g >> 3, chunk = g & 7;
         *reinterpret_cast<uint4*>(prow + slab * kSlab + ((chunk ^ sw) << 4)) = w4;
       }
+      rowsum += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
       ptx::fence_proxy_async_smem();
       ptx::tc_fence_before();
       __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(bar(P_FULL));
+      if (lane == 0) ptx::mbar_arrive(bar(P_FULL + b));
     }
     // partial output of this split
     const int64_t pbase = ((int64_t)h * a.splits + sp) * 128 + r;
     float* po = a.part_o + pbase * kHd;
-    if (ok && nbl > 0 && wait_bar(bar(O_DONE), (uint32_t)((nbl - 1) & 1), abort, a.status)) {
+    if (ok && nbl > 0 && wait_bar(bar(MMA_DONE), 0, abort, a.status)) {
       ptx::tc_fence_after();
 #pragma unroll 1
       for (int c = 0; c < kHd / 16; ++c) {
@@ -398,7 +432,7 @@ sense_status make_map3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d
 }
 
 size_t attn_smem_bytes() {
-  return 1024 + 2 * kTile + kStages * kStageBytes + (8 + 2 * kStages) * 8 + sizeof(AttnShared);
+  return 1024 + 3 * kTile + kStages * kStageBytes + (11 + 2 * kStages) * 8 + sizeof(AttnShared);
 }
 
 int attn_splits(int heads, int nb) {
