@@ -8,15 +8,18 @@
 // (Alg. 3's mask, given as ancestor bit rows).  O = softmax(scale Q K^T +
 // M_full) V.
 //
-// Design (flash-attention over 128-key blocks; one CTA per (head, key split)):
+// Design (flash-attention over 64-key blocks; one CTA per (head, key split)):
 //  - warp 0 (one lane) loads Q [128 x 128] once and, per block, the K tile
-//    [128 keys x 128] and the V^T tile [128 x 128 keys] with 3-D TMA loads
-//    (128-byte swizzle; keys past n are zero-filled) into a 2-stage ring;
+//    [64 keys x 128] and the V^T tile [128 x 64 keys] with 3-D TMA loads
+//    (128-byte swizzle; keys past n are zero-filled) into a 4-stage ring;
 //  - warp 1 (one lane) issues S = Q K^T into one of two fp32 TMEM buffers
-//    (M = 128 tokens, N = 128 keys, K = 128), then O += P V into a third
+//    (M = 128 tokens, N = 64 keys, K = 128), then O += P V into a third
 //    TMEM buffer once the softmax warps have written P (two P buffers, so
 //    the softmax of block j overlaps the product of block j - 1);
-//  - warps 2-5 own one token row each: they read S with tcgen05.ld, apply
+//  - warps 2-9 own half a token row each (two warps per TMEM lane quarter,
+//    32 of a block's 64 keys and 64 of O's 128 dims each; the pair exchanges
+//    row maxima and sums
+//    through shared memory): they read S with tcgen05.ld, apply
 //    the scale and the mask (blocks wholly inside the committed prefix need
 //    none), keep a running reference maximum (log2 domain; O and the row sum
 //    are rescaled only when the block maximum exceeds the reference by more
@@ -45,13 +48,18 @@
 namespace sense {
 namespace {
 
-constexpr int kAttnThreads = 192;
+constexpr int kSoftWarps = 8;                 // two per TMEM lane quarter
+constexpr int kAttnThreads = (2 + kSoftWarps) * 32;
 constexpr int kHd = 128;                  // head dimension
-constexpr int kBN = 128;                  // keys per block
+constexpr int kBN = 64;                   // keys per block
 constexpr int kSlab = 128 * 64 * 2;       // 128 rows x 64 bf16 (one 128-byte swizzle slab)
-constexpr int kTile = 2 * kSlab;          // 128 x 128 bf16
-constexpr int kStages = 2;
-constexpr int kStageBytes = 2 * kTile;    // K tile + V^T tile
+constexpr int kKSlab = kBN * 64 * 2;      // kBN keys x 64 bf16
+constexpr int kQBytes = 2 * kSlab;        // Q: 128 tokens x 128 dims
+constexpr int kPBytes = kSlab;            // P: 128 tokens x 64 keys
+constexpr int kKBytes = 2 * kKSlab;       // K tile: 64 keys x 128 dims
+constexpr int kVBytes = kSlab;            // V^T tile: 128 dims x 64 keys
+constexpr int kStages = 4;
+constexpr int kStageBytes = kKBytes + kVBytes;
 constexpr long long kWaitCycles = 4000000000LL;
 constexpr float kRescale = 8.0f;          // log2 growth that triggers a rescale of O
 
@@ -103,10 +111,11 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// Two floats rounded to bf16 (nearest even) in one conversion: a in the low
+// half, b in the high half.
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-  const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(a));
-  const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(b));
-  return lo | (hi << 16);
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&v);
 }
 
 __global__ void __launch_bounds__(kAttnThreads, 1)
@@ -116,8 +125,8 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* s_q = smem;                       // Q tile
-  uint8_t* s_p = smem + kTile;               // two P tiles
-  uint8_t* s_kv = smem + 3 * kTile;          // stages: K tile, V^T tile
+  uint8_t* s_p = smem + kQBytes;             // two P tiles
+  uint8_t* s_kv = s_p + 2 * kPBytes;         // stages: K tile, V^T tile
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_kv + kStages * kStageBytes);
   // bars: q_full, kv_full[S], kv_empty[S], s_full[2], s_empty[2], p_full[2],
   // p_empty[2], o_done, mma_done
@@ -141,8 +150,8 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     }
     for (int b = 0; b < 2; ++b) {
       ptx::mbar_init(bar(S_FULL + b), 1);
-      ptx::mbar_init(bar(S_EMPTY + b), 4);
-      ptx::mbar_init(bar(P_FULL + b), 4);
+      ptx::mbar_init(bar(S_EMPTY + b), kSoftWarps);
+      ptx::mbar_init(bar(P_FULL + b), kSoftWarps);
       ptx::mbar_init(bar(P_EMPTY + b), 1);
     }
     ptx::mbar_init(bar(O_DONE), 1);
@@ -153,17 +162,17 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     ptx::prefetch_tensormap(&tm_k);
     ptx::prefetch_tensormap(&tm_vt);
   }
-  if (warp == 1) ptx::tmem_alloc(ptx::smem_u32(&sh->tmem_base), 512);
+  if (warp == 1) ptx::tmem_alloc(ptx::smem_u32(&sh->tmem_base), 256);
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
-  const uint32_t tmem = sh->tmem_base;  // S buffers at columns 0 and 128, O at 256
+  const uint32_t tmem = sh->tmem_base;  // S buffers at columns 0 and 64, O at 128
 
   if (warp == 0 && lane == 0 && nbl > 0) {
     // ------------------------------------------------ TMA producer
     const uint64_t pol_stream = ptx::policy_evict_first();
     const uint64_t pol_keep = ptx::policy_evict_last();
-    ptx::mbar_arrive_expect_tx(bar(Q_FULL), kTile);
+    ptx::mbar_arrive_expect_tx(bar(Q_FULL), kQBytes);
     ptx::tma_load_3d(ptx::smem_u32(s_q), &tm_q, bar(Q_FULL), 0, 0, h, pol_keep);
     ptx::tma_load_3d(ptx::smem_u32(s_q + kSlab), &tm_q, bar(Q_FULL), 64, 0, h, pol_keep);
     int issued = 0;
@@ -179,10 +188,8 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
       const int key0 = (j0 + jj) * kBN;
       ptx::mbar_arrive_expect_tx(bar(KV_FULL + s), kStageBytes);
       ptx::tma_load_3d(ptx::smem_u32(st), &tm_k, bar(KV_FULL + s), 0, key0, h, pol_stream);
-      ptx::tma_load_3d(ptx::smem_u32(st + kSlab), &tm_k, bar(KV_FULL + s), 64, key0, h, pol_stream);
-      ptx::tma_load_3d(ptx::smem_u32(st + kTile), &tm_vt, bar(KV_FULL + s), key0, 0, h, pol_stream);
-      ptx::tma_load_3d(ptx::smem_u32(st + kTile + kSlab), &tm_vt, bar(KV_FULL + s), key0 + 64, 0, h,
-                       pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(st + kKSlab), &tm_k, bar(KV_FULL + s), 64, key0, h, pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(st + kKBytes), &tm_vt, bar(KV_FULL + s), key0, 0, h, pol_stream);
       ++issued;
     }
     drain_bar(bar(Q_FULL), 0);
@@ -192,22 +199,20 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     }
   } else if (warp == 1 && lane == 0 && nbl > 0) {
     // ------------------------------------------------ MMA issuer
-    const uint32_t idesc = ptx::idesc_bf16_f32(128, 128);
+    const uint32_t idesc_s = ptx::idesc_bf16_f32(128, kBN);   // S = Q K^T
+    const uint32_t idesc_o = ptx::idesc_bf16_f32(128, kHd);   // O += P V
     const uint32_t q_addr = ptx::smem_u32(s_q), p_addr = ptx::smem_u32(s_p);
     bool ok = wait_bar(bar(Q_FULL), 0, abort, a.status);
     auto pv = [&](int i) -> bool {
       const int pb = i & 1;
       if (!wait_bar(bar(P_FULL + pb), (uint32_t)((i >> 1) & 1), abort, a.status)) return false;
       ptx::tc_fence_after();
-      const uint32_t vt = ptx::smem_u32(s_kv + (i % kStages) * kStageBytes + kTile);
-      const uint32_t pa = p_addr + pb * kTile;
+      const uint32_t vt = ptx::smem_u32(s_kv + (i % kStages) * kStageBytes + kKBytes);
+      const uint32_t pa = p_addr + pb * kPBytes;
 #pragma unroll
-      for (int kc = 0; kc < 2; ++kc)
-#pragma unroll
-        for (int t = 0; t < 4; ++t)
-          ptx::mma_bf16(tmem + 256, ptx::desc_sw128(pa + kc * kSlab + t * 32),
-                        ptx::desc_sw128(vt + kc * kSlab + t * 32), idesc,
-                        (i > 0 || kc > 0 || t > 0) ? 1u : 0u);
+      for (int t = 0; t < kBN / 16; ++t)
+        ptx::mma_bf16(tmem + 2 * kBN, ptx::desc_sw128(pa + t * 32), ptx::desc_sw128(vt + t * 32),
+                      idesc_o, (i > 0 || t > 0) ? 1u : 0u);
       ptx::mma_commit(bar(O_DONE));
       ptx::mma_commit(bar(P_EMPTY + pb));
       ptx::mma_commit(bar(KV_EMPTY + i % kStages));
@@ -226,8 +231,8 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
       for (int kc = 0; kc < 2; ++kc)
 #pragma unroll
         for (int t = 0; t < 4; ++t)
-          ptx::mma_bf16(tmem + 128 * b, ptx::desc_sw128(q_addr + kc * kSlab + t * 32),
-                        ptx::desc_sw128(kt + kc * kSlab + t * 32), idesc,
+          ptx::mma_bf16(tmem + kBN * b, ptx::desc_sw128(q_addr + kc * kSlab + t * 32),
+                        ptx::desc_sw128(kt + kc * kKSlab + t * 32), idesc_s,
                         (kc > 0 || t > 0) ? 1u : 0u);
       ptx::mma_commit(bar(S_FULL + b));
       if (jj > 0 && !pv(jj - 1)) ok = false;
@@ -237,8 +242,18 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     drain_bar(bar(MMA_DONE), 0);
   } else if (warp >= 2) {
     // ------------------------------------------------ softmax / epilogue
-    const int q4 = warp & 3;  // TMEM lane quarter this warp may access
+    // Warps w and w + 4 share TMEM lane quarter w & 3 (rows q4 * 32 + lane);
+    // `half` selects the 32 of a block's 64 keys and the 64 of O's 128 dims
+    // this thread owns.  The pair exchanges row maxima (and at the end row sums)
+    // through its own rows of the free P buffer, synchronised by a 64-thread
+    // named barrier.
+    constexpr int kCols = kBN / 2;
+    const int q4 = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int r = q4 * 32 + lane;
+    const int c0 = half * kCols;
+    const uint32_t pair_bar = 1 + q4;
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory"); };
     const uint32_t lane_base = tmem + ((uint32_t)(q4 * 32) << 16);
     uint32_t mw0 = 0u, mw1 = 0u, mw2 = 0u, mw3 = 0u;
     if (r < a.L) {
@@ -250,52 +265,69 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     }
     const float NEG = -__int_as_float(0x7f800000);
     float ref = NEG, rowsum = 0.0f;
+    // `ok` is kept warp-uniform and no thread leaves the loop early: every
+    // iteration executes both pair barriers, so a failed (aborted) wait in
+    // one warp can never leave its partner blocked in bar.sync.
     bool ok = true;
     const int sw = r & 7;
-    for (int jj = 0; jj < nbl && ok; ++jj) {
+    for (int jj = 0; jj < nbl; ++jj) {
       const int b = jj & 1;
-      if (!wait_bar(bar(S_FULL + b), (uint32_t)((jj >> 1) & 1), abort, a.status)) {
-        ok = false;
-        break;
-      }
-      ptx::tc_fence_after();
-      float sv[kBN];
-      {
-        uint32_t rr[kBN / 16][16];
+      ok = __all_sync(0xffffffffu,
+                      ok && wait_bar(bar(S_FULL + b), (uint32_t)((jj >> 1) & 1), abort, a.status));
+      float sv[kCols];
+      float pmax = NEG;
+      if (ok) {
+        ptx::tc_fence_after();
+        {
+          uint32_t rr[kCols / 16][16];
 #pragma unroll
-        for (int c = 0; c < kBN / 16; ++c) ptx::tmem_ld16_nowait(lane_base + 128 * b + 16 * c, rr[c]);
-        ptx::tmem_ld_wait();
+          for (int c = 0; c < kCols / 16; ++c)
+            ptx::tmem_ld16_nowait(lane_base + kBN * b + c0 + 16 * c, rr[c]);
+          ptx::tmem_ld_wait();
 #pragma unroll
-        for (int c = 0; c < kBN / 16; ++c)
+          for (int c = 0; c < kCols / 16; ++c)
 #pragma unroll
-          for (int e = 0; e < 16; ++e) sv[16 * c + e] = __uint_as_float(rr[c][e]);
-      }
-      ptx::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(bar(S_EMPTY + b));
-      // scale (log2 domain) and mask; blocks inside the prefix are all visible
-      const int key0 = (j0 + jj) * kBN;
-      float bm[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) bm[e] = NEG;
-      if (key0 + kBN <= a.m) {
-#pragma unroll
-        for (int c = 0; c < kBN; ++c) {
-          sv[c] *= a.scale_log2;
-          bm[c & 7] = fmaxf(bm[c & 7], sv[c]);
+            for (int e = 0; e < 16; ++e) sv[16 * c + e] = __uint_as_float(rr[c][e]);
         }
-      } else {
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(bar(S_EMPTY + b));
+        // scale (log2 domain) and mask; blocks inside the prefix are all visible
+        const int key0 = (j0 + jj) * kBN + c0;
+        float bm[8];
 #pragma unroll
-        for (int c = 0; c < kBN; ++c) {
-          const int col = key0 + c;
-          bool vis = col < a.m;
-          if (!vis && r < a.L && col < a.m + a.L) vis = tree_bit(mw0, mw1, mw2, mw3, col - a.m);
-          sv[c] = vis ? sv[c] * a.scale_log2 : NEG;
-          bm[c & 7] = fmaxf(bm[c & 7], sv[c]);
+        for (int e = 0; e < 8; ++e) bm[e] = NEG;
+        if (key0 + kCols <= a.m) {
+#pragma unroll
+          for (int c = 0; c < kCols; ++c) {
+            sv[c] *= a.scale_log2;
+            bm[c & 7] = fmaxf(bm[c & 7], sv[c]);
+          }
+        } else {
+#pragma unroll
+          for (int c = 0; c < kCols; ++c) {
+            const int col = key0 + c;
+            bool vis = col < a.m;
+            if (!vis && r < a.L && col < a.m + a.L) vis = tree_bit(mw0, mw1, mw2, mw3, col - a.m);
+            sv[c] = vis ? sv[c] * a.scale_log2 : NEG;
+            bm[c & 7] = fmaxf(bm[c & 7], sv[c]);
+          }
         }
+        pmax = fmaxf(fmaxf(fmaxf(bm[0], bm[1]), fmaxf(bm[2], bm[3])),
+                     fmaxf(fmaxf(bm[4], bm[5]), fmaxf(bm[6], bm[7])));
       }
-      const float bmax = fmaxf(fmaxf(fmaxf(bm[0], bm[1]), fmaxf(bm[2], bm[3])),
-                               fmaxf(fmaxf(bm[4], bm[5]), fmaxf(bm[6], bm[7])));
+      // P buffer b is free once the product of block jj - 2 is done
+      ok = __all_sync(0xffffffffu, ok && wait_bar(bar(P_EMPTY + b),
+                                                 (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status));
+      // exchange through this row of P buffer b: each thread's first 16-byte
+      // chunk (bytes only this pair touches; written over by P below)
+      uint8_t* pb_row = s_p + b * kPBytes + r * 128;
+      if (ok) *reinterpret_cast<float*>(pb_row + (((4 * half) ^ sw) << 4)) = pmax;
+      pair_sync();
+      const float other = *reinterpret_cast<const float*>(pb_row + (((4 * (1 - half)) ^ sw) << 4));
+      pair_sync();
+      if (!ok) continue;
+      const float bmax = fmaxf(pmax, other);
       float factor = 1.0f;
       bool rescale = false;
       if (ref == NEG) {
@@ -305,44 +337,42 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
         ref = bmax;
         rescale = true;
       }
-      // P buffer b is free once the product of block jj - 2 is done
-      if (!wait_bar(bar(P_EMPTY + b), (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status)) {
-        ok = false;
-        break;
-      }
-      if (rescale) {  // O must hold the product of block jj - 1 before it is scaled
-        if (!wait_bar(bar(O_DONE), (uint32_t)((jj - 1) & 1), abort, a.status)) {
-          ok = false;
-          break;
-        }
+      // O must hold the product of block jj - 1 before it is scaled
+      const bool any_rescale = __any_sync(0xffffffffu, rescale);
+      if (any_rescale) {
+        ok = __all_sync(0xffffffffu,
+                        wait_bar(bar(O_DONE), (uint32_t)((jj - 1) & 1), abort, a.status));
+        if (!ok) continue;
         ptx::tc_fence_after();
 #pragma unroll 1
-        for (int c = 0; c < kHd / 16; ++c) {
+        for (int c = 0; c < kHd / 2 / 16; ++c) {
           uint32_t rr[16];
-          ptx::tmem_ld16(lane_base + 256 + 16 * c, rr);
+          const uint32_t ta = lane_base + 2 * kBN + half * (kHd / 2) + 16 * c;
+          ptx::tmem_ld16(ta, rr);
 #pragma unroll
           for (int e = 0; e < 16; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * factor);
-          ptx::tmem_st16(lane_base + 256 + 16 * c, rr);
+          ptx::tmem_st16(ta, rr);
         }
         rowsum *= factor;
       }
-      // P = 2^(s - ref) as bf16, stored in the swizzled K-major layout
-      uint8_t* prow = s_p + b * kTile + r * 128;
+      // P = 2^(s - ref) as bf16 into this thread's chunks of the swizzled row
+      uint8_t* prow = s_p + b * kPBytes + r * 128;
       float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int g = 0; g < kBN / 8; ++g) {
-        float pv[8];
+      for (int g = 0; g < kCols / 8; ++g) {
+        uint32_t w[4];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float x = sv[8 * g + e];
-          const float pe = (x == NEG || ref == NEG) ? 0.0f : ex2(x - ref);
-          pv[e] = __bfloat162float(__float2bfloat16_rn(pe));
-          ps[e] += pv[e];
+        for (int e = 0; e < 8; e += 2) {
+          const float x0 = sv[8 * g + e], x1 = sv[8 * g + e + 1];
+          const float p0 = (x0 == NEG || ref == NEG) ? 0.0f : ex2(x0 - ref);
+          const float p1 = (x1 == NEG || ref == NEG) ? 0.0f : ex2(x1 - ref);
+          const uint32_t pk = pack_bf16(p0, p1);  // one paired conversion
+          w[e >> 1] = pk;
+          ps[e] += __uint_as_float(pk << 16);          // the rounded values
+          ps[e + 1] += __uint_as_float(pk & 0xffff0000u);
         }
-        const uint4 w4 = make_uint4(pack_bf16(pv[0], pv[1]), pack_bf16(pv[2], pv[3]),
-                                    pack_bf16(pv[4], pv[5]), pack_bf16(pv[6], pv[7]));
-        const int slab = g >> 3, chunk = g & 7;
-        *reinterpret_cast<uint4*>(prow + slab * kSlab + ((chunk ^ sw) << 4)) = w4;
+        *reinterpret_cast<uint4*>(prow + (((4 * half + g) ^ sw) << 4)) =
+            make_uint4(w[0], w[1], w[2], w[3]);
       }
       rowsum += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
       ptx::fence_proxy_async_smem();
@@ -350,33 +380,40 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(bar(P_FULL + b));
     }
-    // partial output of this split
+    // partial output of this split: each thread its 64 dims, row sums combined
     const int64_t pbase = ((int64_t)h * a.splits + sp) * 128 + r;
-    float* po = a.part_o + pbase * kHd;
-    if (ok && nbl > 0 && wait_bar(bar(MMA_DONE), 0, abort, a.status)) {
+    float* po = a.part_o + pbase * kHd + half * (kHd / 2);
+    const bool done =
+        __all_sync(0xffffffffu, ok && nbl > 0 && wait_bar(bar(MMA_DONE), 0, abort, a.status));
+    if (done) {
       ptx::tc_fence_after();
 #pragma unroll 1
-      for (int c = 0; c < kHd / 16; ++c) {
+      for (int c = 0; c < kHd / 2 / 16; ++c) {
         uint32_t rr[16];
-        ptx::tmem_ld16(lane_base + 256 + 16 * c, rr);
+        ptx::tmem_ld16(lane_base + 2 * kBN + half * (kHd / 2) + 16 * c, rr);
 #pragma unroll
         for (int e = 0; e < 16; e += 4)
           *reinterpret_cast<float4*>(po + 16 * c + e) =
               make_float4(__uint_as_float(rr[e]), __uint_as_float(rr[e + 1]),
                           __uint_as_float(rr[e + 2]), __uint_as_float(rr[e + 3]));
       }
-      a.part_ml[pbase * 2] = ref;
-      a.part_ml[pbase * 2 + 1] = rowsum;
-    } else {
-      a.part_ml[pbase * 2] = NEG;
-      a.part_ml[pbase * 2 + 1] = 0.0f;
+    }
+    // every product is done (or the CTA aborted): P buffer 0 is free; the row
+    // sums meet in this row's words of it
+    uint8_t* p0_row = s_p + r * 128;
+    *reinterpret_cast<float*>(p0_row + (((4 * half) ^ sw) << 4)) = rowsum;
+    pair_sync();
+    if (half == 0) {
+      a.part_ml[pbase * 2] = done ? ref : NEG;
+      a.part_ml[pbase * 2 + 1] =
+          done ? rowsum + *reinterpret_cast<const float*>(p0_row + ((4 ^ sw) << 4)) : 0.0f;
     }
   }
   ptx::tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem, 512);
+    ptx::tmem_dealloc(tmem, 256);
   }
 }
 
@@ -415,14 +452,14 @@ tree_attn_combine_kernel(const float* __restrict__ part_o, const float* __restri
 }
 
 sense_status make_map3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
-                       uint64_t stride1, uint64_t stride2) {
+                       uint64_t stride1, uint64_t stride2, uint32_t box_rows) {
   void* fn = nullptr;
   sense_status st = tensor_map_encoder(&fn);
   if (st != SENSE_OK) return st;
   auto enc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
   const cuuint64_t dims[3] = {d0, d1, d2};
   const cuuint64_t strides[2] = {stride1, stride2};
-  const cuuint32_t box[3] = {64, 128, 1};
+  const cuuint32_t box[3] = {64, box_rows, 1};
   const cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -432,7 +469,8 @@ sense_status make_map3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d
 }
 
 size_t attn_smem_bytes() {
-  return 1024 + 3 * kTile + kStages * kStageBytes + (11 + 2 * kStages) * 8 + sizeof(AttnShared);
+  return 1024 + kQBytes + 2 * kPBytes + kStages * kStageBytes + (11 + 2 * kStages) * 8 +
+         sizeof(AttnShared);
 }
 
 int attn_splits(int heads, int nb) {
@@ -489,12 +527,14 @@ sense_status sense_tree_attention(const uint16_t* q, const uint16_t* k_cache,
   const int splits = attn_splits(heads, nb);
   alignas(64) CUtensorMap tm_q, tm_k, tm_vt;
   // Q [H, L, 128]; K [H, capacity, 128] seen up to n keys; V^T [H, 128, capacity] up to n keys
-  sense_status st = make_map3(&tm_q, q, kHd, L, heads, (uint64_t)kHd * 2, (uint64_t)L * kHd * 2);
+  sense_status st =
+      make_map3(&tm_q, q, kHd, L, heads, (uint64_t)kHd * 2, (uint64_t)L * kHd * 2, 128);
   if (st == SENSE_OK)
-    st = make_map3(&tm_k, k_cache, kHd, n, heads, (uint64_t)kHd * 2, (uint64_t)capacity * kHd * 2);
+    st = make_map3(&tm_k, k_cache, kHd, n, heads, (uint64_t)kHd * 2, (uint64_t)capacity * kHd * 2,
+                   kBN);
   if (st == SENSE_OK)
     st = make_map3(&tm_vt, vt_cache, n, kHd, heads, (uint64_t)capacity * 2,
-                   (uint64_t)kHd * capacity * 2);
+                   (uint64_t)kHd * capacity * 2, 128);
   if (st != SENSE_OK) return st;
   AttnArgs a{};
   a.L = L;
