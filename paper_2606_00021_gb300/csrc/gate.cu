@@ -7,7 +7,7 @@
 // runs in two kernels:
 //  1. gate_rows: a persistent grid of warps; each warp takes whole rows
 //     (root or inner-node logits) from an atomic counter and streams a row
-//     through its own 6-stage shared-memory ring with 1-D bulk copies
+//     through its own 3-stage shared-memory ring with 1-D bulk copies
 //     (cp.async.bulk, 4 KB per stage, completion on an mbarrier; every wait
 //     is bounded by clock64 and a timeout sets SENSE_DEVST_TIMEOUT).  Each
 //     lane keeps the running max, the sums exp(x - max) and (x - max)
@@ -33,10 +33,10 @@
 namespace sense {
 namespace {
 
-constexpr int kRowThreads = 256;
+constexpr int kRowThreads = 512;
 constexpr int kWarps = kRowThreads / 32;
 constexpr int kWStageF4 = 256;                     // float4 per warp stage (4 KB)
-constexpr int kWStages = 6;                        // ring depth per warp
+constexpr int kWStages = 3;                        // ring depth per warp
 constexpr int kLaneF4 = kWStageF4 / 32;            // float4 per lane per stage
 constexpr size_t kRingBytes = (size_t)kWarps * kWStages * kWStageF4 * 16;
 constexpr int kStatsInts = 2 + SENSE_MAX_KAPPA;    // argmax, ent flag, top list
