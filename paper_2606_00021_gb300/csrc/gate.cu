@@ -402,16 +402,22 @@ __device__ bool warp_segment(const float* __restrict__ row, int lo4, int hi4, in
   // argmax: this lane's first maximum, read back from its stage
   int bi = 0x7fffffff;
   if (acc.mstage >= 0) {
+    // the lane's float4 of that stage, loaded together (one L2 round trip),
+    // then searched in index order
     const int f0 = acc.mstage * kWStageF4;
-    for (int u = 0; u < kLaneF4 && bi == 0x7fffffff; ++u) {
+    float4 v[kLaneF4];
+#pragma unroll
+    for (int u = 0; u < kLaneF4; ++u) {
       const int j = f0 + lane + 32 * u;
-      if (j >= n4) break;
-      const float4 v = row4[j];
-      const int e = (lo4 + j) * 4;
-      if (v.x == acc.m) bi = e;
-      else if (v.y == acc.m) bi = e + 1;
-      else if (v.z == acc.m) bi = e + 2;
-      else if (v.w == acc.m) bi = e + 3;
+      v[u] = (j < n4) ? row4[j] : make_float4(-FLT_MAX, -FLT_MAX, -FLT_MAX, -FLT_MAX);
+    }
+#pragma unroll
+    for (int u = kLaneF4 - 1; u >= 0; --u) {  // the last hit from the end is the first
+      const int e = (lo4 + f0 + lane + 32 * u) * 4;
+      if (v[u].w == acc.m) bi = e + 3;
+      if (v[u].z == acc.m) bi = e + 2;
+      if (v[u].y == acc.m) bi = e + 1;
+      if (v[u].x == acc.m) bi = e;
     }
   }
   float z0, z1, s0, s1;
