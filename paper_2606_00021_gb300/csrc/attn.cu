@@ -418,7 +418,9 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
 }
 
 // out[h, r, :] = sum_s 2^(ref_s - M) O_s / sum_s 2^(ref_s - M) l_s, one warp
-// per (head, row).
+// per (head, row): lane s holds split s's statistics (32 splits at a time),
+// the weights are shuffled to every lane, and each lane adds its 4 dims of
+// every split with the loads issued together.
 __global__ void __launch_bounds__(256)
 tree_attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_ml,
                          int heads, int splits, int L, float* __restrict__ out) {
@@ -427,24 +429,40 @@ tree_attn_combine_kernel(const float* __restrict__ part_o, const float* __restri
   if (w >= (int64_t)heads * L) return;
   const int h = (int)(w / L), r = (int)(w - (int64_t)h * L);
   const float NEG = -__int_as_float(0x7f800000);
+  const int64_t base = (int64_t)h * splits * 128 + r;  // partial of split s: base + s * 128
   float mx = NEG;
-  for (int s = 0; s < splits; ++s) {
-    const int64_t pb = ((int64_t)h * splits + s) * 128 + r;
-    if (part_ml[pb * 2 + 1] > 0.0f) mx = fmaxf(mx, part_ml[pb * 2]);
+  for (int s0 = 0; s0 < splits; s0 += 32) {
+    const int s = s0 + lane;
+    if (s < splits && part_ml[(base + (int64_t)s * 128) * 2 + 1] > 0.0f)
+      mx = fmaxf(mx, part_ml[(base + (int64_t)s * 128) * 2]);
   }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   float den = 0.0f;
-  for (int s = 0; s < splits; ++s) {
-    const int64_t pb = ((int64_t)h * splits + s) * 128 + r;
-    const float l = part_ml[pb * 2 + 1];
-    if (!(l > 0.0f)) continue;
-    const float f = exp2f(part_ml[pb * 2] - mx);
-    den += f * l;
-    const float4 o = *reinterpret_cast<const float4*>(part_o + pb * kHd + 4 * lane);
-    acc.x += f * o.x;
-    acc.y += f * o.y;
-    acc.z += f * o.z;
-    acc.w += f * o.w;
+  for (int s0 = 0; s0 < splits; s0 += 32) {
+    const int s = s0 + lane;
+    float f = 0.0f, l = 0.0f;
+    if (s < splits) {
+      l = part_ml[(base + (int64_t)s * 128) * 2 + 1];
+      if (l > 0.0f) f = exp2f(part_ml[(base + (int64_t)s * 128) * 2] - mx);
+      else l = 0.0f;
+    }
+    float fl = f * l;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) fl += __shfl_xor_sync(0xffffffffu, fl, off);
+    den += fl;
+    const int n = min(32, splits - s0);
+    for (int t = 0; t < n; ++t) {
+      const float ft = __shfl_sync(0xffffffffu, f, t);
+      if (ft == 0.0f) continue;  // warp-uniform
+      const float4 o = *reinterpret_cast<const float4*>(
+          part_o + (base + (int64_t)(s0 + t) * 128) * kHd + 4 * lane);
+      acc.x += ft * o.x;
+      acc.y += ft * o.y;
+      acc.z += ft * o.z;
+      acc.w += ft * o.w;
+    }
   }
   const float inv = den > 0.0f ? 1.0f / den : 0.0f;
   *reinterpret_cast<float4*>(out + ((int64_t)h * L + r) * kHd + 4 * lane) =
