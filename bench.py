@@ -234,6 +234,16 @@ class Pipeline:
             dyn["anchor"].copy_(g["next_anchor"])  # x~ of the next step
 
 
+DRAFT_KERNELS = ("scan_gemv", "scan_tc", "threshold", "merge", "pad_queries", "gather", "tree",
+                 "project", "ivf_coarse", "ivf_scan", "ctx")
+
+
+def draft_kernel_rate(prof, q, tokens_per_query, steps):
+    """tokens per query x queries / summed time of the drafting kernels."""
+    ms = sum(prof.get(name, (0.0, 0))[0] for name in DRAFT_KERNELS)
+    return q * tokens_per_query * steps / (ms / 1e3) if ms > 0 else None
+
+
 class GraphStep:
     """The whole drafting step captured as one CUDA graph per gate-input set.
     The graphs read the query from a fixed staging buffer; a step copies the
@@ -733,6 +743,12 @@ def main():
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,
             "gate_rows_per_step": float(np.mean(gate_rows_n)),
             "draft_tokens_per_s": value * mean_nodes,
+            # draft tokens (tree nodes) and raw gathered span tokens per second
+            # of the drafting kernels alone (retrieval, gather, tree)
+            "draft_tokens_per_s_drafting_kernels": draft_kernel_rate(prof, cfg["q"], mean_nodes,
+                                                                     args.steps),
+            "span_tokens_per_s_drafting_kernels": draft_kernel_rate(
+                prof, cfg["q"], cfg["k"] * cfg["m"], args.steps),
             "mean_tree_nodes": mean_nodes,
             "trie_compression": trie,
             "roofline": {"bound": "hbm", "kernel": scan_name, "achieved": achieved,
