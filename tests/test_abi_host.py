@@ -82,6 +82,42 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert call(GateParams(float("nan"), 3, 6, 0, 0)) == 1
 
 
+def test_extension_calls_reject_invalid_arguments(lib):
+    p = C.c_void_p(16 * 1024)  # never dereferenced: validation fails first
+    out = C.c_void_p(0)
+    # projection: n, d, v, flags, alignment
+    assert lib.sense_project(p, 0, 64, p, 16, None, 0, p, None) == 1
+    assert lib.sense_project(p, 4, 60, p, 16, None, 0, p, None) == 1
+    assert lib.sense_project(p, 4, 64, p, 129, None, 0, p, None) == 1
+    assert lib.sense_project(p, 4, 64, p, 16, None, 0x10, p, None) == 1
+    assert lib.sense_project(C.c_void_p(16 * 1024 + 4), 4, 64, p, 16, None, 0, p, None) == 1
+    # k-means: dim, ld, k, workspace
+    assert lib.sense_kmeans(p, 100, 12, 12, 8, 1, 0, p, p, None, p, 1 << 20, None) == 1
+    assert lib.sense_kmeans(p, 100, 16, 8, 8, 1, 0, p, p, None, p, 1 << 20, None) == 1
+    assert lib.sense_kmeans(p, 100, 16, 16, 0, 1, 0, p, p, None, p, 1 << 20, None) == 1
+    assert lib.sense_kmeans(p, 100, 16, 16, 8, 1, 0, p, p, None, p, 16, None) == 1
+    # IVF build: v, nlist, pq_m without codebooks, pq_m not dividing v
+    assert lib.sense_ivf_build(p, 100, 24, p, 8, None, 0, None, C.byref(out)) == 1
+    assert lib.sense_ivf_build(p, 100, 64, p, 20000, None, 0, None, C.byref(out)) == 1
+    assert lib.sense_ivf_build(p, 100, 64, p, 8, None, 4, None, C.byref(out)) == 1
+    assert lib.sense_ivf_build(p, 100, 64, p, 8, p, 3, None, C.byref(out)) == 1
+    assert lib.sense_ivf_search(None, p, 1, 1, 1, p, p, None, p, 1 << 20, None) == 1
+    # dynamic buffer: capacity below m, d not a multiple of 8
+    assert lib.sense_ctx_create(4, 64, 8, C.byref(out)) == 1
+    assert lib.sense_ctx_create(64, 60, 8, C.byref(out)) == 1
+    assert lib.sense_ctx_search(None, p, 1, 1, C.c_float(0), p, p, p, p, 1 << 20, None) == 1
+    assert lib.sense_hybrid_drafts(None, p, p, 4, p, p, 4, 1, None, 4, 0, p, None) == 1
+    # tree attention: head dim, L, capacity, prefix beyond capacity, scale
+    args = lambda hd, L, cap, pre, sc: (p, p, p, 2, L, hd, cap, pre, p, 4, C.c_float(sc), p, p,
+                                        1 << 30, None)
+    assert lib.sense_tree_attention(*args(64, 8, 128, 0, 0.1)) == 2
+    assert lib.sense_tree_attention(*args(128, 129, 256, 0, 0.1)) == 1
+    assert lib.sense_tree_attention(*args(128, 8, 100, 0, 0.1)) == 1
+    assert lib.sense_tree_attention(*args(128, 8, 128, 125, 0.1)) == 1
+    assert lib.sense_tree_attention(*args(128, 8, 128, 0, 0.0)) == 1
+    # tree mask covered in test_invalid_arguments_rejected_on_host
+
+
 def test_workspace_sizes(lib):
     assert lib.sense_retrieve_workspace_bytes(None, 1, 1) == 0
     assert lib.sense_soft_gate_workspace_bytes(2, 64, 3) >= 2 * 65 * 4
