@@ -207,7 +207,7 @@ class Pipeline:
                            heads, L, prefix), dev),
                        "heads": heads, "L": L, "capacity": capacity}
 
-    def step(self, query, gate_in):
+    def step(self, query, gate_in, before_gate=None):
         S, cfg = self.S, self.cfg
         self.retrieve(query)
         dyn = getattr(self, "dyn", None)
@@ -225,6 +225,8 @@ class Pipeline:
             S.sense_tree_attention(ver["q"], ver["k"], ver["vt"], ver["prefix"],
                                    self.tree["mask_bits"][0], ver["scale"], out=ver["out"],
                                    workspace=ver["ws"])
+        if before_gate is not None:
+            before_gate()
         root, nodes, hr, hn = gate_in
         S.sense_soft_gate(self.tree, root, nodes, hr, hn, workspace=self.gws, outs=self.gate, **GATE)
         if dyn is not None:
@@ -694,11 +696,19 @@ def main():
         h_gate = []
     torch.cuda.synchronize()
     t0 = time.perf_counter()
+    # the gate's inputs do not depend on retrieval: their host-to-device copies
+    # run on a side stream while the step drafts, and the gate waits for them
+    copy_stream = torch.cuda.Stream(device=dev)
+    copied = torch.cuda.Event()
+    main = torch.cuda.current_stream()
     for it in range(e2e_steps):
         d_query.copy_(h_query, non_blocking=True)
-        for dg, hg in zip(d_gate, h_gate):
-            dg.copy_(hg, non_blocking=True)
-        pipe.step(d_query, d_gate)
+        copy_stream.wait_stream(main)
+        with torch.cuda.stream(copy_stream):
+            for dg, hg in zip(d_gate, h_gate):
+                dg.copy_(hg, non_blocking=True)
+            copied.record(copy_stream)
+        pipe.step(d_query, d_gate, before_gate=lambda: main.wait_event(copied))
         h_scores.copy_(pipe.scores, non_blocking=True)
         h_idx.copy_(pipe.idx, non_blocking=True)
         h_acc.copy_(pipe.gate["accepted"], non_blocking=True)
