@@ -51,14 +51,15 @@ namespace {
 constexpr int kSoftWarps = 8;                 // two per TMEM lane quarter
 constexpr int kAttnThreads = (2 + kSoftWarps) * 32;
 constexpr int kHd = 128;                  // head dimension
-constexpr int kBN = 64;                   // keys per block
+constexpr int kBN = 64;                   // keys per block (64 or 128)
+constexpr int kKS = kBN / 64;             // 64-key slabs per block
 constexpr int kSlab = 128 * 64 * 2;       // 128 rows x 64 bf16 (one 128-byte swizzle slab)
-constexpr int kKSlab = kBN * 64 * 2;      // kBN keys x 64 bf16
+constexpr int kKSlab = kBN * 64 * 2;      // kBN keys x 64 dims
 constexpr int kQBytes = 2 * kSlab;        // Q: 128 tokens x 128 dims
-constexpr int kPBytes = kSlab;            // P: 128 tokens x 64 keys
-constexpr int kKBytes = 2 * kKSlab;       // K tile: 64 keys x 128 dims
-constexpr int kVBytes = kSlab;            // V^T tile: 128 dims x 64 keys
-constexpr int kStages = 4;
+constexpr int kPBytes = kKS * kSlab;      // P: 128 tokens x kBN keys
+constexpr int kKBytes = 2 * kKSlab;       // K tile: kBN keys x 128 dims
+constexpr int kVBytes = kKS * kSlab;      // V^T tile: 128 dims x kBN keys
+constexpr int kStages = (kBN == 64) ? 4 : 2;
 constexpr int kStageBytes = kKBytes + kVBytes;
 constexpr long long kWaitCycles = 4000000000LL;
 constexpr float kRescale = 8.0f;          // log2 growth that triggers a rescale of O
@@ -162,11 +163,12 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     ptx::prefetch_tensormap(&tm_k);
     ptx::prefetch_tensormap(&tm_vt);
   }
-  if (warp == 1) ptx::tmem_alloc(ptx::smem_u32(&sh->tmem_base), 256);
+  constexpr uint32_t kTmemCols = (2 * kBN + kHd <= 256) ? 256 : 512;
+  if (warp == 1) ptx::tmem_alloc(ptx::smem_u32(&sh->tmem_base), kTmemCols);
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
-  const uint32_t tmem = sh->tmem_base;  // S buffers at columns 0 and 64, O at 128
+  const uint32_t tmem = sh->tmem_base;  // S buffers at columns 0 and kBN, O at 2 kBN
 
   if (warp == 0 && lane == 0 && nbl > 0) {
     // ------------------------------------------------ TMA producer
@@ -189,7 +191,10 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
       ptx::mbar_arrive_expect_tx(bar(KV_FULL + s), kStageBytes);
       ptx::tma_load_3d(ptx::smem_u32(st), &tm_k, bar(KV_FULL + s), 0, key0, h, pol_stream);
       ptx::tma_load_3d(ptx::smem_u32(st + kKSlab), &tm_k, bar(KV_FULL + s), 64, key0, h, pol_stream);
-      ptx::tma_load_3d(ptx::smem_u32(st + kKBytes), &tm_vt, bar(KV_FULL + s), key0, 0, h, pol_stream);
+#pragma unroll
+      for (int i = 0; i < kKS; ++i)
+        ptx::tma_load_3d(ptx::smem_u32(st + kKBytes + i * kSlab), &tm_vt, bar(KV_FULL + s),
+                         key0 + 64 * i, 0, h, pol_stream);
       ++issued;
     }
     drain_bar(bar(Q_FULL), 0);
@@ -210,9 +215,12 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
       const uint32_t vt = ptx::smem_u32(s_kv + (i % kStages) * kStageBytes + kKBytes);
       const uint32_t pa = p_addr + pb * kPBytes;
 #pragma unroll
-      for (int t = 0; t < kBN / 16; ++t)
-        ptx::mma_bf16(tmem + 2 * kBN, ptx::desc_sw128(pa + t * 32), ptx::desc_sw128(vt + t * 32),
-                      idesc_o, (i > 0 || t > 0) ? 1u : 0u);
+      for (int ks = 0; ks < kKS; ++ks)
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          ptx::mma_bf16(tmem + 2 * kBN, ptx::desc_sw128(pa + ks * kSlab + t * 32),
+                        ptx::desc_sw128(vt + ks * kSlab + t * 32), idesc_o,
+                        (i > 0 || ks > 0 || t > 0) ? 1u : 0u);
       ptx::mma_commit(bar(O_DONE));
       ptx::mma_commit(bar(P_EMPTY + pb));
       ptx::mma_commit(bar(KV_EMPTY + i % kStages));
@@ -270,6 +278,12 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     // one warp can never leave its partner blocked in bar.sync.
     bool ok = true;
     const int sw = r & 7;
+    constexpr int kChunksT = kCols / 8;  // 16-byte chunks of a P row per thread
+    // logical chunk g (8 keys) of this row in a P tile: slab g / 8, swizzled
+    // position (g % 8) ^ (row % 8) inside the row's 128 bytes
+    auto pchunk = [&](uint8_t* tile, int g) {
+      return tile + (g >> 3) * kSlab + r * 128 + ((((g & 7) ^ sw)) << 4);
+    };
     for (int jj = 0; jj < nbl; ++jj) {
       const int b = jj & 1;
       ok = __all_sync(0xffffffffu,
@@ -321,10 +335,10 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
                                                  (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status));
       // exchange through this row of P buffer b: each thread's first 16-byte
       // chunk (bytes only this pair touches; written over by P below)
-      uint8_t* pb_row = s_p + b * kPBytes + r * 128;
-      if (ok) *reinterpret_cast<float*>(pb_row + (((4 * half) ^ sw) << 4)) = pmax;
+      uint8_t* ptile = s_p + b * kPBytes;
+      if (ok) *reinterpret_cast<float*>(pchunk(ptile, kChunksT * half)) = pmax;
       pair_sync();
-      const float other = *reinterpret_cast<const float*>(pb_row + (((4 * (1 - half)) ^ sw) << 4));
+      const float other = *reinterpret_cast<const float*>(pchunk(ptile, kChunksT * (1 - half)));
       pair_sync();
       if (!ok) continue;
       const float bmax = fmaxf(pmax, other);
@@ -356,7 +370,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
         rowsum *= factor;
       }
       // P = 2^(s - ref) as bf16 into this thread's chunks of the swizzled row
-      uint8_t* prow = s_p + b * kPBytes + r * 128;
+
       float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int g = 0; g < kCols / 8; ++g) {
@@ -371,7 +385,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
           ps[e] += __uint_as_float(pk << 16);          // the rounded values
           ps[e + 1] += __uint_as_float(pk & 0xffff0000u);
         }
-        *reinterpret_cast<uint4*>(prow + (((4 * half + g) ^ sw) << 4)) =
+        *reinterpret_cast<uint4*>(pchunk(ptile, kChunksT * half + g)) =
             make_uint4(w[0], w[1], w[2], w[3]);
       }
       rowsum += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
@@ -400,20 +414,19 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     }
     // every product is done (or the CTA aborted): P buffer 0 is free; the row
     // sums meet in this row's words of it
-    uint8_t* p0_row = s_p + r * 128;
-    *reinterpret_cast<float*>(p0_row + (((4 * half) ^ sw) << 4)) = rowsum;
+    *reinterpret_cast<float*>(pchunk(s_p, kChunksT * half)) = rowsum;
     pair_sync();
     if (half == 0) {
       a.part_ml[pbase * 2] = done ? ref : NEG;
       a.part_ml[pbase * 2 + 1] =
-          done ? rowsum + *reinterpret_cast<const float*>(p0_row + ((4 ^ sw) << 4)) : 0.0f;
+          done ? rowsum + *reinterpret_cast<const float*>(pchunk(s_p, kChunksT)) : 0.0f;
     }
   }
   ptx::tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem, 256);
+    ptx::tmem_dealloc(tmem, kTmemCols);
   }
 }
 
