@@ -36,12 +36,19 @@ from synth.workloads import WORKLOADS  # noqa: E402
 DEFAULT = "llama7b_1m"
 METRIC = "hidden-state top-k retrieval queries/s (whole drafting step)"
 GATE = dict(gamma=0.05, topk=3, window=6, tau=0)
-# DRAM bytes (read + write) per launch of the dominant kernel on the default
-# workload, from one ncu capture (profiles/scan_gemv_llama7b_1m.md): the
-# 262,144-key case read 2.14776 GB and wrote 2.92 MB; traffic grows with the
-# rows scanned, so x4 for the 1,048,576-key store.  None once the kernel
-# changes after the capture.
-NCU_TRAFFIC = {("scan_gemv", "llama7b_1m"): (2.147761e9 + 2.923264e6) * 4}
+# DRAM bytes (read + write) per unit processed by the dominant kernels, each
+# from one ncu capture of a smaller case of the same kernel and shape (the
+# summaries in profiles/), scaled in the bench line by the units of a full
+# step: key rows for the scans (keyed by d), logits rows for the gate's row
+# pass (keyed by V).  Traffic grows in proportion to those units.
+NCU_TRAFFIC_PER_UNIT = {
+    # 262,144 x 4096 keys: 2,147,567,104 B read + 2,790,912 B written
+    ("scan_gemv", 4096): (2147567104 + 2790912) / 262144,
+    # 524,288 x 3584 keys, sample + rest launches of one step
+    ("scan_tc", 3584): (235048448 + 2988800 + 3523437824 + 185600) / 524288,
+    # 4 queries of the k = 64 sweep: 3,774 root / inner-node rows of 128,256 logits
+    ("gate_rows", 128256): (2055664000 + 3651840) / 3773.9375,
+}
 
 
 def peaks():
@@ -566,7 +573,8 @@ def main():
         scan_name = "scan_gemv" if q <= 8 else "scan_tc"
         scan_bytes_per_step = n * d * 2 + q * d * 2
         step_bytes = scan_bytes_per_step  # + the gate rows, added below
-        traffic = NCU_TRAFFIC.get((scan_name, args.workload))
+        per_row = NCU_TRAFFIC_PER_UNIT.get((scan_name, d))
+        traffic = per_row * n if per_row else None
     else:
         # entries scanned per query (probed list sizes, over the distinct batches)
         off = ann["index"].arrays()["offsets"]
@@ -647,7 +655,9 @@ def main():
     g_ms, g_launches = prof.get("gate_rows", (0.0, 0))
     if g_ms > scan_ms:
         scan_name, scan_ms, scan_launches = "gate_rows", g_ms, g_launches
-        scan_bytes_per_step, traffic = gate_bytes_step, None
+        scan_bytes_per_step = gate_bytes_step
+        per_row = NCU_TRAFFIC_PER_UNIT.get(("gate_rows", cfg["vocab"]))
+        traffic = per_row * float(np.mean(gate_rows_n)) if per_row else None
         achieved = scan_bytes_per_step * args.steps / (scan_ms / 1e3) / 1e9
 
     verify_info = None
