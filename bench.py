@@ -427,7 +427,10 @@ def main():
     ap.add_argument("--pq-m", type=int, default=16)
     ap.add_argument("--proj-dim", type=int, default=64)
     ap.add_argument("--graph", action="store_true",
-                    help="time CUDA graph replays of the whole step")
+                    help="time CUDA graph replays of the whole step (per-kernel times then "
+                         "come from an eager pass after the timed region)")
+    ap.add_argument("--no-graph-line", action="store_true",
+                    help="skip the supplementary graph-replay measurement of an eager run")
     ap.add_argument("--dynamic", type=int, default=0, metavar="CAPACITY",
                     help="add the dynamic context buffer of this many positions (q = 1)")
     ap.add_argument("--verify", type=int, default=0, metavar="HEADS",
@@ -563,6 +566,36 @@ def main():
     S.sense_profile_enable(False)
     ms = max_over_ranks(ms, dist, dev)
     launches = sum(v[1] for v in prof.values())
+
+    # Supplementary: the same steps as CUDA graph replays (one graph per
+    # gate-input set), after the eager timed region that the line reports.
+    graph_line = None
+    if graph is None and not args.no_graph_line:
+        try:
+            gstep = GraphStep(pipe, queries[0], gate_sets)
+            for it in range(args.warmup):
+                gstep.step(queries[it % nq], it % n_sets)
+            torch.cuda.synchronize()
+            if dist:
+                dist.barrier()
+            g0 = torch.cuda.Event(enable_timing=True)
+            g1 = torch.cuda.Event(enable_timing=True)
+            g0.record(stream)
+            for it in range(args.steps):
+                gstep.step(queries[it % nq], it % n_sets)
+            g1.record(stream)
+            torch.cuda.synchronize()
+            gms = max_over_ranks(g0.elapsed_time(g1), dist, dev)
+            if S.sense_device_status(clear=True) != 0:
+                raise RuntimeError("device status bits set during graph replays")
+            graph_line = {"value": job_throughput(cfg["q"] * args.steps, world, gms / 1e3),
+                          "ms_per_step": gms / args.steps, "steps": args.steps,
+                          "note": "the same steps replayed as one CUDA graph per gate-input "
+                                  "set, timed after the eager region"}
+            del gstep
+        except Exception as e:  # capture refused: no supplementary line
+            torch.cuda.synchronize()
+            graph_line = {"value": None, "skipped": f"{type(e).__name__}: {e}"}
 
     q, n, d = cfg["q"], cfg["n"], cfg["d"]
     value = job_throughput(q * args.steps, world, ms / 1e3)
@@ -760,6 +793,7 @@ def main():
             "verify": verify_info,
             "launch": "cuda_graph" if graph is not None else "eager",
             "launch_note": graph_note,
+            "graph_replay": graph_line,
             "hbm_gbs": step_bytes * args.steps / (ms / 1e3) / 1e9,
             "gate_rows_per_step": float(np.mean(gate_rows_n)),
             "draft_tokens_per_s": value * mean_nodes,

@@ -12,18 +12,22 @@
 //     is bounded by clock64 and a timeout sets SENSE_DEVST_TIMEOUT).  Each
 //     lane keeps the running max, the sums exp(x - max) and (x - max)
 //     exp(x - max) in packed fp32 pairs (entropy H = log Z - S / Z, with
-//     ex2 in base-2 units), the stage holding its first maximum (the argmax
-//     index is read back once at the end: lowest index among maxima) and a
+//     ex2 in base-2 units), the index of its first maximum (found in the
+//     stage that raised the maximum: lowest index among maxima) and a
 //     top-kappa list under (logit desc, index asc).  A lower bound of the
 //     row's kappa-th largest value, seeded from the lane maxima of the
 //     first stage and refreshed from the lists after stages 1, 3, 7, 15, 31,
 //     keeps list updates (warp-voted) off the common path.  All combining is
 //     done with warp shuffles: no block barriers.  A node is an inner node
 //     iff the next node in preorder is its child, so the test is O(1).
+//     With at most one row per SM (a single query's tree) the same warp
+//     pass runs as one block per row instead, its warps on consecutive
+//     slices, merged in shared memory (gate_row_block_kernel).
 //  2. gate_decide: one block per query evaluates B_em, B_ent, B_topk, the
 //     lookahead B_con, G, the accepted prefix lengths L_i, i*, and writes
 //     the accepted tokens, the next node, its argmax (streaming that row if
 //     it is a leaf) and h_next.
+#include <cooperative_groups.h>
 #include <float.h>
 
 #include "common.cuh"
@@ -32,6 +36,8 @@
 
 namespace sense {
 namespace {
+
+namespace cg = cooperative_groups;
 
 constexpr int kRowThreads = 512;
 constexpr int kWarps = kRowThreads / 32;
@@ -116,7 +122,7 @@ template <int KM>
 struct RowAcc {
   float m = -FLT_MAX;       // running max (also the argmax value)
   uint64_t z = 0, s = 0;    // packed pairs: sum exp(x - m), sum ((x - m) log2 e) exp(x - m)
-  int mstage = -1;          // stage holding this thread's first maximum
+  int am = 0x7fffffff;      // index of this thread's first maximum
   float lb = -FLT_MAX;      // lower bound of the row's kappa-th largest value
   TopList<KM> tl;
 
@@ -136,16 +142,23 @@ struct RowAcc {
   // Folds one stage: kLaneF4 float4 of this lane (element indices
   // idx[u] * 4 + e, increasing).  Padding slots hold -FLT_MAX.  Called by
   // all 32 lanes of a warp together (it votes).
-  __device__ __forceinline__ void add(const float4 (&x)[kLaneF4], const int (&idx)[kLaneF4],
-                                      int st) {
+  __device__ __forceinline__ void add(const float4 (&x)[kLaneF4], const int (&idx)[kLaneF4]) {
     float cm = -FLT_MAX;
 #pragma unroll
     for (int u = 0; u < kLaneF4; ++u)
       cm = fmaxf(cm, fmaxf(fmaxf(x[u].x, x[u].y), fmaxf(x[u].z, x[u].w)));
     const bool live = cm > -FLT_MAX;  // false past the end of the range
-    if (live && cm > m) {
+    if (live && cm > m) {  // a new maximum: its first index in this stage
       rescale(cm);
-      mstage = st;
+      int first = 0x7fffffff;
+#pragma unroll
+      for (int u = kLaneF4 - 1; u >= 0; --u) {  // the last hit from the end is the first
+        if (x[u].w == cm) first = idx[u] * 4 + 3;
+        if (x[u].z == cm) first = idx[u] * 4 + 2;
+        if (x[u].y == cm) first = idx[u] * 4 + 1;
+        if (x[u].x == cm) first = idx[u] * 4;
+      }
+      am = first;
     }
     float thr = fmaxf(tl.v[KM - 1], lb);
     if (__any_sync(0xffffffffu, live && cm >= thr)) {
@@ -190,17 +203,14 @@ struct RowAcc {
   }
 };
 
+// Warp-wide best (value desc, index asc) in two warp reductions: the
+// largest order-preserving value code, then the smallest index holding it
+// (-0 and +0 share a code, as they compare equal).
 __device__ __forceinline__ ArgMax warp_best(ArgMax a) {
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    const float ov = __shfl_xor_sync(0xffffffffu, a.v, off);
-    const int oi = __shfl_xor_sync(0xffffffffu, a.i, off);
-    if (better(ov, oi, a.v, a.i)) {
-      a.v = ov;
-      a.i = oi;
-    }
-  }
-  return a;
+  const uint32_t c = score_code(a.v);
+  const uint32_t cm = __reduce_max_sync(0xffffffffu, c);
+  const uint32_t im = __reduce_min_sync(0xffffffffu, c == cm ? (uint32_t)a.i : 0xffffffffu);
+  return ArgMax{code_score(cm), (int)im};
 }
 
 // Bounded wait on an mbarrier phase; false after ~2 s.
@@ -243,7 +253,7 @@ __device__ __forceinline__ float warp_kth(const TopList<KM>& tl, int kappa) {
 
 // Statistics of one segment of a row, merged by the row's last warp.
 struct Partial {
-  double z, s;  // relative to m
+  float z, s;  // relative to m
   float m;
   float bv;
   int bi;
@@ -253,38 +263,38 @@ struct Partial {
 };
 
 // Row statistics from its segment partials, written to out.  Called by a
-// whole warp: lane g holds partial g (segs <= 32), then warp reductions.
-__device__ void finish_row(const Partial* parts, int segs, int vocab, int kappa, float thr,
-                           int unnormalized, int32_t* __restrict__ out) {
+// whole warp: each lane brings one partial (p, or none when p is null),
+// then warp reductions.
+__device__ void finish_row(const Partial* p, int vocab, int kappa, float thr, int unnormalized,
+                           int32_t* __restrict__ out) {
   const int lane = threadIdx.x & 31;
-  const bool has = lane < segs;
+  const bool has = p != nullptr;
   float m = -FLT_MAX, bv = -FLT_MAX;
-  double pz = 0.0, ps = 0.0;
+  float pz = 0.0f, ps = 0.0f;
   int bi = 0x7fffffff;
   float tv[SENSE_MAX_KAPPA];
   int ti[SENSE_MAX_KAPPA];
   if (has) {
-    const Partial& p = parts[lane];
-    m = p.m;
-    pz = p.z;
-    ps = p.s;
-    bv = p.bv;
-    bi = p.bi;
+    m = p->m;
+    pz = p->z;
+    ps = p->s;
+    bv = p->bv;
+    bi = p->bi;
   }
 #pragma unroll
   for (int r = 0; r < SENSE_MAX_KAPPA; ++r) {
-    tv[r] = (has && r < kappa) ? parts[lane].tv[r] : -FLT_MAX;
-    ti[r] = (has && r < kappa) ? parts[lane].ti[r] : 0x7fffffff;
+    tv[r] = (has && r < kappa) ? p->tv[r] : -FLT_MAX;
+    ti[r] = (has && r < kappa) ? p->ti[r] : 0x7fffffff;
   }
   float M = m;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-  double Z = 0.0, Sx = 0.0;
-  if (has && pz > 0.0) {
+  float Z = 0.0f, Sx = 0.0f;
+  if (has && pz > 0.0f) {
     const float d = m - M;
-    const double sc = (double)exp2_ftz(d * kLog2e);
+    const float sc = exp2_ftz(d * kLog2e);
     Z = pz * sc;
-    Sx = sc * (ps + (double)d * pz);
+    Sx = sc * (ps + d * pz);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -307,7 +317,7 @@ __device__ void finish_row(const Partial* parts, int segs, int vocab, int kappa,
     if (hx == w.i && hv == w.v) ++head;
   }
   if (lane == 0) {
-    const float H = logf((float)Z) - (float)(Sx / Z);
+    const float H = logf(Z) - Sx / Z;
     const float score = unnormalized ? H : H / logf((float)vocab);
     out[0] = b.i;
     out[1] = (score > thr) ? 1 : 0;
@@ -393,33 +403,12 @@ __device__ bool warp_segment(const float* __restrict__ row, int lo4, int hi4, in
       }
       acc.lb = b;
     }
-    acc.add(x, idx, i);
-    if (((i + 2) & (i + 1)) == 0 && i < 32)  // after stages 1, 3, 7, 15, 31
+    acc.add(x, idx);
+    if (((i + 2) & (i + 1)) == 0 && i < 32 && i + 1 < n)  // after stages 1, 3, 7, 15, 31
       acc.lb = fmaxf(acc.lb, warp_kth<KM>(acc.tl, kappa));
   }
   seq += (uint32_t)n;
   if (!ok) return false;
-  // argmax: this lane's first maximum, read back from its stage
-  int bi = 0x7fffffff;
-  if (acc.mstage >= 0) {
-    // the lane's float4 of that stage, loaded together (one L2 round trip),
-    // then searched in index order
-    const int f0 = acc.mstage * kWStageF4;
-    float4 v[kLaneF4];
-#pragma unroll
-    for (int u = 0; u < kLaneF4; ++u) {
-      const int j = f0 + lane + 32 * u;
-      v[u] = (j < n4) ? row4[j] : make_float4(-FLT_MAX, -FLT_MAX, -FLT_MAX, -FLT_MAX);
-    }
-#pragma unroll
-    for (int u = kLaneF4 - 1; u >= 0; --u) {  // the last hit from the end is the first
-      const int e = (lo4 + f0 + lane + 32 * u) * 4;
-      if (v[u].w == acc.m) bi = e + 3;
-      if (v[u].z == acc.m) bi = e + 2;
-      if (v[u].y == acc.m) bi = e + 1;
-      if (v[u].x == acc.m) bi = e;
-    }
-  }
   float z0, z1, s0, s1;
   upk(acc.z, z0, z1);
   upk(acc.s, s0, s1);
@@ -428,19 +417,19 @@ __device__ bool warp_segment(const float* __restrict__ row, int lo4, int hi4, in
   float M = acc.m;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-  double z = 0.0, s = 0.0;
+  float z = 0.0f, s = 0.0f;
   if (lz > 0.0f) {  // rescale this lane's sums to the row max
     const float d = acc.m - M;
     const float sc = exp2_ftz(d * kLog2e);
-    z = (double)(lz * sc);
-    s = (double)(sc * (ls + d * lz));
+    z = lz * sc;
+    s = sc * (ls + d * lz);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     z += __shfl_xor_sync(0xffffffffu, z, off);
     s += __shfl_xor_sync(0xffffffffu, s, off);
   }
-  const ArgMax am = warp_best(ArgMax{acc.m, bi});
+  const ArgMax am = warp_best(ArgMax{acc.m, acc.am});
   if (lane == 0) {
     out->z = z;
     out->s = s;
@@ -521,7 +510,7 @@ gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__
     int32_t* out = stats + (int64_t)rid * kStatsInts;
     if (segs == 1) {
       __syncwarp();
-      finish_row(&s_part[wid], 1, vocab, kappa, thr, unnormalized, out);
+      finish_row(lane == 0 ? &s_part[wid] : nullptr, vocab, kappa, thr, unnormalized, out);
     } else {
       // the row's last segment to finish merges the partials
       unsigned last = 0;
@@ -532,11 +521,97 @@ gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__
       last = __shfl_sync(0xffffffffu, last, 0);
       if (last) {
         __threadfence();
-        finish_row(parts + (int64_t)rid * segs, segs, vocab, kappa, thr, unnormalized, out);
+        finish_row(lane < segs ? parts + (int64_t)rid * segs + lane : nullptr, vocab, kappa, thr,
+                   unnormalized, out);
         if (lane == 0) done[rid] = 0u;
       }
     }
     __syncwarp();
+  }
+}
+
+// Few rows with short slices: NC blocks per row (a cluster of NC blocks
+// when NC > 1), whose kWarps * NC warps stream consecutive slices of seg4
+// float4 each through their own rings.  Each block keeps its warps'
+// partials in shared memory; warp 0 of the cluster's first block merges
+// them all, reading the other block's partials through distributed shared
+// memory.  No task counter, no partials in global memory, no grid-wide
+// atomics: the row's latency is one streaming pass plus block and cluster
+// barriers.
+template <int KM, int NC>
+__global__ void __launch_bounds__(kRowThreads, 1)
+gate_row_block_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ num_nodes,
+                      int cap, const float* __restrict__ root_logits,
+                      const float* __restrict__ node_logits, int vocab, int kappa, float thr,
+                      int unnormalized, int seg4, int32_t* __restrict__ stats, uint32_t* status) {
+  static_assert(NC >= 1 && NC * kWarps <= 32, "one merging warp holds every partial");
+  extern __shared__ __align__(128) float4 ring_all[];
+  __shared__ __align__(8) uint64_t bars_all[kWarps * kWStages];
+  __shared__ Partial s_part[kWarps];
+  __shared__ int s_fail;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int rid = blockIdx.x / NC;  // q * (cap + 1) + slot
+  const int crank = blockIdx.x - rid * NC;  // rank in the cluster (clusters of NC along x)
+  const int q = rid / (cap + 1);
+  const int slot = rid - q * (cap + 1);  // 0 = root, 1 + n = node n
+  const float* row;
+  if (slot == 0) {
+    row = root_logits + (int64_t)q * vocab;
+  } else {
+    const int nd = slot - 1;
+    const int nn = min(num_nodes[q], cap);
+    const bool inner = (nd + 1 < nn) && parent[(int64_t)q * cap + nd + 1] == nd;
+    if (!inner) return;  // depends on the row only: the whole cluster leaves
+    row = node_logits + ((int64_t)q * cap + nd) * vocab;
+  }
+  if (threadIdx.x == 0) {
+    for (int b = 0; b < kWarps * kWStages; ++b) ptx::mbar_init(ptx::smem_u32(bars_all + b), 1);
+    ptx::fence_barrier_init();
+    s_fail = 0;
+  }
+  __syncthreads();
+  const int n4 = vocab >> 2;
+  const int lo4 = min(n4, (crank * kWarps + wid) * seg4);
+  const int hi4 = min(n4, lo4 + seg4);
+  if (lo4 < hi4) {
+    float4* ring = ring_all + (size_t)wid * kWStages * kWStageF4;
+    uint64_t* bars = bars_all + wid * kWStages;
+    const uint64_t pol = (lane == 0) ? ptx::policy_evict_first() : 0ull;
+    uint32_t seq = 0;
+    if (!warp_segment<KM>(row, lo4, hi4, kappa, ring, bars, seq, pol, &s_part[wid])) {
+      if (lane == 0) {
+        raise_status(status, SENSE_DEVST_TIMEOUT);
+        s_fail = 1;
+      }
+    }
+  } else if (lane == 0) {  // empty slice: a neutral partial
+    Partial& p = s_part[wid];
+    p.z = 0.0f;
+    p.s = 0.0f;
+    p.m = -FLT_MAX;
+    p.bv = -FLT_MAX;
+    p.bi = 0x7fffffff;
+    for (int r = 0; r < SENSE_MAX_KAPPA; ++r) {
+      p.tv[r] = -FLT_MAX;
+      p.ti[r] = 0x7fffffff;
+    }
+  }
+  int32_t* out = stats + (int64_t)rid * kStatsInts;
+  if constexpr (NC == 1) {
+    __syncthreads();
+    if (wid == 0 && !s_fail)
+      finish_row(lane < kWarps ? &s_part[lane] : nullptr, vocab, kappa, thr, unnormalized, out);
+  } else {
+    cg::cluster_group cl = cg::this_cluster();
+    cl.sync();  // every block's partials (and failure flag) are written
+    if (crank == 0 && wid == 0) {
+      const int src = lane / kWarps;  // block holding this lane's partial
+      const Partial* pp = cl.map_shared_rank(&s_part[lane - src * kWarps], src);
+      bool fail = false;
+      for (int r = 0; r < NC; ++r) fail |= *cl.map_shared_rank(&s_fail, r) != 0;
+      if (!fail) finish_row(lane < NC * kWarps ? pp : nullptr, vocab, kappa, thr, unnormalized, out);
+    }
+    cl.sync();  // the other blocks' shared memory stays alive until it is read
   }
 }
 
@@ -737,20 +812,57 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
   ws += align256(rows * kStatsInts * sizeof(int32_t));
   unsigned* next_task = reinterpret_cast<unsigned*>(ws);
   ws += 256;
-  const int segs = gate_segments(a.q, a.cap, a.vocab);
   const int n4 = a.vocab >> 2;
-  const int seg4 = (n4 + segs - 1) / segs;
-  Partial* parts = reinterpret_cast<Partial*>(ws);
-  unsigned* done = nullptr;
-  if (segs > 1) done = reinterpret_cast<unsigned*>(ws + align256(rows * segs * sizeof(Partial)));
-  sense_status st = cuda_check(cudaMemsetAsync(next_task, 0, sizeof(unsigned), s),
-                               "clear gate task counter");
-  if (st != SENSE_OK) return st;
-  if (segs > 1) {
-    st = cuda_check(cudaMemsetAsync(done, 0, rows * sizeof(unsigned), s), "clear gate counters");
+  sense_status st = SENSE_OK;
+  // Few rows, each warp's slice inside its ring: blocks per row (two as a
+  // cluster when the rows leave room for it).
+  const int64_t sms = sm_count();
+  const bool pair = 2 * (int64_t)rows <= sms &&
+                    (n4 + 2 * kWarps - 1) / (2 * kWarps) <= kWStages * kWStageF4;
+  const bool single = (int64_t)rows <= sms && (n4 + kWarps - 1) / kWarps <= kWStages * kWStageF4;
+  if (pair || single) {
+    const int nc = pair ? 2 : 1;
+    const int slice4 = (n4 + nc * kWarps - 1) / (nc * kWarps);
+    void (*kern)(const int32_t*, const int32_t*, int, const float*, const float*, int, int, float,
+                 int, int, int32_t*, uint32_t*);
+    if (pair) kern = (a.kappa <= 4) ? gate_row_block_kernel<4, 2>
+                                     : gate_row_block_kernel<SENSE_MAX_KAPPA, 2>;
+    else kern = (a.kappa <= 4) ? gate_row_block_kernel<4, 1>
+                               : gate_row_block_kernel<SENSE_MAX_KAPPA, 1>;
+    st = cuda_check(
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kRingBytes),
+        "cudaFuncSetAttribute(gate_row_block)");
     if (st != SENSE_OK) return st;
-  }
-  {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(rows * nc));
+    cfg.blockDim = dim3(kRowThreads);
+    cfg.dynamicSmemBytes = kRingBytes;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)nc;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    LaunchScope ls(K_GATE_ROWS, s);
+    st = cuda_check(cudaLaunchKernelEx(&cfg, kern, a.parent, a.num_nodes, a.cap, a.root_logits,
+                                       a.node_logits, a.vocab, a.kappa, a.thr, a.unnormalized,
+                                       slice4, stats, a.status),
+                    "launch gate_row_block");
+    if (st != SENSE_OK) return st;
+  } else {
+    const int segs = gate_segments(a.q, a.cap, a.vocab);
+    const int seg4 = (n4 + segs - 1) / segs;
+    Partial* parts = reinterpret_cast<Partial*>(ws);
+    unsigned* done = nullptr;
+    if (segs > 1) done = reinterpret_cast<unsigned*>(ws + align256(rows * segs * sizeof(Partial)));
+    st = cuda_check(cudaMemsetAsync(next_task, 0, sizeof(unsigned), s), "clear gate task counter");
+    if (st != SENSE_OK) return st;
+    if (segs > 1) {
+      st = cuda_check(cudaMemsetAsync(done, 0, rows * sizeof(unsigned), s), "clear gate counters");
+      if (st != SENSE_OK) return st;
+    }
     auto k4 = gate_rows_kernel<4>;
     auto k16 = gate_rows_kernel<SENSE_MAX_KAPPA>;
     auto kern = (a.kappa <= 4) ? k4 : k16;

@@ -21,6 +21,7 @@
 //    memory, become the output scores and indices.
 #include "common.cuh"
 #include "launch.h"
+#include "tc_ptx.cuh"
 
 namespace sense {
 namespace {
@@ -272,7 +273,139 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
 // each hold a key >= T), so only list prefixes >= T are candidates; they are
 // gathered into shared memory, selected and sorted.  If the gathered set
 // would not fit, every key of every list is used instead.
+//
+// Small merges (the lists fit in kFastKeys keys, at most kRankHeads lists)
+// take a short path: one bulk copy brings every list into shared memory, T
+// is the head of rank k - 1 (ranks counted against warp-sorted groups of
+// heads by binary search), and each gathered candidate's rank among the
+// candidates is its output slot, so no radix passes or block-wide sorting
+// network run.  Nonzero keys are distinct (a key row lives in one list),
+// which makes the ranks a permutation.
 constexpr int kGather = 4096;
+constexpr int kFastKeys = 20480;   // list keys staged by the short path (160 KB)
+constexpr int kFastCand = 1024;    // candidates it ranks
+constexpr int kRankHeads = 1024;   // lists it ranks
+constexpr long long kCopyWaitCycles = 4000000000LL;
+
+__device__ __forceinline__ bool wait_copy(uint32_t bar) {
+  if (ptx::mbar_try_wait(bar, 0)) return true;
+  const long long t0 = clock64();
+  while (!ptx::mbar_try_wait(bar, 0)) {
+    if (clock64() - t0 > kCopyWaitCycles) return false;
+  }
+  return true;
+}
+
+// The short path; returns false (block-uniform) when the candidates do not
+// suit it, leaving the general path to run.  On a timed-out copy it marks the
+// outputs and status and returns true.
+__device__ bool merge_lists_short(const uint64_t* __restrict__ src, int nlists, int k,
+                                  float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
+                                  uint32_t* status, uint64_t* s_keys) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ uint64_t s_t;
+  __shared__ unsigned s_got;
+  __shared__ int s_ok;
+  uint64_t* s_cand = s_keys + kFastKeys;
+  uint64_t* s_grp = s_cand + kFastCand;  // heads in sorted groups of 32
+  const int total = nlists * k;
+  const uint32_t b = ptx::smem_u32(&bar);
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(b, 1);
+    ptx::fence_barrier_init();
+    const uint32_t bytes = (uint32_t)total * 8u;
+    ptx::mbar_arrive_expect_tx(b, bytes);
+    const uint64_t pol = ptx::policy_evict_first();
+    for (uint32_t off = 0; off < bytes; off += 32768u)
+      ptx::bulk_load(ptx::smem_u32(s_keys) + off, reinterpret_cast<const char*>(src) + off,
+                     min(32768u, bytes - off), b, pol);
+    s_t = 0ull;
+    s_got = 0u;
+  }
+  __syncthreads();
+  const bool arrived = wait_copy(b);
+  if (!__syncthreads_and(arrived)) {
+    if (threadIdx.x == 0) {
+      raise_status(status, SENSE_DEVST_TIMEOUT);
+      wait_copy(b);  // give the copy a second bound before the block leaves
+    }
+    for (int r = threadIdx.x; r < k; r += blockDim.x) {
+      out_scores[r] = 0.0f;
+      out_idx[r] = -1;
+    }
+    __syncthreads();
+    return true;
+  }
+  // T: the k-th largest nonzero head (0 when fewer than k heads are
+  // nonzero; nonzero keys are distinct).  Heads are cut into groups of 32,
+  // each sorted (descending) by one warp with a bitonic network over
+  // shuffles; a head's rank is the sum over groups of the heads above it,
+  // found by binary search.
+  if (nlists >= k) {
+    const int lane = threadIdx.x & 31;
+    const int ngroups = (nlists + 31) >> 5;
+    for (int g = threadIdx.x >> 5; g < ngroups; g += blockDim.x >> 5) {
+      const int i = g * 32 + lane;
+      uint64_t h = (i < nlists) ? s_keys[(int64_t)i * k] : 0ull;
+#pragma unroll
+      for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+          const uint64_t o = __shfl_xor_sync(0xffffffffu, h, stride);
+          const bool keep_max = ((lane & stride) == 0) == ((lane & size) == 0);
+          h = keep_max ? (h > o ? h : o) : (h < o ? h : o);
+        }
+      }
+      s_grp[i] = h;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < nlists; i += blockDim.x) {
+      const uint64_t h = s_keys[(int64_t)i * k];
+      if (h == 0ull) continue;
+      int rank = 0;
+      for (int g = 0; g < ngroups; ++g) {
+        const uint64_t* grp = s_grp + g * 32;
+        // heads of group g above h (a prefix, the group being descending):
+        // the longest prefix of at most 31 found by halving steps, then slot 31
+        int lo = 0;
+#pragma unroll
+        for (int step = 16; step > 0; step >>= 1)
+          if (grp[lo + step - 1] > h) lo += step;
+        rank += lo + ((lo == 31 && grp[31] > h) ? 1 : 0);
+      }
+      if (rank == k - 1) s_t = h;
+    }
+  }
+  __syncthreads();
+  const uint64_t t = s_t;
+  for (int l = threadIdx.x; l < nlists; l += blockDim.x) {
+    const uint64_t* lb = s_keys + (int64_t)l * k;
+    for (int r = 0; r < k; ++r) {
+      const uint64_t c = lb[r];
+      if (c < t || c == 0ull) break;
+      const unsigned p = atomicAdd(&s_got, 1u);
+      if (p < (unsigned)kFastCand) s_cand[p] = c;
+    }
+  }
+  __syncthreads();
+  const int got = (int)s_got;
+  if (threadIdx.x == 0) s_ok = (got >= k && got <= kFastCand);
+  __syncthreads();
+  if (!s_ok) return false;
+  for (int i = threadIdx.x; i < got; i += blockDim.x) {
+    const uint64_t c = s_cand[i];
+    int rank = 0;
+    for (int j = 0; j < got; ++j) {
+      const uint64_t o = s_cand[j];
+      rank += (o > c) || (o == c && j < i);
+    }
+    if (rank < k) {
+      out_scores[rank] = code_score((uint32_t)(c >> 32));
+      out_idx[rank] = (int32_t)cand_index(c);
+    }
+  }
+  return true;
+}
 
 __global__ void __launch_bounds__(kSelThreads, 1)
 merge_lists_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
@@ -285,6 +418,12 @@ merge_lists_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
   __shared__ uint64_t sel[SENSE_MAX_K];
   const int q = blockIdx.x;
   const uint64_t* src = lists + (int64_t)q * nlists * k;
+  if ((int64_t)nlists * k <= kFastKeys && nlists <= kRankHeads && ((nlists * k) & 1) == 0 &&
+      (reinterpret_cast<uintptr_t>(src) & 15) == 0) {
+    if (merge_lists_short(src, nlists, k, out_scores + (int64_t)q * k, out_idx + (int64_t)q * k,
+                          status, s_keys))
+      return;
+  }
   // 1. lower bound from the list heads
   for (int b = threadIdx.x; b < nlists; b += blockDim.x) s_keys[b] = src[(int64_t)b * k];
   __syncthreads();
@@ -404,7 +543,7 @@ sense_status launch_merge_lists(const uint64_t* lists, int nlists, int q, int k,
   sense_status st = set_smem(merge_lists_kernel, kSmemKeys * sizeof(uint64_t));
   if (st != SENSE_OK) return st;
   LaunchScope ls(K_MERGE, s);
-  merge_lists_kernel<<<q, 256, kSmemKeys * sizeof(uint64_t), s>>>(
+  merge_lists_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(
       lists, nlists, k, out_scores, out_idx, status);
   return cuda_check(cudaGetLastError(), "launch merge_lists");
 }

@@ -309,6 +309,9 @@ def _gate_case(q, k, m, v, d, cap, seed, plant=True):
     (2, 32, 16, 32000, 64, 0.01, 2, 9, 0, False),
     (2, 8, 4, 512, 0, 1.5, 4, 2, 0, True),
     (2, 3, 16, 128, 0, -1.0, 16, 1, 0, False),
+    (1, 32, 16, 32000, 64, 0.05, 3, 6, 0, False),   # one query: two blocks per row
+    (1, 4, 4, 64, 0, 0.5, 16, 3, 1, False),         # slices of one float4, empty slices
+    (1, 16, 8, 40000, 0, 0.05, 5, 4, 0, False),     # one block per row, three stages a warp
 ])
 def test_gate_matches_oracle(S, q, k, m, v, cap, gamma, kappa, w, tau, unnorm):
     dev = torch.device("cuda")
