@@ -47,7 +47,7 @@ NCU_TRAFFIC_PER_UNIT = {
     # 524,288 x 3584 keys, sample + rest launches of one step
     ("scan_tc", 3584): (235048448 + 2988800 + 3523437824 + 185600) / 524288,
     # 4 queries of the k = 64 sweep: 3,774 root / inner-node rows of 128,256 logits
-    ("gate_rows", 128256): (2055664000 + 3651840) / 3773.9375,
+    ("gate_rows", 128256): (1939918336 + 3338240) / 3773.9375,
 }
 
 

@@ -399,17 +399,21 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     float* po = a.part_o + pbase * kHd + half * (kHd / 2);
     const bool done =
         __all_sync(0xffffffffu, ok && nbl > 0 && wait_bar(bar(MMA_DONE), 0, abort, a.status));
-    if (done) {
+    if (done && q4 * 32 < a.L) {  // rows past L are padding: not written
       ptx::tc_fence_after();
-#pragma unroll 1
-      for (int c = 0; c < kHd / 2 / 16; ++c) {
-        uint32_t rr[16];
-        ptx::tmem_ld16(lane_base + 2 * kBN + half * (kHd / 2) + 16 * c, rr);
+      uint32_t rr[kHd / 2 / 16][16];
 #pragma unroll
-        for (int e = 0; e < 16; e += 4)
-          *reinterpret_cast<float4*>(po + 16 * c + e) =
-              make_float4(__uint_as_float(rr[e]), __uint_as_float(rr[e + 1]),
-                          __uint_as_float(rr[e + 2]), __uint_as_float(rr[e + 3]));
+      for (int c = 0; c < kHd / 2 / 16; ++c)
+        ptx::tmem_ld16_nowait(lane_base + 2 * kBN + half * (kHd / 2) + 16 * c, rr[c]);
+      ptx::tmem_ld_wait();
+      if (r < a.L) {
+#pragma unroll
+        for (int c = 0; c < kHd / 2 / 16; ++c)
+#pragma unroll
+          for (int e = 0; e < 16; e += 4)
+            *reinterpret_cast<float4*>(po + 16 * c + e) =
+                make_float4(__uint_as_float(rr[c][e]), __uint_as_float(rr[c][e + 1]),
+                            __uint_as_float(rr[c][e + 2]), __uint_as_float(rr[c][e + 3]));
       }
     }
     // every product is done (or the CTA aborted): P buffer 0 is free; the row

@@ -190,6 +190,110 @@ threshold_kernel(const uint64_t* __restrict__ lists, int64_t len, int k,
   }
 }
 
+// Short path of merge_kernel for a pool staged in shared memory (distinct
+// nonzero keys, at most 32 * kPoolGroups of them).  The pool is cut into
+// groups of 32; a group's maximum is a head, and the k-th largest head T
+// bounds the k-th largest key from below (k groups hold a key >= T).  Heads
+// are ranked against warp-sorted groups of heads by binary search; the keys
+// >= T (a few dozen for a random pool) are then placed by their rank among
+// themselves.  Returns false (block-uniform) when the candidates do not
+// suit it, leaving the radix path to run.
+constexpr int kPoolGroups = 1024;  // heads ranked by the short path
+constexpr int kPoolCand = 512;     // candidates placed by rank (in `sel`), O(c^2 / threads)
+constexpr int kPoolAll = 256;      // pools this small are ranked whole
+
+__device__ __forceinline__ uint64_t warp_max64(uint64_t x) {
+  // distinct keys: the largest high word, then the largest low word under it
+  const uint32_t hi = (uint32_t)(x >> 32);
+  const uint32_t hm = __reduce_max_sync(0xffffffffu, hi);
+  const uint32_t lm = __reduce_max_sync(0xffffffffu, hi == hm ? (uint32_t)x : 0u);
+  return ((uint64_t)hm << 32) | lm;
+}
+
+__device__ bool merge_pool_short(const uint64_t* s_keys, int cnt, int k, int pad_short,
+                                 uint64_t* cand, float* __restrict__ out_scores,
+                                 int32_t* __restrict__ out_idx) {
+  __shared__ uint64_t s_heads[kPoolGroups];  // group maxima, then sorted in groups of 32
+  __shared__ uint64_t s_t;
+  __shared__ unsigned s_got;
+  __shared__ int s_ok;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  const int ngr = (cnt + 31) >> 5;
+  if (threadIdx.x == 0) {
+    s_t = 0ull;
+    s_got = 0u;
+  }
+  // heads: group maxima, sorted descending within each group of 32 heads
+  const int nhg = (ngr + 31) >> 5;
+  for (int hg = warp; hg < nhg; hg += nwarps) {
+    uint64_t h = 0ull;  // the maximum of group hg * 32 + lane
+    for (int u = 0; u < 32; ++u) {  // group g's keys, read across the warp by lane u's group
+      const int gu = hg * 32 + u;
+      const int i = gu * 32 + lane;
+      const uint64_t x = (gu < ngr && i < cnt) ? s_keys[i] : 0ull;
+      const uint64_t m = warp_max64(x);
+      if (lane == u) h = m;
+    }
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        const uint64_t o = __shfl_xor_sync(0xffffffffu, h, stride);
+        const bool keep_max = ((lane & stride) == 0) == ((lane & size) == 0);
+        h = keep_max ? (h > o ? h : o) : (h < o ? h : o);
+      }
+    }
+    s_heads[hg * 32 + lane] = h;
+  }
+  __syncthreads();
+  // T: the head of rank k - 1 among the nonzero heads (0 when fewer than k)
+  for (int i = threadIdx.x; i < nhg * 32; i += blockDim.x) {
+    const uint64_t h = s_heads[i];
+    if (h == 0ull) continue;
+    int rank = 0;
+    for (int hg = 0; hg < nhg; ++hg) {
+      const uint64_t* grp = s_heads + hg * 32;
+      int lo = 0;
+#pragma unroll
+      for (int step = 16; step > 0; step >>= 1)
+        if (grp[lo + step - 1] > h) lo += step;
+      rank += lo + ((lo == 31 && grp[31] > h) ? 1 : 0);
+    }
+    if (rank == k - 1) s_t = h;
+  }
+  __syncthreads();
+  const uint64_t t = s_t;
+  for (int i = threadIdx.x; i < cnt; i += blockDim.x) {
+    const uint64_t c = s_keys[i];
+    if (c != 0ull && c >= t) {
+      const unsigned p = atomicAdd(&s_got, 1u);
+      if (p < (unsigned)kPoolCand) cand[p] = c;
+    }
+  }
+  __syncthreads();
+  const int got = (int)s_got;
+  if (threadIdx.x == 0) s_ok = got <= kPoolCand && (got >= k || pad_short);
+  __syncthreads();
+  if (!s_ok) return false;
+  for (int i = threadIdx.x; i < got; i += blockDim.x) {
+    const uint64_t c = cand[i];
+    int rank = 0;
+    for (int j = 0; j < got; ++j) {
+      const uint64_t o = cand[j];
+      rank += (o > c) || (o == c && j < i);
+    }
+    if (rank < k) {
+      out_scores[rank] = code_score((uint32_t)(c >> 32));
+      out_idx[rank] = (int32_t)cand_index(c);
+    }
+  }
+  for (int r = got + threadIdx.x; r < k; r += blockDim.x) {  // a short pool: -inf, -1
+    out_scores[r] = -__int_as_float(0x7f800000);
+    out_idx[r] = -1;
+  }
+  return true;
+}
+
 __global__ void __launch_bounds__(kSelThreads, 1)
 merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
              int64_t pool_cap, int k, float* __restrict__ out_scores,
@@ -208,6 +312,12 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
     for (int64_t i = threadIdx.x; i < cnt; i += blockDim.x) s_keys[i] = src[i];
     __syncthreads();
   }
+  // the short path needs a pruning threshold (k group heads) or a tiny pool
+  if (staged && cnt > 0 && cnt <= 32 * kPoolGroups &&
+      (cnt <= kPoolAll || (cnt + 31) / 32 >= (int64_t)k) &&
+      merge_pool_short(s_keys, (int)cnt, k, pad_short, sel, out_scores + (int64_t)q * k,
+                       out_idx + (int64_t)q * k))
+    return;
   auto get = [&](int64_t i) { return staged ? s_keys[i] : src[i]; };
   uint64_t prefix, pmask;
   bool ok = radix_select(get, cnt, k, 0, hist, &dig, &prefix, &pmask);
