@@ -26,7 +26,9 @@
 //  2. gate_decide: one block per query evaluates B_em, B_ent, B_topk, the
 //     lookahead B_con, G, the accepted prefix lengths L_i, i*, and writes
 //     the accepted tokens, the next node, its argmax (streaming that row if
-//     it is a leaf) and h_next.
+//     it is a leaf) and h_next.  When they fit, the query's Gamma, tokens,
+//     parents and row statistics are first staged in shared memory with
+//     independent loads, so that the block pays one round trip for them.
 #include <cooperative_groups.h>
 #include <float.h>
 
@@ -617,18 +619,62 @@ gate_row_block_kernel(const int32_t* __restrict__ parent, const int32_t* __restr
 
 constexpr int kDecideThreads = 1024;
 
+// Shared memory of a staged decide block: Gamma, tokens, parents and the
+// row statistics of one query, then the flags.
+size_t decide_stage_bytes(int k, int m, int cap) {
+  return sizeof(int32_t) * ((size_t)k * m + 2 * (size_t)cap + (size_t)(cap + 1) * kStatsInts) +
+         (size_t)k * m;
+}
+constexpr size_t kDecideStageMax = 96 * 1024;
+
+// 4-byte asynchronous global -> shared copy (no register round trip: every
+// copy of a thread is in flight at once); cp_async_wait_all() completes them.
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(ptx::smem_u32(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
 __global__ void __launch_bounds__(kDecideThreads)
-gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats) {
-  extern __shared__ uint8_t s_flags[];  // [k*m]: bit0 valid, bit1 em, bit2 ent, bit3 topk, bit4 G
+gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats, int staged) {
+  // dynamic: staged ? [Gamma k*m][tokens cap][parents cap][stats (cap+1) rows] : nothing,
+  // then flags [k*m]: bit0 valid, bit1 em, bit2 ent, bit3 topk, bit4 G
+  extern __shared__ __align__(16) int32_t s_dyn[];
   __shared__ int s_L[SENSE_MAX_K];
   __shared__ int s_best[32];
-  __shared__ int s_istar, s_lstar, s_next;
+  __shared__ int s_istar, s_lstar, s_next, s_nn;
   __shared__ ArgMax s_w[32];
   const int q = blockIdx.x;
   const int k = a.k, m = a.m, cap = a.cap, km = k * m;
   const int32_t* gam = a.gamma + (int64_t)q * km;
   const int32_t* tok = a.tokens + (int64_t)q * cap;
+  const int32_t* par = a.parent + (int64_t)q * cap;
   const int32_t* st = stats + (int64_t)q * (cap + 1) * kStatsInts;
+  uint8_t* s_flags = reinterpret_cast<uint8_t*>(s_dyn);
+  if (staged) {  // one round trip for everything the block reads more than once
+    int32_t* sg = s_dyn;
+    int32_t* stk = sg + km;
+    int32_t* spr = stk + cap;
+    int32_t* sst = spr + cap;
+    for (int i = threadIdx.x; i < km; i += blockDim.x) cp_async4(sg + i, gam + i);
+    for (int i = threadIdx.x; i < cap; i += blockDim.x) {
+      cp_async4(stk + i, tok + i);
+      cp_async4(spr + i, par + i);
+    }
+    for (int i = threadIdx.x; i < (cap + 1) * kStatsInts; i += blockDim.x) cp_async4(sst + i, st + i);
+    if (threadIdx.x == 0) cp_async4(&s_nn, a.num_nodes + q);
+    cp_async_wait_all();
+    s_flags = reinterpret_cast<uint8_t*>(sst + (cap + 1) * kStatsInts);
+    gam = sg;
+    tok = stk;
+    par = spr;
+    st = sst;
+    __syncthreads();
+  } else if (threadIdx.x == 0) {
+    s_nn = a.num_nodes[q];
+  }
 
   for (int e = threadIdx.x; e < km; e += blockDim.x) {
     const int j = e % m;
@@ -732,8 +778,8 @@ gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats) {
     for (int i = threadIdx.x; i < (a.d >> 3); i += blockDim.x) o4[i] = h4[i];
   }
   // next anchor: argmax of the next node's logits row.
-  const int nn = min(a.num_nodes[q], cap);
-  const bool have = (nxt < 0) || ((nxt + 1 < nn) && a.parent[(int64_t)q * cap + nxt + 1] == nxt);
+  const int nn = min(s_nn, cap);
+  const bool have = (nxt < 0) || ((nxt + 1 < nn) && par[nxt + 1] == nxt);
   if (have) {
     if (threadIdx.x == 0) a.next_anchor[q] = st[(int64_t)(nxt + 1) * kStatsInts];
     return;
@@ -881,10 +927,18 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     st = cuda_check(cudaGetLastError(), "launch gate_rows");
     if (st != SENSE_OK) return st;
   }
-  const size_t smem = (size_t)a.k * a.m;
+  const size_t staged_smem = decide_stage_bytes(a.k, a.m, a.cap);
+  const int staged = staged_smem <= kDecideStageMax ? 1 : 0;
+  const size_t smem = staged ? staged_smem : (size_t)a.k * a.m;
+  if (smem > 48 * 1024) {
+    st = cuda_check(cudaFuncSetAttribute(gate_decide_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                    "cudaFuncSetAttribute(gate_decide)");
+    if (st != SENSE_OK) return st;
+  }
   LaunchScope ls(K_GATE_DECIDE, s);
   const int threads = (a.k * a.m <= 4096) ? 256 : kDecideThreads;
-  gate_decide_kernel<<<a.q, threads, smem, s>>>(a, stats);
+  gate_decide_kernel<<<a.q, threads, smem, s>>>(a, stats, staged);
   return cuda_check(cudaGetLastError(), "launch gate_decide");
 }
 
