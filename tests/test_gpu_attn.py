@@ -40,6 +40,8 @@ def _tree(seed, k, m_span, vocab, cap):
 @pytest.mark.parametrize("heads,k,m_span,cap,prefix,capacity", [
     (2, 3, 3, 8, 5, 128), (4, 16, 8, 64, 300, 512), (32, 32, 16, 128, 3968, 4096),
     (3, 1, 1, 1, 0, 128), (8, 24, 8, 100, 1000, 1152), (1, 40, 16, 128, 130, 384),
+    (4, 32, 16, 64, 2000, 2176),   # exactly 64 draft tokens (two lane quarters)
+    (4, 32, 16, 65, 2000, 2176),   # one row into the third quarter
 ])
 def test_tree_attention_matches_oracle(S, heads, k, m_span, cap, prefix, capacity):
     dev = torch.device("cuda")
