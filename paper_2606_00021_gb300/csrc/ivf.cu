@@ -548,22 +548,21 @@ __global__ void residual_kernel(const float* __restrict__ x, int64_t n, int v,
 // ---------------------------------------------------------------------------
 
 // PQ lookup table of each query: lut[qi][m][b] = <q_m, B_m[b]> (dsub terms in
-// index order).  One block per query; shared by all of its probe blocks.
+// index order).  One block per (sub-quantizer m, query), one thread per
+// codeword b: every codeword row is loaded at once (one round trip).
 __global__ void __launch_bounds__(256)
 pq_lut_kernel(const float* __restrict__ queries, int v, const float* __restrict__ cb, int pq_m,
               int dsub, float* __restrict__ lut) {
   __shared__ float sq[128];
-  const int qi = blockIdx.x;
-  for (int j = threadIdx.x; j < v; j += blockDim.x) sq[j] = queries[(int64_t)qi * v + j];
+  const int m = blockIdx.x, qi = blockIdx.y;
+  for (int j = threadIdx.x; j < dsub; j += blockDim.x)
+    sq[j] = queries[(int64_t)qi * v + m * dsub + j];
   __syncthreads();
-  float* out = lut + (int64_t)qi * pq_m * 256;
-  for (int e = threadIdx.x; e < pq_m * 256; e += blockDim.x) {
-    const int m = e >> 8;
-    const float* bb = cb + (int64_t)e * dsub;
-    float s = 0.0f;
-    for (int j = 0; j < dsub; ++j) s = madd(s, sq[m * dsub + j], bb[j]);
-    out[e] = s;
-  }
+  const int e = m * 256 + threadIdx.x;  // blockDim.x == 256 codewords
+  const float* bb = cb + (int64_t)e * dsub;
+  float s = 0.0f;
+  for (int j = 0; j < dsub; ++j) s = madd(s, sq[j], bb[j]);
+  lut[(int64_t)qi * pq_m * 256 + e] = s;
 }
 
 constexpr int kScanThreads = 256;
@@ -981,7 +980,8 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
   }
   if (ix->pq_m > 0) {
     LaunchScope ls(K_IVF_COARSE, s);
-    pq_lut_kernel<<<q, 256, 0, s>>>(queries, ix->v, ix->codebooks, ix->pq_m, ix->dsub, lut);
+    pq_lut_kernel<<<dim3(ix->pq_m, q), 256, 0, s>>>(queries, ix->v, ix->codebooks, ix->pq_m,
+                                                     ix->dsub, lut);
     st = cuda_check(cudaGetLastError(), "launch pq lut");
     if (st != SENSE_OK) return st;
   }
