@@ -16,6 +16,11 @@
 //  - k-means sums are 2^-31 fixed-point integers (order-free atomics),
 //    divided in fp64.
 // Kernels:
+//  project_bulk_kernel   one or a few query rows: x, the mean and each
+//                        warp's row of W arrive by one bulk copy each, one
+//                        warp per output; with normalisation the row's
+//                        blocks form a cluster and block 0 normalises the
+//                        gathered outputs (distributed shared memory)
 //  project_rows_kernel   row staged in shared memory, one warp per output:
 //                        query batches
 //  project_tile_kernel   16 rows x 32 outputs per block, 16 warps, each lane
@@ -33,11 +38,14 @@
 //  ivf_scan_kernel       one block per (probe, query): flat dot products or
 //                        LUT sums, candidates appended to the query's pool;
 //                        the exact top-k of the pool is the existing merge.
+#include <cooperative_groups.h>
+
 #include <algorithm>
 #include <vector>
 
 #include "common.cuh"
 #include "launch.h"
+#include "tc_ptx.cuh"
 
 struct sense_ivf {
   int64_t n;
@@ -89,6 +97,116 @@ __device__ __forceinline__ float4 load_x4(const uint16_t* xr, const float* mu, i
   }
   return x;
 }
+
+constexpr long long kBulkWaitCycles = 4000000000LL;
+
+// Block (output group of 8, row): the row of x (bf16), the mean and the W
+// rows of the block's outputs are brought in by one bulk copy each on one
+// mbarrier, so the block pays a single round trip; warp w then computes
+// output 8 * blockIdx.x + w from shared memory in the order of
+// project_rows_kernel (lane l: its 4-column groups ascending; butterfly).
+// NORM: the blocks of a row are one cluster (gridDim.x <= 8); block 0
+// gathers the v outputs through distributed shared memory and writes the
+// row divided by its L2 norm, in the order of normalize_rows_kernel.  A
+// copy that never lands (bounded wait) sets SENSE_DEVST_TIMEOUT; the row is
+// then left unwritten.
+template <bool NORM>
+__global__ void __launch_bounds__(256)
+project_bulk_kernel(const uint16_t* __restrict__ x, int d, const float* __restrict__ w, int v,
+                    const float* __restrict__ mu, float* __restrict__ out, uint32_t* status) {
+  extern __shared__ __align__(128) uint8_t smb[];
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ float s_out[8];
+  __shared__ int s_fail;
+  uint16_t* sxb = reinterpret_cast<uint16_t*>(smb);                   // [d]
+  float* smu = reinterpret_cast<float*>(smb + (size_t)d * 2);         // [d] when mu
+  float* sw = smu + (mu ? d : 0);                                     // [8][d]
+  const int64_t row = blockIdx.y;
+  const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int o = blockIdx.x * 8 + wid;
+  const int nw = min(8, v - (int)blockIdx.x * 8);
+  const uint32_t b = ptx::smem_u32(&bar);
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(b, 1);
+    ptx::fence_barrier_init();
+    s_fail = 0;
+    const uint32_t bytes = (uint32_t)d * 2u + (mu ? (uint32_t)d * 4u : 0u) + (uint32_t)nw * d * 4u;
+    ptx::mbar_arrive_expect_tx(b, bytes);
+    const uint64_t pol = ptx::policy_evict_first();
+    ptx::bulk_load(ptx::smem_u32(sxb), x + row * d, (uint32_t)d * 2u, b, pol);
+    if (mu) ptx::bulk_load(ptx::smem_u32(smu), mu, (uint32_t)d * 4u, b, pol);
+    for (int k = 0; k < nw; ++k)
+      ptx::bulk_load(ptx::smem_u32(sw + (size_t)k * d), w + (int64_t)(blockIdx.x * 8 + k) * d,
+                     (uint32_t)d * 4u, b, pol);
+  }
+  __syncthreads();
+  bool got = ptx::mbar_try_wait(b, 0);
+  if (!got) {
+    const long long t0 = clock64();
+    while (!(got = ptx::mbar_try_wait(b, 0)) && clock64() - t0 <= kBulkWaitCycles) {
+    }
+  }
+  if (!got) s_fail = 1;
+  __syncthreads();
+  const bool fail = s_fail != 0;
+  if (fail && threadIdx.x == 0) raise_status(status, SENSE_DEVST_TIMEOUT);
+  float acc = 0.0f;
+  if (!fail && o < v) {
+    const float* wr = sw + (size_t)wid * d;
+    for (int j0 = 4 * lane; j0 < d; j0 += 128) {
+      const uint2 xw = *reinterpret_cast<const uint2*>(sxb + j0);
+      float4 xv = make_float4(bf_lo(xw.x), bf_hi(xw.x), bf_lo(xw.y), bf_hi(xw.y));
+      if (mu) {
+        const float4 m = *reinterpret_cast<const float4*>(smu + j0);
+        xv = make_float4(__fsub_rn(xv.x, m.x), __fsub_rn(xv.y, m.y), __fsub_rn(xv.z, m.z),
+                         __fsub_rn(xv.w, m.w));
+      }
+      const float4 wv = *reinterpret_cast<const float4*>(wr + j0);
+      acc = madd(acc, xv.x, wv.x);
+      acc = madd(acc, xv.y, wv.y);
+      acc = madd(acc, xv.z, wv.z);
+      acc = madd(acc, xv.w, wv.w);
+    }
+    acc = butterfly(acc);
+  }
+  if constexpr (!NORM) {
+    if (!fail && o < v && lane == 0) out[row * v + o] = acc;
+  } else {
+    namespace cg = cooperative_groups;
+    cg::cluster_group cl = cg::this_cluster();
+    if (lane == 0) s_out[wid] = acc;
+    cl.sync();  // every block's outputs and failure flag are written
+    if (blockIdx.x == 0 && wid == 0) {
+      bool any_fail = false;
+      for (unsigned r = 0; r < gridDim.x; ++r) any_fail |= *cl.map_shared_rank(&s_fail, r) != 0;
+      if (!any_fail) {
+        float part[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int oo = 32 * t + lane;
+          part[t] = (oo < v) ? *cl.map_shared_rank(&s_out[oo & 7], (unsigned)(oo >> 3)) : 0.0f;
+        }
+        float ss = 0.0f;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          for (int l = 0; l < 32 && 32 * t + l < v; ++l) {
+            const float e = __shfl_sync(0xffffffffu, part[t], l);
+            ss = madd(ss, e, e);
+          }
+        }
+        const float nrm = __fsqrt_rn(ss);
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          if (32 * t + lane < v)
+            out[row * v + 32 * t + lane] = nrm > 0.0f ? __fdiv_rn(part[t], nrm) : 0.0f;
+      }
+    }
+    cl.sync();  // the other blocks' shared memory stays alive until it is read
+  }
+}
+
+size_t project_bulk_smem(int d, bool mean) { return (size_t)d * 2 + (mean ? (size_t)d * 4 : 0) + 32 * (size_t)d; }
+constexpr size_t kProjectBulkMax = 200 * 1024;
 
 // Block (output group, row): the centred row is staged in shared memory once;
 // warp w computes output 8 * blockIdx.x + w, streaming its row of W.
@@ -721,6 +839,42 @@ sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float*
   if (!aligned(x, 16) || !aligned(basis, 16) || (mean && !aligned(mean, 16)) || !aligned(out, 4))
     return fail(SENSE_ERR_INVALID_ARG, "x, basis and mean must be 16-byte aligned");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int groups = (v + 7) / 8;
+  const size_t bulk_smem = project_bulk_smem(d, mean != nullptr);
+  if (n <= 64 && bulk_smem <= kProjectBulkMax) {
+    // one query batch: bulk copies, normalisation fused when a row's blocks fit a cluster
+    uint32_t* status = device_status_word();
+    if (!status) return SENSE_ERR_OOM;
+    const bool fuse = (flags & SENSE_PROJECT_NORMALIZE) && groups <= 8;
+    void (*kern)(const uint16_t*, int, const float*, int, const float*, float*, uint32_t*) =
+        fuse ? project_bulk_kernel<true> : project_bulk_kernel<false>;
+    sense_status st = cuda_check(
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bulk_smem),
+        "cudaFuncSetAttribute(project_bulk)");
+    if (st != SENSE_OK) return st;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)groups, (unsigned)n);
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = bulk_smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = fuse ? (unsigned)groups : 1u;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    {
+      LaunchScope ls(K_PROJECT, s);
+      st = cuda_check(cudaLaunchKernelEx(&cfg, kern, x, (int)d, basis, (int)v, mean, out, status),
+                      "launch project_bulk");
+      if (st != SENSE_OK) return st;
+    }
+    if (fuse || !(flags & SENSE_PROJECT_NORMALIZE)) return SENSE_OK;
+    LaunchScope ls(K_PROJECT, s);
+    normalize_rows_kernel<<<(unsigned)((n * 32 + 255) / 256), 256, 0, s>>>(out, n, v);
+    return cuda_check(cudaGetLastError(), "launch normalize rows");
+  }
   {
     LaunchScope ls(K_PROJECT, s);
     if (n * v <= 16384 && n <= 65535 && d <= 12288) {

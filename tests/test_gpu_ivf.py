@@ -50,6 +50,7 @@ def _dev(a):
 @pytest.mark.parametrize("n,d,v,centre,norm", [
     (1, 4096, 64, True, True), (5, 1000, 16, False, True), (300, 4096, 64, True, True),
     (333, 1000, 48, True, False), (40, 512, 128, False, True), (2000, 256, 20, True, True),
+    (3, 768, 20, True, False), (64, 4096, 64, True, True), (2, 2048, 60, True, True),
 ])
 def test_project_matches_oracle(S, n, d, v, centre, norm):
     rng = np.random.default_rng(n + d + v)
