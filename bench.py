@@ -699,8 +699,8 @@ def main():
         n_keys = v["prefix"] + v["L"]
         vbytes = 2 * v["heads"] * n_keys * 128 * 2 + v["heads"] * v["L"] * 128 * (2 + 4)
         vflops = 4 * v["heads"] * v["L"] * n_keys * 128
-        t_ms, t_launches = prof.get("tree_attn", (0.0, 0))
-        per = t_ms / max(1, t_launches // 2) / 1e3  # main kernel + combine per step
+        t_ms, _ = prof.get("tree_attn", (0.0, 0))
+        per = t_ms / args.steps / 1e3  # every attention launch of a step (main + any combine)
         verify_info = {"heads": v["heads"], "head_dim": 128, "draft_tokens": v["L"],
                        "prefix": v["prefix"], "cache_capacity": v["capacity"],
                        "us_per_step": per * 1e6,

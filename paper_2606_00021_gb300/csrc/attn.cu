@@ -27,14 +27,18 @@
 //    P = 2^(s - ref) (ex2.approx) as bf16 into shared memory in the
 //    128-byte-swizzled K-major layout the MMA reads, and sum the bf16
 //    values of P into the row sum;
-//  - each split writes its unnormalised O, reference maximum and row sum;
-//    a combine kernel rescales the splits to a common maximum and divides.
+//  - each split keeps its unnormalised O, reference maximum and row sum;
+//    with at most 8 splits per head the splits are one cluster and merge
+//    in place (each CTA combines every splits-th row from the others'
+//    shared memory, rescaled to a common maximum, and divides), else they
+//    go to global memory for a combine kernel.
 // The key range is split so that heads x splits fill the SMs: the cache
 // (2 x n x 128 x 2 bytes per head) is streamed once.
 // Every mbarrier wait gives up after ~2 s of clock64 time: it sets
 // SENSE_DEVST_TIMEOUT and an abort flag that releases the other roles; the
 // producer then waits (bounded) for its copies in flight, the MMA thread for
 // its MMAs, and the CTA frees its TMEM before returning.
+#include <cooperative_groups.h>
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -71,6 +75,8 @@ struct AttnArgs {
   int mask_words;
   float* part_o;   // [H, splits, 128, 128]
   float* part_ml;  // [H, splits, 128, 2]: reference maximum (log2), row sum
+  float* out;      // [H, L, 128] (fused combine)
+  int fused;       // the splits of a head form a cluster and combine in place
   uint32_t* status;
 };
 
@@ -394,9 +400,16 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(bar(P_FULL + b));
     }
-    // partial output of this split: each thread its 64 dims, row sums combined
+    // partial output of this split: each thread its 64 dims, row sums
+    // combined; into global memory, or (fused) into this CTA's shared memory
+    // where the K/V stages were (every load has landed, every product is
+    // done once MMA_DONE has completed)
     const int64_t pbase = ((int64_t)h * a.splits + sp) * 128 + r;
-    float* po = a.part_o + pbase * kHd + half * (kHd / 2);
+    float* so = reinterpret_cast<float*>(s_kv);  // fused: [128][128] partial O
+    float* sml = so + 128 * kHd;                  // fused: [128][2] statistics
+    float* po = a.fused ? so + r * kHd + half * (kHd / 2)
+                        : a.part_o + pbase * kHd + half * (kHd / 2);
+    float* pml = a.fused ? sml + 2 * r : a.part_ml + pbase * 2;
     const bool done =
         __all_sync(0xffffffffu, ok && nbl > 0 && wait_bar(bar(MMA_DONE), 0, abort, a.status));
     if (done && q4 * 32 < a.L) {  // rows past L are padding: not written
@@ -421,9 +434,8 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     *reinterpret_cast<float*>(pchunk(s_p, kChunksT * half)) = rowsum;
     pair_sync();
     if (half == 0) {
-      a.part_ml[pbase * 2] = done ? ref : NEG;
-      a.part_ml[pbase * 2 + 1] =
-          done ? rowsum + *reinterpret_cast<const float*>(pchunk(s_p, kChunksT)) : 0.0f;
+      pml[0] = done ? ref : NEG;
+      pml[1] = done ? rowsum + *reinterpret_cast<const float*>(pchunk(s_p, kChunksT)) : 0.0f;
     }
   }
   ptx::tc_fence_before();
@@ -431,6 +443,54 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
   if (warp == 1) {
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+  if (a.fused) {
+    // the head's splits (one cluster) merge their partials: row r is done by
+    // CTA r % splits, one warp per row, reading every split's statistics and
+    // rows through distributed shared memory, in the order of
+    // tree_attn_combine_kernel
+    namespace cg = cooperative_groups;
+    cg::cluster_group cl = cg::this_cluster();
+    cl.sync();
+    const int nsp = a.splits;
+    const float* so = reinterpret_cast<const float*>(s_kv);
+    const float* sml = so + 128 * kHd;
+    const float NEG = -__int_as_float(0x7f800000);
+    for (int r = sp + nsp * warp; r < a.L; r += nsp * (kAttnThreads / 32)) {
+      float ref_s = NEG, l_s = 0.0f;
+      if (lane < nsp) {
+        const float* m = cl.map_shared_rank(sml, (unsigned)lane) + 2 * r;
+        ref_s = m[0];
+        l_s = m[1];
+      }
+      float mx = (lane < nsp && l_s > 0.0f) ? ref_s : NEG;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+      float f = 0.0f, l = 0.0f;
+      if (lane < nsp) {
+        l = l_s;
+        if (l > 0.0f) f = exp2f(ref_s - mx);
+        else l = 0.0f;
+      }
+      float fl = f * l;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) fl += __shfl_xor_sync(0xffffffffu, fl, off);
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int t = 0; t < nsp; ++t) {
+        const float ft = __shfl_sync(0xffffffffu, f, t);
+        if (ft == 0.0f) continue;  // warp-uniform
+        const float4 o =
+            *reinterpret_cast<const float4*>(cl.map_shared_rank(so, (unsigned)t) + r * kHd + 4 * lane);
+        acc.x += ft * o.x;
+        acc.y += ft * o.y;
+        acc.z += ft * o.z;
+        acc.w += ft * o.w;
+      }
+      const float inv = fl > 0.0f ? 1.0f / fl : 0.0f;
+      *reinterpret_cast<float4*>(a.out + ((int64_t)h * a.L + r) * kHd + 4 * lane) =
+          make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+    }
+    cl.sync();  // the other CTAs' shared memory stays alive until it is read
   }
 }
 
@@ -589,12 +649,28 @@ sense_status sense_tree_attention(const uint16_t* q, const uint16_t* k_cache,
   st = cuda_check(cudaFuncSetAttribute(tree_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem), "cudaFuncSetAttribute(tree_attn)");
   if (st != SENSE_OK) return st;
+  // up to 8 splits per head: the splits form a cluster and combine in place
+  a.out = out;
+  a.fused = splits <= 8 ? 1 : 0;
   {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)heads, (unsigned)splits);
+    cfg.blockDim = dim3(kAttnThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = a.fused ? (unsigned)splits : 1u;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     LaunchScope ls(K_TREE_ATTN, s);
-    tree_attn_kernel<<<dim3(heads, splits), kAttnThreads, smem, s>>>(tm_q, tm_k, tm_vt, a);
-    st = cuda_check(cudaGetLastError(), "launch tree attention");
+    st = cuda_check(cudaLaunchKernelEx(&cfg, tree_attn_kernel, tm_q, tm_k, tm_vt, a),
+                    "launch tree attention");
     if (st != SENSE_OK) return st;
   }
+  if (a.fused) return SENSE_OK;
   LaunchScope ls(K_TREE_ATTN, s);
   const int64_t threads = (int64_t)heads * L * 32;
   tree_attn_combine_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(
