@@ -199,6 +199,7 @@ def _check_tree(got, want, q, cap):
     (3, 8, 8, 5, 0), (4, 32, 16, 3, 64), (2, 256, 16, 4, 0), (2, 256, 16, 50, 128),
     (3, 1, 5, 3, 0), (2, 64, 1, 10, 0), (2, 1024, 8, 3, 0), (2, 300, 27, 2, 4000),
     (2, 512, 16, 3, 7), (1, 17, 32, 2, 1),
+    (2, 128, 32, 3, 200), (1, 128, 8, 2, 0), (2, 129, 4, 3, 50),  # small-path boundary
 ])
 def test_tree_matches_oracle(S, q, k, m, vocab, cap):
     dev = torch.device("cuda")
@@ -312,6 +313,7 @@ def _gate_case(q, k, m, v, d, cap, seed, plant=True):
     (1, 32, 16, 32000, 64, 0.05, 3, 6, 0, False),   # one query: two blocks per row
     (1, 4, 4, 64, 0, 0.5, 16, 3, 1, False),         # slices of one float4, empty slices
     (1, 16, 8, 40000, 0, 0.05, 5, 4, 0, False),     # one block per row, three stages a warp
+    (1, 16, 16, 128256, 64, 0.05, 3, 6, 0, False),  # one query, long rows: split rows merged
 ])
 def test_gate_matches_oracle(S, q, k, m, v, cap, gamma, kappa, w, tau, unnorm):
     dev = torch.device("cuda")
