@@ -202,7 +202,10 @@ sense_status sense_retrieve_topk_noalloc(const sense_datastore* ds, const uint16
  * principal axes); mean [d] f32 or NULL.  With SENSE_PROJECT_NORMALIZE each
  * row is then divided by its L2 norm (zero rows stay zero).  out [n, v] f32.
  * Limits: d % 8 == 0, 1 <= v <= SENSE_MAX_PROJ_DIM; x, basis, mean 16-byte
- * aligned.  The PCA basis itself is fitted offline by the caller.
+ * aligned.  The PCA basis itself is fitted offline by the caller.  For
+ * small batches the rows are staged by bulk copies whose wait is bounded: a
+ * copy that never lands sets SENSE_DEVST_TIMEOUT and leaves its row
+ * unwritten.
  */
 sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float* basis, int32_t v,
                            const float* mean, uint32_t flags, float* out, sense_stream_t stream);
@@ -479,7 +482,8 @@ sense_status sense_tree_mask_full(const uint32_t* mask_bits, const int32_t* num_
  *   out [heads, L, 128] f32.  Probabilities are rounded to bf16 before the
  *   product with V (fp32 accumulation throughout).
  *   workspace: sense_tree_attention_workspace_bytes(heads, L, prefix_len)
- *   bytes, 256-byte aligned.
+ *   bytes, 256-byte aligned (used only when a head's keys are split over
+ *   more than 8 CTAs; up to 8 splits merge on chip).
  * Limits: d_head == 128, 1 <= L <= 128, capacity % 128 == 0, prefix_len +
  * L <= capacity, scale > 0; q, caches and out 16-byte aligned.
  */
