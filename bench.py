@@ -372,8 +372,9 @@ def run_reference(args, cfg, name):
     t_scan, t_down = [], []
     total = args.warmup + args.steps
     t_all0 = time.perf_counter()
+    avail = keys.shape[0] // slice_rows  # distinct slices held (up to 4)
     for it in range(total):
-        lo = (it % 4) * slice_rows
+        lo = (it % avail) * slice_rows
         t0 = time.perf_counter()
         s = O.scores(kb[lo:lo + slice_rows], qb)
         t1 = time.perf_counter()
