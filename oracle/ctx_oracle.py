@@ -9,8 +9,8 @@ Alg. 1 fills it with R.Update(h, y) after prefill and R.Update(H_align[i*,
 0:L*+1], a) after every accepted step: pairs of a hidden state and the token
 it predicted.  Alg. 2 searches it with DynSearch(h, C_d, x~), adds a score
 boost delta to its results (s = [s_s; s_d + delta]) and reranks the union
-with Eq. 8.  The paper does not define DynSearch or the buffer's size; the
-readings below are stated in the design doc's list of readings as well:
+with Eq. 8.  The paper does not define DynSearch or the buffer's size; this
+module reads them as follows:
 
 * an entry is a position p of the generated sequence: its key is the hidden
   state h_p that predicted token y_{p+1}, L2-normalised and stored as bf16
