@@ -17,21 +17,23 @@ pipeline in numpy:
   ivf_search     coarse top-nprobe, list scan, exact top-k of the
                  approximate scores
 
-Precision.  FAISS computes in fp32, and every step here ends in an integer
-decision (a cell, a code, a probe set, a top-k index), so the oracle takes
-those decisions in fp32 with a stated evaluation order, each product
-rounded to fp32 before it is added (no fused multiply-add):
-  * dot products and squared distances in the projected space (dimension
-    <= 128) are summed term by term from index 0 upwards (``dot_seq``);
-  * the projection's long dot products (the hidden size d) are summed in 32
-    interleaved partial sums - partial l takes the 4-column groups g with
-    g mod 32 = l, in ascending column order - which are then combined by a
-    butterfly: 16 rounds ... 1 round, partial l += partial (l xor s) for
-    s = 16, 8, 4, 2, 1 (``dot_lanes``).
+Precision.  The projection (query and key construction) is a plain linear
+map followed by a normalisation, and its oracle is that definition in fp64:
+y = (x - mu) W^T summed exactly in fp64 over the hidden size, then y / ||y||.
+The CUDA path computes it in fp32; the tests compare the two within an
+error bound derived from the fp32 arithmetic, not bit for bit.
+
+Every later step ends in an integer decision (a cell, a code, a probe set, a
+top-k index).  FAISS takes those decisions in fp32, and so does this oracle,
+on vectors it is given (the tests hand both sides the same projected
+vectors): dot products and squared distances in the projected space
+(dimension <= 128) are the plain left-to-right sums, each product rounded
+to fp32 before it is added (no fused multiply-add; ``dot_seq``, ``l2_seq``).
 k-means means are accumulated in 2^-31 fixed point (integer sums do not
-depend on the order of the members) and divided in fp64.  These orders are
-readings: the paper does not state them.  Pins in tests/test_oracle_ivf.py compare
-every function against fp64 arithmetic, brute force and special cases.
+depend on the order of the members) and divided in fp64.  The left-to-right
+fp32 sum and the fixed-point mean are readings: the paper does not state an
+evaluation order.  Pins in tests/test_oracle_ivf.py compare every function
+against exact arithmetic, brute force and special cases.
 """
 from __future__ import annotations
 
@@ -71,27 +73,6 @@ def l2_seq(a: np.ndarray, b: np.ndarray) -> np.ndarray:
     return acc
 
 
-def dot_lanes(a: np.ndarray, b: np.ndarray) -> np.ndarray:
-    """sum_j a[..., j] * b[..., j] in fp32 over 32 interleaved partial sums
-    of 4-column groups, combined by an xor butterfly (see the module
-    docstring).  a [..., n], b [..., n]."""
-    a = np.asarray(a, dtype=F32)
-    b = np.asarray(b, dtype=F32)
-    shape = np.broadcast_shapes(a.shape[:-1], b.shape[:-1])
-    n = a.shape[-1]
-    part = np.zeros(shape + (32,), dtype=F32)
-    for g0 in range(0, n, 128):          # one round of 32 groups of 4
-        for lane in range(32):
-            for u in range(4):
-                j = g0 + 4 * lane + u
-                if j < n:
-                    part[..., lane] = (part[..., lane] + (a[..., j] * b[..., j])).astype(F32)
-    lanes = np.arange(32)
-    for s in (16, 8, 4, 2, 1):
-        part = (part + part[..., lanes ^ s]).astype(F32)
-    return part[..., 0]
-
-
 def _l2_normalize(y: np.ndarray) -> np.ndarray:
     """y / ||y|| per row in fp32 (zero rows stay zero)."""
     nrm = np.sqrt(dot_seq(y, y)).astype(F32)
@@ -107,19 +88,27 @@ def _l2_normalize(y: np.ndarray) -> np.ndarray:
 
 
 def project(x_bits: np.ndarray, basis: np.ndarray, mean=None, normalize: bool = True):
-    """PCA projection of bf16 hidden states, then (optionally) unit L2 norm.
+    """PCA projection of bf16 hidden states, then (optionally) unit L2 norm,
+    in fp64 (App. E: PCA to v dimensions, then L2Norm; Alg. 2 builds the
+    query as k = L2Norm(PCA(h))).
 
-    x_bits [n, d] uint16 (bf16), basis [v, d] f32 (rows = principal axes),
-    mean [d] f32 or None.  y[i, o] = sum_j (x[i, j] - mean[j]) * basis[o, j]
-    (fp32, the centred value rounded to fp32, ``dot_lanes`` order); with
-    ``normalize``, y[i] / ||y[i]|| (``dot_seq`` order over the v outputs).
+    x_bits [n, d] uint16 (bf16), basis [v, d] (row o = principal axis o),
+    mean [d] or None.  The PCA coordinates are y[i, o] = sum_j (x[i, j] -
+    mean[j]) * basis[o, j]; with ``normalize``, y[i] / ||y[i]|| (a zero row
+    stays zero).  Returns float64 [n, v].
     """
-    x = bf16_bits_to_f64(np.asarray(x_bits)).astype(F32)  # exact
-    w = np.asarray(basis, dtype=F32)
+    x = bf16_bits_to_f64(np.asarray(x_bits))  # exact
+    w = np.asarray(basis, dtype=np.float64)
     if mean is not None:
-        x = (x - np.asarray(mean, dtype=F32)[None, :]).astype(F32)
-    y = dot_lanes(x[:, None, :], w[None, :, :])
-    return _l2_normalize(y) if normalize else y
+        x = x - np.asarray(mean, dtype=np.float64)[None, :]
+    y = x @ w.T
+    if not normalize:
+        return y
+    nrm = np.sqrt((y * y).sum(axis=1))
+    out = np.zeros_like(y)
+    nz = nrm > 0
+    out[nz] = y[nz] / nrm[nz, None]
+    return out
 
 
 # ----------------------------------------------------------------------------

@@ -52,40 +52,24 @@ def test_dot_exact_on_dyadic_values_and_order_matters():
     assert I.dot_seq(x[:, ::-1].copy(), np.ones_like(x))[0] == 2.0 ** -23
 
 
-def test_dot_lanes_order_and_bound():
-    rng = np.random.default_rng(12)
-    a = rng.standard_normal((30, 1000)).astype(np.float32)
-    b = rng.standard_normal((30, 1000)).astype(np.float32)
-    ex = np.sum(a.astype(np.float64) * b, axis=1)
-    bound = 1000 * U * np.sum(np.abs(a.astype(np.float64) * b), axis=1)
-    assert np.all(np.abs(I.dot_lanes(a, b) - ex) <= bound)
-    # lane partials: column 128 joins lane 0 (with columns 0..3), column 4
-    # starts lane 1; the butterfly then adds lane 1 to lane 0 last
-    x = np.zeros((1, 256), np.float32)
-    x[0, 0], x[0, 128], x[0, 4] = 1.0, 2.0 ** -24, 2.0 ** -24
-    # lane 0: 1 + 2^-24 -> 1 (ties to even); lane 1: 2^-24; final 1 + 2^-24 -> 1
-    assert I.dot_lanes(x, np.ones_like(x))[0] == 1.0
-    x[0, 132] = 2.0 ** -24  # lane 1 now holds 2^-23: 1 + 2^-23 is exact
-    assert I.dot_lanes(x, np.ones_like(x))[0] == 1.0 + 2.0 ** -23
-
-
 # ---------------------------------------------------------------- projection
 
-def test_project_matches_fp64_and_is_unit():
+def test_project_exact_on_dyadic_inputs():
+    """Small dyadic inputs: every product and sum is a short binary fraction,
+    so the fp64 result must equal exact rational arithmetic."""
+    from fractions import Fraction as F
     rng = np.random.default_rng(3)
-    x = synth.gaussian_rows_f32(40, 512, seed=3).to(torch.bfloat16)
+    n, d, v = 4, 24, 5
+    xv = rng.integers(-6, 7, (n, d)) / 8.0
+    x = torch.tensor(xv, dtype=torch.float32).to(torch.bfloat16)
     xb = _bits(x)
-    w = rng.standard_normal((16, 512)).astype(np.float32) / np.sqrt(512)
-    mu = rng.standard_normal(512).astype(np.float32) * 0.1
+    w = (rng.integers(-9, 10, (v, d)) / 16.0).astype(np.float32)
+    mu = (rng.integers(-3, 4, d) / 4.0).astype(np.float32)
     y = I.project(xb, w, mu, normalize=False)
-    xf = O.bf16_bits_to_f64(xb)
-    xc = (xf - mu).astype(np.float32).astype(np.float64)  # centring is rounded to fp32 first
-    ex = xc @ w.astype(np.float64).T
-    bound = 512 * U * (np.abs(xc) @ np.abs(w.astype(np.float64)).T) * 1.01 + 1e-30
-    assert np.all(np.abs(y - ex) <= bound)
-    yn = I.project(xb, w, mu)
-    np.testing.assert_allclose(np.linalg.norm(yn.astype(np.float64), axis=1), 1.0, atol=1e-6)
-    np.testing.assert_allclose(yn, ex / np.linalg.norm(ex, axis=1, keepdims=True), atol=2e-6)
+    for i in range(n):
+        for o in range(v):
+            ex = sum((F(float(xv[i, j])) - F(float(mu[j]))) * F(float(w[o, j])) for j in range(d))
+            assert F(float(y[i, o])) == ex
 
 
 def test_project_coordinate_basis_and_zero_row():
@@ -94,11 +78,47 @@ def test_project_coordinate_basis_and_zero_row():
     sel = [5, 0, 63, 17]
     w = np.eye(64, dtype=np.float32)[sel]
     y = I.project(xb, w, normalize=False)
-    np.testing.assert_array_equal(y, O.bf16_bits_to_f64(xb)[:, sel].astype(np.float32))
+    np.testing.assert_array_equal(y, O.bf16_bits_to_f64(xb)[:, sel])
+    # a signed permutation of coordinates only permutes and flips them
+    w2 = -np.eye(64, dtype=np.float32)[sel[::-1]]
+    np.testing.assert_array_equal(I.project(xb, w2, normalize=False), -y[:, ::-1])
     # centring on the row itself gives a zero row, left at zero by the norm
     mu = O.bf16_bits_to_f64(xb[2]).astype(np.float32)
     z = I.project(xb[2:3], w, mu)
     assert np.all(z == 0)
+
+
+def test_project_orthonormal_basis_keeps_lengths_and_angles():
+    """With a full orthonormal basis (v = d) the PCA coordinates are a
+    rotation: lengths and inner products of centred rows are preserved."""
+    rng = np.random.default_rng(13)
+    d = 96
+    x = synth.gaussian_rows_f32(10, d, seed=13).to(torch.bfloat16)
+    xb = _bits(x)
+    w = np.linalg.qr(rng.standard_normal((d, d)))[0].T
+    mu = 0.2 * rng.standard_normal(d)
+    y = I.project(xb, w, mu, normalize=False)
+    xc = O.bf16_bits_to_f64(xb) - mu
+    np.testing.assert_allclose(np.linalg.norm(y, axis=1), np.linalg.norm(xc, axis=1), rtol=1e-12)
+    np.testing.assert_allclose(y[0] @ y[1], xc[0] @ xc[1], rtol=1e-10)
+
+
+def test_project_normalised_rows_and_translation():
+    rng = np.random.default_rng(14)
+    x = synth.gaussian_rows_f32(20, 128, seed=14).to(torch.bfloat16)
+    xb = _bits(x)
+    w = rng.standard_normal((16, 128)) / np.sqrt(128)
+    mu = 0.1 * rng.standard_normal(128)
+    y = I.project(xb, w, mu, normalize=False)
+    # centring is a translation of the PCA coordinates by -W mu
+    np.testing.assert_allclose(y, I.project(xb, w, normalize=False) - w @ mu, atol=1e-12)
+    yn = I.project(xb, w, mu)
+    np.testing.assert_allclose(np.linalg.norm(yn, axis=1), 1.0, atol=1e-14)
+    # the normalised row points along y: positive multiple, and a scaled
+    # basis (c > 0) gives the same unit rows
+    cos = (yn * y).sum(1) / np.linalg.norm(y, axis=1)
+    np.testing.assert_allclose(cos, 1.0, atol=1e-14)
+    np.testing.assert_allclose(I.project(xb, 3.0 * w, mu), yn, atol=1e-14)
 
 
 # ---------------------------------------------------------------- k-means
