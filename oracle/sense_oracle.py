@@ -23,7 +23,8 @@ for floating point, following the step order and notation of the paper:
   tree_mask_full        static KV cache) from Alg. 3's mask M
   tree_attention       the masked attention of the verify forward (Alg. 1)
                         under that mask
-  soft_gate            §3.3 Eqs. 11-19 and App. C.4 Alg. 4
+  soft_gate            §3.3 Eqs. 11-19 (with App. C.4's normalised entropy
+                        and look-ahead window)
 
 Readings where the paper is silent or ambiguous are stated at each function.
 
@@ -399,9 +400,9 @@ def tree_attention(q_bits: np.ndarray, k_bits: np.ndarray, v_bits: np.ndarray, m
 
 
 def _softmax_entropy(rows: np.ndarray) -> np.ndarray:
-    """Shannon entropy (nats) of softmax(rows) along the last axis, fp64.
-
-    Alg. 4: P~ = Softmax(P), E = -sum_v P~ log P~ (with 0 log 0 = 0).
+    """Shannon entropy (nats) of softmax(rows) along the last axis, fp64:
+    -sum_v p_v log p_v over the softmax probabilities p (0 log 0 = 0), the
+    entropy of Eq. 14 taken of the logits' distribution as App. C.4 does.
     """
     x = np.asarray(rows, dtype=np.float64)
     z = x - x.max(axis=-1, keepdims=True)
@@ -415,8 +416,8 @@ def _softmax_entropy(rows: np.ndarray) -> np.ndarray:
 def _in_topk(rows: np.ndarray, tok: np.ndarray, kappa: int) -> np.ndarray:
     """I(tok in TopK(row, kappa)) with the total order (value desc, index asc).
 
-    Alg. 4 line "Y_k = TopK(P, k)" does not say how ties at the boundary are
-    broken.  Reading: the lower vocabulary index wins, so the token is in the
+    Eq. 15's top-k set does not say how ties at its boundary are broken.
+    Reading: the lower vocabulary index wins, so the token is in the
     top-kappa iff fewer than kappa entries precede it in that order.
     """
     x = np.asarray(rows, dtype=np.float32)
@@ -432,39 +433,43 @@ def soft_gate(tokens, parent, num_nodes, gamma, root_logits, node_logits,
               root_hidden, node_hidden, *, gamma_thr=0.05, kappa=3, window=6,
               tau=0, unnormalized_entropy=False, return_masks=False,
               ent_band=0.0):
-    """Soft-gated evaluation of every candidate path of every query.
+    """Soft-gated evaluation of every candidate path of every query (§3.3).
 
     Inputs per query q (leading axis): the tree (tokens, parent, num_nodes,
     gamma [k, M]) and the target outputs on it: root_logits [V] = p (the
     state before the draft), node_logits [cap, V] = P' (one row per tree
     node), root_hidden [d] = h, node_hidden [cap, d] = H'.
 
-    Alignment (§3.2.3 Eq. 11; Alg. 1 "H_align, P_align <- [h; Gamma(H')]"):
-    position j of candidate i is predicted by the row P_align[i, j], which is
-    p for j = 0 and P'[gamma[i, j-1]] for j >= 1.  The draft token there is
-    D[i, j] = tokens[gamma[i, j]].  (Reading of the garbled shape
-    "M x (N+1)": N candidates, each with its root row plus M positions.)
+    Candidate i is the path of nodes gamma[i, 0], gamma[i, 1], ...; its draft
+    token at position j is D[i, j] = tokens[gamma[i, j]].  The target's
+    prediction for position j comes from the state just before it (Eq. 11,
+    the alignment that prepends p and h): the root row p for j = 0 and the
+    row of node gamma[i, j-1] otherwise.  (The printed shape "M x (N+1)" is
+    read as N candidates, each with its root row plus M positions.)
 
-    Masks follow Alg. 4 in its order:
-      Y = argmax_v P_align (lowest index among equal maxima);
-      B_em = I(D == Y)                                         (Eq. 13)
-      E = entropy(softmax(P_align)); B_ent = I(E / log|V| > gamma)  (Alg. 4;
-          ``unnormalized_entropy`` uses Eq. 14's E > gamma instead)
-      B_topk = I(D in TopK(P_align, kappa))                    (Eq. 15)
-      Bbar = Pad(1 - B_em, (0, W), 1); R = Conv1D(Bbar, 1_W)[:, 1:M+1];
-      B_con = I(R <= tau)  (Alg. 4 writes R == 0, Eq. 16 writes R <= tau;
-          tau = 0 makes them equal)                            (Eq. 16)
-      G = B_em or (B_ent and (B_topk or B_con))                (Eq. 17)
-      L_i = sum_j CumProd(G, dim 1)[i, j] - 1;  i* = argmax_i L_i  (Eq. 18)
-    Reading: i* is the lowest candidate rank among the maximal L_i.
+    For each position (i, j), with r its predicting row:
+      * Eq. 12-13: em = 1 when D[i, j] is the greedy token of r (the lowest
+        index among equal maxima);
+      * Eq. 14: ent = 1 when the entropy of softmax(r), in nats and divided
+        by log|V|, exceeds gamma_thr (the normalisation is App. C.4's;
+        ``unnormalized_entropy`` compares the raw entropy as Eq. 14 prints);
+      * Eq. 15: topk = 1 when fewer than kappa vocabulary entries come before
+        D[i, j] in the order (value desc, index asc) of r;
+      * Eq. 16: con = 1 when the positions j+1 .. j+W of the same candidate
+        hold at most tau mismatches (1 - em), positions past the span
+        counting as mismatches (the window looks strictly ahead: App. C.4
+        pads with ones on the right and drops the first output);
+      * Eq. 17: G = em or (ent and (topk or con)).
+    Eq. 18: n_i is the number of leading ones of G[i, :], the accepted
+    length; L_i = n_i - 1 (App. C.4 and Alg. 1 index the accepted tokens
+    D[i, 0 .. L_i]); i* is the lowest candidate rank with the largest L_i.
     Positions whose node was dropped by the tree's node cap (gamma = -1)
-    count as mismatches (Bbar = 1, like the padding) and have G = 0.
+    have em = ent = topk = G = 0 and count as mismatches inside a window.
 
-    Next state (Eq. 19; Alg. 1): accepted tokens a = D[i*, 0:L*+1];
-    the next node is gamma[i*, L*] (-1, the root, when L* = -1);
-    h_next = H_align[i*, L*+1] is that node's hidden state (h when -1) and
-    p_next = P_align[i*, L*+1] is that node's logits row, whose argmax is
-    the next anchor token.
+    Next state (Eq. 19; Alg. 1): accepted tokens a = D[i*, 0 .. L*]; the next
+    node is gamma[i*, L*] (-1, the root, when L* = -1); h_next is that
+    node's hidden state (h when -1) and p_next its logits row, whose greedy
+    token is the next anchor.
 
     ``ent_band`` > 0 also reports, per query, whether any evaluated
     position had a normalised entropy within ``ent_band`` of the threshold
@@ -496,49 +501,45 @@ def soft_gate(tokens, parent, num_nodes, gamma, root_logits, node_logits,
             out[key] = np.zeros((qn, k, m), dtype=np.uint8)
     for q in range(qn):
         g = gamma[q].astype(np.int64)
-        valid = g >= 0
-        d_tok = np.where(valid, tokens[q][np.where(valid, g, 0)], -1)
-        # P_align[i, j]: root row for j == 0, else the row of node gamma[i, j-1]
-        b_em = np.zeros((k, m), dtype=np.int64)
-        b_ent = np.zeros((k, m), dtype=np.int64)
-        b_topk = np.zeros((k, m), dtype=np.int64)
+        kept = g >= 0
+        em = np.zeros((k, m), dtype=bool)
+        ent = np.zeros((k, m), dtype=bool)
+        top = np.zeros((k, m), dtype=bool)
         amb = False
         for i in range(k):
-            rows = np.empty((m, v), dtype=np.float32)
             for j in range(m):
-                if j == 0:
-                    rows[j] = root_logits[q]
-                elif valid[i, j - 1]:
-                    rows[j] = node_logits[q, g[i, j - 1]]
-                else:
-                    rows[j] = root_logits[q]  # unused: position is dropped
-            y = np.argmax(rows, axis=-1)
-            b_em[i] = (d_tok[i] == y) & valid[i]
-            ent = _softmax_entropy(rows)
-            score = ent if unnormalized_entropy else ent / math.log(v)
-            b_ent[i] = (score > gamma_thr) & valid[i]
-            if ent_band > 0:
-                amb |= bool(np.any(valid[i] & (np.abs(score - gamma_thr) < ent_band)))
-            b_topk[i] = _in_topk(rows, d_tok[i], kappa) & valid[i]
-        # Bbar = Pad(1 - B_em, (0, W), value 1); dropped positions are 1 too.
-        bbar = np.ones((k, m + w), dtype=np.int64)
-        bbar[:, :m] = np.where(valid, 1 - b_em, 1)
-        # Conv1D with a ones kernel of width W (no padding): out[t] =
-        # sum_{u<W} bbar[t+u], t = 0..M; keep t = 1..M.
-        conv = np.zeros((k, m + 1), dtype=np.int64)
-        for t in range(m + 1):
-            conv[:, t] = bbar[:, t:t + w].sum(axis=1)
-        r_cnt = conv[:, 1:m + 1]
-        b_con = (r_cnt <= tau).astype(np.int64) * valid
-        gmask = (b_em | (b_ent & (b_topk | b_con))) & valid
-        gseq = np.cumprod(gmask, axis=1)
-        li = gseq.sum(axis=1) - 1
-        istar = int(np.argmax(li))
+                if not kept[i, j]:
+                    continue
+                tok = int(tokens[q, g[i, j]])
+                row = root_logits[q] if j == 0 else node_logits[q, g[i, j - 1]]
+                em[i, j] = tok == int(np.argmax(row))  # first maximum
+                h = _softmax_entropy(row)
+                score = h if unnormalized_entropy else h / math.log(v)
+                ent[i, j] = score > gamma_thr
+                if ent_band > 0 and abs(score - gamma_thr) < ent_band:
+                    amb = True
+                top[i, j] = bool(_in_topk(row, np.array(tok), kappa))
+        # mismatch indicator per position; dropped positions and the
+        # positions past the span (j >= M) are mismatches
+        miss = ~(em & kept)
+        con = np.zeros((k, m), dtype=bool)
+        for i in range(k):
+            for j in range(m):
+                ahead = [bool(miss[i, u]) if u < m else True for u in range(j + 1, j + w + 1)]
+                con[i, j] = kept[i, j] and sum(ahead) <= tau
+        gmask = (em | (ent & (top | con))) & kept
+        n_acc = np.zeros(k, dtype=np.int64)
+        for i in range(k):
+            while n_acc[i] < m and gmask[i, n_acc[i]]:
+                n_acc[i] += 1
+        li = n_acc - 1
+        istar = int(np.argmax(li))  # the first (lowest rank) maximum
         lstar = int(li[istar])
         out["i_star"][q] = istar
         out["L_star"][q] = lstar
         out["n_accept"][q] = lstar + 1
-        out["accepted"][q, :lstar + 1] = d_tok[istar, :lstar + 1]
+        for j in range(lstar + 1):
+            out["accepted"][q, j] = tokens[q, g[istar, j]]
         nxt = int(g[istar, lstar]) if lstar >= 0 else -1
         out["next_node"][q] = nxt
         prow = root_logits[q] if nxt < 0 else node_logits[q, nxt]
@@ -547,8 +548,8 @@ def soft_gate(tokens, parent, num_nodes, gamma, root_logits, node_logits,
         out["G"][q] = gmask.astype(np.uint8)
         out["ambiguous"][q] = amb
         if return_masks:
-            out["B_em"][q] = b_em
-            out["B_ent"][q] = b_ent
-            out["B_topk"][q] = b_topk
-            out["B_con"][q] = b_con
+            out["B_em"][q] = em
+            out["B_ent"][q] = ent & kept
+            out["B_topk"][q] = top & kept
+            out["B_con"][q] = con
     return out
