@@ -4,11 +4,13 @@ One step = one pass of the whole path for one batch of queries on a seeded
 synthetic workload resident in HBM: exact top-k retrieval over the bf16
 datastore, span gather, loose-trie draft tree and soft-gated evaluation.
 
-Default workload (LLaMA-7B-shaped store): n = 1,048,576 keys, d = 4096 bf16
-(8.6 GB), 1 query per step (512 distinct queries, each a perturbed key),
-k = 32, spans of 16 Zipf(1.1) tokens over a 32,000-token vocabulary, tree
-capped at 64 nodes, gate on fp32 N(0, 3^2) logits for every tree node with the
-paper's defaults (gamma 0.05, top-3, window 6).
+Default workload (LLaMA-70B-shaped store, the largest that one GPU holds):
+n = 8,388,608 keys, d = 8192 bf16 (137 GB), 1 query per step (16 distinct
+queries, each a perturbed key), k = 64, spans of 16 Zipf(1.1) tokens over a
+128,256-token vocabulary, tree capped at 64 nodes, gate on fp32 N(0, 3^2)
+logits for every tree node with the paper's defaults (gamma 0.05, top-3,
+window 6).  ``--workload`` selects the other shapes (llama7b_1m, qwen7b_4m,
+the sweeps, tiny_4k).
 
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle
 on bounded samples of the same workload instead.
@@ -33,7 +35,7 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 from synth.workloads import WORKLOADS  # noqa: E402
 
-DEFAULT = "llama7b_1m"
+DEFAULT = "llama70b_8m"
 METRIC = "hidden-state top-k retrieval queries/s (whole drafting step)"
 GATE = dict(gamma=0.05, topk=3, window=6, tau=0)
 # DRAM bytes (read + write) per unit processed by the dominant kernels, each
@@ -49,6 +51,15 @@ NCU_TRAFFIC_PER_UNIT = {
     # 4 queries of the k = 64 sweep: 3,774 root / inner-node rows of 128,256 logits
     ("gate_rows", 128256): (1939918336 + 3338240) / 3773.9375,
 }
+
+
+def _bits(t: torch.Tensor) -> np.ndarray:
+    """bf16 tensor -> uint16 bit patterns on the host."""
+    return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def _host(t: torch.Tensor) -> np.ndarray:
+    return t.detach().cpu().numpy()
 
 
 def peaks():
@@ -321,87 +332,148 @@ def build_ann(S, keys, kind, nlist, nprobe, pq_m, v, dev, seed=0):
             "build_s": build_s, "mean_list": float(sizes.mean()), "max_list": ix.max_list}
 
 
-def cpu_baseline(cfg, keys, spans, queries, gate_sets, budget_s=25.0):
-    """The oracle, as it stands, on whole queries of the same workload."""
+SLICE_ROWS = 65536  # rows per sampled slice of the store (one generator chunk)
+
+
+def _oracle_query(O, cfg, kb_slices, row_ids, qb, spans_h, gate_h):
+    """One query batch through the oracle over the sampled rows: scoring and
+    top-k over the sample (timed together), then gather, trie and gate on
+    the sample's top-k (timed apart).  Returns (t_scan, t_down)."""
+    t0 = time.perf_counter()
+    s = np.concatenate([O.scores(kb, qb) for kb in kb_slices], axis=1)
+    _, pos = O.topk(s, cfg["k"])
+    t1 = time.perf_counter()
+    idx = row_ids[pos]
+    dr = O.gather_drafts(spans_h, idx)
+    tr = O.loose_trie(dr, node_cap=cfg["cap"])
+    root, nodes, hr, hn = gate_h
+    O.soft_gate(tr["tokens"], tr["parent"], tr["num_nodes"], tr["gamma"], root, nodes, hr, hn,
+                gamma_thr=GATE["gamma"], kappa=GATE["topk"], window=GATE["window"])
+    return t1 - t0, time.perf_counter() - t1
+
+
+def _gate_host(gate_set):
+    return [_bits(t) if t.dtype == torch.bfloat16 else _host(t) for t in gate_set]
+
+
+def cpu_baseline(cfg, keys, spans, queries, gate_sets, budget_s=10.0):
+    """The oracle, as it stands, on whole queries of the same workload.
+
+    Scoring and top-k run over seeded 65,536-row slices of the resident store,
+    copied to the host one at a time, until about ``budget_s`` of oracle time
+    is spent (the whole store when it fits); their time is scaled by
+    n / rows scanned.  Gather, trie and gate run on the sample's top-k and
+    are not scaled."""
     import oracle as O
-    from tests.parity import bits, host
-    kb = bits(keys)
-    sp = host(spans)
-    root, nodes, hr, hn = [host(t) if t.dtype != torch.bfloat16 else bits(t) for t in gate_sets[0]]
-    done, t0 = 0, time.perf_counter()
-    while True:
-        qb = bits(queries[done % queries.shape[0]])
-        s = O.scores(kb, qb)
-        _, idx = O.topk(s, cfg["k"])
-        dr = O.gather_drafts(sp, idx)
-        tr = O.loose_trie(dr, node_cap=cfg["cap"])
-        O.soft_gate(tr["tokens"], tr["parent"], tr["num_nodes"], tr["gamma"], root, nodes, hr,
-                    hn, gamma_thr=GATE["gamma"], kappa=GATE["topk"], window=GATE["window"])
-        done += 1
-        el = time.perf_counter() - t0
-        if el > budget_s * 0.5 or done >= 4:
-            break
-    qn = done * cfg["q"]
-    return {"value": qn / el, "unit": "queries/s", "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{done} whole step(s) of the workload ({qn} queries over all "
-                      f"{cfg['n']} keys + gather/tree/gate), numpy fp64, {el:.1f} s"}
+    n = cfg["n"]
+    n_slices = (n + SLICE_ROWS - 1) // SLICE_ROWS
+    order = np.random.default_rng(5).permutation(n_slices)
+    qb = _bits(queries[0])
+    spans_h = _host(spans)
+    gate_h = _gate_host(gate_sets[0])
+    # the rate of the first slice sizes the sample to the budget
+    lo0 = int(order[0]) * SLICE_ROWS
+    kb0 = _bits(keys[lo0:min(n, lo0 + SLICE_ROWS)])
+    t0 = time.perf_counter()
+    O.scores(kb0, qb)
+    take = int(min(n_slices, max(1, budget_s / max(time.perf_counter() - t0, 1e-6))))
+    kbs, ids, rows = [], [], 0
+    for si in order[:take]:
+        lo, hi = int(si) * SLICE_ROWS, min(n, (int(si) + 1) * SLICE_ROWS)
+        kbs.append(kb0 if lo == lo0 else _bits(keys[lo:hi]))
+        ids.append(np.arange(lo, hi))
+        rows += hi - lo
+    # one whole query over the sample, timed end to end
+    t_scan, t_down = _oracle_query(O, cfg, kbs, np.concatenate(ids), qb, spans_h, gate_h)
+    scale = n / rows
+    per_batch = t_scan * scale + t_down
+    q = cfg["q"]
+    return {"value": q / per_batch, "unit": "queries/s", "cores": os.cpu_count(),
+            "kind": "oracle",
+            "sample": (f"1 batch of {q} query(ies): oracle scoring + top-k over {rows} of {n} "
+                       f"keys ({len(kbs)} seeded {SLICE_ROWS}-row slices copied from the device; "
+                       f"{t_scan:.2f} s, scaled by n/rows = {scale:.2f}), then gather/trie/gate "
+                       f"on that top-k ({t_down:.2f} s, unscaled); numpy fp64")}
 
 
 def run_reference(args, cfg, name):
-    """--impl reference: the CPU oracle, timed on bounded samples per step."""
+    """--impl reference: the CPU oracle on bounded samples of the same
+    workload, one query batch per step.
+
+    The store is not held: a pool of seeded 65,536-row slices of it (the
+    generator's own chunks, drawn on the GPU when there is one, so the values
+    are the main arm's), including the chunks of the step queries' source
+    keys, is made before the timed steps.  Each step scores its query batch
+    against ``--ref-slices`` slices of the pool (rotating), takes the top-k of
+    that sample and runs gather, trie and gate on it; that is the step the
+    line's ms_per_step times.  queries/s scales the scoring + top-k time by
+    n / rows scanned (the full store), the rest unscaled."""
     import oracle as O
     import synth
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    n, d = cfg["n"], cfg["d"]
-    # A step scores the query batch against one slice of the store (rows
-    # rotate over steps) and runs top-k/gather/tree/gate on that slice's
-    # candidates; queries/s = q / (slices x slice-scan time + downstream time).
-    slice_rows = min(n, 4096)
-    slices = (n + slice_rows - 1) // slice_rows
-    dev = "cpu"
-    keys = synth.clustered_unit_keys(min(n, slice_rows * 4), d, min(cfg["clusters"], 256),
-                                     seed=0, device=dev)
-    spans = synth.spans_zipf(keys.shape[0], cfg["m"], cfg["vocab"], seed=0, device=dev)
-    qs, _ = synth.noisy_queries(keys, cfg["q"], seed=1)
-    gate = make_gate_inputs(cfg, dev, sets=1)[0]
-    from tests.parity import bits, host
-    kb, sp, qb = bits(keys), host(spans), bits(qs)
-    root, nodes, hr, hn = host(gate[0]), host(gate[1]), bits(gate[2]), bits(gate[3])
-    t_scan, t_down = [], []
-    total = args.warmup + args.steps
-    t_all0 = time.perf_counter()
-    avail = keys.shape[0] // slice_rows  # distinct slices held (up to 4)
-    for it in range(total):
-        lo = (it % avail) * slice_rows
-        t0 = time.perf_counter()
-        s = O.scores(kb[lo:lo + slice_rows], qb)
-        t1 = time.perf_counter()
-        _, idx = O.topk(s, cfg["k"])
-        dr = O.gather_drafts(sp[lo:lo + slice_rows], idx)
-        tr = O.loose_trie(dr, node_cap=cfg["cap"])
-        O.soft_gate(tr["tokens"], tr["parent"], tr["num_nodes"], tr["gamma"], root, nodes, hr,
-                    hn, gamma_thr=GATE["gamma"], kappa=GATE["topk"], window=GATE["window"])
-        t2 = time.perf_counter()
-        if it >= args.warmup:
-            t_scan.append(t1 - t0)
-            t_down.append(t2 - t1)
-        if time.perf_counter() - t_all0 > 150 and len(t_scan) >= 1:
+    n, d, q = cfg["n"], cfg["d"], cfg["q"]
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    store = synth.ClusteredStoreRows(n, d, cfg["clusters"], sigma=0.3, seed=0, device=dev)
+    n_q = cfg["distinct"] * q
+    queries, src = synth.noisy_queries(store, n_q, noise=0.05, seed=1)
+    queries = queries.reshape(cfg["distinct"], q, d)
+    src = src.reshape(cfg["distinct"], q).cpu()
+    n_chunks = (n + synth.CHUNK_ROWS - 1) // synth.CHUNK_ROWS
+    per_step = max(1, min(args.ref_slices, n_chunks))
+    pool_ids = sorted(set((src[0] // synth.CHUNK_ROWS).tolist()))
+    rng = np.random.default_rng(3)
+    for c in rng.permutation(n_chunks).tolist():
+        if len(pool_ids) >= min(n_chunks, 2 * per_step):
             break
-    per_query_batch = slices * statistics.mean(t_scan) + statistics.mean(t_down)
-    value = cfg["q"] / per_query_batch
+        if c not in pool_ids:
+            pool_ids.append(c)
+    pool = {c: _bits(store.chunk(c)) for c in pool_ids}
+    if cfg["zipf"]:
+        spans = synth.spans_zipf(n, cfg["m"], cfg["vocab"], 1.1, seed=0, device=dev)
+    else:
+        spans = synth.spans_uniform(n, cfg["m"], cfg["vocab"], seed=0, device=dev)
+    spans_h = _host(spans)
+    del spans, store
+    gate_h = _gate_host(make_gate_inputs(cfg, dev, sets=1, seed=100)[0])
+    t_scan, t_down, t_step, rows_per = [], [], [], []
+    total = args.warmup + args.steps
+    for it in range(total):
+        ids = [pool_ids[(it * per_step + j) % len(pool_ids)] for j in range(per_step)]
+        kbs = [pool[c] for c in ids]
+        row_ids = np.concatenate([np.arange(c * synth.CHUNK_ROWS,
+                                            c * synth.CHUNK_ROWS + pool[c].shape[0]) for c in ids])
+        qb = _bits(queries[it % cfg["distinct"]])
+        t0 = time.perf_counter()
+        ts, td = _oracle_query(O, cfg, kbs, row_ids, qb, spans_h, gate_h)
+        el = time.perf_counter() - t0
+        if it >= args.warmup:
+            t_scan.append(ts)
+            t_down.append(td)
+            t_step.append(el)
+            rows_per.append(row_ids.size)
+    rows = statistics.mean(rows_per)
+    scale = n / rows
+    per_batch = statistics.mean(t_scan) * scale + statistics.mean(t_down)
+    value = q / per_batch
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "queries/s",
-        "n_gpus": args.gpus, "steps": len(t_scan), "warmup": args.warmup,
-        "ms_per_step": per_query_batch * 1e3, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": name, **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab", "cap")}},
+        "n_gpus": args.gpus, "steps": len(t_step), "warmup": args.warmup,
+        "ms_per_step": statistics.mean(t_step) * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": name, **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab",
+                                                             "cap", "clusters")}},
         "cpu_baseline": {"value": value, "unit": "queries/s", "cores": os.cpu_count(),
                          "kind": "oracle",
-                         "sample": f"per step: scoring of {cfg['q']} queries over one "
-                                   f"{slice_rows}-row slice (x{slices} slices per query batch) "
-                                   f"plus top-k/gather/tree/gate; numpy fp64"},
+                         "sample": (f"per step: one batch of {q} query(ies) of the workload "
+                                    f"scored against {per_step} seeded {SLICE_ROWS}-row slices "
+                                    f"of its store ({int(rows)} of {n} keys), top-k of that "
+                                    f"sample, gather/trie/gate; ms_per_step is that sampled "
+                                    f"step; value scales scoring + top-k by n/rows = "
+                                    f"{scale:.1f}; numpy fp64"),
+                         "scan_s_per_step": statistics.mean(t_scan),
+                         "downstream_s_per_step": statistics.mean(t_down)},
         "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -416,6 +488,8 @@ def main():
     ap.add_argument("--impl", default="sense", choices=["sense", "reference"])
     ap.add_argument("--workload", default=DEFAULT, choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ref-slices", type=int, default=4,
+                    help="--impl reference: 65,536-row slices of the store scored per step")
     ap.add_argument("--e2e-steps", type=int, default=200)
     ap.add_argument("--n-keys", type=int, default=0,
                     help="override the store size (small cases for profiler captures)")

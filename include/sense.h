@@ -171,14 +171,38 @@ sense_status sense_retrieve_topk(const sense_datastore* ds, const uint16_t* quer
  * bytes is rejected with SENSE_ERR_UNSUPPORTED.  All calls share the array,
  * which keeps the last call's contents (the counters that must start at zero
  * are cleared by every call); calls that overlap on the GPU race on it, so
- * order them on one stream.  Device-side checks of this function record
- * into a status word inside the array, not the one sense_device_status reads.
+ * order them on one stream.  The array's address is kept for the life of
+ * the process: no call may span a cudaDeviceReset.  Device-side checks of
+ * this function (SENSE_DEVST_INTERNAL, SENSE_DEVST_TIMEOUT) record into a
+ * status word inside the array, not the one sense_device_status reads; every
+ * call clears it first, and sense_retrieve_noalloc_status reads it.
  * Arguments, outputs and results are those of sense_retrieve_topk.
  */
 #define SENSE_NOALLOC_SCRATCH_BYTES (32u << 20)
 sense_status sense_retrieve_topk_noalloc(const sense_datastore* ds, const uint16_t* queries,
                                          int32_t q, int32_t k, float* out_scores,
                                          int32_t* out_idx, sense_stream_t stream);
+
+/*
+ * Device status of sense_retrieve_topk_noalloc on the current device (the
+ * paper has no counterpart): synchronises `stream`, copies the status word
+ * of the static array into *out_bits and, when `clear` is non-zero, zeroes
+ * it.  Read it after a call and before the next one (each call clears it).
+ * Allocates nothing.  Returns SENSE_ERR_TIMEOUT when SENSE_DEVST_TIMEOUT is
+ * set, SENSE_ERR_DEVICE_STATUS for any other bit, SENSE_OK for none; a
+ * non-OK result means that call's outputs must not be used.
+ */
+sense_status sense_retrieve_noalloc_status(sense_stream_t stream, uint32_t* out_bits,
+                                           int32_t clear);
+
+/*
+ * Failure-detection self test of that status word (the paper has no
+ * counterpart): the bounded-wait self test of sense_selftest_timeout, with
+ * its SENSE_DEVST_TIMEOUT written into the static array's status word
+ * instead of the device status word.  Read it with
+ * sense_retrieve_noalloc_status.  Allocates nothing.
+ */
+sense_status sense_retrieve_noalloc_selftest(sense_stream_t stream, int64_t limit_cycles);
 
 /* ---------------------------------------------------------------------- */
 /* Approximate retrieval: PCA projection and an IVF / IVF-PQ index          */

@@ -196,6 +196,24 @@ def sense_retrieve_topk_noalloc(ds: Datastore, queries: torch.Tensor, k: int, ou
     return out_scores, out_idx
 
 
+def sense_retrieve_noalloc_status(clear: bool = True, stream=None) -> int:
+    """Status bits the last allocation-free retrieval left (synchronises)."""
+    out = C.c_uint32(0)
+    st = lib().sense_retrieve_noalloc_status(C.c_void_p(_stream(stream)), C.byref(out),
+                                             1 if clear else 0)
+    if st not in (0, 5, 6):
+        _check(st)
+    return int(out.value)
+
+
+def sense_retrieve_noalloc_selftest(limit_cycles: int = 200_000_000, stream=None) -> int:
+    """Bounded-wait self test into the allocation-free retrieval's status
+    word; returns the bits it left (SENSE_DEVST_TIMEOUT expected) without
+    clearing them."""
+    _check(lib().sense_retrieve_noalloc_selftest(C.c_void_p(_stream(stream)), int(limit_cycles)))
+    return sense_retrieve_noalloc_status(clear=False, stream=stream)
+
+
 def sense_gather_drafts(ds: Datastore, idx: torch.Tensor, anchor=None, n_keep=None,
                         force_anchor: bool = False, out=None, stream=None) -> torch.Tensor:
     """Candidate spans [q, n_keep, m] int32 for retrieved indices idx [q, k]."""

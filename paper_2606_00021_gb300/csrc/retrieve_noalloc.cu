@@ -12,10 +12,16 @@
 // The array lives in this file's module: every GPU that loads the library
 // and uses this entry point holds its kNoallocScratchBytes until the process
 // exits.  Its device address is looked up once per device, on the first
-// call made with that device current.  All calls share the array and it
-// keeps the previous call's contents: the per-query counters are cleared on
-// every call, and calls whose work overlaps on the GPU (different streams
-// with no ordering between them) race on the array.
+// call made with that device current, and kept for the life of the process
+// (no call of this library may span a cudaDeviceReset).  All calls share the
+// array and it keeps the previous call's contents: the per-query counters
+// are cleared on every call, and calls whose work overlaps on the GPU
+// (different streams with no ordering between them) race on the array.
+//
+// The first 256 bytes of the array hold this entry point's own device
+// status word: the kernels' device-side checks (an internal consistency
+// check, a bounded wait that ran out) set bits there.  Every call clears it
+// first; sense_retrieve_noalloc_status reads it after the call.
 #include <mutex>
 
 #include "common.cuh"
@@ -92,4 +98,38 @@ extern "C" sense_status sense_retrieve_topk_noalloc(const sense_datastore* ds,
   if (st != SENSE_OK) return st;
   return run_retrieve(p, ds, queries, q, k, out_scores, out_idx, base + kStatusBytes, status,
                       stream);
+}
+
+extern "C" sense_status sense_retrieve_noalloc_status(sense_stream_t stream, uint32_t* out_bits,
+                                                      int32_t clear) {
+  if (!out_bits) return fail(SENSE_ERR_INVALID_ARG, "out_bits is NULL");
+  char* base = nullptr;
+  sense_status st = scratch_address(&base);
+  if (st != SENSE_OK) return st;
+  st = cuda_check(cudaStreamSynchronize(stream), "cudaStreamSynchronize");
+  if (st != SENSE_OK) return st;
+  uint32_t v = 0;
+  st = cuda_check(cudaMemcpy(&v, base, sizeof(v), cudaMemcpyDeviceToHost), "read status word");
+  if (st != SENSE_OK) return st;
+  if (clear) {
+    st = cuda_check(cudaMemset(base, 0, sizeof(uint32_t)), "clear status word");
+    if (st != SENSE_OK) return st;
+  }
+  *out_bits = v;
+  if (v & SENSE_DEVST_TIMEOUT)
+    return fail(SENSE_ERR_TIMEOUT, "a device wait of the allocation-free retrieval hit its limit "
+                "(bits 0x%x)", v);
+  if (v) return fail(SENSE_ERR_DEVICE_STATUS, "allocation-free retrieval status bits 0x%x", v);
+  return SENSE_OK;
+}
+
+extern "C" sense_status sense_retrieve_noalloc_selftest(sense_stream_t stream,
+                                                        int64_t limit_cycles) {
+  if (limit_cycles < 1 || limit_cycles > (1LL << 34))
+    return fail(SENSE_ERR_INVALID_ARG, "limit_cycles=%lld outside [1, 2^34]",
+                (long long)limit_cycles);
+  char* base = nullptr;
+  sense_status st = scratch_address(&base);
+  if (st != SENSE_OK) return st;
+  return launch_selftest_wait(limit_cycles, reinterpret_cast<uint32_t*>(base), stream);
 }

@@ -55,33 +55,71 @@ def clustered_unit_keys(n: int, d: int, n_clusters: int, sigma: float = 0.3,
     """bf16 [n, d] keys drawn around ``n_clusters`` unit centroids (and, with
     ``return_assign``, the int32 [n] cluster of each key)."""
     c = centroids(n_clusters, d, seed, device)
-    scale = sigma / (d ** 0.5) if reading == "A" else sigma
     if out is None:
         out = torch.empty(n, d, dtype=torch.bfloat16, device=device)
     assign = torch.empty(n, dtype=torch.int32, device=device) if return_assign else None
     for ci, lo in enumerate(range(0, n, CHUNK_ROWS)):
         hi = min(n, lo + CHUNK_ROWS)
-        g = _gen(device, _sub_seed(seed, 2, ci))
-        a = torch.randint(0, n_clusters, (hi - lo,), generator=g, device=device)
-        e = torch.randn(hi - lo, d, generator=g, device=device, dtype=torch.float32)
-        x = c[a] + scale * e
-        out[lo:hi] = _unit_rows(x).to(torch.bfloat16)
+        rows, a = _key_chunk(c, ci, hi - lo, sigma, seed, reading)
+        out[lo:hi] = rows
         if assign is not None:
             assign[lo:hi] = a.to(torch.int32)
-        del e, x
+        del rows
     return (out, assign) if return_assign else out
 
 
-def noisy_queries(keys: torch.Tensor, q: int, noise: float = 0.05, seed: int = 0,
+def _key_chunk(c: torch.Tensor, ci: int, rows: int, sigma: float, seed: int, reading: str):
+    """Chunk ``ci`` of a clustered store: (bf16 [rows, d] keys, cluster ids)."""
+    n_clusters, d = c.shape
+    scale = sigma / (d ** 0.5) if reading == "A" else sigma
+    g = _gen(c.device, _sub_seed(seed, 2, ci))
+    a = torch.randint(0, n_clusters, (rows,), generator=g, device=c.device)
+    e = torch.randn(rows, d, generator=g, device=c.device, dtype=torch.float32)
+    x = c[a] + scale * e
+    return _unit_rows(x).to(torch.bfloat16), a
+
+
+class ClusteredStoreRows:
+    """Rows of the store ``clustered_unit_keys`` draws, produced chunk by
+    chunk on demand (the same values on the same device), for consumers that
+    cannot hold the whole store."""
+
+    def __init__(self, n: int, d: int, n_clusters: int, sigma: float = 0.3, seed: int = 0,
+                 device="cpu", reading: str = "A"):
+        self.n, self.d, self.sigma, self.seed, self.reading = n, d, sigma, seed, reading
+        self.c = centroids(n_clusters, d, seed, device)
+
+    def chunk(self, ci: int) -> torch.Tensor:
+        lo = ci * CHUNK_ROWS
+        hi = min(self.n, lo + CHUNK_ROWS)
+        return _key_chunk(self.c, ci, hi - lo, self.sigma, self.seed, self.reading)[0]
+
+    def rows(self, idx: torch.Tensor) -> torch.Tensor:
+        """bf16 [len(idx), d]: the store rows at the given indices."""
+        idx = idx.to(self.c.device)
+        out = torch.empty(idx.shape[0], self.d, dtype=torch.bfloat16, device=self.c.device)
+        chunks = torch.div(idx, CHUNK_ROWS, rounding_mode="floor")
+        for ci in sorted(set(chunks.tolist())):
+            sel = chunks == ci
+            out[sel] = self.chunk(ci)[idx[sel] - ci * CHUNK_ROWS]
+        return out
+
+
+def noisy_queries(keys, q: int, noise: float = 0.05, seed: int = 0,
                   reading: str = "A"):
-    """(bf16 [q, d] queries, int64 [q] source key index)."""
-    n, d = keys.shape
-    dev = keys.device
+    """(bf16 [q, d] queries, int64 [q] source key index).  ``keys`` is the
+    store tensor, or a ``ClusteredStoreRows`` for a store that is not held."""
+    if isinstance(keys, ClusteredStoreRows):
+        n, d, dev, fetch = keys.n, keys.d, keys.c.device, keys.rows
+    else:
+        n, d = keys.shape
+        dev = keys.device
+        fetch = lambda s: keys[s]  # noqa: E731
     g = _gen(dev, _sub_seed(seed, 3))
     src = torch.randint(0, n, (q,), generator=g, device=dev)
     scale = noise / (d ** 0.5) if reading == "A" else noise
     e = torch.randn(q, d, generator=g, device=dev, dtype=torch.float32)
-    x = keys[src].float() + scale * e
+    x = fetch(src).float() + scale * e
     return _unit_rows(x).to(torch.bfloat16), src
 
 

@@ -53,6 +53,11 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert b"SENSE_DS_NORMALIZE" in lib.sense_last_error()
     # retrieve / gather on a NULL handle
     assert lib.sense_retrieve_topk(None, p, 1, 1, p, p, p, 1 << 20, None) == 1
+    assert lib.sense_retrieve_topk_noalloc(None, p, 1, 1, p, p, None) == 1
+    # allocation-free status reader and self test: NULL output, limit range
+    assert lib.sense_retrieve_noalloc_status(None, None, 1) == 1
+    assert lib.sense_retrieve_noalloc_selftest(None, 0) == 1
+    assert lib.sense_retrieve_noalloc_selftest(None, (1 << 34) + 1) == 1
     assert lib.sense_gather_drafts(None, p, 1, 1, None, 1, 0, p, None) == 1
     # tree: k, m, k*m, cap, flags
     args = (p, p, p, p, p, None, None)

@@ -1,11 +1,14 @@
 """Parity at the workloads' full sizes, in the launch configuration bench.py
 times (one call per query batch, the same k, m, cap and gate parameters).
 
-The full stores are too large for the oracle to score every key, so
-retrieval is checked on sampled outputs the oracle computes one by one: for
-each query, the oracle scores (a) every key it returned, (b) every key of the
+Retrieval is checked exhaustively for a seeded subset of queries: the oracle
+scores every key of the store (copied to the host in 65,536-row slices) and
+the full top-k rule applies (4 steps of the 1M-key store, 1 step of the
+137 GB store, every query of one 16-query batch of the 4M-key store and of
+the 64-query batches of the 2M-key sweeps, every query of the tiny store).  The other checked queries use sampled outputs the
+oracle computes one by one: (a) every key returned, (b) every key of the
 query's source cluster and (c) a seeded random sample of the store (about
-1 GB of keys).  The returned scores must match, the order must agree, no
+1 GB of keys).  Their returned scores must match, the order must agree, no
 sampled key may beat the returned k-th by more than the tolerance, and the
 query's source key must be returned.  Gather, tree and gate run on seeded
 inputs drawn from each workload's distributions and are compared bit for bit
@@ -20,7 +23,7 @@ import torch
 import oracle as O
 import synth
 from synth.workloads import WORKLOADS
-from tests.parity import SCORE_TOL, bits, host
+from tests.parity import SCORE_TOL, bits, check_topk, host
 
 pytestmark = pytest.mark.gpu
 cuda = pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")
@@ -68,9 +71,27 @@ def _check_query(keys, assign_h, q_bits, src, sc, ix, k, sample_rows):
     assert src in set(ret.tolist()), "the query's source key was not returned"
 
 
+def _exhaustive_scores(keys, q_bits):
+    """The oracle's scores of every key of the store for the given queries
+    (fp64 [q, n]), the keys copied to the host one 65,536-row slice at a
+    time."""
+    n = keys.shape[0]
+    out = np.empty((q_bits.shape[0], n), dtype=np.float64)
+    for lo in range(0, n, 65536):
+        hi = min(n, lo + 65536)
+        out[:, lo:hi] = O.scores(bits(keys[lo:hi]), q_bits)
+    return out
+
+
+# queries checked against every key of the store: (query batches, queries per batch)
+EXHAUSTIVE = {"tiny_4k": (1, 8), "llama7b_1m": (4, 1), "llama70b_8m": (1, 1),
+              "qwen7b_4m": (1, 16), "sweep_2m_k16": (1, 64), "sweep_2m_k64": (1, 64),
+              "sweep_2m_k256": (1, 64)}
+
+
 @cuda
 @pytest.mark.parametrize("name", ["tiny_4k", "llama7b_1m", "qwen7b_4m", "llama70b_8m",
-                                  "sweep_2m_k256"])
+                                  "sweep_2m_k16", "sweep_2m_k64", "sweep_2m_k256"])
 def test_full_size_retrieval(S, name):
     cfg = WORKLOADS[name]
     dev = torch.device("cuda")
@@ -87,19 +108,39 @@ def test_full_size_retrieval(S, name):
     rng = np.random.default_rng(7)
     n_sample = min(n, (1 << 30) // (d * 2))
     sample_rows = np.sort(rng.choice(n, size=n_sample, replace=False))
-    checked = 0
+    results = []
     for b in range(batches):
         qb = qs[b * q:(b + 1) * q].contiguous()
         sc, ix = S.sense_retrieve_topk(ds, qb, k, workspace=ws)
         torch.cuda.synchronize()
         assert S.sense_device_status(clear=True) == 0
-        # every query of the batch (up to 64)
+        results.append((qb, host(sc), host(ix)))
+    ex_b, ex_q = EXHAUSTIVE.get(name, (0, 0))
+    checked = exhaustive = 0
+    if ex_b:
+        q_bits = np.concatenate([bits(results[b][0][:ex_q]) for b in range(ex_b)])
+        full = _exhaustive_scores(keys, q_bits)
+        row = 0
+        for b in range(ex_b):
+            _, sc_h, ix_h = results[b]
+            for qi in range(ex_q):
+                check_topk(sc_h[qi], ix_h[qi], full[row], k)
+                assert int(src[b * q + qi]) in set(ix_h[qi].tolist())
+                row += 1
+                exhaustive += 1
+        del full
+    for b in range(batches):
+        qb, sc_h, ix_h = results[b]
+        # every query of the batch (up to 64) not already checked exhaustively
         pick = range(q) if q <= 64 else sorted(rng.choice(q, size=64, replace=False).tolist())
         for qi in pick:
-            _check_query(keys, assign_h, bits(qb[qi:qi + 1]), int(src[b * q + qi]), sc[qi],
-                         ix[qi], k, sample_rows)
+            if b < ex_b and qi < ex_q:
+                continue
+            _check_query(keys, assign_h, bits(qb[qi:qi + 1]), int(src[b * q + qi]),
+                         torch.from_numpy(sc_h[qi]), torch.from_numpy(ix_h[qi]), k, sample_rows)
             checked += 1
-    assert checked >= 3
+    assert checked + exhaustive >= 3
+    assert exhaustive == ex_b * ex_q
     del ds, keys, spans, assign, qs, ws
     _free()
 
@@ -134,14 +175,17 @@ def test_full_size_gather_and_tree(S, name):
 
 
 @cuda
-@pytest.mark.parametrize("name,nq,plant", [
-    ("tiny_4k", 8, True), ("llama7b_1m", 4, False), ("llama7b_1m", 4, True),
-    ("qwen7b_4m", 3, True), ("llama70b_8m", 3, True), ("sweep_2m_k16", 4, True),
-    ("sweep_2m_k64", 2, True), ("sweep_2m_k256", 1, True), ("sweep_2m_k256", 1, False),
+@pytest.mark.parametrize("name,nq,plant,seed", [
+    ("tiny_4k", 8, True, 7), ("llama7b_1m", 4, False, 5), ("llama7b_1m", 4, True, 5),
+    ("qwen7b_4m", 3, True, 7), ("llama70b_8m", 3, True, 7), ("sweep_2m_k16", 4, True, 7),
+    ("sweep_2m_k64", 2, True, 7), ("sweep_2m_k256", 1, True, 5), ("sweep_2m_k256", 1, False, 5),
 ])
-def test_full_size_gate(S, name, nq, plant):
+def test_full_size_gate(S, name, nq, plant, seed):
     """Gate at the workload's vocabulary, hidden size, k, m and cap on seeded
-    trees (spans drawn from a small vocabulary so that prefixes are shared)."""
+    trees (spans drawn from a small vocabulary so that prefixes are shared).
+    The logits seeds are chosen so that no query has a normalised entropy
+    within the 1e-4 band of the threshold (the fixture check below allows at
+    most one such query per case, and never all of them)."""
     cfg = WORKLOADS[name]
     dev = torch.device("cuda")
     k, m, v, d = cfg["k"], cfg["m"], cfg["vocab"], cfg["d"]
@@ -156,12 +200,12 @@ def test_full_size_gate(S, name, nq, plant):
         sp[qi] = rows
     tr = O.loose_trie(sp, node_cap=cfg["cap"])
     cap = tr["tokens"].shape[1]
-    root = synth.gate_logits(nq, 1, v, seed=5)[:, 0].contiguous()
-    nodes = synth.gate_logits(nq, cap, v, seed=6)
+    root = synth.gate_logits(nq, 1, v, seed=seed)[:, 0].contiguous()
+    nodes = synth.gate_logits(nq, cap, v, seed=seed + 1)
     if plant:
         synth.plant_gate_rows(root, nodes, torch.from_numpy(tr["tokens"]),
                               torch.from_numpy(tr["parent"]), torch.from_numpy(tr["num_nodes"]),
-                              seed=5)
+                              seed=seed)
     hr = synth.gate_hidden(nq, 1, d, seed=5)[:, 0].contiguous()
     hn = synth.gate_hidden(nq, cap, d, seed=6)
     tree = {key: torch.from_numpy(tr[key]).to(dev) for key in
@@ -174,7 +218,7 @@ def test_full_size_gate(S, name, nq, plant):
                        kappa=GATE["topk"], window=GATE["window"], tau=GATE["tau"],
                        ent_band=1e-4)
     ok = ~want["ambiguous"]
-    assert ok.any(), "every query hit the entropy ambiguity band"
+    assert ok.any() and (~ok).sum() <= 1, "fixture: too many near-threshold entropies"
     for key in ("i_star", "L_star", "n_accept", "next_node", "next_anchor"):
         np.testing.assert_array_equal(host(got[key])[ok], want[key][ok], err_msg=key)
     np.testing.assert_array_equal(host(got["accepted"])[ok], want["accepted"][ok])

@@ -329,7 +329,7 @@ def test_gate_matches_oracle(S, q, k, m, v, cap, gamma, kappa, w, tau, unnorm):
                        host(nodes), bits(hr), bits(hn), gamma_thr=gamma, kappa=kappa,
                        window=w, tau=tau, unnormalized_entropy=unnorm, ent_band=1e-4)
     ok = ~want["ambiguous"]
-    assert ok.mean() >= 0.5, "too many near-threshold entropies in the fixture"
+    assert ok.any() and (~ok).sum() <= 1, "fixture: too many near-threshold entropies"
     for key in ("i_star", "L_star", "n_accept", "next_node", "next_anchor"):
         np.testing.assert_array_equal(host(got[key])[ok], want[key][ok], err_msg=key)
     np.testing.assert_array_equal(host(got["accepted"])[ok], want["accepted"][ok])
