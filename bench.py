@@ -136,11 +136,17 @@ def job_throughput(units_per_rank: int, world: int, seconds: float) -> float:
     return world * units_per_rank / seconds
 
 
-def make_workload(cfg, dev, seed=0):
+def make_workload(cfg, dev, seed=0, key_recipe=None):
     import synth
     n, d, m = cfg["n"], cfg["d"], cfg["m"]
-    keys, assign = synth.clustered_unit_keys(n, d, cfg["clusters"], sigma=0.3, seed=seed,
-                                             device=dev, return_assign=True)
+    if key_recipe and key_recipe.get("kind") == "subspace":
+        keys, assign = synth.subspace_unit_keys(n, d, cfg["clusters"], rank=key_recipe["rank"],
+                                                decay=key_recipe["decay"], sigma=0.3,
+                                                iso=key_recipe["iso"], seed=seed, device=dev,
+                                                return_assign=True)
+    else:
+        keys, assign = synth.clustered_unit_keys(n, d, cfg["clusters"], sigma=0.3, seed=seed,
+                                                 device=dev, return_assign=True)
     if cfg["zipf"]:
         spans = synth.spans_zipf(n, m, cfg["vocab"], 1.1, seed=seed, device=dev)
     else:
@@ -302,7 +308,8 @@ def build_ann(S, keys, kind, nlist, nprobe, pq_m, v, dev, seed=0):
     cov = (xc.T @ xc / xc.shape[0]).double().cpu().numpy()
     del sample, xc
     import scipy.linalg
-    _, evecs = scipy.linalg.eigh(cov, subset_by_index=[d - v, d - 1])
+    evals, evecs = scipy.linalg.eigh(cov, subset_by_index=[d - v, d - 1])
+    energy = float(evals.sum() / np.trace(cov))  # variance kept by the v components
     basis = torch.from_numpy(np.ascontiguousarray(evecs[:, ::-1].T)).float().to(dev).contiguous()
     mean = mean.contiguous()
     del cov, evecs
@@ -329,6 +336,7 @@ def build_ann(S, keys, kind, nlist, nprobe, pq_m, v, dev, seed=0):
     return {"index": ix, "basis": basis, "mean": mean, "nprobe": nprobe, "kind": kind,
             "keys_proj": kp,
             "nlist": nlist, "pq_m": pq_m if kind == "ivfpq" else 0, "v": v,
+            "pca_energy": energy,
             "build_s": build_s, "mean_list": float(sizes.mean()), "max_list": ix.max_list}
 
 
@@ -497,6 +505,12 @@ def main():
                     help="override the queries per step (small cases for profiler captures)")
     ap.add_argument("--retrieval", default="exact", choices=["exact", "ivfpq", "ivfflat"],
                     help="exact scan of the full keys, or the PCA + IVF index of App. E")
+    ap.add_argument("--keys", default="clustered", choices=["clustered", "subspace"],
+                    help="key recipe: isotropic clusters in d dimensions, or clusters and "
+                         "spread inside a low-dimensional subspace (power-law spectrum)")
+    ap.add_argument("--key-rank", type=int, default=256)
+    ap.add_argument("--key-decay", type=float, default=1.0)
+    ap.add_argument("--key-iso", type=float, default=0.05)
     ap.add_argument("--nlist", type=int, default=4096)
     ap.add_argument("--nprobe", type=int, default=32)
     ap.add_argument("--pq-m", type=int, default=16)
@@ -541,7 +555,9 @@ def main():
     _build.build()
     S.lib()
 
-    keys, spans, queries, assign = make_workload(cfg, dev, seed=rank)
+    key_recipe = ({"kind": "subspace", "rank": args.key_rank, "decay": args.key_decay,
+                   "iso": args.key_iso} if args.keys == "subspace" else {"kind": "clustered"})
+    keys, spans, queries, assign = make_workload(cfg, dev, seed=rank, key_recipe=key_recipe)
     cap = cfg["cap"] if cfg["cap"] > 0 else cfg["k"] * cfg["m"]
     gate_bytes = cfg["q"] * (cap + 1) * cfg["vocab"] * 4
     n_sets = 4 if gate_bytes < (2 << 30) else 1
@@ -721,6 +737,7 @@ def main():
         ann.pop("keys_proj")
         retrieval = {"kind": ann["kind"], "proj_dim": v_, "nlist": nl, "nprobe": ann["nprobe"],
                      "pq_m": pq_m, "build_s": round(ann["build_s"], 3),
+                     "pca_energy": ann["pca_energy"],
                      "mean_list": ann["mean_list"], "max_list": ann["max_list"],
                      "entries_scanned_per_query": per_q,
                      "recall_at_k_vs_exact": float(np.mean(hits)),
@@ -881,6 +898,7 @@ def main():
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded clustered unit-norm keys, Zipf spans, N(0,9) logits)",
             "config": {"workload": args.workload, "retrieval": args.retrieval,
+                       "keys": key_recipe,
                        "dynamic_capacity": args.dynamic, "verify_heads": args.verify,
                        **{k: cfg[k] for k in ("n", "d", "q", "k", "m", "vocab", "cap", "clusters")},
                        "key_bytes": n * d * 2,

@@ -11,6 +11,12 @@ chunk, independent of the device that draws them):
   sphere and stored as bf16.  Noise reading "A" draws N(0, sigma^2/d) per
   coordinate (noise vector norm ~ sigma); reading "B" draws N(0, sigma^2)
   per coordinate.
+* subspace keys (approximate-retrieval studies): the clusters and the spread
+  within them live in a random ``rank``-dimensional subspace of R^d whose
+  coordinates have a power-law spectrum (scale (i+1)^-decay), plus a small
+  isotropic noise of norm ~``iso``; back on the unit sphere, bf16.  Hidden
+  states concentrate their energy in few directions like this; isotropic
+  clusters in d dimensions do not.
 * queries: a uniformly chosen key plus Gaussian noise (same readings), back
   on the unit sphere, as bf16; the source key index is returned.
 * lattice keys/queries: entries from {-3..3} * 2^-6 (exact in bf16, and all
@@ -121,6 +127,34 @@ def noisy_queries(keys, q: int, noise: float = 0.05, seed: int = 0,
     e = torch.randn(q, d, generator=g, device=dev, dtype=torch.float32)
     x = fetch(src).float() + scale * e
     return _unit_rows(x).to(torch.bfloat16), src
+
+
+def subspace_unit_keys(n: int, d: int, n_clusters: int, rank: int = 256, decay: float = 1.0,
+                       sigma: float = 0.3, iso: float = 0.05, seed: int = 0, device="cpu",
+                       out: torch.Tensor | None = None, return_assign: bool = False):
+    """bf16 [n, d] unit keys whose clusters and within-cluster spread lie in a
+    random ``rank``-dimensional subspace (power-law coordinate scales), plus
+    isotropic noise of norm ~``iso`` (and, with ``return_assign``, the int32
+    cluster of each key)."""
+    g = _gen(device, _sub_seed(seed, 13))
+    basis = torch.linalg.qr(torch.randn(d, rank, generator=g, device=device))[0]  # [d, rank]
+    scale = torch.arange(1, rank + 1, device=device, dtype=torch.float32).pow(-decay)
+    scale = scale / scale.norm()
+    cz = torch.randn(n_clusters, rank, generator=g, device=device) * scale
+    if out is None:
+        out = torch.empty(n, d, dtype=torch.bfloat16, device=device)
+    assign = torch.empty(n, dtype=torch.int32, device=device) if return_assign else None
+    for ci, lo in enumerate(range(0, n, CHUNK_ROWS)):
+        hi = min(n, lo + CHUNK_ROWS)
+        gc = _gen(device, _sub_seed(seed, 14, ci))
+        a = torch.randint(0, n_clusters, (hi - lo,), generator=gc, device=device)
+        z = cz[a] + sigma * scale * torch.randn(hi - lo, rank, generator=gc, device=device)
+        x = z @ basis.T + (iso / d ** 0.5) * torch.randn(hi - lo, d, generator=gc, device=device)
+        out[lo:hi] = _unit_rows(x).to(torch.bfloat16)
+        if assign is not None:
+            assign[lo:hi] = a.to(torch.int32)
+        del z, x
+    return (out, assign) if return_assign else out
 
 
 def lattice_rows(n: int, d: int, seed: int = 0, device="cpu") -> torch.Tensor:
