@@ -125,6 +125,56 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
+// The head's splits (one cluster) merge their partials: row r is done by
+// CTA r % splits, one warp per row, reading every split's statistics and rows
+// through distributed shared memory, in the order of
+// tree_attn_combine_kernel.  `so` is this CTA's partial O [128][128] f32
+// followed by its statistics [128][2].
+__device__ __forceinline__ void cluster_merge(const float* so, const AttnArgs& a, int h, int sp,
+                                              int warp, int lane) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  cl.sync();
+  const int nsp = a.splits;
+  const float* sml = so + 128 * kHd;
+  const float NEG = -__int_as_float(0x7f800000);
+  for (int r = sp + nsp * warp; r < a.L; r += nsp * (kAttnThreads / 32)) {
+    float ref_s = NEG, l_s = 0.0f;
+    if (lane < nsp) {
+      const float* m = cl.map_shared_rank(sml, (unsigned)lane) + 2 * r;
+      ref_s = m[0];
+      l_s = m[1];
+    }
+    float mx = (lane < nsp && l_s > 0.0f) ? ref_s : NEG;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    float f = 0.0f, l = 0.0f;
+    if (lane < nsp) {
+      l = l_s;
+      if (l > 0.0f) f = exp2f(ref_s - mx);
+      else l = 0.0f;
+    }
+    float fl = f * l;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) fl += __shfl_xor_sync(0xffffffffu, fl, off);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int t = 0; t < nsp; ++t) {
+      const float ft = __shfl_sync(0xffffffffu, f, t);
+      if (ft == 0.0f) continue;  // warp-uniform
+      const float4 o =
+          *reinterpret_cast<const float4*>(cl.map_shared_rank(so, (unsigned)t) + r * kHd + 4 * lane);
+      acc.x += ft * o.x;
+      acc.y += ft * o.y;
+      acc.z += ft * o.z;
+      acc.w += ft * o.w;
+    }
+    const float inv = fl > 0.0f ? 1.0f / fl : 0.0f;
+    *reinterpret_cast<float4*>(a.out + ((int64_t)h * a.L + r) * kHd + 4 * lane) =
+        make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+  }
+  cl.sync();  // the other CTAs' shared memory stays alive until it is read
+}
+
 __global__ void __launch_bounds__(kAttnThreads, 1)
 tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                  const __grid_constant__ CUtensorMap tm_vt, const AttnArgs a) {
@@ -444,54 +494,465 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
   }
-  if (a.fused) {
-    // the head's splits (one cluster) merge their partials: row r is done by
-    // CTA r % splits, one warp per row, reading every split's statistics and
-    // rows through distributed shared memory, in the order of
-    // tree_attn_combine_kernel
-    namespace cg = cooperative_groups;
-    cg::cluster_group cl = cg::this_cluster();
-    cl.sync();
-    const int nsp = a.splits;
-    const float* so = reinterpret_cast<const float*>(s_kv);
-    const float* sml = so + 128 * kHd;
-    const float NEG = -__int_as_float(0x7f800000);
-    for (int r = sp + nsp * warp; r < a.L; r += nsp * (kAttnThreads / 32)) {
-      float ref_s = NEG, l_s = 0.0f;
-      if (lane < nsp) {
-        const float* m = cl.map_shared_rank(sml, (unsigned)lane) + 2 * r;
-        ref_s = m[0];
-        l_s = m[1];
-      }
-      float mx = (lane < nsp && l_s > 0.0f) ? ref_s : NEG;
+  if (a.fused) cluster_merge(reinterpret_cast<const float*>(s_kv), a, h, sp, warp, lane);
+}
+
+// ---------------------------------------------------------------------------
+// Transposed products for trees of at most 64 nodes.
+//
+// With L <= 64 draft tokens, half of the M = 128 rows of S = Q K^T and of
+// O = P V are padding, and an MMA of M <= 128 costs about N cycles per K = 16
+// step whatever M is.  This kernel computes both products transposed, with
+// the 64 token columns as N:
+//   S^T = K Q^T   (M = 128 keys of a block, N = 64 tokens, K = 128 dims)
+//   O^T += V^T P^T (M = 128 dims, N = 64 tokens, K = 128 keys)
+// which halves the tensor time per key and, with 128-key blocks, halves the
+// exponentials per key (no padding rows).  In TMEM a softmax thread now owns
+// one key (a lane) and 32 token columns, so the row statistics need cross-
+// thread reductions; they are only needed when the lazy-rescale test fires:
+//  - every thread keeps the per-token reference maxima ref_t of its 32
+//    tokens (the same values in every thread of a token half);
+//  - per block, each thread tests whether any visible score exceeds its
+//    token's reference by more than 2^8 (log2 domain); one barrier-reduction
+//    over the 256 softmax threads decides for the CTA;
+//  - only then (always on the first block) the block maxima per token are
+//    reduced (a 31-shuffle transposing reduction per warp, the four lane
+//    quarters through shared memory), the references raised, and the
+//    thread's row sums and its O^T columns rescaled;
+//  - P = 2^(s - ref_t) is rounded to bf16 and written to P[token][key] in the
+//    swizzled K-major layout the product reads; each thread adds its rounded
+//    values into per-token partial row sums, reduced across keys once at
+//    the end.
+// K and V^T tiles have separate rings (3 and 2 stages of 32 KB), so keys can
+// be loaded ahead while the products of earlier blocks still hold their
+// V^T tiles.  The split partials and their merge are those of
+// tree_attn_kernel.
+constexpr int kTB = 128;                  // keys per block
+constexpr int kTN = 64;                   // token columns (N of both products)
+constexpr int kTSlabQ = kTN * 128;        // 64 rows x 64 bf16 (one swizzle slab)
+constexpr int kTQBytes = 2 * kTSlabQ;     // Q: 64 tokens x 128 dims
+constexpr int kTPBytes = 2 * kTSlabQ;     // P: 64 tokens x 128 keys
+constexpr int kTSlab = 128 * 128;         // 128 rows x 64 bf16
+constexpr int kTKBytes = 2 * kTSlab;      // K tile: 128 keys x 128 dims
+constexpr int kTVBytes = 2 * kTSlab;      // V^T tile: 128 dims x 128 keys
+constexpr int kTKStages = 3;
+constexpr int kTVStages = 2;
+constexpr int kTNBars = 1 + 2 * kTKStages + 2 * kTVStages + 8 + 2;
+
+struct AttnTShared {
+  uint32_t tmem_base;
+  int abort;
+  uint32_t maskT[kTN][2];   // tree key j: bit t of word t / 32 set iff node j is visible to token t
+  float4 qmax[kTN];         // per token: block maxima of the four lane quarters
+  float4 qsum[kTN];         // per token: row sums of the four lane quarters
+  float ref[kTN];           // per token: reference maximum (log2 domain)
+  float factor[kTN];        // per token: rescale factor of the last raise
+};
+
+size_t attn_t_smem_bytes() {
+  return 1024 + kTQBytes + 2 * kTPBytes + kTKStages * kTKBytes + kTVStages * kTVBytes +
+         kTNBars * 8 + 16 + sizeof(AttnTShared);
+}
+
+// Barrier over the 256 softmax threads that also returns whether any of them
+// passed `p` (bar.red.or).
+__device__ __forceinline__ bool soft_any(bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.or.pred po, 2, 256, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)p)
+      : "memory");
+  return r != 0;
+}
+__device__ __forceinline__ void soft_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+// After the call, lane i holds op over the warp's 32 lanes of v[i] (each
+// lane passes 32 values indexed by token).  Five exchange rounds: in round
+// `off` a lane keeps the half of its remaining values selected by its bit
+// `off` and receives the partner's copy of that half.
+template <bool kMax>
+__device__ __forceinline__ float transpose_reduce(float (&v)[32], int lane) {
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      float f = 0.0f, l = 0.0f;
-      if (lane < nsp) {
-        l = l_s;
-        if (l > 0.0f) f = exp2f(ref_s - mx);
-        else l = 0.0f;
-      }
-      float fl = f * l;
+  for (int off = 16; off > 0; off >>= 1) {
+    const bool upper = (lane & off) != 0;
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) fl += __shfl_xor_sync(0xffffffffu, fl, off);
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int t = 0; t < nsp; ++t) {
-        const float ft = __shfl_sync(0xffffffffu, f, t);
-        if (ft == 0.0f) continue;  // warp-uniform
-        const float4 o =
-            *reinterpret_cast<const float4*>(cl.map_shared_rank(so, (unsigned)t) + r * kHd + 4 * lane);
-        acc.x += ft * o.x;
-        acc.y += ft * o.y;
-        acc.z += ft * o.z;
-        acc.w += ft * o.w;
-      }
-      const float inv = fl > 0.0f ? 1.0f / fl : 0.0f;
-      *reinterpret_cast<float4*>(a.out + ((int64_t)h * a.L + r) * kHd + 4 * lane) =
-          make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+    for (int i = 0; i < off; ++i) {
+      const float keep = upper ? v[i + off] : v[i];
+      const float send = upper ? v[i] : v[i + off];
+      const float got = __shfl_xor_sync(0xffffffffu, send, off);
+      v[i] = kMax ? fmaxf(keep, got) : keep + got;
     }
-    cl.sync();  // the other CTAs' shared memory stays alive until it is read
   }
+  return v[0];
+}
+
+__global__ void __launch_bounds__(kAttnThreads, 1)
+tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                   const __grid_constant__ CUtensorMap tm_vt, const AttnArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* s_q = smem;                          // Q tile (B of S^T)
+  uint8_t* s_p = s_q + kTQBytes;                // two P tiles (B of O^T)
+  uint8_t* s_k = s_p + 2 * kTPBytes;            // K ring (A of S^T)
+  uint8_t* s_v = s_k + kTKStages * kTKBytes;    // V^T ring (A of O^T)
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_v + kTVStages * kTVBytes);
+  const int Q_FULL = 0, K_FULL = 1, K_EMPTY = 1 + kTKStages, V_FULL = 1 + 2 * kTKStages,
+            V_EMPTY = V_FULL + kTVStages, S_FULL = V_EMPTY + kTVStages, S_EMPTY = S_FULL + 2,
+            P_FULL = S_EMPTY + 2, P_EMPTY = P_FULL + 2, O_DONE = P_EMPTY + 2,
+            MMA_DONE = O_DONE + 1;
+  AttnTShared* sh = reinterpret_cast<AttnTShared*>(
+      (reinterpret_cast<uintptr_t>(bars + kTNBars) + 15) & ~static_cast<uintptr_t>(15));
+  volatile int* abort = &sh->abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x, sp = blockIdx.y;
+  const int j0 = sp * a.bps;
+  const int j1 = min(a.nb, j0 + a.bps);
+  const int nbl = max(0, j1 - j0);
+  auto bar = [&](int i) { return ptx::smem_u32(bars + i); };
+
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(bar(Q_FULL), 1);
+    for (int s = 0; s < kTKStages; ++s) {
+      ptx::mbar_init(bar(K_FULL + s), 1);
+      ptx::mbar_init(bar(K_EMPTY + s), 1);
+    }
+    for (int s = 0; s < kTVStages; ++s) {
+      ptx::mbar_init(bar(V_FULL + s), 1);
+      ptx::mbar_init(bar(V_EMPTY + s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      ptx::mbar_init(bar(S_FULL + b), 1);
+      ptx::mbar_init(bar(S_EMPTY + b), kSoftWarps);
+      ptx::mbar_init(bar(P_FULL + b), kSoftWarps);
+      ptx::mbar_init(bar(P_EMPTY + b), 1);
+    }
+    ptx::mbar_init(bar(O_DONE), 1);
+    ptx::mbar_init(bar(MMA_DONE), 1);
+    sh->abort = 0;
+    ptx::fence_barrier_init();
+    ptx::prefetch_tensormap(&tm_q);
+    ptx::prefetch_tensormap(&tm_k);
+    ptx::prefetch_tensormap(&tm_vt);
+  }
+  if (warp == 1) ptx::tmem_alloc(ptx::smem_u32(&sh->tmem_base), 256);
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = sh->tmem_base;  // S^T buffers at columns 0 and kTN, O^T at 2 kTN
+
+  if (warp == 0 && lane == 0 && nbl > 0) {
+    // ------------------------------------------------ TMA producer
+    // K and V^T tiles are issued in block order as their ring slots free up;
+    // the slot tests do not block, so a late V^T slot does not hold back
+    // the next K tile.
+    const uint64_t pol_stream = ptx::policy_evict_first();
+    const uint64_t pol_keep = ptx::policy_evict_last();
+    ptx::mbar_arrive_expect_tx(bar(Q_FULL), kTQBytes);
+    ptx::tma_load_3d(ptx::smem_u32(s_q), &tm_q, bar(Q_FULL), 0, 0, h, pol_keep);
+    ptx::tma_load_3d(ptx::smem_u32(s_q + kTSlabQ), &tm_q, bar(Q_FULL), 64, 0, h, pol_keep);
+    int jk = 0, jv = 0;
+    long long t0 = clock64();
+    while ((jk < nbl || jv < nbl) && !*abort) {
+      bool moved = false;
+      if (jk < nbl && ptx::mbar_try_wait(bar(K_EMPTY + jk % kTKStages),
+                                         (uint32_t)(((jk / kTKStages) & 1) ^ 1))) {
+        const int s = jk % kTKStages;
+        uint8_t* st = s_k + s * kTKBytes;
+        const int key0 = (j0 + jk) * kTB;
+        ptx::mbar_arrive_expect_tx(bar(K_FULL + s), kTKBytes);
+        ptx::tma_load_3d(ptx::smem_u32(st), &tm_k, bar(K_FULL + s), 0, key0, h, pol_stream);
+        ptx::tma_load_3d(ptx::smem_u32(st + kTSlab), &tm_k, bar(K_FULL + s), 64, key0, h,
+                         pol_stream);
+        ++jk;
+        moved = true;
+      }
+      if (jv < nbl && jv < jk &&
+          ptx::mbar_try_wait(bar(V_EMPTY + jv % kTVStages), (uint32_t)(((jv / kTVStages) & 1) ^ 1))) {
+        const int s = jv % kTVStages;
+        uint8_t* st = s_v + s * kTVBytes;
+        const int key0 = (j0 + jv) * kTB;
+        ptx::mbar_arrive_expect_tx(bar(V_FULL + s), kTVBytes);
+        ptx::tma_load_3d(ptx::smem_u32(st), &tm_vt, bar(V_FULL + s), key0, 0, h, pol_stream);
+        ptx::tma_load_3d(ptx::smem_u32(st + kTSlab), &tm_vt, bar(V_FULL + s), key0 + 64, 0, h,
+                         pol_stream);
+        ++jv;
+        moved = true;
+      }
+      if (moved) {
+        t0 = clock64();
+      } else if (clock64() - t0 > kWaitCycles) {
+        *abort = 1;
+        raise_status(a.status, SENSE_DEVST_TIMEOUT);
+      }
+    }
+    drain_bar(bar(Q_FULL), 0);
+    if (*abort) {  // wait (bounded) for the copies that may still be in flight
+      for (int j = max(0, jk - kTKStages); j < jk; ++j)
+        drain_bar(bar(K_FULL + j % kTKStages), (uint32_t)((j / kTKStages) & 1));
+      for (int j = max(0, jv - kTVStages); j < jv; ++j)
+        drain_bar(bar(V_FULL + j % kTVStages), (uint32_t)((j / kTVStages) & 1));
+    }
+  } else if (warp == 1 && lane == 0 && nbl > 0) {
+    // ------------------------------------------------ MMA issuer
+    const uint32_t idesc = ptx::idesc_bf16_f32(128, kTN);
+    const uint32_t q_addr = ptx::smem_u32(s_q), p_addr = ptx::smem_u32(s_p);
+    bool ok = wait_bar(bar(Q_FULL), 0, abort, a.status);
+    auto pv = [&](int i) -> bool {
+      const int pb = i & 1, sv = i % kTVStages;
+      if (!wait_bar(bar(P_FULL + pb), (uint32_t)((i >> 1) & 1), abort, a.status) ||
+          !wait_bar(bar(V_FULL + sv), (uint32_t)((i / kTVStages) & 1), abort, a.status))
+        return false;
+      ptx::tc_fence_after();
+      const uint32_t vt = ptx::smem_u32(s_v + sv * kTVBytes);
+      const uint32_t pa = p_addr + pb * kTPBytes;
+#pragma unroll
+      for (int ks = 0; ks < 2; ++ks)
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          ptx::mma_bf16(tmem + 2 * kTN, ptx::desc_sw128(vt + ks * kTSlab + t * 32),
+                        ptx::desc_sw128(pa + ks * kTSlabQ + t * 32), idesc,
+                        (i > 0 || ks > 0 || t > 0) ? 1u : 0u);
+      ptx::mma_commit(bar(O_DONE));
+      ptx::mma_commit(bar(P_EMPTY + pb));
+      ptx::mma_commit(bar(V_EMPTY + sv));
+      return true;
+    };
+    for (int jj = 0; jj < nbl && ok; ++jj) {
+      const int s = jj % kTKStages, b = jj & 1;
+      if (!wait_bar(bar(K_FULL + s), (uint32_t)((jj / kTKStages) & 1), abort, a.status) ||
+          !wait_bar(bar(S_EMPTY + b), (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      const uint32_t kt = ptx::smem_u32(s_k + s * kTKBytes);
+#pragma unroll
+      for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          ptx::mma_bf16(tmem + kTN * b, ptx::desc_sw128(kt + kc * kTSlab + t * 32),
+                        ptx::desc_sw128(q_addr + kc * kTSlabQ + t * 32), idesc,
+                        (kc > 0 || t > 0) ? 1u : 0u);
+      ptx::mma_commit(bar(S_FULL + b));
+      ptx::mma_commit(bar(K_EMPTY + s));
+      if (jj > 0 && !pv(jj - 1)) ok = false;
+    }
+    if (ok) pv(nbl - 1);
+    ptx::mma_commit(bar(MMA_DONE));
+    drain_bar(bar(MMA_DONE), 0);
+  } else if (warp >= 2) {
+    // ------------------------------------------------ softmax / epilogue
+    // Warp w owns TMEM lane quarter q4 = w & 3: keys 32 q4 + lane of a block
+    // in S^T, dims 32 q4 + lane in O^T; `half` selects its 32 token columns.
+    const int q4 = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const int tb = 32 * half;                 // first token of this thread
+    const uint32_t lane_base = tmem + ((uint32_t)(q4 * 32) << 16);
+    const int kl = 32 * q4 + lane;            // this thread's key within a block
+    const float NEG = -__int_as_float(0x7f800000);
+    // transposed tree mask: warp w' = w - 2 ballots tokens 32 (w' & 1) + lane
+    // for tree keys j in [16 (w' >> 1), +16)
+    {
+      const int wp = warp - 2;
+      const int t = 32 * (wp & 1) + lane;
+      uint32_t m0 = 0u, m1 = 0u;
+      if (t < a.L) {
+        const uint32_t* mr = a.mask + (int64_t)t * a.mask_words;
+        m0 = mr[0];
+        if (a.mask_words > 1) m1 = mr[1];
+      }
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int j = 16 * (wp >> 1) + i;
+        const uint32_t bit = ((j < 32 ? m0 : m1) >> (j & 31)) & 1u;
+        const uint32_t word = __ballot_sync(0xffffffffu, bit != 0u && j < a.L);
+        if (lane == 0) sh->maskT[j][wp & 1] = word;
+      }
+    }
+    if (warp < 4) sh->ref[32 * (warp - 2) + lane] = NEG;
+    soft_sync();
+    float psum[32];
+#pragma unroll
+    for (int u = 0; u < 32; ++u) psum[u] = 0.0f;
+    const float4* ref4 = reinterpret_cast<const float4*>(sh->ref + tb);
+    // P[token][key]: slab kl / 64, 16-byte chunk (kl % 64) / 8 swizzled by
+    // token % 8 inside the token's 128-byte row, 2 bytes per key
+    const int g = (kl & 63) >> 3;
+    const uint32_t p_off = (uint32_t)((kl >> 6) * kTSlabQ + ((kl & 7) << 1));
+    bool ok = true;
+    for (int jj = 0; jj < nbl; ++jj) {
+      const int b = jj & 1;
+      ok = __all_sync(0xffffffffu,
+                      ok && wait_bar(bar(S_FULL + b), (uint32_t)((jj >> 1) & 1), abort, a.status));
+      float x[32];
+      uint32_t vis = 0u;  // visibility of this thread's 32 tokens
+      if (ok) {
+        ptx::tc_fence_after();
+        {
+          uint32_t rr[2][16];
+          ptx::tmem_ld16_nowait(lane_base + kTN * b + tb, rr[0]);
+          ptx::tmem_ld16_nowait(lane_base + kTN * b + tb + 16, rr[1]);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            x[e] = __uint_as_float(rr[0][e]) * a.scale_log2;
+            x[16 + e] = __uint_as_float(rr[1][e]) * a.scale_log2;
+          }
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(bar(S_EMPTY + b));
+        const int key = (j0 + jj) * kTB + kl;
+        if (key < a.m) {
+          vis = a.L >= tb + 32 ? 0xffffffffu : (a.L <= tb ? 0u : ((1u << (a.L - tb)) - 1u));
+        } else if (key < a.m + a.L) {
+          vis = sh->maskT[key - a.m][half];
+        }
+      }
+      // lazy-rescale test over the CTA
+      bool exceed = false;
+#pragma unroll
+      for (int u4 = 0; u4 < 8; ++u4) {
+        const float4 r4 = ref4[u4];
+        exceed |= ((vis >> (4 * u4)) & 1u) && (x[4 * u4] > r4.x + kRescale);
+        exceed |= ((vis >> (4 * u4 + 1)) & 1u) && (x[4 * u4 + 1] > r4.y + kRescale);
+        exceed |= ((vis >> (4 * u4 + 2)) & 1u) && (x[4 * u4 + 2] > r4.z + kRescale);
+        exceed |= ((vis >> (4 * u4 + 3)) & 1u) && (x[4 * u4 + 3] > r4.w + kRescale);
+      }
+      // P buffer b is free once the product of block jj - 2 is done; after
+      // this wait at most the product of block jj - 1 is still running, so
+      // the O_DONE phase tested below is that product's
+      ok = __all_sync(0xffffffffu, ok && wait_bar(bar(P_EMPTY + b),
+                                                 (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status));
+      if (soft_any(ok && exceed)) {
+        {
+          float bm[32];
+#pragma unroll
+          for (int u = 0; u < 32; ++u) bm[u] = ((vis >> u) & 1u) ? x[u] : NEG;
+          const float wmax = transpose_reduce<true>(bm, lane);  // token tb + lane, this quarter
+          reinterpret_cast<float*>(&sh->qmax[tb + lane])[q4] = wmax;
+        }
+        soft_sync();
+        if (q4 == 0) {  // one thread per token raises its reference
+          const int t = tb + lane;
+          const float4 qm = sh->qmax[t];
+          const float m4 = fmaxf(fmaxf(qm.x, qm.y), fmaxf(qm.z, qm.w));
+          const float r = sh->ref[t];
+          float f = 1.0f;
+          if (m4 > r + kRescale) {
+            if (r != NEG) f = ex2(r - m4);
+            sh->ref[t] = m4;
+          }
+          sh->factor[t] = f;
+        }
+        soft_sync();
+        const float4* f4 = reinterpret_cast<const float4*>(sh->factor + tb);
+        bool rescale = false;
+#pragma unroll
+        for (int u4 = 0; u4 < 8; ++u4) {
+          const float4 f = f4[u4];
+          psum[4 * u4] *= f.x;
+          psum[4 * u4 + 1] *= f.y;
+          psum[4 * u4 + 2] *= f.z;
+          psum[4 * u4 + 3] *= f.w;
+          rescale |= (f.x != 1.0f) || (f.y != 1.0f) || (f.z != 1.0f) || (f.w != 1.0f);
+        }
+        // this warp's O^T columns (its tokens, its dims) must hold the
+        // product of block jj - 1 before they are scaled
+        if (__any_sync(0xffffffffu, rescale) && ok) {
+          ok = __all_sync(0xffffffffu,
+                          wait_bar(bar(O_DONE), (uint32_t)((jj - 1) & 1), abort, a.status));
+          if (ok) {
+            ptx::tc_fence_after();
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+              uint32_t rr[16];
+              const uint32_t ta = lane_base + 2 * kTN + tb + 16 * c;
+              ptx::tmem_ld16(ta, rr);
+#pragma unroll
+              for (int e = 0; e < 16; ++e)
+                rr[e] = __float_as_uint(__uint_as_float(rr[e]) * sh->factor[tb + 16 * c + e]);
+              ptx::tmem_st16(ta, rr);
+            }
+          }
+        }
+      }
+      if (!ok) continue;
+      uint8_t* prow = s_p + b * kTPBytes + p_off + tb * 128;
+#pragma unroll
+      for (int u4 = 0; u4 < 8; ++u4) {
+        const float4 r4 = ref4[u4];
+        const float rv[4] = {r4.x, r4.y, r4.z, r4.w};
+#pragma unroll
+        for (int e = 0; e < 4; e += 2) {
+          const int u = 4 * u4 + e;
+          const float p0 = ((vis >> u) & 1u) ? ex2(x[u] - rv[e]) : 0.0f;
+          const float p1 = ((vis >> (u + 1)) & 1u) ? ex2(x[u + 1] - rv[e + 1]) : 0.0f;
+          const uint32_t pk = pack_bf16(p0, p1);
+          psum[u] += __uint_as_float(pk << 16);
+          psum[u + 1] += __uint_as_float(pk & 0xffff0000u);
+          *reinterpret_cast<uint16_t*>(prow + u * 128 + ((g ^ (u & 7)) << 4)) =
+              (uint16_t)(pk & 0xffffu);
+          *reinterpret_cast<uint16_t*>(prow + (u + 1) * 128 + ((g ^ ((u + 1) & 7)) << 4)) =
+              (uint16_t)(pk >> 16);
+        }
+      }
+      ptx::fence_proxy_async_smem();
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(bar(P_FULL + b));
+    }
+    // row sums: this warp's 32 keys, then the four lane quarters
+    const float wsum = transpose_reduce<false>(psum, lane);  // token tb + lane
+    reinterpret_cast<float*>(&sh->qsum[tb + lane])[q4] = wsum;
+    const bool done =
+        __all_sync(0xffffffffu, ok && nbl > 0 && wait_bar(bar(MMA_DONE), 0, abort, a.status));
+    soft_sync();
+    // partial output of this split in row layout [token][dim]: into global
+    // memory, or (fused) into this CTA's shared memory where the K ring was
+    // (every load has landed, every product is done once MMA_DONE completed)
+    float* so = reinterpret_cast<float*>(s_k);   // fused: [128][128] partial O
+    float* sml = so + 128 * kHd;                  // fused: [128][2] statistics
+    const int dim = 32 * q4 + lane;
+    const int64_t pbase = ((int64_t)h * a.splits + sp) * 128;
+    if (done && tb < a.L) {
+      ptx::tc_fence_after();
+      uint32_t rr[2][16];
+      ptx::tmem_ld16_nowait(lane_base + 2 * kTN + tb, rr[0]);
+      ptx::tmem_ld16_nowait(lane_base + 2 * kTN + tb + 16, rr[1]);
+      ptx::tmem_ld_wait();
+#pragma unroll
+      for (int u = 0; u < 32; ++u) {
+        const int t = tb + u;
+        if (t < a.L) {
+          const float v = __uint_as_float(rr[u >> 4][u & 15]);
+          if (a.fused) so[t * kHd + dim] = v;
+          else a.part_o[(pbase + t) * kHd + dim] = v;
+        }
+      }
+    }
+    if (q4 == 0) {
+      const int t = tb + lane;
+      const float4 qs = sh->qsum[t];
+      float* pml = a.fused ? sml + 2 * t : a.part_ml + (pbase + t) * 2;
+      if (t < a.L) {
+        pml[0] = done ? sh->ref[t] : NEG;
+        pml[1] = done ? (qs.x + qs.y) + (qs.z + qs.w) : 0.0f;
+      }
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, 256);
+  }
+  if (a.fused) cluster_merge(reinterpret_cast<const float*>(s_k), a, h, sp, warp, lane);
 }
 
 // out[h, r, :] = sum_s 2^(ref_s - M) O_s / sum_s 2^(ref_s - M) l_s, one warp
@@ -577,6 +1038,76 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// Trees of at most 64 nodes: the transposed-product kernel over 128-key
+// blocks (splits of a head merged in their cluster when <= 8, else by
+// tree_attn_combine_kernel through the workspace).
+sense_status launch_attn_t(const uint16_t* q, const uint16_t* k_cache, const uint16_t* vt_cache,
+                           int heads, int L, int capacity, int prefix_len,
+                           const uint32_t* mask_bits, int mask_words, float scale, float* out,
+                           void* workspace, uint32_t* status, cudaStream_t s) {
+  const int n = prefix_len + L;
+  const int nb = (n + kTB - 1) / kTB;
+  const int splits = attn_splits(heads, nb);
+  alignas(64) CUtensorMap tm_q, tm_k, tm_vt;
+  // Q [H, L, 128] in boxes of 64 rows (rows past L read as zero); K [H,
+  // capacity, 128] seen up to n keys in boxes of 128 keys; V^T [H, 128,
+  // capacity] up to n keys
+  sense_status st =
+      make_map3(&tm_q, q, kHd, L, heads, (uint64_t)kHd * 2, (uint64_t)L * kHd * 2, kTN);
+  if (st == SENSE_OK)
+    st = make_map3(&tm_k, k_cache, kHd, n, heads, (uint64_t)kHd * 2, (uint64_t)capacity * kHd * 2,
+                   kTB);
+  if (st == SENSE_OK)
+    st = make_map3(&tm_vt, vt_cache, n, kHd, heads, (uint64_t)capacity * 2,
+                   (uint64_t)kHd * capacity * 2, 128);
+  if (st != SENSE_OK) return st;
+  AttnArgs a{};
+  a.L = L;
+  a.m = prefix_len;
+  a.n = n;
+  a.nb = nb;
+  a.splits = splits;
+  a.bps = (nb + splits - 1) / splits;
+  a.scale_log2 = scale * 1.4426950408889634f;
+  a.mask = mask_bits;
+  a.mask_words = mask_words;
+  char* ws = static_cast<char*>(workspace);
+  a.part_o = reinterpret_cast<float*>(ws);
+  a.part_ml = reinterpret_cast<float*>(ws + align256((size_t)heads * splits * 128 * kHd * 4));
+  a.status = status;
+  a.out = out;
+  a.fused = splits <= 8 ? 1 : 0;
+  const size_t smem = attn_t_smem_bytes();
+  st = cuda_check(cudaFuncSetAttribute(tree_attn_t_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                  "cudaFuncSetAttribute(tree_attn_t)");
+  if (st != SENSE_OK) return st;
+  {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)heads, (unsigned)splits);
+    cfg.blockDim = dim3(kAttnThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = a.fused ? (unsigned)splits : 1u;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    LaunchScope ls(K_TREE_ATTN, s);
+    st = cuda_check(cudaLaunchKernelEx(&cfg, tree_attn_t_kernel, tm_q, tm_k, tm_vt, a),
+                    "launch tree attention (transposed)");
+    if (st != SENSE_OK) return st;
+  }
+  if (a.fused) return SENSE_OK;
+  LaunchScope ls(K_TREE_ATTN, s);
+  const int64_t threads = (int64_t)heads * L * 32;
+  tree_attn_combine_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(
+      a.part_o, a.part_ml, heads, splits, L, out);
+  return cuda_check(cudaGetLastError(), "launch tree attention combine");
+}
+
 }  // namespace
 }  // namespace sense
 
@@ -618,6 +1149,8 @@ sense_status sense_tree_attention(const uint16_t* q, const uint16_t* k_cache,
   if (!status) return SENSE_ERR_OOM;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int n = prefix_len + L;
+  if (L <= kTN) return launch_attn_t(q, k_cache, vt_cache, heads, L, capacity, prefix_len, mask_bits,
+                                     mask_words, scale, out, workspace, status, s);
   const int nb = (n + kBN - 1) / kBN;
   const int splits = attn_splits(heads, nb);
   alignas(64) CUtensorMap tm_q, tm_k, tm_vt;

@@ -42,6 +42,13 @@ def _tree(seed, k, m_span, vocab, cap):
     (3, 1, 1, 1, 0, 128), (8, 24, 8, 100, 1000, 1152), (1, 40, 16, 128, 130, 384),
     (4, 32, 16, 64, 2000, 2176),   # exactly 64 draft tokens (two lane quarters)
     (4, 32, 16, 65, 2000, 2176),   # one row into the third quarter
+    # trees of <= 64 nodes (transposed products over 128-key blocks):
+    (2, 16, 8, 64, 3000, 3200),    # 24 key splits: merged through the workspace
+    (1, 8, 4, 32, 8000, 8192),     # 63 key splits (more than one warp of splits)
+    (8, 24, 8, 64, 1000, 1152),    # tree keys straddle two key blocks; 9 splits
+    (32, 24, 8, 64, 1000, 1152),   # the same in a cluster of 4 splits, one without blocks
+    (4, 5, 4, 20, 0, 128),         # no committed prefix: every key is a tree node
+    (6, 2, 16, 17, 129, 256),      # a 16-node chain and a branch, prefix past a block edge
 ])
 def test_tree_attention_matches_oracle(S, heads, k, m_span, cap, prefix, capacity):
     dev = torch.device("cuda")
@@ -67,14 +74,16 @@ def test_tree_attention_matches_oracle(S, heads, k, m_span, cap, prefix, capacit
 
 
 @cuda
-def test_tree_attention_large_logits_rescale(S):
+@pytest.mark.parametrize("heads,capacity,prefix", [(2, 1024, 900), (40, 4096, 3900)])
+def test_tree_attention_large_logits_rescale(S, heads, capacity, prefix):
     """Keys aligned with the queries make later blocks' logits exceed the
     running maximum by far more than 2^8: the lazy rescale of O must keep the
-    result exact within the tolerance."""
+    result exact within the tolerance (one key block per split, and about
+    eleven blocks per split)."""
     dev = torch.device("cuda")
     tr = _tree(5, 8, 4, 3, 32)
     L = int(tr["num_nodes"][0])
-    heads, D, capacity, prefix = 2, 128, 1024, 900
+    D = 128
     g = torch.Generator().manual_seed(4)
     q = torch.randn(heads, L, D, generator=g)
     kc = 0.05 * torch.randn(heads, capacity, D, generator=g)
