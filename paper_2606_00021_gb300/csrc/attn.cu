@@ -648,8 +648,8 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
   if (warp == 0 && lane == 0 && nbl > 0) {
     // ------------------------------------------------ TMA producer
     // K and V^T tiles are issued in block order as their ring slots free up;
-    // the slot tests do not block, so a late V^T slot does not hold back
-    // the next K tile.
+    // the slot tests do not block (test_wait), so a late V^T slot does not
+    // hold back the next K tile or the other way round.
     const uint64_t pol_stream = ptx::policy_evict_first();
     const uint64_t pol_keep = ptx::policy_evict_last();
     ptx::mbar_arrive_expect_tx(bar(Q_FULL), kTQBytes);
@@ -659,8 +659,8 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     long long t0 = clock64();
     while ((jk < nbl || jv < nbl) && !*abort) {
       bool moved = false;
-      if (jk < nbl && ptx::mbar_try_wait(bar(K_EMPTY + jk % kTKStages),
-                                         (uint32_t)(((jk / kTKStages) & 1) ^ 1))) {
+      if (jk < nbl && ptx::mbar_test_wait(bar(K_EMPTY + jk % kTKStages),
+                                          (uint32_t)(((jk / kTKStages) & 1) ^ 1))) {
         const int s = jk % kTKStages;
         uint8_t* st = s_k + s * kTKBytes;
         const int key0 = (j0 + jk) * kTB;
@@ -672,7 +672,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
         moved = true;
       }
       if (jv < nbl && jv < jk &&
-          ptx::mbar_try_wait(bar(V_EMPTY + jv % kTVStages), (uint32_t)(((jv / kTVStages) & 1) ^ 1))) {
+          ptx::mbar_test_wait(bar(V_EMPTY + jv % kTVStages), (uint32_t)(((jv / kTVStages) & 1) ^ 1))) {
         const int s = jv % kTVStages;
         uint8_t* st = s_v + s * kTVBytes;
         const int key0 = (j0 + jv) * kTB;
