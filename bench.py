@@ -190,12 +190,19 @@ class Pipeline:
         self.gws = S.alloc_workspace(S.sense_soft_gate_workspace_bytes(q, self.cap, GATE["topk"]), dev)
 
     def use_ann(self, ann, dev):
-        """Retrieve through the projected IVF index instead of the exact scan."""
+        """Retrieve through the projected IVF index instead of the exact scan;
+        with ann["rerank"] = N' > 0 the index returns N' candidates whose exact
+        similarity to the full query ranks them (Eq. 8's sim) before the top k
+        are kept."""
         q, k = self.cfg["q"], self.cfg["k"]
         self.ann = ann
+        kk = max(k, ann.get("rerank", 0))
         self.qproj = torch.empty(q, ann["index"].v, dtype=torch.float32, device=dev)
+        if ann.get("rerank", 0):
+            self.cand_s = torch.empty(q, kk, dtype=torch.float32, device=dev)
+            self.cand_i = torch.empty(q, kk, dtype=torch.int32, device=dev)
         self.ws = self.S.alloc_workspace(
-            self.S.sense_ivf_search_workspace_bytes(ann["index"], q, k, ann["nprobe"]), dev)
+            self.S.sense_ivf_search_workspace_bytes(ann["index"], q, kk, ann["nprobe"]), dev)
 
     def retrieve(self, query):
         S, cfg = self.S, self.cfg
@@ -204,8 +211,13 @@ class Pipeline:
         else:
             a = self.ann
             S.sense_project(query, a["basis"], a["mean"], out=self.qproj)
-            S.sense_ivf_search(a["index"], self.qproj, cfg["k"], a["nprobe"], self.scores,
-                               self.idx, workspace=self.ws)
+            if a.get("rerank", 0):
+                S.sense_ivf_search(a["index"], self.qproj, a["rerank"], a["nprobe"], self.cand_s,
+                                   self.cand_i, workspace=self.ws)
+                S.sense_rescore_topk(self.ds, query, self.cand_i, cfg["k"], self.scores, self.idx)
+            else:
+                S.sense_ivf_search(a["index"], self.qproj, cfg["k"], a["nprobe"], self.scores,
+                                   self.idx, workspace=self.ws)
 
     def use_dynamic(self, ctx, kd, delta, dev):
         """Hybrid retrieval (Alg. 2): the dynamic buffer is searched beside the
@@ -263,7 +275,7 @@ class Pipeline:
 
 
 DRAFT_KERNELS = ("scan_gemv", "scan_tc", "threshold", "merge", "pad_queries", "gather", "tree",
-                 "project", "ivf_coarse", "ivf_scan", "ctx")
+                 "project", "ivf_coarse", "ivf_scan", "ctx", "rescore")
 
 
 def draft_kernel_rate(prof, q, tokens_per_query, steps):
@@ -513,6 +525,9 @@ def main():
     ap.add_argument("--key-rank", type=int, default=256)
     ap.add_argument("--key-decay", type=float, default=1.0)
     ap.add_argument("--key-iso", type=float, default=0.05)
+    ap.add_argument("--rerank", type=int, default=0, metavar="N_PRIME",
+                    help="approximate retrieval: take N' candidates from the index and keep "
+                         "the top k by their exact similarity to the full query (Eq. 8)")
     ap.add_argument("--nlist", type=int, default=4096)
     ap.add_argument("--nprobe", type=int, default=32)
     ap.add_argument("--pq-m", type=int, default=16)
@@ -571,6 +586,7 @@ def main():
     if args.retrieval != "exact":
         ann = build_ann(S, keys, args.retrieval, args.nlist, args.nprobe, args.pq_m,
                         args.proj_dim, dev, seed=rank)
+        ann["rerank"] = args.rerank
         pipe.use_ann(ann, dev)
     if args.verify:
         if cfg["q"] != 1 or pipe.cap > 128:
@@ -717,6 +733,8 @@ def main():
         kb = {"project": v_ * d * 4 + q * d * 2 + q * v_ * 4,
               "ivf_coarse": nl * v_ * 4 + q * nl * 8,
               "ivf_scan": q * per_q * entry}
+        if ann.get("rerank", 0):
+            kb["rescore"] = q * ann["rerank"] * (d * 2 + 4)
         scan_name = max(kb, key=lambda name: prof.get(name, (0.0, 0))[0])
         scan_bytes_per_step = kb[scan_name]
         step_bytes = sum(kb.values())
@@ -742,6 +760,7 @@ def main():
                      "pca_energy": ann["pca_energy"],
                      "mean_list": ann["mean_list"], "max_list": ann["max_list"],
                      "entries_scanned_per_query": per_q,
+                     "rerank_candidates": ann.get("rerank", 0),
                      "recall_at_k_vs_exact": float(np.mean(hits)),
                      "recall_at_k_vs_exact_projected": float(np.mean(hits_p)),
                      "recall_queries": len(hits)}

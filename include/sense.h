@@ -82,6 +82,7 @@ typedef enum sense_status {
 
 /* Limits. */
 #define SENSE_MAX_K 1024          /* retrieval top-k                          */
+#define SENSE_MAX_RESCORE 1024    /* shortlist length of sense_rescore_topk   */
 #define SENSE_MAX_M 32            /* span length                              */
 #define SENSE_MAX_TREE_TOKENS 8192 /* k * m accepted by sense_build_tree      */
 #define SENSE_MAX_KAPPA 16        /* gate top-k                               */
@@ -313,6 +314,28 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
                               int32_t nprobe, float* out_scores, int32_t* out_idx,
                               int32_t* out_probes, void* workspace, size_t workspace_bytes,
                               sense_stream_t stream);
+
+/*
+ * Exact re-scoring of an approximate shortlist (Sec. 3.2.2 Eq. 8: the
+ * composite score ranks the N' retrieved candidates D_ret by sim(h, k_i),
+ * the similarity of the full hidden state to each candidate's key, and keeps
+ * the top N).  For each query q, the score of candidate c is
+ * <queries[q], keys[cand_idx[q, c]]> over the datastore's stored bf16 keys
+ * with fp32 accumulation (the arithmetic of sense_retrieve_topk), and the k
+ * best candidates are written in the order (score desc, key index asc).
+ *
+ * queries: bf16 [q, d] (the full hidden states), 16-byte aligned;
+ * cand_idx: int32 [q, n_cand] key indices, -1 for an empty slot (what
+ * sense_ivf_search writes when fewer than N' keys were found);
+ * out_scores: f32 [q, k], out_idx: int32 [q, k]; slots beyond the valid
+ * candidates get -inf / -1.  Device pointers owned by the caller; no
+ * workspace.  Limits: 1 <= q <= 65535, 1 <= k <= n_cand <= SENSE_MAX_RESCORE.
+ * An index outside [0, n) is treated as empty and sets
+ * SENSE_DEVST_BAD_INDEX.  Asynchronous on `stream`.
+ */
+sense_status sense_rescore_topk(const sense_datastore* ds, const uint16_t* queries, int32_t q,
+                                const int32_t* cand_idx, int32_t n_cand, int32_t k,
+                                float* out_scores, int32_t* out_idx, sense_stream_t stream);
 
 /* ---------------------------------------------------------------------- */
 /* a4. Span gather                                                          */

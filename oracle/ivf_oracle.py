@@ -16,6 +16,8 @@ pipeline in numpy:
   ivf_build      cell assignment, inverted lists, flat vectors or PQ codes
   ivf_search     coarse top-nprobe, list scan, exact top-k of the
                  approximate scores
+  rescore_topk   Eq. 8's sim(h, k_i) over the N' retrieved candidates,
+                 exactly, and the top N of them
 
 Precision.  The projection (query and key construction) is a plain linear
 map followed by a normalisation, and its oracle is that definition in fp64:
@@ -39,7 +41,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from .sense_oracle import bf16_bits_to_f64
+from .sense_oracle import bf16_bits_to_f64, scores
 
 F32 = np.float32
 FIX = float(2 ** 31)  # fixed-point scale of the k-means sums
@@ -253,6 +255,33 @@ def ivf_search(index: dict, centroids: np.ndarray, queries: np.ndarray, nprobe: 
         out_s[qi, :len(o)] = s[o]
         out_i[qi, :len(o)] = i[o]
     return out_s, out_i, probes
+
+
+def rescore_topk(keys_bits: np.ndarray, queries_bits: np.ndarray, cand: np.ndarray, k: int):
+    """Exact similarity of each query's candidates, then its top k (Sec.
+    3.2.2 Eq. 8: the approximate search returns N' candidates D_ret, the
+    composite score ranks them by sim(h, k_i) between the full hidden state
+    and each candidate's key, and Top-N keeps N of them).
+
+    keys_bits [n, d] and queries_bits [q, d] bf16 bit patterns, cand [q, N']
+    int key indices with -1 for an empty slot.  sim is the fp64 inner
+    product of the stored bf16 values (``scores``).  The top k are ordered
+    by (score desc, key index asc); slots beyond the valid candidates hold
+    -inf / -1.  Returns (scores [q, k] f64, idx [q, k] int32).
+    """
+    cand = np.asarray(cand)
+    nq = cand.shape[0]
+    out_s = np.full((nq, k), -np.inf)
+    out_i = np.full((nq, k), -1, dtype=np.int32)
+    for qi in range(nq):
+        c = cand[qi][cand[qi] >= 0].astype(np.int64)
+        if c.size == 0:
+            continue
+        s = scores(np.asarray(keys_bits)[c], np.asarray(queries_bits)[qi:qi + 1])[0]
+        order = np.lexsort((c, -s))[:k]
+        out_s[qi, :order.size] = s[order]
+        out_i[qi, :order.size] = c[order]
+    return out_s, out_i
 
 
 def recall_at_k(approx_idx: np.ndarray, exact_idx: np.ndarray) -> float:

@@ -214,6 +214,27 @@ def sense_retrieve_noalloc_selftest(limit_cycles: int = 200_000_000, stream=None
     return sense_retrieve_noalloc_status(clear=False, stream=stream)
 
 
+def sense_rescore_topk(ds: Datastore, queries: torch.Tensor, cand_idx: torch.Tensor, k: int,
+                       out_scores=None, out_idx=None, stream=None):
+    """Exact scores of a shortlist of key indices per query (-1 = empty) and
+    the top k of it by (score desc, index asc): Eq. 8's sim(h, k_i) over the
+    approximate search's candidates."""
+    _need(queries, "queries", torch.bfloat16, 2)
+    _need(cand_idx, "cand_idx", torch.int32, 2)
+    q, n_cand = cand_idx.shape
+    if queries.shape != (q, ds.d):
+        raise ValueError("queries must be [q, d] with q = cand_idx rows")
+    dev = queries.device
+    if out_scores is None:
+        out_scores = torch.empty(q, k, dtype=torch.float32, device=dev)
+    if out_idx is None:
+        out_idx = _i32((q, k), dev)
+    _check(lib().sense_rescore_topk(C.c_void_p(ds.handle), queries.data_ptr(), q,
+                                    cand_idx.data_ptr(), n_cand, k, out_scores.data_ptr(),
+                                    out_idx.data_ptr(), C.c_void_p(_stream(stream))))
+    return out_scores, out_idx
+
+
 def sense_gather_drafts(ds: Datastore, idx: torch.Tensor, anchor=None, n_keep=None,
                         force_anchor: bool = False, out=None, stream=None) -> torch.Tensor:
     """Candidate spans [q, n_keep, m] int32 for retrieved indices idx [q, k]."""

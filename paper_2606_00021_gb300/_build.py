@@ -19,7 +19,7 @@ OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libsense.so")
 
 SOURCES = ["api.cu", "scan_gemv.cu", "scan_tc.cu", "select.cu", "draft.cu", "gate.cu",
-           "retrieve_noalloc.cu", "ivf.cu", "ctx.cu", "attn.cu"]
+           "retrieve_noalloc.cu", "ivf.cu", "ctx.cu", "attn.cu", "rescore.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-Xptxas", "-v"]

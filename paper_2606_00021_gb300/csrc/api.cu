@@ -32,7 +32,7 @@ const char* const kKernelNames[K_COUNT] = {
     "normalize", "scan_gemv", "scan_tc", "threshold", "merge",
     "gather",    "tree",      "gate_rows", "gate_decide", "pad_queries",
     "tree_mask", "project",  "kmeans",    "ivf_build", "ivf_coarse",
-    "ivf_scan",  "ctx",       "tree_attn"};
+    "ivf_scan",  "ctx",       "tree_attn", "rescore"};
 
 cudaEvent_t take_event() {
   if (!g_ev_pool.empty()) {
@@ -379,6 +379,24 @@ sense_status sense_retrieve_topk(const sense_datastore* ds, const uint16_t* quer
   if (!status) return SENSE_ERR_OOM;
   return run_retrieve(p, ds, queries, q, k, out_scores, out_idx, static_cast<char*>(workspace),
                       status, stream);
+}
+
+sense_status sense_rescore_topk(const sense_datastore* ds, const uint16_t* queries, int32_t q,
+                                const int32_t* cand_idx, int32_t n_cand, int32_t k,
+                                float* out_scores, int32_t* out_idx, sense_stream_t stream) {
+  sense_status st = check_ds(ds);
+  if (st != SENSE_OK) return st;
+  if (!queries || !cand_idx || !out_scores || !out_idx)
+    return fail(SENSE_ERR_INVALID_ARG, "queries, candidates and outputs must be non-NULL");
+  if (q < 1 || q > 65535) return fail(SENSE_ERR_INVALID_ARG, "q=%d outside [1, 65535]", q);
+  if (n_cand < 1 || n_cand > SENSE_MAX_RESCORE)
+    return fail(SENSE_ERR_INVALID_ARG, "n_cand=%d outside [1, %d]", n_cand, SENSE_MAX_RESCORE);
+  if (k < 1 || k > n_cand) return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, n_cand=%d]", k, n_cand);
+  if (!aligned(queries, 16)) return fail(SENSE_ERR_INVALID_ARG, "queries must be 16-byte aligned");
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  return launch_rescore(ds->keys, ds->n, ds->d, queries, q, cand_idx, n_cand, k, out_scores,
+                        out_idx, status, stream);
 }
 
 sense_status sense_gather_drafts(const sense_datastore* ds, const int32_t* idx, int32_t q,

@@ -131,14 +131,14 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 // tree_attn_combine_kernel.  `so` is this CTA's partial O [128][128] f32
 // followed by its statistics [128][2].
 __device__ __forceinline__ void cluster_merge(const float* so, const AttnArgs& a, int h, int sp,
-                                              int warp, int lane) {
+                                              int warp, int lane, int nwarps) {
   namespace cg = cooperative_groups;
   cg::cluster_group cl = cg::this_cluster();
   cl.sync();
   const int nsp = a.splits;
   const float* sml = so + 128 * kHd;
   const float NEG = -__int_as_float(0x7f800000);
-  for (int r = sp + nsp * warp; r < a.L; r += nsp * (kAttnThreads / 32)) {
+  for (int r = sp + nsp * warp; r < a.L; r += nsp * nwarps) {
     float ref_s = NEG, l_s = 0.0f;
     if (lane < nsp) {
       const float* m = cl.map_shared_rank(sml, (unsigned)lane) + 2 * r;
@@ -494,7 +494,8 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
   }
-  if (a.fused) cluster_merge(reinterpret_cast<const float*>(s_kv), a, h, sp, warp, lane);
+  if (a.fused)
+    cluster_merge(reinterpret_cast<const float*>(s_kv), a, h, sp, warp, lane, kAttnThreads / 32);
 }
 
 // ---------------------------------------------------------------------------
@@ -529,6 +530,9 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
 // tree_attn_kernel.
 constexpr int kTB = 128;                  // keys per block
 constexpr int kTN = 64;                   // token columns (N of both products)
+constexpr int kTSoftWarps = 16;           // four per TMEM lane quarter
+constexpr int kTTok = kTN / 4;            // token columns per softmax thread
+constexpr int kTThreads = (2 + kTSoftWarps) * 32;
 constexpr int kTSlabQ = kTN * 128;        // 64 rows x 64 bf16 (one swizzle slab)
 constexpr int kTQBytes = 2 * kTSlabQ;     // Q: 64 tokens x 128 dims
 constexpr int kTPBytes = 2 * kTSlabQ;     // P: 64 tokens x 128 keys
@@ -554,30 +558,33 @@ size_t attn_t_smem_bytes() {
          kTNBars * 8 + 16 + sizeof(AttnTShared);
 }
 
-// Barrier over the 256 softmax threads that also returns whether any of them
+// Barrier over the softmax threads that also returns whether any of them
 // passed `p` (bar.red.or).
 __device__ __forceinline__ bool soft_any(bool p) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred pi, po;\n\t"
       "setp.ne.u32 pi, %1, 0;\n\t"
-      "bar.red.or.pred po, 2, 256, pi;\n\t"
+      "bar.red.or.pred po, 2, %2, pi;\n\t"
       "selp.u32 %0, 1, 0, po;\n\t}"
       : "=r"(r)
-      : "r"((uint32_t)p)
+      : "r"((uint32_t)p), "n"(kTSoftWarps * 32)
       : "memory");
   return r != 0;
 }
-__device__ __forceinline__ void soft_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+__device__ __forceinline__ void soft_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kTSoftWarps * 32) : "memory");
+}
 
-// After the call, lane i holds op over the warp's 32 lanes of v[i] (each
-// lane passes 32 values indexed by token).  Five exchange rounds: in round
-// `off` a lane keeps the half of its remaining values selected by its bit
-// `off` and receives the partner's copy of that half.
+// Lane i (and lane i ^ 16) ends up with op over the warp's 32 lanes of
+// v[i % 16] (each lane passes 16 values indexed by token).  Four exchange
+// rounds: in round `off` a lane keeps the half of its remaining values
+// selected by its bit `off` and receives the partner's copy of that half;
+// a last exchange combines the two half-warps.
 template <bool kMax>
-__device__ __forceinline__ float transpose_reduce(float (&v)[32], int lane) {
+__device__ __forceinline__ float transpose_reduce(float (&v)[kTTok], int lane) {
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
+  for (int off = kTTok / 2; off > 0; off >>= 1) {
     const bool upper = (lane & off) != 0;
 #pragma unroll
     for (int i = 0; i < off; ++i) {
@@ -587,10 +594,11 @@ __device__ __forceinline__ float transpose_reduce(float (&v)[32], int lane) {
       v[i] = kMax ? fmaxf(keep, got) : keep + got;
     }
   }
-  return v[0];
+  const float other = __shfl_xor_sync(0xffffffffu, v[0], 16);
+  return kMax ? fmaxf(v[0], other) : v[0] + other;
 }
 
-__global__ void __launch_bounds__(kAttnThreads, 1)
+__global__ void __launch_bounds__(kTThreads, 1)
 tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_vt, const AttnArgs a) {
   extern __shared__ uint8_t smem_raw[];
@@ -627,8 +635,8 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     }
     for (int b = 0; b < 2; ++b) {
       ptx::mbar_init(bar(S_FULL + b), 1);
-      ptx::mbar_init(bar(S_EMPTY + b), kSoftWarps);
-      ptx::mbar_init(bar(P_FULL + b), kSoftWarps);
+      ptx::mbar_init(bar(S_EMPTY + b), kTSoftWarps);
+      ptx::mbar_init(bar(P_FULL + b), kTSoftWarps);
       ptx::mbar_init(bar(P_EMPTY + b), 1);
     }
     ptx::mbar_init(bar(O_DONE), 1);
@@ -748,15 +756,16 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
   } else if (warp >= 2) {
     // ------------------------------------------------ softmax / epilogue
     // Warp w owns TMEM lane quarter q4 = w & 3: keys 32 q4 + lane of a block
-    // in S^T, dims 32 q4 + lane in O^T; `half` selects its 32 token columns.
+    // in S^T, dims 32 q4 + lane in O^T; `tg` = (w - 2) / 4 selects its 16
+    // token columns.
     const int q4 = warp & 3;
-    const int half = (warp - 2) >> 2;
-    const int tb = 32 * half;                 // first token of this thread
+    const int tg = (warp - 2) >> 2;
+    const int tb = kTTok * tg;                // first token of this thread
     const uint32_t lane_base = tmem + ((uint32_t)(q4 * 32) << 16);
     const int kl = 32 * q4 + lane;            // this thread's key within a block
     const float NEG = -__int_as_float(0x7f800000);
     // transposed tree mask: warp w' = w - 2 ballots tokens 32 (w' & 1) + lane
-    // for tree keys j in [16 (w' >> 1), +16)
+    // for tree keys j in [8 (w' >> 1), +8)
     {
       const int wp = warp - 2;
       const int t = 32 * (wp & 1) + lane;
@@ -767,8 +776,8 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
         if (a.mask_words > 1) m1 = mr[1];
       }
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int j = 16 * (wp >> 1) + i;
+      for (int i = 0; i < 8; ++i) {
+        const int j = 8 * (wp >> 1) + i;
         const uint32_t bit = ((j < 32 ? m0 : m1) >> (j & 31)) & 1u;
         const uint32_t word = __ballot_sync(0xffffffffu, bit != 0u && j < a.L);
         if (lane == 0) sh->maskT[j][wp & 1] = word;
@@ -776,9 +785,12 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     }
     if (warp < 4) sh->ref[32 * (warp - 2) + lane] = NEG;
     soft_sync();
-    float psum[32];
+    // tokens of this thread that exist (t < L)
+    const uint32_t live = a.L >= tb + kTTok ? 0xffffu : (a.L <= tb ? 0u : ((1u << (a.L - tb)) - 1u));
+    const int mshift = tb & 31;               // this thread's tokens in a maskT word
+    float psum[kTTok];
 #pragma unroll
-    for (int u = 0; u < 32; ++u) psum[u] = 0.0f;
+    for (int u = 0; u < kTTok; ++u) psum[u] = 0.0f;
     const float4* ref4 = reinterpret_cast<const float4*>(sh->ref + tb);
     // P[token][key]: slab kl / 64, 16-byte chunk (kl % 64) / 8 swizzled by
     // token % 8 inside the token's 128-byte row, 2 bytes per key
@@ -787,42 +799,39 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     bool ok = true;
     for (int jj = 0; jj < nbl; ++jj) {
       const int b = jj & 1;
+      const int key0 = (j0 + jj) * kTB;
       ok = __all_sync(0xffffffffu,
                       ok && wait_bar(bar(S_FULL + b), (uint32_t)((jj >> 1) & 1), abort, a.status));
-      float x[32];
-      uint32_t vis = 0u;  // visibility of this thread's 32 tokens
+      float x[kTTok];                         // log2-domain scores (-inf: not visible)
+      bool exceed = false;
       if (ok) {
         ptx::tc_fence_after();
-        {
-          uint32_t rr[2][16];
-          ptx::tmem_ld16_nowait(lane_base + kTN * b + tb, rr[0]);
-          ptx::tmem_ld16_nowait(lane_base + kTN * b + tb + 16, rr[1]);
-          ptx::tmem_ld_wait();
-#pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            x[e] = __uint_as_float(rr[0][e]) * a.scale_log2;
-            x[16 + e] = __uint_as_float(rr[1][e]) * a.scale_log2;
-          }
-        }
+        uint32_t rr[kTTok];
+        ptx::tmem_ld16(lane_base + kTN * b + tb, rr);
         ptx::tc_fence_before();
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(bar(S_EMPTY + b));
-        const int key = (j0 + jj) * kTB + kl;
-        if (key < a.m) {
-          vis = a.L >= tb + 32 ? 0xffffffffu : (a.L <= tb ? 0u : ((1u << (a.L - tb)) - 1u));
-        } else if (key < a.m + a.L) {
-          vis = sh->maskT[key - a.m][half];
-        }
-      }
-      // lazy-rescale test over the CTA
-      bool exceed = false;
+        const int key = key0 + kl;
 #pragma unroll
-      for (int u4 = 0; u4 < 8; ++u4) {
-        const float4 r4 = ref4[u4];
-        exceed |= ((vis >> (4 * u4)) & 1u) && (x[4 * u4] > r4.x + kRescale);
-        exceed |= ((vis >> (4 * u4 + 1)) & 1u) && (x[4 * u4 + 1] > r4.y + kRescale);
-        exceed |= ((vis >> (4 * u4 + 2)) & 1u) && (x[4 * u4 + 2] > r4.z + kRescale);
-        exceed |= ((vis >> (4 * u4 + 3)) & 1u) && (x[4 * u4 + 3] > r4.w + kRescale);
+        for (int u = 0; u < kTTok; ++u) x[u] = __uint_as_float(rr[u]) * a.scale_log2;
+        if (!(key0 + kTB <= a.m && live == 0xffffu)) {  // not a block inside the prefix
+          uint32_t vis = 0u;
+          if (key < a.m) vis = live;
+          else if (key < a.m + a.L) vis = (sh->maskT[key - a.m][tb >> 5] >> mshift) & 0xffffu;
+#pragma unroll
+          for (int u = 0; u < kTTok; ++u)
+            if (!((vis >> u) & 1u)) x[u] = NEG;
+        }
+        // a visible score above its token's reference by more than 2^8 (the
+        // first visible score of a token always is: its reference is -inf)
+        float dmax = NEG;
+#pragma unroll
+        for (int u4 = 0; u4 < kTTok / 4; ++u4) {
+          const float4 r4 = ref4[u4];
+          dmax = fmaxf(dmax, fmaxf(fmaxf(x[4 * u4] - r4.x, x[4 * u4 + 1] - r4.y),
+                                   fmaxf(x[4 * u4 + 2] - r4.z, x[4 * u4 + 3] - r4.w)));
+        }
+        exceed = dmax > kRescale;  // -inf - -inf = NaN compares false
       }
       // P buffer b is free once the product of block jj - 2 is done; after
       // this wait at most the product of block jj - 1 is still running, so
@@ -831,14 +840,14 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
                                                  (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status));
       if (soft_any(ok && exceed)) {
         {
-          float bm[32];
+          float bm[kTTok];  // block maxima per token
 #pragma unroll
-          for (int u = 0; u < 32; ++u) bm[u] = ((vis >> u) & 1u) ? x[u] : NEG;
-          const float wmax = transpose_reduce<true>(bm, lane);  // token tb + lane, this quarter
-          reinterpret_cast<float*>(&sh->qmax[tb + lane])[q4] = wmax;
+          for (int u = 0; u < kTTok; ++u) bm[u] = x[u];
+          const float wmax = transpose_reduce<true>(bm, lane);  // token tb + lane % 16
+          if (lane < kTTok) reinterpret_cast<float*>(&sh->qmax[tb + lane])[q4] = wmax;
         }
         soft_sync();
-        if (q4 == 0) {  // one thread per token raises its reference
+        if (q4 == 0 && lane < kTTok) {  // one thread per token raises its reference
           const int t = tb + lane;
           const float4 qm = sh->qmax[t];
           const float m4 = fmaxf(fmaxf(qm.x, qm.y), fmaxf(qm.z, qm.w));
@@ -854,7 +863,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
         const float4* f4 = reinterpret_cast<const float4*>(sh->factor + tb);
         bool rescale = false;
 #pragma unroll
-        for (int u4 = 0; u4 < 8; ++u4) {
+        for (int u4 = 0; u4 < kTTok / 4; ++u4) {
           const float4 f = f4[u4];
           psum[4 * u4] *= f.x;
           psum[4 * u4 + 1] *= f.y;
@@ -869,30 +878,34 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
                           wait_bar(bar(O_DONE), (uint32_t)((jj - 1) & 1), abort, a.status));
           if (ok) {
             ptx::tc_fence_after();
+            uint32_t rr[kTTok];
+            const uint32_t ta = lane_base + 2 * kTN + tb;
+            ptx::tmem_ld16(ta, rr);
 #pragma unroll
-            for (int c = 0; c < 2; ++c) {
-              uint32_t rr[16];
-              const uint32_t ta = lane_base + 2 * kTN + tb + 16 * c;
-              ptx::tmem_ld16(ta, rr);
-#pragma unroll
-              for (int e = 0; e < 16; ++e)
-                rr[e] = __float_as_uint(__uint_as_float(rr[e]) * sh->factor[tb + 16 * c + e]);
-              ptx::tmem_st16(ta, rr);
+            for (int u4 = 0; u4 < kTTok / 4; ++u4) {
+              const float4 f = f4[u4];
+              rr[4 * u4] = __float_as_uint(__uint_as_float(rr[4 * u4]) * f.x);
+              rr[4 * u4 + 1] = __float_as_uint(__uint_as_float(rr[4 * u4 + 1]) * f.y);
+              rr[4 * u4 + 2] = __float_as_uint(__uint_as_float(rr[4 * u4 + 2]) * f.z);
+              rr[4 * u4 + 3] = __float_as_uint(__uint_as_float(rr[4 * u4 + 3]) * f.w);
             }
+            ptx::tmem_st16(ta, rr);
           }
         }
       }
       if (!ok) continue;
+      // P = 2^(x - ref) rounded to bf16 into P[token][this key]; every
+      // visible x is at most ref + 2^8 here; invisible -> 0
       uint8_t* prow = s_p + b * kTPBytes + p_off + tb * 128;
 #pragma unroll
-      for (int u4 = 0; u4 < 8; ++u4) {
+      for (int u4 = 0; u4 < kTTok / 4; ++u4) {
         const float4 r4 = ref4[u4];
         const float rv[4] = {r4.x, r4.y, r4.z, r4.w};
 #pragma unroll
         for (int e = 0; e < 4; e += 2) {
           const int u = 4 * u4 + e;
-          const float p0 = ((vis >> u) & 1u) ? ex2(x[u] - rv[e]) : 0.0f;
-          const float p1 = ((vis >> (u + 1)) & 1u) ? ex2(x[u + 1] - rv[e + 1]) : 0.0f;
+          const float p0 = x[u] == NEG ? 0.0f : ex2(x[u] - rv[e]);
+          const float p1 = x[u + 1] == NEG ? 0.0f : ex2(x[u + 1] - rv[e + 1]);
           const uint32_t pk = pack_bf16(p0, p1);
           psum[u] += __uint_as_float(pk << 16);
           psum[u + 1] += __uint_as_float(pk & 0xffff0000u);
@@ -908,8 +921,8 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
       if (lane == 0) ptx::mbar_arrive(bar(P_FULL + b));
     }
     // row sums: this warp's 32 keys, then the four lane quarters
-    const float wsum = transpose_reduce<false>(psum, lane);  // token tb + lane
-    reinterpret_cast<float*>(&sh->qsum[tb + lane])[q4] = wsum;
+    const float wsum = transpose_reduce<false>(psum, lane);  // token tb + lane % 16
+    if (lane < kTTok) reinterpret_cast<float*>(&sh->qsum[tb + lane])[q4] = wsum;
     const bool done =
         __all_sync(0xffffffffu, ok && nbl > 0 && wait_bar(bar(MMA_DONE), 0, abort, a.status));
     soft_sync();
@@ -922,21 +935,19 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     const int64_t pbase = ((int64_t)h * a.splits + sp) * 128;
     if (done && tb < a.L) {
       ptx::tc_fence_after();
-      uint32_t rr[2][16];
-      ptx::tmem_ld16_nowait(lane_base + 2 * kTN + tb, rr[0]);
-      ptx::tmem_ld16_nowait(lane_base + 2 * kTN + tb + 16, rr[1]);
-      ptx::tmem_ld_wait();
+      uint32_t rr[kTTok];
+      ptx::tmem_ld16(lane_base + 2 * kTN + tb, rr);
 #pragma unroll
-      for (int u = 0; u < 32; ++u) {
+      for (int u = 0; u < kTTok; ++u) {
         const int t = tb + u;
         if (t < a.L) {
-          const float v = __uint_as_float(rr[u >> 4][u & 15]);
+          const float v = __uint_as_float(rr[u]);
           if (a.fused) so[t * kHd + dim] = v;
           else a.part_o[(pbase + t) * kHd + dim] = v;
         }
       }
     }
-    if (q4 == 0) {
+    if (q4 == 0 && lane < kTTok) {
       const int t = tb + lane;
       const float4 qs = sh->qsum[t];
       float* pml = a.fused ? sml + 2 * t : a.part_ml + (pbase + t) * 2;
@@ -952,7 +963,8 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, 256);
   }
-  if (a.fused) cluster_merge(reinterpret_cast<const float*>(s_k), a, h, sp, warp, lane);
+  if (a.fused)
+    cluster_merge(reinterpret_cast<const float*>(s_k), a, h, sp, warp, lane, kTThreads / 32);
 }
 
 // out[h, r, :] = sum_s 2^(ref_s - M) O_s / sum_s 2^(ref_s - M) l_s, one warp
@@ -1085,7 +1097,7 @@ sense_status launch_attn_t(const uint16_t* q, const uint16_t* k_cache, const uin
   {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)heads, (unsigned)splits);
-    cfg.blockDim = dim3(kAttnThreads);
+    cfg.blockDim = dim3(kTThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];

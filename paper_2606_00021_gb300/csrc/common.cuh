@@ -42,6 +42,7 @@ enum KernelId {
   K_IVF_SCAN,
   K_CTX,
   K_TREE_ATTN,
+  K_RESCORE,
   K_COUNT
 };
 

@@ -85,6 +85,11 @@ sense_status launch_scan_tc(const uint16_t* keys, int64_t n, int d, const uint16
                             uint64_t* out, uint32_t* counts, int64_t pool_cap, uint32_t* status,
                             cudaStream_t s);
 sense_status launch_selftest_wait(long long limit, uint32_t* status, cudaStream_t s);
+// Exact scores of a shortlist of n_cand key indices per query (-1 = empty),
+// top k by (score desc, index asc).
+sense_status launch_rescore(const uint16_t* keys, int64_t n, int d, const uint16_t* queries, int q,
+                            const int32_t* cand, int n_cand, int k, float* out_scores,
+                            int32_t* out_idx, uint32_t* status, cudaStream_t s);
 sense_status launch_pad_queries(const uint16_t* src, int qg, int d, uint16_t* dst, int nq,
                                 cudaStream_t s);
 size_t scan_tc_smem_bytes(int d, int nq);

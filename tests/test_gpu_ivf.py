@@ -270,3 +270,66 @@ def test_projected_pipeline_and_recall(S):
     _, fi = S.sense_ivf_search(flat, qp, k, 24)
     exact = np.argsort(-(qp_h.astype(np.float64) @ kp_h.astype(np.float64).T), axis=1)[:, :k]
     assert I.recall_at_k(host(fi), exact) > 0.9
+
+
+# ---------------------------------------------------------------- shortlist re-scoring (Eq. 8 sim)
+
+@cuda
+@pytest.mark.parametrize("n,d,q,n_cand,k,empty", [
+    (50000, 512, 5, 300, 32, 0), (20000, 4096, 3, 1024, 64, 100), (9000, 256, 2, 1, 1, 0),
+    (9000, 256, 4, 40, 40, 30), (70000, 8192, 1, 256, 32, 0),
+])
+def test_rescore_matches_oracle(S, n, d, q, n_cand, k, empty):
+    """Exact re-scoring of a shortlist: scores within 2e-3 of the oracle's
+    fp64 inner products, the top-k rule of the exact search restricted to
+    the candidates, and empty slots (-1) skipped and padded with -inf / -1."""
+    from tests.parity import check_topk
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(n + n_cand)
+    keys = synth.clustered_unit_keys(n, d, 64, seed=n % 97, device=dev)
+    qs, _ = synth.noisy_queries(keys, q, seed=5)
+    ds = S.sense_datastore_build(keys, synth.spans_uniform(n, 2, 50, seed=1, device=dev))
+    cand = np.stack([rng.permutation(n)[:n_cand] for _ in range(q)]).astype(np.int32)
+    for qi in range(q):
+        cand[qi, rng.permutation(n_cand)[:empty]] = -1
+    sc, ix = S.sense_rescore_topk(ds, qs, _dev(cand), k)
+    torch.cuda.synchronize()
+    assert S.sense_device_status(clear=True) == 0
+    ws, wi = I.rescore_topk(bits(keys), bits(qs), cand, k)
+    for qi in range(q):
+        valid = int((wi[qi] >= 0).sum())
+        assert host(ix[qi])[valid:].tolist() == [-1] * (k - valid)
+        assert np.all(host(sc[qi])[valid:] == -np.inf)
+        row = np.full(n, -np.inf)
+        c = cand[qi][cand[qi] >= 0]
+        row[c] = I.scores(bits(keys)[c], bits(qs[qi:qi + 1]))[0]
+        check_topk(host(sc[qi])[:valid], host(ix[qi])[:valid], row, valid)
+
+
+@cuda
+def test_rescore_lattice_bit_exact_and_bad_index(S):
+    """Lattice keys and queries: every score is exact in fp32, so scores,
+    order and ties (lower key index first) must equal the oracle bit for
+    bit.  An index outside [0, n) is skipped and reported."""
+    dev = torch.device("cuda")
+    n, d, q, n_cand, k = 6000, 512, 3, 500, 100
+    keys = synth.lattice_rows(n, d, seed=7, device=dev)
+    qs = synth.lattice_rows(q, d, seed=8, device=dev)
+    ds = S.sense_datastore_build(keys, synth.spans_uniform(n, 2, 50, seed=1, device=dev))
+    rng = np.random.default_rng(3)
+    cand = np.stack([rng.permutation(n)[:n_cand] for _ in range(q)]).astype(np.int32)
+    sc, ix = S.sense_rescore_topk(ds, qs, _dev(cand), k)
+    torch.cuda.synchronize()
+    assert S.sense_device_status(clear=True) == 0
+    ws, wi = I.rescore_topk(bits(keys), bits(qs), cand, k)
+    np.testing.assert_array_equal(host(ix), wi)
+    np.testing.assert_array_equal(host(sc).astype(np.float64), ws)
+    bad = cand.copy()
+    bad[0, 7] = n + 5
+    bad[1, 0] = 1 << 30
+    sc2, ix2 = S.sense_rescore_topk(ds, qs, _dev(bad), k)
+    torch.cuda.synchronize()
+    assert S.sense_device_status(clear=True) == S.DEVST_BAD_INDEX
+    bad[bad >= n] = -1
+    ws2, wi2 = I.rescore_topk(bits(keys), bits(qs), bad, k)
+    np.testing.assert_array_equal(host(ix2), wi2)

@@ -285,3 +285,44 @@ def test_ivf_pq_exact_codebooks_reduce_to_flat():
 
 def test_recall_at_k():
     assert I.recall_at_k(np.array([[1, 2, 3]]), np.array([[3, 4, 1]])) == pytest.approx(2 / 3)
+
+
+# ---------------------------------------------------------------- shortlist re-scoring (Eq. 8 sim)
+
+def test_rescore_topk_exact_on_lattice_and_ordering():
+    """Lattice keys make every score an exact short binary fraction: the
+    re-scored top k must equal brute force with rational arithmetic, ties
+    broken by the lower key index, empty slots (-1) skipped and padded."""
+    from fractions import Fraction as F
+    rng = np.random.default_rng(21)
+    n, d = 40, 16
+    kv = rng.integers(-3, 4, (n, d)) / 64.0
+    qv = rng.integers(-3, 4, (3, d)) / 64.0
+    kb = _bits(torch.tensor(kv, dtype=torch.float32).to(torch.bfloat16))
+    qb = _bits(torch.tensor(qv, dtype=torch.float32).to(torch.bfloat16))
+    cand = np.array([rng.permutation(n)[:12], np.r_[rng.permutation(n)[:5], [-1] * 7],
+                     np.r_[[-1] * 10, [3, 17]]], dtype=np.int32)
+    for k in (1, 4, 8):
+        s, i = I.rescore_topk(kb, qb, cand, k)
+        for qi in range(3):
+            c = [int(x) for x in cand[qi] if x >= 0]
+            ex = sorted(((sum(F(float(qv[qi, j])) * F(float(kv[r, j])) for j in range(d)), r)
+                         for r in c), key=lambda t: (-t[0], t[1]))[:k]
+            assert [r for _, r in ex] == i[qi, :len(ex)].tolist()
+            assert [float(v) for v, _ in ex] == s[qi, :len(ex)].tolist()
+            assert np.all(i[qi, len(ex):] == -1) and np.all(s[qi, len(ex):] == -np.inf)
+
+
+def test_rescore_of_every_key_is_exhaustive_search():
+    # a shortlist holding every key reduces to the exact top-k of the store
+    rng = np.random.default_rng(22)
+    x = synth.gaussian_rows_f32(300, 32, seed=22).to(torch.bfloat16)
+    q = synth.gaussian_rows_f32(2, 32, seed=23).to(torch.bfloat16)
+    kb, qb = _bits(x), _bits(q)
+    cand = np.stack([rng.permutation(300) for _ in range(2)]).astype(np.int32)
+    s, i = I.rescore_topk(kb, qb, cand, 25)
+    full = O.bf16_bits_to_f64(qb) @ O.bf16_bits_to_f64(kb).T
+    for qi in range(2):
+        o = np.lexsort((np.arange(300), -full[qi]))[:25]
+        assert i[qi].tolist() == o.tolist()
+        np.testing.assert_allclose(s[qi], full[qi, o], rtol=0, atol=1e-12)
