@@ -509,25 +509,28 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant
 //   O^T += V^T P^T (M = 128 dims, N = 64 tokens, K = 128 keys)
 // which halves the tensor time per key and, with 128-key blocks, halves the
 // exponentials per key (no padding rows).  In TMEM a softmax thread now owns
-// one key (a lane) and 32 token columns, so the row statistics need cross-
-// thread reductions; they are only needed when the lazy-rescale test fires:
-//  - every thread keeps the per-token reference maxima ref_t of its 32
-//    tokens (the same values in every thread of a token half);
+// one key (a lane) and 16 token columns; 16 softmax warps cover the 128
+// keys x 64 tokens of a block.  The row statistics need cross-thread
+// reductions, but only when the lazy-rescale test fires:
+//  - the four warps that share 16 tokens (one per TMEM lane quarter) keep
+//    the tokens' reference maxima in shared memory;
 //  - per block, each thread tests whether any visible score exceeds its
 //    token's reference by more than 2^8 (log2 domain); one barrier-reduction
-//    over the 256 softmax threads decides for the CTA;
+//    over the four warps decides for them;
 //  - only then (always on the first block) the block maxima per token are
-//    reduced (a 31-shuffle transposing reduction per warp, the four lane
-//    quarters through shared memory), the references raised, and the
-//    thread's row sums and its O^T columns rescaled;
+//    reduced (a transposing shuffle reduction per warp, the four lane
+//    quarters through shared memory), the references raised, and the row
+//    sums and O^T columns of those tokens rescaled;
 //  - P = 2^(s - ref_t) is rounded to bf16 and written to P[token][key] in the
 //    swizzled K-major layout the product reads; each thread adds its rounded
 //    values into per-token partial row sums, reduced across keys once at
 //    the end.
-// K and V^T tiles have separate rings (3 and 2 stages of 32 KB), so keys can
-// be loaded ahead while the products of earlier blocks still hold their
-// V^T tiles.  The split partials and their merge are those of
-// tree_attn_kernel.
+// The MMA thread issues the scores of a block as soon as its K tile and one
+// of three S^T buffers are free, ahead of the value products, so the softmax
+// warps never wait behind a product.  K and V^T tiles have separate rings
+// (3 and 2 stages of 32 KB), so keys can be loaded ahead while the products
+// of earlier blocks still hold their V^T tiles.  The split partials and
+// their merge are those of tree_attn_kernel.
 constexpr int kTB = 128;                  // keys per block
 constexpr int kTN = 64;                   // token columns (N of both products)
 constexpr int kTSoftWarps = 16;           // four per TMEM lane quarter
@@ -541,7 +544,9 @@ constexpr int kTKBytes = 2 * kTSlab;      // K tile: 128 keys x 128 dims
 constexpr int kTVBytes = 2 * kTSlab;      // V^T tile: 128 dims x 128 keys
 constexpr int kTKStages = 3;
 constexpr int kTVStages = 2;
-constexpr int kTNBars = 1 + 2 * kTKStages + 2 * kTVStages + 8 + 2;
+constexpr int kTSBufs = 3;                // S^T buffers in TMEM
+constexpr int kTOCol = kTSBufs * kTN;     // TMEM column of O^T
+constexpr int kTNBars = 1 + 2 * kTKStages + 2 * kTVStages + 2 * kTSBufs + 4 + 2;
 
 struct AttnTShared {
   uint32_t tmem_base;
@@ -558,22 +563,28 @@ size_t attn_t_smem_bytes() {
          kTNBars * 8 + 16 + sizeof(AttnTShared);
 }
 
-// Barrier over the softmax threads that also returns whether any of them
-// passed `p` (bar.red.or).
-__device__ __forceinline__ bool soft_any(bool p) {
+__device__ __forceinline__ void soft_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kTSoftWarps * 32) : "memory");
+}
+
+// The four warps of token group `tg` (one per lane quarter) share the
+// reference maxima of their 16 tokens: a barrier over them (ids 3..6) that
+// also returns whether any of their threads passed `p`, and a plain one
+// (ids 7..10).
+__device__ __forceinline__ bool group_any(int tg, bool p) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred pi, po;\n\t"
       "setp.ne.u32 pi, %1, 0;\n\t"
-      "bar.red.or.pred po, 2, %2, pi;\n\t"
+      "bar.red.or.pred po, %2, 128, pi;\n\t"
       "selp.u32 %0, 1, 0, po;\n\t}"
       : "=r"(r)
-      : "r"((uint32_t)p), "n"(kTSoftWarps * 32)
+      : "r"((uint32_t)p), "r"(3 + tg)
       : "memory");
   return r != 0;
 }
-__device__ __forceinline__ void soft_sync() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kTSoftWarps * 32) : "memory");
+__device__ __forceinline__ void group_sync(int tg) {
+  asm volatile("bar.sync %0, 128;" ::"r"(7 + tg) : "memory");
 }
 
 // Lane i (and lane i ^ 16) ends up with op over the warp's 32 lanes of
@@ -610,8 +621,8 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
   uint8_t* s_v = s_k + kTKStages * kTKBytes;    // V^T ring (A of O^T)
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_v + kTVStages * kTVBytes);
   const int Q_FULL = 0, K_FULL = 1, K_EMPTY = 1 + kTKStages, V_FULL = 1 + 2 * kTKStages,
-            V_EMPTY = V_FULL + kTVStages, S_FULL = V_EMPTY + kTVStages, S_EMPTY = S_FULL + 2,
-            P_FULL = S_EMPTY + 2, P_EMPTY = P_FULL + 2, O_DONE = P_EMPTY + 2,
+            V_EMPTY = V_FULL + kTVStages, S_FULL = V_EMPTY + kTVStages, S_EMPTY = S_FULL + kTSBufs,
+            P_FULL = S_EMPTY + kTSBufs, P_EMPTY = P_FULL + 2, O_DONE = P_EMPTY + 2,
             MMA_DONE = O_DONE + 1;
   AttnTShared* sh = reinterpret_cast<AttnTShared*>(
       (reinterpret_cast<uintptr_t>(bars + kTNBars) + 15) & ~static_cast<uintptr_t>(15));
@@ -633,9 +644,11 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
       ptx::mbar_init(bar(V_FULL + s), 1);
       ptx::mbar_init(bar(V_EMPTY + s), 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kTSBufs; ++b) {
       ptx::mbar_init(bar(S_FULL + b), 1);
       ptx::mbar_init(bar(S_EMPTY + b), kTSoftWarps);
+    }
+    for (int b = 0; b < 2; ++b) {
       ptx::mbar_init(bar(P_FULL + b), kTSoftWarps);
       ptx::mbar_init(bar(P_EMPTY + b), 1);
     }
@@ -651,7 +664,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
-  const uint32_t tmem = sh->tmem_base;  // S^T buffers at columns 0 and kTN, O^T at 2 kTN
+  const uint32_t tmem = sh->tmem_base;  // S^T buffers at columns kTN b (b < 3), O^T at kTOCol
 
   if (warp == 0 && lane == 0 && nbl > 0) {
     // ------------------------------------------------ TMA producer
@@ -707,50 +720,64 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     }
   } else if (warp == 1 && lane == 0 && nbl > 0) {
     // ------------------------------------------------ MMA issuer
+    // Score products run ahead of the value products as far as the three
+    // S^T buffers allow (a block's scores are released as soon as the
+    // softmax has read them), so the softmax never waits behind a value
+    // product; the barrier tests do not block (test_wait).
     const uint32_t idesc = ptx::idesc_bf16_f32(128, kTN);
     const uint32_t q_addr = ptx::smem_u32(s_q), p_addr = ptx::smem_u32(s_p);
     bool ok = wait_bar(bar(Q_FULL), 0, abort, a.status);
-    auto pv = [&](int i) -> bool {
-      const int pb = i & 1, sv = i % kTVStages;
-      if (!wait_bar(bar(P_FULL + pb), (uint32_t)((i >> 1) & 1), abort, a.status) ||
-          !wait_bar(bar(V_FULL + sv), (uint32_t)((i / kTVStages) & 1), abort, a.status))
-        return false;
-      ptx::tc_fence_after();
-      const uint32_t vt = ptx::smem_u32(s_v + sv * kTVBytes);
-      const uint32_t pa = p_addr + pb * kTPBytes;
+    ptx::tc_fence_after();
+    int js = 0, jp = 0;
+    long long t0 = clock64();
+    while (ok && jp < nbl) {
+      bool moved = false;
+      if (js < nbl && ptx::mbar_test_wait(bar(K_FULL + js % kTKStages), (uint32_t)((js / kTKStages) & 1)) &&
+          ptx::mbar_test_wait(bar(S_EMPTY + js % kTSBufs), (uint32_t)(((js / kTSBufs) & 1) ^ 1))) {
+        ptx::tc_fence_after();
+        const uint32_t kt = ptx::smem_u32(s_k + (js % kTKStages) * kTKBytes);
+        const uint32_t sd = tmem + kTN * (js % kTSBufs);
 #pragma unroll
-      for (int ks = 0; ks < 2; ++ks)
+        for (int kc = 0; kc < 2; ++kc)
 #pragma unroll
-        for (int t = 0; t < 4; ++t)
-          ptx::mma_bf16(tmem + 2 * kTN, ptx::desc_sw128(vt + ks * kTSlab + t * 32),
-                        ptx::desc_sw128(pa + ks * kTSlabQ + t * 32), idesc,
-                        (i > 0 || ks > 0 || t > 0) ? 1u : 0u);
-      ptx::mma_commit(bar(O_DONE));
-      ptx::mma_commit(bar(P_EMPTY + pb));
-      ptx::mma_commit(bar(V_EMPTY + sv));
-      return true;
-    };
-    for (int jj = 0; jj < nbl && ok; ++jj) {
-      const int s = jj % kTKStages, b = jj & 1;
-      if (!wait_bar(bar(K_FULL + s), (uint32_t)((jj / kTKStages) & 1), abort, a.status) ||
-          !wait_bar(bar(S_EMPTY + b), (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status)) {
-        ok = false;
-        break;
+          for (int t = 0; t < 4; ++t)
+            ptx::mma_bf16(sd, ptx::desc_sw128(kt + kc * kTSlab + t * 32),
+                          ptx::desc_sw128(q_addr + kc * kTSlabQ + t * 32), idesc,
+                          (kc > 0 || t > 0) ? 1u : 0u);
+        ptx::mma_commit(bar(S_FULL + js % kTSBufs));
+        ptx::mma_commit(bar(K_EMPTY + js % kTKStages));
+        ++js;
+        moved = true;
       }
-      ptx::tc_fence_after();
-      const uint32_t kt = ptx::smem_u32(s_k + s * kTKBytes);
+      if (jp < js && ptx::mbar_test_wait(bar(P_FULL + (jp & 1)), (uint32_t)((jp >> 1) & 1)) &&
+          ptx::mbar_test_wait(bar(V_FULL + jp % kTVStages), (uint32_t)((jp / kTVStages) & 1))) {
+        ptx::tc_fence_after();
+        const int pb = jp & 1, sv = jp % kTVStages;
+        const uint32_t vt = ptx::smem_u32(s_v + sv * kTVBytes);
+        const uint32_t pa = p_addr + pb * kTPBytes;
 #pragma unroll
-      for (int kc = 0; kc < 2; ++kc)
+        for (int ks = 0; ks < 2; ++ks)
 #pragma unroll
-        for (int t = 0; t < 4; ++t)
-          ptx::mma_bf16(tmem + kTN * b, ptx::desc_sw128(kt + kc * kTSlab + t * 32),
-                        ptx::desc_sw128(q_addr + kc * kTSlabQ + t * 32), idesc,
-                        (kc > 0 || t > 0) ? 1u : 0u);
-      ptx::mma_commit(bar(S_FULL + b));
-      ptx::mma_commit(bar(K_EMPTY + s));
-      if (jj > 0 && !pv(jj - 1)) ok = false;
+          for (int t = 0; t < 4; ++t)
+            ptx::mma_bf16(tmem + kTOCol, ptx::desc_sw128(vt + ks * kTSlab + t * 32),
+                          ptx::desc_sw128(pa + ks * kTSlabQ + t * 32), idesc,
+                          (jp > 0 || ks > 0 || t > 0) ? 1u : 0u);
+        ptx::mma_commit(bar(O_DONE));
+        ptx::mma_commit(bar(P_EMPTY + pb));
+        ptx::mma_commit(bar(V_EMPTY + sv));
+        ++jp;
+        moved = true;
+      }
+      if (moved) {
+        t0 = clock64();
+      } else if (*abort) {
+        ok = false;
+      } else if (clock64() - t0 > kWaitCycles) {
+        *abort = 1;
+        raise_status(a.status, SENSE_DEVST_TIMEOUT);
+        ok = false;
+      }
     }
-    if (ok) pv(nbl - 1);
     ptx::mma_commit(bar(MMA_DONE));
     drain_bar(bar(MMA_DONE), 0);
   } else if (warp >= 2) {
@@ -784,7 +811,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
       }
     }
     if (warp < 4) sh->ref[32 * (warp - 2) + lane] = NEG;
-    soft_sync();
+    soft_sync();  // every warp's maskT words and the references are in place
     // tokens of this thread that exist (t < L)
     const uint32_t live = a.L >= tb + kTTok ? 0xffffu : (a.L <= tb ? 0u : ((1u << (a.L - tb)) - 1u));
     const int mshift = tb & 31;               // this thread's tokens in a maskT word
@@ -798,19 +825,20 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     const uint32_t p_off = (uint32_t)((kl >> 6) * kTSlabQ + ((kl & 7) << 1));
     bool ok = true;
     for (int jj = 0; jj < nbl; ++jj) {
-      const int b = jj & 1;
+      const int b = jj & 1;                     // P buffer
+      const int sb = jj % kTSBufs;              // S^T buffer
       const int key0 = (j0 + jj) * kTB;
-      ok = __all_sync(0xffffffffu,
-                      ok && wait_bar(bar(S_FULL + b), (uint32_t)((jj >> 1) & 1), abort, a.status));
+      ok = __all_sync(0xffffffffu, ok && wait_bar(bar(S_FULL + sb), (uint32_t)((jj / kTSBufs) & 1),
+                                                 abort, a.status));
       float x[kTTok];                         // log2-domain scores (-inf: not visible)
       bool exceed = false;
       if (ok) {
         ptx::tc_fence_after();
         uint32_t rr[kTTok];
-        ptx::tmem_ld16(lane_base + kTN * b + tb, rr);
+        ptx::tmem_ld16(lane_base + kTN * sb + tb, rr);
         ptx::tc_fence_before();
         __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(bar(S_EMPTY + b));
+        if (lane == 0) ptx::mbar_arrive(bar(S_EMPTY + sb));
         const int key = key0 + kl;
 #pragma unroll
         for (int u = 0; u < kTTok; ++u) x[u] = __uint_as_float(rr[u]) * a.scale_log2;
@@ -838,7 +866,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
       // the O_DONE phase tested below is that product's
       ok = __all_sync(0xffffffffu, ok && wait_bar(bar(P_EMPTY + b),
                                                  (uint32_t)(((jj >> 1) & 1) ^ 1), abort, a.status));
-      if (soft_any(ok && exceed)) {
+      if (group_any(tg, ok && exceed)) {
         {
           float bm[kTTok];  // block maxima per token
 #pragma unroll
@@ -846,7 +874,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
           const float wmax = transpose_reduce<true>(bm, lane);  // token tb + lane % 16
           if (lane < kTTok) reinterpret_cast<float*>(&sh->qmax[tb + lane])[q4] = wmax;
         }
-        soft_sync();
+        group_sync(tg);
         if (q4 == 0 && lane < kTTok) {  // one thread per token raises its reference
           const int t = tb + lane;
           const float4 qm = sh->qmax[t];
@@ -859,7 +887,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
           }
           sh->factor[t] = f;
         }
-        soft_sync();
+        group_sync(tg);
         const float4* f4 = reinterpret_cast<const float4*>(sh->factor + tb);
         bool rescale = false;
 #pragma unroll
@@ -879,7 +907,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
           if (ok) {
             ptx::tc_fence_after();
             uint32_t rr[kTTok];
-            const uint32_t ta = lane_base + 2 * kTN + tb;
+            const uint32_t ta = lane_base + kTOCol + tb;
             ptx::tmem_ld16(ta, rr);
 #pragma unroll
             for (int u4 = 0; u4 < kTTok / 4; ++u4) {
@@ -925,7 +953,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     if (lane < kTTok) reinterpret_cast<float*>(&sh->qsum[tb + lane])[q4] = wsum;
     const bool done =
         __all_sync(0xffffffffu, ok && nbl > 0 && wait_bar(bar(MMA_DONE), 0, abort, a.status));
-    soft_sync();
+    group_sync(tg);
     // partial output of this split in row layout [token][dim]: into global
     // memory, or (fused) into this CTA's shared memory where the K ring was
     // (every load has landed, every product is done once MMA_DONE completed)
@@ -936,7 +964,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     if (done && tb < a.L) {
       ptx::tc_fence_after();
       uint32_t rr[kTTok];
-      ptx::tmem_ld16(lane_base + 2 * kTN + tb, rr);
+      ptx::tmem_ld16(lane_base + kTOCol + tb, rr);
 #pragma unroll
       for (int u = 0; u < kTTok; ++u) {
         const int t = tb + u;
