@@ -247,18 +247,26 @@ class Pipeline:
 
     def step(self, query, gate_in, before_gate=None):
         S, cfg = self.S, self.cfg
-        self.retrieve(query)
         dyn = getattr(self, "dyn", None)
-        if dyn is None:
-            S.sense_gather_drafts(self.ds, self.idx, out=self.drafts)
-        else:
-            S.sense_ctx_search(dyn["ctx"], query, dyn["kd"], dyn["delta"], outs=dyn["outs"],
-                               workspace=dyn["ws"])
-            S.sense_hybrid_drafts(self.ds, self.scores, self.idx, dyn["outs"], dyn["anchor"],
-                                  cfg["k"], True, out=self.drafts)
         ver = getattr(self, "verify", None)
-        S.sense_build_tree(self.drafts, node_cap=cfg["cap"], mask_bits=ver is not None,
-                           outs=self.tree)
+        if self.ann is None and dyn is None:
+            # exact retrieval, gather and trie in one call (one kernel per
+            # query after the scan on the single-pass path)
+            outs = self.tree
+            outs["scores"], outs["idx"], outs["spans"] = self.scores, self.idx, self.drafts
+            S.sense_draft(self.ds, query, cfg["k"], node_cap=cfg["cap"], mask_bits=ver is not None,
+                          outs=outs, workspace=self.ws)
+        else:
+            self.retrieve(query)
+            if dyn is None:
+                S.sense_gather_drafts(self.ds, self.idx, out=self.drafts)
+            else:
+                S.sense_ctx_search(dyn["ctx"], query, dyn["kd"], dyn["delta"], outs=dyn["outs"],
+                                   workspace=dyn["ws"])
+                S.sense_hybrid_drafts(self.ds, self.scores, self.idx, dyn["outs"], dyn["anchor"],
+                                      cfg["k"], True, out=self.drafts)
+            S.sense_build_tree(self.drafts, node_cap=cfg["cap"], mask_bits=ver is not None,
+                               outs=self.tree)
         if ver is not None:
             S.sense_tree_attention(ver["q"], ver["k"], ver["vt"], ver["prefix"],
                                    self.tree["mask_bits"][0], ver["scale"], out=ver["out"],
@@ -275,7 +283,7 @@ class Pipeline:
 
 
 DRAFT_KERNELS = ("scan_gemv", "scan_tc", "threshold", "merge", "pad_queries", "gather", "tree",
-                 "project", "ivf_coarse", "ivf_scan", "ctx", "rescore")
+                 "project", "ivf_coarse", "ivf_scan", "ctx", "rescore", "draft")
 
 
 def draft_kernel_rate(prof, q, tokens_per_query, steps):
@@ -610,9 +618,17 @@ def main():
                     "delta": args.delta, "n_keep": cfg["k"], "anchor": "previous step's x~",
                     "update": "accepted path appended every step (device-side count)"}
 
+    # warm-up, profiled: the kernel family with the largest share is the one
+    # the timed region brackets with CUDA events (the roofline kernel); the
+    # other launches run unbracketed there, and their times come from an
+    # eager pass of the same steps after the timed region
+    S.sense_profile_enable(True)
     for it in range(args.warmup):
         pipe.step(queries[it % nq], gate_sets[it % n_sets])
     torch.cuda.synchronize()
+    warm = {name: S.sense_profile_query(name) for name in S.sense_profile_names()}
+    live_family = max(warm, key=lambda name: warm[name][0])
+    S.sense_profile_enable(False)
     if S.sense_device_status(clear=True) != 0:
         raise RuntimeError("device status bits set after warm-up")
     graph, graph_error = None, None
@@ -662,6 +678,7 @@ def main():
                       f"eager pass of the same {args.steps} steps")
     else:
         S.sense_profile_enable(True)
+        S.sense_profile_filter([live_family])
         e0.record(stream)
         for it in range(args.steps):
             pipe.step(queries[it % nq], gate_sets[it % n_sets])
@@ -671,7 +688,18 @@ def main():
             dist.barrier()
         clk = clocks.stop()
         ms = e0.elapsed_time(e1)
+        live = S.sense_profile_query(live_family)
+        # every family, from an eager pass of the same steps
+        S.sense_profile_enable(True)
+        for it in range(args.steps):
+            pipe.step(queries[it % nq], gate_sets[it % n_sets])
+        torch.cuda.synchronize()
+        graph_note = (f"timed region: {args.steps} eager steps with CUDA events around the "
+                      f"{live_family} launches only; the other kernels' times (kernel_ms) come "
+                      f"from an eager pass of the same {args.steps} steps after it")
     prof = {name: S.sense_profile_query(name) for name in S.sense_profile_names()}
+    if graph is None:
+        prof[live_family] = live
     S.sense_profile_enable(False)
     ms = max_over_ranks(ms, dist, dev)
     launches = sum(v[1] for v in prof.values())

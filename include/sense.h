@@ -485,6 +485,27 @@ sense_status sense_build_tree(const int32_t* spans, int32_t q, int32_t k, int32_
                               int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
                               int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream);
 
+/*
+ * The drafting step of one query batch in one call (the paper has no
+ * separate counterpart: it is Sec. 3.2.2 Eq. 7 retrieval, the D_ret span
+ * gather and the Sec. 3.2.3 Eq. 9 loose trie, composed): the same results,
+ * bit for bit, as sense_retrieve_topk, then sense_gather_drafts without an
+ * anchor (n_keep = k), then sense_build_tree on the gathered spans.
+ * Arguments are those calls' arguments; out_spans is int32 [q, k, m] with
+ * m = the datastore's span length, 16-byte aligned; the workspace is
+ * sense_retrieve_workspace_bytes(ds, q, k) bytes, 256-byte aligned.  For
+ * the single-pass retrieval (q <= 4, k <= 128, the exact scan's fused
+ * lists) the merge, the gather and the trie run as one kernel per query;
+ * otherwise the calls' own launches run in order.  Errors and device status
+ * are those of the three calls.
+ */
+sense_status sense_draft(const sense_datastore* ds, const uint16_t* queries, int32_t q, int32_t k,
+                         void* workspace, size_t workspace_bytes, int32_t node_cap, uint32_t flags,
+                         float* out_scores, int32_t* out_idx, int32_t* out_spans,
+                         int32_t* out_num_nodes, int32_t* out_tokens, int32_t* out_parent,
+                         int32_t* out_depth, int32_t* out_gamma, uint32_t* out_mask_bits,
+                         sense_stream_t stream);
+
 /* ---------------------------------------------------------------------- */
 /* Tree attention mask over a static KV cache                               */
 /* ---------------------------------------------------------------------- */
@@ -628,6 +649,14 @@ sense_status sense_selftest_timeout(sense_stream_t stream, int64_t limit_cycles)
  * summed device time in milliseconds and the number of launches.
  */
 sense_status sense_profile_enable(int32_t on);
+/*
+ * Restricts the bracketing to the comma-separated kernel families in
+ * `names` (NULL or "" = every family) until the next sense_profile_enable,
+ * which selects every family again.  Each bracketed launch adds two event
+ * records to its stream; filtering keeps them off the launches that are not
+ * being measured.  SENSE_ERR_INVALID_ARG for an unknown family name.
+ */
+sense_status sense_profile_filter(const char* names);
 int32_t sense_profile_count(void);
 const char* sense_profile_name(int32_t i);
 sense_status sense_profile_query(const char* name, double* total_ms, int64_t* launches);

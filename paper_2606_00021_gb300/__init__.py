@@ -276,6 +276,44 @@ def sense_build_tree(spans: torch.Tensor, node_cap: int = 0, mask_bits: bool = F
     return o
 
 
+def sense_draft(ds: Datastore, queries: torch.Tensor, k: int, node_cap: int = 0,
+                mask_bits: bool = False, outs: dict | None = None, workspace=None, stream=None):
+    """Retrieval, span gather and loose trie of one query batch in one call;
+    the results of sense_retrieve_topk, sense_gather_drafts (no anchor) and
+    sense_build_tree.  Returns a dict: scores, idx, spans and the tree
+    arrays (num_nodes, tokens, parent, depth, gamma[, mask_bits], cap)."""
+    _need(queries, "queries", torch.bfloat16, 2)
+    q = queries.shape[0]
+    if queries.shape[1] != ds.d:
+        raise ValueError("queries must have d columns")
+    m = ds.m
+    cap = node_cap if node_cap > 0 else k * m
+    dev = queries.device
+    o = outs if outs is not None else {}
+    o.setdefault("scores", torch.empty(q, k, dtype=torch.float32, device=dev))
+    o.setdefault("idx", _i32((q, k), dev))
+    o.setdefault("spans", _i32((q, k, m), dev))
+    o.setdefault("num_nodes", _i32((q,), dev))
+    o.setdefault("tokens", _i32((q, cap), dev))
+    o.setdefault("parent", _i32((q, cap), dev))
+    o.setdefault("depth", _i32((q, cap), dev))
+    o.setdefault("gamma", _i32((q, k, m), dev))
+    if mask_bits:
+        o.setdefault("mask_bits", torch.empty(q, cap, (cap + 31) // 32, dtype=torch.int32,
+                                              device=dev))
+    if workspace is None:
+        workspace = alloc_workspace(sense_retrieve_workspace_bytes(ds, q, k), dev)
+    _check(lib().sense_draft(C.c_void_p(ds.handle), queries.data_ptr(), q, k,
+                             workspace.data_ptr(), workspace.numel(), node_cap,
+                             1 if mask_bits else 0, o["scores"].data_ptr(), o["idx"].data_ptr(),
+                             o["spans"].data_ptr(), o["num_nodes"].data_ptr(),
+                             o["tokens"].data_ptr(), o["parent"].data_ptr(),
+                             o["depth"].data_ptr(), o["gamma"].data_ptr(),
+                             _ptr(o.get("mask_bits")), C.c_void_p(_stream(stream))))
+    o["cap"] = cap
+    return o
+
+
 def sense_tree_mask_full(tree: dict, prefix_len: torch.Tensor, cache_len: int,
                          out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """Additive static-KV attention mask [q, cap, cache_len] f32 of a tree
@@ -626,6 +664,13 @@ def sense_selftest_timeout(limit_cycles: int = 200_000_000, stream=None) -> int:
 
 def sense_profile_enable(on: bool = True):
     _check(lib().sense_profile_enable(1 if on else 0))
+
+
+def sense_profile_filter(names=None):
+    """Bracket only these kernel families (iterable of names; None = all)
+    while profiling is on; reset by sense_profile_enable."""
+    arg = None if names is None else ",".join(names).encode()
+    _check(lib().sense_profile_filter(arg))
 
 
 def sense_profile_query(name: str):

@@ -33,6 +33,8 @@ SIGNATURES = {
     "sense_gather_drafts": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_i32, c_u32, c_p, c_p]),
     "sense_build_tree": (c_i32, [c_p, c_i32, c_i32, c_i32, c_i32, c_u32, c_p, c_p, c_p, c_p,
                                  c_p, c_p, c_p]),
+    "sense_draft": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_size, c_i32, c_u32, c_p, c_p, c_p, c_p,
+                            c_p, c_p, c_p, c_p, c_p, c_p]),
     "sense_tree_mask_full": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_i32, c_p, c_p]),
     "sense_project": (c_i32, [c_p, c_i64, c_i32, c_p, c_i32, c_p, c_u32, c_p, c_p]),
     "sense_kmeans_workspace_bytes": (c_size, [c_i64, c_i32, c_i32]),
@@ -64,6 +66,7 @@ SIGNATURES = {
                                 c_p, c_p, c_i32, C.POINTER(GateParams), c_p, c_p, c_p, c_p, c_p,
                                 c_p, c_p, c_p, c_p, c_size, c_p]),
     "sense_selftest_timeout": (c_i32, [c_p, c_i64]),
+    "sense_profile_filter": (c_i32, [C.c_char_p]),
     "sense_profile_enable": (c_i32, [c_i32]),
     "sense_profile_count": (c_i32, []),
     "sense_profile_name": (C.c_char_p, [c_i32]),

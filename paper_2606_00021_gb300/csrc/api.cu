@@ -26,13 +26,14 @@ struct ProfRec {
   cudaEvent_t a, b;
 };
 bool g_prof_on = false;
+bool g_prof_family[K_COUNT];  // families bracketed while profiling is on
 std::vector<ProfRec> g_prof;
 std::vector<cudaEvent_t> g_ev_pool;
 const char* const kKernelNames[K_COUNT] = {
     "normalize", "scan_gemv", "scan_tc", "threshold", "merge",
     "gather",    "tree",      "gate_rows", "gate_decide", "pad_queries",
     "tree_mask", "project",  "kmeans",    "ivf_build", "ivf_coarse",
-    "ivf_scan",  "ctx",       "tree_attn", "rescore"};
+    "ivf_scan",  "ctx",       "tree_attn", "rescore",   "draft"};
 
 cudaEvent_t take_event() {
   if (!g_ev_pool.empty()) {
@@ -100,7 +101,7 @@ int sm_count() {
 }
 
 LaunchScope::LaunchScope(KernelId id, cudaStream_t s) : id_(id), s_(s), slot_(-1) {
-  if (!g_prof_on) return;
+  if (!g_prof_on || !g_prof_family[id]) return;
   std::lock_guard<std::mutex> lk(g_mu);
   ProfRec r{id, take_event(), take_event()};
   cudaEventRecord(r.a, s);
@@ -439,6 +440,56 @@ sense_status sense_build_tree(const int32_t* spans, int32_t q, int32_t k, int32_
                      out_depth, out_gamma, out_mask_bits, status, stream);
 }
 
+sense_status sense_draft(const sense_datastore* ds, const uint16_t* queries, int32_t q, int32_t k,
+                         void* workspace, size_t workspace_bytes, int32_t node_cap, uint32_t flags,
+                         float* out_scores, int32_t* out_idx, int32_t* out_spans,
+                         int32_t* out_num_nodes, int32_t* out_tokens, int32_t* out_parent,
+                         int32_t* out_depth, int32_t* out_gamma, uint32_t* out_mask_bits,
+                         sense_stream_t stream) {
+  sense_status st = check_ds(ds);
+  if (st != SENSE_OK) return st;
+  if (!queries || !out_scores || !out_idx || !workspace || !out_spans || !out_num_nodes ||
+      !out_tokens || !out_parent || !out_depth || !out_gamma)
+    return fail(SENSE_ERR_INVALID_ARG, "queries, workspace and outputs must be non-NULL");
+  if (q < 1) return fail(SENSE_ERR_INVALID_ARG, "q=%d must be >= 1", q);
+  if (k < 1 || k > SENSE_MAX_K || (int64_t)k > ds->n)
+    return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, min(n=%lld, %d)]", k, (long long)ds->n, SENSE_MAX_K);
+  const int m = ds->m;
+  if ((int64_t)k * m > SENSE_MAX_TREE_TOKENS)
+    return fail(SENSE_ERR_INVALID_ARG, "k*m=%d exceeds %d", k * m, SENSE_MAX_TREE_TOKENS);
+  if (node_cap < 0) return fail(SENSE_ERR_INVALID_ARG, "node_cap=%d must be >= 0", node_cap);
+  if (flags & ~SENSE_TREE_MASK_BITS) return fail(SENSE_ERR_INVALID_ARG, "unknown tree flags 0x%x", flags);
+  const bool bits = (flags & SENSE_TREE_MASK_BITS) != 0;
+  if (bits && !out_mask_bits) return fail(SENSE_ERR_INVALID_ARG, "SENSE_TREE_MASK_BITS needs out_mask_bits");
+  if (!aligned(queries, 16) || !aligned(out_spans, 16))
+    return fail(SENSE_ERR_INVALID_ARG, "queries and out_spans must be 16-byte aligned");
+  if (q > 8 && ds->n > 2147483647LL - 1024)
+    return fail(SENSE_ERR_UNSUPPORTED, "batched (q > 8) retrieval supports n <= 2^31 - 1025");
+  if (!aligned(workspace, 256)) return fail(SENSE_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  const RetrievePlan p = make_plan(ds, q, k);
+  if (workspace_bytes < p.total)
+    return fail(SENSE_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", workspace_bytes, p.total);
+  const int cap = node_cap > 0 ? node_cap : k * m;
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  char* ws = static_cast<char*>(workspace);
+  if (p.fused && draft_fused_fits(k, m)) {
+    // single-pass scan, then merge + gather + trie in one kernel per query
+    uint64_t* pool = reinterpret_cast<uint64_t*>(ws + p.off_pool);
+    st = launch_scan_gemv_topk(ds->keys, ds->n, ds->d, queries, q, k, p.fused_blocks, pool, stream);
+    if (st != SENSE_OK) return st;
+    return launch_draft_fused(pool, p.fused_blocks, q, k, out_scores, out_idx, ds->spans, ds->n, m,
+                              out_spans, cap, bits ? 1 : 0, out_num_nodes, out_tokens, out_parent,
+                              out_depth, out_gamma, out_mask_bits, status, stream);
+  }
+  st = run_retrieve(p, ds, queries, q, k, out_scores, out_idx, ws, status, stream);
+  if (st != SENSE_OK) return st;
+  st = launch_gather(ds->spans, ds->n, m, out_idx, q, k, nullptr, k, 0, out_spans, status, stream);
+  if (st != SENSE_OK) return st;
+  return launch_tree(out_spans, q, k, m, cap, bits ? 1 : 0, out_num_nodes, out_tokens, out_parent,
+                     out_depth, out_gamma, out_mask_bits, status, stream);
+}
+
 sense_status sense_tree_mask_full(const uint32_t* mask_bits, const int32_t* num_nodes, int32_t q,
                                   int32_t cap, const int32_t* prefix_len, int32_t cache_len,
                                   float* out, sense_stream_t stream) {
@@ -546,6 +597,28 @@ sense_status sense_profile_enable(int32_t on) {
   }
   g_prof.clear();
   g_prof_on = on != 0;
+  for (int i = 0; i < K_COUNT; ++i) g_prof_family[i] = true;
+  return SENSE_OK;
+}
+
+sense_status sense_profile_filter(const char* names) {
+  bool sel[K_COUNT];
+  for (int i = 0; i < K_COUNT; ++i) sel[i] = (names == nullptr || names[0] == 0);
+  if (names && names[0]) {
+    const char* p = names;
+    while (*p) {
+      const char* e = strchr(p, ',');
+      const size_t len = e ? (size_t)(e - p) : strlen(p);
+      int id = -1;
+      for (int i = 0; i < K_COUNT; ++i)
+        if (strlen(kKernelNames[i]) == len && strncmp(p, kKernelNames[i], len) == 0) id = i;
+      if (id < 0) return fail(SENSE_ERR_INVALID_ARG, "unknown kernel family in '%s'", names);
+      sel[id] = true;
+      p = e ? e + 1 : p + len;
+    }
+  }
+  std::lock_guard<std::mutex> lk(g_mu);
+  for (int i = 0; i < K_COUNT; ++i) g_prof_family[i] = sel[i];
   return SENSE_OK;
 }
 

@@ -43,6 +43,7 @@ enum KernelId {
   K_CTX,
   K_TREE_ATTN,
   K_RESCORE,
+  K_DRAFT,
   K_COUNT
 };
 

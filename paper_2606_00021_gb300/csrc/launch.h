@@ -85,6 +85,16 @@ sense_status launch_scan_tc(const uint16_t* keys, int64_t n, int d, const uint16
                             uint64_t* out, uint32_t* counts, int64_t pool_cap, uint32_t* status,
                             cudaStream_t s);
 sense_status launch_selftest_wait(long long limit, uint32_t* status, cudaStream_t s);
+// The single-query drafting tail fused in one kernel per query: merge of the
+// single-pass scan's `nlists` lists, span gather, small-tree trie (k <=
+// 128; draft_fused_fits(k, m)).  Outputs as launch_merge_lists,
+// launch_gather (no anchor) and launch_tree.
+bool draft_fused_fits(int k, int m);
+sense_status launch_draft_fused(const uint64_t* lists, int nlists, int q, int k, float* out_scores,
+                                int32_t* out_idx, const int32_t* spans, int64_t n, int m,
+                                int32_t* out_spans, int cap, int mask_bits, int32_t* num_nodes,
+                                int32_t* tokens, int32_t* parent, int32_t* depth, int32_t* gamma,
+                                uint32_t* mask, uint32_t* status, cudaStream_t s);
 // Exact scores of a shortlist of n_cand key indices per query (-1 = empty),
 // top k by (score desc, index asc).
 sense_status launch_rescore(const uint16_t* keys, int64_t n, int d, const uint16_t* queries, int q,

@@ -20,6 +20,7 @@
 //  - merge: per query, the k largest pool keys, bitonic-sorted in shared
 //    memory, become the output scores and indices.
 #include "common.cuh"
+#include "draft_dev.cuh"
 #include "launch.h"
 #include "tc_ptx.cuh"
 
@@ -517,16 +518,15 @@ __device__ bool merge_lists_short(const uint64_t* __restrict__ src, int nlists, 
   return true;
 }
 
-__global__ void __launch_bounds__(kSelThreads, 1)
-merge_lists_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
-                   float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
-                   uint32_t* status) {
-  extern __shared__ uint64_t s_keys[];  // [kSmemKeys]
+// Merge of query q's nlists sorted lists of k keys into its top k, by one
+// block of kSelThreads threads; s_keys holds kSmemKeys keys.
+__device__ void merge_lists_block(const uint64_t* __restrict__ lists, int nlists, int k,
+                                  float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
+                                  uint32_t* status, int q, uint64_t* s_keys) {
   __shared__ unsigned hist[256];
   __shared__ Digit dig;
   __shared__ unsigned n_sel, n_got;
   __shared__ uint64_t sel[SENSE_MAX_K];
-  const int q = blockIdx.x;
   const uint64_t* src = lists + (int64_t)q * nlists * k;
   if ((int64_t)nlists * k <= kFastKeys && nlists <= kRankHeads && ((nlists * k) & 1) == 0 &&
       (reinterpret_cast<uintptr_t>(src) & 15) == 0) {
@@ -612,6 +612,39 @@ merge_lists_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
   }
 }
 
+__global__ void __launch_bounds__(kSelThreads, 1)
+merge_lists_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
+                   float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
+                   uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];  // [kSmemKeys]
+  merge_lists_block(lists, nlists, k, out_scores, out_idx, status, blockIdx.x, s_keys);
+}
+
+// The single-query drafting tail in one block per query: the merge of the
+// scan's per-block lists into the top k, the span gather of those k keys
+// and the small-tree trie of the gathered spans, one after the other.  Each
+// phase reads what the previous one wrote to global memory (visible inside
+// the block after a barrier); the trie reuses the merge's shared memory.
+__global__ void __launch_bounds__(kSelThreads, 1)
+draft_fused_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
+                   float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
+                   const int32_t* __restrict__ spans, int64_t n, int m, int32_t* out_spans,
+                   int cap, int mask_words, int32_t* __restrict__ num_nodes,
+                   int32_t* __restrict__ tokens, int32_t* __restrict__ parent,
+                   int32_t* __restrict__ depth, int32_t* __restrict__ gamma,
+                   uint32_t* __restrict__ mask, uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];  // [kSmemKeys]
+  __shared__ int scratch[32];
+  __shared__ int sv[3];
+  const int q = blockIdx.x;
+  merge_lists_block(lists, nlists, k, out_scores, out_idx, status, q, s_keys);
+  __syncthreads();
+  gather_block(spans, n, m, out_idx, k, nullptr, k, 0, out_spans, status, q, scratch);
+  __syncthreads();
+  tree_small_block(out_spans, k, m, cap, mask_words, num_nodes, tokens, parent, depth, gamma,
+                   mask, status, q, reinterpret_cast<int*>(s_keys), scratch, sv);
+}
+
 template <class K>
 sense_status set_smem(K kern, size_t bytes) {
   return cuda_check(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -656,6 +689,25 @@ sense_status launch_merge_lists(const uint64_t* lists, int nlists, int q, int k,
   merge_lists_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(
       lists, nlists, k, out_scores, out_idx, status);
   return cuda_check(cudaGetLastError(), "launch merge_lists");
+}
+
+sense_status launch_draft_fused(const uint64_t* lists, int nlists, int q, int k, float* out_scores,
+                                int32_t* out_idx, const int32_t* spans, int64_t n, int m,
+                                int32_t* out_spans, int cap, int mask_bits, int32_t* num_nodes,
+                                int32_t* tokens, int32_t* parent, int32_t* depth, int32_t* gamma,
+                                uint32_t* mask, uint32_t* status, cudaStream_t s) {
+  sense_status st = set_smem(draft_fused_kernel, kSmemKeys * sizeof(uint64_t));
+  if (st != SENSE_OK) return st;
+  LaunchScope ls(K_DRAFT, s);
+  draft_fused_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(
+      lists, nlists, k, out_scores, out_idx, spans, n, m, out_spans, cap, (cap + 31) / 32,
+      num_nodes, tokens, parent, depth, gamma, mask_bits ? mask : nullptr, status);
+  return cuda_check(cudaGetLastError(), "launch draft_fused");
+}
+
+bool draft_fused_fits(int k, int m) {
+  return k <= kTreeSmallK && sizeof(int) * ((size_t)3 * k * m + (size_t)5 * k) <=
+                                 kSmemKeys * sizeof(uint64_t);
 }
 
 sense_status launch_merge(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap, int q,

@@ -55,6 +55,7 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert lib.sense_retrieve_topk(None, p, 1, 1, p, p, p, 1 << 20, None) == 1
     assert lib.sense_retrieve_topk_noalloc(None, p, 1, 1, p, p, None) == 1
     assert lib.sense_rescore_topk(None, p, 1, p, 8, 4, p, p, None) == 1
+    assert lib.sense_draft(None, p, 1, 8, p, 1 << 20, 0, 0, p, p, p, p, p, p, p, p, None, None) == 1
     # allocation-free status reader and self test: NULL output, limit range
     assert lib.sense_retrieve_noalloc_status(None, None, 1) == 1
     assert lib.sense_retrieve_noalloc_selftest(None, 0) == 1

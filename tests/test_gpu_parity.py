@@ -387,3 +387,39 @@ def test_bounded_wait_reports_timeout_and_context_survives(S):
     full = O.scores(bits(keys), bits(qs))
     for qi in range(16):
         check_topk(host(sc[qi]), host(ix[qi]), full[qi], 8)
+
+
+# ---------------------------------------------------------------- drafting step in one call
+
+@cuda
+@pytest.mark.parametrize("n,d,m,q,k,cap,with_bits", [
+    (50000, 512, 16, 1, 32, 64, True),      # the single-query path: one fused kernel
+    (50000, 512, 16, 2, 128, 0, False),     # uncapped, 128 candidates
+    (70000, 4096, 8, 4, 8, 10, True),       # cap below the node count
+    (20000, 256, 32, 3, 64, 128, False),    # long spans
+    (50000, 512, 16, 8, 32, 64, True),      # sampled-threshold retrieval (separate launches)
+    (30000, 512, 16, 16, 64, 100, True),    # tensor-core retrieval (separate launches)
+    (30000, 512, 4, 1, 200, 0, False),      # k > 128: the large trie (separate launches)
+])
+def test_draft_equals_separate_calls(S, n, d, m, q, k, cap, with_bits):
+    """sense_draft is bit-identical to retrieve + gather + tree called one by
+    one (which the other tests compare with the oracle), on every path."""
+    dev = torch.device("cuda")
+    keys = synth.clustered_unit_keys(n, d, 64, seed=n % 89, device=dev)
+    spans = synth.spans_uniform(n, m, 6, seed=m, device=dev)  # few tokens: shared prefixes
+    ds = S.sense_datastore_build(keys, spans)
+    qs, _ = synth.noisy_queries(keys, q, seed=q + k)
+    for _ in range(2):  # twice in a row: nothing left over from the first call matters
+        got = S.sense_draft(ds, qs, k, node_cap=cap, mask_bits=with_bits)
+        sc, ix = S.sense_retrieve_topk(ds, qs, k)
+        dr = S.sense_gather_drafts(ds, ix)
+        tr = S.sense_build_tree(dr, node_cap=cap, mask_bits=with_bits)
+        torch.cuda.synchronize()
+        assert S.sense_device_status(clear=True) == 0
+        assert torch.equal(got["scores"], sc) and torch.equal(got["idx"], ix)
+        assert torch.equal(got["spans"], dr)
+        for key in ("num_nodes", "tokens", "parent", "depth", "gamma") + (("mask_bits",) if with_bits else ()):
+            assert torch.equal(got[key], tr[key]), key
+    full = O.scores(bits(keys), bits(qs))
+    for qi in range(q):
+        check_topk(host(got["scores"][qi]), host(got["idx"][qi]), full[qi], k)
