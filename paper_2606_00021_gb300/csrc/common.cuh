@@ -77,6 +77,17 @@ __device__ __forceinline__ uint64_t cand_key(float s, uint32_t idx) {
 }
 __device__ __forceinline__ uint32_t cand_index(uint64_t c) { return ~(uint32_t)c; }
 
+// Programmatic dependent launch: a kernel launched with
+// cudaLaunchAttributeProgrammaticStreamSerialization may be scheduled
+// before the kernel ahead of it in the stream has finished; pdl_wait()
+// blocks until that kernel has completed and its memory is visible (a
+// no-op for a normal launch).  pdl_launch_dependents() lets the next such
+// kernel be scheduled while this one still runs.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ void raise_status(uint32_t* st, uint32_t bits) {
   if (st) atomicOr(st, bits);
 }

@@ -471,6 +471,8 @@ gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__
   extern __shared__ __align__(128) float4 ring_all[];
   __shared__ __align__(8) uint64_t bars_all[kWarps * kWStages];
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  pdl_wait();
+  pdl_launch_dependents();
   if (threadIdx.x == 0) {
     for (int b = 0; b < kWarps * kWStages; ++b) ptx::mbar_init(ptx::smem_u32(bars_all + b), 1);
     ptx::fence_barrier_init();
@@ -552,6 +554,8 @@ gate_row_block_kernel(const int32_t* __restrict__ parent, const int32_t* __restr
   __shared__ Partial s_part[kWarps];
   __shared__ int s_fail;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  pdl_wait();  // the tree (and everything before it) is complete
+  pdl_launch_dependents();
   const int rid = blockIdx.x / NC;  // q * (cap + 1) + slot
   const int crank = blockIdx.x - rid * NC;  // rank in the cluster (clusters of NC along x)
   const int q = rid / (cap + 1);
@@ -646,6 +650,7 @@ gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats, int staged) {
   __shared__ int s_best[32];
   __shared__ int s_istar, s_lstar, s_next, s_nn;
   __shared__ ArgMax s_w[32];
+  pdl_wait();  // every row statistic is written
   const int q = blockIdx.x;
   const int k = a.k, m = a.m, cap = a.cap, km = k * m;
   const int32_t* gam = a.gamma + (int64_t)q * km;
@@ -884,13 +889,15 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     cfg.blockDim = dim3(kRowThreads);
     cfg.dynamicSmemBytes = kRingBytes;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = (unsigned)nc;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     LaunchScope ls(K_GATE_ROWS, s);
     st = cuda_check(cudaLaunchKernelEx(&cfg, kern, a.parent, a.num_nodes, a.cap, a.root_logits,
                                        a.node_logits, a.vocab, a.kappa, a.thr, a.unnormalized,
@@ -936,10 +943,20 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
                     "cudaFuncSetAttribute(gate_decide)");
     if (st != SENSE_OK) return st;
   }
-  LaunchScope ls(K_GATE_DECIDE, s);
   const int threads = (a.k * a.m <= 4096) ? 256 : kDecideThreads;
-  gate_decide_kernel<<<a.q, threads, smem, s>>>(a, stats, staged);
-  return cuda_check(cudaGetLastError(), "launch gate_decide");
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)a.q);
+  cfg.blockDim = dim3((unsigned)threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  LaunchScope ls(K_GATE_DECIDE, s);
+  return cuda_check(cudaLaunchKernelEx(&cfg, gate_decide_kernel, a, (const int32_t*)stats, staged),
+                    "launch gate_decide");
 }
 
 }  // namespace sense

@@ -128,6 +128,7 @@ scan_gemv_topk_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
   constexpr int K = KPL * 32;   // list length per warp
   constexpr int L = 8 * K;      // entries per query per block (8 warps)
   extern __shared__ uint4 s_q[];  // [Q][C] bf16 chunks, then the lists
+  pdl_launch_dependents();      // the merge may be scheduled; it waits for this grid
   const int C = d >> 3;
   const uint4* qsrc = reinterpret_cast<const uint4*>(queries);
   for (int i = threadIdx.x; i < Q * C; i += blockDim.x) s_q[i] = qsrc[i];

@@ -637,6 +637,8 @@ draft_fused_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
   __shared__ int scratch[32];
   __shared__ int sv[3];
   const int q = blockIdx.x;
+  pdl_wait();  // the scan's lists are complete
+  pdl_launch_dependents();
   merge_lists_block(lists, nlists, k, out_scores, out_idx, status, q, s_keys);
   __syncthreads();
   gather_block(spans, n, m, out_idx, k, nullptr, k, 0, out_spans, status, q, scratch);
@@ -698,11 +700,22 @@ sense_status launch_draft_fused(const uint64_t* lists, int nlists, int q, int k,
                                 uint32_t* mask, uint32_t* status, cudaStream_t s) {
   sense_status st = set_smem(draft_fused_kernel, kSmemKeys * sizeof(uint64_t));
   if (st != SENSE_OK) return st;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)q);
+  cfg.blockDim = dim3(kSelThreads);
+  cfg.dynamicSmemBytes = kSmemKeys * sizeof(uint64_t);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
   LaunchScope ls(K_DRAFT, s);
-  draft_fused_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(
-      lists, nlists, k, out_scores, out_idx, spans, n, m, out_spans, cap, (cap + 31) / 32,
-      num_nodes, tokens, parent, depth, gamma, mask_bits ? mask : nullptr, status);
-  return cuda_check(cudaGetLastError(), "launch draft_fused");
+  return cuda_check(cudaLaunchKernelEx(&cfg, draft_fused_kernel, lists, nlists, k, out_scores,
+                                       out_idx, spans, n, m, out_spans, cap, (cap + 31) / 32,
+                                       num_nodes, tokens, parent, depth, gamma,
+                                       mask_bits ? mask : nullptr, status),
+                    "launch draft_fused");
 }
 
 bool draft_fused_fits(int k, int m) {
