@@ -203,6 +203,9 @@ class Pipeline:
             self.cand_i = torch.empty(q, kk, dtype=torch.int32, device=dev)
         self.ws = self.S.alloc_workspace(
             self.S.sense_ivf_search_workspace_bytes(ann["index"], q, kk, ann["nprobe"]), dev)
+        import ctypes
+        self.ann_ws = self.S.alloc_workspace(self.S.lib().sense_ann_draft_workspace_bytes(
+            ctypes.c_void_p(ann["index"].handle), q, k, ann["nprobe"], ann.get("rerank", 0)), dev)
 
     def retrieve(self, query):
         S, cfg = self.S, self.cfg
@@ -249,13 +252,19 @@ class Pipeline:
         S, cfg = self.S, self.cfg
         dyn = getattr(self, "dyn", None)
         ver = getattr(self, "verify", None)
-        if self.ann is None and dyn is None:
-            # exact retrieval, gather and trie in one call (one kernel per
+        if dyn is None:
+            # retrieval, gather and trie in one call (exact: one kernel per
             # query after the scan on the single-pass path)
             outs = self.tree
             outs["scores"], outs["idx"], outs["spans"] = self.scores, self.idx, self.drafts
-            S.sense_draft(self.ds, query, cfg["k"], node_cap=cfg["cap"], mask_bits=ver is not None,
-                          outs=outs, workspace=self.ws)
+            if self.ann is None:
+                S.sense_draft(self.ds, query, cfg["k"], node_cap=cfg["cap"],
+                              mask_bits=ver is not None, outs=outs, workspace=self.ws)
+            else:
+                a = self.ann
+                S.sense_ann_draft(a["index"], self.ds, query, a["basis"], a["mean"], cfg["k"],
+                                  a["nprobe"], rerank=a.get("rerank", 0), node_cap=cfg["cap"],
+                                  mask_bits=ver is not None, outs=outs, workspace=self.ann_ws)
         else:
             self.retrieve(query)
             if dyn is None:

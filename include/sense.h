@@ -337,6 +337,31 @@ sense_status sense_rescore_topk(const sense_datastore* ds, const uint16_t* queri
                                 const int32_t* cand_idx, int32_t n_cand, int32_t k,
                                 float* out_scores, int32_t* out_idx, sense_stream_t stream);
 
+/*
+ * The approximate drafting step of one query batch in one call (App. E:
+ * k = L2Norm(PCA(h)) searched in an IVF / IVF-PQ index, Sec. 3.2.2 Eq. 7
+ * ANN; optionally Eq. 8's exact re-scoring of N' = rerank candidates; then
+ * the D_ret span gather and the Sec. 3.2.3 Eq. 9 loose trie): the results,
+ * bit for bit, of sense_project (normalised), sense_ivf_search (k, or
+ * rerank candidates followed by sense_rescore_topk to k), sense_gather_drafts
+ * without an anchor and sense_build_tree.  queries: bf16 [q, d] hidden
+ * states with d = the datastore's d; basis [v, d] and mean [d] (nullable)
+ * as for sense_project, v = the index's dimension; rerank = 0 (no
+ * re-scoring) or in [k, SENSE_MAX_RESCORE].  The workspace is
+ * sense_ann_draft_workspace_bytes(ix, q, k, nprobe, rerank) bytes, 256-byte
+ * aligned; outputs as sense_draft.  Errors and device status are those of
+ * the composed calls.
+ */
+size_t sense_ann_draft_workspace_bytes(const sense_ivf* ix, int32_t q, int32_t k, int32_t nprobe,
+                                       int32_t rerank);
+sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, const uint16_t* queries,
+                             int32_t q, const float* basis, const float* mean, int32_t k,
+                             int32_t nprobe, int32_t rerank, int32_t node_cap, uint32_t flags,
+                             void* workspace, size_t workspace_bytes, float* out_scores,
+                             int32_t* out_idx, int32_t* out_spans, int32_t* out_num_nodes,
+                             int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
+                             int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream);
+
 /* ---------------------------------------------------------------------- */
 /* a4. Span gather                                                          */
 /* ---------------------------------------------------------------------- */

@@ -451,6 +451,50 @@ def sense_ivf_search_workspace_bytes(ix: IvfIndex, q: int, k: int, nprobe: int) 
     return int(lib().sense_ivf_search_workspace_bytes(C.c_void_p(ix.handle), q, k, nprobe))
 
 
+def sense_ann_draft(ix: "IvfIndex", ds: Datastore, queries: torch.Tensor, basis: torch.Tensor,
+                    mean: torch.Tensor | None, k: int, nprobe: int, rerank: int = 0,
+                    node_cap: int = 0, mask_bits: bool = False, outs: dict | None = None,
+                    workspace=None, stream=None):
+    """Projection, IVF search (with optional exact re-scoring of `rerank`
+    candidates), span gather and loose trie of one query batch in one call;
+    the results of those calls one by one.  Returns a dict like sense_draft."""
+    _need(queries, "queries", torch.bfloat16, 2)
+    _need(basis, "basis", torch.float32, 2)
+    if mean is not None:
+        _need(mean, "mean", torch.float32, 1)
+    q = queries.shape[0]
+    if queries.shape[1] != ds.d:
+        raise ValueError("queries must have d columns")
+    m = ds.m
+    cap = node_cap if node_cap > 0 else k * m
+    dev = queries.device
+    o = outs if outs is not None else {}
+    o.setdefault("scores", torch.empty(q, k, dtype=torch.float32, device=dev))
+    o.setdefault("idx", _i32((q, k), dev))
+    o.setdefault("spans", _i32((q, k, m), dev))
+    o.setdefault("num_nodes", _i32((q,), dev))
+    o.setdefault("tokens", _i32((q, cap), dev))
+    o.setdefault("parent", _i32((q, cap), dev))
+    o.setdefault("depth", _i32((q, cap), dev))
+    o.setdefault("gamma", _i32((q, k, m), dev))
+    if mask_bits:
+        o.setdefault("mask_bits", torch.empty(q, cap, (cap + 31) // 32, dtype=torch.int32,
+                                              device=dev))
+    if workspace is None:
+        need = lib().sense_ann_draft_workspace_bytes(C.c_void_p(ix.handle), q, k, nprobe, rerank)
+        workspace = alloc_workspace(need, dev)
+    _check(lib().sense_ann_draft(C.c_void_p(ix.handle), C.c_void_p(ds.handle), queries.data_ptr(),
+                                 q, basis.data_ptr(), _ptr(mean), k, nprobe, rerank, node_cap,
+                                 1 if mask_bits else 0, workspace.data_ptr(), workspace.numel(),
+                                 o["scores"].data_ptr(), o["idx"].data_ptr(), o["spans"].data_ptr(),
+                                 o["num_nodes"].data_ptr(), o["tokens"].data_ptr(),
+                                 o["parent"].data_ptr(), o["depth"].data_ptr(),
+                                 o["gamma"].data_ptr(), _ptr(o.get("mask_bits")),
+                                 C.c_void_p(_stream(stream))))
+    o["cap"] = cap
+    return o
+
+
 def sense_ivf_search(ix: IvfIndex, queries: torch.Tensor, k: int, nprobe: int,
                      out_scores=None, out_idx=None, want_probes: bool = False, workspace=None,
                      stream=None):

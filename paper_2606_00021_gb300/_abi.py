@@ -29,6 +29,9 @@ SIGNATURES = {
     "sense_retrieve_topk_noalloc": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_p, c_p]),
     "sense_retrieve_noalloc_status": (c_i32, [c_p, C.POINTER(c_u32), c_i32]),
     "sense_retrieve_noalloc_selftest": (c_i32, [c_p, c_i64]),
+    "sense_ann_draft_workspace_bytes": (c_size, [c_p, c_i32, c_i32, c_i32, c_i32]),
+    "sense_ann_draft": (c_i32, [c_p, c_p, c_p, c_i32, c_p, c_p, c_i32, c_i32, c_i32, c_i32, c_u32,
+                                c_p, c_size, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p]),
     "sense_rescore_topk": (c_i32, [c_p, c_p, c_i32, c_p, c_i32, c_i32, c_p, c_p, c_p]),
     "sense_gather_drafts": (c_i32, [c_p, c_p, c_i32, c_i32, c_p, c_i32, c_u32, c_p, c_p]),
     "sense_build_tree": (c_i32, [c_p, c_i32, c_i32, c_i32, c_i32, c_u32, c_p, c_p, c_p, c_p,

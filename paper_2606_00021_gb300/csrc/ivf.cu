@@ -1156,4 +1156,80 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
   return launch_merge_short(pool, counts, p.pool_cap, q, k, out_scores, out_idx, status, s);
 }
 
+size_t sense_ann_draft_workspace_bytes(const sense_ivf* ix, int32_t q, int32_t k, int32_t nprobe,
+                                       int32_t rerank) {
+  if (!ix || q < 1 || k < 1 || nprobe < 1 || rerank < 0) return 0;
+  const int kk = std::max(k, rerank);
+  size_t b = align256((size_t)q * ix->v * 4);
+  if (rerank > 0) b += 2 * align256((size_t)q * kk * 4);
+  return b + sense_ivf_search_workspace_bytes(ix, q, kk, nprobe);
+}
+
+sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, const uint16_t* queries,
+                             int32_t q, const float* basis, const float* mean, int32_t k,
+                             int32_t nprobe, int32_t rerank, int32_t node_cap, uint32_t flags,
+                             void* workspace, size_t workspace_bytes, float* out_scores,
+                             int32_t* out_idx, int32_t* out_spans, int32_t* out_num_nodes,
+                             int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
+                             int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream) {
+  if (!ix || !ds) return fail(SENSE_ERR_INVALID_ARG, "index and datastore must be non-NULL");
+  if (!queries || !basis || !workspace || !out_scores || !out_idx || !out_spans ||
+      !out_num_nodes || !out_tokens || !out_parent || !out_depth || !out_gamma)
+    return fail(SENSE_ERR_INVALID_ARG, "queries, basis, workspace and outputs must be non-NULL");
+  if (ds->device != current_device() || ix->device != current_device())
+    return fail(SENSE_ERR_INVALID_ARG, "index and datastore must live on the current device");
+  if (q < 1 || q > 65535) return fail(SENSE_ERR_INVALID_ARG, "q=%d outside [1, 65535]", q);
+  if (k < 1 || k > SENSE_MAX_K) return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, %d]", k, SENSE_MAX_K);
+  if (rerank < 0 || (rerank > 0 && (rerank < k || rerank > SENSE_MAX_RESCORE)))
+    return fail(SENSE_ERR_INVALID_ARG, "rerank=%d must be 0 or in [k=%d, %d]", rerank, k,
+                SENSE_MAX_RESCORE);
+  const int m = ds->m;
+  if ((int64_t)k * m > SENSE_MAX_TREE_TOKENS)
+    return fail(SENSE_ERR_INVALID_ARG, "k*m=%d exceeds %d", k * m, SENSE_MAX_TREE_TOKENS);
+  if (node_cap < 0) return fail(SENSE_ERR_INVALID_ARG, "node_cap=%d must be >= 0", node_cap);
+  if (flags & ~SENSE_TREE_MASK_BITS) return fail(SENSE_ERR_INVALID_ARG, "unknown tree flags 0x%x", flags);
+  const bool bits = (flags & SENSE_TREE_MASK_BITS) != 0;
+  if (bits && !out_mask_bits) return fail(SENSE_ERR_INVALID_ARG, "SENSE_TREE_MASK_BITS needs out_mask_bits");
+  if (!aligned(workspace, 256) || !aligned(out_spans, 16))
+    return fail(SENSE_ERR_INVALID_ARG, "workspace must be 256-byte and out_spans 16-byte aligned");
+  const size_t need = sense_ann_draft_workspace_bytes(ix, q, k, nprobe, rerank);
+  if (workspace_bytes < need)
+    return fail(SENSE_ERR_INVALID_ARG, "workspace of %zu bytes < %zu", workspace_bytes, need);
+  const int kk = std::max(k, rerank);
+  char* ws = static_cast<char*>(workspace);
+  float* qproj = reinterpret_cast<float*>(ws);
+  ws += align256((size_t)q * ix->v * 4);
+  float* cand_s = nullptr;
+  int32_t* cand_i = nullptr;
+  if (rerank > 0) {
+    cand_s = reinterpret_cast<float*>(ws);
+    ws += align256((size_t)q * kk * 4);
+    cand_i = reinterpret_cast<int32_t*>(ws);
+    ws += align256((size_t)q * kk * 4);
+  }
+  const size_t ivf_bytes = sense_ivf_search_workspace_bytes(ix, q, kk, nprobe);
+  // query construction (Alg. 2: k = L2Norm(PCA(h))), search, optional
+  // exact re-scoring (Eq. 8), gather and trie
+  sense_status st = sense_project(queries, q, ds->d, basis, ix->v, mean, SENSE_PROJECT_NORMALIZE,
+                                  qproj, stream);
+  if (st != SENSE_OK) return st;
+  if (rerank > 0) {
+    st = sense_ivf_search(ix, qproj, q, rerank, nprobe, cand_s, cand_i, nullptr, ws, ivf_bytes,
+                          stream);
+    if (st != SENSE_OK) return st;
+    st = sense_rescore_topk(ds, queries, q, cand_i, rerank, k, out_scores, out_idx, stream);
+  } else {
+    st = sense_ivf_search(ix, qproj, q, k, nprobe, out_scores, out_idx, nullptr, ws, ivf_bytes,
+                          stream);
+  }
+  if (st != SENSE_OK) return st;
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  const int cap = node_cap > 0 ? node_cap : k * m;
+  st = launch_gather(ds->spans, ds->n, m, out_idx, q, k, nullptr, k, 0, out_spans, status, stream);
+  if (st != SENSE_OK) return st;
+  return launch_tree(out_spans, q, k, m, cap, bits ? 1 : 0, out_num_nodes, out_tokens, out_parent,
+                     out_depth, out_gamma, out_mask_bits, status, stream);
+}
+
 }  // extern "C"

@@ -333,3 +333,51 @@ def test_rescore_lattice_bit_exact_and_bad_index(S):
     bad[bad >= n] = -1
     ws2, wi2 = I.rescore_topk(bits(keys), bits(qs), bad, k)
     np.testing.assert_array_equal(host(ix2), wi2)
+
+
+# ---------------------------------------------------------------- approximate drafting step in one call
+
+@cuda
+@pytest.mark.parametrize("pq,rerank,q,k,cap", [
+    (False, 0, 1, 32, 64), (True, 0, 1, 32, 64), (True, 128, 1, 32, 64), (True, 64, 3, 16, 0),
+    (False, 40, 2, 40, 30),
+])
+def test_ann_draft_equals_separate_calls(S, pq, rerank, q, k, cap):
+    """sense_ann_draft is bit-identical to projection, IVF search (and the
+    exact re-scoring), gather and trie called one by one."""
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(17 + k)
+    n, d, v, nlist = 20000, 512, 32, 64
+    keys = synth.clustered_unit_keys(n, d, 32, seed=19, device=dev)
+    spans = synth.spans_uniform(n, 8, 5, seed=2, device=dev)
+    ds = S.sense_datastore_build(keys, spans)
+    basis = _dev(np.linalg.qr(rng.standard_normal((d, v)))[0].T.astype(np.float32).copy())
+    mean = _dev((0.01 * rng.standard_normal(d)).astype(np.float32))
+    kp = S.sense_project(keys, basis, mean)
+    cent = S.sense_kmeans(kp[:4096].contiguous(), kp[:nlist].clone(), 3, True)
+    cb = None
+    if pq:
+        _, res = S.sense_ivf_residuals(kp[:4096].contiguous(), cent)
+        cb = torch.stack([S.sense_kmeans(res[:, 4 * mm:4 * mm + 4].contiguous(),
+                                         res[:256, 4 * mm:4 * mm + 4].contiguous(), 3, False)
+                          for mm in range(v // 4)])
+    ix = S.sense_ivf_build(kp, cent, cb)
+    qs, _ = synth.noisy_queries(keys, q, seed=23)
+    for _ in range(2):
+        got = S.sense_ann_draft(ix, ds, qs, basis, mean, k, 8, rerank=rerank, node_cap=cap,
+                                mask_bits=True)
+        qp = S.sense_project(qs, basis, mean)
+        if rerank:
+            _, ci = S.sense_ivf_search(ix, qp, rerank, 8)
+            sc, idx = S.sense_rescore_topk(ds, qs, ci, k)
+        else:
+            sc, idx = S.sense_ivf_search(ix, qp, k, 8)
+        dr = S.sense_gather_drafts(ds, idx)
+        tr = S.sense_build_tree(dr, node_cap=cap, mask_bits=True)
+        torch.cuda.synchronize()
+        assert S.sense_device_status(clear=True) == 0
+        assert torch.equal(got["scores"], sc) and torch.equal(got["idx"], idx)
+        assert torch.equal(got["spans"], dr)
+        for key in ("num_nodes", "tokens", "parent", "depth", "gamma", "mask_bits"):
+            assert torch.equal(got[key], tr[key]), key
+    ix.close()
