@@ -41,6 +41,8 @@ __global__ void gather_kernel(const int32_t* __restrict__ spans, int64_t n, int 
                               const int32_t* __restrict__ idx, int k,
                               const int32_t* __restrict__ anchor, int n_keep, int force,
                               int32_t* __restrict__ out, uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   __shared__ int scratch[32];
   gather_block(spans, n, m, idx, k, anchor, n_keep, force, out, status, blockIdx.x, scratch);
 }
@@ -63,6 +65,8 @@ tree_kernel(const int32_t* __restrict__ spans, int k, int m, int cap, int mask_w
             int32_t* __restrict__ num_nodes, int32_t* __restrict__ tokens,
             int32_t* __restrict__ parent, int32_t* __restrict__ depth,
             int32_t* __restrict__ gamma, uint32_t* __restrict__ mask, uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   extern __shared__ int sm[];
   const int km = k * m;
   int kp = 1;
@@ -268,6 +272,8 @@ tree_small_kernel(const int32_t* __restrict__ spans, int k, int m, int cap, int 
                   int32_t* __restrict__ num_nodes, int32_t* __restrict__ tokens,
                   int32_t* __restrict__ parent, int32_t* __restrict__ depth,
                   int32_t* __restrict__ gamma, uint32_t* __restrict__ mask, uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   extern __shared__ int sm[];
   __shared__ int scratch[32];
   __shared__ int sv[3];
@@ -322,9 +328,9 @@ sense_status launch_gather(const int32_t* spans, int64_t n, int m, const int32_t
                            int32_t* out_spans, uint32_t* status, cudaStream_t s) {
   const int threads = ((k + 31) / 32) * 32;
   LaunchScope ls(K_GATHER, s);
-  gather_kernel<<<q, threads, 0, s>>>(spans, n, m, idx, k, anchor, n_keep, force, out_spans,
-                                      status);
-  return cuda_check(cudaGetLastError(), "launch gather");
+  return cuda_check(launch_pdl(gather_kernel, dim3(q), dim3(threads), 0, s, spans, n, m, idx, k,
+                              anchor, n_keep, force, out_spans, status),
+                    "launch gather");
 }
 
 size_t tree_smem_bytes(int k, int m) {
@@ -343,10 +349,10 @@ sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int
         tree_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(tree_small)");
     LaunchScope ls(K_TREE, s);
-    tree_small_kernel<<<q, kTreeSmallThreads, smem, s>>>(spans, k, m, cap, words, num_nodes,
-                                                          tokens, parent, depth, gamma,
-                                                          mask_bits ? mask : nullptr, status);
-    return cuda_check(cudaGetLastError(), "launch tree_small");
+    return cuda_check(launch_pdl(tree_small_kernel, dim3(q), dim3(kTreeSmallThreads), smem, s,
+                                 spans, k, m, cap, words, num_nodes, tokens, parent, depth, gamma,
+                                 mask_bits ? mask : nullptr, status),
+                      "launch tree_small");
   }
   const size_t smem = tree_smem_bytes(k, m);
   cudaError_t e = cudaFuncSetAttribute(tree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -357,9 +363,10 @@ sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int
   // block barriers of a small tree cheaper
   int threads = 128;
   while (threads < k) threads <<= 1;
-  tree_kernel<<<q, threads, smem, s>>>(spans, k, m, cap, words, num_nodes, tokens, parent,
-                                            depth, gamma, mask_bits ? mask : nullptr, status);
-  return cuda_check(cudaGetLastError(), "launch tree");
+  return cuda_check(launch_pdl(tree_kernel, dim3(q), dim3(threads), smem, s, spans, k, m, cap,
+                              words, num_nodes, tokens, parent, depth, gamma,
+                              mask_bits ? mask : nullptr, status),
+                    "launch tree");
 }
 
 sense_status launch_tree_mask_full(const uint32_t* mask_bits, const int32_t* num_nodes,

@@ -114,6 +114,8 @@ template <bool NORM>
 __global__ void __launch_bounds__(256)
 project_bulk_kernel(const uint16_t* __restrict__ x, int d, const float* __restrict__ w, int v,
                     const float* __restrict__ mu, float* __restrict__ out, uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   extern __shared__ __align__(128) uint8_t smb[];
   __shared__ __align__(8) uint64_t bar;
   __shared__ float s_out[8];
@@ -214,6 +216,8 @@ __global__ void __launch_bounds__(256)
 project_rows_kernel(const uint16_t* __restrict__ x, int64_t n, int d,
                     const float* __restrict__ w, int v, const float* __restrict__ mu,
                     float* __restrict__ out) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   extern __shared__ __align__(16) float sx[];  // [d]
   const int64_t row = blockIdx.y;
   const int lane = threadIdx.x & 31;
@@ -263,6 +267,8 @@ __global__ void __launch_bounds__(512)
 project_tile_kernel(const uint16_t* __restrict__ x, int64_t n, int d,
                     const float* __restrict__ w, int v, const float* __restrict__ mu,
                     float* __restrict__ out) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   __shared__ __align__(16) float xs[kPtRows][kPtCols];
   __shared__ __align__(16) float ws[kPtOuts][kPtCols];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -334,6 +340,8 @@ project_tile_kernel(const uint16_t* __restrict__ x, int64_t n, int d,
 // sum of squares in index order from shuffled values, then scales its part.
 __global__ void __launch_bounds__(256)
 normalize_rows_kernel(float* __restrict__ y, int64_t n, int v) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   const int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (i >= n) return;  // warp-uniform
@@ -368,6 +376,8 @@ template <int D, int MODE, bool VEC>
 __global__ void __launch_bounds__(128)
 assign_kernel(const float* __restrict__ x, int64_t n, int ld, const float* __restrict__ c,
               int k, int32_t* __restrict__ out_assign, uint64_t* __restrict__ pool) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   constexpr int kTile = (D <= 16) ? 256 : (8192 / D);
   __shared__ __align__(16) float cs[kTile * D];
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -428,12 +438,15 @@ sense_status launch_assign_mode(const float* x, int64_t n, int dim, int ld, cons
                                 int32_t* out_assign, uint64_t* pool, cudaStream_t s) {
   const dim3 grid((unsigned)((n + 127) / 128));
   const bool vec = (reinterpret_cast<uintptr_t>(x) % 16 == 0) && (ld % 4 == 0);
+  cudaError_t e = cudaSuccess;
 #define SENSE_ASSIGN_CASE(DD)                                                               \
   case DD:                                                                                  \
     if (vec)                                                                                \
-      assign_kernel<DD, MODE, true><<<grid, 128, 0, s>>>(x, n, ld, c, k, out_assign, pool); \
+      e = launch_pdl(assign_kernel<DD, MODE, true>, grid, dim3(128), 0, s, x, n, ld, c, k,        \
+                     out_assign, pool);                                                         \
     else                                                                                    \
-      assign_kernel<DD, MODE, false><<<grid, 128, 0, s>>>(x, n, ld, c, k, out_assign, pool); \
+      e = launch_pdl(assign_kernel<DD, MODE, false>, grid, dim3(128), 0, s, x, n, ld, c, k,       \
+                     out_assign, pool);                                                         \
     break;
   switch (dim) {
     SENSE_ASSIGN_CASE(4)
@@ -446,7 +459,7 @@ sense_status launch_assign_mode(const float* x, int64_t n, int dim, int ld, cons
       return fail(SENSE_ERR_UNSUPPORTED, "dimension %d not in {4, 8, 16, 32, 64, 128}", dim);
   }
 #undef SENSE_ASSIGN_CASE
-  return cuda_check(cudaGetLastError(), "launch assign");
+  return cuda_check(e, "launch assign");
 }
 
 // ---------------------------------------------------------------------------
@@ -671,6 +684,8 @@ __global__ void residual_kernel(const float* __restrict__ x, int64_t n, int v,
 __global__ void __launch_bounds__(256)
 pq_lut_kernel(const float* __restrict__ queries, int v, const float* __restrict__ cb, int pq_m,
               int dsub, float* __restrict__ lut) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   __shared__ float sq[128];
   const int m = blockIdx.x, qi = blockIdx.y;
   for (int j = threadIdx.x; j < dsub; j += blockDim.x)
@@ -697,6 +712,8 @@ ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries,
                 const float* __restrict__ probe_score, const int32_t* __restrict__ probe_cell,
                 uint64_t* __restrict__ pool, uint32_t* __restrict__ counts, int64_t pool_cap,
                 uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   extern __shared__ __align__(16) float sm[];
   const int p = blockIdx.x, qi = blockIdx.y;
   const int v = ix.v;
@@ -857,13 +874,15 @@ sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float*
     cfg.blockDim = dim3(256);
     cfg.dynamicSmemBytes = bulk_smem;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = fuse ? (unsigned)groups : 1u;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     {
       LaunchScope ls(K_PROJECT, s);
       st = cuda_check(cudaLaunchKernelEx(&cfg, kern, x, (int)d, basis, (int)v, mean, out, status),
@@ -872,25 +891,29 @@ sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float*
     }
     if (fuse || !(flags & SENSE_PROJECT_NORMALIZE)) return SENSE_OK;
     LaunchScope ls(K_PROJECT, s);
-    normalize_rows_kernel<<<(unsigned)((n * 32 + 255) / 256), 256, 0, s>>>(out, n, v);
-    return cuda_check(cudaGetLastError(), "launch normalize rows");
+    return cuda_check(launch_pdl(normalize_rows_kernel, dim3((unsigned)((n * 32 + 255) / 256)),
+                                 dim3(256), 0, s, out, n, v),
+                      "launch normalize rows");
   }
   {
     LaunchScope ls(K_PROJECT, s);
+    cudaError_t e = cudaSuccess;
     if (n * v <= 16384 && n <= 65535 && d <= 12288) {
       const dim3 grid((unsigned)((v + 7) / 8), (unsigned)n);
-      project_rows_kernel<<<grid, 256, (size_t)d * 4, s>>>(x, n, d, basis, v, mean, out);
+      e = launch_pdl(project_rows_kernel, grid, dim3(256), (size_t)d * 4, s, x, n, d, basis, v,
+                     mean, out);
     } else {
       const dim3 grid((unsigned)((n + kPtRows - 1) / kPtRows), (unsigned)((v + kPtOuts - 1) / kPtOuts));
-      project_tile_kernel<<<grid, 512, 0, s>>>(x, n, d, basis, v, mean, out);
+      e = launch_pdl(project_tile_kernel, grid, dim3(512), 0, s, x, n, d, basis, v, mean, out);
     }
-    sense_status st = cuda_check(cudaGetLastError(), "launch project");
+    sense_status st = cuda_check(e, "launch project");
     if (st != SENSE_OK) return st;
   }
   if (flags & SENSE_PROJECT_NORMALIZE) {
     LaunchScope ls(K_PROJECT, s);
-    normalize_rows_kernel<<<(unsigned)((n * 32 + 255) / 256), 256, 0, s>>>(out, n, v);
-    return cuda_check(cudaGetLastError(), "launch normalize rows");
+    return cuda_check(launch_pdl(normalize_rows_kernel, dim3((unsigned)((n * 32 + 255) / 256)),
+                                 dim3(256), 0, s, out, n, v),
+                      "launch normalize rows");
   }
   return SENSE_OK;
 }
@@ -1134,9 +1157,9 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
   }
   if (ix->pq_m > 0) {
     LaunchScope ls(K_IVF_COARSE, s);
-    pq_lut_kernel<<<dim3(ix->pq_m, q), 256, 0, s>>>(queries, ix->v, ix->codebooks, ix->pq_m,
-                                                     ix->dsub, lut);
-    st = cuda_check(cudaGetLastError(), "launch pq lut");
+    st = cuda_check(launch_pdl(pq_lut_kernel, dim3(ix->pq_m, q), dim3(256), 0, s, queries, ix->v,
+                               (const float*)ix->codebooks, ix->pq_m, ix->dsub, lut),
+                    "launch pq lut");
     if (st != SENSE_OK) return st;
   }
   st = launch_merge(coarse, nullptr, ix->nlist, q, nprobe, pscore, pcell, status, s);
@@ -1147,10 +1170,10 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
                                          (int)smem), "smem attribute");
     if (st != SENSE_OK) return st;
     LaunchScope ls(K_IVF_SCAN, s);
-    ivf_scan_kernel<<<dim3(nprobe, q), kScanThreads, smem, s>>>(*ix, queries, lut, nprobe, pscore,
-                                                                pcell, pool, counts, p.pool_cap,
-                                                                status);
-    st = cuda_check(cudaGetLastError(), "launch ivf scan");
+    st = cuda_check(launch_pdl(ivf_scan_kernel, dim3(nprobe, q), dim3(kScanThreads), smem, s, *ix,
+                               queries, (const float*)lut, nprobe, (const float*)pscore,
+                               (const int32_t*)pcell, pool, counts, p.pool_cap, status),
+                    "launch ivf scan");
     if (st != SENSE_OK) return st;
   }
   return launch_merge_short(pool, counts, p.pool_cap, q, k, out_scores, out_idx, status, s);

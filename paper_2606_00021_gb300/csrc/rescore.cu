@@ -47,6 +47,8 @@ rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
                const uint16_t* __restrict__ queries, const int32_t* __restrict__ cand,
                int n_cand, int n2, int k, float* __restrict__ out_scores,
                int32_t* __restrict__ out_idx, uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   namespace cg = cooperative_groups;
   cg::cluster_group cl = cg::this_cluster();
   __shared__ uint64_t s_mine[kRsMaxPer];
@@ -135,13 +137,15 @@ sense_status launch_rescore(const uint16_t* keys, int64_t n, int d, const uint16
   cfg.blockDim = dim3(kRsThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = kRsCtas;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   LaunchScope ls(K_RESCORE, s);
   return cuda_check(cudaLaunchKernelEx(&cfg, rescore_kernel, keys, n, d, queries, cand, n_cand, n2,
                                        k, out_scores, out_idx, status),

@@ -299,6 +299,8 @@ __global__ void __launch_bounds__(kSelThreads, 1)
 merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
              int64_t pool_cap, int k, float* __restrict__ out_scores,
              int32_t* __restrict__ out_idx, uint32_t* status, int pad_short) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   extern __shared__ uint64_t s_keys[];
   __shared__ unsigned hist[256];
   __shared__ Digit dig;
@@ -616,6 +618,8 @@ __global__ void __launch_bounds__(kSelThreads, 1)
 merge_lists_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
                    float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
                    uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
   extern __shared__ uint64_t s_keys[];  // [kSmemKeys]
   merge_lists_block(lists, nlists, k, out_scores, out_idx, status, blockIdx.x, s_keys);
 }
@@ -688,9 +692,10 @@ sense_status launch_merge_lists(const uint64_t* lists, int nlists, int q, int k,
   sense_status st = set_smem(merge_lists_kernel, kSmemKeys * sizeof(uint64_t));
   if (st != SENSE_OK) return st;
   LaunchScope ls(K_MERGE, s);
-  merge_lists_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(
-      lists, nlists, k, out_scores, out_idx, status);
-  return cuda_check(cudaGetLastError(), "launch merge_lists");
+  return cuda_check(launch_pdl(merge_lists_kernel, dim3(q), dim3(kSelThreads),
+                              kSmemKeys * sizeof(uint64_t), s, lists, nlists, k, out_scores,
+                              out_idx, status),
+                    "launch merge_lists");
 }
 
 sense_status launch_draft_fused(const uint64_t* lists, int nlists, int q, int k, float* out_scores,
@@ -729,9 +734,10 @@ sense_status launch_merge(const uint64_t* pool, const uint32_t* counts, int64_t 
   sense_status st = set_smem(merge_kernel, kSmemKeys * sizeof(uint64_t));
   if (st != SENSE_OK) return st;
   LaunchScope ls(K_MERGE, s);
-  merge_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(pool, counts, pool_cap, k,
-                                                                   out_scores, out_idx, status, 0);
-  return cuda_check(cudaGetLastError(), "launch merge");
+  return cuda_check(launch_pdl(merge_kernel, dim3(q), dim3(kSelThreads),
+                              kSmemKeys * sizeof(uint64_t), s, pool, counts, pool_cap, k,
+                              out_scores, out_idx, status, 0),
+                    "launch merge");
 }
 
 sense_status launch_merge_short(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap,
@@ -740,9 +746,10 @@ sense_status launch_merge_short(const uint64_t* pool, const uint32_t* counts, in
   sense_status st = set_smem(merge_kernel, kSmemKeys * sizeof(uint64_t));
   if (st != SENSE_OK) return st;
   LaunchScope ls(K_MERGE, s);
-  merge_kernel<<<q, kSelThreads, kSmemKeys * sizeof(uint64_t), s>>>(pool, counts, pool_cap, k,
-                                                                   out_scores, out_idx, status, 1);
-  return cuda_check(cudaGetLastError(), "launch merge");
+  return cuda_check(launch_pdl(merge_kernel, dim3(q), dim3(kSelThreads),
+                              kSmemKeys * sizeof(uint64_t), s, pool, counts, pool_cap, k,
+                              out_scores, out_idx, status, 1),
+                    "launch merge");
 }
 
 }  // namespace sense
