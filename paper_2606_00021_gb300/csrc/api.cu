@@ -5,6 +5,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <map>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -88,6 +89,18 @@ uint32_t* device_status_word() {
     g_status[dev] = static_cast<uint32_t*>(p);
   }
   return g_status[dev];
+}
+
+cudaError_t func_smem(const void* f, int bytes) {
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, int> done;
+  const int dev = current_device();
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = done.find({f, dev});
+  if (it != done.end() && it->second >= bytes) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done[{f, dev}] = bytes;
+  return e;
 }
 
 int sm_count() {

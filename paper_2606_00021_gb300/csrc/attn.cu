@@ -1118,8 +1118,7 @@ sense_status launch_attn_t(const uint16_t* q, const uint16_t* k_cache, const uin
   a.out = out;
   a.fused = splits <= 8 ? 1 : 0;
   const size_t smem = attn_t_smem_bytes();
-  st = cuda_check(cudaFuncSetAttribute(tree_attn_t_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+  st = cuda_check(func_smem(reinterpret_cast<const void*>(tree_attn_t_kernel), (int)smem),
                   "cudaFuncSetAttribute(tree_attn_t)");
   if (st != SENSE_OK) return st;
   {
@@ -1219,8 +1218,7 @@ sense_status sense_tree_attention(const uint16_t* q, const uint16_t* k_cache,
   a.part_ml = reinterpret_cast<float*>(ws + align256((size_t)heads * splits * 128 * kHd * 4));
   a.status = status;
   const size_t smem = attn_smem_bytes();
-  st = cuda_check(cudaFuncSetAttribute(tree_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem), "cudaFuncSetAttribute(tree_attn)");
+  st = cuda_check(func_smem(reinterpret_cast<const void*>(tree_attn_kernel), (int)smem), "cudaFuncSetAttribute(tree_attn)");
   if (st != SENSE_OK) return st;
   // up to 8 splits per head: the splits form a cluster and combine in place
   a.out = out;

@@ -22,6 +22,10 @@ sense_status cuda_check(cudaError_t e, const char* what);
 uint32_t* device_status_word();
 // Number of SMs of the current device (cached per device).
 int sm_count();
+// cudaFuncSetAttribute(f, MaxDynamicSharedMemorySize, bytes), skipped when
+// a value at least as large was already set for f on the current device
+// (the attribute call costs host time on every launch otherwise).
+cudaError_t func_smem(const void* f, int bytes);
 
 enum KernelId {
   K_NORMALIZE = 0,

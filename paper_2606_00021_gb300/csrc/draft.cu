@@ -345,8 +345,7 @@ sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int
   const int words = (cap + 31) / 32;
   if (k <= kTreeSmallK) {
     const size_t smem = sizeof(int) * ((size_t)3 * k * m + (size_t)5 * k);
-    cudaError_t e = cudaFuncSetAttribute(
-        tree_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = func_smem(reinterpret_cast<const void*>(tree_small_kernel), (int)smem);
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(tree_small)");
     LaunchScope ls(K_TREE, s);
     return cuda_check(launch_pdl(tree_small_kernel, dim3(q), dim3(kTreeSmallThreads), smem, s,
@@ -355,8 +354,7 @@ sense_status launch_tree(const int32_t* spans, int q, int k, int m, int cap, int
                       "launch tree_small");
   }
   const size_t smem = tree_smem_bytes(k, m);
-  cudaError_t e = cudaFuncSetAttribute(tree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+  cudaError_t e = func_smem(reinterpret_cast<const void*>(tree_kernel), (int)smem);
   if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(tree)");
   LaunchScope ls(K_TREE, s);
   // one thread per candidate row at least; fewer threads make the many

@@ -881,7 +881,7 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     else kern = (a.kappa <= 4) ? gate_row_block_kernel<4, 1>
                                : gate_row_block_kernel<SENSE_MAX_KAPPA, 1>;
     st = cuda_check(
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kRingBytes),
+        func_smem(reinterpret_cast<const void*>(kern), (int)kRingBytes),
         "cudaFuncSetAttribute(gate_row_block)");
     if (st != SENSE_OK) return st;
     cudaLaunchConfig_t cfg = {};
@@ -920,7 +920,7 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     auto k16 = gate_rows_kernel<SENSE_MAX_KAPPA>;
     auto kern = (a.kappa <= 4) ? k4 : k16;
     st = cuda_check(
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kRingBytes),
+        func_smem(reinterpret_cast<const void*>(kern), (int)kRingBytes),
         "cudaFuncSetAttribute(gate_rows)");
     if (st != SENSE_OK) return st;
     // persistent: one block of kWarps row-streaming warps per SM; with few
@@ -938,8 +938,7 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
   const int staged = staged_smem <= kDecideStageMax ? 1 : 0;
   const size_t smem = staged ? staged_smem : (size_t)a.k * a.m;
   if (smem > 48 * 1024) {
-    st = cuda_check(cudaFuncSetAttribute(gate_decide_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+    st = cuda_check(func_smem(reinterpret_cast<const void*>(gate_decide_kernel), (int)smem),
                     "cudaFuncSetAttribute(gate_decide)");
     if (st != SENSE_OK) return st;
   }

@@ -866,7 +866,7 @@ sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float*
     void (*kern)(const uint16_t*, int, const float*, int, const float*, float*, uint32_t*) =
         fuse ? project_bulk_kernel<true> : project_bulk_kernel<false>;
     sense_status st = cuda_check(
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bulk_smem),
+        func_smem(reinterpret_cast<const void*>(kern), (int)bulk_smem),
         "cudaFuncSetAttribute(project_bulk)");
     if (st != SENSE_OK) return st;
     cudaLaunchConfig_t cfg = {};
@@ -1054,8 +1054,7 @@ sense_status sense_ivf_build(const float* vecs, int64_t n, int32_t v, const floa
     if (st != SENSE_OK) return cleanup(st);
     const size_t hsm = (size_t)nlist * 4;
     if (hsm > 48 * 1024) {
-      st = cuda_check(cudaFuncSetAttribute(cell_hist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)hsm), "smem attribute");
+      st = cuda_check(func_smem(reinterpret_cast<const void*>(cell_hist_kernel), (int)hsm), "smem attribute");
       if (st != SENSE_OK) return cleanup(st);
     }
     cell_hist_kernel<<<nb, 256, hsm, s>>>(cell, n, nlist, hist);
@@ -1063,16 +1062,14 @@ sense_status sense_ivf_build(const float* vecs, int64_t n, int32_t v, const floa
     cell_offsets_kernel<<<1, 1024, 0, s>>>(ix->offsets, nlist, dmax);
     const size_t psm = (size_t)nlist * 8;
     if (psm > 48 * 1024) {
-      st = cuda_check(cudaFuncSetAttribute(cell_place_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)psm), "smem attribute");
+      st = cuda_check(func_smem(reinterpret_cast<const void*>(cell_place_kernel), (int)psm), "smem attribute");
       if (st != SENSE_OK) return cleanup(st);
     }
     cell_place_kernel<<<nb, 32, psm, s>>>(cell, n, nlist, ix->offsets, base, pos, ix->ids);
     if (codebooks) {
       const size_t csm = (size_t)pq_m * 256 * ix->dsub * 4;
       if (csm > 48 * 1024) {
-        st = cuda_check(cudaFuncSetAttribute(pq_encode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)csm), "smem attribute");
+        st = cuda_check(func_smem(reinterpret_cast<const void*>(pq_encode_kernel), (int)csm), "smem attribute");
         if (st != SENSE_OK) return cleanup(st);
       }
       pq_encode_kernel<<<(unsigned)((n + 31) / 32), 256, csm, s>>>(vecs, n, v, ix->centroids, cell,
@@ -1166,8 +1163,7 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
   if (st != SENSE_OK) return st;
   {
     const size_t smem = scan_smem_bytes(ix);
-    st = cuda_check(cudaFuncSetAttribute(ivf_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem), "smem attribute");
+    st = cuda_check(func_smem(reinterpret_cast<const void*>(ivf_scan_kernel), (int)smem), "smem attribute");
     if (st != SENSE_OK) return st;
     LaunchScope ls(K_IVF_SCAN, s);
     st = cuda_check(launch_pdl(ivf_scan_kernel, dim3(nprobe, q), dim3(kScanThreads), smem, s, *ix,

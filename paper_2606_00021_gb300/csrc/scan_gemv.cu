@@ -217,7 +217,7 @@ sense_status launch_topk_q(const uint16_t* keys, int64_t n, int d, const uint16_
   auto kern = scan_gemv_topk_kernel<Q, KPL, UNROLL>;
   const size_t smem = fused_smem_bytes(Q, d, KPL * 32);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = func_smem(reinterpret_cast<const void*>(kern), (int)smem);
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(scan_gemv_topk)");
   }
   LaunchScope ls(K_SCAN_GEMV, s);
@@ -241,7 +241,7 @@ sense_status launch_q_mode(const uint16_t* keys, int64_t n, int d, const uint16_
   auto kern = scan_gemv_kernel<Q, MODE, UNROLL>;
   const size_t smem = (size_t)Q * d * 2;
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = func_smem(reinterpret_cast<const void*>(kern), (int)smem);
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(scan_gemv)");
   }
   int per_sm = 0;

@@ -399,7 +399,7 @@ sense_status launch_scan_tc(const uint16_t* keys, int64_t n, int d, const uint16
   if (grid > units) grid = units;
   if (grid < 1) grid = 1;
   auto run = [&](auto kern) -> sense_status {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = func_smem(reinterpret_cast<const void*>(kern), (int)smem);
     if (e != cudaSuccess) return cuda_check(e, "cudaFuncSetAttribute(scan_tc)");
     LaunchScope ls(K_SCAN_TC, s);
     kern<<<(unsigned)grid, kThreads, smem, s>>>(tm_keys, tm_q, a);

@@ -653,8 +653,7 @@ draft_fused_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
 
 template <class K>
 sense_status set_smem(K kern, size_t bytes) {
-  return cuda_check(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)bytes),
+  return cuda_check(func_smem(reinterpret_cast<const void*>(kern), (int)bytes),
                     "cudaFuncSetAttribute(select)");
 }
 
