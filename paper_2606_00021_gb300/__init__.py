@@ -40,8 +40,25 @@ def _check(st: int):
 
 def _stream(stream) -> int:
     if stream is None:
+        raw = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+        if raw is not None:
+            return raw(torch.cuda.current_device())
         stream = torch.cuda.current_stream()
     return stream.cuda_stream
+
+
+class Prepared:
+    """A library call whose arguments were marshalled once (device pointers,
+    sizes, the stream).  Calling it issues the call again: the buffers keep
+    their addresses and their contents may change between calls.  Returned by
+    the prepare_* functions for per-step calls whose host-side marshalling
+    would otherwise cost more than the kernels they launch."""
+
+    def __init__(self, fn, args, keep):
+        self._fn, self._args, self._keep = fn, args, keep
+
+    def __call__(self):
+        _check(self._fn(*self._args))
 
 
 def _ptr(t):
@@ -277,11 +294,13 @@ def sense_build_tree(spans: torch.Tensor, node_cap: int = 0, mask_bits: bool = F
 
 
 def sense_draft(ds: Datastore, queries: torch.Tensor, k: int, node_cap: int = 0,
-                mask_bits: bool = False, outs: dict | None = None, workspace=None, stream=None):
+                mask_bits: bool = False, outs: dict | None = None, workspace=None, stream=None,
+                prepare: bool = False):
     """Retrieval, span gather and loose trie of one query batch in one call;
     the results of sense_retrieve_topk, sense_gather_drafts (no anchor) and
     sense_build_tree.  Returns a dict: scores, idx, spans and the tree
-    arrays (num_nodes, tokens, parent, depth, gamma[, mask_bits], cap)."""
+    arrays (num_nodes, tokens, parent, depth, gamma[, mask_bits], cap).
+    With prepare=True nothing runs: returns (Prepared call, dict)."""
     _need(queries, "queries", torch.bfloat16, 2)
     q = queries.shape[0]
     if queries.shape[1] != ds.d:
@@ -303,14 +322,15 @@ def sense_draft(ds: Datastore, queries: torch.Tensor, k: int, node_cap: int = 0,
                                               device=dev))
     if workspace is None:
         workspace = alloc_workspace(sense_retrieve_workspace_bytes(ds, q, k), dev)
-    _check(lib().sense_draft(C.c_void_p(ds.handle), queries.data_ptr(), q, k,
-                             workspace.data_ptr(), workspace.numel(), node_cap,
-                             1 if mask_bits else 0, o["scores"].data_ptr(), o["idx"].data_ptr(),
-                             o["spans"].data_ptr(), o["num_nodes"].data_ptr(),
-                             o["tokens"].data_ptr(), o["parent"].data_ptr(),
-                             o["depth"].data_ptr(), o["gamma"].data_ptr(),
-                             _ptr(o.get("mask_bits")), C.c_void_p(_stream(stream))))
+    args = (C.c_void_p(ds.handle), queries.data_ptr(), q, k, workspace.data_ptr(),
+            workspace.numel(), node_cap, 1 if mask_bits else 0, o["scores"].data_ptr(),
+            o["idx"].data_ptr(), o["spans"].data_ptr(), o["num_nodes"].data_ptr(),
+            o["tokens"].data_ptr(), o["parent"].data_ptr(), o["depth"].data_ptr(),
+            o["gamma"].data_ptr(), _ptr(o.get("mask_bits")), C.c_void_p(_stream(stream)))
     o["cap"] = cap
+    if prepare:
+        return Prepared(lib().sense_draft, args, (ds, queries, workspace, dict(o))), o
+    _check(lib().sense_draft(*args))
     return o
 
 
@@ -454,10 +474,11 @@ def sense_ivf_search_workspace_bytes(ix: IvfIndex, q: int, k: int, nprobe: int) 
 def sense_ann_draft(ix: "IvfIndex", ds: Datastore, queries: torch.Tensor, basis: torch.Tensor,
                     mean: torch.Tensor | None, k: int, nprobe: int, rerank: int = 0,
                     node_cap: int = 0, mask_bits: bool = False, outs: dict | None = None,
-                    workspace=None, stream=None):
+                    workspace=None, stream=None, prepare: bool = False):
     """Projection, IVF search (with optional exact re-scoring of `rerank`
     candidates), span gather and loose trie of one query batch in one call;
-    the results of those calls one by one.  Returns a dict like sense_draft."""
+    the results of those calls one by one.  Returns a dict like sense_draft
+    (with prepare=True: (Prepared call, dict), nothing run)."""
     _need(queries, "queries", torch.bfloat16, 2)
     _need(basis, "basis", torch.float32, 2)
     if mean is not None:
@@ -483,15 +504,17 @@ def sense_ann_draft(ix: "IvfIndex", ds: Datastore, queries: torch.Tensor, basis:
     if workspace is None:
         need = lib().sense_ann_draft_workspace_bytes(C.c_void_p(ix.handle), q, k, nprobe, rerank)
         workspace = alloc_workspace(need, dev)
-    _check(lib().sense_ann_draft(C.c_void_p(ix.handle), C.c_void_p(ds.handle), queries.data_ptr(),
-                                 q, basis.data_ptr(), _ptr(mean), k, nprobe, rerank, node_cap,
-                                 1 if mask_bits else 0, workspace.data_ptr(), workspace.numel(),
-                                 o["scores"].data_ptr(), o["idx"].data_ptr(), o["spans"].data_ptr(),
-                                 o["num_nodes"].data_ptr(), o["tokens"].data_ptr(),
-                                 o["parent"].data_ptr(), o["depth"].data_ptr(),
-                                 o["gamma"].data_ptr(), _ptr(o.get("mask_bits")),
-                                 C.c_void_p(_stream(stream))))
+    args = (C.c_void_p(ix.handle), C.c_void_p(ds.handle), queries.data_ptr(), q,
+            basis.data_ptr(), _ptr(mean), k, nprobe, rerank, node_cap, 1 if mask_bits else 0,
+            workspace.data_ptr(), workspace.numel(), o["scores"].data_ptr(), o["idx"].data_ptr(),
+            o["spans"].data_ptr(), o["num_nodes"].data_ptr(), o["tokens"].data_ptr(),
+            o["parent"].data_ptr(), o["depth"].data_ptr(), o["gamma"].data_ptr(),
+            _ptr(o.get("mask_bits")), C.c_void_p(_stream(stream)))
     o["cap"] = cap
+    if prepare:
+        return Prepared(lib().sense_ann_draft, args,
+                        (ix, ds, queries, basis, mean, workspace, dict(o))), o
+    _check(lib().sense_ann_draft(*args))
     return o
 
 
@@ -662,8 +685,10 @@ def sense_soft_gate(tree: dict, root_logits: torch.Tensor, node_logits: torch.Te
                     root_hidden: torch.Tensor, node_hidden: torch.Tensor, gamma: float = 0.05,
                     topk: int = 3, window: int = 6, tau: int = 0,
                     unnormalized_entropy: bool = False, want_G: bool = False,
-                    workspace=None, outs: dict | None = None, stream=None) -> dict:
-    """Soft-gated evaluation of every draft path; returns a dict of device tensors."""
+                    workspace=None, outs: dict | None = None, stream=None,
+                    prepare: bool = False):
+    """Soft-gated evaluation of every draft path; returns a dict of device
+    tensors (with prepare=True: (Prepared call, dict), nothing run)."""
     for name in ("num_nodes", "tokens", "parent", "gamma"):
         _need(tree[name], name, torch.int32)
     q, k, m = tree["gamma"].shape
@@ -688,14 +713,18 @@ def sense_soft_gate(tree: dict, root_logits: torch.Tensor, node_logits: torch.Te
         workspace = alloc_workspace(sense_soft_gate_workspace_bytes(q, cap, topk), dev)
     p = _abi.GateParams(float(gamma), int(topk), int(window), int(tau),
                         1 if unnormalized_entropy else 0)
-    _check(lib().sense_soft_gate(
-        tree["tokens"].data_ptr(), tree["parent"].data_ptr(), tree["num_nodes"].data_ptr(),
-        tree["gamma"].data_ptr(), q, k, m, cap, root_logits.data_ptr(), node_logits.data_ptr(),
-        vocab, root_hidden.data_ptr(), node_hidden.data_ptr(), d, C.byref(p),
-        o["i_star"].data_ptr(), o["L_star"].data_ptr(), o["n_accept"].data_ptr(),
-        o["accepted"].data_ptr(), o["next_node"].data_ptr(), o["next_anchor"].data_ptr(),
-        o["h_next"].data_ptr(), _ptr(o.get("G")), workspace.data_ptr(), workspace.numel(),
-        C.c_void_p(_stream(stream))))
+    args = (tree["tokens"].data_ptr(), tree["parent"].data_ptr(), tree["num_nodes"].data_ptr(),
+            tree["gamma"].data_ptr(), q, k, m, cap, root_logits.data_ptr(),
+            node_logits.data_ptr(), vocab, root_hidden.data_ptr(), node_hidden.data_ptr(), d,
+            C.byref(p), o["i_star"].data_ptr(), o["L_star"].data_ptr(), o["n_accept"].data_ptr(),
+            o["accepted"].data_ptr(), o["next_node"].data_ptr(), o["next_anchor"].data_ptr(),
+            o["h_next"].data_ptr(), _ptr(o.get("G")), workspace.data_ptr(), workspace.numel(),
+            C.c_void_p(_stream(stream)))
+    if prepare:
+        return Prepared(lib().sense_soft_gate, args,
+                        (dict(tree), root_logits, node_logits, root_hidden, node_hidden, p,
+                         workspace, dict(o))), o
+    _check(lib().sense_soft_gate(*args))
     return o
 
 

@@ -423,3 +423,34 @@ def test_draft_equals_separate_calls(S, n, d, m, q, k, cap, with_bits):
     full = O.scores(bits(keys), bits(qs))
     for qi in range(q):
         check_topk(host(got["scores"][qi]), host(got["idx"][qi]), full[qi], k)
+
+
+@cuda
+def test_prepared_calls_follow_buffer_contents(S):
+    """A prepared call reissues the same call on the same buffers: after the
+    query buffer's contents change, it gives what a fresh call gives."""
+    dev = torch.device("cuda")
+    n, d, m, q, k, cap, v = 30000, 512, 8, 1, 16, 32, 1000
+    keys = synth.clustered_unit_keys(n, d, 64, seed=41, device=dev)
+    spans = synth.spans_uniform(n, m, 6, seed=42, device=dev)
+    ds = S.sense_datastore_build(keys, spans)
+    qbuf = torch.empty(q, d, dtype=torch.bfloat16, device=dev)
+    call, outs = S.sense_draft(ds, qbuf, k, node_cap=cap, prepare=True)
+    root = synth.gate_logits(q, 1, v, seed=3, device=dev)[:, 0].contiguous()
+    nodes = synth.gate_logits(q, cap, v, seed=4, device=dev)
+    hr = synth.gate_hidden(q, 1, d, seed=3, device=dev)[:, 0].contiguous()
+    hn = synth.gate_hidden(q, cap, d, seed=4, device=dev)
+    gcall, gouts = S.sense_soft_gate(outs, root, nodes, hr, hn, prepare=True)
+    for seed in (5, 6, 7):
+        qs, _ = synth.noisy_queries(keys, q, seed=seed)
+        qbuf.copy_(qs)
+        call()
+        gcall()
+        want = S.sense_draft(ds, qs, k, node_cap=cap)
+        wg = S.sense_soft_gate(want, root, nodes, hr, hn)
+        torch.cuda.synchronize()
+        assert S.sense_device_status(clear=True) == 0
+        for key in ("scores", "idx", "spans", "num_nodes", "tokens", "parent", "gamma"):
+            assert torch.equal(outs[key], want[key]), key
+        for key in ("i_star", "L_star", "next_node", "next_anchor", "accepted", "h_next"):
+            assert torch.equal(gouts[key], wg[key]), key
