@@ -656,9 +656,21 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     ptx::mbar_init(bar(MMA_DONE), 1);
     sh->abort = 0;
     ptx::fence_barrier_init();
-    ptx::prefetch_tensormap(&tm_q);
-    ptx::prefetch_tensormap(&tm_k);
-    ptx::prefetch_tensormap(&tm_vt);
+    if (nbl > 0) {  // Q and the first K and V^T tiles go out before the block barrier
+      const uint64_t pol_stream = ptx::policy_evict_first();
+      const uint64_t pol_keep = ptx::policy_evict_last();
+      const int key0 = j0 * kTB;
+      ptx::mbar_arrive_expect_tx(bar(Q_FULL), kTQBytes);
+      ptx::tma_load_3d(ptx::smem_u32(s_q), &tm_q, bar(Q_FULL), 0, 0, h, pol_keep);
+      ptx::tma_load_3d(ptx::smem_u32(s_q + kTSlabQ), &tm_q, bar(Q_FULL), 64, 0, h, pol_keep);
+      ptx::mbar_arrive_expect_tx(bar(K_FULL), kTKBytes);
+      ptx::tma_load_3d(ptx::smem_u32(s_k), &tm_k, bar(K_FULL), 0, key0, h, pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(s_k + kTSlab), &tm_k, bar(K_FULL), 64, key0, h, pol_stream);
+      ptx::mbar_arrive_expect_tx(bar(V_FULL), kTVBytes);
+      ptx::tma_load_3d(ptx::smem_u32(s_v), &tm_vt, bar(V_FULL), key0, 0, h, pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(s_v + kTSlab), &tm_vt, bar(V_FULL), key0 + 64, 0, h,
+                       pol_stream);
+    }
   }
   if (warp == 1) ptx::tmem_alloc(ptx::smem_u32(&sh->tmem_base), 256);
   ptx::tc_fence_before();
@@ -672,11 +684,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     // the slot tests do not block (test_wait), so a late V^T slot does not
     // hold back the next K tile or the other way round.
     const uint64_t pol_stream = ptx::policy_evict_first();
-    const uint64_t pol_keep = ptx::policy_evict_last();
-    ptx::mbar_arrive_expect_tx(bar(Q_FULL), kTQBytes);
-    ptx::tma_load_3d(ptx::smem_u32(s_q), &tm_q, bar(Q_FULL), 0, 0, h, pol_keep);
-    ptx::tma_load_3d(ptx::smem_u32(s_q + kTSlabQ), &tm_q, bar(Q_FULL), 64, 0, h, pol_keep);
-    int jk = 0, jv = 0;
+    int jk = 1, jv = 1;  // block 0's tiles and Q were issued with the barriers
     long long t0 = clock64();
     while ((jk < nbl || jv < nbl) && !*abort) {
       bool moved = false;
