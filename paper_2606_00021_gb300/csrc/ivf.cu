@@ -373,14 +373,13 @@ normalize_rows_kernel(float* __restrict__ y, int64_t n, int v) {
 //  ARGMIN_L2: out_assign[i] = arg min_c ||x_i - c||^2 (first minimum)
 //  ALL_IP:    x = cells, c = queries: pool[c * n + i] = key(<x_i, c>, i)
 template <int D, int MODE, bool VEC>
-__global__ void __launch_bounds__(128)
-assign_kernel(const float* __restrict__ x, int64_t n, int ld, const float* __restrict__ c,
-              int k, int32_t* __restrict__ out_assign, uint64_t* __restrict__ pool) {
-  pdl_wait();  // inputs written by the kernels before this one
-  pdl_launch_dependents();
+__device__ __forceinline__ void assign_block(const float* __restrict__ x, int64_t n, int ld,
+                                             const float* __restrict__ c, int k,
+                                             int32_t* __restrict__ out_assign,
+                                             uint64_t* __restrict__ pool, int block) {
   constexpr int kTile = (D <= 16) ? 256 : (8192 / D);
   __shared__ __align__(16) float cs[kTile * D];
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t i = (int64_t)block * blockDim.x + threadIdx.x;
   const bool live = i < n;
   float xr[D];
   if (VEC) {  // 16-byte row loads (x 16-byte aligned, ld % 4 == 0)
@@ -431,6 +430,70 @@ assign_kernel(const float* __restrict__ x, int64_t n, int ld, const float* __res
     }
   }
   if (MODE != ALL_IP && live) out_assign[i] = arg;
+}
+
+template <int D, int MODE, bool VEC>
+__global__ void __launch_bounds__(128)
+assign_kernel(const float* __restrict__ x, int64_t n, int ld, const float* __restrict__ c,
+              int k, int32_t* __restrict__ out_assign, uint64_t* __restrict__ pool) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
+  assign_block<D, MODE, VEC>(x, n, ld, c, k, out_assign, pool, blockIdx.x);
+}
+
+// The query-side work of an IVF-PQ search in one launch: blocks [0, nbc)
+// write the coarse keys of 128 cells each for every query (the ALL_IP
+// assignment above), the following pq_m x q blocks the lookup table
+// LUT[qi][m][b] = <q_m, B_m[b]> of one sub-quantizer and query (fp32 sums
+// over the sub-vector's coordinates in order).
+template <int D>
+__global__ void __launch_bounds__(128)
+coarse_lut_kernel(const float* __restrict__ cells, int64_t nlist, const float* __restrict__ queries,
+                  int q, uint64_t* __restrict__ coarse, const float* __restrict__ cb, int pq_m,
+                  int dsub, float* __restrict__ lut, int nbc) {
+  pdl_wait();  // the projected queries are complete
+  pdl_launch_dependents();
+  if ((int)blockIdx.x < nbc) {
+    assign_block<D, ALL_IP, true>(cells, nlist, D, queries, q, nullptr, coarse, blockIdx.x);
+    return;
+  }
+  __shared__ float sq[128];
+  const int b = (int)blockIdx.x - nbc;
+  const int m = b % pq_m, qi = b / pq_m;
+  for (int j = threadIdx.x; j < dsub; j += blockDim.x) sq[j] = queries[(int64_t)qi * D + m * dsub + j];
+  __syncthreads();
+  for (int w = threadIdx.x; w < 256; w += blockDim.x) {
+    const int e = m * 256 + w;
+    const float* bb = cb + (int64_t)e * dsub;
+    float s = 0.0f;
+    for (int j = 0; j < dsub; ++j) s = madd(s, sq[j], bb[j]);
+    lut[(int64_t)qi * pq_m * 256 + e] = s;
+  }
+}
+
+sense_status launch_coarse_lut(const sense_ivf* ix, const float* queries, int q, uint64_t* coarse,
+                               float* lut, cudaStream_t s) {
+  const int nbc = (ix->nlist + 127) / 128;
+  const dim3 grid((unsigned)(nbc + ix->pq_m * q));
+  cudaError_t e = cudaSuccess;
+#define SENSE_COARSE_LUT_CASE(DD)                                                            \
+  case DD:                                                                                  \
+    e = launch_pdl(coarse_lut_kernel<DD>, grid, dim3(128), 0, s, (const float*)ix->centroids,  \
+                   (int64_t)ix->nlist, queries, q, coarse, (const float*)ix->codebooks,       \
+                   ix->pq_m, ix->dsub, lut, nbc);                                             \
+    break;
+  switch (ix->v) {
+    SENSE_COARSE_LUT_CASE(4)
+    SENSE_COARSE_LUT_CASE(8)
+    SENSE_COARSE_LUT_CASE(16)
+    SENSE_COARSE_LUT_CASE(32)
+    SENSE_COARSE_LUT_CASE(64)
+    SENSE_COARSE_LUT_CASE(128)
+    default:
+      return fail(SENSE_ERR_UNSUPPORTED, "dimension %d not in {4, 8, 16, 32, 64, 128}", ix->v);
+  }
+#undef SENSE_COARSE_LUT_CASE
+  return cuda_check(e, "launch coarse + lut");
 }
 
 template <int MODE>
@@ -681,23 +744,6 @@ __global__ void residual_kernel(const float* __restrict__ x, int64_t n, int v,
 // PQ lookup table of each query: lut[qi][m][b] = <q_m, B_m[b]> (dsub terms in
 // index order).  One block per (sub-quantizer m, query), one thread per
 // codeword b: every codeword row is loaded at once (one round trip).
-__global__ void __launch_bounds__(256)
-pq_lut_kernel(const float* __restrict__ queries, int v, const float* __restrict__ cb, int pq_m,
-              int dsub, float* __restrict__ lut) {
-  pdl_wait();  // inputs written by the kernels before this one
-  pdl_launch_dependents();
-  __shared__ float sq[128];
-  const int m = blockIdx.x, qi = blockIdx.y;
-  for (int j = threadIdx.x; j < dsub; j += blockDim.x)
-    sq[j] = queries[(int64_t)qi * v + m * dsub + j];
-  __syncthreads();
-  const int e = m * 256 + threadIdx.x;  // blockDim.x == 256 codewords
-  const float* bb = cb + (int64_t)e * dsub;
-  float s = 0.0f;
-  for (int j = 0; j < dsub; ++j) s = madd(s, sq[j], bb[j]);
-  lut[(int64_t)qi * pq_m * 256 + e] = s;
-}
-
 constexpr int kScanThreads = 256;
 constexpr int kFlatStride = 132;  // padded row stride (floats) of staged vectors, v <= 128
 
@@ -1115,12 +1161,18 @@ size_t sense_ivf_search_workspace_bytes(const sense_ivf* ix, int32_t q, int32_t 
   return search_plan(ix, q, nprobe).total;
 }
 
-sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t q, int32_t k,
-                              int32_t nprobe, float* out_scores, int32_t* out_idx,
-                              int32_t* out_probes, void* workspace, size_t workspace_bytes,
-                              sense_stream_t stream) {
+}  // extern "C"
+
+namespace {
+// Validation, coarse scores, probe selection, PQ tables and the list scan of
+// a search: each query's scanned candidates are left in the workspace's
+// pool (`*pool`, `*counts`, `*pool_cap` keys per query).
+sense_status ivf_scan_pool(const sense_ivf* ix, const float* queries, int32_t q, int32_t k,
+                           int32_t nprobe, int32_t* out_probes, void* workspace,
+                           size_t workspace_bytes, cudaStream_t s, uint64_t** pool_out,
+                           uint32_t** counts_out, int64_t* pool_cap_out, uint32_t** status_out) {
   if (!ix) return fail(SENSE_ERR_INVALID_ARG, "ix is NULL");
-  if (!queries || !out_scores || !out_idx || !workspace)
+  if (!queries || !workspace)
     return fail(SENSE_ERR_INVALID_ARG, "queries, outputs and workspace must be non-NULL");
   if (q < 1 || q > 65535) return fail(SENSE_ERR_INVALID_ARG, "q=%d outside [1, 65535]", q);
   if (k < 1 || k > SENSE_MAX_K) return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, %d]", k, SENSE_MAX_K);
@@ -1135,7 +1187,6 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
   if (current_device() != ix->device) return fail(SENSE_ERR_INVALID_ARG, "index lives on device %d", ix->device);
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   char* ws = static_cast<char*>(workspace);
   auto* coarse = reinterpret_cast<uint64_t*>(ws + p.off_coarse);
   auto* pscore = reinterpret_cast<float*>(ws + p.off_pscore);
@@ -1145,18 +1196,15 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
   auto* lut = reinterpret_cast<float*>(ws + p.off_lut);
   sense_status st = cuda_check(cudaMemsetAsync(counts, 0, (size_t)q * 4, s), "clear counts");
   if (st != SENSE_OK) return st;
-  {
+  if (ix->pq_m > 0) {  // coarse keys and lookup tables in one launch
+    LaunchScope ls(K_IVF_COARSE, s);
+    st = launch_coarse_lut(ix, queries, q, coarse, lut, s);
+    if (st != SENSE_OK) return st;
+  } else {
     LaunchScope ls(K_IVF_COARSE, s);
     // cells as rows, queries staged: pool row qi holds key(<q_qi, c>, c)
     st = launch_assign_mode<ALL_IP>(ix->centroids, ix->nlist, ix->v, ix->v, queries, q, nullptr,
                                     coarse, s);
-    if (st != SENSE_OK) return st;
-  }
-  if (ix->pq_m > 0) {
-    LaunchScope ls(K_IVF_COARSE, s);
-    st = cuda_check(launch_pdl(pq_lut_kernel, dim3(ix->pq_m, q), dim3(256), 0, s, queries, ix->v,
-                               (const float*)ix->codebooks, ix->pq_m, ix->dsub, lut),
-                    "launch pq lut");
     if (st != SENSE_OK) return st;
   }
   st = launch_merge(coarse, nullptr, ix->nlist, q, nprobe, pscore, pcell, status, s);
@@ -1172,7 +1220,32 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
                     "launch ivf scan");
     if (st != SENSE_OK) return st;
   }
-  return launch_merge_short(pool, counts, p.pool_cap, q, k, out_scores, out_idx, status, s);
+  *pool_out = pool;
+  *counts_out = counts;
+  *pool_cap_out = p.pool_cap;
+  *status_out = status;
+  return SENSE_OK;
+}
+}  // namespace
+
+extern "C" {
+
+sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t q, int32_t k,
+                              int32_t nprobe, float* out_scores, int32_t* out_idx,
+                              int32_t* out_probes, void* workspace, size_t workspace_bytes,
+                              sense_stream_t stream) {
+  if (!ix) return fail(SENSE_ERR_INVALID_ARG, "ix is NULL");
+  if (!queries || !out_scores || !out_idx || !workspace)
+    return fail(SENSE_ERR_INVALID_ARG, "queries, outputs and workspace must be non-NULL");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint64_t* pool = nullptr;
+  uint32_t* counts = nullptr;
+  uint32_t* status = nullptr;
+  int64_t pool_cap = 0;
+  sense_status st = ivf_scan_pool(ix, queries, q, k, nprobe, out_probes, workspace,
+                                  workspace_bytes, s, &pool, &counts, &pool_cap, &status);
+  if (st != SENSE_OK) return st;
+  return launch_merge_short(pool, counts, pool_cap, q, k, out_scores, out_idx, status, s);
 }
 
 size_t sense_ann_draft_workspace_bytes(const sense_ivf* ix, int32_t q, int32_t k, int32_t nprobe,
@@ -1227,11 +1300,26 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
     ws += align256((size_t)q * kk * 4);
   }
   const size_t ivf_bytes = sense_ivf_search_workspace_bytes(ix, q, kk, nprobe);
+  const int cap = node_cap > 0 ? node_cap : k * m;
+  const bool fused = draft_fused_fits(k, m);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   // query construction (Alg. 2: k = L2Norm(PCA(h))), search, optional
   // exact re-scoring (Eq. 8), gather and trie
   sense_status st = sense_project(queries, q, ds->d, basis, ix->v, mean, SENSE_PROJECT_NORMALIZE,
                                   qproj, stream);
   if (st != SENSE_OK) return st;
+  if (rerank == 0 && fused) {  // pool merge, gather and trie in one kernel per query
+    uint64_t* pool = nullptr;
+    uint32_t* counts = nullptr;
+    uint32_t* status = nullptr;
+    int64_t pool_cap = 0;
+    st = ivf_scan_pool(ix, qproj, q, k, nprobe, nullptr, ws, ivf_bytes, s, &pool, &counts,
+                       &pool_cap, &status);
+    if (st != SENSE_OK) return st;
+    return launch_pool_draft(pool, counts, pool_cap, q, k, out_scores, out_idx, ds->spans, ds->n,
+                             m, out_spans, cap, bits ? 1 : 0, out_num_nodes, out_tokens,
+                             out_parent, out_depth, out_gamma, out_mask_bits, status, s);
+  }
   if (rerank > 0) {
     st = sense_ivf_search(ix, qproj, q, rerank, nprobe, cand_s, cand_i, nullptr, ws, ivf_bytes,
                           stream);
@@ -1244,7 +1332,10 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
   if (st != SENSE_OK) return st;
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
-  const int cap = node_cap > 0 ? node_cap : k * m;
+  if (fused)  // gather and trie in one kernel per query
+    return launch_span_draft(out_idx, q, k, ds->spans, ds->n, m, out_spans, cap, bits ? 1 : 0,
+                             out_num_nodes, out_tokens, out_parent, out_depth, out_gamma,
+                             out_mask_bits, status, s);
   st = launch_gather(ds->spans, ds->n, m, out_idx, q, k, nullptr, k, 0, out_spans, status, stream);
   if (st != SENSE_OK) return st;
   return launch_tree(out_spans, q, k, m, cap, bits ? 1 : 0, out_num_nodes, out_tokens, out_parent,

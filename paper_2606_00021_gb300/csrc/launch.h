@@ -95,6 +95,22 @@ sense_status launch_draft_fused(const uint64_t* lists, int nlists, int q, int k,
                                 int32_t* out_spans, int cap, int mask_bits, int32_t* num_nodes,
                                 int32_t* tokens, int32_t* parent, int32_t* depth, int32_t* gamma,
                                 uint32_t* mask, uint32_t* status, cudaStream_t s);
+// The approximate drafting tail fused in one kernel per query: the top k
+// of the list scan's pool (short pools padded, as launch_merge_short), span
+// gather, small-tree trie (draft_fused_fits(k, m)).
+sense_status launch_pool_draft(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap,
+                               int q, int k, float* out_scores, int32_t* out_idx,
+                               const int32_t* spans, int64_t n, int m, int32_t* out_spans, int cap,
+                               int mask_bits, int32_t* num_nodes, int32_t* tokens,
+                               int32_t* parent, int32_t* depth, int32_t* gamma, uint32_t* mask,
+                               uint32_t* status, cudaStream_t s);
+// Span gather of k key indices per query and the small-tree trie fused in
+// one kernel per query (draft_fused_fits(k, m)).
+sense_status launch_span_draft(const int32_t* idx, int q, int k, const int32_t* spans, int64_t n,
+                               int m, int32_t* out_spans, int cap, int mask_bits,
+                               int32_t* num_nodes, int32_t* tokens, int32_t* parent,
+                               int32_t* depth, int32_t* gamma, uint32_t* mask, uint32_t* status,
+                               cudaStream_t s);
 // Exact scores of a shortlist of n_cand key indices per query (-1 = empty),
 // top k by (score desc, index asc).
 sense_status launch_rescore(const uint16_t* keys, int64_t n, int d, const uint16_t* queries, int q,

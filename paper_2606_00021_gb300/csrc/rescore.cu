@@ -7,28 +7,55 @@
 // same arithmetic as the exact scan) and selects the top k of the shortlist
 // in the order (score desc, key index asc).
 //
-// A query's shortlist is a gather of N' scattered key rows (2 MB for 256
-// rows of 4096 dims), so one query is spread over a cluster of kRsCtas CTAs:
-// CTA r scores every kRsCtas-th candidate, one warp per candidate with the
-// whole row's 16-byte loads of a lane issued together (the query stays in
-// L1), and keeps the candidate keys (score code, inverted index) in its
-// shared memory.  CTA 0 then gathers the cluster's keys through distributed
-// shared memory, sorts them with a block bitonic network and writes the top
-// k.  Slots with index -1 (fewer candidates than N') are empty; an index
-// outside [0, n) is empty too and sets SENSE_DEVST_BAD_INDEX.
+// A query's shortlist is a gather of N' scattered key rows (4 MB for 512
+// rows of 4096 dims), paced by how many bytes are in flight, so one query is
+// spread over a cluster of C CTAs (16 where the device schedules clusters
+// that wide, else 8) and each CTA keeps 24 rows in flight:
+//  1. CTA r takes the candidates [r * per, (r + 1) * per), per =
+//     ceil(N' / C); warp w of the CTA takes every 8th of them.  Lane 0 of
+//     the warp streams its candidates' rows through a 3-stage ring of
+//     8 KB shared-memory stages with 1-D bulk copies (cp.async.bulk,
+//     completion on an mbarrier, every wait bounded); a row longer than a
+//     stage takes several stages.  Lane l accumulates chunks l, l + 32, ...
+//     of 8 bf16 in increasing order, then a butterfly sums the lanes.
+//  2. Warp 0 sorts the CTA's candidate keys (score code, inverted index)
+//     in registers with a bitonic network.
+//  3. After a cluster barrier every CTA copies the C sorted lists through
+//     distributed shared memory, and the rank of each of its own keys is its
+//     position in its list plus, per other list, a binary-search count of
+//     the keys ahead of it; keys ranked below k are written in place.
+// Slots with index -1 (fewer candidates than N') are empty; an index
+// outside [0, n) is empty too and sets SENSE_DEVST_BAD_INDEX.  A copy that
+// never lands sets SENSE_DEVST_TIMEOUT and drops the warp's later
+// candidates.
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "launch.h"
+#include "tc_ptx.cuh"
 
 namespace sense {
 namespace {
 
-constexpr int kRsCtas = 8;       // CTAs per query (one cluster)
-constexpr int kRsThreads = 512;  // 16 warps
-constexpr int kRsMaxPer = (SENSE_MAX_RESCORE + kRsCtas - 1) / kRsCtas;
-constexpr int kRsBatch = 16;     // 16-byte loads in flight per lane
+namespace cg = cooperative_groups;
+
+constexpr int kRsThreads = 256;                  // 8 warps
+constexpr int kRsWarps = kRsThreads / 32;
+constexpr int kRsStage = 8192;                   // bytes per ring stage
+constexpr int kRsChunks = kRsStage / 16;         // 16-byte chunks per stage
+constexpr int kRsLaneChunks = kRsChunks / 32;
+constexpr int kRsDepth = 3;                      // stages per warp ring
+constexpr int kRsListMax = 128;                  // candidates per CTA (N' / C)
+constexpr int kRsWarpMax = kRsListMax / kRsWarps;
+constexpr long long kRsWaitCycles = 4000000000LL;
+
+constexpr size_t kRsRingBytes = (size_t)kRsWarps * kRsDepth * kRsStage;
+constexpr size_t kRsSmemBytes = kRsRingBytes + sizeof(uint64_t) * kRsWarps * kRsDepth +
+                                sizeof(uint64_t) * (kRsListMax + SENSE_MAX_RESCORE) +
+                                sizeof(int32_t) * kRsWarps * kRsWarpMax;
 
 __device__ __forceinline__ float dot8(uint4 kv, uint4 qv, float acc) {
   acc = fmaf(bf_lo(kv.x), bf_lo(qv.x), acc);
@@ -42,87 +69,249 @@ __device__ __forceinline__ float dot8(uint4 kv, uint4 qv, float acc) {
   return acc;
 }
 
-__global__ void __launch_bounds__(kRsThreads)
+// Bounded wait on an mbarrier phase; false after ~2 s.
+__device__ __forceinline__ bool rs_wait(uint32_t bar, uint32_t parity) {
+  if (ptx::mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!ptx::mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > kRsWaitCycles) return false;
+  }
+  return true;
+}
+
+// Bitonic sort, descending, of the 32 * KPL keys a warp holds (element
+// lane + 32 r in x[r]).
+template <int KPL>
+__device__ __forceinline__ void warp_sort_desc(uint64_t (&x)[KPL]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int size = 2; size <= 32 * KPL; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      if (stride >= 32) {  // partner in register r ^ (stride / 32) of the same lane
+        const int rs = stride >> 5;
+#pragma unroll
+        for (int r = 0; r < KPL; ++r) {
+          if (r & rs) continue;
+          const bool desc = (((lane + 32 * r) & size) == 0);
+          const uint64_t a = x[r], b = x[r | rs];
+          const uint64_t hi = a > b ? a : b, lo = a > b ? b : a;
+          x[r] = desc ? hi : lo;
+          x[r | rs] = desc ? lo : hi;
+        }
+      } else {
+        const bool lower = (lane & stride) == 0;
+#pragma unroll
+        for (int r = 0; r < KPL; ++r) {
+          const uint64_t p = __shfl_xor_sync(0xffffffffu, x[r], stride);
+          const bool desc = (((lane + 32 * r) & size) == 0);
+          const bool keep_max = (lower == desc);
+          x[r] = keep_max ? (x[r] > p ? x[r] : p) : (x[r] < p ? x[r] : p);
+        }
+      }
+    }
+  }
+}
+
+template <int KPL>
+__global__ void __launch_bounds__(kRsThreads, 1)
 rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
                const uint16_t* __restrict__ queries, const int32_t* __restrict__ cand,
-               int n_cand, int n2, int k, float* __restrict__ out_scores,
+               int n_cand, int k, float* __restrict__ out_scores,
                int32_t* __restrict__ out_idx, uint32_t* status) {
+  constexpr int L = 32 * KPL;  // sorted-list length per CTA (padded with empty keys)
   pdl_wait();  // inputs written by the kernels before this one
   pdl_launch_dependents();
-  namespace cg = cooperative_groups;
   cg::cluster_group cl = cg::this_cluster();
-  __shared__ uint64_t s_mine[kRsMaxPer];
-  __shared__ uint64_t s_all[SENSE_MAX_RESCORE];
+  extern __shared__ __align__(128) unsigned char rs_smem[];
+  uint4* ring = reinterpret_cast<uint4*>(rs_smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(rs_smem + kRsRingBytes);
+  uint64_t* s_list = bars + kRsWarps * kRsDepth;  // this CTA's keys, then sorted
+  uint64_t* s_all = s_list + kRsListMax;          // the cluster's sorted lists
+  int32_t* s_cidx = reinterpret_cast<int32_t*>(s_all + SENSE_MAX_RESCORE);
+  __shared__ unsigned s_total;
+
+  const int C = (int)cl.num_blocks();
   const int r = (int)cl.block_rank();
   const int qi = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nw = blockDim.x >> 5;
-  const int per = (n_cand + kRsCtas - 1) / kRsCtas;
-  const uint16_t* qrow = queries + (int64_t)qi * d;
-  const int chunks = d >> 3;  // 8 bf16 per 16-byte chunk
-  for (int i = threadIdx.x; i < per; i += blockDim.x) s_mine[i] = 0ull;
+  const int per = (n_cand + C - 1) / C;  // <= L (chosen by the host)
+  const int lo = min(r * per, n_cand);
+  const int cnt = min(per, n_cand - lo);
+  if (threadIdx.x == 0) {
+    for (int b = 0; b < kRsWarps * kRsDepth; ++b) ptx::mbar_init(ptx::smem_u32(bars + b), 1);
+    ptx::fence_barrier_init();
+    s_total = 0u;
+  }
+  for (int i = threadIdx.x; i < kRsListMax; i += blockDim.x) s_list[i] = 0ull;
   __syncthreads();
-  for (int i = warp; i < per; i += nw) {
-    const int c = r + kRsCtas * i;
-    if (c >= n_cand) break;  // warp-uniform
-    const int32_t idx = cand[(int64_t)qi * n_cand + c];
-    if (idx < 0) continue;  // warp-uniform
-    if ((int64_t)idx >= n) {
-      if (lane == 0) raise_status(status, SENSE_DEVST_BAD_INDEX);
-      continue;
-    }
-    const uint16_t* krow = keys + (int64_t)idx * d;
-    float acc = 0.0f;
-    for (int j0 = 0; j0 < chunks; j0 += 32 * kRsBatch) {
-      uint4 kv[kRsBatch];
-#pragma unroll
-      for (int t = 0; t < kRsBatch; ++t) {
-        const int j = j0 + 32 * t + lane;
-        kv[t] = j < chunks ? ld_stream_v4(krow + 8 * j) : make_uint4(0u, 0u, 0u, 0u);
+
+  // 1. score the warp's candidates
+  const int nwc = cnt > warp ? (cnt - warp + kRsWarps - 1) / kRsWarps : 0;  // <= kRsWarpMax
+  int32_t my = -1;  // lane j: key index of the warp's j-th candidate, -1 if empty
+  if (lane < nwc) {
+    const int32_t idx = cand[(int64_t)qi * n_cand + lo + warp + kRsWarps * lane];
+    if ((int64_t)idx >= n) raise_status(status, SENSE_DEVST_BAD_INDEX);
+    else my = idx;  // -1 (or any negative) stays empty
+  }
+  if (my < -1) my = -1;
+  const unsigned valid = __ballot_sync(0xffffffffu, my >= 0);
+  const int nv = __popc(valid);
+  int32_t* wcidx = s_cidx + warp * kRsWarpMax;
+  if (my >= 0) wcidx[__popc(valid & ((1u << lane) - 1u))] = my;
+  __syncwarp();
+  const int rowb = 2 * d;
+  const int spr = (rowb + kRsStage - 1) / kRsStage;  // stages per row
+  const int total = nv * spr;
+  uint64_t* wbars = bars + warp * kRsDepth;
+  uint4* wring = ring + (size_t)warp * kRsDepth * kRsChunks;
+  const uint64_t pol = ptx::policy_evict_first();
+  auto issue = [&](int g) {  // lane 0: stage g of the warp's stream
+    const int v = g / spr, piece = g - v * spr;
+    const int off = piece * kRsStage;
+    const int bytes = min(kRsStage, rowb - off);
+    const uint32_t bar = ptx::smem_u32(wbars + g % kRsDepth);
+    ptx::mbar_arrive_expect_tx(bar, (uint32_t)bytes);
+    ptx::bulk_load(ptx::smem_u32(wring + (size_t)(g % kRsDepth) * kRsChunks),
+                   reinterpret_cast<const char*>(keys + (int64_t)wcidx[v] * d) + off,
+                   (uint32_t)bytes, bar, pol);
+  };
+  if (lane == 0)
+    for (int g = 0; g < min(kRsDepth, total); ++g) issue(g);
+  const uint16_t* qrow = queries + (int64_t)qi * d;
+  float acc = 0.0f;
+  for (int g = 0; g < total; ++g) {
+    const bool got = rs_wait(ptx::smem_u32(wbars + g % kRsDepth), (uint32_t)(g / kRsDepth) & 1u);
+    if (!__all_sync(0xffffffffu, got)) {
+      if (lane == 0) {  // let the copies in flight land before giving up
+        for (int j = g; j < min(total, g + kRsDepth); ++j)
+          rs_wait(ptx::smem_u32(wbars + j % kRsDepth), (uint32_t)(j / kRsDepth) & 1u);
+        raise_status(status, SENSE_DEVST_TIMEOUT);
       }
-#pragma unroll
-      for (int t = 0; t < kRsBatch; ++t) {
-        const int j = j0 + 32 * t + lane;
-        if (j < chunks)
-          acc = dot8(kv[t], __ldg(reinterpret_cast<const uint4*>(qrow + 8 * j)), acc);
-      }
+      break;
     }
+    const int v = g / spr, piece = g - v * spr;
+    const int nc = min(kRsChunks, (rowb - piece * kRsStage) >> 4);
+    const uint4* st = wring + (size_t)(g % kRsDepth) * kRsChunks;
+    const uint4* q4 = reinterpret_cast<const uint4*>(qrow) + piece * kRsChunks;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-    if (lane == 0) s_mine[i] = cand_key(acc, (uint32_t)idx);
+    for (int u = 0; u < kRsLaneChunks; ++u) {
+      const int j = lane + 32 * u;
+      if (j < nc) acc = dot8(st[j], __ldg(q4 + j), acc);
+    }
+    __syncwarp();  // every lane has read the stage: its buffer takes stage g + depth
+    if (lane == 0 && g + kRsDepth < total) {
+      ptx::fence_proxy_async_smem();
+      issue(g + kRsDepth);
+    }
+    if (piece == spr - 1) {
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+      if (lane == 0) s_list[warp + kRsWarps * v] = cand_key(acc, (uint32_t)wcidx[v]);
+      acc = 0.0f;
+    }
+  }
+  __syncthreads();
+
+  // 2. sort this CTA's keys
+  if (warp == 0) {
+    uint64_t x[KPL];
+#pragma unroll
+    for (int i = 0; i < KPL; ++i) x[i] = s_list[lane + 32 * i];
+    warp_sort_desc<KPL>(x);
+#pragma unroll
+    for (int i = 0; i < KPL; ++i) s_list[lane + 32 * i] = x[i];
   }
   cl.sync();
-  if (r == 0) {
-    for (int c = threadIdx.x; c < n2; c += blockDim.x) {
-      uint64_t v = 0ull;
-      if (c < n_cand) v = *cl.map_shared_rank(s_mine + c / kRsCtas, (unsigned)(c % kRsCtas));
-      s_all[c] = v;
+
+  // 3. copy the cluster's lists, rank this CTA's keys among them
+  for (int t = threadIdx.x; t < C * L; t += blockDim.x) {  // C * L: a multiple of blockDim
+    const uint64_t v = *cl.map_shared_rank(s_list + (t % L), (unsigned)(t / L));
+    s_all[t] = v;
+    const unsigned nz = __ballot_sync(0xffffffffu, v != 0ull);
+    if (lane == 0) atomicAdd(&s_total, (unsigned)__popc(nz));
+  }
+  cl.sync();  // no CTA reads another's shared memory after this
+  float* os = out_scores + (int64_t)qi * k;
+  int32_t* oi = out_idx + (int64_t)qi * k;
+  for (int t0 = 0; t0 < L * C; t0 += blockDim.x) {  // L * C is a multiple of blockDim
+    const int t = t0 + threadIdx.x;
+    const int p = t / C, b = t - p * C;
+    const uint64_t x = s_all[r * L + p];
+    int ahead = 0;  // keys of list b ahead of x: larger, or equal in an earlier list
+    if (x != 0ull && b != r) {
+      const uint64_t* lb = s_all + b * L;
+      int a = 0, e = L;
+      while (a < e) {
+        const int mid = (a + e) >> 1;
+        const uint64_t y = lb[mid];
+        if (y > x || (y == x && b < r)) a = mid + 1;
+        else e = mid;
+      }
+      ahead = a;
     }
-    __syncthreads();
-    // bitonic sort of n2 keys, largest first
-    for (int size = 2; size <= n2; size <<= 1) {
-      for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        for (int i = threadIdx.x; i < n2 / 2; i += blockDim.x) {
-          const int lo = 2 * i - (i & (stride - 1));
-          const int hi = lo + stride;
-          const bool desc = ((lo & size) == 0);
-          const uint64_t a = s_all[lo], b = s_all[hi];
-          if ((a < b) == desc) {
-            s_all[lo] = b;
-            s_all[hi] = a;
-          }
-        }
-        __syncthreads();
+    for (int off = C >> 1; off > 0; off >>= 1) ahead += __shfl_xor_sync(0xffffffffu, ahead, off);
+    if (b == 0 && x != 0ull) {
+      const int rank = p + ahead;
+      if (rank < k) {
+        os[rank] = code_score((uint32_t)(x >> 32));
+        oi[rank] = (int32_t)cand_index(x);
       }
     }
+  }
+  if (r == 0) {  // fewer valid candidates than k: -inf, -1
     const float NEG = -__int_as_float(0x7f800000);
-    for (int t = threadIdx.x; t < k; t += blockDim.x) {
-      const uint64_t key = s_all[t];
-      out_scores[(int64_t)qi * k + t] = key ? code_score((uint32_t)(key >> 32)) : NEG;
-      out_idx[(int64_t)qi * k + t] = key ? (int32_t)cand_index(key) : -1;
+    for (int t = (int)s_total + threadIdx.x; t < k; t += blockDim.x) {
+      os[t] = NEG;
+      oi[t] = -1;
     }
   }
-  cl.sync();  // the other CTAs' shared memory stays alive until it is read
+}
+
+using RescoreFn = void (*)(const uint16_t*, int64_t, int, const uint16_t*, const int32_t*, int, int,
+                           float*, int32_t*, uint32_t*);
+constexpr int kMaxDev = 64;
+
+// Cluster width per device: 16 when a cluster of 16 of these CTAs can be
+// resident, else 8 (the portable size).  Attributes are set once.
+sense_status rescore_setup(int dev, int* width) {
+  static std::mutex mu;
+  static int widths[kMaxDev] = {0};
+  std::lock_guard<std::mutex> lk(mu);
+  if (dev >= 0 && dev < kMaxDev && widths[dev] > 0) {
+    *width = widths[dev];
+    return SENSE_OK;
+  }
+  const RescoreFn fns[3] = {rescore_kernel<1>, rescore_kernel<2>, rescore_kernel<4>};
+  for (RescoreFn f : fns) {
+    sense_status st = cuda_check(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      (int)kRsSmemBytes),
+                                 "rescore shared-memory attribute");
+    if (st != SENSE_OK) return st;
+    st = cuda_check(cudaFuncSetAttribute(f, cudaFuncAttributeNonPortableClusterSizeAllowed, 1),
+                    "rescore cluster attribute");
+    if (st != SENSE_OK) return st;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(16, 1);
+  cfg.blockDim = dim3(kRsThreads);
+  cfg.dynamicSmemBytes = kRsSmemBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 16;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int nclusters = 0;
+  int w = 8;
+  if (cudaOccupancyMaxActiveClusters(&nclusters, fns[2], &cfg) == cudaSuccess && nclusters >= 1)
+    w = 16;
+  else
+    (void)cudaGetLastError();  // the query's failure only means "not 16"
+  if (dev >= 0 && dev < kMaxDev) widths[dev] = w;
+  *width = w;
+  return SENSE_OK;
 }
 
 }  // namespace
@@ -130,16 +319,21 @@ rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
 sense_status launch_rescore(const uint16_t* keys, int64_t n, int d, const uint16_t* queries, int q,
                             const int32_t* cand, int n_cand, int k, float* out_scores,
                             int32_t* out_idx, uint32_t* status, cudaStream_t s) {
-  int n2 = 2;
-  while (n2 < n_cand) n2 <<= 1;
+  int C = 8, dev = 0;
+  sense_status st = cuda_check(cudaGetDevice(&dev), "cudaGetDevice");
+  if (st != SENSE_OK) return st;
+  st = rescore_setup(dev, &C);
+  if (st != SENSE_OK) return st;
+  const int per = (n_cand + C - 1) / C;  // <= SENSE_MAX_RESCORE / 8 = kRsListMax
+  const RescoreFn fn = per <= 32 ? rescore_kernel<1> : per <= 64 ? rescore_kernel<2> : rescore_kernel<4>;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(kRsCtas, (unsigned)q);
+  cfg.gridDim = dim3((unsigned)C, (unsigned)q);
   cfg.blockDim = dim3(kRsThreads);
-  cfg.dynamicSmemBytes = 0;
+  cfg.dynamicSmemBytes = kRsSmemBytes;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kRsCtas;
+  attr[0].val.clusterDim.x = (unsigned)C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -147,8 +341,8 @@ sense_status launch_rescore(const uint16_t* keys, int64_t n, int d, const uint16
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   LaunchScope ls(K_RESCORE, s);
-  return cuda_check(cudaLaunchKernelEx(&cfg, rescore_kernel, keys, n, d, queries, cand, n_cand, n2,
-                                       k, out_scores, out_idx, status),
+  return cuda_check(cudaLaunchKernelEx(&cfg, fn, keys, n, d, queries, cand, n_cand, k, out_scores,
+                                       out_idx, status),
                     "launch rescore");
 }
 

@@ -295,18 +295,110 @@ __device__ bool merge_pool_short(const uint64_t* s_keys, int cnt, int k, int pad
   return true;
 }
 
-__global__ void __launch_bounds__(kSelThreads, 1)
-merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
-             int64_t pool_cap, int k, float* __restrict__ out_scores,
-             int32_t* __restrict__ out_idx, uint32_t* status, int pad_short) {
-  pdl_wait();  // inputs written by the kernels before this one
-  pdl_launch_dependents();
-  extern __shared__ uint64_t s_keys[];
+// Selection for pools much longer than k that the group-head bound cannot
+// prune (k above the number of 32-key groups): keys are binned by their
+// score code, (code - min) >> sh with sh chosen so that the range spans at
+// most kBins bins, which keeps bins in code order.  A suffix count of the
+// bin histogram finds the bin B holding the k-th largest key; the keys of
+// bins >= B are scattered bucket by bucket into shared memory, and each
+// key's rank is the count of keys in higher bins plus the larger keys of its
+// own bucket (equal keys ordered by position).  Ranks below k are written,
+// sorted.  Uses the shared memory past the pool: 2 kBins words of counts and
+// cursors, then kBinCap keys.  Returns false (block-uniform) when the
+// selected bins hold more than kBinCap keys (codes bunched in a few bins).
+constexpr int kBins = 2 * kSelThreads;  // two bins per thread in the scan
+constexpr int kBinCap = 4096;
+
+__device__ bool merge_pool_binned(const uint64_t* s_keys, int cnt, int k,
+                                  float* __restrict__ out_scores,
+                                  int32_t* __restrict__ out_idx) {
+  __shared__ uint32_t s_lo, s_hi;
+  __shared__ int s_bin, s_above;
+  __shared__ int scan_scratch[32];
+  uint32_t* count = reinterpret_cast<uint32_t*>(const_cast<uint64_t*>(s_keys) + cnt);  // [kBins]
+  uint32_t* start = count + kBins;                                     // [kBins]
+  uint64_t* buf = reinterpret_cast<uint64_t*>(start + kBins);          // [kBinCap]
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    s_lo = 0xffffffffu;
+    s_hi = 0u;
+    s_bin = -1;
+    s_above = 0;
+  }
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x) count[b] = 0u;
+  __syncthreads();
+  uint32_t lo = 0xffffffffu, hi = 0u;
+  for (int i = threadIdx.x; i < cnt; i += blockDim.x) {
+    const uint32_t c = (uint32_t)(s_keys[i] >> 32);
+    lo = min(lo, c);
+    hi = max(hi, c);
+  }
+  lo = __reduce_min_sync(0xffffffffu, lo);
+  hi = __reduce_max_sync(0xffffffffu, hi);
+  if (lane == 0) {
+    atomicMin(&s_lo, lo);
+    atomicMax(&s_hi, hi);
+  }
+  __syncthreads();
+  const uint32_t clo = s_lo;
+  const uint32_t range = s_hi - clo;  // codes span [clo, clo + range]
+  int sh = 0;
+  while (sh < 32 && (range >> sh) >= (uint32_t)kBins) ++sh;
+  auto bin_of = [&](uint64_t key) { return (int)(((uint32_t)(key >> 32) - clo) >> sh); };
+  for (int i = threadIdx.x; i < cnt; i += blockDim.x) atomicAdd(&count[bin_of(s_keys[i])], 1u);
+  __syncthreads();
+  // thread t holds bins kBins-1-2t and kBins-2-2t: the scan runs from the top bin down
+  const int d0 = kBins - 1 - 2 * (int)threadIdx.x, d1 = d0 - 1;
+  const int c0 = (int)count[d0], c1 = (int)count[d1];
+  int total = 0;
+  const int ex = block_exclusive_scan(c0 + c1, scan_scratch, &total);
+  start[d0] = (uint32_t)ex;
+  start[d1] = (uint32_t)(ex + c0);
+  if (ex < k && k <= ex + c0) {
+    s_bin = d0;
+    s_above = ex;
+  } else if (ex + c0 < k && k <= ex + c0 + c1) {
+    s_bin = d1;
+    s_above = ex + c0;
+  }
+  __syncthreads();
+  const int B = s_bin;
+  if (B < 0 || s_above + (int)count[B] > kBinCap) return false;  // block-uniform
+  for (int i = threadIdx.x; i < cnt; i += blockDim.x) {
+    const uint64_t key = s_keys[i];
+    const int b = bin_of(key);
+    if (b >= B) buf[atomicAdd(&start[b], 1u)] = key;  // start[b] ends at the bucket's end
+  }
+  __syncthreads();
+  const int nsel = s_above + (int)count[B];
+  for (int p = threadIdx.x; p < nsel; p += blockDim.x) {
+    const uint64_t key = buf[p];
+    const int b = bin_of(key);
+    const int e = (int)start[b], s0 = e - (int)count[b];
+    int r = s0;  // keys in higher bins
+    for (int j = s0; j < e; ++j) {
+      const uint64_t o = buf[j];
+      r += (o > key) || (o == key && j < p);
+    }
+    if (r < k) {
+      out_scores[r] = code_score((uint32_t)(key >> 32));
+      out_idx[r] = (int32_t)cand_index(key);
+    }
+  }
+  return true;
+}
+
+// Top k of query q's pool into out_scores / out_idx rows q (one block per
+// query, s_keys: kSmemKeys of shared memory).  Every return is
+// block-uniform, so a caller may continue after a block barrier.
+__device__ void merge_pool_block(const uint64_t* __restrict__ pool,
+                                 const uint32_t* __restrict__ counts, int64_t pool_cap, int k,
+                                 float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
+                                 uint32_t* status, int pad_short, int q, uint64_t* s_keys) {
   __shared__ unsigned hist[256];
   __shared__ Digit dig;
   __shared__ unsigned n_sel;
   __shared__ uint64_t sel[SENSE_MAX_K];
-  const int q = blockIdx.x;
   const uint64_t* src = pool + (int64_t)q * pool_cap;
   int64_t cnt = counts ? (int64_t)counts[q] : pool_cap;  // no counts: every slot is used
   if (cnt > pool_cap) cnt = pool_cap;
@@ -320,6 +412,9 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
       (cnt <= kPoolAll || (cnt + 31) / 32 >= (int64_t)k) &&
       merge_pool_short(s_keys, (int)cnt, k, pad_short, sel, out_scores + (int64_t)q * k,
                        out_idx + (int64_t)q * k))
+    return;
+  if (staged && cnt >= k && cnt + kBins + kBinCap <= kSmemKeys &&
+      merge_pool_binned(s_keys, (int)cnt, k, out_scores + (int64_t)q * k, out_idx + (int64_t)q * k))
     return;
   auto get = [&](int64_t i) { return staged ? s_keys[i] : src[i]; };
   uint64_t prefix, pmask;
@@ -378,6 +473,17 @@ merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ cou
     out_scores[(int64_t)q * k + r] = real ? code_score((uint32_t)(c >> 32)) : -__int_as_float(0x7f800000);
     out_idx[(int64_t)q * k + r] = real ? (int32_t)cand_index(c) : -1;
   }
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1)
+merge_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
+             int64_t pool_cap, int k, float* __restrict__ out_scores,
+             int32_t* __restrict__ out_idx, uint32_t* status, int pad_short) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
+  extern __shared__ uint64_t s_keys[];
+  merge_pool_block(pool, counts, pool_cap, k, out_scores, out_idx, status, pad_short, blockIdx.x,
+                   s_keys);
 }
 
 // Exact top-k of `nlists` lists of k keys per query, each list sorted in
@@ -651,6 +757,52 @@ draft_fused_kernel(const uint64_t* __restrict__ lists, int nlists, int k,
                    mask, status, q, reinterpret_cast<int*>(s_keys), scratch, sv);
 }
 
+// The approximate drafting tail in one block per query: the top k of the
+// list scan's pool (a short pool padded with -inf / -1), the span gather of
+// those keys and the small-tree trie, one after the other, as in
+// draft_fused_kernel.
+__global__ void __launch_bounds__(kSelThreads, 1)
+pool_draft_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
+                  int64_t pool_cap, int k, float* __restrict__ out_scores,
+                  int32_t* __restrict__ out_idx, const int32_t* __restrict__ spans, int64_t n,
+                  int m, int32_t* out_spans, int cap, int mask_words,
+                  int32_t* __restrict__ num_nodes, int32_t* __restrict__ tokens,
+                  int32_t* __restrict__ parent, int32_t* __restrict__ depth,
+                  int32_t* __restrict__ gamma, uint32_t* __restrict__ mask, uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];  // [kSmemKeys]
+  __shared__ int scratch[32];
+  __shared__ int sv[3];
+  const int q = blockIdx.x;
+  pdl_wait();  // the scan's pool is complete
+  pdl_launch_dependents();
+  merge_pool_block(pool, counts, pool_cap, k, out_scores, out_idx, status, 1, q, s_keys);
+  __syncthreads();
+  gather_block(spans, n, m, out_idx, k, nullptr, k, 0, out_spans, status, q, scratch);
+  __syncthreads();
+  tree_small_block(out_spans, k, m, cap, mask_words, num_nodes, tokens, parent, depth, gamma,
+                   mask, status, q, reinterpret_cast<int*>(s_keys), scratch, sv);
+}
+
+// The span gather of k given key indices and the small-tree trie in one
+// block per query (the tail after a shortlist re-scoring).
+__global__ void __launch_bounds__(kSelThreads, 1)
+span_draft_kernel(const int32_t* __restrict__ idx, int k, const int32_t* __restrict__ spans,
+                  int64_t n, int m, int32_t* out_spans, int cap, int mask_words,
+                  int32_t* __restrict__ num_nodes, int32_t* __restrict__ tokens,
+                  int32_t* __restrict__ parent, int32_t* __restrict__ depth,
+                  int32_t* __restrict__ gamma, uint32_t* __restrict__ mask, uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];  // [kSmemKeys], the trie's scratch
+  __shared__ int scratch[32];
+  __shared__ int sv[3];
+  const int q = blockIdx.x;
+  pdl_wait();  // the indices are complete
+  pdl_launch_dependents();
+  gather_block(spans, n, m, idx, k, nullptr, k, 0, out_spans, status, q, scratch);
+  __syncthreads();
+  tree_small_block(out_spans, k, m, cap, mask_words, num_nodes, tokens, parent, depth, gamma,
+                   mask, status, q, reinterpret_cast<int*>(s_keys), scratch, sv);
+}
+
 template <class K>
 sense_status set_smem(K kern, size_t bytes) {
   return cuda_check(func_smem(reinterpret_cast<const void*>(kern), (int)bytes),
@@ -720,6 +872,38 @@ sense_status launch_draft_fused(const uint64_t* lists, int nlists, int q, int k,
                                        num_nodes, tokens, parent, depth, gamma,
                                        mask_bits ? mask : nullptr, status),
                     "launch draft_fused");
+}
+
+sense_status launch_pool_draft(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap,
+                               int q, int k, float* out_scores, int32_t* out_idx,
+                               const int32_t* spans, int64_t n, int m, int32_t* out_spans, int cap,
+                               int mask_bits, int32_t* num_nodes, int32_t* tokens,
+                               int32_t* parent, int32_t* depth, int32_t* gamma, uint32_t* mask,
+                               uint32_t* status, cudaStream_t s) {
+  sense_status st = set_smem(pool_draft_kernel, kSmemKeys * sizeof(uint64_t));
+  if (st != SENSE_OK) return st;
+  LaunchScope ls(K_DRAFT, s);
+  return cuda_check(launch_pdl(pool_draft_kernel, dim3((unsigned)q), dim3(kSelThreads),
+                              kSmemKeys * sizeof(uint64_t), s, pool, counts, pool_cap, k,
+                              out_scores, out_idx, spans, n, m, out_spans, cap, (cap + 31) / 32,
+                              num_nodes, tokens, parent, depth, gamma, mask_bits ? mask : nullptr,
+                              status),
+                    "launch pool_draft");
+}
+
+sense_status launch_span_draft(const int32_t* idx, int q, int k, const int32_t* spans, int64_t n,
+                               int m, int32_t* out_spans, int cap, int mask_bits,
+                               int32_t* num_nodes, int32_t* tokens, int32_t* parent,
+                               int32_t* depth, int32_t* gamma, uint32_t* mask, uint32_t* status,
+                               cudaStream_t s) {
+  sense_status st = set_smem(span_draft_kernel, kSmemKeys * sizeof(uint64_t));
+  if (st != SENSE_OK) return st;
+  LaunchScope ls(K_DRAFT, s);
+  return cuda_check(launch_pdl(span_draft_kernel, dim3((unsigned)q), dim3(kSelThreads),
+                              kSmemKeys * sizeof(uint64_t), s, idx, k, spans, n, m, out_spans, cap,
+                              (cap + 31) / 32, num_nodes, tokens, parent, depth, gamma,
+                              mask_bits ? mask : nullptr, status),
+                    "launch span_draft");
 }
 
 bool draft_fused_fits(int k, int m) {

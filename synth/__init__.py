@@ -137,7 +137,10 @@ def subspace_unit_keys(n: int, d: int, n_clusters: int, rank: int = 256, decay: 
     isotropic noise of norm ~``iso`` (and, with ``return_assign``, the int32
     cluster of each key)."""
     g = _gen(device, _sub_seed(seed, 13))
-    basis = torch.linalg.qr(torch.randn(d, rank, generator=g, device=device))[0]  # [d, rank]
+    # the orthonormal basis is factored on the host in fp64 (no device linear-algebra
+    # library needed; the same basis on every machine up to fp64 rounding)
+    draw = torch.randn(d, rank, generator=g, device=device)
+    basis = torch.linalg.qr(draw.double().cpu())[0].float().to(device)  # [d, rank]
     scale = torch.arange(1, rank + 1, device=device, dtype=torch.float32).pow(-decay)
     scale = scale / scale.norm()
     cz = torch.randn(n_clusters, rank, generator=g, device=device) * scale

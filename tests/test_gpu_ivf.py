@@ -172,8 +172,13 @@ def test_ivf_build_matches_oracle(S, n, v, nlist, pq_m):
 @pytest.mark.parametrize("n,v,nlist,pq_m,q,k,nprobe", [
     (6000, 64, 64, 0, 1, 32, 8), (6000, 64, 64, 16, 7, 100, 8), (6000, 64, 64, 16, 64, 16, 64),
     (9000, 16, 300, 4, 5, 64, 1), (3000, 32, 40, 0, 33, 256, 3), (2000, 64, 16, 16, 3, 500, 2),
+    (20000, 64, 64, 16, 4, 512, 16), (12000, 32, 64, 16, 3, 300, 32), (20000, 64, 64, 0, 2, 1024, 64),
 ])
 def test_ivf_search_matches_oracle(S, n, v, nlist, pq_m, q, k, nprobe):
+    """Probes, indices and scores bit-identical to the oracle's search: the
+    pool merge's short path (k below the number of 32-key groups), its
+    binned path (larger k), the radix path (a pool too long for the binned
+    path's shared memory) and short pools padded with -inf / -1."""
     rng, x, cent, cb = _index_inputs(7 * n + q, n, v, nlist, pq_m)
     qs = _clustered(rng, q, v, 8)
     ix = S.sense_ivf_build(_dev(x), _dev(cent), None if cb is None else _dev(cb))
@@ -277,7 +282,8 @@ def test_projected_pipeline_and_recall(S):
 @cuda
 @pytest.mark.parametrize("n,d,q,n_cand,k,empty", [
     (50000, 512, 5, 300, 32, 0), (20000, 4096, 3, 1024, 64, 100), (9000, 256, 2, 1, 1, 0),
-    (9000, 256, 4, 40, 40, 30), (70000, 8192, 1, 256, 32, 0),
+    (9000, 256, 4, 40, 40, 30), (70000, 8192, 1, 256, 32, 0), (5000, 4104, 2, 600, 50, 20),
+    (8000, 4096, 1, 512, 32, 0), (8000, 4096, 1, 513, 32, 0), (3000, 64, 2, 1000, 999, 5),
 ])
 def test_rescore_matches_oracle(S, n, d, q, n_cand, k, empty):
     """Exact re-scoring of a shortlist: scores within 2e-3 of the oracle's
@@ -307,17 +313,22 @@ def test_rescore_matches_oracle(S, n, d, q, n_cand, k, empty):
 
 
 @cuda
-def test_rescore_lattice_bit_exact_and_bad_index(S):
+@pytest.mark.parametrize("d,n_cand,k,dup", [(512, 500, 100, 0), (512, 1024, 1024, 40),
+                                             (8200, 17, 5, 3), (512, 64, 64, 0)])
+def test_rescore_lattice_bit_exact_and_bad_index(S, d, n_cand, k, dup):
     """Lattice keys and queries: every score is exact in fp32, so scores,
     order and ties (lower key index first) must equal the oracle bit for
-    bit.  An index outside [0, n) is skipped and reported."""
+    bit, at the largest shortlist and with repeated candidates (each copy
+    is scored and kept).  An index outside [0, n) is skipped and reported."""
     dev = torch.device("cuda")
-    n, d, q, n_cand, k = 6000, 512, 3, 500, 100
+    n, q = 6000, 3
     keys = synth.lattice_rows(n, d, seed=7, device=dev)
     qs = synth.lattice_rows(q, d, seed=8, device=dev)
     ds = S.sense_datastore_build(keys, synth.spans_uniform(n, 2, 50, seed=1, device=dev))
     rng = np.random.default_rng(3)
     cand = np.stack([rng.permutation(n)[:n_cand] for _ in range(q)]).astype(np.int32)
+    if dup:
+        cand[:, :dup] = cand[:, n_cand - dup:]
     sc, ix = S.sense_rescore_topk(ds, qs, _dev(cand), k)
     torch.cuda.synchronize()
     assert S.sense_device_status(clear=True) == 0
@@ -338,16 +349,20 @@ def test_rescore_lattice_bit_exact_and_bad_index(S):
 # ---------------------------------------------------------------- approximate drafting step in one call
 
 @cuda
-@pytest.mark.parametrize("pq,rerank,q,k,cap", [
-    (False, 0, 1, 32, 64), (True, 0, 1, 32, 64), (True, 128, 1, 32, 64), (True, 64, 3, 16, 0),
-    (False, 40, 2, 40, 30),
+@pytest.mark.parametrize("pq,rerank,q,k,cap,nlist,nprobe", [
+    (False, 0, 1, 32, 64, 64, 8), (True, 0, 1, 32, 64, 64, 8), (True, 128, 1, 32, 64, 64, 8),
+    (True, 64, 3, 16, 0, 64, 8), (False, 40, 2, 40, 30, 64, 8),
+    (True, 0, 2, 200, 64, 64, 8), (True, 300, 1, 200, 0, 64, 8),
+    (False, 0, 2, 128, 64, 1024, 1), (True, 0, 1, 100, 0, 1024, 1),
 ])
-def test_ann_draft_equals_separate_calls(S, pq, rerank, q, k, cap):
+def test_ann_draft_equals_separate_calls(S, pq, rerank, q, k, cap, nlist, nprobe):
     """sense_ann_draft is bit-identical to projection, IVF search (and the
-    exact re-scoring), gather and trie called one by one."""
+    exact re-scoring), gather and trie called one by one: with the fused
+    tails (k <= 128), without them (k = 200), and with a probed list shorter
+    than k (the pool is padded with -inf / -1)."""
     dev = torch.device("cuda")
     rng = np.random.default_rng(17 + k)
-    n, d, v, nlist = 20000, 512, 32, 64
+    n, d, v = 20000, 512, 32
     keys = synth.clustered_unit_keys(n, d, 32, seed=19, device=dev)
     spans = synth.spans_uniform(n, 8, 5, seed=2, device=dev)
     ds = S.sense_datastore_build(keys, spans)
@@ -364,19 +379,28 @@ def test_ann_draft_equals_separate_calls(S, pq, rerank, q, k, cap):
     ix = S.sense_ivf_build(kp, cent, cb)
     qs, _ = synth.noisy_queries(keys, q, seed=23)
     for _ in range(2):
-        got = S.sense_ann_draft(ix, ds, qs, basis, mean, k, 8, rerank=rerank, node_cap=cap,
+        got = S.sense_ann_draft(ix, ds, qs, basis, mean, k, nprobe, rerank=rerank, node_cap=cap,
                                 mask_bits=True)
+        torch.cuda.synchronize()
+        st_one = S.sense_device_status(clear=True)
         qp = S.sense_project(qs, basis, mean)
         if rerank:
-            _, ci = S.sense_ivf_search(ix, qp, rerank, 8)
+            _, ci = S.sense_ivf_search(ix, qp, rerank, nprobe)
             sc, idx = S.sense_rescore_topk(ds, qs, ci, k)
         else:
-            sc, idx = S.sense_ivf_search(ix, qp, k, 8)
+            sc, idx = S.sense_ivf_search(ix, qp, k, nprobe)
         dr = S.sense_gather_drafts(ds, idx)
         tr = S.sense_build_tree(dr, node_cap=cap, mask_bits=True)
         torch.cuda.synchronize()
-        assert S.sense_device_status(clear=True) == 0
+        # the same status as the composed calls: none, or for a short pool
+        # the -1 slots' rows (bad index, then negative tokens in the trie)
+        assert S.sense_device_status(clear=True) == st_one
         assert torch.equal(got["scores"], sc) and torch.equal(got["idx"], idx)
+        if nprobe == 1:  # a short pool: the padding is part of the result
+            assert (idx == -1).any()
+            assert st_one == S.DEVST_BAD_INDEX | S.DEVST_BAD_TOKEN
+        else:
+            assert st_one == 0
         assert torch.equal(got["spans"], dr)
         for key in ("num_nodes", "tokens", "parent", "depth", "gamma", "mask_bits"):
             assert torch.equal(got[key], tr[key]), key
