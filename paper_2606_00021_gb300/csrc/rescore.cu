@@ -16,14 +16,17 @@
 //     the warp streams its candidates' rows through a 3-stage ring of
 //     8 KB shared-memory stages with 1-D bulk copies (cp.async.bulk,
 //     completion on an mbarrier, every wait bounded); a row longer than a
-//     stage takes several stages.  Lane l accumulates chunks l, l + 32, ...
-//     of 8 bf16 in increasing order, then a butterfly sums the lanes.
+//     stage takes several stages.  Lane l holds its query chunks in
+//     registers and accumulates chunks l, l + 64, ... and l + 32, l + 96,
+//     ... of 8 bf16 in two fp32 sums (each in increasing order), added
+//     before a butterfly sums the lanes.
 //  2. Warp 0 sorts the CTA's candidate keys (score code, inverted index)
 //     in registers with a bitonic network.
-//  3. After a cluster barrier every CTA copies the C sorted lists through
-//     distributed shared memory, and the rank of each of its own keys is its
-//     position in its list plus, per other list, a binary-search count of
-//     the keys ahead of it; keys ranked below k are written in place.
+//  3. Each CTA stores its sorted list into every CTA of the cluster through
+//     distributed shared memory; after one cluster barrier the rank of each
+//     of its own keys is its position in its list plus, per other list, a
+//     binary-search count of the keys ahead of it; keys ranked below k are
+//     written in place.
 // Slots with index -1 (fewer candidates than N') are empty; an index
 // outside [0, n) is empty too and sets SENSE_DEVST_BAD_INDEX.  A copy that
 // never lands sets SENSE_DEVST_TIMEOUT and drops the warp's later
@@ -113,6 +116,15 @@ __device__ __forceinline__ void warp_sort_desc(uint64_t (&x)[KPL]) {
   }
 }
 
+// Split cluster barrier: every thread arrives (relaxed, nothing to
+// publish) and later waits; between the two the CTA runs its own work.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+
 template <int KPL>
 __global__ void __launch_bounds__(kRsThreads, 1)
 rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
@@ -144,6 +156,7 @@ rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
     s_total = 0u;
   }
   for (int i = threadIdx.x; i < kRsListMax; i += blockDim.x) s_list[i] = 0ull;
+  cluster_arrive_relaxed();  // waited for before the first remote store
   __syncthreads();
 
   // 1. score the warp's candidates
@@ -178,8 +191,19 @@ rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
   };
   if (lane == 0)
     for (int g = 0; g < min(kRsDepth, total); ++g) issue(g);
-  const uint16_t* qrow = queries + (int64_t)qi * d;
-  float acc = 0.0f;
+  // the query chunks a lane multiplies: loaded once when a row is one
+  // stage, else with each stage, always all before the products
+  const uint4* qrow4 = reinterpret_cast<const uint4*>(queries + (int64_t)qi * d);
+  uint4 qv[kRsLaneChunks];
+  auto load_q = [&](int piece, int nc) {
+#pragma unroll
+    for (int u = 0; u < kRsLaneChunks; ++u) {
+      const int j = lane + 32 * u;
+      qv[u] = j < nc ? __ldg(qrow4 + piece * kRsChunks + j) : make_uint4(0u, 0u, 0u, 0u);
+    }
+  };
+  if (spr == 1) load_q(0, rowb >> 4);
+  float acc0 = 0.0f, acc1 = 0.0f;  // even and odd chunks of the lane
   for (int g = 0; g < total; ++g) {
     const bool got = rs_wait(ptx::smem_u32(wbars + g % kRsDepth), (uint32_t)(g / kRsDepth) & 1u);
     if (!__all_sync(0xffffffffu, got)) {
@@ -193,11 +217,12 @@ rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
     const int v = g / spr, piece = g - v * spr;
     const int nc = min(kRsChunks, (rowb - piece * kRsStage) >> 4);
     const uint4* st = wring + (size_t)(g % kRsDepth) * kRsChunks;
-    const uint4* q4 = reinterpret_cast<const uint4*>(qrow) + piece * kRsChunks;
+    if (spr > 1) load_q(piece, nc);
 #pragma unroll
-    for (int u = 0; u < kRsLaneChunks; ++u) {
+    for (int u = 0; u < kRsLaneChunks; u += 2) {
       const int j = lane + 32 * u;
-      if (j < nc) acc = dot8(st[j], __ldg(q4 + j), acc);
+      if (j < nc) acc0 = dot8(st[j], qv[u], acc0);
+      if (j + 32 < nc) acc1 = dot8(st[j + 32], qv[u + 1], acc1);
     }
     __syncwarp();  // every lane has read the stage: its buffer takes stage g + depth
     if (lane == 0 && g + kRsDepth < total) {
@@ -205,15 +230,18 @@ rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
       issue(g + kRsDepth);
     }
     if (piece == spr - 1) {
+      float acc = acc0 + acc1;
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
       if (lane == 0) s_list[warp + kRsWarps * v] = cand_key(acc, (uint32_t)wcidx[v]);
-      acc = 0.0f;
+      acc0 = 0.0f;
+      acc1 = 0.0f;
     }
   }
   __syncthreads();
 
-  // 2. sort this CTA's keys
+  // 2. sort this CTA's keys and store the sorted list into every CTA's
+  //    copy of the cluster's lists (row r of s_all)
   if (warp == 0) {
     uint64_t x[KPL];
 #pragma unroll
@@ -222,16 +250,17 @@ rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
 #pragma unroll
     for (int i = 0; i < KPL; ++i) s_list[lane + 32 * i] = x[i];
   }
-  cl.sync();
+  cluster_wait();  // every CTA of the cluster is running
+  __syncthreads();
+  for (int t = threadIdx.x; t < C * L; t += blockDim.x)
+    *cl.map_shared_rank(s_all + r * L + (t % L), (unsigned)(t / L)) = s_list[t % L];
+  cl.sync();  // the lists are complete; no remote access after this
 
-  // 3. copy the cluster's lists, rank this CTA's keys among them
+  // 3. rank this CTA's keys among the cluster's lists
   for (int t = threadIdx.x; t < C * L; t += blockDim.x) {  // C * L: a multiple of blockDim
-    const uint64_t v = *cl.map_shared_rank(s_list + (t % L), (unsigned)(t / L));
-    s_all[t] = v;
-    const unsigned nz = __ballot_sync(0xffffffffu, v != 0ull);
+    const unsigned nz = __ballot_sync(0xffffffffu, s_all[t] != 0ull);
     if (lane == 0) atomicAdd(&s_total, (unsigned)__popc(nz));
   }
-  cl.sync();  // no CTA reads another's shared memory after this
   float* os = out_scores + (int64_t)qi * k;
   int32_t* oi = out_idx + (int64_t)qi * k;
   for (int t0 = 0; t0 < L * C; t0 += blockDim.x) {  // L * C is a multiple of blockDim
@@ -259,6 +288,7 @@ rescore_kernel(const uint16_t* __restrict__ keys, int64_t n, int d,
       }
     }
   }
+  __syncthreads();  // s_total complete
   if (r == 0) {  // fewer valid candidates than k: -inf, -1
     const float NEG = -__int_as_float(0x7f800000);
     for (int t = (int)s_total + threadIdx.x; t < k; t += blockDim.x) {
