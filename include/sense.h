@@ -321,8 +321,11 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
  * the similarity of the full hidden state to each candidate's key, and keeps
  * the top N).  For each query q, the score of candidate c is
  * <queries[q], keys[cand_idx[q, c]]> over the datastore's stored bf16 keys
- * with fp32 accumulation (the arithmetic of sense_retrieve_topk), and the k
- * best candidates are written in the order (score desc, key index asc).
+ * with fp32 accumulation (the precision of sense_retrieve_topk; the
+ * summation order differs, so a score may differ from that call's in the
+ * last bits), and the k best candidates are written in the order (score
+ * desc, key index asc).  A candidate that appears twice is scored and kept
+ * twice.
  *
  * queries: bf16 [q, d] (the full hidden states), 16-byte aligned;
  * cand_idx: int32 [q, n_cand] key indices, -1 for an empty slot (what
@@ -331,7 +334,9 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
  * candidates get -inf / -1.  Device pointers owned by the caller; no
  * workspace.  Limits: 1 <= q <= 65535, 1 <= k <= n_cand <= SENSE_MAX_RESCORE.
  * An index outside [0, n) is treated as empty and sets
- * SENSE_DEVST_BAD_INDEX.  Asynchronous on `stream`.
+ * SENSE_DEVST_BAD_INDEX; a key-row copy that never lands sets
+ * SENSE_DEVST_TIMEOUT and drops that warp's remaining candidates.
+ * Asynchronous on `stream`.
  */
 sense_status sense_rescore_topk(const sense_datastore* ds, const uint16_t* queries, int32_t q,
                                 const int32_t* cand_idx, int32_t n_cand, int32_t k,
