@@ -631,7 +631,10 @@ sense_status sense_tree_attention(const uint16_t* q, const uint16_t* k_cache,
  *   (1..SENSE_MAX_WINDOW), tau (>= 0), flags.  Paper defaults (App. E):
  *   gamma 0.05, kappa 3, W 6, tau 0.
  *   workspace: at least sense_soft_gate_workspace_bytes(q, cap, kappa)
- *   bytes of device scratch, 256-byte aligned.
+ *   bytes of device scratch, 256-byte aligned, zero-filled before its
+ *   first use and used by no other call: it holds per-query counters that
+ *   let the last row of a query run the decision in the same launch, and
+ *   every call leaves them zero.
  *   Limits: vocab >= kappa, vocab % 4 == 0; d % 8 == 0; k * m <=
  *   SENSE_MAX_TREE_TOKENS; logits 16-byte aligned.
  */

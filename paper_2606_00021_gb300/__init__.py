@@ -165,8 +165,10 @@ def sense_retrieve_workspace_bytes(ds: Datastore, q: int, k: int) -> int:
 
 
 def alloc_workspace(nbytes: int, device=None) -> torch.Tensor:
+    """Device scratch of at least nbytes, zero-filled (the soft gate keeps
+    counters there that must start at zero)."""
     dev = device or torch.device("cuda", torch.cuda.current_device())
-    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=dev)
+    return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=dev)
 
 
 def sense_retrieve_topk(ds: Datastore, queries: torch.Tensor, k: int, out_scores=None,

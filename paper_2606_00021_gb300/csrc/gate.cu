@@ -534,93 +534,6 @@ gate_rows_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__
   }
 }
 
-// Few rows with short slices: NC blocks per row (a cluster of NC blocks
-// when NC > 1), whose kWarps * NC warps stream consecutive slices of seg4
-// float4 each through their own rings.  Each block keeps its warps'
-// partials in shared memory; warp 0 of the cluster's first block merges
-// them all, reading the other block's partials through distributed shared
-// memory.  No task counter, no partials in global memory, no grid-wide
-// atomics: the row's latency is one streaming pass plus block and cluster
-// barriers.
-template <int KM, int NC>
-__global__ void __launch_bounds__(kRowThreads, 1)
-gate_row_block_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ num_nodes,
-                      int cap, const float* __restrict__ root_logits,
-                      const float* __restrict__ node_logits, int vocab, int kappa, float thr,
-                      int unnormalized, int seg4, int32_t* __restrict__ stats, uint32_t* status) {
-  static_assert(NC >= 1 && NC * kWarps <= 32, "one merging warp holds every partial");
-  extern __shared__ __align__(128) float4 ring_all[];
-  __shared__ __align__(8) uint64_t bars_all[kWarps * kWStages];
-  __shared__ Partial s_part[kWarps];
-  __shared__ int s_fail;
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  pdl_wait();  // the tree (and everything before it) is complete
-  pdl_launch_dependents();
-  const int rid = blockIdx.x / NC;  // q * (cap + 1) + slot
-  const int crank = blockIdx.x - rid * NC;  // rank in the cluster (clusters of NC along x)
-  const int q = rid / (cap + 1);
-  const int slot = rid - q * (cap + 1);  // 0 = root, 1 + n = node n
-  const float* row;
-  if (slot == 0) {
-    row = root_logits + (int64_t)q * vocab;
-  } else {
-    const int nd = slot - 1;
-    const int nn = min(num_nodes[q], cap);
-    const bool inner = (nd + 1 < nn) && parent[(int64_t)q * cap + nd + 1] == nd;
-    if (!inner) return;  // depends on the row only: the whole cluster leaves
-    row = node_logits + ((int64_t)q * cap + nd) * vocab;
-  }
-  if (threadIdx.x == 0) {
-    for (int b = 0; b < kWarps * kWStages; ++b) ptx::mbar_init(ptx::smem_u32(bars_all + b), 1);
-    ptx::fence_barrier_init();
-    s_fail = 0;
-  }
-  __syncthreads();
-  const int n4 = vocab >> 2;
-  const int lo4 = min(n4, (crank * kWarps + wid) * seg4);
-  const int hi4 = min(n4, lo4 + seg4);
-  if (lo4 < hi4) {
-    float4* ring = ring_all + (size_t)wid * kWStages * kWStageF4;
-    uint64_t* bars = bars_all + wid * kWStages;
-    const uint64_t pol = (lane == 0) ? ptx::policy_evict_first() : 0ull;
-    uint32_t seq = 0;
-    if (!warp_segment<KM>(row, lo4, hi4, kappa, ring, bars, seq, pol, &s_part[wid])) {
-      if (lane == 0) {
-        raise_status(status, SENSE_DEVST_TIMEOUT);
-        s_fail = 1;
-      }
-    }
-  } else if (lane == 0) {  // empty slice: a neutral partial
-    Partial& p = s_part[wid];
-    p.z = 0.0f;
-    p.s = 0.0f;
-    p.m = -FLT_MAX;
-    p.bv = -FLT_MAX;
-    p.bi = 0x7fffffff;
-    for (int r = 0; r < SENSE_MAX_KAPPA; ++r) {
-      p.tv[r] = -FLT_MAX;
-      p.ti[r] = 0x7fffffff;
-    }
-  }
-  int32_t* out = stats + (int64_t)rid * kStatsInts;
-  if constexpr (NC == 1) {
-    __syncthreads();
-    if (wid == 0 && !s_fail)
-      finish_row(lane < kWarps ? &s_part[lane] : nullptr, vocab, kappa, thr, unnormalized, out);
-  } else {
-    cg::cluster_group cl = cg::this_cluster();
-    cl.sync();  // every block's partials (and failure flag) are written
-    if (crank == 0 && wid == 0) {
-      const int src = lane / kWarps;  // block holding this lane's partial
-      const Partial* pp = cl.map_shared_rank(&s_part[lane - src * kWarps], src);
-      bool fail = false;
-      for (int r = 0; r < NC; ++r) fail |= *cl.map_shared_rank(&s_fail, r) != 0;
-      if (!fail) finish_row(lane < NC * kWarps ? pp : nullptr, vocab, kappa, thr, unnormalized, out);
-    }
-    cl.sync();  // the other blocks' shared memory stays alive until it is read
-  }
-}
-
 constexpr int kDecideThreads = 1024;
 
 // Shared memory of a staged decide block: Gamma, tokens, parents and the
@@ -641,17 +554,18 @@ __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
-__global__ void __launch_bounds__(kDecideThreads)
-gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats, int staged) {
-  // dynamic: staged ? [Gamma k*m][tokens cap][parents cap][stats (cap+1) rows] : nothing,
-  // then flags [k*m]: bit0 valid, bit1 em, bit2 ent, bit3 topk, bit4 G
-  extern __shared__ __align__(16) int32_t s_dyn[];
+// The decision of query q by one block (any multiple of 32 threads up to
+// 1024).  s_dyn: staged ? [Gamma k*m][tokens cap][parents cap][stats
+// (cap+1) rows] : nothing, then flags [k*m]: bit0 valid, bit1 em, bit2 ent,
+// bit3 topk, bit4 G.  `fresh` (staged only): the statistics were written
+// by other blocks of the running grid, so they are read from L2 with plain
+// loads rather than copied through L1.
+__device__ __forceinline__ void decide_block(const GateArgs& a, const int32_t* __restrict__ stats, int staged,
+                             int q, int32_t* s_dyn, bool fresh) {
   __shared__ int s_L[SENSE_MAX_K];
   __shared__ int s_best[32];
   __shared__ int s_istar, s_lstar, s_next, s_nn;
   __shared__ ArgMax s_w[32];
-  pdl_wait();  // every row statistic is written
-  const int q = blockIdx.x;
   const int k = a.k, m = a.m, cap = a.cap, km = k * m;
   const int32_t* gam = a.gamma + (int64_t)q * km;
   const int32_t* tok = a.tokens + (int64_t)q * cap;
@@ -668,7 +582,10 @@ gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats, int staged) {
       cp_async4(stk + i, tok + i);
       cp_async4(spr + i, par + i);
     }
-    for (int i = threadIdx.x; i < (cap + 1) * kStatsInts; i += blockDim.x) cp_async4(sst + i, st + i);
+    if (fresh)
+      for (int i = threadIdx.x; i < (cap + 1) * kStatsInts; i += blockDim.x) sst[i] = __ldcg(st + i);
+    else
+      for (int i = threadIdx.x; i < (cap + 1) * kStatsInts; i += blockDim.x) cp_async4(sst + i, st + i);
     if (threadIdx.x == 0) cp_async4(&s_nn, a.num_nodes + q);
     cp_async_wait_all();
     s_flags = reinterpret_cast<uint8_t*>(sst + (cap + 1) * kStatsInts);
@@ -829,6 +746,129 @@ gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats, int staged) {
   }
 }
 
+// The streaming pass of one row by the NC blocks of its cluster (all of
+// them call it); warp 0 of block 0 writes the row's statistics to `out`.
+template <int KM, int NC>
+__device__ void row_block_pass(const float* __restrict__ row, int vocab, int kappa, float thr,
+                               int unnormalized, int seg4, int32_t* __restrict__ out,
+                               uint32_t* status, int crank, float4* ring_all, uint64_t* bars_all,
+                               Partial* s_part, int& s_fail) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    for (int b = 0; b < kWarps * kWStages; ++b) ptx::mbar_init(ptx::smem_u32(bars_all + b), 1);
+    ptx::fence_barrier_init();
+    s_fail = 0;
+  }
+  __syncthreads();
+  const int n4 = vocab >> 2;
+  const int lo4 = min(n4, (crank * kWarps + wid) * seg4);
+  const int hi4 = min(n4, lo4 + seg4);
+  if (lo4 < hi4) {
+    float4* ring = ring_all + (size_t)wid * kWStages * kWStageF4;
+    uint64_t* bars = bars_all + wid * kWStages;
+    const uint64_t pol = (lane == 0) ? ptx::policy_evict_first() : 0ull;
+    uint32_t seq = 0;
+    if (!warp_segment<KM>(row, lo4, hi4, kappa, ring, bars, seq, pol, &s_part[wid])) {
+      if (lane == 0) {
+        raise_status(status, SENSE_DEVST_TIMEOUT);
+        s_fail = 1;
+      }
+    }
+  } else if (lane == 0) {  // empty slice: a neutral partial
+    Partial& p = s_part[wid];
+    p.z = 0.0f;
+    p.s = 0.0f;
+    p.m = -FLT_MAX;
+    p.bv = -FLT_MAX;
+    p.bi = 0x7fffffff;
+    for (int r = 0; r < SENSE_MAX_KAPPA; ++r) {
+      p.tv[r] = -FLT_MAX;
+      p.ti[r] = 0x7fffffff;
+    }
+  }
+  if constexpr (NC == 1) {
+    __syncthreads();
+    if (wid == 0 && !s_fail)
+      finish_row(lane < kWarps ? &s_part[lane] : nullptr, vocab, kappa, thr, unnormalized, out);
+  } else {
+    cg::cluster_group cl = cg::this_cluster();
+    cl.sync();  // every block's partials (and failure flag) are written
+    if (crank == 0 && wid == 0) {
+      const int src = lane / kWarps;  // block holding this lane's partial
+      const Partial* pp = cl.map_shared_rank(&s_part[lane - src * kWarps], src);
+      bool fail = false;
+      for (int r = 0; r < NC; ++r) fail |= *cl.map_shared_rank(&s_fail, r) != 0;
+      if (!fail) finish_row(lane < NC * kWarps ? pp : nullptr, vocab, kappa, thr, unnormalized, out);
+    }
+    cl.sync();  // the other blocks' shared memory stays alive until it is read
+  }
+}
+
+// Few rows with short slices: NC blocks per row (a cluster of NC blocks
+// when NC > 1), whose kWarps * NC warps stream consecutive slices of seg4
+// float4 each through their own rings.  Each block keeps its warps'
+// partials in shared memory; warp 0 of the cluster's first block merges
+// them all, reading the other block's partials through distributed shared
+// memory.  No task counter, no partials in global memory, no grid-wide
+// atomics: the row's latency is one streaming pass plus block and cluster
+// barriers.  With `decide_done` set, the decision of each query runs in the
+// same launch: every row slot of query q (rows without logits included)
+// counts itself on decide_done[q] after its statistics are written, and the
+// first block of the slot that arrives last runs the decide block and
+// resets the counter to zero for the next call.
+template <int KM, int NC>
+__global__ void __launch_bounds__(kRowThreads, 1)
+gate_row_block_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ num_nodes,
+                      int cap, const float* __restrict__ root_logits,
+                      const float* __restrict__ node_logits, int vocab, int kappa, float thr,
+                      int unnormalized, int seg4, int32_t* __restrict__ stats, uint32_t* status,
+                      GateArgs a, int staged, unsigned* __restrict__ decide_done) {
+  static_assert(NC >= 1 && NC * kWarps <= 32, "one merging warp holds every partial");
+  extern __shared__ __align__(128) float4 ring_all[];
+  __shared__ __align__(8) uint64_t bars_all[kWarps * kWStages];
+  __shared__ Partial s_part[kWarps];
+  __shared__ int s_fail;
+  __shared__ int s_last;
+  pdl_wait();  // the tree (and everything before it) is complete
+  pdl_launch_dependents();
+  const int rid = blockIdx.x / NC;  // q * (cap + 1) + slot
+  const int crank = blockIdx.x - rid * NC;  // rank in the cluster (clusters of NC along x)
+  const int q = rid / (cap + 1);
+  const int slot = rid - q * (cap + 1);  // 0 = root, 1 + n = node n
+  const float* row = nullptr;
+  if (slot == 0) {
+    row = root_logits + (int64_t)q * vocab;
+  } else {
+    const int nd = slot - 1;
+    const int nn = min(num_nodes[q], cap);
+    const bool inner = (nd + 1 < nn) && parent[(int64_t)q * cap + nd + 1] == nd;
+    // depends on the row only: the whole cluster skips the row
+    if (inner) row = node_logits + ((int64_t)q * cap + nd) * vocab;
+  }
+  if (row) row_block_pass<KM, NC>(row, vocab, kappa, thr, unnormalized, seg4,
+                                  stats + (int64_t)rid * kStatsInts, status, crank, ring_all,
+                                  bars_all, s_part, s_fail);
+  if (decide_done == nullptr || crank != 0) return;
+  __threadfence();  // this block's statistics before its count
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const bool last = atomicAdd(&decide_done[q], 1u) == (unsigned)cap;  // cap + 1 slots
+    if (last) atomicExch(&decide_done[q], 0u);
+    s_last = last;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();  // every slot's statistics are visible
+  decide_block(a, stats, staged, q, reinterpret_cast<int32_t*>(ring_all), true);
+}
+
+__global__ void __launch_bounds__(kDecideThreads)
+gate_decide_kernel(GateArgs a, const int32_t* __restrict__ stats, int staged) {
+  extern __shared__ __align__(16) int32_t s_dyn[];
+  pdl_wait();  // every row statistic is written
+  decide_block(a, stats, staged, blockIdx.x, s_dyn, false);
+}
+
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 }  // namespace
@@ -851,7 +891,8 @@ size_t gate_workspace_bytes(int q, int cap, int kappa) {
   const size_t rows = (size_t)q * (cap + 1);
   const int segs = gate_segments(q, cap, 1 << 30);  // upper bound over vocabularies
   size_t b = align256(rows * kStatsInts * sizeof(int32_t));
-  b += 256;  // task counter
+  b += 256;                                      // task counter
+  b += align256((size_t)q * sizeof(unsigned));  // per-query decide counters
   if (segs > 1) b += align256(rows * segs * sizeof(Partial)) + align256(rows * sizeof(unsigned));
   return b;
 }
@@ -863,7 +904,11 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
   ws += align256(rows * kStatsInts * sizeof(int32_t));
   unsigned* next_task = reinterpret_cast<unsigned*>(ws);
   ws += 256;
+  unsigned* decide_done = reinterpret_cast<unsigned*>(ws);  // zero between calls
+  ws += align256((size_t)a.q * sizeof(unsigned));
   const int n4 = a.vocab >> 2;
+  const size_t staged_smem = decide_stage_bytes(a.k, a.m, a.cap);
+  const int staged = staged_smem <= kDecideStageMax ? 1 : 0;
   sense_status st = SENSE_OK;
   // Few rows, each warp's slice inside its ring: blocks per row (two as a
   // cluster when the rows leave room for it).
@@ -875,7 +920,7 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     const int nc = pair ? 2 : 1;
     const int slice4 = (n4 + nc * kWarps - 1) / (nc * kWarps);
     void (*kern)(const int32_t*, const int32_t*, int, const float*, const float*, int, int, float,
-                 int, int, int32_t*, uint32_t*);
+                 int, int, int32_t*, uint32_t*, GateArgs, int, unsigned*);
     if (pair) kern = (a.kappa <= 4) ? gate_row_block_kernel<4, 2>
                                      : gate_row_block_kernel<SENSE_MAX_KAPPA, 2>;
     else kern = (a.kappa <= 4) ? gate_row_block_kernel<4, 1>
@@ -898,12 +943,16 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
+    // the decision runs in the same launch (in the last row slot of each
+    // query) when its staged inputs fit the ring's shared memory
+    unsigned* fuse = staged ? decide_done : nullptr;
     LaunchScope ls(K_GATE_ROWS, s);
     st = cuda_check(cudaLaunchKernelEx(&cfg, kern, a.parent, a.num_nodes, a.cap, a.root_logits,
                                        a.node_logits, a.vocab, a.kappa, a.thr, a.unnormalized,
-                                       slice4, stats, a.status),
+                                       slice4, stats, a.status, a, staged, fuse),
                     "launch gate_row_block");
     if (st != SENSE_OK) return st;
+    if (fuse) return SENSE_OK;
   } else {
     const int segs = gate_segments(a.q, a.cap, a.vocab);
     const int seg4 = (n4 + segs - 1) / segs;
@@ -934,8 +983,6 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     st = cuda_check(cudaGetLastError(), "launch gate_rows");
     if (st != SENSE_OK) return st;
   }
-  const size_t staged_smem = decide_stage_bytes(a.k, a.m, a.cap);
-  const int staged = staged_smem <= kDecideStageMax ? 1 : 0;
   const size_t smem = staged ? staged_smem : (size_t)a.k * a.m;
   if (smem > 48 * 1024) {
     st = cuda_check(func_smem(reinterpret_cast<const void*>(gate_decide_kernel), (int)smem),
