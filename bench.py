@@ -229,8 +229,9 @@ class Pipeline:
         q = self.cfg["q"]
         self.dyn = {"ctx": ctx, "kd": kd, "delta": delta, "outs": {},
                     "ws": self.S.alloc_workspace(self.S.lib().sense_ctx_search_workspace_bytes(
-                        __import__("ctypes").c_void_p(ctx.handle), q, kd), dev),
-                    "anchor": torch.zeros(q, dtype=torch.int32, device=dev)}
+                        __import__("ctypes").c_void_p(ctx.handle), q, kd), dev)}
+        # x~ of the next step: the gate writes it, the next step's rerank reads it
+        self.gate["next_anchor"] = torch.zeros(q, dtype=torch.int32, device=dev)
 
     def use_verify(self, heads, prefix, dev, seed=0):
         """Adds the tree-masked attention of the verify forward (Alg. 1) on a
@@ -292,43 +293,58 @@ class Pipeline:
                 before_gate()
             self._prepared(("gate", stream) + tuple(t.data_ptr() for t in gate_in), make_gate)()
             return
-        if dyn is None:
-            # retrieval, gather and trie in one call (exact: one kernel per
-            # query after the scan on the single-pass path)
-            outs = self.tree
-            outs["scores"], outs["idx"], outs["spans"] = self.scores, self.idx, self.drafts
-            if self.ann is None:
-                S.sense_draft(self.ds, query, cfg["k"], node_cap=cfg["cap"],
-                              mask_bits=ver is not None, outs=outs, workspace=self.ws)
-            else:
-                a = self.ann
-                S.sense_ann_draft(a["index"], self.ds, query, a["basis"], a["mean"], cfg["k"],
-                                  a["nprobe"], rerank=a.get("rerank", 0), node_cap=cfg["cap"],
-                                  mask_bits=ver is not None, outs=outs, workspace=self.ann_ws)
-        else:
-            self.retrieve(query)
-            if dyn is None:
-                S.sense_gather_drafts(self.ds, self.idx, out=self.drafts)
-            else:
-                S.sense_ctx_search(dyn["ctx"], query, dyn["kd"], dyn["delta"], outs=dyn["outs"],
-                                   workspace=dyn["ws"])
-                S.sense_hybrid_drafts(self.ds, self.scores, self.idx, dyn["outs"], dyn["anchor"],
-                                      cfg["k"], True, out=self.drafts)
-            S.sense_build_tree(self.drafts, node_cap=cfg["cap"], mask_bits=ver is not None,
-                               outs=self.tree)
-        if ver is not None:
-            S.sense_tree_attention(ver["q"], ver["k"], ver["vt"], ver["prefix"],
-                                   self.tree["mask_bits"][0], ver["scale"], out=ver["out"],
-                                   workspace=ver["ws"])
+        # with the dynamic buffer or the verify attention: the step's calls,
+        # recorded once per buffer set (arguments marshalled once) and issued
+        # again every step
+        def make_pre():
+            with S.record_calls() as calls:
+                if dyn is None:
+                    # retrieval, gather and trie in one call (exact: one kernel
+                    # per query after the scan on the single-pass path)
+                    outs = self.tree
+                    outs["scores"], outs["idx"], outs["spans"] = self.scores, self.idx, self.drafts
+                    if self.ann is None:
+                        S.sense_draft(self.ds, query, cfg["k"], node_cap=cfg["cap"],
+                                      mask_bits=ver is not None, outs=outs, workspace=self.ws)
+                    else:
+                        a = self.ann
+                        S.sense_ann_draft(a["index"], self.ds, query, a["basis"], a["mean"],
+                                          cfg["k"], a["nprobe"], rerank=a.get("rerank", 0),
+                                          node_cap=cfg["cap"], mask_bits=ver is not None,
+                                          outs=outs, workspace=self.ann_ws)
+                else:
+                    self.retrieve(query)
+                    S.sense_ctx_search(dyn["ctx"], query, dyn["kd"], dyn["delta"],
+                                       outs=dyn["outs"], workspace=dyn["ws"])
+                    S.sense_hybrid_drafts(self.ds, self.scores, self.idx, dyn["outs"],
+                                          self.gate["next_anchor"], cfg["k"], True,
+                                          out=self.drafts)
+                    S.sense_build_tree(self.drafts, node_cap=cfg["cap"],
+                                       mask_bits=ver is not None, outs=self.tree)
+                if ver is not None:
+                    S.sense_tree_attention(ver["q"], ver["k"], ver["vt"], ver["prefix"],
+                                           self.tree["mask_bits"][0], ver["scale"], out=ver["out"],
+                                           workspace=ver["ws"])
+            return calls
+
+        def make_post():
+            root, nodes, hr, hn = gate_in
+            with S.record_calls() as calls:
+                S.sense_soft_gate(self.tree, root, nodes, hr, hn, workspace=self.gws,
+                                  outs=self.gate, **GATE)
+                if dyn is not None:  # R.Update with the accepted path
+                    g = self.gate
+                    S.sense_ctx_append_path(dyn["ctx"], hr[0], hn[0], self.tree["gamma"][0],
+                                            g["i_star"][:1], g["n_accept"][:1], g["accepted"][0])
+            return calls
+
+        stream = S._stream(None)
+        for c in self._prepared(("pre", stream, query.data_ptr()), make_pre):
+            c()
         if before_gate is not None:
             before_gate()
-        root, nodes, hr, hn = gate_in
-        S.sense_soft_gate(self.tree, root, nodes, hr, hn, workspace=self.gws, outs=self.gate, **GATE)
-        if dyn is not None:
-            g = self.gate
-            S.sense_ctx_append_path(dyn["ctx"], hr[0], hn[0], self.tree["gamma"][0],
-                                    g["i_star"][:1], g["n_accept"][:1], g["accepted"][0])
-            dyn["anchor"].copy_(g["next_anchor"])  # x~ of the next step
+        for c in self._prepared(("post", stream) + tuple(t.data_ptr() for t in gate_in), make_post):
+            c()
 
 
 DRAFT_KERNELS = ("scan_gemv", "scan_tc", "threshold", "merge", "pad_queries", "gather", "tree",

@@ -8,6 +8,7 @@ library's CUDA kernels; there is no CPU path.
 """
 from __future__ import annotations
 
+import contextlib
 import ctypes as C
 from dataclasses import dataclass, field
 
@@ -59,6 +60,35 @@ class Prepared:
 
     def __call__(self):
         _check(self._fn(*self._args))
+
+
+_recorder = None  # list of Prepared calls while record_calls() is active
+
+
+def _call(fn, *args):
+    """Runs a stream-ordered library call, or records it as a Prepared call
+    inside record_calls()."""
+    if _recorder is not None:
+        _recorder.append(Prepared(fn, args, None))
+        return
+    _check(fn(*args))
+
+
+@contextlib.contextmanager
+def record_calls():
+    """Inside the block the per-step library calls (retrieval, projection,
+    search, re-scoring, gather, trie, masks, attention, dynamic buffer, gate)
+    are recorded instead of run, with their arguments marshalled: the block
+    yields the list of Prepared calls, to be issued again in order.  Output
+    buffers the calls allocate are allocated once, here; every buffer must
+    stay alive while the calls are used.  Calls that read results back to
+    the host are not recorded and must not appear in the block."""
+    global _recorder
+    prev, _recorder = _recorder, []
+    try:
+        yield _recorder
+    finally:
+        _recorder = prev
 
 
 def _ptr(t):
@@ -186,10 +216,10 @@ def sense_retrieve_topk(ds: Datastore, queries: torch.Tensor, k: int, out_scores
     need = sense_retrieve_workspace_bytes(ds, q, k)
     if workspace is None:
         workspace = alloc_workspace(need, dev)
-    _check(lib().sense_retrieve_topk(C.c_void_p(ds.handle), queries.data_ptr(), q, k,
+    _call(lib().sense_retrieve_topk, C.c_void_p(ds.handle), queries.data_ptr(), q, k,
                                      out_scores.data_ptr(), out_idx.data_ptr(),
                                      workspace.data_ptr(), workspace.numel(),
-                                     C.c_void_p(_stream(stream))))
+                                     C.c_void_p(_stream(stream)))
     return out_scores, out_idx
 
 
@@ -248,9 +278,9 @@ def sense_rescore_topk(ds: Datastore, queries: torch.Tensor, cand_idx: torch.Ten
         out_scores = torch.empty(q, k, dtype=torch.float32, device=dev)
     if out_idx is None:
         out_idx = _i32((q, k), dev)
-    _check(lib().sense_rescore_topk(C.c_void_p(ds.handle), queries.data_ptr(), q,
+    _call(lib().sense_rescore_topk, C.c_void_p(ds.handle), queries.data_ptr(), q,
                                     cand_idx.data_ptr(), n_cand, k, out_scores.data_ptr(),
-                                    out_idx.data_ptr(), C.c_void_p(_stream(stream))))
+                                    out_idx.data_ptr(), C.c_void_p(_stream(stream)))
     return out_scores, out_idx
 
 
@@ -264,9 +294,9 @@ def sense_gather_drafts(ds: Datastore, idx: torch.Tensor, anchor=None, n_keep=No
         _need(anchor, "anchor", torch.int32, 1)
     if out is None:
         out = _i32((q, keep, ds.m), idx.device)
-    _check(lib().sense_gather_drafts(C.c_void_p(ds.handle), idx.data_ptr(), q, k, _ptr(anchor),
+    _call(lib().sense_gather_drafts, C.c_void_p(ds.handle), idx.data_ptr(), q, k, _ptr(anchor),
                                      keep, 1 if force_anchor else 0, out.data_ptr(),
-                                     C.c_void_p(_stream(stream))))
+                                     C.c_void_p(_stream(stream)))
     return out
 
 
@@ -286,11 +316,11 @@ def sense_build_tree(spans: torch.Tensor, node_cap: int = 0, mask_bits: bool = F
     if mask_bits:
         o.setdefault("mask_bits", torch.empty(q, cap, (cap + 31) // 32, dtype=torch.int32,
                                               device=dev))
-    _check(lib().sense_build_tree(spans.data_ptr(), q, k, m, node_cap, 1 if mask_bits else 0,
+    _call(lib().sense_build_tree, spans.data_ptr(), q, k, m, node_cap, 1 if mask_bits else 0,
                                   o["num_nodes"].data_ptr(), o["tokens"].data_ptr(),
                                   o["parent"].data_ptr(), o["depth"].data_ptr(),
                                   o["gamma"].data_ptr(), _ptr(o.get("mask_bits")),
-                                  C.c_void_p(_stream(stream))))
+                                  C.c_void_p(_stream(stream)))
     o["cap"] = cap
     return o
 
@@ -332,7 +362,7 @@ def sense_draft(ds: Datastore, queries: torch.Tensor, k: int, node_cap: int = 0,
     o["cap"] = cap
     if prepare:
         return Prepared(lib().sense_draft, args, (ds, queries, workspace, dict(o))), o
-    _check(lib().sense_draft(*args))
+    _call(lib().sense_draft, *args)
     return o
 
 
@@ -348,9 +378,9 @@ def sense_tree_mask_full(tree: dict, prefix_len: torch.Tensor, cache_len: int,
     if out is None:
         out = torch.empty(q, cap, cache_len, dtype=torch.float32, device=bits.device)
     _need(out, "out", torch.float32, 3)
-    _check(lib().sense_tree_mask_full(bits.data_ptr(), tree["num_nodes"].data_ptr(), q, cap,
+    _call(lib().sense_tree_mask_full, bits.data_ptr(), tree["num_nodes"].data_ptr(), q, cap,
                                       prefix_len.data_ptr(), cache_len, out.data_ptr(),
-                                      C.c_void_p(_stream(stream))))
+                                      C.c_void_p(_stream(stream)))
     return out
 
 
@@ -372,9 +402,9 @@ def sense_project(x: torch.Tensor, basis: torch.Tensor, mean: torch.Tensor | Non
     if out is None:
         out = torch.empty(n, v, dtype=torch.float32, device=x.device)
     _need(out, "out", torch.float32, 2)
-    _check(lib().sense_project(x.data_ptr(), n, d, basis.data_ptr(), v, _ptr(mean),
+    _call(lib().sense_project, x.data_ptr(), n, d, basis.data_ptr(), v, _ptr(mean),
                                1 if normalize else 0, out.data_ptr(),
-                               C.c_void_p(_stream(stream))))
+                               C.c_void_p(_stream(stream)))
     return out
 
 
@@ -516,7 +546,7 @@ def sense_ann_draft(ix: "IvfIndex", ds: Datastore, queries: torch.Tensor, basis:
     if prepare:
         return Prepared(lib().sense_ann_draft, args,
                         (ix, ds, queries, basis, mean, workspace, dict(o))), o
-    _check(lib().sense_ann_draft(*args))
+    _call(lib().sense_ann_draft, *args)
     return o
 
 
@@ -536,10 +566,10 @@ def sense_ivf_search(ix: IvfIndex, queries: torch.Tensor, k: int, nprobe: int,
     probes = _i32((q, nprobe), dev) if want_probes else None
     if workspace is None:
         workspace = alloc_workspace(sense_ivf_search_workspace_bytes(ix, q, k, nprobe), dev)
-    _check(lib().sense_ivf_search(C.c_void_p(ix.handle), queries.data_ptr(), q, k, nprobe,
+    _call(lib().sense_ivf_search, C.c_void_p(ix.handle), queries.data_ptr(), q, k, nprobe,
                                   out_scores.data_ptr(), out_idx.data_ptr(), _ptr(probes),
                                   workspace.data_ptr(), workspace.numel(),
-                                  C.c_void_p(_stream(stream))))
+                                  C.c_void_p(_stream(stream)))
     return (out_scores, out_idx, probes) if want_probes else (out_scores, out_idx)
 
 
@@ -588,8 +618,8 @@ def sense_ctx_append(ctx: ContextBuffer, hidden: torch.Tensor, tokens: torch.Ten
     _need(tokens, "tokens", torch.int32, 1)
     if hidden.shape[0] != tokens.shape[0] or hidden.shape[1] != ctx.d:
         raise ValueError("hidden must be [t, d] and tokens [t]")
-    _check(lib().sense_ctx_append(C.c_void_p(ctx.handle), hidden.data_ptr(), tokens.data_ptr(),
-                                  hidden.shape[0], C.c_void_p(_stream(stream))))
+    _call(lib().sense_ctx_append, C.c_void_p(ctx.handle), hidden.data_ptr(), tokens.data_ptr(),
+                                  hidden.shape[0], C.c_void_p(_stream(stream)))
 
 
 def sense_ctx_append_path(ctx: ContextBuffer, root_hidden: torch.Tensor,
@@ -603,11 +633,11 @@ def sense_ctx_append_path(ctx: ContextBuffer, root_hidden: torch.Tensor,
     _need(gamma, "gamma", torch.int32, 2)
     for t, name in ((i_star, "i_star"), (n_accept, "n_accept"), (accepted, "accepted")):
         _need(t, name, torch.int32, 1)
-    _check(lib().sense_ctx_append_path(C.c_void_p(ctx.handle), root_hidden.data_ptr(),
+    _call(lib().sense_ctx_append_path, C.c_void_p(ctx.handle), root_hidden.data_ptr(),
                                        node_hidden.data_ptr(), node_hidden.shape[0],
                                        gamma.data_ptr(), gamma.shape[0], i_star.data_ptr(),
                                        n_accept.data_ptr(), accepted.data_ptr(),
-                                       C.c_void_p(_stream(stream))))
+                                       C.c_void_p(_stream(stream)))
 
 
 def sense_ctx_search(ctx: ContextBuffer, queries: torch.Tensor, k: int, delta: float = 0.0,
@@ -623,10 +653,10 @@ def sense_ctx_search(ctx: ContextBuffer, queries: torch.Tensor, k: int, delta: f
     if workspace is None:
         workspace = alloc_workspace(lib().sense_ctx_search_workspace_bytes(
             C.c_void_p(ctx.handle), q, k), dev)
-    _check(lib().sense_ctx_search(C.c_void_p(ctx.handle), queries.data_ptr(), q, k,
+    _call(lib().sense_ctx_search, C.c_void_p(ctx.handle), queries.data_ptr(), q, k,
                                   C.c_float(delta), o["scores"].data_ptr(), o["pos"].data_ptr(),
                                   o["spans"].data_ptr(), workspace.data_ptr(), workspace.numel(),
-                                  C.c_void_p(_stream(stream))))
+                                  C.c_void_p(_stream(stream)))
     return o
 
 
@@ -644,12 +674,12 @@ def sense_hybrid_drafts(ds: Datastore, static_scores: torch.Tensor, static_idx: 
         _need(anchor, "anchor", torch.int32, 1)
     if out is None:
         out = _i32((q, keep, ds.m), static_idx.device)
-    _check(lib().sense_hybrid_drafts(C.c_void_p(ds.handle), static_scores.data_ptr(),
+    _call(lib().sense_hybrid_drafts, C.c_void_p(ds.handle), static_scores.data_ptr(),
                                      static_idx.data_ptr(), ks,
                                      None if dyn is None else dyn["scores"].data_ptr(),
                                      None if dyn is None else dyn["spans"].data_ptr(), kd, q,
                                      _ptr(anchor), keep, 1 if force_anchor else 0,
-                                     out.data_ptr(), C.c_void_p(_stream(stream))))
+                                     out.data_ptr(), C.c_void_p(_stream(stream)))
     return out
 
 
@@ -671,11 +701,11 @@ def sense_tree_attention(q: torch.Tensor, k_cache: torch.Tensor, vt_cache: torch
     if workspace is None:
         workspace = alloc_workspace(
             lib().sense_tree_attention_workspace_bytes(heads, L, prefix_len), q.device)
-    _check(lib().sense_tree_attention(q.data_ptr(), k_cache.data_ptr(), vt_cache.data_ptr(), heads,
+    _call(lib().sense_tree_attention, q.data_ptr(), k_cache.data_ptr(), vt_cache.data_ptr(), heads,
                                       L, dh, cap, prefix_len, mask_bits.data_ptr(),
                                       mask_bits.shape[1], C.c_float(scale), out.data_ptr(),
                                       workspace.data_ptr(), workspace.numel(),
-                                      C.c_void_p(_stream(stream))))
+                                      C.c_void_p(_stream(stream)))
     return out
 
 
@@ -726,7 +756,7 @@ def sense_soft_gate(tree: dict, root_logits: torch.Tensor, node_logits: torch.Te
         return Prepared(lib().sense_soft_gate, args,
                         (dict(tree), root_logits, node_logits, root_hidden, node_hidden, p,
                          workspace, dict(o))), o
-    _check(lib().sense_soft_gate(*args))
+    _call(lib().sense_soft_gate, *args)
     return o
 
 

@@ -17,11 +17,12 @@
 //  - ctx_append_kernel: one warp per appended row: fp64 norm, bf16 key into
 //    ring slot p mod C, token into the token ring (rows: a host-given block,
 //    or the accepted path H_align[i*, 0:L*+1] read through Gamma);
-//  - ctx_bump_kernel: advances the counter after the rows are written;
+//  - ctx_bump_kernel: advances the counter after host-given rows are
+//    written (the accepted path's kernel advances it itself);
 //  - ctx_score_kernel: one warp per (entry, query): fp32 dot product of the
 //    bf16 key and query + delta -> candidate key in the query's pool;
-//  - the exact top-k of the pool is the shared merge; ctx_spans_kernel
-//    turns the winners into positions and spans;
+//  - ctx_pool_kernel (select.cu): the exact top-k of the pool (the shared
+//    merge), then the winners' positions and spans, one block per query;
 //  - hybrid_kernel: one block per query sorts the union of static and
 //    dynamic candidates by (score desc, union index asc), applies the
 //    anchor-first stable partition and the forced anchor, and copies the
@@ -78,33 +79,38 @@ ctx_append_kernel(const uint16_t* __restrict__ hidden, const int32_t* __restrict
   append_row(hidden + (int64_t)i * d, tok[i], (*count + i) % cap, d, keys, ring);
 }
 
-// Accepted path of one step: warp j < n_accept appends H_align[i*, j] (the
-// root state for j = 0, else the state of node Gamma[i*, j-1]) with the
-// accepted token a_j.
-__global__ void __launch_bounds__(256)
+// Accepted path of one step, one block of m warps: warp j < n_accept
+// appends H_align[i*, j] (the root state for j = 0, else the state of node
+// Gamma[i*, j-1]) with the accepted token a_j; then thread 0 advances the
+// counter by n_accept clamped to [0, m].
+__global__ void __launch_bounds__(1024)
 ctx_append_path_kernel(const uint16_t* __restrict__ root, const uint16_t* __restrict__ nodes,
                        int n_nodes, const int32_t* __restrict__ gamma, int k, int m,
                        const int32_t* __restrict__ i_star, const int32_t* __restrict__ n_accept,
-                       const int32_t* __restrict__ accepted, const int64_t* __restrict__ count,
+                       const int32_t* __restrict__ accepted, int64_t* __restrict__ count,
                        int cap, int d, uint16_t* __restrict__ keys, int32_t* __restrict__ ring,
                        uint32_t* status) {
-  const int j = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  pdl_wait();  // the gate's outputs are complete
+  pdl_launch_dependents();
+  const int j = threadIdx.x >> 5;
   const int na = *n_accept, is = *i_star;
-  if (j >= na || j >= m) return;  // warp-uniform
-  if (is < 0 || is >= k || na > m) {
-    if ((threadIdx.x & 31) == 0) raise_status(status, SENSE_DEVST_BAD_INDEX);
-    return;
-  }
-  const uint16_t* x = root;
-  if (j > 0) {
-    const int node = gamma[(int64_t)is * m + j - 1];
-    if (node < 0 || node >= n_nodes) {
-      if ((threadIdx.x & 31) == 0) raise_status(status, SENSE_DEVST_BAD_INDEX);
-      return;
+  const int64_t base = *count;
+  if (j < na && j < m) {  // warp-uniform
+    bool ok = !(is < 0 || is >= k || na > m);
+    const uint16_t* x = root;
+    if (ok && j > 0) {
+      const int node = gamma[(int64_t)is * m + j - 1];
+      if (node < 0 || node >= n_nodes) ok = false;
+      else x = nodes + (int64_t)node * d;
     }
-    x = nodes + (int64_t)node * d;
+    if (!ok) {
+      if ((threadIdx.x & 31) == 0) raise_status(status, SENSE_DEVST_BAD_INDEX);
+    } else {
+      append_row(x, accepted[j], (base + j) % cap, d, keys, ring);
+    }
   }
-  append_row(x, accepted[j], (*count + j) % cap, d, keys, ring);
+  __syncthreads();  // every row read the counter before it moves
+  if (threadIdx.x == 0) *count = base + (na < 0 ? 0 : (na > m ? m : na));
 }
 
 // count += t (host value) or += *t_dev (clamped to [0, m_max]).
@@ -126,11 +132,16 @@ __device__ __forceinline__ void ctx_range_dev(int64_t count, int cap, int m, int
 }
 
 // Grid-stride over (query, entry) pairs, one warp each; also records the
-// number of searchable entries as every query's pool count.
+// number of searchable entries as every query's pool count.  A lane's eight
+// 16-byte key loads of a row piece are issued together; its chunks j = lane,
+// lane + 32, ... are summed in increasing order.
 __global__ void __launch_bounds__(256)
 ctx_score_kernel(const uint16_t* __restrict__ keys, const uint16_t* __restrict__ queries, int q,
                  int d, int cap, int m, const int64_t* __restrict__ count, float delta,
                  uint64_t* __restrict__ pool, uint32_t* __restrict__ counts) {
+  pdl_wait();  // the buffer and the query are complete
+  pdl_launch_dependents();
+  constexpr int kBatch = 8;
   const int lane = threadIdx.x & 31;
   int64_t lo;
   int n_valid;
@@ -138,46 +149,40 @@ ctx_score_kernel(const uint16_t* __restrict__ keys, const uint16_t* __restrict__
   const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
   if (gw < q && lane == 0) counts[gw] = (uint32_t)n_valid;
+  const int chunks = d >> 3;
   for (int64_t w = gw; w < (int64_t)n_valid * q; w += nw) {
     const int qi = (int)(w / n_valid);
     const int e = (int)(w - (int64_t)qi * n_valid);
-    const uint16_t* kr = keys + ((lo + e) % cap) * d;
-    const uint16_t* qr = queries + (int64_t)qi * d;
+    const uint4* kr = reinterpret_cast<const uint4*>(keys + ((lo + e) % cap) * d);
+    const uint4* qr = reinterpret_cast<const uint4*>(queries + (int64_t)qi * d);
     float acc = 0.0f;
-    for (int j = 8 * lane; j < d; j += 256) {
-      const uint4 a = *reinterpret_cast<const uint4*>(kr + j);
-      const uint4 b = *reinterpret_cast<const uint4*>(qr + j);
-      acc = fmaf(bf_lo(a.x), bf_lo(b.x), acc);
-      acc = fmaf(bf_hi(a.x), bf_hi(b.x), acc);
-      acc = fmaf(bf_lo(a.y), bf_lo(b.y), acc);
-      acc = fmaf(bf_hi(a.y), bf_hi(b.y), acc);
-      acc = fmaf(bf_lo(a.z), bf_lo(b.z), acc);
-      acc = fmaf(bf_hi(a.z), bf_hi(b.z), acc);
-      acc = fmaf(bf_lo(a.w), bf_lo(b.w), acc);
-      acc = fmaf(bf_hi(a.w), bf_hi(b.w), acc);
+    for (int j0 = 0; j0 < chunks; j0 += 32 * kBatch) {
+      uint4 kv[kBatch];
+#pragma unroll
+      for (int t = 0; t < kBatch; ++t) {
+        const int j = j0 + 32 * t + lane;
+        kv[t] = j < chunks ? ld_stream_v4(kr + j) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int t = 0; t < kBatch; ++t) {
+        const int j = j0 + 32 * t + lane;
+        if (j < chunks) {
+          const uint4 a = kv[t], b = __ldg(qr + j);
+          acc = fmaf(bf_lo(a.x), bf_lo(b.x), acc);
+          acc = fmaf(bf_hi(a.x), bf_hi(b.x), acc);
+          acc = fmaf(bf_lo(a.y), bf_lo(b.y), acc);
+          acc = fmaf(bf_hi(a.y), bf_hi(b.y), acc);
+          acc = fmaf(bf_lo(a.z), bf_lo(b.z), acc);
+          acc = fmaf(bf_hi(a.z), bf_hi(b.z), acc);
+          acc = fmaf(bf_lo(a.w), bf_lo(b.w), acc);
+          acc = fmaf(bf_hi(a.w), bf_hi(b.w), acc);
+        }
+      }
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
     if (lane == 0) pool[(int64_t)qi * cap + e] = cand_key(acc + delta, (uint32_t)e);
   }
-}
-
-// One thread per (slot, span token).
-__global__ void ctx_spans_kernel(const int32_t* __restrict__ rel, int q, int k,
-                                 const int64_t* __restrict__ count, int cap, int m,
-                                 const int32_t* __restrict__ ring, int64_t* __restrict__ out_pos,
-                                 int32_t* __restrict__ out_spans) {
-  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= (int64_t)q * k * m) return;
-  const int64_t slot = t / m;
-  const int j = (int)(t - slot * m);
-  int64_t lo;
-  int n_valid;
-  ctx_range_dev(*count, cap, m, &lo, &n_valid);
-  const int e = rel[slot];
-  const int64_t p = lo + e;
-  if (j == 0) out_pos[slot] = e < 0 ? -1 : p;
-  out_spans[t] = e < 0 ? -1 : ring[(p + j) % cap];
 }
 
 // One block (1024 threads) per query.  Union index u < ks: static rank u;
@@ -191,6 +196,8 @@ hybrid_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
   __shared__ uint64_t key[kHybridMax];
   __shared__ int dest[kHybridMax];
   __shared__ int n_live;
+  pdl_wait();  // both candidate lists are complete
+  pdl_launch_dependents();
   const int qi = blockIdx.x;
   const int tot = ks + kd;
   int pw = 1;
@@ -373,15 +380,12 @@ sense_status sense_ctx_append_path(sense_ctx* c, const uint16_t* root_hidden,
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  {
-    LaunchScope ls(K_CTX, s);
-    ctx_append_path_kernel<<<(unsigned)((c->m * 32 + 255) / 256), 256, 0, s>>>(
-        root_hidden, node_hidden, n_nodes, gamma, k, c->m, i_star, n_accept, accepted, c->count,
-        c->cap, c->d, c->keys, c->tokens, status);
-  }
   LaunchScope ls(K_CTX, s);
-  ctx_bump_kernel<<<1, 1, 0, s>>>(c->count, 0, n_accept, c->m);
-  return cuda_check(cudaGetLastError(), "launch ctx append path");
+  return cuda_check(launch_pdl(ctx_append_path_kernel, dim3(1), dim3((unsigned)(c->m * 32)), 0, s,
+                               root_hidden, node_hidden, n_nodes, gamma, k, c->m, i_star,
+                               n_accept, accepted, c->count, c->cap, c->d, c->keys, c->tokens,
+                               status),
+                    "launch ctx append path");
 }
 
 size_t sense_ctx_search_workspace_bytes(const sense_ctx* c, int32_t q, int32_t k) {
@@ -416,17 +420,15 @@ sense_status sense_ctx_search(const sense_ctx* c, const uint16_t* queries, int32
     const int64_t want = ((int64_t)q * c->cap * 32 + 255) / 256;
     const int64_t floor_q = ((int64_t)q * 32 + 255) / 256;  // at least one warp per query
     const int64_t blocks = std::max(floor_q, std::min<int64_t>(want, (int64_t)sm_count() * 16));
-    ctx_score_kernel<<<(unsigned)blocks, 256, 0, s>>>(c->keys, queries, q, c->d, c->cap, c->m,
-                                                      c->count, delta, pool, counts);
-    sense_status st = cuda_check(cudaGetLastError(), "launch ctx score");
+    sense_status st = cuda_check(
+        launch_pdl(ctx_score_kernel, dim3((unsigned)blocks), dim3(256), 0, s, c->keys, queries, q,
+                   c->d, c->cap, c->m, (const int64_t*)c->count, delta, pool, counts),
+        "launch ctx score");
     if (st != SENSE_OK) return st;
   }
-  sense_status st = launch_merge_short(pool, counts, c->cap, q, k, out_scores, rel, status, s);
-  if (st != SENSE_OK) return st;
-  LaunchScope ls(K_CTX, s);
-  ctx_spans_kernel<<<(unsigned)(((int64_t)q * k * c->m + 255) / 256), 256, 0, s>>>(
-      rel, q, k, c->count, c->cap, c->m, c->tokens, out_pos, out_spans);
-  return cuda_check(cudaGetLastError(), "launch ctx spans");
+  // top k of each pool, then the winners' positions and spans, one block per query
+  return launch_ctx_pool(pool, counts, c->cap, q, k, out_scores, rel, c->count, c->m, c->tokens,
+                         out_pos, out_spans, status, s);
 }
 
 sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_scores,
@@ -449,10 +451,11 @@ sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_
   if (!status) return SENSE_ERR_OOM;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   LaunchScope ls(K_CTX, s);
-  hybrid_kernel<<<q, 1024, 0, s>>>(ds->spans, ds->n, ds->m, static_scores, static_idx, ks,
-                                   dyn_scores, dyn_spans, kd, anchor, n_keep,
-                                   (flags & SENSE_GATHER_FORCE_ANCHOR) ? 1 : 0, out_spans, status);
-  return cuda_check(cudaGetLastError(), "launch hybrid drafts");
+  return cuda_check(launch_pdl(hybrid_kernel, dim3((unsigned)q), dim3(1024), 0, s,
+                               (const int32_t*)ds->spans, ds->n, ds->m, static_scores, static_idx,
+                               ks, dyn_scores, dyn_spans, kd, anchor, n_keep,
+                               (flags & SENSE_GATHER_FORCE_ANCHOR) ? 1 : 0, out_spans, status),
+                    "launch hybrid drafts");
 }
 
 }  // extern "C"

@@ -104,6 +104,12 @@ sense_status launch_pool_draft(const uint64_t* pool, const uint32_t* counts, int
                                int mask_bits, int32_t* num_nodes, int32_t* tokens,
                                int32_t* parent, int32_t* depth, int32_t* gamma, uint32_t* mask,
                                uint32_t* status, cudaStream_t s);
+// DynSearch's tail: top k of each query's pool of pool_cap (= ring
+// capacity) scored positions, then positions and spans of the winners.
+sense_status launch_ctx_pool(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap, int q,
+                             int k, float* out_scores, int32_t* rel, const int64_t* count, int m,
+                             const int32_t* ring, int64_t* out_pos, int32_t* out_spans,
+                             uint32_t* status, cudaStream_t s);
 // Span gather of k key indices per query and the small-tree trie fused in
 // one kernel per query (draft_fused_fits(k, m)).
 sense_status launch_span_draft(const int32_t* idx, int q, int k, const int32_t* spans, int64_t n,

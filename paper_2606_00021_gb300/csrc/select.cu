@@ -783,6 +783,36 @@ pool_draft_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict_
                    mask, status, q, reinterpret_cast<int*>(s_keys), scratch, sv);
 }
 
+// DynSearch's tail in one block per query: the top k of the query's pool of
+// buffered positions (a short pool padded with -inf / -1), then each
+// winner's absolute position and its span from the token ring.  Entry e of
+// the pool is position lo + e, lo = max(0, count - cap) the oldest position
+// the ring still holds.
+__global__ void __launch_bounds__(kSelThreads, 1)
+ctx_pool_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
+                int64_t pool_cap, int k, float* __restrict__ out_scores,
+                int32_t* __restrict__ rel, const int64_t* __restrict__ count, int m,
+                const int32_t* __restrict__ ring, int64_t* __restrict__ out_pos,
+                int32_t* __restrict__ out_spans, uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];  // [kSmemKeys]
+  const int q = blockIdx.x;
+  pdl_wait();  // the scores are complete
+  pdl_launch_dependents();
+  merge_pool_block(pool, counts, pool_cap, k, out_scores, rel, status, 1, q, s_keys);
+  __syncthreads();
+  const int64_t cnt = *count;
+  const int64_t cap = pool_cap;  // the pool holds one slot per ring position
+  const int64_t lo = cnt > cap ? cnt - cap : 0;
+  for (int t = threadIdx.x; t < k * m; t += blockDim.x) {
+    const int r = t / m, j = t - r * m;
+    const int64_t slot = (int64_t)q * k + r;
+    const int e = rel[slot];
+    const int64_t p = lo + e;
+    if (j == 0) out_pos[slot] = e < 0 ? -1 : p;
+    out_spans[slot * m + j] = e < 0 ? -1 : ring[(p + j) % cap];
+  }
+}
+
 // The span gather of k given key indices and the small-tree trie in one
 // block per query (the tail after a shortlist re-scoring).
 __global__ void __launch_bounds__(kSelThreads, 1)
@@ -889,6 +919,19 @@ sense_status launch_pool_draft(const uint64_t* pool, const uint32_t* counts, int
                               num_nodes, tokens, parent, depth, gamma, mask_bits ? mask : nullptr,
                               status),
                     "launch pool_draft");
+}
+
+sense_status launch_ctx_pool(const uint64_t* pool, const uint32_t* counts, int64_t pool_cap, int q,
+                             int k, float* out_scores, int32_t* rel, const int64_t* count, int m,
+                             const int32_t* ring, int64_t* out_pos, int32_t* out_spans,
+                             uint32_t* status, cudaStream_t s) {
+  sense_status st = set_smem(ctx_pool_kernel, kSmemKeys * sizeof(uint64_t));
+  if (st != SENSE_OK) return st;
+  LaunchScope ls(K_CTX, s);
+  return cuda_check(launch_pdl(ctx_pool_kernel, dim3((unsigned)q), dim3(kSelThreads),
+                              kSmemKeys * sizeof(uint64_t), s, pool, counts, pool_cap, k,
+                              out_scores, rel, count, m, ring, out_pos, out_spans, status),
+                    "launch ctx pool");
 }
 
 sense_status launch_span_draft(const int32_t* idx, int q, int k, const int32_t* spans, int64_t n,

@@ -454,3 +454,70 @@ def test_prepared_calls_follow_buffer_contents(S):
             assert torch.equal(outs[key], want[key]), key
         for key in ("i_star", "L_star", "next_node", "next_anchor", "accepted", "h_next"):
             assert torch.equal(gouts[key], wg[key]), key
+
+
+@cuda
+def test_recorded_calls_follow_buffer_contents(S):
+    """record_calls() marshals a step's calls once (retrieval, hybrid
+    rerank with the dynamic buffer, trie, gate, R.Update): issuing them
+    again on changed query contents gives what fresh calls give, and the
+    recording itself runs nothing."""
+    dev = torch.device("cuda")
+    n, d, m, q, k, kd, cap, v = 30000, 512, 8, 1, 16, 8, 32, 1000
+    keys = synth.clustered_unit_keys(n, d, 64, seed=51, device=dev)
+    spans = synth.spans_uniform(n, m, 6, seed=52, device=dev)
+    ds = S.sense_datastore_build(keys, spans)
+    root = synth.gate_logits(q, 1, v, seed=3, device=dev)[:, 0].contiguous()
+    nodes = synth.gate_logits(q, cap, v, seed=4, device=dev)
+    hr = synth.gate_hidden(q, 1, d, seed=3, device=dev)[:, 0].contiguous()
+    hn = synth.gate_hidden(q, cap, d, seed=4, device=dev)
+
+    def step(ctx, query, anchor, outs):
+        sc, ix = S.sense_retrieve_topk(ds, query, k, outs.get("sc"), outs.get("ix"),
+                                       outs.get("ws"))
+        outs["sc"], outs["ix"] = sc, ix
+        dyn = S.sense_ctx_search(ctx, query, kd, 0.05, outs=outs.setdefault("dyn", {}),
+                                 workspace=outs.get("dws"))
+        dr = S.sense_hybrid_drafts(ds, sc, ix, dyn, anchor, k, True, out=outs.get("dr"))
+        outs["dr"] = dr
+        tr = S.sense_build_tree(dr, node_cap=cap, outs=outs.setdefault("tree", {}))
+        g = S.sense_soft_gate(tr, root, nodes, hr, hn, outs=outs.setdefault("gate", {}),
+                              workspace=outs.get("gws"))
+        S.sense_ctx_append_path(ctx, hr[0], hn[0], tr["gamma"][0], g["i_star"][:1],
+                                g["n_accept"][:1], g["accepted"][0])
+        return outs
+
+    def fresh_ctx():
+        ctx = S.sense_ctx_create(256, d, m)
+        rows = synth.gate_hidden(1, 40, d, seed=9, device=dev)[0].contiguous()
+        S.sense_ctx_append(ctx, rows, torch.arange(40, dtype=torch.int32, device=dev))
+        return ctx
+
+    ctx_a, ctx_b = fresh_ctx(), fresh_ctx()
+    qbuf = torch.zeros(q, d, dtype=torch.bfloat16, device=dev)
+    anchor_a = torch.zeros(q, dtype=torch.int32, device=dev)
+    outs_a = {"ws": S.alloc_workspace(S.sense_retrieve_workspace_bytes(ds, q, k), dev),
+              "dws": S.alloc_workspace(S.lib().sense_ctx_search_workspace_bytes(
+                  __import__("ctypes").c_void_p(ctx_a.handle), q, kd), dev),
+              "gws": S.alloc_workspace(S.sense_soft_gate_workspace_bytes(q, cap, 3), dev)}
+    before = ctx_a.count
+    with S.record_calls() as calls:
+        step(ctx_a, qbuf, anchor_a, outs_a)
+    torch.cuda.synchronize()
+    assert ctx_a.count == before and len(calls) == 6  # nothing ran
+    anchor_b = torch.zeros(q, dtype=torch.int32, device=dev)
+    for seed in (5, 6, 7):
+        qs, _ = synth.noisy_queries(keys, q, seed=seed)
+        qbuf.copy_(qs)
+        for c in calls:
+            c()
+        want = step(ctx_b, qs, anchor_b, {})
+        torch.cuda.synchronize()
+        assert S.sense_device_status(clear=True) == 0
+        for key in ("sc", "ix", "dr"):
+            assert torch.equal(outs_a[key], want[key]), key
+        for key in ("num_nodes", "tokens", "gamma"):
+            assert torch.equal(outs_a["tree"][key], want["tree"][key]), key
+        for key in ("i_star", "n_accept", "accepted", "next_anchor"):
+            assert torch.equal(outs_a["gate"][key], want["gate"][key]), key
+        assert ctx_a.count == ctx_b.count
