@@ -336,7 +336,9 @@ sense_status sense_ivf_search(const sense_ivf* ix, const float* queries, int32_t
  * An index outside [0, n) is treated as empty and sets
  * SENSE_DEVST_BAD_INDEX; a key-row copy that never lands sets
  * SENSE_DEVST_TIMEOUT and drops that warp's remaining candidates.
- * Asynchronous on `stream`.
+ * Asynchronous on `stream`.  A query runs on a cluster of 16 CTAs where the
+ * device can hold one, else 8; SENSE_RESCORE_CLUSTER=8 in the environment
+ * (read once per process) selects 8.
  */
 sense_status sense_rescore_topk(const sense_datastore* ds, const uint16_t* queries, int32_t q,
                                 const int32_t* cand_idx, int32_t n_cand, int32_t k,

@@ -132,16 +132,17 @@ __device__ __forceinline__ void ctx_range_dev(int64_t count, int cap, int m, int
 }
 
 // Grid-stride over (query, entry) pairs, one warp each; also records the
-// number of searchable entries as every query's pool count.  A lane's eight
-// 16-byte key loads of a row piece are issued together; its chunks j = lane,
-// lane + 32, ... are summed in increasing order.
+// number of searchable entries as every query's pool count.  A lane's
+// sixteen 16-byte key loads of a row piece (a whole 4096-dimensional row)
+// are issued together; its chunks j = lane, lane + 32, ... are summed in
+// increasing order.
 __global__ void __launch_bounds__(256)
 ctx_score_kernel(const uint16_t* __restrict__ keys, const uint16_t* __restrict__ queries, int q,
                  int d, int cap, int m, const int64_t* __restrict__ count, float delta,
                  uint64_t* __restrict__ pool, uint32_t* __restrict__ counts) {
   pdl_wait();  // the buffer and the query are complete
   pdl_launch_dependents();
-  constexpr int kBatch = 8;
+  constexpr int kBatch = 16;
   const int lane = threadIdx.x & 31;
   int64_t lo;
   int n_valid;

@@ -34,6 +34,8 @@
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
+#include <cstdlib>
+#include <cstring>
 #include <mutex>
 
 #include "common.cuh"
@@ -303,7 +305,8 @@ using RescoreFn = void (*)(const uint16_t*, int64_t, int, const uint16_t*, const
 constexpr int kMaxDev = 64;
 
 // Cluster width per device: 16 when a cluster of 16 of these CTAs can be
-// resident, else 8 (the portable size).  Attributes are set once.
+// resident, else 8 (the portable size); SENSE_RESCORE_CLUSTER=8 in the
+// environment selects 8 regardless.  Attributes are set once.
 sense_status rescore_setup(int dev, int* width) {
   static std::mutex mu;
   static int widths[kMaxDev] = {0};
@@ -335,10 +338,14 @@ sense_status rescore_setup(int dev, int* width) {
   cfg.numAttrs = 1;
   int nclusters = 0;
   int w = 8;
-  if (cudaOccupancyMaxActiveClusters(&nclusters, fns[2], &cfg) == cudaSuccess && nclusters >= 1)
-    w = 16;
-  else
-    (void)cudaGetLastError();  // the query's failure only means "not 16"
+  const char* force = std::getenv("SENSE_RESCORE_CLUSTER");
+  const bool portable = force && std::strcmp(force, "8") == 0;
+  if (!portable) {
+    if (cudaOccupancyMaxActiveClusters(&nclusters, fns[2], &cfg) == cudaSuccess && nclusters >= 1)
+      w = 16;
+    else
+      (void)cudaGetLastError();  // the query's failure only means "not 16"
+  }
   if (dev >= 0 && dev < kMaxDev) widths[dev] = w;
   *width = w;
   return SENSE_OK;

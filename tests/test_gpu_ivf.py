@@ -194,6 +194,68 @@ def test_ivf_search_matches_oracle(S, n, v, nlist, pq_m, q, k, nprobe):
 
 
 @cuda
+@pytest.mark.parametrize("n,k", [(6000, 600), (3000, 300)])
+def test_ivf_search_equal_scores(S, n, k):
+    """Every vector identical: every candidate ties, so the top k are the k
+    lowest key indices.  Longer pools put more keys in one score bin than
+    the binned selection holds and take the radix path (n = 6000); shorter
+    ones rank a single bucket (n = 3000)."""
+    rng = np.random.default_rng(n)
+    v, nlist = 32, 4
+    one = _unit(rng, 1, v)
+    x = np.repeat(one, n, axis=0).astype(np.float32)
+    cent = _unit(rng, nlist, v)
+    qs = _unit(rng, 2, v)
+    ix = S.sense_ivf_build(_dev(x), _dev(cent))
+    sc, idx = S.sense_ivf_search(ix, _dev(qs), k, nlist)
+    torch.cuda.synchronize()
+    assert S.sense_device_status(clear=True) == 0
+    index = I.ivf_build(x, cent, None)
+    ws, wi, _ = I.ivf_search(index, cent, qs, nlist, k)
+    np.testing.assert_array_equal(host(idx), wi)
+    np.testing.assert_array_equal(host(sc), ws)
+    assert host(idx)[0].tolist() == list(range(k))
+    ix.close()
+
+
+@cuda
+def test_rescore_portable_cluster_width():
+    """The re-scoring kernel's portable cluster width (8 CTAs per query,
+    used where a cluster of 16 cannot be resident), forced through
+    SENSE_RESCORE_CLUSTER in a fresh process: bit-exact on lattice keys at
+    shortlists that need 1, 2 and 4 keys per lane in the per-CTA sort."""
+    import subprocess
+    import sys
+    code = r"""
+import numpy as np, torch, sys
+sys.path.insert(0, '.')
+import paper_2606_00021_gb300 as S, synth
+from oracle import ivf_oracle as I
+from tests.parity import bits, host
+dev = torch.device('cuda')
+n, d, q = 6000, 512, 2
+keys = synth.lattice_rows(n, d, seed=7, device=dev)
+qs = synth.lattice_rows(q, d, seed=8, device=dev)
+ds = S.sense_datastore_build(keys, synth.spans_uniform(n, 2, 50, seed=1, device=dev))
+rng = np.random.default_rng(3)
+for n_cand, k in ((200, 50), (500, 100), (1024, 1024)):
+    cand = np.stack([rng.permutation(n)[:n_cand] for _ in range(q)]).astype(np.int32)
+    sc, ix = S.sense_rescore_topk(ds, qs, torch.from_numpy(cand).to(dev), k)
+    torch.cuda.synchronize()
+    assert S.sense_device_status(clear=True) == 0
+    ws, wi = I.rescore_topk(bits(keys), bits(qs), cand, k)
+    np.testing.assert_array_equal(host(ix), wi)
+    np.testing.assert_array_equal(host(sc).astype(np.float64), ws)
+print('ok')
+"""
+    env = dict(__import__("os").environ, SENSE_RESCORE_CLUSTER="8")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
+                       cwd=os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                       timeout=600)
+    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stderr[-3000:]
+
+
+@cuda
 def test_ivf_golden_on_gpu(S):
     """The hand-worked index, embedded in 16 dimensions: the extra
     coordinates are zero, their codebooks code zero first, and the golden
