@@ -656,13 +656,12 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     ptx::mbar_init(bar(MMA_DONE), 1);
     sh->abort = 0;
     ptx::fence_barrier_init();
-    if (nbl > 0) {  // Q and the first K and V^T tiles go out before the block barrier
+    if (nbl > 0 && (j0 + 1) * kTB <= a.m) {
+      // the first K and V^T tiles go out before the block barrier when they
+      // hold committed keys only (nothing launched before this kernel
+      // writes those); Q waits for the dependency below
       const uint64_t pol_stream = ptx::policy_evict_first();
-      const uint64_t pol_keep = ptx::policy_evict_last();
       const int key0 = j0 * kTB;
-      ptx::mbar_arrive_expect_tx(bar(Q_FULL), kTQBytes);
-      ptx::tma_load_3d(ptx::smem_u32(s_q), &tm_q, bar(Q_FULL), 0, 0, h, pol_keep);
-      ptx::tma_load_3d(ptx::smem_u32(s_q + kTSlabQ), &tm_q, bar(Q_FULL), 64, 0, h, pol_keep);
       ptx::mbar_arrive_expect_tx(bar(K_FULL), kTKBytes);
       ptx::tma_load_3d(ptx::smem_u32(s_k), &tm_k, bar(K_FULL), 0, key0, h, pol_stream);
       ptx::tma_load_3d(ptx::smem_u32(s_k + kTSlab), &tm_k, bar(K_FULL), 64, key0, h, pol_stream);
@@ -676,6 +675,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
+  pdl_launch_dependents();
   const uint32_t tmem = sh->tmem_base;  // S^T buffers at columns kTN b (b < 3), O^T at kTOCol
 
   if (warp == 0 && lane == 0 && nbl > 0) {
@@ -684,31 +684,50 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     // the slot tests do not block (test_wait), so a late V^T slot does not
     // hold back the next K tile or the other way round.
     const uint64_t pol_stream = ptx::policy_evict_first();
-    int jk = 1, jv = 1;  // block 0's tiles and Q were issued with the barriers
+    auto committed = [&](int j) { return (j0 + j + 1) * kTB <= a.m; };
+    auto issue_k = [&](int j) {
+      const int s = j % kTKStages;
+      uint8_t* st = s_k + s * kTKBytes;
+      const int key0 = (j0 + j) * kTB;
+      ptx::mbar_arrive_expect_tx(bar(K_FULL + s), kTKBytes);
+      ptx::tma_load_3d(ptx::smem_u32(st), &tm_k, bar(K_FULL + s), 0, key0, h, pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(st + kTSlab), &tm_k, bar(K_FULL + s), 64, key0, h,
+                       pol_stream);
+    };
+    auto issue_v = [&](int j) {
+      const int s = j % kTVStages;
+      uint8_t* st = s_v + s * kTVBytes;
+      const int key0 = (j0 + j) * kTB;
+      ptx::mbar_arrive_expect_tx(bar(V_FULL + s), kTVBytes);
+      ptx::tma_load_3d(ptx::smem_u32(st), &tm_vt, bar(V_FULL + s), key0, 0, h, pol_stream);
+      ptx::tma_load_3d(ptx::smem_u32(st + kTSlab), &tm_vt, bar(V_FULL + s), key0 + 64, 0, h,
+                       pol_stream);
+    };
+    // block 0's tiles went out with the barriers when committed; the other
+    // free ring slots take further committed blocks before the dependency
+    // wait, everything else (Q, draft keys) after it
+    int jk = committed(0) ? 1 : 0, jv = jk;
+    for (; jk < min(nbl, kTKStages) && committed(jk); ++jk) issue_k(jk);
+    for (; jv < min(nbl, kTVStages) && jv < jk; ++jv) issue_v(jv);
+    pdl_wait();  // Q, the tree's keys and the mask are written
+    ptx::mbar_arrive_expect_tx(bar(Q_FULL), kTQBytes);
+    {
+      const uint64_t pol_keep = ptx::policy_evict_last();
+      ptx::tma_load_3d(ptx::smem_u32(s_q), &tm_q, bar(Q_FULL), 0, 0, h, pol_keep);
+      ptx::tma_load_3d(ptx::smem_u32(s_q + kTSlabQ), &tm_q, bar(Q_FULL), 64, 0, h, pol_keep);
+    }
     long long t0 = clock64();
     while ((jk < nbl || jv < nbl) && !*abort) {
       bool moved = false;
       if (jk < nbl && ptx::mbar_test_wait(bar(K_EMPTY + jk % kTKStages),
                                           (uint32_t)(((jk / kTKStages) & 1) ^ 1))) {
-        const int s = jk % kTKStages;
-        uint8_t* st = s_k + s * kTKBytes;
-        const int key0 = (j0 + jk) * kTB;
-        ptx::mbar_arrive_expect_tx(bar(K_FULL + s), kTKBytes);
-        ptx::tma_load_3d(ptx::smem_u32(st), &tm_k, bar(K_FULL + s), 0, key0, h, pol_stream);
-        ptx::tma_load_3d(ptx::smem_u32(st + kTSlab), &tm_k, bar(K_FULL + s), 64, key0, h,
-                         pol_stream);
+        issue_k(jk);
         ++jk;
         moved = true;
       }
       if (jv < nbl && jv < jk &&
           ptx::mbar_test_wait(bar(V_EMPTY + jv % kTVStages), (uint32_t)(((jv / kTVStages) & 1) ^ 1))) {
-        const int s = jv % kTVStages;
-        uint8_t* st = s_v + s * kTVBytes;
-        const int key0 = (j0 + jv) * kTB;
-        ptx::mbar_arrive_expect_tx(bar(V_FULL + s), kTVBytes);
-        ptx::tma_load_3d(ptx::smem_u32(st), &tm_vt, bar(V_FULL + s), key0, 0, h, pol_stream);
-        ptx::tma_load_3d(ptx::smem_u32(st + kTSlab), &tm_vt, bar(V_FULL + s), key0 + 64, 0, h,
-                         pol_stream);
+        issue_v(jv);
         ++jv;
         moved = true;
       }
@@ -789,6 +808,7 @@ tree_attn_t_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_consta
     ptx::mma_commit(bar(MMA_DONE));
     drain_bar(bar(MMA_DONE), 0);
   } else if (warp >= 2) {
+    pdl_wait();  // the mask and the outputs' previous readers are done
     // ------------------------------------------------ softmax / epilogue
     // Warp w owns TMEM lane quarter q4 = w & 3: keys 32 q4 + lane of a block
     // in S^T, dims 32 q4 + lane in O^T; `tg` = (w - 2) / 4 selects its 16
@@ -1135,13 +1155,15 @@ sense_status launch_attn_t(const uint16_t* q, const uint16_t* k_cache, const uin
     cfg.blockDim = dim3(kTThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 1;
     attr[0].val.clusterDim.y = a.fused ? (unsigned)splits : 1u;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     LaunchScope ls(K_TREE_ATTN, s);
     st = cuda_check(cudaLaunchKernelEx(&cfg, tree_attn_t_kernel, tm_q, tm_k, tm_vt, a),
                     "launch tree attention (transposed)");
