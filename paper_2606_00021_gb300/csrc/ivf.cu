@@ -111,11 +111,10 @@ constexpr long long kBulkWaitCycles = 4000000000LL;
 // copy that never lands (bounded wait) sets SENSE_DEVST_TIMEOUT; the row is
 // then left unwritten.
 template <bool NORM>
-__global__ void __launch_bounds__(256)
-project_bulk_kernel(const uint16_t* __restrict__ x, int d, const float* __restrict__ w, int v,
-                    const float* __restrict__ mu, float* __restrict__ out, uint32_t* status) {
-  pdl_wait();  // inputs written by the kernels before this one
-  pdl_launch_dependents();
+__device__ __forceinline__ void project_bulk_block(const uint16_t* __restrict__ x, int d,
+                                                   const float* __restrict__ w, int v,
+                                                   const float* __restrict__ mu,
+                                                   float* __restrict__ out, uint32_t* status) {
   extern __shared__ __align__(128) uint8_t smb[];
   __shared__ __align__(8) uint64_t bar;
   __shared__ float s_out[8];
@@ -205,6 +204,15 @@ project_bulk_kernel(const uint16_t* __restrict__ x, int d, const float* __restri
     }
     cl.sync();  // the other blocks' shared memory stays alive until it is read
   }
+}
+
+template <bool NORM>
+__global__ void __launch_bounds__(256)
+project_bulk_kernel(const uint16_t* __restrict__ x, int d, const float* __restrict__ w, int v,
+                    const float* __restrict__ mu, float* __restrict__ out, uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
+  project_bulk_block<NORM>(x, d, w, v, mu, out, status);
 }
 
 size_t project_bulk_smem(int d, bool mean) { return (size_t)d * 2 + (mean ? (size_t)d * 4 : 0) + 32 * (size_t)d; }
@@ -471,6 +479,48 @@ coarse_lut_kernel(const float* __restrict__ cells, int64_t nlist, const float* _
   }
 }
 
+// The query side of an approximate search in one launch, per query row:
+// the normalised projection (project_bulk_kernel<true>: the row's blocks
+// form one cluster, block 0 writes the unit row), then, after the cluster
+// barrier that makes that row visible, the cluster's C blocks write the
+// coarse keys of every cell (blocks of 256 cells, the ALL_IP assignment
+// above, block b of the cells taken by cluster block b mod C) and the PQ
+// lookup tables (sub-quantizer m by cluster block m mod C), with the
+// arithmetic of coarse_lut_kernel.  It also empties the row's candidate
+// pool for the list scan (counts[row] = 0).
+template <int D>
+__global__ void __launch_bounds__(256)
+project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __restrict__ w,
+                      const float* __restrict__ mu, float* __restrict__ out,
+                      const float* __restrict__ cells, int64_t nlist,
+                      uint64_t* __restrict__ coarse, const float* __restrict__ cb, int pq_m,
+                      int dsub, float* __restrict__ lut, uint32_t* __restrict__ counts,
+                      uint32_t* status) {
+  pdl_wait();  // inputs written by the kernels before this one
+  pdl_launch_dependents();
+  project_bulk_block<true>(x, d, w, D, mu, out, status);  // ends on a cluster barrier
+  const int64_t row = blockIdx.y;
+  if (blockIdx.x == 0 && threadIdx.x == 0) counts[row] = 0u;  // the list scan's pool is empty
+  const float* qrow = out + row * D;
+  const int C = (int)gridDim.x, r = (int)blockIdx.x;
+  const int nblk = (int)((nlist + blockDim.x - 1) / blockDim.x);
+  for (int b = r; b < nblk; b += C)
+    assign_block<D, ALL_IP, true>(cells, nlist, D, qrow, 1, nullptr, coarse + row * nlist, b);
+  __shared__ float sq[128];
+  for (int m = r; m < pq_m; m += C) {
+    __syncthreads();
+    for (int j = threadIdx.x; j < dsub; j += blockDim.x) sq[j] = qrow[m * dsub + j];
+    __syncthreads();
+    for (int cw = threadIdx.x; cw < 256; cw += blockDim.x) {
+      const int e = m * 256 + cw;
+      const float* bb = cb + (int64_t)e * dsub;
+      float s = 0.0f;
+      for (int j = 0; j < dsub; ++j) s = madd(s, sq[j], bb[j]);
+      lut[row * pq_m * 256 + e] = s;
+    }
+  }
+}
+
 sense_status launch_coarse_lut(const sense_ivf* ix, const float* queries, int q, uint64_t* coarse,
                                float* lut, cudaStream_t s) {
   const int nbc = (ix->nlist + 127) / 128;
@@ -494,6 +544,59 @@ sense_status launch_coarse_lut(const sense_ivf* ix, const float* queries, int q,
   }
 #undef SENSE_COARSE_LUT_CASE
   return cuda_check(e, "launch coarse + lut");
+}
+
+size_t project_bulk_smem(int d, bool mean);
+constexpr size_t kProjectCoarseMax = 180 * 1024;  // + 33 KB static for D = 64
+
+// Launches project_coarse_kernel when the row's projection blocks fit one
+// cluster and its shared memory; *done = false (nothing launched) otherwise.
+sense_status launch_project_coarse(const uint16_t* x, int n, int d, const float* basis,
+                                   const float* mean, float* out, const sense_ivf* ix,
+                                   uint64_t* coarse, float* lut, uint32_t* counts, cudaStream_t s,
+                                   bool* done) {
+  *done = false;
+  const int v = ix->v;
+  const size_t smem = project_bulk_smem(d, mean != nullptr);
+  const bool vdim = v == 4 || v == 8 || v == 16 || v == 32 || v == 64;
+  if (!vdim || n > 64 || (v + 7) / 8 > 8 || smem > kProjectCoarseMax) return SENSE_OK;
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  void (*kern)(const uint16_t*, int, const float*, const float*, float*, const float*, int64_t,
+               uint64_t*, const float*, int, int, float*, uint32_t*, uint32_t*) = nullptr;
+  switch (v) {
+    case 4: kern = project_coarse_kernel<4>; break;
+    case 8: kern = project_coarse_kernel<8>; break;
+    case 16: kern = project_coarse_kernel<16>; break;
+    case 32: kern = project_coarse_kernel<32>; break;
+    default: kern = project_coarse_kernel<64>; break;
+  }
+  sense_status st = cuda_check(func_smem(reinterpret_cast<const void*>(kern), (int)smem),
+                               "cudaFuncSetAttribute(project_coarse)");
+  if (st != SENSE_OK) return st;
+  const int groups = (v + 7) / 8;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)groups, (unsigned)n);
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)groups;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  LaunchScope ls(K_PROJECT, s);
+  st = cuda_check(cudaLaunchKernelEx(&cfg, kern, x, d, basis, mean, out,
+                                     (const float*)ix->centroids, (int64_t)ix->nlist, coarse,
+                                     (const float*)ix->codebooks, ix->pq_m, ix->dsub, lut, counts,
+                                     status),
+                  "launch project + coarse");
+  if (st == SENSE_OK) *done = true;
+  return st;
 }
 
 template <int MODE>
@@ -1170,7 +1273,8 @@ namespace {
 sense_status ivf_scan_pool(const sense_ivf* ix, const float* queries, int32_t q, int32_t k,
                            int32_t nprobe, int32_t* out_probes, void* workspace,
                            size_t workspace_bytes, cudaStream_t s, uint64_t** pool_out,
-                           uint32_t** counts_out, int64_t* pool_cap_out, uint32_t** status_out) {
+                           uint32_t** counts_out, int64_t* pool_cap_out, uint32_t** status_out,
+                           bool coarse_done = false) {
   if (!ix) return fail(SENSE_ERR_INVALID_ARG, "ix is NULL");
   if (!queries || !workspace)
     return fail(SENSE_ERR_INVALID_ARG, "queries, outputs and workspace must be non-NULL");
@@ -1194,9 +1298,14 @@ sense_status ivf_scan_pool(const sense_ivf* ix, const float* queries, int32_t q,
   auto* counts = reinterpret_cast<uint32_t*>(ws + p.off_counts);
   auto* pool = reinterpret_cast<uint64_t*>(ws + p.off_pool);
   auto* lut = reinterpret_cast<float*>(ws + p.off_lut);
-  sense_status st = cuda_check(cudaMemsetAsync(counts, 0, (size_t)q * 4, s), "clear counts");
-  if (st != SENSE_OK) return st;
-  if (ix->pq_m > 0) {  // coarse keys and lookup tables in one launch
+  sense_status st = SENSE_OK;
+  if (coarse_done) {  // coarse keys, tables and empty pools written by project_coarse_kernel
+  } else {
+    st = cuda_check(cudaMemsetAsync(counts, 0, (size_t)q * 4, s), "clear counts");
+    if (st != SENSE_OK) return st;
+  }
+  if (coarse_done) {
+  } else if (ix->pq_m > 0) {  // coarse keys and lookup tables in one launch
     LaunchScope ls(K_IVF_COARSE, s);
     st = launch_coarse_lut(ix, queries, q, coarse, lut, s);
     if (st != SENSE_OK) return st;
@@ -1303,35 +1412,42 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
   const int cap = node_cap > 0 ? node_cap : k * m;
   const bool fused = draft_fused_fits(k, m);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // query construction (Alg. 2: k = L2Norm(PCA(h))), search, optional
-  // exact re-scoring (Eq. 8), gather and trie
-  sense_status st = sense_project(queries, q, ds->d, basis, ix->v, mean, SENSE_PROJECT_NORMALIZE,
-                                  qproj, stream);
+  if (!aligned(queries, 16) || !aligned(basis, 16) || (mean && !aligned(mean, 16)))
+    return fail(SENSE_ERR_INVALID_ARG, "queries, basis and mean must be 16-byte aligned");
+  // query construction (Alg. 2: k = L2Norm(PCA(h))) with the coarse keys and
+  // lookup tables in the same launch when it fits, search, optional exact
+  // re-scoring (Eq. 8), gather and trie
+  const SearchPlan plan = search_plan(ix, q, nprobe);
+  bool coarse_done = false;
+  sense_status st = launch_project_coarse(
+      queries, q, ds->d, basis, mean, qproj, ix, reinterpret_cast<uint64_t*>(ws + plan.off_coarse),
+      reinterpret_cast<float*>(ws + plan.off_lut), reinterpret_cast<uint32_t*>(ws + plan.off_counts),
+      s, &coarse_done);
   if (st != SENSE_OK) return st;
-  if (rerank == 0 && fused) {  // pool merge, gather and trie in one kernel per query
-    uint64_t* pool = nullptr;
-    uint32_t* counts = nullptr;
-    uint32_t* status = nullptr;
-    int64_t pool_cap = 0;
-    st = ivf_scan_pool(ix, qproj, q, k, nprobe, nullptr, ws, ivf_bytes, s, &pool, &counts,
-                       &pool_cap, &status);
+  if (!coarse_done) {
+    st = sense_project(queries, q, ds->d, basis, ix->v, mean, SENSE_PROJECT_NORMALIZE, qproj,
+                       stream);
     if (st != SENSE_OK) return st;
+  }
+  uint64_t* pool = nullptr;
+  uint32_t* counts = nullptr;
+  uint32_t* status = nullptr;
+  int64_t pool_cap = 0;
+  st = ivf_scan_pool(ix, qproj, q, rerank > 0 ? rerank : k, nprobe, nullptr, ws, ivf_bytes, s,
+                     &pool, &counts, &pool_cap, &status, coarse_done);
+  if (st != SENSE_OK) return st;
+  if (rerank == 0 && fused)  // pool merge, gather and trie in one kernel per query
     return launch_pool_draft(pool, counts, pool_cap, q, k, out_scores, out_idx, ds->spans, ds->n,
                              m, out_spans, cap, bits ? 1 : 0, out_num_nodes, out_tokens,
                              out_parent, out_depth, out_gamma, out_mask_bits, status, s);
-  }
   if (rerank > 0) {
-    st = sense_ivf_search(ix, qproj, q, rerank, nprobe, cand_s, cand_i, nullptr, ws, ivf_bytes,
-                          stream);
+    st = launch_merge_short(pool, counts, pool_cap, q, rerank, cand_s, cand_i, status, s);
     if (st != SENSE_OK) return st;
     st = sense_rescore_topk(ds, queries, q, cand_i, rerank, k, out_scores, out_idx, stream);
   } else {
-    st = sense_ivf_search(ix, qproj, q, k, nprobe, out_scores, out_idx, nullptr, ws, ivf_bytes,
-                          stream);
+    st = launch_merge_short(pool, counts, pool_cap, q, k, out_scores, out_idx, status, s);
   }
   if (st != SENSE_OK) return st;
-  uint32_t* status = device_status_word();
-  if (!status) return SENSE_ERR_OOM;
   if (fused)  // gather and trie in one kernel per query
     return launch_span_draft(out_idx, q, k, ds->spans, ds->n, m, out_spans, cap, bits ? 1 : 0,
                              out_num_nodes, out_tokens, out_parent, out_depth, out_gamma,
