@@ -35,6 +35,11 @@
 //                        histograms, a column scan, one warp placing each
 //                        block's ids in order)
 //  pq_encode_kernel      residual sub-vector -> nearest of 256 codewords
+//  coarse_lut_kernel     a search's coarse keys and PQ lookup tables in one
+//                        launch (blocks of cells, then blocks of codebooks)
+//  project_coarse_kernel the approximate drafting step's query side: the
+//                        normalised projection cluster, then its blocks
+//                        write the coarse keys and lookup tables
 //  ivf_scan_kernel       one block per (probe, query): flat dot products or
 //                        LUT sums, candidates appended to the query's pool;
 //                        the exact top-k of the pool is the existing merge.
