@@ -428,6 +428,7 @@ def build_ann(S, keys, kind, nlist, nprobe, pq_m, v, dev, seed=0):
 
 
 SLICE_ROWS = 65536  # rows per sampled slice of the store (one generator chunk)
+REF_BUDGET_S = 150.0  # --impl reference: oracle time of the whole run, about
 
 
 def _oracle_query(O, cfg, kb_slices, row_ids, qb, spans_h, gate_h):
@@ -532,13 +533,29 @@ def run_reference(args, cfg, name):
     spans_h = _host(spans)
     del spans, store
     gate_h = _gate_host(make_gate_inputs(cfg, dev, sets=1, seed=100)[0])
-    t_scan, t_down, t_step, rows_per = [], [], [], []
     total = args.warmup + args.steps
+    # rows per step: --ref-slices slices, fewer when the whole run would
+    # exceed about REF_BUDGET_S (one untimed calibration step sizes it)
+    c0 = pool_ids[0]
+    ts1, td1 = _oracle_query(O, cfg, [pool[c0]], np.arange(c0 * synth.CHUNK_ROWS,
+                                                           c0 * synth.CHUNK_ROWS + pool[c0].shape[0]),
+                             _bits(queries[0]), spans_h, gate_h)
+    per_row = ts1 / pool[c0].shape[0]
+    step_budget = REF_BUDGET_S / total
+    rows_cap = per_step * SLICE_ROWS
+    rows_step = int(min(rows_cap, max(4096, (step_budget - td1) / max(per_row, 1e-12))))
+    t_scan, t_down, t_step, rows_per = [], [], [], []
     for it in range(total):
         ids = [pool_ids[(it * per_step + j) % len(pool_ids)] for j in range(per_step)]
-        kbs = [pool[c] for c in ids]
-        row_ids = np.concatenate([np.arange(c * synth.CHUNK_ROWS,
-                                            c * synth.CHUNK_ROWS + pool[c].shape[0]) for c in ids])
+        kbs, row_ids, left = [], [], rows_step
+        for c in ids:
+            if left <= 0:
+                break
+            r = min(left, pool[c].shape[0])
+            kbs.append(pool[c][:r])
+            row_ids.append(np.arange(c * synth.CHUNK_ROWS, c * synth.CHUNK_ROWS + r))
+            left -= r
+        row_ids = np.concatenate(row_ids)
         qb = _bits(queries[it % cfg["distinct"]])
         t0 = time.perf_counter()
         ts, td = _oracle_query(O, cfg, kbs, row_ids, qb, spans_h, gate_h)
@@ -562,11 +579,13 @@ def run_reference(args, cfg, name):
         "cpu_baseline": {"value": value, "unit": "queries/s", "cores": os.cpu_count(),
                          "kind": "oracle",
                          "sample": (f"per step: one batch of {q} query(ies) of the workload "
-                                    f"scored against {per_step} seeded {SLICE_ROWS}-row slices "
-                                    f"of its store ({int(rows)} of {n} keys), top-k of that "
-                                    f"sample, gather/trie/gate; ms_per_step is that sampled "
-                                    f"step; value scales scoring + top-k by n/rows = "
-                                    f"{scale:.1f}; numpy fp64"),
+                                    f"scored against {int(rows)} of its {n} keys (seeded "
+                                    f"{SLICE_ROWS}-row slices of the store, at most "
+                                    f"{per_step}, fewer rows when {total} steps would exceed "
+                                    f"~{REF_BUDGET_S:.0f} s), top-k of that sample, "
+                                    f"gather/trie/gate; ms_per_step is that sampled step; "
+                                    f"value scales scoring + top-k by n/rows = {scale:.1f}; "
+                                    f"numpy fp64"),
                          "scan_s_per_step": statistics.mean(t_scan),
                          "downstream_s_per_step": statistics.mean(t_down)},
         "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
