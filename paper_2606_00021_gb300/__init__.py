@@ -217,9 +217,9 @@ def sense_retrieve_topk(ds: Datastore, queries: torch.Tensor, k: int, out_scores
     if workspace is None:
         workspace = alloc_workspace(need, dev)
     _call(lib().sense_retrieve_topk, C.c_void_p(ds.handle), queries.data_ptr(), q, k,
-                                     out_scores.data_ptr(), out_idx.data_ptr(),
-                                     workspace.data_ptr(), workspace.numel(),
-                                     C.c_void_p(_stream(stream)))
+          out_scores.data_ptr(), out_idx.data_ptr(),
+          workspace.data_ptr(), workspace.numel(),
+          C.c_void_p(_stream(stream)))
     return out_scores, out_idx
 
 
@@ -279,8 +279,8 @@ def sense_rescore_topk(ds: Datastore, queries: torch.Tensor, cand_idx: torch.Ten
     if out_idx is None:
         out_idx = _i32((q, k), dev)
     _call(lib().sense_rescore_topk, C.c_void_p(ds.handle), queries.data_ptr(), q,
-                                    cand_idx.data_ptr(), n_cand, k, out_scores.data_ptr(),
-                                    out_idx.data_ptr(), C.c_void_p(_stream(stream)))
+          cand_idx.data_ptr(), n_cand, k, out_scores.data_ptr(),
+          out_idx.data_ptr(), C.c_void_p(_stream(stream)))
     return out_scores, out_idx
 
 
@@ -295,8 +295,8 @@ def sense_gather_drafts(ds: Datastore, idx: torch.Tensor, anchor=None, n_keep=No
     if out is None:
         out = _i32((q, keep, ds.m), idx.device)
     _call(lib().sense_gather_drafts, C.c_void_p(ds.handle), idx.data_ptr(), q, k, _ptr(anchor),
-                                     keep, 1 if force_anchor else 0, out.data_ptr(),
-                                     C.c_void_p(_stream(stream)))
+          keep, 1 if force_anchor else 0, out.data_ptr(),
+          C.c_void_p(_stream(stream)))
     return out
 
 
@@ -317,10 +317,10 @@ def sense_build_tree(spans: torch.Tensor, node_cap: int = 0, mask_bits: bool = F
         o.setdefault("mask_bits", torch.empty(q, cap, (cap + 31) // 32, dtype=torch.int32,
                                               device=dev))
     _call(lib().sense_build_tree, spans.data_ptr(), q, k, m, node_cap, 1 if mask_bits else 0,
-                                  o["num_nodes"].data_ptr(), o["tokens"].data_ptr(),
-                                  o["parent"].data_ptr(), o["depth"].data_ptr(),
-                                  o["gamma"].data_ptr(), _ptr(o.get("mask_bits")),
-                                  C.c_void_p(_stream(stream)))
+          o["num_nodes"].data_ptr(), o["tokens"].data_ptr(),
+          o["parent"].data_ptr(), o["depth"].data_ptr(),
+          o["gamma"].data_ptr(), _ptr(o.get("mask_bits")),
+          C.c_void_p(_stream(stream)))
     o["cap"] = cap
     return o
 
@@ -379,8 +379,8 @@ def sense_tree_mask_full(tree: dict, prefix_len: torch.Tensor, cache_len: int,
         out = torch.empty(q, cap, cache_len, dtype=torch.float32, device=bits.device)
     _need(out, "out", torch.float32, 3)
     _call(lib().sense_tree_mask_full, bits.data_ptr(), tree["num_nodes"].data_ptr(), q, cap,
-                                      prefix_len.data_ptr(), cache_len, out.data_ptr(),
-                                      C.c_void_p(_stream(stream)))
+          prefix_len.data_ptr(), cache_len, out.data_ptr(),
+          C.c_void_p(_stream(stream)))
     return out
 
 
@@ -403,8 +403,8 @@ def sense_project(x: torch.Tensor, basis: torch.Tensor, mean: torch.Tensor | Non
         out = torch.empty(n, v, dtype=torch.float32, device=x.device)
     _need(out, "out", torch.float32, 2)
     _call(lib().sense_project, x.data_ptr(), n, d, basis.data_ptr(), v, _ptr(mean),
-                               1 if normalize else 0, out.data_ptr(),
-                               C.c_void_p(_stream(stream)))
+          1 if normalize else 0, out.data_ptr(),
+          C.c_void_p(_stream(stream)))
     return out
 
 
@@ -567,9 +567,9 @@ def sense_ivf_search(ix: IvfIndex, queries: torch.Tensor, k: int, nprobe: int,
     if workspace is None:
         workspace = alloc_workspace(sense_ivf_search_workspace_bytes(ix, q, k, nprobe), dev)
     _call(lib().sense_ivf_search, C.c_void_p(ix.handle), queries.data_ptr(), q, k, nprobe,
-                                  out_scores.data_ptr(), out_idx.data_ptr(), _ptr(probes),
-                                  workspace.data_ptr(), workspace.numel(),
-                                  C.c_void_p(_stream(stream)))
+          out_scores.data_ptr(), out_idx.data_ptr(), _ptr(probes),
+          workspace.data_ptr(), workspace.numel(),
+          C.c_void_p(_stream(stream)))
     return (out_scores, out_idx, probes) if want_probes else (out_scores, out_idx)
 
 
@@ -619,7 +619,7 @@ def sense_ctx_append(ctx: ContextBuffer, hidden: torch.Tensor, tokens: torch.Ten
     if hidden.shape[0] != tokens.shape[0] or hidden.shape[1] != ctx.d:
         raise ValueError("hidden must be [t, d] and tokens [t]")
     _call(lib().sense_ctx_append, C.c_void_p(ctx.handle), hidden.data_ptr(), tokens.data_ptr(),
-                                  hidden.shape[0], C.c_void_p(_stream(stream)))
+          hidden.shape[0], C.c_void_p(_stream(stream)))
 
 
 def sense_ctx_append_path(ctx: ContextBuffer, root_hidden: torch.Tensor,
@@ -634,10 +634,10 @@ def sense_ctx_append_path(ctx: ContextBuffer, root_hidden: torch.Tensor,
     for t, name in ((i_star, "i_star"), (n_accept, "n_accept"), (accepted, "accepted")):
         _need(t, name, torch.int32, 1)
     _call(lib().sense_ctx_append_path, C.c_void_p(ctx.handle), root_hidden.data_ptr(),
-                                       node_hidden.data_ptr(), node_hidden.shape[0],
-                                       gamma.data_ptr(), gamma.shape[0], i_star.data_ptr(),
-                                       n_accept.data_ptr(), accepted.data_ptr(),
-                                       C.c_void_p(_stream(stream)))
+          node_hidden.data_ptr(), node_hidden.shape[0],
+          gamma.data_ptr(), gamma.shape[0], i_star.data_ptr(),
+          n_accept.data_ptr(), accepted.data_ptr(),
+          C.c_void_p(_stream(stream)))
 
 
 def sense_ctx_search(ctx: ContextBuffer, queries: torch.Tensor, k: int, delta: float = 0.0,
@@ -654,9 +654,9 @@ def sense_ctx_search(ctx: ContextBuffer, queries: torch.Tensor, k: int, delta: f
         workspace = alloc_workspace(lib().sense_ctx_search_workspace_bytes(
             C.c_void_p(ctx.handle), q, k), dev)
     _call(lib().sense_ctx_search, C.c_void_p(ctx.handle), queries.data_ptr(), q, k,
-                                  C.c_float(delta), o["scores"].data_ptr(), o["pos"].data_ptr(),
-                                  o["spans"].data_ptr(), workspace.data_ptr(), workspace.numel(),
-                                  C.c_void_p(_stream(stream)))
+          C.c_float(delta), o["scores"].data_ptr(), o["pos"].data_ptr(),
+          o["spans"].data_ptr(), workspace.data_ptr(), workspace.numel(),
+          C.c_void_p(_stream(stream)))
     return o
 
 
@@ -675,11 +675,11 @@ def sense_hybrid_drafts(ds: Datastore, static_scores: torch.Tensor, static_idx: 
     if out is None:
         out = _i32((q, keep, ds.m), static_idx.device)
     _call(lib().sense_hybrid_drafts, C.c_void_p(ds.handle), static_scores.data_ptr(),
-                                     static_idx.data_ptr(), ks,
-                                     None if dyn is None else dyn["scores"].data_ptr(),
-                                     None if dyn is None else dyn["spans"].data_ptr(), kd, q,
-                                     _ptr(anchor), keep, 1 if force_anchor else 0,
-                                     out.data_ptr(), C.c_void_p(_stream(stream)))
+          static_idx.data_ptr(), ks,
+          None if dyn is None else dyn["scores"].data_ptr(),
+          None if dyn is None else dyn["spans"].data_ptr(), kd, q,
+          _ptr(anchor), keep, 1 if force_anchor else 0,
+          out.data_ptr(), C.c_void_p(_stream(stream)))
     return out
 
 
@@ -702,10 +702,10 @@ def sense_tree_attention(q: torch.Tensor, k_cache: torch.Tensor, vt_cache: torch
         workspace = alloc_workspace(
             lib().sense_tree_attention_workspace_bytes(heads, L, prefix_len), q.device)
     _call(lib().sense_tree_attention, q.data_ptr(), k_cache.data_ptr(), vt_cache.data_ptr(), heads,
-                                      L, dh, cap, prefix_len, mask_bits.data_ptr(),
-                                      mask_bits.shape[1], C.c_float(scale), out.data_ptr(),
-                                      workspace.data_ptr(), workspace.numel(),
-                                      C.c_void_p(_stream(stream)))
+          L, dh, cap, prefix_len, mask_bits.data_ptr(),
+          mask_bits.shape[1], C.c_float(scale), out.data_ptr(),
+          workspace.data_ptr(), workspace.numel(),
+          C.c_void_p(_stream(stream)))
     return out
 
 
