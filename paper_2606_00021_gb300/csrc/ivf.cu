@@ -50,6 +50,7 @@
 
 #include "common.cuh"
 #include "launch.h"
+#include "select_dev.cuh"
 #include "tc_ptx.cuh"
 
 struct sense_ivf {
@@ -492,7 +493,9 @@ coarse_lut_kernel(const float* __restrict__ cells, int64_t nlist, const float* _
 // above, block b of the cells taken by cluster block b mod C) and the PQ
 // lookup tables (sub-quantizer m by cluster block m mod C), with the
 // arithmetic of coarse_lut_kernel.  It also empties the row's candidate
-// pool for the list scan (counts[row] = 0).
+// pool for the list scan (counts[row] = 0).  After a second cluster barrier
+// block 0 selects the row's nprobe best cells from the coarse keys (the
+// block merge of merge_kernel, in the projection's shared memory).
 template <int D>
 __global__ void __launch_bounds__(256)
 project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __restrict__ w,
@@ -500,7 +503,8 @@ project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __rest
                       const float* __restrict__ cells, int64_t nlist,
                       uint64_t* __restrict__ coarse, const float* __restrict__ cb, int pq_m,
                       int dsub, float* __restrict__ lut, uint32_t* __restrict__ counts,
-                      uint32_t* status) {
+                      int nprobe, float* __restrict__ pscore, int32_t* __restrict__ pcell,
+                      int smem_keys, uint32_t* status) {
   pdl_wait();  // inputs written by the kernels before this one
   pdl_launch_dependents();
   project_bulk_block<true>(x, d, w, D, mu, out, status);  // ends on a cluster barrier
@@ -523,6 +527,12 @@ project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __rest
       for (int j = 0; j < dsub; ++j) s = madd(s, sq[j], bb[j]);
       lut[row * pq_m * 256 + e] = s;
     }
+  }
+  cooperative_groups::this_cluster().sync();  // every block's coarse keys are written
+  if (r == 0) {
+    extern __shared__ __align__(128) uint8_t smb_keys[];
+    merge_pool_block(coarse, nullptr, nlist, nprobe, pscore, pcell, status, 0, (int)row,
+                     reinterpret_cast<uint64_t*>(smb_keys), smem_keys);
   }
 }
 
@@ -552,23 +562,25 @@ sense_status launch_coarse_lut(const sense_ivf* ix, const float* queries, int q,
 }
 
 size_t project_bulk_smem(int d, bool mean);
-constexpr size_t kProjectCoarseMax = 180 * 1024;  // + 33 KB static for D = 64
+constexpr size_t kProjectCoarseMax = 172 * 1024;  // + 51 KB static for D = 64 (<= 227 KB)
 
 // Launches project_coarse_kernel when the row's projection blocks fit one
 // cluster and its shared memory; *done = false (nothing launched) otherwise.
 sense_status launch_project_coarse(const uint16_t* x, int n, int d, const float* basis,
                                    const float* mean, float* out, const sense_ivf* ix,
-                                   uint64_t* coarse, float* lut, uint32_t* counts, cudaStream_t s,
-                                   bool* done) {
+                                   uint64_t* coarse, float* lut, uint32_t* counts, int nprobe,
+                                   float* pscore, int32_t* pcell, cudaStream_t s, bool* done) {
   *done = false;
   const int v = ix->v;
-  const size_t smem = project_bulk_smem(d, mean != nullptr);
+  // the shared memory also stages the row's coarse keys for the cell selection
+  const size_t smem = std::max(project_bulk_smem(d, mean != nullptr), (size_t)ix->nlist * 8);
   const bool vdim = v == 4 || v == 8 || v == 16 || v == 32 || v == 64;
   if (!vdim || n > 64 || (v + 7) / 8 > 8 || smem > kProjectCoarseMax) return SENSE_OK;
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
   void (*kern)(const uint16_t*, int, const float*, const float*, float*, const float*, int64_t,
-               uint64_t*, const float*, int, int, float*, uint32_t*, uint32_t*) = nullptr;
+               uint64_t*, const float*, int, int, float*, uint32_t*, int, float*, int32_t*, int,
+               uint32_t*) = nullptr;
   switch (v) {
     case 4: kern = project_coarse_kernel<4>; break;
     case 8: kern = project_coarse_kernel<8>; break;
@@ -598,7 +610,7 @@ sense_status launch_project_coarse(const uint16_t* x, int n, int d, const float*
   st = cuda_check(cudaLaunchKernelEx(&cfg, kern, x, d, basis, mean, out,
                                      (const float*)ix->centroids, (int64_t)ix->nlist, coarse,
                                      (const float*)ix->codebooks, ix->pq_m, ix->dsub, lut, counts,
-                                     status),
+                                     nprobe, pscore, pcell, (int)(smem / 8), status),
                   "launch project + coarse");
   if (st == SENSE_OK) *done = true;
   return st;
@@ -1321,8 +1333,10 @@ sense_status ivf_scan_pool(const sense_ivf* ix, const float* queries, int32_t q,
                                     coarse, s);
     if (st != SENSE_OK) return st;
   }
-  st = launch_merge(coarse, nullptr, ix->nlist, q, nprobe, pscore, pcell, status, s);
-  if (st != SENSE_OK) return st;
+  if (!coarse_done) {  // else the best cells were selected with the coarse keys
+    st = launch_merge(coarse, nullptr, ix->nlist, q, nprobe, pscore, pcell, status, s);
+    if (st != SENSE_OK) return st;
+  }
   {
     const size_t smem = scan_smem_bytes(ix);
     st = cuda_check(func_smem(reinterpret_cast<const void*>(ivf_scan_kernel), (int)smem), "smem attribute");
@@ -1427,7 +1441,8 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
   sense_status st = launch_project_coarse(
       queries, q, ds->d, basis, mean, qproj, ix, reinterpret_cast<uint64_t*>(ws + plan.off_coarse),
       reinterpret_cast<float*>(ws + plan.off_lut), reinterpret_cast<uint32_t*>(ws + plan.off_counts),
-      s, &coarse_done);
+      nprobe, reinterpret_cast<float*>(ws + plan.off_pscore),
+      reinterpret_cast<int32_t*>(ws + plan.off_pcell), s, &coarse_done);
   if (st != SENSE_OK) return st;
   if (!coarse_done) {
     st = sense_project(queries, q, ds->d, basis, ix->v, mean, SENSE_PROJECT_NORMALIZE, qproj,
