@@ -215,16 +215,31 @@ __device__ void tree_small_block(const int32_t* __restrict__ spans, int k, int m
     s_lcp[p] = l;
   }
   __syncthreads();
-  //    bases: nodes created by sorted rows before p; nodes first reached by ranks before r
-  for (int i = threadIdx.x; i < k; i += blockDim.x) {
-    int b = 0, pr = 0;
-    for (int t = 0; t < i; ++t) {
-      b += m - s_lcp[t];
-      pr += m - s_mll[t];
+  //    bases: nodes created by sorted rows before p; nodes first reached by
+  //    ranks before r (exclusive prefix sums by warp 0, 32 rows a step)
+  if (wid == 0) {
+    int cb = 0, cp = 0;  // sums of the rows before this step's
+    for (int i0 = 0; i0 < k; i0 += 32) {
+      const int i = i0 + lane;
+      const int vb = i < k ? m - s_lcp[i] : 0, vp = i < k ? m - s_mll[i] : 0;
+      int xb = vb, xp = vp;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int tb = __shfl_up_sync(0xffffffffu, xb, off);
+        const int tp = __shfl_up_sync(0xffffffffu, xp, off);
+        if (lane >= off) {
+          xb += tb;
+          xp += tp;
+        }
+      }
+      if (i < k) {
+        s_base[i] = cb + xb - vb;
+        s_pre[i] = cp + xp - vp;
+      }
+      cb += __shfl_sync(0xffffffffu, xb, 31);
+      cp += __shfl_sync(0xffffffffu, xp, 31);
     }
-    s_base[i] = b;
-    s_pre[i] = pr;
-    if (i == k - 1) s_total = b + m - s_lcp[i];
+    if (lane == 0) s_total = cb;
   }
   __syncthreads();
   const int U = s_total;
