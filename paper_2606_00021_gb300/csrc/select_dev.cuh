@@ -135,17 +135,18 @@ __device__ bool merge_pool_short(const uint64_t* s_keys, int cnt, int k, int pad
     s_t = 0ull;
     s_got = 0u;
   }
-  // heads: group maxima, sorted descending within each group of 32 heads
+  // heads: group maxima (every warp takes groups in turn), then sorted
+  // descending within each group of 32 heads; groups past the pool are 0
   const int nhg = (ngr + 31) >> 5;
+  for (int g = warp; g < ngr; g += nwarps) {
+    const int i = g * 32 + lane;
+    const uint64_t m = warp_max64(i < cnt ? s_keys[i] : 0ull);
+    if (lane == 0) s_heads[g] = m;
+  }
+  for (int g = ngr + threadIdx.x; g < nhg * 32; g += blockDim.x) s_heads[g] = 0ull;
+  __syncthreads();
   for (int hg = warp; hg < nhg; hg += nwarps) {
-    uint64_t h = 0ull;  // the maximum of group hg * 32 + lane
-    for (int u = 0; u < 32; ++u) {  // group g's keys, read across the warp by lane u's group
-      const int gu = hg * 32 + u;
-      const int i = gu * 32 + lane;
-      const uint64_t x = (gu < ngr && i < cnt) ? s_keys[i] : 0ull;
-      const uint64_t m = warp_max64(x);
-      if (lane == u) h = m;
-    }
+    uint64_t h = s_heads[hg * 32 + lane];
 #pragma unroll
     for (int size = 2; size <= 32; size <<= 1) {
 #pragma unroll
