@@ -313,14 +313,16 @@ class Pipeline:
                                           node_cap=cfg["cap"], mask_bits=ver is not None,
                                           outs=outs, workspace=self.ann_ws)
                 else:
+                    # static retrieval, then DynSearch, the hybrid rerank and the
+                    # trie in one call
                     self.retrieve(query)
-                    S.sense_ctx_search(dyn["ctx"], query, dyn["kd"], dyn["delta"],
-                                       outs=dyn["outs"], workspace=dyn["ws"])
-                    S.sense_hybrid_drafts(self.ds, self.scores, self.idx, dyn["outs"],
-                                          self.gate["next_anchor"], cfg["k"], True,
-                                          out=self.drafts)
-                    S.sense_build_tree(self.drafts, node_cap=cfg["cap"],
-                                       mask_bits=ver is not None, outs=self.tree)
+                    outs = self.tree
+                    outs["dyn"], outs["spans"] = dyn["outs"], self.drafts
+                    S.sense_dyn_draft(self.ds, dyn["ctx"], query, self.scores, self.idx,
+                                      dyn["kd"], dyn["delta"], self.gate["next_anchor"],
+                                      cfg["k"], True, node_cap=cfg["cap"],
+                                      mask_bits=ver is not None, outs=outs,
+                                      workspace=dyn["ws"])
                 if ver is not None:
                     S.sense_tree_attention(ver["q"], ver["k"], ver["vt"], ver["prefix"],
                                            self.tree["mask_bits"][0], ver["scale"], out=ver["out"],

@@ -486,6 +486,32 @@ sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_
                                  const int32_t* anchor, int32_t n_keep, uint32_t flags,
                                  int32_t* out_spans, sense_stream_t stream);
 
+/*
+ * The hybrid drafting step's buffer side and tail in one call (Alg. 2:
+ * DynSearch over the buffer with the delta boost, the union D_all with the
+ * static results reranked by Eq. 8, then the Sec. 3.2.3 Eq. 9 loose trie of
+ * the kept rows): the results, bit for bit, of sense_ctx_search(ctx,
+ * queries, q, kd, delta) into dyn_scores [q, kd] f32, dyn_pos [q, kd] int64,
+ * dyn_spans [q, kd, m] int32, then sense_hybrid_drafts(ds, static_scores,
+ * static_idx, ks, ..., anchor, n_keep, flags) into out_spans [q, n_keep, m],
+ * then sense_build_tree(out_spans, q, n_keep, m, node_cap, tree_flags) into
+ * the tree outputs (as sense_build_tree).  The datastore and the buffer
+ * share d and m.  workspace: sense_ctx_search_workspace_bytes(ctx, q, kd)
+ * bytes, 256-byte aligned.  When n_keep <= 128 (and the trie fits shared
+ * memory) it is two kernels: the buffer's scores, then one block per query
+ * for the rest; otherwise the three calls' launches.  Errors and device
+ * status are those of the composed calls.
+ */
+sense_status sense_dyn_draft(const sense_datastore* ds, const sense_ctx* ctx,
+                             const uint16_t* queries, int32_t q, const float* static_scores,
+                             const int32_t* static_idx, int32_t ks, int32_t kd, float delta,
+                             const int32_t* anchor, int32_t n_keep, uint32_t flags,
+                             int32_t node_cap, uint32_t tree_flags, void* workspace,
+                             size_t workspace_bytes, float* dyn_scores, int64_t* dyn_pos,
+                             int32_t* dyn_spans, int32_t* out_spans, int32_t* out_num_nodes,
+                             int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
+                             int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream);
+
 /* ---------------------------------------------------------------------- */
 /* a5. Loose trie (draft tree)                                              */
 /* ---------------------------------------------------------------------- */

@@ -683,6 +683,54 @@ def sense_hybrid_drafts(ds: Datastore, static_scores: torch.Tensor, static_idx: 
     return out
 
 
+def sense_dyn_draft(ds: Datastore, ctx: ContextBuffer, queries: torch.Tensor,
+                    static_scores: torch.Tensor, static_idx: torch.Tensor, kd: int,
+                    delta: float = 0.0, anchor: torch.Tensor | None = None,
+                    n_keep: int | None = None, force_anchor: bool = False, node_cap: int = 0,
+                    mask_bits: bool = False, outs: dict | None = None, workspace=None,
+                    stream=None) -> dict:
+    """DynSearch, the hybrid rerank and the loose trie in one call: the dict
+    of sense_ctx_search's outputs ("dyn": scores, pos, spans), the kept
+    drafts ("spans" [q, n_keep, m]) and the tree (as sense_build_tree)."""
+    _need(queries, "queries", torch.bfloat16, 2)
+    _need(static_scores, "static_scores", torch.float32, 2)
+    _need(static_idx, "static_idx", torch.int32, 2)
+    if anchor is not None:
+        _need(anchor, "anchor", torch.int32, 1)
+    q, ks = static_idx.shape
+    m = ctx.m
+    keep = ks + kd if n_keep is None else n_keep
+    cap = node_cap if node_cap > 0 else keep * m
+    dev = queries.device
+    o = outs if outs is not None else {}
+    dyn = o.setdefault("dyn", {})
+    dyn.setdefault("scores", torch.empty(q, kd, dtype=torch.float32, device=dev))
+    dyn.setdefault("pos", torch.empty(q, kd, dtype=torch.int64, device=dev))
+    dyn.setdefault("spans", _i32((q, kd, m), dev))
+    o.setdefault("spans", _i32((q, keep, m), dev))
+    o.setdefault("num_nodes", _i32((q,), dev))
+    o.setdefault("tokens", _i32((q, cap), dev))
+    o.setdefault("parent", _i32((q, cap), dev))
+    o.setdefault("depth", _i32((q, cap), dev))
+    o.setdefault("gamma", _i32((q, keep, m), dev))
+    if mask_bits:
+        o.setdefault("mask_bits", torch.empty(q, cap, (cap + 31) // 32, dtype=torch.int32,
+                                              device=dev))
+    if workspace is None:
+        workspace = alloc_workspace(lib().sense_ctx_search_workspace_bytes(
+            C.c_void_p(ctx.handle), q, kd), dev)
+    _call(lib().sense_dyn_draft, C.c_void_p(ds.handle), C.c_void_p(ctx.handle),
+          queries.data_ptr(), q, static_scores.data_ptr(), static_idx.data_ptr(), ks, kd,
+          C.c_float(delta), _ptr(anchor), keep, 1 if force_anchor else 0, node_cap,
+          1 if mask_bits else 0, workspace.data_ptr(), workspace.numel(),
+          dyn["scores"].data_ptr(), dyn["pos"].data_ptr(), dyn["spans"].data_ptr(),
+          o["spans"].data_ptr(), o["num_nodes"].data_ptr(), o["tokens"].data_ptr(),
+          o["parent"].data_ptr(), o["depth"].data_ptr(), o["gamma"].data_ptr(),
+          _ptr(o.get("mask_bits")), C.c_void_p(_stream(stream)))
+    o["cap"] = cap
+    return o
+
+
 def sense_tree_attention(q: torch.Tensor, k_cache: torch.Tensor, vt_cache: torch.Tensor,
                          prefix_len: int, mask_bits: torch.Tensor, scale: float,
                          out: torch.Tensor | None = None, workspace=None,

@@ -32,7 +32,9 @@
 #include <algorithm>
 
 #include "common.cuh"
+#include "draft_dev.cuh"
 #include "launch.h"
+#include "select_dev.cuh"
 
 struct sense_ctx {
   int32_t cap;
@@ -48,6 +50,7 @@ namespace sense {
 namespace {
 
 constexpr int kHybridMax = 2048;  // static + dynamic candidates per query
+constexpr size_t kDynDraftSmemMax = 180 * 1024;  // dyn_draft_kernel: + 42 KB static
 
 // Writes the key and token of one position; `x` is its bf16 hidden state.
 __device__ void append_row(const uint16_t* __restrict__ x, int32_t token, int64_t slot, int d,
@@ -186,20 +189,17 @@ ctx_score_kernel(const uint16_t* __restrict__ keys, const uint16_t* __restrict__
   }
 }
 
-// One block (1024 threads) per query.  Union index u < ks: static rank u;
-// u >= ks: dynamic rank u - ks.
-__global__ void __launch_bounds__(1024)
-hybrid_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
-              const float* __restrict__ s_scores, const int32_t* __restrict__ s_idx, int ks,
-              const float* __restrict__ d_scores, const int32_t* __restrict__ d_spans, int kd,
-              const int32_t* __restrict__ anchor, int n_keep, int force,
-              int32_t* __restrict__ out, uint32_t* status) {
+// Query qi by one block (any multiple of 32 threads).  Union index u < ks:
+// static rank u; u >= ks: dynamic rank u - ks.  The dynamic lists are read
+// from L2 (a fused caller writes them earlier in the same launch).
+__device__ void hybrid_block(const int32_t* __restrict__ spans, int64_t n, int m,
+                             const float* __restrict__ s_scores, const int32_t* __restrict__ s_idx,
+                             int ks, const float* d_scores, const int32_t* d_spans, int kd,
+                             const int32_t* __restrict__ anchor, int n_keep, int force,
+                             int32_t* __restrict__ out, uint32_t* status, int qi) {
   __shared__ uint64_t key[kHybridMax];
   __shared__ int dest[kHybridMax];
   __shared__ int n_live;
-  pdl_wait();  // both candidate lists are complete
-  pdl_launch_dependents();
-  const int qi = blockIdx.x;
   const int tot = ks + kd;
   int pw = 1;
   while (pw < tot) pw <<= 1;
@@ -214,7 +214,7 @@ hybrid_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
       if (idx >= 0 && idx < n) kk = cand_key(s_scores[(int64_t)qi * ks + u], (uint32_t)u);
       else raise_status(status, SENSE_DEVST_BAD_INDEX);
     } else if (u < tot) {
-      const float s = d_scores[(int64_t)qi * kd + (u - ks)];
+      const float s = __ldcg(d_scores + (int64_t)qi * kd + (u - ks));
       if (s > -__int_as_float(0x7f800000)) kk = cand_key(s, (uint32_t)u);
     }
     if (kk) atomicAdd(&n_live, 1);
@@ -241,7 +241,7 @@ hybrid_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
   const int live = n_live;
   auto first_token = [&](int u) -> int {
     if (u < ks) return spans[(int64_t)s_idx[(int64_t)qi * ks + u] * m];
-    return d_spans[((int64_t)qi * kd + (u - ks)) * m];
+    return __ldcg(d_spans + ((int64_t)qi * kd + (u - ks)) * m);
   };
   // stable partition (anchor matches first), one warp, 32 candidates a step
   if (threadIdx.x < 32) {
@@ -271,11 +271,70 @@ hybrid_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
     if (o < live) {
       const int u = dest[o];
       v = (u < ks) ? spans[(int64_t)s_idx[(int64_t)qi * ks + u] * m + j]
-                   : d_spans[((int64_t)qi * kd + (u - ks)) * m + j];
+                   : __ldcg(d_spans + ((int64_t)qi * kd + (u - ks)) * m + j);
     }
     if (force && has_anchor && j == 0 && (o == 0 || o == n_keep - 1)) v = a;
     out[obase + e] = v;
   }
+}
+
+__global__ void __launch_bounds__(1024)
+hybrid_kernel(const int32_t* __restrict__ spans, int64_t n, int m,
+              const float* __restrict__ s_scores, const int32_t* __restrict__ s_idx, int ks,
+              const float* __restrict__ d_scores, const int32_t* __restrict__ d_spans, int kd,
+              const int32_t* __restrict__ anchor, int n_keep, int force,
+              int32_t* __restrict__ out, uint32_t* status) {
+  pdl_wait();  // both candidate lists are complete
+  pdl_launch_dependents();
+  hybrid_block(spans, n, m, s_scores, s_idx, ks, d_scores, d_spans, kd, anchor, n_keep, force, out,
+               status, blockIdx.x);
+}
+
+// The hybrid drafting tail of one query by one block of 1024 threads: the
+// top kd of the buffer's scored positions (the pool merge) with their
+// positions and spans, the union with the static results reranked
+// (hybrid_block) and the small-tree trie of the kept spans, each phase
+// reading the previous one's global writes after a block barrier; the trie
+// reuses the merge's shared memory.
+__global__ void __launch_bounds__(1024, 1)
+dyn_draft_kernel(const uint64_t* __restrict__ pool, const uint32_t* __restrict__ counts,
+                 int cap, int kd, float* __restrict__ dyn_scores, int32_t* __restrict__ rel,
+                 const int64_t* __restrict__ count, const int32_t* __restrict__ ring,
+                 int64_t* __restrict__ dyn_pos, int32_t* __restrict__ dyn_spans,
+                 const int32_t* __restrict__ spans, int64_t n, int m,
+                 const float* __restrict__ s_scores, const int32_t* __restrict__ s_idx, int ks,
+                 const int32_t* __restrict__ anchor, int n_keep, int force,
+                 int32_t* __restrict__ out_spans, int node_cap, int mask_words,
+                 int32_t* __restrict__ num_nodes, int32_t* __restrict__ tokens,
+                 int32_t* __restrict__ parent, int32_t* __restrict__ depth,
+                 int32_t* __restrict__ gamma, uint32_t* __restrict__ mask, int smem_keys,
+                 uint32_t* status) {
+  extern __shared__ uint64_t s_keys[];
+  __shared__ int scratch[32];
+  __shared__ int sv[3];
+  const int q = blockIdx.x;
+  pdl_wait();  // the buffer's scores and the static results are complete
+  pdl_launch_dependents();
+  merge_pool_block(pool, counts, cap, kd, dyn_scores, rel, status, 1, q, s_keys, smem_keys);
+  __syncthreads();
+  {  // positions and spans of the dynamic winners (as ctx_pool_kernel)
+    const int64_t cnt = *count;
+    const int64_t lo = cnt > cap ? cnt - cap : 0;
+    for (int t = threadIdx.x; t < kd * m; t += blockDim.x) {
+      const int r = t / m, j = t - r * m;
+      const int64_t slot = (int64_t)q * kd + r;
+      const int e = rel[slot];
+      const int64_t p = lo + e;
+      if (j == 0) dyn_pos[slot] = e < 0 ? -1 : p;
+      dyn_spans[slot * m + j] = e < 0 ? -1 : ring[(p + j) % cap];
+    }
+  }
+  __syncthreads();
+  hybrid_block(spans, n, m, s_scores, s_idx, ks, dyn_scores, dyn_spans, kd, anchor, n_keep, force,
+               out_spans, status, q);
+  __syncthreads();
+  tree_small_block(out_spans, n_keep, m, node_cap, mask_words, num_nodes, tokens, parent, depth,
+                   gamma, mask, status, q, reinterpret_cast<int*>(s_keys), scratch, sv);
 }
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -394,11 +453,16 @@ size_t sense_ctx_search_workspace_bytes(const sense_ctx* c, int32_t q, int32_t k
   return align256((size_t)q * c->cap * 8) + align256((size_t)q * 4) + align256((size_t)q * k * 4);
 }
 
-sense_status sense_ctx_search(const sense_ctx* c, const uint16_t* queries, int32_t q, int32_t k,
-                              float delta, float* out_scores, int64_t* out_pos, int32_t* out_spans,
-                              void* workspace, size_t workspace_bytes, sense_stream_t stream) {
+}  // extern "C"
+
+namespace {
+// Validation of a DynSearch and its scoring launch (ctx_score_kernel): every
+// query's pool of scored positions is left in the workspace.
+sense_status ctx_score(const sense_ctx* c, const uint16_t* queries, int32_t q, int32_t k,
+                       float delta, void* workspace, size_t workspace_bytes, cudaStream_t s,
+                       uint64_t** pool_out, uint32_t** counts_out, int32_t** rel_out) {
   if (!c) return fail(SENSE_ERR_INVALID_ARG, "ctx is NULL");
-  if (!queries || !out_scores || !out_pos || !out_spans || !workspace)
+  if (!queries || !workspace)
     return fail(SENSE_ERR_INVALID_ARG, "queries, outputs and workspace must be non-NULL");
   if (q < 1 || q > 65535) return fail(SENSE_ERR_INVALID_ARG, "q=%d outside [1, 65535]", q);
   if (k < 1 || k > SENSE_MAX_K) return fail(SENSE_ERR_INVALID_ARG, "k=%d outside [1, %d]", k, SENSE_MAX_K);
@@ -409,34 +473,29 @@ sense_status sense_ctx_search(const sense_ctx* c, const uint16_t* queries, int32
     return fail(SENSE_ERR_INVALID_ARG, "workspace of %zu bytes < %zu", workspace_bytes,
                 sense_ctx_search_workspace_bytes(c, q, k));
   if (current_device() != c->device) return fail(SENSE_ERR_INVALID_ARG, "ctx lives on device %d", c->device);
-  uint32_t* status = device_status_word();
-  if (!status) return SENSE_ERR_OOM;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   char* ws = static_cast<char*>(workspace);
   auto* pool = reinterpret_cast<uint64_t*>(ws);
   auto* counts = reinterpret_cast<uint32_t*>(ws + align256((size_t)q * c->cap * 8));
   auto* rel = reinterpret_cast<int32_t*>(ws + align256((size_t)q * c->cap * 8) + align256((size_t)q * 4));
-  {
-    LaunchScope ls(K_CTX, s);
-    const int64_t want = ((int64_t)q * c->cap * 32 + 255) / 256;
-    const int64_t floor_q = ((int64_t)q * 32 + 255) / 256;  // at least one warp per query
-    const int64_t blocks = std::max(floor_q, std::min<int64_t>(want, (int64_t)sm_count() * 16));
-    sense_status st = cuda_check(
-        launch_pdl(ctx_score_kernel, dim3((unsigned)blocks), dim3(256), 0, s, c->keys, queries, q,
-                   c->d, c->cap, c->m, (const int64_t*)c->count, delta, pool, counts),
-        "launch ctx score");
-    if (st != SENSE_OK) return st;
-  }
-  // top k of each pool, then the winners' positions and spans, one block per query
-  return launch_ctx_pool(pool, counts, c->cap, q, k, out_scores, rel, c->count, c->m, c->tokens,
-                         out_pos, out_spans, status, s);
+  LaunchScope ls(K_CTX, s);
+  const int64_t want = ((int64_t)q * c->cap * 32 + 255) / 256;
+  const int64_t floor_q = ((int64_t)q * 32 + 255) / 256;  // at least one warp per query
+  const int64_t blocks = std::max(floor_q, std::min<int64_t>(want, (int64_t)sm_count() * 16));
+  sense_status st = cuda_check(
+      launch_pdl(ctx_score_kernel, dim3((unsigned)blocks), dim3(256), 0, s, c->keys, queries, q,
+                 c->d, c->cap, c->m, (const int64_t*)c->count, delta, pool, counts),
+      "launch ctx score");
+  *pool_out = pool;
+  *counts_out = counts;
+  *rel_out = rel;
+  return st;
 }
 
-sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_scores,
-                                 const int32_t* static_idx, int32_t ks, const float* dyn_scores,
-                                 const int32_t* dyn_spans, int32_t kd, int32_t q,
-                                 const int32_t* anchor, int32_t n_keep, uint32_t flags,
-                                 int32_t* out_spans, sense_stream_t stream) {
+// Validation of a hybrid rerank's arguments (sense_hybrid_drafts).
+sense_status check_hybrid(const sense_datastore* ds, const float* static_scores,
+                          const int32_t* static_idx, int32_t ks, const float* dyn_scores,
+                          const int32_t* dyn_spans, int32_t kd, int32_t q, const int32_t* anchor,
+                          int32_t n_keep, uint32_t flags, const int32_t* out_spans) {
   if (!ds) return fail(SENSE_ERR_INVALID_ARG, "ds is NULL");
   if (q < 1 || q > 65535) return fail(SENSE_ERR_INVALID_ARG, "q=%d outside [1, 65535]", q);
   if (ks < 0 || kd < 0 || ks + kd < 1 || ks + kd > kHybridMax)
@@ -448,6 +507,40 @@ sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_
   if (flags & ~SENSE_GATHER_FORCE_ANCHOR) return fail(SENSE_ERR_INVALID_ARG, "unknown flags 0x%x", flags);
   if ((flags & SENSE_GATHER_FORCE_ANCHOR) && !anchor)
     return fail(SENSE_ERR_INVALID_ARG, "SENSE_GATHER_FORCE_ANCHOR needs anchor");
+  return SENSE_OK;
+}
+}  // namespace
+
+extern "C" {
+
+sense_status sense_ctx_search(const sense_ctx* c, const uint16_t* queries, int32_t q, int32_t k,
+                              float delta, float* out_scores, int64_t* out_pos, int32_t* out_spans,
+                              void* workspace, size_t workspace_bytes, sense_stream_t stream) {
+  if (!c) return fail(SENSE_ERR_INVALID_ARG, "ctx is NULL");
+  if (!queries || !out_scores || !out_pos || !out_spans || !workspace)
+    return fail(SENSE_ERR_INVALID_ARG, "queries, outputs and workspace must be non-NULL");
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint64_t* pool = nullptr;
+  uint32_t* counts = nullptr;
+  int32_t* rel = nullptr;
+  sense_status st = ctx_score(c, queries, q, k, delta, workspace, workspace_bytes, s, &pool,
+                              &counts, &rel);
+  if (st != SENSE_OK) return st;
+  // top k of each pool, then the winners' positions and spans, one block per query
+  return launch_ctx_pool(pool, counts, c->cap, q, k, out_scores, rel, c->count, c->m, c->tokens,
+                         out_pos, out_spans, status, s);
+}
+
+sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_scores,
+                                 const int32_t* static_idx, int32_t ks, const float* dyn_scores,
+                                 const int32_t* dyn_spans, int32_t kd, int32_t q,
+                                 const int32_t* anchor, int32_t n_keep, uint32_t flags,
+                                 int32_t* out_spans, sense_stream_t stream) {
+  sense_status st = check_hybrid(ds, static_scores, static_idx, ks, dyn_scores, dyn_spans, kd, q,
+                                 anchor, n_keep, flags, out_spans);
+  if (st != SENSE_OK) return st;
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
@@ -457,6 +550,68 @@ sense_status sense_hybrid_drafts(const sense_datastore* ds, const float* static_
                                ks, dyn_scores, dyn_spans, kd, anchor, n_keep,
                                (flags & SENSE_GATHER_FORCE_ANCHOR) ? 1 : 0, out_spans, status),
                     "launch hybrid drafts");
+}
+
+sense_status sense_dyn_draft(const sense_datastore* ds, const sense_ctx* c,
+                             const uint16_t* queries, int32_t q, const float* static_scores,
+                             const int32_t* static_idx, int32_t ks, int32_t kd, float delta,
+                             const int32_t* anchor, int32_t n_keep, uint32_t flags,
+                             int32_t node_cap, uint32_t tree_flags, void* workspace,
+                             size_t workspace_bytes, float* dyn_scores, int64_t* dyn_pos,
+                             int32_t* dyn_spans, int32_t* out_spans, int32_t* out_num_nodes,
+                             int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
+                             int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream) {
+  if (!ds || !c) return fail(SENSE_ERR_INVALID_ARG, "datastore and buffer must be non-NULL");
+  if (ds->m != c->m || ds->d != c->d)
+    return fail(SENSE_ERR_INVALID_ARG, "datastore and buffer must share d and m");
+  if (!dyn_scores || !dyn_pos || !dyn_spans || !out_num_nodes || !out_tokens || !out_parent ||
+      !out_depth || !out_gamma)
+    return fail(SENSE_ERR_INVALID_ARG, "outputs must be non-NULL");
+  const int m = c->m;
+  sense_status st = check_hybrid(ds, static_scores, static_idx, ks, dyn_scores, dyn_spans, kd, q,
+                                 anchor, n_keep, flags, out_spans);
+  if (st != SENSE_OK) return st;
+  if ((int64_t)n_keep * m > SENSE_MAX_TREE_TOKENS)
+    return fail(SENSE_ERR_INVALID_ARG, "n_keep*m=%d exceeds %d", n_keep * m, SENSE_MAX_TREE_TOKENS);
+  if (node_cap < 0) return fail(SENSE_ERR_INVALID_ARG, "node_cap=%d must be >= 0", node_cap);
+  if (tree_flags & ~SENSE_TREE_MASK_BITS)
+    return fail(SENSE_ERR_INVALID_ARG, "unknown tree flags 0x%x", tree_flags);
+  const bool bits = (tree_flags & SENSE_TREE_MASK_BITS) != 0;
+  if (bits && !out_mask_bits) return fail(SENSE_ERR_INVALID_ARG, "SENSE_TREE_MASK_BITS needs out_mask_bits");
+  const size_t trie_bytes = sizeof(int) * ((size_t)3 * n_keep * m + (size_t)5 * n_keep);
+  const size_t smem = std::max((size_t)c->cap * 8, trie_bytes);
+  if (!draft_fused_fits(n_keep, m) || smem > kDynDraftSmemMax) {  // the calls one by one
+    st = sense_ctx_search(c, queries, q, kd, delta, dyn_scores, dyn_pos, dyn_spans, workspace,
+                          workspace_bytes, stream);
+    if (st != SENSE_OK) return st;
+    st = sense_hybrid_drafts(ds, static_scores, static_idx, ks, dyn_scores, dyn_spans, kd, q,
+                             anchor, n_keep, flags, out_spans, stream);
+    if (st != SENSE_OK) return st;
+    return sense_build_tree(out_spans, q, n_keep, m, node_cap, tree_flags, out_num_nodes,
+                            out_tokens, out_parent, out_depth, out_gamma, out_mask_bits, stream);
+  }
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint64_t* pool = nullptr;
+  uint32_t* counts = nullptr;
+  int32_t* rel = nullptr;
+  st = ctx_score(c, queries, q, kd, delta, workspace, workspace_bytes, s, &pool, &counts, &rel);
+  if (st != SENSE_OK) return st;
+  st = cuda_check(func_smem(reinterpret_cast<const void*>(dyn_draft_kernel), (int)smem),
+                  "cudaFuncSetAttribute(dyn_draft)");
+  if (st != SENSE_OK) return st;
+  const int cap_nodes = node_cap > 0 ? node_cap : n_keep * m;
+  LaunchScope ls(K_CTX, s);
+  return cuda_check(
+      launch_pdl(dyn_draft_kernel, dim3((unsigned)q), dim3(1024), smem, s, (const uint64_t*)pool,
+                 (const uint32_t*)counts, c->cap, kd, dyn_scores, rel, (const int64_t*)c->count,
+                 (const int32_t*)c->tokens, dyn_pos, dyn_spans, (const int32_t*)ds->spans, ds->n,
+                 m, static_scores, static_idx, ks, anchor, n_keep,
+                 (flags & SENSE_GATHER_FORCE_ANCHOR) ? 1 : 0, out_spans, cap_nodes,
+                 (cap_nodes + 31) / 32, out_num_nodes, out_tokens, out_parent, out_depth,
+                 out_gamma, bits ? out_mask_bits : nullptr, (int)(smem / 8), status),
+      "launch dyn draft");
 }
 
 }  // extern "C"

@@ -71,7 +71,7 @@ __device__ void gather_block(const int32_t* __restrict__ spans, int64_t n, int m
   int64_t i = -1;
   bool valid = false;
   if (r < k) {
-    i = idx[(int64_t)q * k + r];
+    i = __ldcg(idx + (int64_t)q * k + r);  // L2: a fused caller wrote idx in this launch
     valid = (i >= 0 && i < n);
     if (!valid) raise_status(status, SENSE_DEVST_BAD_INDEX);
   }
@@ -114,7 +114,8 @@ __device__ void gather_block(const int32_t* __restrict__ spans, int64_t n, int m
 //      decides their lexicographic order (ties by row index), so a's sorted
 //      position is the count of rows before it; the largest LCP of a with a
 //      lower-ranked row, mll[a], is kept too;
-//   2. LCP with the sorted predecessor and the preorder bases (direct sums);
+//   2. LCP with the sorted predecessor and the preorder bases (a warp's
+//      prefix scan);
 //   3. node of (sorted row p, depth j): walk back to the last row p' <= p
 //      with lcp[p'] <= j (its creator);
 //   4. node cap: the node of row r at depth j is first reached by rank r iff
@@ -153,7 +154,7 @@ __device__ void tree_small_block(const int32_t* __restrict__ spans, int k, int m
   if (threadIdx.x == 0) s_bad = 0;
   __syncthreads();
   for (int i = threadIdx.x; i < km; i += blockDim.x) {
-    const int t = src[i];
+    const int t = __ldcg(src + i);  // L2: a fused caller wrote the spans in this launch
     s_tok[i] = t;
     if (t < 0) s_bad = 1;
   }

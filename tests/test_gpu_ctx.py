@@ -204,3 +204,42 @@ def test_ctx_step_replays_as_cuda_graph(S):
         ht = np.concatenate([acc[:4]] * rep)
         _check_search(out, hh, ht, cap, m, bits(qs.cpu()), 6, 0.0)
     ctx.close()
+
+
+@cuda
+@pytest.mark.parametrize("cap,m,fill,ks,kd,keep,force,node_cap,q", [
+    (4096, 16, 3000, 32, 16, 32, True, 64, 1),     # the bench's shape: fused tail
+    (256, 8, 30, 20, 30, 40, False, 0, 2),         # fewer searchable entries than kd
+    (512, 4, 600, 8, 8, 10, True, 7, 3),           # ring wrapped, tight node cap
+    (128, 8, 100, 100, 60, 150, False, 0, 1),      # n_keep > 128: the calls one by one
+])
+def test_dyn_draft_equals_separate_calls(S, cap, m, fill, ks, kd, keep, force, node_cap, q):
+    """sense_dyn_draft is bit-identical to sense_ctx_search, then
+    sense_hybrid_drafts, then sense_build_tree (with mask bits), in its
+    fused form (n_keep <= 128) and in its fallback."""
+    dev = torch.device("cuda")
+    d, n = 256, 5000
+    keys = synth.clustered_unit_keys(n, d, 16, seed=cap + ks, device=dev)
+    spans = synth.spans_uniform(n, m, 7, seed=m, device=dev)  # small vocab: shared prefixes
+    ds = S.sense_datastore_build(keys, spans)
+    ctx = S.sense_ctx_create(cap, d, m)
+    h = synth.gaussian_rows_f32(fill, d, seed=fill).to(torch.bfloat16).to(dev)
+    tok = torch.from_numpy(np.random.default_rng(fill).integers(0, 7, fill).astype(np.int32))
+    S.sense_ctx_append(ctx, h, tok.to(dev))
+    qs, _ = synth.noisy_queries(keys, q, seed=3)
+    sc, ix = S.sense_retrieve_topk(ds, qs, ks)
+    anchor = torch.from_numpy(np.arange(q, dtype=np.int32) % 7).to(dev)
+    for _ in range(2):
+        got = S.sense_dyn_draft(ds, ctx, qs, sc, ix, kd, delta=0.05, anchor=anchor,
+                                n_keep=keep, force_anchor=force, node_cap=node_cap,
+                                mask_bits=True)
+        dyn = S.sense_ctx_search(ctx, qs, kd, 0.05)
+        dr = S.sense_hybrid_drafts(ds, sc, ix, dyn, anchor, keep, force)
+        tr = S.sense_build_tree(dr, node_cap=node_cap, mask_bits=True)
+        torch.cuda.synchronize()
+        assert S.sense_device_status(clear=True) == 0
+        for key in ("scores", "pos", "spans"):
+            assert torch.equal(got["dyn"][key], dyn[key]), key
+        assert torch.equal(got["spans"], dr)
+        for key in ("num_nodes", "tokens", "parent", "depth", "gamma", "mask_bits"):
+            assert torch.equal(got[key], tr[key]), key
