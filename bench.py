@@ -211,16 +211,11 @@ class Pipeline:
         S, cfg = self.S, self.cfg
         if self.ann is None:
             S.sense_retrieve_topk(self.ds, query, cfg["k"], self.scores, self.idx, self.ws)
-        else:
+        else:  # projection, search (and re-scoring) in one call
             a = self.ann
-            S.sense_project(query, a["basis"], a["mean"], out=self.qproj)
-            if a.get("rerank", 0):
-                S.sense_ivf_search(a["index"], self.qproj, a["rerank"], a["nprobe"], self.cand_s,
-                                   self.cand_i, workspace=self.ws)
-                S.sense_rescore_topk(self.ds, query, self.cand_i, cfg["k"], self.scores, self.idx)
-            else:
-                S.sense_ivf_search(a["index"], self.qproj, cfg["k"], a["nprobe"], self.scores,
-                                   self.idx, workspace=self.ws)
+            S.sense_ann_search(a["index"], self.ds, query, a["basis"], a["mean"], cfg["k"],
+                               a["nprobe"], rerank=a.get("rerank", 0), out_scores=self.scores,
+                               out_idx=self.idx, workspace=self.ann_ws)
 
     def use_dynamic(self, ctx, kd, delta, dev):
         """Hybrid retrieval (Alg. 2): the dynamic buffer is searched beside the

@@ -369,6 +369,19 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
                              int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
                              int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream);
 
+/*
+ * The approximate retrieval of sense_ann_draft without its gather and trie
+ * (the static side of a hybrid step, Alg. 2): out_scores / out_idx [q, k]
+ * exactly as sense_ann_draft writes them.  The workspace is
+ * sense_ann_draft_workspace_bytes(ix, q, k, nprobe, rerank) bytes; the
+ * datastore supplies the keys of the re-scoring (rerank > 0) and d.
+ */
+sense_status sense_ann_search(const sense_ivf* ix, const sense_datastore* ds,
+                              const uint16_t* queries, int32_t q, const float* basis,
+                              const float* mean, int32_t k, int32_t nprobe, int32_t rerank,
+                              void* workspace, size_t workspace_bytes, float* out_scores,
+                              int32_t* out_idx, sense_stream_t stream);
+
 /* ---------------------------------------------------------------------- */
 /* a4. Span gather                                                          */
 /* ---------------------------------------------------------------------- */

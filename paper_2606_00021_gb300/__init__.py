@@ -550,6 +550,33 @@ def sense_ann_draft(ix: "IvfIndex", ds: Datastore, queries: torch.Tensor, basis:
     return o
 
 
+def sense_ann_search(ix: "IvfIndex", ds: Datastore, queries: torch.Tensor, basis: torch.Tensor,
+                     mean: torch.Tensor | None, k: int, nprobe: int, rerank: int = 0,
+                     out_scores=None, out_idx=None, workspace=None, stream=None):
+    """sense_ann_draft's retrieval alone (projection, IVF search, optional
+    exact re-scoring): (scores f32 [q, k], idx int32 [q, k])."""
+    _need(queries, "queries", torch.bfloat16, 2)
+    _need(basis, "basis", torch.float32, 2)
+    if mean is not None:
+        _need(mean, "mean", torch.float32, 1)
+    q = queries.shape[0]
+    if queries.shape[1] != ds.d:
+        raise ValueError("queries must have d columns")
+    dev = queries.device
+    if out_scores is None:
+        out_scores = torch.empty(q, k, dtype=torch.float32, device=dev)
+    if out_idx is None:
+        out_idx = _i32((q, k), dev)
+    if workspace is None:
+        need = lib().sense_ann_draft_workspace_bytes(C.c_void_p(ix.handle), q, k, nprobe, rerank)
+        workspace = alloc_workspace(need, dev)
+    _call(lib().sense_ann_search, C.c_void_p(ix.handle), C.c_void_p(ds.handle),
+          queries.data_ptr(), q, basis.data_ptr(), _ptr(mean), k, nprobe, rerank,
+          workspace.data_ptr(), workspace.numel(), out_scores.data_ptr(), out_idx.data_ptr(),
+          C.c_void_p(_stream(stream)))
+    return out_scores, out_idx
+
+
 def sense_ivf_search(ix: IvfIndex, queries: torch.Tensor, k: int, nprobe: int,
                      out_scores=None, out_idx=None, want_probes: bool = False, workspace=None,
                      stream=None):

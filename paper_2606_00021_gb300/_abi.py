@@ -61,6 +61,8 @@ SIGNATURES = {
                                  c_p]),
     "sense_hybrid_drafts": (c_i32, [c_p, c_p, c_p, c_i32, c_p, c_p, c_i32, c_i32, c_p, c_i32,
                                     c_u32, c_p, c_p]),
+    "sense_ann_search": (c_i32, [c_p, c_p, c_p, c_i32, c_p, c_p, c_i32, c_i32, c_i32, c_p, c_size,
+                                 c_p, c_p, c_p]),
     "sense_dyn_draft": (c_i32, [c_p, c_p, c_p, c_i32, c_p, c_p, c_i32, c_i32, C.c_float, c_p,
                                 c_i32, c_u32, c_i32, c_u32, c_p, c_size, c_p, c_p, c_p, c_p, c_p,
                                 c_p, c_p, c_p, c_p, c_p, c_p]),

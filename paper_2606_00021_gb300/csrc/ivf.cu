@@ -1385,16 +1385,22 @@ size_t sense_ann_draft_workspace_bytes(const sense_ivf* ix, int32_t q, int32_t k
   return b + sense_ivf_search_workspace_bytes(ix, q, kk, nprobe);
 }
 
-sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, const uint16_t* queries,
-                             int32_t q, const float* basis, const float* mean, int32_t k,
-                             int32_t nprobe, int32_t rerank, int32_t node_cap, uint32_t flags,
-                             void* workspace, size_t workspace_bytes, float* out_scores,
-                             int32_t* out_idx, int32_t* out_spans, int32_t* out_num_nodes,
-                             int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
-                             int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream) {
+}  // extern "C"
+
+namespace {
+// sense_ann_draft (draft = true) and sense_ann_search (draft = false: the
+// step ends with the top k, the span and tree outputs are unused).
+sense_status ann_step(bool draft, const sense_ivf* ix, const sense_datastore* ds,
+                      const uint16_t* queries, int32_t q, const float* basis, const float* mean,
+                      int32_t k, int32_t nprobe, int32_t rerank, int32_t node_cap,
+                      uint32_t flags, void* workspace, size_t workspace_bytes, float* out_scores,
+                      int32_t* out_idx, int32_t* out_spans, int32_t* out_num_nodes,
+                      int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
+                      int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream) {
   if (!ix || !ds) return fail(SENSE_ERR_INVALID_ARG, "index and datastore must be non-NULL");
-  if (!queries || !basis || !workspace || !out_scores || !out_idx || !out_spans ||
-      !out_num_nodes || !out_tokens || !out_parent || !out_depth || !out_gamma)
+  if (!queries || !basis || !workspace || !out_scores || !out_idx ||
+      (draft && (!out_spans || !out_num_nodes || !out_tokens || !out_parent || !out_depth ||
+                 !out_gamma)))
     return fail(SENSE_ERR_INVALID_ARG, "queries, basis, workspace and outputs must be non-NULL");
   if (ds->device != current_device() || ix->device != current_device())
     return fail(SENSE_ERR_INVALID_ARG, "index and datastore must live on the current device");
@@ -1404,13 +1410,14 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
     return fail(SENSE_ERR_INVALID_ARG, "rerank=%d must be 0 or in [k=%d, %d]", rerank, k,
                 SENSE_MAX_RESCORE);
   const int m = ds->m;
-  if ((int64_t)k * m > SENSE_MAX_TREE_TOKENS)
+  if (draft && (int64_t)k * m > SENSE_MAX_TREE_TOKENS)
     return fail(SENSE_ERR_INVALID_ARG, "k*m=%d exceeds %d", k * m, SENSE_MAX_TREE_TOKENS);
   if (node_cap < 0) return fail(SENSE_ERR_INVALID_ARG, "node_cap=%d must be >= 0", node_cap);
   if (flags & ~SENSE_TREE_MASK_BITS) return fail(SENSE_ERR_INVALID_ARG, "unknown tree flags 0x%x", flags);
   const bool bits = (flags & SENSE_TREE_MASK_BITS) != 0;
-  if (bits && !out_mask_bits) return fail(SENSE_ERR_INVALID_ARG, "SENSE_TREE_MASK_BITS needs out_mask_bits");
-  if (!aligned(workspace, 256) || !aligned(out_spans, 16))
+  if (draft && bits && !out_mask_bits)
+    return fail(SENSE_ERR_INVALID_ARG, "SENSE_TREE_MASK_BITS needs out_mask_bits");
+  if (!aligned(workspace, 256) || (draft && !aligned(out_spans, 16)))
     return fail(SENSE_ERR_INVALID_ARG, "workspace must be 256-byte and out_spans 16-byte aligned");
   const size_t need = sense_ann_draft_workspace_bytes(ix, q, k, nprobe, rerank);
   if (workspace_bytes < need)
@@ -1429,7 +1436,7 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
   }
   const size_t ivf_bytes = sense_ivf_search_workspace_bytes(ix, q, kk, nprobe);
   const int cap = node_cap > 0 ? node_cap : k * m;
-  const bool fused = draft_fused_fits(k, m);
+  const bool fused = draft && draft_fused_fits(k, m);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (!aligned(queries, 16) || !aligned(basis, 16) || (mean && !aligned(mean, 16)))
     return fail(SENSE_ERR_INVALID_ARG, "queries, basis and mean must be 16-byte aligned");
@@ -1467,7 +1474,7 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
   } else {
     st = launch_merge_short(pool, counts, pool_cap, q, k, out_scores, out_idx, status, s);
   }
-  if (st != SENSE_OK) return st;
+  if (st != SENSE_OK || !draft) return st;
   if (fused)  // gather and trie in one kernel per query
     return launch_span_draft(out_idx, q, k, ds->spans, ds->n, m, out_spans, cap, bits ? 1 : 0,
                              out_num_nodes, out_tokens, out_parent, out_depth, out_gamma,
@@ -1476,6 +1483,31 @@ sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, con
   if (st != SENSE_OK) return st;
   return launch_tree(out_spans, q, k, m, cap, bits ? 1 : 0, out_num_nodes, out_tokens, out_parent,
                      out_depth, out_gamma, out_mask_bits, status, stream);
+}
+}  // namespace
+
+extern "C" {
+
+sense_status sense_ann_draft(const sense_ivf* ix, const sense_datastore* ds, const uint16_t* queries,
+                             int32_t q, const float* basis, const float* mean, int32_t k,
+                             int32_t nprobe, int32_t rerank, int32_t node_cap, uint32_t flags,
+                             void* workspace, size_t workspace_bytes, float* out_scores,
+                             int32_t* out_idx, int32_t* out_spans, int32_t* out_num_nodes,
+                             int32_t* out_tokens, int32_t* out_parent, int32_t* out_depth,
+                             int32_t* out_gamma, uint32_t* out_mask_bits, sense_stream_t stream) {
+  return ann_step(true, ix, ds, queries, q, basis, mean, k, nprobe, rerank, node_cap, flags,
+                  workspace, workspace_bytes, out_scores, out_idx, out_spans, out_num_nodes,
+                  out_tokens, out_parent, out_depth, out_gamma, out_mask_bits, stream);
+}
+
+sense_status sense_ann_search(const sense_ivf* ix, const sense_datastore* ds,
+                              const uint16_t* queries, int32_t q, const float* basis,
+                              const float* mean, int32_t k, int32_t nprobe, int32_t rerank,
+                              void* workspace, size_t workspace_bytes, float* out_scores,
+                              int32_t* out_idx, sense_stream_t stream) {
+  return ann_step(false, ix, ds, queries, q, basis, mean, k, nprobe, rerank, 0, 0, workspace,
+                  workspace_bytes, out_scores, out_idx, nullptr, nullptr, nullptr, nullptr,
+                  nullptr, nullptr, nullptr, stream);
 }
 
 }  // extern "C"

@@ -59,6 +59,7 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert lib.sense_ann_draft(None, None, p, 1, p, None, 8, 4, 0, 0, 0, p, 1 << 20, p, p, p, p,
                                p, p, p, p, None, None) == 1
     assert lib.sense_ann_draft_workspace_bytes(None, 1, 8, 4, 0) == 0
+    assert lib.sense_ann_search(None, None, p, 1, p, None, 8, 4, 0, p, 1 << 20, p, p, None) == 1
     assert lib.sense_dyn_draft(None, None, p, 1, p, p, 8, 4, 0.0, None, 8, 0, 0, 0, p, 1 << 20,
                                p, p, p, p, p, p, p, p, p, None, None) == 1
     # allocation-free status reader and self test: NULL output, limit range

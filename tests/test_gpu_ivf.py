@@ -458,6 +458,13 @@ def test_ann_draft_equals_separate_calls(S, pq, rerank, q, k, cap, nlist, nprobe
         # the -1 slots' rows (bad index, then negative tokens in the trie)
         assert S.sense_device_status(clear=True) == st_one
         assert torch.equal(got["scores"], sc) and torch.equal(got["idx"], idx)
+        sc2, ix2 = S.sense_ann_search(ix, ds, qs, basis, mean, k, nprobe, rerank=rerank)
+        torch.cuda.synchronize()
+        assert torch.equal(sc2, sc) and torch.equal(ix2, idx)
+        if nprobe > 1:
+            assert S.sense_device_status(clear=True) == 0
+        else:
+            S.sense_device_status(clear=True)
         if nprobe == 1:  # a short pool: the padding is part of the result
             assert (idx == -1).any()
             assert st_one == S.DEVST_BAD_INDEX | S.DEVST_BAD_TOKEN
