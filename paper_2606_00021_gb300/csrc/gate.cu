@@ -47,6 +47,7 @@ constexpr int kWStageF4 = 256;                     // float4 per warp stage (4 K
 constexpr int kWStages = 3;                        // ring depth per warp
 constexpr int kLaneF4 = kWStageF4 / 32;            // float4 per lane per stage
 constexpr size_t kRingBytes = (size_t)kWarps * kWStages * kWStageF4 * 16;
+constexpr size_t kRowSmemMax = 216 * 1024;  // dynamic shared memory of a row block (+ ~8 KB static)
 constexpr int kStatsInts = 2 + SENSE_MAX_KAPPA;    // argmax, ent flag, top list
 constexpr int kMaxSegs = 16;
 constexpr long long kWaitCycles = 4000000000LL;
@@ -169,12 +170,9 @@ struct RowAcc {
         const float xs[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const bool want = live && xs[e] >= thr;
-          if (__any_sync(0xffffffffu, want)) {
-            if (want) {
-              tl.push(xs[e], idx[u] * 4 + e);
-              thr = fmaxf(tl.v[KM - 1], lb);
-            }
+          if (live && xs[e] >= thr) {  // per-lane list: no vote needed
+            tl.push(xs[e], idx[u] * 4 + e);
+            thr = fmaxf(tl.v[KM - 1], lb);
           }
         }
       }
@@ -554,14 +552,33 @@ __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
+// Issues the asynchronous copies of query q's Gamma, tokens and parents into
+// a staged decide block's shared memory (completed by the same threads'
+// cp_async_wait_all() in decide_block).
+__device__ __forceinline__ void decide_stage_inputs(const GateArgs& a, int q, int32_t* s_dyn) {
+  const int km = a.k * a.m, cap = a.cap;
+  int32_t* sg = s_dyn;
+  int32_t* stk = sg + km;
+  int32_t* spr = stk + cap;
+  const int32_t* gam = a.gamma + (int64_t)q * km;
+  const int32_t* tok = a.tokens + (int64_t)q * cap;
+  const int32_t* par = a.parent + (int64_t)q * cap;
+  for (int i = threadIdx.x; i < km; i += blockDim.x) cp_async4(sg + i, gam + i);
+  for (int i = threadIdx.x; i < cap; i += blockDim.x) {
+    cp_async4(stk + i, tok + i);
+    cp_async4(spr + i, par + i);
+  }
+}
+
 // The decision of query q by one block (any multiple of 32 threads up to
 // 1024).  s_dyn: staged ? [Gamma k*m][tokens cap][parents cap][stats
 // (cap+1) rows] : nothing, then flags [k*m]: bit0 valid, bit1 em, bit2 ent,
 // bit3 topk, bit4 G.  `fresh` (staged only): the statistics were written
 // by other blocks of the running grid, so they are read from L2 with plain
-// loads rather than copied through L1.
+// loads rather than copied through L1.  `prestaged`: the same threads
+// already issued decide_stage_inputs into s_dyn.
 __device__ __forceinline__ void decide_block(const GateArgs& a, const int32_t* __restrict__ stats, int staged,
-                             int q, int32_t* s_dyn, bool fresh) {
+                             int q, int32_t* s_dyn, bool fresh, bool prestaged = false) {
   __shared__ int s_L[SENSE_MAX_K];
   __shared__ int s_best[32];
   __shared__ int s_istar, s_lstar, s_next, s_nn;
@@ -577,14 +594,23 @@ __device__ __forceinline__ void decide_block(const GateArgs& a, const int32_t* _
     int32_t* stk = sg + km;
     int32_t* spr = stk + cap;
     int32_t* sst = spr + cap;
-    for (int i = threadIdx.x; i < km; i += blockDim.x) cp_async4(sg + i, gam + i);
-    for (int i = threadIdx.x; i < cap; i += blockDim.x) {
-      cp_async4(stk + i, tok + i);
-      cp_async4(spr + i, par + i);
-    }
-    if (fresh)
-      for (int i = threadIdx.x; i < (cap + 1) * kStatsInts; i += blockDim.x) sst[i] = __ldcg(st + i);
-    else
+    if (!prestaged) decide_stage_inputs(a, q, s_dyn);
+    if (fresh) {  // four loads per thread in flight before their stores
+      const int ns = (cap + 1) * kStatsInts;
+      for (int i0 = threadIdx.x; i0 < ns; i0 += 4 * blockDim.x) {
+        int32_t v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int i = i0 + u * blockDim.x;
+          v[u] = i < ns ? __ldcg(st + i) : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int i = i0 + u * blockDim.x;
+          if (i < ns) sst[i] = v[u];
+        }
+      }
+    } else
       for (int i = threadIdx.x; i < (cap + 1) * kStatsInts; i += blockDim.x) cp_async4(sst + i, st + i);
     if (threadIdx.x == 0) cp_async4(&s_nn, a.num_nodes + q);
     cp_async_wait_all();
@@ -822,7 +848,7 @@ gate_row_block_kernel(const int32_t* __restrict__ parent, const int32_t* __restr
                       int cap, const float* __restrict__ root_logits,
                       const float* __restrict__ node_logits, int vocab, int kappa, float thr,
                       int unnormalized, int seg4, int32_t* __restrict__ stats, uint32_t* status,
-                      GateArgs a, int staged, unsigned* __restrict__ decide_done) {
+                      GateArgs a, int staged, unsigned* __restrict__ decide_done, int prestage) {
   static_assert(NC >= 1 && NC * kWarps <= 32, "one merging warp holds every partial");
   extern __shared__ __align__(128) float4 ring_all[];
   __shared__ __align__(8) uint64_t bars_all[kWarps * kWStages];
@@ -845,6 +871,10 @@ gate_row_block_kernel(const int32_t* __restrict__ parent, const int32_t* __restr
     // depends on the row only: the whole cluster skips the row
     if (inner) row = node_logits + ((int64_t)q * cap + nd) * vocab;
   }
+  // the decision's inputs that the trie wrote go to shared memory past the
+  // ring now, so the block that runs the decision waits only for the stats
+  int32_t* s_dec = reinterpret_cast<int32_t*>(reinterpret_cast<char*>(ring_all) + kRingBytes);
+  if (decide_done != nullptr && prestage && crank == 0) decide_stage_inputs(a, q, s_dec);
   if (row) row_block_pass<KM, NC>(row, vocab, kappa, thr, unnormalized, seg4,
                                   stats + (int64_t)rid * kStatsInts, status, crank, ring_all,
                                   bars_all, s_part, s_fail);
@@ -857,9 +887,13 @@ gate_row_block_kernel(const int32_t* __restrict__ parent, const int32_t* __restr
     s_last = last;
   }
   __syncthreads();
-  if (!s_last) return;
+  if (!s_last) {
+    if (prestage) cp_async_wait_all();  // no copy into this block's memory outlives it
+    return;
+  }
   __threadfence();  // every slot's statistics are visible
-  decide_block(a, stats, staged, q, reinterpret_cast<int32_t*>(ring_all), true);
+  if (prestage) decide_block(a, stats, staged, q, s_dec, true, true);
+  else decide_block(a, stats, staged, q, reinterpret_cast<int32_t*>(ring_all), true);
 }
 
 __global__ void __launch_bounds__(kDecideThreads)
@@ -920,19 +954,23 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     const int nc = pair ? 2 : 1;
     const int slice4 = (n4 + nc * kWarps - 1) / (nc * kWarps);
     void (*kern)(const int32_t*, const int32_t*, int, const float*, const float*, int, int, float,
-                 int, int, int32_t*, uint32_t*, GateArgs, int, unsigned*);
+                 int, int, int32_t*, uint32_t*, GateArgs, int, unsigned*, int);
     if (pair) kern = (a.kappa <= 4) ? gate_row_block_kernel<4, 2>
                                      : gate_row_block_kernel<SENSE_MAX_KAPPA, 2>;
     else kern = (a.kappa <= 4) ? gate_row_block_kernel<4, 1>
                                : gate_row_block_kernel<SENSE_MAX_KAPPA, 1>;
+    // the decision's staged inputs past the ring when they fit beside it
+    const size_t dec_bytes = (staged_smem + 15) & ~(size_t)15;
+    const int prestage = (staged && kRingBytes + dec_bytes <= kRowSmemMax) ? 1 : 0;
+    const size_t row_smem = kRingBytes + (prestage ? dec_bytes : 0);
     st = cuda_check(
-        func_smem(reinterpret_cast<const void*>(kern), (int)kRingBytes),
+        func_smem(reinterpret_cast<const void*>(kern), (int)row_smem),
         "cudaFuncSetAttribute(gate_row_block)");
     if (st != SENSE_OK) return st;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(rows * nc));
     cfg.blockDim = dim3(kRowThreads);
-    cfg.dynamicSmemBytes = kRingBytes;
+    cfg.dynamicSmemBytes = row_smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -949,7 +987,7 @@ sense_status launch_gate(const GateArgs& a, cudaStream_t s) {
     LaunchScope ls(K_GATE_ROWS, s);
     st = cuda_check(cudaLaunchKernelEx(&cfg, kern, a.parent, a.num_nodes, a.cap, a.root_logits,
                                        a.node_logits, a.vocab, a.kappa, a.thr, a.unnormalized,
-                                       slice4, stats, a.status, a, staged, fuse),
+                                       slice4, stats, a.status, a, staged, fuse, prestage),
                     "launch gate_row_block");
     if (st != SENSE_OK) return st;
     if (fuse) return SENSE_OK;
