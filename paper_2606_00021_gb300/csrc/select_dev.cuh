@@ -102,8 +102,8 @@ __device__ bool radix_select(Get get, int64_t cnt, int k, int low, unsigned* his
   return true;
 }
 
-// Short path of merge_kernel for a pool staged in shared memory (distinct
-// nonzero keys, at most 32 * kPoolGroups of them).  The pool is cut into
+// Short path of merge_kernel for a pool of distinct nonzero keys (at most
+// 32 * kPoolGroups of them).  The pool is cut into
 // groups of 32; a group's maximum is a head, and the k-th largest head T
 // bounds the k-th largest key from below (k groups hold a key >= T).  Heads
 // are ranked against warp-sorted groups of heads by binary search; the keys
@@ -122,7 +122,10 @@ __device__ __forceinline__ uint64_t warp_max64(uint64_t x) {
   return ((uint64_t)hm << 32) | lm;
 }
 
-__device__ bool merge_pool_short(const uint64_t* s_keys, int cnt, int k, int pad_short,
+// The keys are read where they are, in the pool (L2 loads, four per thread
+// in flight; a fused caller writes the pool earlier in the same launch):
+// both passes over them are coalesced, so no staging copy is needed.
+__device__ bool merge_pool_short(const uint64_t* __restrict__ keys, int cnt, int k, int pad_short,
                                  uint64_t* cand, float* __restrict__ out_scores,
                                  int32_t* __restrict__ out_idx) {
   __shared__ uint64_t s_heads[kPoolGroups];  // group maxima, then sorted in groups of 32
@@ -138,10 +141,21 @@ __device__ bool merge_pool_short(const uint64_t* s_keys, int cnt, int k, int pad
   // heads: group maxima (every warp takes groups in turn), then sorted
   // descending within each group of 32 heads; groups past the pool are 0
   const int nhg = (ngr + 31) >> 5;
-  for (int g = warp; g < ngr; g += nwarps) {
-    const int i = g * 32 + lane;
-    const uint64_t m = warp_max64(i < cnt ? s_keys[i] : 0ull);
-    if (lane == 0) s_heads[g] = m;
+  for (int g0 = warp; g0 < ngr; g0 += 4 * nwarps) {
+    uint64_t x[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = (g0 + u * nwarps) * 32 + lane;
+      x[u] = i < cnt ? __ldcg(keys + i) : 0ull;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int g = g0 + u * nwarps;  // warp-uniform
+      if (g < ngr) {
+        const uint64_t m = warp_max64(x[u]);
+        if (lane == 0) s_heads[g] = m;
+      }
+    }
   }
   for (int g = ngr + threadIdx.x; g < nhg * 32; g += blockDim.x) s_heads[g] = 0ull;
   __syncthreads();
@@ -176,11 +190,20 @@ __device__ bool merge_pool_short(const uint64_t* s_keys, int cnt, int k, int pad
   }
   __syncthreads();
   const uint64_t t = s_t;
-  for (int i = threadIdx.x; i < cnt; i += blockDim.x) {
-    const uint64_t c = s_keys[i];
-    if (c != 0ull && c >= t) {
-      const unsigned p = atomicAdd(&s_got, 1u);
-      if (p < (unsigned)kPoolCand) cand[p] = c;
+  for (int i0 = threadIdx.x; i0 < cnt; i0 += 4 * blockDim.x) {
+    uint64_t x[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = i0 + u * blockDim.x;
+      x[u] = i < cnt ? __ldcg(keys + i) : 0ull;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const uint64_t c = x[u];
+      if (c != 0ull && c >= t) {
+        const unsigned p = atomicAdd(&s_got, 1u);
+        if (p < (unsigned)kPoolCand) cand[p] = c;
+      }
     }
   }
   __syncthreads();
@@ -316,18 +339,18 @@ __device__ void merge_pool_block(const uint64_t* __restrict__ pool,
   const uint64_t* src = pool + (int64_t)q * pool_cap;
   int64_t cnt = counts ? (int64_t)counts[q] : pool_cap;  // no counts: every slot is used
   if (cnt > pool_cap) cnt = pool_cap;
+  // the short path (pool read in place) needs a pruning threshold (k group
+  // heads) or a tiny pool
+  if (cnt > 0 && cnt <= 32 * kPoolGroups && (cnt <= kPoolAll || (cnt + 31) / 32 >= (int64_t)k) &&
+      merge_pool_short(src, (int)cnt, k, pad_short, sel, out_scores + (int64_t)q * k,
+                       out_idx + (int64_t)q * k))
+    return;
   const bool staged = cnt <= smem_keys;
   if (staged) {
     // L2 loads: a fused caller's pool was written earlier in the same launch
     for (int64_t i = threadIdx.x; i < cnt; i += blockDim.x) s_keys[i] = __ldcg(src + i);
     __syncthreads();
   }
-  // the short path needs a pruning threshold (k group heads) or a tiny pool
-  if (staged && cnt > 0 && cnt <= 32 * kPoolGroups &&
-      (cnt <= kPoolAll || (cnt + 31) / 32 >= (int64_t)k) &&
-      merge_pool_short(s_keys, (int)cnt, k, pad_short, sel, out_scores + (int64_t)q * k,
-                       out_idx + (int64_t)q * k))
-    return;
   if (staged && cnt >= k && (int)blockDim.x == kSelThreads && cnt + kBins + kBinCap <= smem_keys &&
       merge_pool_binned(s_keys, (int)cnt, k, out_scores + (int64_t)q * k, out_idx + (int64_t)q * k))
     return;
