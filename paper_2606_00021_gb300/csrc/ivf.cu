@@ -867,10 +867,22 @@ __global__ void residual_kernel(const float* __restrict__ x, int64_t n, int v,
 constexpr int kScanThreads = 256;
 constexpr int kFlatStride = 132;  // padded row stride (floats) of staged vectors, v <= 128
 
+// 16-byte asynchronous global -> shared copy through L2 (cp.async.cg);
+// cp_async_wait() completes the thread's copies.
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(ptx::smem_u32(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
 // One block per (probe p, query qi).  Flat: each thread scores one staged
 // vector (<q, x> in index order).  PQ: the block stages the query's lookup
-// table in shared memory; each thread reads one code row and sums
-// coarse + LUT[0][c_0] + ... + LUT[pq_m-1][c_{pq_m-1}].
+// table in shared memory (copies issued before the probe's cell is read,
+// which they do not depend on); each thread reads its code row (16 codes
+// per 16-byte load when pq_m % 16 == 0) and sums
+// coarse + LUT[0][c_0] + ... + LUT[pq_m-1][c_{pq_m-1}] in that order.
 // Candidates go to the query's pool (warp-aggregated append).
 __global__ void __launch_bounds__(kScanThreads)
 ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries,
@@ -886,28 +898,45 @@ ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries,
   float* sq = sm;                  // [v]
   float* stage = sm + 128;         // flat: [kScanThreads][kFlatStride]; pq: LUT [pq_m][256]
   const float* q = queries + (int64_t)qi * v;
-  for (int j = threadIdx.x; j < v; j += blockDim.x) sq[j] = q[j];
+  if (ix.pq_m > 0) {  // the lookup table goes to shared memory while the cell is read
+    const float4* src = reinterpret_cast<const float4*>(lut + (int64_t)qi * ix.pq_m * 256);
+    for (int e = threadIdx.x; e < ix.pq_m * 64; e += blockDim.x)
+      cp_async16(reinterpret_cast<float4*>(stage) + e, src + e);
+  } else {
+    for (int j = threadIdx.x; j < v; j += blockDim.x) sq[j] = q[j];
+  }
   const int cell = probe_cell[(int64_t)qi * nprobe + p];
   const float coarse = probe_score[(int64_t)qi * nprobe + p];
   if (cell < 0 || cell >= ix.nlist) {
+    cp_async_wait();
     if (threadIdx.x == 0) raise_status(status, SENSE_DEVST_INTERNAL);
     return;
   }
-  __syncthreads();
   const int64_t lo = ix.offsets[cell], hi = ix.offsets[cell + 1];
+  cp_async_wait();
+  __syncthreads();
   uint64_t* dst = pool + (int64_t)qi * pool_cap;
   if (ix.pq_m > 0) {
-    const float4* src = reinterpret_cast<const float4*>(lut + (int64_t)qi * ix.pq_m * 256);
-    for (int e = threadIdx.x; e < ix.pq_m * 64; e += blockDim.x)
-      reinterpret_cast<float4*>(stage)[e] = src[e];
-    __syncthreads();
+    const bool wide = (ix.pq_m & 15) == 0;
     for (int64_t s0 = lo; s0 < hi; s0 += blockDim.x) {
       const int64_t slot = s0 + threadIdx.x;
       const bool live = slot < hi;
       float s = coarse;
       if (live) {
         const uint8_t* cr = ix.codes + slot * ix.pq_m;
-        for (int m = 0; m < ix.pq_m; ++m) s = __fadd_rn(s, stage[(m << 8) + cr[m]]);
+        if (wide) {
+          for (int m0 = 0; m0 < ix.pq_m; m0 += 16) {
+            const uint4 w4 = __ldg(reinterpret_cast<const uint4*>(cr + m0));
+            const uint32_t w[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+            for (int b = 0; b < 16; ++b) {
+              const uint32_t c = (w[b >> 2] >> (8 * (b & 3))) & 255u;
+              s = __fadd_rn(s, stage[((m0 + b) << 8) + c]);
+            }
+          }
+        } else {
+          for (int m = 0; m < ix.pq_m; ++m) s = __fadd_rn(s, stage[(m << 8) + cr[m]]);
+        }
       }
       const uint32_t at = warp_append(&counts[qi], live);
       if (live) {
