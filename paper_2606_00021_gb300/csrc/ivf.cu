@@ -488,11 +488,11 @@ coarse_lut_kernel(const float* __restrict__ cells, int64_t nlist, const float* _
 // The query side of an approximate search in one launch, per query row:
 // the normalised projection (project_bulk_kernel<true>: the row's blocks
 // form one cluster, block 0 writes the unit row), then, after the cluster
-// barrier that makes that row visible, the cluster's C blocks write the
-// coarse keys of every cell (blocks of 256 cells, the ALL_IP assignment
-// above, block b of the cells taken by cluster block b mod C) and the PQ
-// lookup tables (sub-quantizer m by cluster block m mod C), with the
-// arithmetic of coarse_lut_kernel.  It also empties the row's candidate
+// barrier that makes that row visible, the cluster's C blocks compute the
+// coarse keys of every cell (tiles of 256 cells, tile b taken by cluster
+// block b mod C; the ALL_IP arithmetic) into block 0's shared memory and
+// write the PQ lookup tables (sub-quantizer m by cluster block m mod C),
+// with the arithmetic of coarse_lut_kernel.  It also empties the row's candidate
 // pool for the list scan (counts[row] = 0).  After a second cluster barrier
 // block 0 selects the row's nprobe best cells from the coarse keys (the
 // block merge of merge_kernel, in the projection's shared memory).
@@ -501,20 +501,63 @@ __global__ void __launch_bounds__(256)
 project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __restrict__ w,
                       const float* __restrict__ mu, float* __restrict__ out,
                       const float* __restrict__ cells, int64_t nlist,
-                      uint64_t* __restrict__ coarse, const float* __restrict__ cb, int pq_m,
-                      int dsub, float* __restrict__ lut, uint32_t* __restrict__ counts,
-                      int nprobe, float* __restrict__ pscore, int32_t* __restrict__ pcell,
-                      int smem_keys, uint32_t* status) {
+                      const float* __restrict__ cb, int pq_m, int dsub, float* __restrict__ lut,
+                      uint32_t* __restrict__ counts, int nprobe, float* __restrict__ pscore,
+                      int32_t* __restrict__ pcell, int keys_off, uint32_t* status) {
   pdl_wait();  // inputs written by the kernels before this one
   pdl_launch_dependents();
   project_bulk_block<true>(x, d, w, D, mu, out, status);  // ends on a cluster barrier
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  extern __shared__ __align__(128) uint8_t smd[];
   const int64_t row = blockIdx.y;
   if (blockIdx.x == 0 && threadIdx.x == 0) counts[row] = 0u;  // the list scan's pool is empty
   const float* qrow = out + row * D;
   const int C = (int)gridDim.x, r = (int)blockIdx.x;
-  const int nblk = (int)((nlist + blockDim.x - 1) / blockDim.x);
-  for (int b = r; b < nblk; b += C)
-    assign_block<D, ALL_IP, true>(cells, nlist, D, qrow, 1, nullptr, coarse + row * nlist, b);
+  __shared__ float sqr[D];  // the normalised row
+  for (int j = threadIdx.x; j < D; j += blockDim.x) sqr[j] = qrow[j];
+  // coarse keys: tiles of 256 cells staged in shared memory by coalesced
+  // loads (row stride D + 1: conflict-free reads), each thread one cell's
+  // in-order dot product (the ALL_IP arithmetic), the key stored straight
+  // into block 0's shared memory for the cell selection
+  constexpr int kTileCells = 256;
+  float* tile = reinterpret_cast<float*>(smd);  // [kTileCells][D + 1]
+  uint64_t* keys0 = cl.map_shared_rank(reinterpret_cast<uint64_t*>(smd + keys_off), 0);
+  const int ntile = (int)((nlist + kTileCells - 1) / kTileCells);
+  for (int b = r; b < ntile; b += C) {
+    const int64_t c0 = (int64_t)b * kTileCells;
+    const int rows = (int)min((int64_t)kTileCells, nlist - c0);
+    __syncthreads();  // the previous tile (and sqr) are complete / used
+    const float4* src4 = reinterpret_cast<const float4*>(cells + c0 * D);
+    const int n4 = rows * (D / 4);
+    for (int e0 = threadIdx.x; e0 < n4; e0 += 16 * blockDim.x) {  // sixteen loads in flight
+      float4 v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int e = e0 + u * blockDim.x;
+        v[u] = e < n4 ? __ldg(src4 + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int e = e0 + u * blockDim.x;
+        if (e < n4) {
+          float* dst = tile + (e / (D / 4)) * (D + 1) + 4 * (e % (D / 4));
+          dst[0] = v[u].x;
+          dst[1] = v[u].y;
+          dst[2] = v[u].z;
+          dst[3] = v[u].w;
+        }
+      }
+    }
+    __syncthreads();
+    for (int t = threadIdx.x; t < rows; t += blockDim.x) {
+      const float* xr = tile + t * (D + 1);
+      float sc = 0.0f;
+#pragma unroll 8
+      for (int j = 0; j < D; ++j) sc = madd(sc, xr[j], sqr[j]);
+      keys0[c0 + t] = cand_key(sc, (uint32_t)(c0 + t));
+    }
+  }
   __shared__ float sq[128];
   for (int m = r; m < pq_m; m += C) {
     __syncthreads();
@@ -528,12 +571,10 @@ project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __rest
       lut[row * pq_m * 256 + e] = s;
     }
   }
-  cooperative_groups::this_cluster().sync();  // every block's coarse keys are written
-  if (r == 0) {
-    extern __shared__ __align__(128) uint8_t smb_keys[];
-    merge_pool_block(coarse, nullptr, nlist, nprobe, pscore, pcell, status, 0, (int)row,
-                     reinterpret_cast<uint64_t*>(smb_keys), smem_keys);
-  }
+  cl.sync();  // every block's coarse keys are in block 0's shared memory
+  if (r == 0)
+    merge_pool_block(nullptr, nullptr, nlist, nprobe, pscore, pcell, status, 0, (int)row,
+                     reinterpret_cast<uint64_t*>(smd + keys_off), (int)nlist, true);
 }
 
 sense_status launch_coarse_lut(const sense_ivf* ix, const float* queries, int q, uint64_t* coarse,
@@ -562,24 +603,27 @@ sense_status launch_coarse_lut(const sense_ivf* ix, const float* queries, int q,
 }
 
 size_t project_bulk_smem(int d, bool mean);
-constexpr size_t kProjectCoarseMax = 172 * 1024;  // + 51 KB static for D = 64 (<= 227 KB)
+constexpr size_t kProjectCoarseMax = 200 * 1024;  // + ~20 KB static (<= 227 KB)
 
 // Launches project_coarse_kernel when the row's projection blocks fit one
 // cluster and its shared memory; *done = false (nothing launched) otherwise.
 sense_status launch_project_coarse(const uint16_t* x, int n, int d, const float* basis,
-                                   const float* mean, float* out, const sense_ivf* ix,
-                                   uint64_t* coarse, float* lut, uint32_t* counts, int nprobe,
-                                   float* pscore, int32_t* pcell, cudaStream_t s, bool* done) {
+                                   const float* mean, float* out, const sense_ivf* ix, float* lut,
+                                   uint32_t* counts, int nprobe, float* pscore, int32_t* pcell,
+                                   cudaStream_t s, bool* done) {
   *done = false;
   const int v = ix->v;
-  // the shared memory also stages the row's coarse keys for the cell selection
-  const size_t smem = std::max(project_bulk_smem(d, mean != nullptr), (size_t)ix->nlist * 8);
+  // the projection's shared memory is reused for the cell tiles; the row's
+  // coarse keys follow it (block 0's copy is the one used)
+  const size_t keys_off =
+      (std::max(project_bulk_smem(d, mean != nullptr), (size_t)256 * (v + 1) * 4) + 127) & ~(size_t)127;
+  const size_t smem = keys_off + (size_t)ix->nlist * 8;
   const bool vdim = v == 4 || v == 8 || v == 16 || v == 32 || v == 64;
   if (!vdim || n > 64 || (v + 7) / 8 > 8 || smem > kProjectCoarseMax) return SENSE_OK;
   uint32_t* status = device_status_word();
   if (!status) return SENSE_ERR_OOM;
   void (*kern)(const uint16_t*, int, const float*, const float*, float*, const float*, int64_t,
-               uint64_t*, const float*, int, int, float*, uint32_t*, int, float*, int32_t*, int,
+               const float*, int, int, float*, uint32_t*, int, float*, int32_t*, int,
                uint32_t*) = nullptr;
   switch (v) {
     case 4: kern = project_coarse_kernel<4>; break;
@@ -608,9 +652,9 @@ sense_status launch_project_coarse(const uint16_t* x, int n, int d, const float*
   cfg.numAttrs = 2;
   LaunchScope ls(K_PROJECT, s);
   st = cuda_check(cudaLaunchKernelEx(&cfg, kern, x, d, basis, mean, out,
-                                     (const float*)ix->centroids, (int64_t)ix->nlist, coarse,
+                                     (const float*)ix->centroids, (int64_t)ix->nlist,
                                      (const float*)ix->codebooks, ix->pq_m, ix->dsub, lut, counts,
-                                     nprobe, pscore, pcell, (int)(smem / 8), status),
+                                     nprobe, pscore, pcell, (int)keys_off, status),
                   "launch project + coarse");
   if (st == SENSE_OK) *done = true;
   return st;
@@ -1475,8 +1519,8 @@ sense_status ann_step(bool draft, const sense_ivf* ix, const sense_datastore* ds
   const SearchPlan plan = search_plan(ix, q, nprobe);
   bool coarse_done = false;
   sense_status st = launch_project_coarse(
-      queries, q, ds->d, basis, mean, qproj, ix, reinterpret_cast<uint64_t*>(ws + plan.off_coarse),
-      reinterpret_cast<float*>(ws + plan.off_lut), reinterpret_cast<uint32_t*>(ws + plan.off_counts),
+      queries, q, ds->d, basis, mean, qproj, ix, reinterpret_cast<float*>(ws + plan.off_lut),
+      reinterpret_cast<uint32_t*>(ws + plan.off_counts),
       nprobe, reinterpret_cast<float*>(ws + plan.off_pscore),
       reinterpret_cast<int32_t*>(ws + plan.off_pcell), s, &coarse_done);
   if (st != SENSE_OK) return st;

@@ -125,9 +125,14 @@ __device__ __forceinline__ uint64_t warp_max64(uint64_t x) {
 // The keys are read where they are, in the pool (L2 loads, four per thread
 // in flight; a fused caller writes the pool earlier in the same launch):
 // both passes over them are coalesced, so no staging copy is needed.
+template <bool SMEM = false>  // SMEM: the keys are in shared memory
 __device__ bool merge_pool_short(const uint64_t* __restrict__ keys, int cnt, int k, int pad_short,
                                  uint64_t* cand, float* __restrict__ out_scores,
                                  int32_t* __restrict__ out_idx) {
+  auto key_at = [&](int i) -> uint64_t {
+    if constexpr (SMEM) return keys[i];
+    else return __ldcg(keys + i);
+  };
   __shared__ uint64_t s_heads[kPoolGroups];  // group maxima, then sorted in groups of 32
   __shared__ uint64_t s_t;
   __shared__ unsigned s_got;
@@ -146,7 +151,7 @@ __device__ bool merge_pool_short(const uint64_t* __restrict__ keys, int cnt, int
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int i = (g0 + u * nwarps) * 32 + lane;
-      x[u] = i < cnt ? __ldcg(keys + i) : 0ull;
+      x[u] = i < cnt ? key_at(i) : 0ull;
     }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
@@ -195,7 +200,7 @@ __device__ bool merge_pool_short(const uint64_t* __restrict__ keys, int cnt, int
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int i = i0 + u * blockDim.x;
-      x[u] = i < cnt ? __ldcg(keys + i) : 0ull;
+      x[u] = i < cnt ? key_at(i) : 0ull;
     }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
@@ -325,28 +330,34 @@ __device__ bool merge_pool_binned(const uint64_t* s_keys, int cnt, int k,
 
 // Top k of query q's pool into out_scores / out_idx rows q (one block per
 // query; s_keys: smem_keys keys of shared memory, kSmemKeys for the merge
-// kernels).  The binned path runs only with kSelThreads threads.  Every
-// return is block-uniform, so a caller may continue after a block barrier.
+// kernels).  With `in_smem` the pool_cap keys are already in s_keys (pool
+// and counts unused).  The binned path runs only with kSelThreads threads.
+// Every return is block-uniform, so a caller may continue after a block
+// barrier.
 __device__ void merge_pool_block(const uint64_t* __restrict__ pool,
                                  const uint32_t* __restrict__ counts, int64_t pool_cap, int k,
                                  float* __restrict__ out_scores, int32_t* __restrict__ out_idx,
                                  uint32_t* status, int pad_short, int q, uint64_t* s_keys,
-                                 int smem_keys = kSmemKeys) {
+                                 int smem_keys = kSmemKeys, bool in_smem = false) {
   __shared__ unsigned hist[256];
   __shared__ Digit dig;
   __shared__ unsigned n_sel;
   __shared__ uint64_t sel[SENSE_MAX_K];
-  const uint64_t* src = pool + (int64_t)q * pool_cap;
-  int64_t cnt = counts ? (int64_t)counts[q] : pool_cap;  // no counts: every slot is used
+  const uint64_t* src = in_smem ? s_keys : pool + (int64_t)q * pool_cap;
+  int64_t cnt = (counts && !in_smem) ? (int64_t)counts[q] : pool_cap;  // else every slot is used
   if (cnt > pool_cap) cnt = pool_cap;
-  // the short path (pool read in place) needs a pruning threshold (k group
-  // heads) or a tiny pool
-  if (cnt > 0 && cnt <= 32 * kPoolGroups && (cnt <= kPoolAll || (cnt + 31) / 32 >= (int64_t)k) &&
-      merge_pool_short(src, (int)cnt, k, pad_short, sel, out_scores + (int64_t)q * k,
-                       out_idx + (int64_t)q * k))
+  // the short path (pool read where it is) needs a pruning threshold (k
+  // group heads) or a tiny pool
+  const bool short_ok =
+      cnt > 0 && cnt <= 32 * kPoolGroups && (cnt <= kPoolAll || (cnt + 31) / 32 >= (int64_t)k);
+  if (short_ok &&
+      (in_smem ? merge_pool_short<true>(src, (int)cnt, k, pad_short, sel, out_scores + (int64_t)q * k,
+                                        out_idx + (int64_t)q * k)
+               : merge_pool_short<false>(src, (int)cnt, k, pad_short, sel,
+                                         out_scores + (int64_t)q * k, out_idx + (int64_t)q * k)))
     return;
-  const bool staged = cnt <= smem_keys;
-  if (staged) {
+  const bool staged = in_smem || cnt <= smem_keys;
+  if (staged && !in_smem) {
     // L2 loads: a fused caller's pool was written earlier in the same launch
     for (int64_t i = threadIdx.x; i < cnt; i += blockDim.x) s_keys[i] = __ldcg(src + i);
     __syncthreads();
