@@ -358,8 +358,21 @@ __device__ void merge_pool_block(const uint64_t* __restrict__ pool,
     return;
   const bool staged = in_smem || cnt <= smem_keys;
   if (staged && !in_smem) {
-    // L2 loads: a fused caller's pool was written earlier in the same launch
-    for (int64_t i = threadIdx.x; i < cnt; i += blockDim.x) s_keys[i] = __ldcg(src + i);
+    // L2 loads (a fused caller's pool was written earlier in the same
+    // launch), eight per thread in flight before their stores
+    for (int64_t i0 = threadIdx.x; i0 < cnt; i0 += 8 * (int64_t)blockDim.x) {
+      uint64_t v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int64_t i = i0 + u * (int64_t)blockDim.x;
+        v[u] = i < cnt ? __ldcg(src + i) : 0ull;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int64_t i = i0 + u * (int64_t)blockDim.x;
+        if (i < cnt) s_keys[i] = v[u];
+      }
+    }
     __syncthreads();
   }
   if (staged && cnt >= k && (int)blockDim.x == kSelThreads && cnt + kBins + kBinCap <= smem_keys &&
