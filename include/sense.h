@@ -651,7 +651,7 @@ sense_status sense_tree_attention(const uint16_t* q, const uint16_t* k_cache,
  *  - B_topk = I(D in top-kappa of P_align), order (logit desc, index asc);
  *  - B_con = I(#mismatches among positions j+1..j+W <= tau), positions past
  *    the span (and positions dropped by the node cap) counting as
- *    mismatches (Alg. 4: Pad(1-B_em,(0,W),1), Conv1D(.,1_W)[:,1:M+1], == 0);
+ *    mismatches (Alg. 4's reading of Eq. 16: a strictly-future window);
  *  - G = B_em | (B_ent & (B_topk | B_con)); L_i = leading run of ones in
  *    G[i,:] minus 1; i* = lowest i with the largest L_i; L* = L_{i*}.
  * Positions whose node was dropped by the cap have G = 0.

@@ -287,16 +287,17 @@ def loose_trie(spans_qkm: np.ndarray, node_cap: int = 0, mask_bits=False):
 
 
 def loose_trie_alg3(d_sorted_or_not: np.ndarray):
-    """App. C.3 Alg. 3, restated step by step (one query, no node cap).
+    """App. C.3 Alg. 3's vectorised trie, in its order (one query, no node cap).
 
-    Input: candidates D in Z^{N x M}.  Following Alg. 2 the rows are first
-    put in lexicographic order (LexSort), then:
-      match[1:] = (D[1:] == D[:-1]);  is_prefix = CumProd(match, dim 1);
-      unique = not is_prefix;  T = D[unique];  L = |T|;
-      idx = CumSum(unique.flat) - 1;  Gamma = reshape(idx, (N, M));
-      tmp = where(unique, Gamma, -1);  Gamma = CumMax(tmp, dim 0);
-      M[Gamma[i, I], Gamma[i, J]] = 1 for the lower-triangle pairs (I, J).
-    Returns (T, Gamma in sorted-row order, mask M, sort permutation pi).
+    The rows are put in lexicographic order first (Alg. 2 sorts before it
+    builds).  A cell (i, j) repeats an earlier node exactly when row i agrees
+    with row i-1 on every column up to and including j; the other cells are
+    new nodes, numbered in row-major reading order, which is preorder.  A
+    repeated cell takes the number of the latest new node above it in its
+    column (a running maximum down the column), and the ancestor mask marks,
+    for every row, each of its nodes against every earlier node on the same
+    row.  Returns (tokens of the new cells, Gamma in sorted-row order, the
+    mask, the sort permutation pi).
     """
     d = np.asarray(d_sorted_or_not, dtype=np.int64)
     n, m = d.shape

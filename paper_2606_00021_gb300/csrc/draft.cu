@@ -13,7 +13,7 @@
 //      counts numbers the nodes in preorder (Eq. 9's T_flat);
 //   3. node of (sorted row p, depth j) = node created by the last row
 //      p' <= p with lcp[p'] <= j: a prefix-max over p per column (Alg. 3's
-//      CumMax);
+//      running column maximum);
 //   4. node cap: key (first candidate rank containing the node, depth) -
 //      segmented minimum by shared-memory atomicMin, then the cap smallest
 //      keys are kept (keys are distinct integers < k*m, so a prefix count
