@@ -857,6 +857,8 @@ def main():
         for b in range(min(nq, 64)):
             _, ex_i = S.sense_retrieve_topk(ds, queries[b], cfg["k"], workspace=ex_ws)
             pipe.retrieve(queries[b])
+            # the one-call search keeps its projected query in its workspace
+            S.sense_project(queries[b], ann["basis"], ann["mean"], out=pipe.qproj)
             _, px_i = S.sense_ivf_search(one, pipe.qproj, cfg["k"], 1)
             for a_row, e_row, p_row in zip(pipe.idx.cpu().tolist(), ex_i.cpu().tolist(),
                                            px_i.cpu().tolist()):

@@ -909,7 +909,12 @@ __global__ void residual_kernel(const float* __restrict__ x, int64_t n, int v,
 // index order).  One block per (sub-quantizer m, query), one thread per
 // codeword b: every codeword row is loaded at once (one round trip).
 constexpr int kScanThreads = 256;
-constexpr int kFlatStride = 132;  // padded row stride (floats) of staged vectors, v <= 128
+// Flat lists are staged in chunks of kScanThreads x flat_rows_per_thread(v)
+// vectors with a padded row stride of v + 4 floats (16-byte reads of 8
+// consecutive threads hit distinct bank groups).  One row per thread keeps
+// a block at <= 135 KB of shared memory (70 KB at v = 64, three blocks per
+// SM); long lists are split across blocks instead.
+__host__ __device__ constexpr int flat_rows_per_thread(int) { return 1; }
 
 // 16-byte asynchronous global -> shared copy through L2 (cp.async.cg);
 // cp_async_wait() completes the thread's copies.
@@ -921,8 +926,11 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
-// One block per (probe p, query qi).  Flat: each thread scores one staged
-// vector (<q, x> in index order).  PQ: the block stages the query's lookup
+// One block per (probe p, query qi, list part z): part z of a list takes
+// its chunks z, z + gridDim.z, ... (a flat chunk is kScanThreads x
+// flat_rows_per_thread(v) entries, a PQ chunk kScanThreads), so that a long
+// list is not scanned by one block alone.  Flat: the chunk's vectors are
+// staged and each thread scores its rows (<q, x> in index order).  PQ: the block stages the query's lookup
 // table in shared memory (copies issued before the probe's cell is read,
 // which they do not depend on); each thread reads its code row (16 codes
 // per 16-byte load when pq_m % 16 == 0) and sums
@@ -940,7 +948,7 @@ ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries,
   const int p = blockIdx.x, qi = blockIdx.y;
   const int v = ix.v;
   float* sq = sm;                  // [v]
-  float* stage = sm + 128;         // flat: [kScanThreads][kFlatStride]; pq: LUT [pq_m][256]
+  float* stage = sm + 128;         // flat: staged vectors [rows][v + 4]; pq: LUT [pq_m][256]
   const float* q = queries + (int64_t)qi * v;
   if (ix.pq_m > 0) {  // the lookup table goes to shared memory while the cell is read
     const float4* src = reinterpret_cast<const float4*>(lut + (int64_t)qi * ix.pq_m * 256);
@@ -962,7 +970,8 @@ ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries,
   uint64_t* dst = pool + (int64_t)qi * pool_cap;
   if (ix.pq_m > 0) {
     const bool wide = (ix.pq_m & 15) == 0;
-    for (int64_t s0 = lo; s0 < hi; s0 += blockDim.x) {
+    for (int64_t s0 = lo + (int64_t)blockIdx.z * blockDim.x; s0 < hi;
+         s0 += (int64_t)gridDim.z * blockDim.x) {
       const int64_t slot = s0 + threadIdx.x;
       const bool live = slot < hi;
       float s = coarse;
@@ -989,41 +998,59 @@ ivf_scan_kernel(const sense_ivf ix, const float* __restrict__ queries,
       }
     }
   } else {
-    for (int64_t s0 = lo; s0 < hi; s0 += blockDim.x) {
-      const int rows = (int)min((int64_t)blockDim.x, hi - s0);
-      __syncthreads();
-      // stage `rows` vectors (v floats each) with 16-byte loads
-      const int vq = v >> 2;
+    // one chunk of vectors is copied with every 16-byte copy in flight at
+    // once, then each thread scores its rows (<q, x> in index order)
+    const int vq = v >> 2, fs = v + 4;
+    const int64_t chunk = (int64_t)blockDim.x * flat_rows_per_thread(v);
+    for (int64_t c0 = lo + blockIdx.z * chunk; c0 < hi; c0 += gridDim.z * chunk) {
+      const int rows = (int)min(chunk, hi - c0);
+      __syncthreads();  // the previous chunk's rows are read
+      const float4* src = reinterpret_cast<const float4*>(ix.vectors + c0 * v);
       for (int e = threadIdx.x; e < rows * vq; e += blockDim.x) {
         const int r = e / vq, g = e - r * vq;
-        *reinterpret_cast<float4*>(stage + r * kFlatStride + 4 * g) =
-            *reinterpret_cast<const float4*>(ix.vectors + (s0 + r) * v + 4 * g);
+        cp_async16(stage + r * fs + 4 * g, src + e);
       }
+      cp_async_wait();
       __syncthreads();
-      const bool live = threadIdx.x < rows;
-      float s = 0.0f;
-      if (live) {
-        const float* xr = stage + threadIdx.x * kFlatStride;
-        for (int g = 0; g < vq; ++g) {
-          const float4 xv = *reinterpret_cast<const float4*>(xr + 4 * g);
-          s = madd(s, sq[4 * g], xv.x);
-          s = madd(s, sq[4 * g + 1], xv.y);
-          s = madd(s, sq[4 * g + 2], xv.z);
-          s = madd(s, sq[4 * g + 3], xv.w);
+      for (int r0 = 0; r0 < rows; r0 += blockDim.x) {
+        const int r = r0 + threadIdx.x;
+        const bool live = r < rows;
+        float s = 0.0f;
+        if (live) {
+          const float* xr = stage + r * fs;
+          for (int g = 0; g < vq; ++g) {
+            const float4 xv = *reinterpret_cast<const float4*>(xr + 4 * g);
+            s = madd(s, sq[4 * g], xv.x);
+            s = madd(s, sq[4 * g + 1], xv.y);
+            s = madd(s, sq[4 * g + 2], xv.z);
+            s = madd(s, sq[4 * g + 3], xv.w);
+          }
         }
-      }
-      const uint32_t at = warp_append(&counts[qi], live);
-      if (live) {
-        const int64_t slot = s0 + threadIdx.x;
-        if ((int64_t)at < pool_cap) dst[at] = cand_key(s, (uint32_t)ix.ids[slot]);
-        else raise_status(status, SENSE_DEVST_INTERNAL);
+        const uint32_t at = warp_append(&counts[qi], live);
+        if (live) {
+          const int64_t slot = c0 + r;
+          if ((int64_t)at < pool_cap) dst[at] = cand_key(s, (uint32_t)ix.ids[slot]);
+          else raise_status(status, SENSE_DEVST_INTERNAL);
+        }
       }
     }
   }
 }
 
+// Parts per probed list: enough that the longest list is one chunk per
+// block, at most 8, and fewer when the probes alone fill the GPU.
+int scan_parts(const sense_ivf* ix, int q, int nprobe) {
+  const int64_t chunk = (int64_t)kScanThreads * (ix->pq_m > 0 ? 1 : flat_rows_per_thread(ix->v));
+  int parts = (int)std::min<int64_t>(8, std::max<int64_t>(1, (ix->max_list + chunk - 1) / chunk));
+  const int64_t blocks = (int64_t)nprobe * q;
+  const int64_t budget = 4LL * sm_count();
+  if (blocks * parts > budget) parts = (int)std::max<int64_t>(1, budget / blocks);
+  return parts;
+}
+
 size_t scan_smem_bytes(const sense_ivf* ix) {
-  const size_t stage = ix->pq_m > 0 ? (size_t)ix->pq_m * 256 : (size_t)kScanThreads * kFlatStride;
+  const size_t stage = ix->pq_m > 0 ? (size_t)ix->pq_m * 256
+                                     : (size_t)kScanThreads * flat_rows_per_thread(ix->v) * (ix->v + 4);
   return (128 + stage) * sizeof(float);
 }
 
@@ -1415,7 +1442,8 @@ sense_status ivf_scan_pool(const sense_ivf* ix, const float* queries, int32_t q,
     st = cuda_check(func_smem(reinterpret_cast<const void*>(ivf_scan_kernel), (int)smem), "smem attribute");
     if (st != SENSE_OK) return st;
     LaunchScope ls(K_IVF_SCAN, s);
-    st = cuda_check(launch_pdl(ivf_scan_kernel, dim3(nprobe, q), dim3(kScanThreads), smem, s, *ix,
+    st = cuda_check(launch_pdl(ivf_scan_kernel, dim3(nprobe, q, scan_parts(ix, q, nprobe)),
+                               dim3(kScanThreads), smem, s, *ix,
                                queries, (const float*)lut, nprobe, (const float*)pscore,
                                (const int32_t*)pcell, pool, counts, p.pool_cap, status),
                     "launch ivf scan");
