@@ -10,7 +10,8 @@
 //    128-row tiles of the scan's tile set);
 //  - warp 0 (one lane) streams, per 64-column slice of d, both 128 x 64 key
 //    tiles and the padded nq x 64 query tile with 2-D TMA loads (128-byte
-//    swizzle, keys marked evict-first in L2) into a multi-stage ring;
+//    swizzle, keys marked evict-first in L2) into a multi-stage ring, two
+//    consecutive slices per stage up to 32 queries;
 //  - warp 1 (one lane) issues tcgen05.mma kind::f16 (M = 128 keys,
 //    N = nq queries, K = 16) into fp32 TMEM accumulators: two tiles x two
 //    buffers, so the epilogue of one unit overlaps the MMAs of the next;
@@ -47,6 +48,7 @@ struct TcArgs {
   int64_t n_half;  // 128-row work tiles
   int64_t n_work;  // n_half * 128
   int kc;      // 64-column slices of d
+  int cps;     // slices per ring stage
   int stages;
   uint32_t tmem_cols;
   const uint64_t* thresh;
@@ -99,7 +101,11 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tm_keys,
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int S = a.stages;
-  const uint32_t stage_bytes = 2 * kTileBytes + a.nq * kBlockK * 2;
+  const int cps = a.cps;
+  // a stage holds cps consecutive 64-column slices: slice c of tile t at
+  // (2 c + t) kTileBytes, then the query slices (nq x 64 each)
+  const uint32_t q_off = (uint32_t)(2 * cps * kTileBytes);
+  const uint32_t stage_bytes = (uint32_t)cps * (2 * kTileBytes + a.nq * kBlockK * 2);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
   // bars: full[S], empty[S], acc_full[2], acc_empty[2], mma_done
   Shared* sh = reinterpret_cast<Shared*>(bars + 2 * S + 5);
@@ -146,19 +152,25 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tm_keys,
     for (int64_t u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
       const int64_t t0 = key_tile<MODE>(2 * u);
       const int64_t t1 = (2 * u + 1 < a.n_half) ? key_tile<MODE>(2 * u + 1) : dummy_tile;
-      for (int kc = 0; kc < a.kc; ++kc) {
+      for (int kc = 0; kc < a.kc; kc += cps) {
         if (!wait_bar(bar(EMPTY + s), ph ^ 1u, abort, a.status)) {
           ok = false;
           break;
         }
         uint8_t* st = smem + (size_t)s * stage_bytes;
+        // slices past d (the last stage when kc % cps != 0) are zero-filled
+        // and still count their full box bytes
         ptx::mbar_arrive_expect_tx(bar(FULL + s), stage_bytes);
-        ptx::tma_load_2d(ptx::smem_u32(st), &tm_keys, bar(FULL + s), kc * kBlockK,
-                         (int32_t)(t0 * 128), pol_keys);
-        ptx::tma_load_2d(ptx::smem_u32(st + kTileBytes), &tm_keys, bar(FULL + s), kc * kBlockK,
-                         (int32_t)(t1 * 128), pol_keys);
-        ptx::tma_load_2d(ptx::smem_u32(st + 2 * kTileBytes), &tm_q, bar(FULL + s), kc * kBlockK,
-                         0, pol_q);
+        for (int c = 0; c < cps; ++c) {
+          const int col = (kc + c) * kBlockK;
+          ptx::tma_load_2d(ptx::smem_u32(st + (2 * c) * kTileBytes), &tm_keys, bar(FULL + s), col,
+                           (int32_t)(t0 * 128), pol_keys);
+          ptx::tma_load_2d(ptx::smem_u32(st + (2 * c + 1) * kTileBytes), &tm_keys, bar(FULL + s),
+                           col, (int32_t)(t1 * 128), pol_keys);
+        }
+        for (int c = 0; c < cps; ++c)
+          ptx::tma_load_2d(ptx::smem_u32(st + q_off + c * a.nq * kBlockK * 2), &tm_q, bar(FULL + s),
+                           (kc + c) * kBlockK, 0, pol_q);
         ++issued;
         if (++s == S) {
           s = 0;
@@ -192,19 +204,23 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tm_keys,
       ptx::tc_fence_after();
       const uint32_t d0 = tmem + (uint32_t)((2 * b) * a.nq);
       const uint32_t d1 = tmem + (uint32_t)((2 * b + 1) * a.nq);
-      for (int kc = 0; kc < a.kc; ++kc) {
+      for (int kc = 0; kc < a.kc; kc += cps) {
         if (!wait_bar(bar(FULL + s), ph, abort, a.status)) {
           ok = false;
           break;
         }
         ptx::tc_fence_after();
         const uint32_t st = ptx::smem_u32(smem + (size_t)s * stage_bytes);
+        for (int c = 0; c < cps; ++c) {
+          const uint32_t ta = st + (uint32_t)(2 * c) * kTileBytes;
+          const uint32_t qa = st + q_off + (uint32_t)(c * a.nq * kBlockK * 2);
 #pragma unroll
-        for (int kk = 0; kk < kBlockK / 16; ++kk) {
-          const uint64_t db = ptx::desc_sw128(st + 2 * kTileBytes + kk * 32);
-          const uint32_t acc = (kc | kk) != 0;
-          ptx::mma_bf16(d0, ptx::desc_sw128(st + kk * 32), db, idesc, acc);
-          ptx::mma_bf16(d1, ptx::desc_sw128(st + kTileBytes + kk * 32), db, idesc, acc);
+          for (int kk = 0; kk < kBlockK / 16; ++kk) {
+            const uint64_t db = ptx::desc_sw128(qa + kk * 32);
+            const uint32_t acc = (kc | c | kk) != 0;
+            ptx::mma_bf16(d0, ptx::desc_sw128(ta + kk * 32), db, idesc, acc);
+            ptx::mma_bf16(d1, ptx::desc_sw128(ta + kTileBytes + kk * 32), db, idesc, acc);
+          }
         }
         ptx::mma_commit(bar(EMPTY + s));
         if (++s == S) {
@@ -336,8 +352,14 @@ sense_status make_map(CUtensorMap* m, const void* base, int64_t rows, int d, int
   return SENSE_OK;
 }
 
-int stages_for(int nq) {
-  const int stage = 2 * kTileBytes + nq * kBlockK * 2;
+// 64-column slices per ring stage: consecutive slices of a key row go out
+// in one stage, so each row is requested cps x 128 contiguous bytes at a
+// time.  Two slices keep three stages (192 KB of keys) in flight up to 32
+// queries; past that they would cut the ring to two stages.
+int slices_per_stage(int nq) { return nq <= 32 ? 2 : 1; }
+
+int stages_for(int nq, int cps) {
+  const int stage = cps * (2 * kTileBytes + nq * kBlockK * 2);
   const int budget = 227 * 1024 - 1024 - 512 - 8 * 128;
   int s = budget / stage;
   return s > 8 ? 8 : s;
@@ -347,8 +369,9 @@ int stages_for(int nq) {
 
 size_t scan_tc_smem_bytes(int d, int nq) {
   (void)d;
-  const int S = stages_for(nq);
-  const size_t stage = 2 * kTileBytes + (size_t)nq * kBlockK * 2;
+  const int cps = slices_per_stage(nq);
+  const int S = stages_for(nq, cps);
+  const size_t stage = (size_t)cps * (2 * kTileBytes + (size_t)nq * kBlockK * 2);
   return 1024 + S * stage + (2 * S + 5) * 8 + sizeof(Shared) + 8 * 128;
 }
 
@@ -384,7 +407,12 @@ sense_status launch_scan_tc(const uint16_t* keys, int64_t n, int d, const uint16
   a.n_half = n_half;
   a.n_work = n_half * 128;
   a.kc = (d + kBlockK - 1) / kBlockK;
-  a.stages = stages_for(nq);
+  a.cps = slices_per_stage(nq);
+  a.stages = stages_for(nq, a.cps);
+  if (a.stages < 2) {
+    a.cps = 1;
+    a.stages = stages_for(nq, 1);
+  }
   uint32_t cols = 32;
   while (cols < (uint32_t)(4 * nq)) cols <<= 1;
   a.tmem_cols = cols;

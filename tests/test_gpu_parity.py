@@ -79,7 +79,7 @@ def test_retrieve_tensor_path_matches_oracle(S, n, d, q, k, clusters):
 @pytest.mark.parametrize("n,d,q,k", [(20000, 256, 1, 64), (20000, 256, 8, 17),
                                      (150000, 128, 3, 100), (4096, 64, 2, 4096 // 4),
                                      (20000, 256, 16, 64), (150000, 192, 40, 100),
-                                     (9000, 64, 129, 33)])
+                                     (9000, 64, 129, 33), (30000, 192, 24, 50)])
 def test_retrieve_lattice_bit_exact(S, n, d, q, k):
     """Lattice entries make every fp32 sum exact: scores, order and ties
     (lower index first) must equal the oracle bit for bit."""
