@@ -48,8 +48,9 @@ NCU_TRAFFIC_PER_UNIT = {
     ("scan_gemv", 4096): (2147567104 + 2790912) / 262144,
     # 262,144 x 8192 keys: 4,295,055,872 B read + 2,958,336 B written
     ("scan_gemv", 8192): (4295055872 + 2958336) / 262144,
-    # 524,288 x 3584 keys, sample + rest launches of one step
-    ("scan_tc", 3584): (235048448 + 2988800 + 3523437824 + 185600) / 524288,
+    # 524,288 x 3584 keys, sample + rest launches of one step (two slices
+    # per ring stage)
+    ("scan_tc", 3584): (235059200 + 3039488 + 3523413504 + 171008) / 524288,
     # 4 queries of the k = 64 sweep: 3,774 root / inner-node rows of 128,256 logits
     ("gate_rows", 128256): (1939918336 + 3338240) / 3773.9375,
 }

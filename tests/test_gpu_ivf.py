@@ -474,3 +474,53 @@ def test_ann_draft_equals_separate_calls(S, pq, rerank, q, k, cap, nlist, nprobe
         for key in ("num_nodes", "tokens", "parent", "depth", "gamma", "mask_bits"):
             assert torch.equal(got[key], tr[key]), key
     ix.close()
+
+
+@cuda
+@pytest.mark.parametrize("v,nlist,nprobe,pq", [
+    (64, 2048, 33, False),   # one 256-cell tile per block of the 8-block cluster
+    (64, 4096, 64, True),    # two tiles per block
+    (64, 6144, 17, False),   # three tiles per block
+    (64, 8192, 64, False),   # four tiles per block
+    (64, 4096, 100, False),
+    (16, 4096, 32, False),   # two blocks, eight tiles each
+    (64, 4096, 1, False),
+])
+def test_ann_search_cell_selection(S, v, nlist, nprobe, pq):
+    """The query-side launch's cell selection (coarse keys of the cluster's
+    blocks merged in block 0's shared memory) probes the same cells as the
+    coarse scores and merge called one by one: k = 1024 over short lists
+    returns every scanned entry, so equal results mean equal cell sets."""
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(nlist + nprobe)
+    n, d, q, k = 20000, 512, 2, 1024
+    keys = synth.clustered_unit_keys(n, d, 64, seed=29, device=dev)
+    spans = synth.spans_uniform(n, 8, 5, seed=2, device=dev)
+    ds = S.sense_datastore_build(keys, spans)
+    basis = _dev(np.linalg.qr(rng.standard_normal((d, v)))[0].T.astype(np.float32).copy())
+    mean = _dev((0.01 * rng.standard_normal(d)).astype(np.float32))
+    kp = S.sense_project(keys, basis, mean)
+    cent = S.sense_kmeans(kp, kp[:nlist].clone(), 2, True)
+    cb = None
+    if pq:
+        _, res = S.sense_ivf_residuals(kp, cent)
+        cb = torch.stack([S.sense_kmeans(res[:, 4 * mm:4 * mm + 4].contiguous(),
+                                         res[:256, 4 * mm:4 * mm + 4].contiguous(), 2, False)
+                          for mm in range(v // 4)])
+    ix = S.sense_ivf_build(kp, cent, cb)
+    qs, _ = synth.noisy_queries(keys, q, seed=31)
+    sc, idx = S.sense_ann_search(ix, ds, qs, basis, mean, k, nprobe)
+    torch.cuda.synchronize()
+    st_one = S.sense_device_status(clear=True)
+    qp = S.sense_project(qs, basis, mean)
+    sc2, idx2, probes = S.sense_ivf_search(ix, qp, k, nprobe, want_probes=True)
+    torch.cuda.synchronize()
+    assert S.sense_device_status(clear=True) == st_one
+    sizes = (ix.arrays()["offsets"][1:] - ix.arrays()["offsets"][:-1])
+    scanned = sizes[probes.long()].sum(dim=1)
+    assert int(scanned.max()) < k  # the whole pool is in the result
+    assert torch.equal(sc, sc2) and torch.equal(idx, idx2)
+    for qi in range(q):
+        got = set(idx[qi][idx[qi] >= 0].tolist())
+        assert len(got) == int(scanned[qi])
+    ix.close()
