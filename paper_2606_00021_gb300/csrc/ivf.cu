@@ -46,6 +46,7 @@
 #include <cooperative_groups.h>
 
 #include <algorithm>
+#include <mutex>
 #include <vector>
 
 #include "common.cuh"
@@ -106,12 +107,12 @@ __device__ __forceinline__ float4 load_x4(const uint16_t* xr, const float* mu, i
 
 constexpr long long kBulkWaitCycles = 4000000000LL;
 
-// Block (output group of 8, row): the row of x (bf16), the mean and the W
-// rows of the block's outputs are brought in by one bulk copy each on one
-// mbarrier, so the block pays a single round trip; warp w then computes
-// output 8 * blockIdx.x + w from shared memory in the order of
+// Block (output group of opb <= 8, row): the row of x (bf16), the mean and
+// the W rows of the block's outputs are brought in by one bulk copy each on
+// one mbarrier, so the block pays a single round trip; warp w < opb then
+// computes output opb * blockIdx.x + w from shared memory in the order of
 // project_rows_kernel (lane l: its 4-column groups ascending; butterfly).
-// NORM: the blocks of a row are one cluster (gridDim.x <= 8); block 0
+// NORM: the blocks of a row are one cluster (gridDim.x <= 16); block 0
 // gathers the v outputs through distributed shared memory and writes the
 // row divided by its L2 norm, in the order of normalize_rows_kernel.  A
 // copy that never lands (bounded wait) sets SENSE_DEVST_TIMEOUT; the row is
@@ -120,18 +121,19 @@ template <bool NORM>
 __device__ __forceinline__ void project_bulk_block(const uint16_t* __restrict__ x, int d,
                                                    const float* __restrict__ w, int v,
                                                    const float* __restrict__ mu,
-                                                   float* __restrict__ out, uint32_t* status) {
+                                                   float* __restrict__ out, uint32_t* status,
+                                                   int opb = 8) {
   extern __shared__ __align__(128) uint8_t smb[];
   __shared__ __align__(8) uint64_t bar;
   __shared__ float s_out[8];
   __shared__ int s_fail;
   uint16_t* sxb = reinterpret_cast<uint16_t*>(smb);                   // [d]
   float* smu = reinterpret_cast<float*>(smb + (size_t)d * 2);         // [d] when mu
-  float* sw = smu + (mu ? d : 0);                                     // [8][d]
+  float* sw = smu + (mu ? d : 0);                                     // [opb][d]
   const int64_t row = blockIdx.y;
   const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int o = blockIdx.x * 8 + wid;
-  const int nw = min(8, v - (int)blockIdx.x * 8);
+  const int nw = min(opb, v - (int)blockIdx.x * opb);  // outputs of this block
+  const int o = wid < nw ? (int)blockIdx.x * opb + wid : v;
   const uint32_t b = ptx::smem_u32(&bar);
   if (threadIdx.x == 0) {
     ptx::mbar_init(b, 1);
@@ -143,7 +145,7 @@ __device__ __forceinline__ void project_bulk_block(const uint16_t* __restrict__ 
     ptx::bulk_load(ptx::smem_u32(sxb), x + row * d, (uint32_t)d * 2u, b, pol);
     if (mu) ptx::bulk_load(ptx::smem_u32(smu), mu, (uint32_t)d * 4u, b, pol);
     for (int k = 0; k < nw; ++k)
-      ptx::bulk_load(ptx::smem_u32(sw + (size_t)k * d), w + (int64_t)(blockIdx.x * 8 + k) * d,
+      ptx::bulk_load(ptx::smem_u32(sw + (size_t)k * d), w + (int64_t)(blockIdx.x * opb + k) * d,
                      (uint32_t)d * 4u, b, pol);
   }
   __syncthreads();
@@ -191,7 +193,7 @@ __device__ __forceinline__ void project_bulk_block(const uint16_t* __restrict__ 
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           const int oo = 32 * t + lane;
-          part[t] = (oo < v) ? *cl.map_shared_rank(&s_out[oo & 7], (unsigned)(oo >> 3)) : 0.0f;
+          part[t] = (oo < v) ? *cl.map_shared_rank(&s_out[oo % opb], (unsigned)(oo / opb)) : 0.0f;
         }
         float ss = 0.0f;
 #pragma unroll
@@ -221,7 +223,9 @@ project_bulk_kernel(const uint16_t* __restrict__ x, int d, const float* __restri
   project_bulk_block<NORM>(x, d, w, v, mu, out, status);
 }
 
-size_t project_bulk_smem(int d, bool mean) { return (size_t)d * 2 + (mean ? (size_t)d * 4 : 0) + 32 * (size_t)d; }
+size_t project_bulk_smem(int d, bool mean, int opb = 8) {
+  return (size_t)d * 2 + (mean ? (size_t)d * 4 : 0) + (size_t)opb * 4 * d;
+}
 constexpr size_t kProjectBulkMax = 200 * 1024;
 
 // Block (output group, row): the centred row is staged in shared memory once;
@@ -503,10 +507,10 @@ project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __rest
                       const float* __restrict__ cells, int64_t nlist,
                       const float* __restrict__ cb, int pq_m, int dsub, float* __restrict__ lut,
                       uint32_t* __restrict__ counts, int nprobe, float* __restrict__ pscore,
-                      int32_t* __restrict__ pcell, int keys_off, uint32_t* status) {
+                      int32_t* __restrict__ pcell, int keys_off, int opb, uint32_t* status) {
   pdl_wait();  // inputs written by the kernels before this one
   pdl_launch_dependents();
-  project_bulk_block<true>(x, d, w, D, mu, out, status);  // ends on a cluster barrier
+  project_bulk_block<true>(x, d, w, D, mu, out, status, opb);  // ends on a cluster barrier
   namespace cg = cooperative_groups;
   cg::cluster_group cl = cg::this_cluster();
   extern __shared__ __align__(128) uint8_t smd[];
@@ -602,8 +606,49 @@ sense_status launch_coarse_lut(const sense_ivf* ix, const float* queries, int q,
   return cuda_check(e, "launch coarse + lut");
 }
 
-size_t project_bulk_smem(int d, bool mean);
 constexpr size_t kProjectCoarseMax = 200 * 1024;  // + ~20 KB static (<= 227 KB)
+
+using ProjectCoarseFn = void (*)(const uint16_t*, int, const float*, const float*, float*,
+                                 const float*, int64_t, const float*, int, int, float*, uint32_t*,
+                                 int, float*, int32_t*, int, int, uint32_t*);
+
+// Whether clusters of 16 blocks of `smem` bytes can run (non-portable size;
+// the occupancy query's answer is cached per device and size).
+bool cluster16_ok(ProjectCoarseFn kern, size_t smem) {
+  constexpr int kMaxDev = 64;
+  static std::mutex mu;
+  static size_t asked[kMaxDev] = {};
+  static bool answer[kMaxDev] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (asked[dev] == smem) return answer[dev];
+  bool ok = cudaFuncSetAttribute(reinterpret_cast<const void*>(kern),
+                                 cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess &&
+            func_smem(reinterpret_cast<const void*>(kern), (int)smem) == cudaSuccess;
+  if (ok) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(16, 1);
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 16;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int nclusters = 0;
+    ok = cudaOccupancyMaxActiveClusters(&nclusters, kern, &cfg) == cudaSuccess && nclusters >= 1;
+  }
+  if (!ok) (void)cudaGetLastError();  // the failed query only means "not 16"
+  asked[dev] = smem;
+  answer[dev] = ok;
+  return ok;
+}
 
 // Launches project_coarse_kernel when the row's projection blocks fit one
 // cluster and its shared memory; *done = false (nothing launched) otherwise.
@@ -613,18 +658,9 @@ sense_status launch_project_coarse(const uint16_t* x, int n, int d, const float*
                                    cudaStream_t s, bool* done) {
   *done = false;
   const int v = ix->v;
-  // the projection's shared memory is reused for the cell tiles; the row's
-  // coarse keys follow it (block 0's copy is the one used)
-  const size_t keys_off =
-      (std::max(project_bulk_smem(d, mean != nullptr), (size_t)256 * (v + 1) * 4) + 127) & ~(size_t)127;
-  const size_t smem = keys_off + (size_t)ix->nlist * 8;
   const bool vdim = v == 4 || v == 8 || v == 16 || v == 32 || v == 64;
-  if (!vdim || n > 64 || (v + 7) / 8 > 8 || smem > kProjectCoarseMax) return SENSE_OK;
-  uint32_t* status = device_status_word();
-  if (!status) return SENSE_ERR_OOM;
-  void (*kern)(const uint16_t*, int, const float*, const float*, float*, const float*, int64_t,
-               const float*, int, int, float*, uint32_t*, int, float*, int32_t*, int,
-               uint32_t*) = nullptr;
+  if (!vdim || n > 64) return SENSE_OK;
+  ProjectCoarseFn kern = nullptr;
   switch (v) {
     case 4: kern = project_coarse_kernel<4>; break;
     case 8: kern = project_coarse_kernel<8>; break;
@@ -632,10 +668,29 @@ sense_status launch_project_coarse(const uint16_t* x, int n, int d, const float*
     case 32: kern = project_coarse_kernel<32>; break;
     default: kern = project_coarse_kernel<64>; break;
   }
+  // the projection's shared memory is reused for the cell tiles; the row's
+  // coarse keys follow it (block 0's copy is the one used).  Four outputs
+  // per block (16 blocks at v = 64: half the W rows per block and one cell
+  // tile each) when a cluster of that size can run, else eight.
+  size_t keys_off = 0, smem = 0;
+  int opb = 4;
+  auto size_for = [&](int ob) {
+    keys_off = (std::max(project_bulk_smem(d, mean != nullptr, ob), (size_t)256 * (v + 1) * 4) + 127) &
+               ~(size_t)127;
+    smem = keys_off + (size_t)ix->nlist * 8;
+  };
+  size_for(opb);
+  if ((v + opb - 1) / opb > 8 && (smem > kProjectCoarseMax || !cluster16_ok(kern, smem))) {
+    opb = 8;
+    size_for(opb);
+  }
+  if (smem > kProjectCoarseMax) return SENSE_OK;
+  uint32_t* status = device_status_word();
+  if (!status) return SENSE_ERR_OOM;
   sense_status st = cuda_check(func_smem(reinterpret_cast<const void*>(kern), (int)smem),
                                "cudaFuncSetAttribute(project_coarse)");
   if (st != SENSE_OK) return st;
-  const int groups = (v + 7) / 8;
+  const int groups = (v + opb - 1) / opb;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)groups, (unsigned)n);
   cfg.blockDim = dim3(256);
@@ -654,7 +709,7 @@ sense_status launch_project_coarse(const uint16_t* x, int n, int d, const float*
   st = cuda_check(cudaLaunchKernelEx(&cfg, kern, x, d, basis, mean, out,
                                      (const float*)ix->centroids, (int64_t)ix->nlist,
                                      (const float*)ix->codebooks, ix->pq_m, ix->dsub, lut, counts,
-                                     nprobe, pscore, pcell, (int)keys_off, status),
+                                     nprobe, pscore, pcell, (int)keys_off, opb, status),
                   "launch project + coarse");
   if (st == SENSE_OK) *done = true;
   return st;
