@@ -104,7 +104,7 @@ __device__ bool radix_select(Get get, int64_t cnt, int k, int low, unsigned* his
 
 // Short path of merge_kernel for a pool of distinct nonzero keys (at most
 // 32 * kPoolGroups of them).  The pool is cut into
-// groups of 32; a group's maximum is a head, and the k-th largest head T
+// groups of at most 32; a group's maximum is a head, and the k-th largest head T
 // bounds the k-th largest key from below (k groups hold a key >= T).  Heads
 // are ranked against warp-sorted groups of heads by binary search; the keys
 // >= T (a few dozen for a random pool) are then placed by their rank among
@@ -114,17 +114,14 @@ constexpr int kPoolGroups = 1024;  // heads ranked by the short path
 constexpr int kPoolCand = 512;     // candidates placed by rank (in `sel`), O(c^2 / threads)
 constexpr int kPoolAll = 256;      // pools this small are ranked whole
 
-__device__ __forceinline__ uint64_t warp_max64(uint64_t x) {
-  // distinct keys: the largest high word, then the largest low word under it
-  const uint32_t hi = (uint32_t)(x >> 32);
-  const uint32_t hm = __reduce_max_sync(0xffffffffu, hi);
-  const uint32_t lm = __reduce_max_sync(0xffffffffu, hi == hm ? (uint32_t)x : 0u);
-  return ((uint64_t)hm << 32) | lm;
-}
-
-// The keys are read where they are, in the pool (L2 loads, four per thread
+// The keys are read where they are, in the pool (L2 loads, eight per thread
 // in flight; a fused caller writes the pool earlier in the same launch):
 // both passes over them are coalesced, so no staging copy is needed.
+// Group g of the ngr = ceil(cnt / 32) groups holds the keys g, g + ngr,
+// g + 2 ngr, ... (at most 32); its head (maximum) is formed by a team of
+// adjacent lanes in registers.  Any partition into groups gives the same
+// guarantee: the k-th largest head T has k distinct keys at or above it,
+// so every key of the top k is >= T and is collected.
 template <bool SMEM = false>  // SMEM: the keys are in shared memory
 __device__ bool merge_pool_short(const uint64_t* __restrict__ keys, int cnt, int k, int pad_short,
                                  uint64_t* cand, float* __restrict__ out_scores,
@@ -143,24 +140,33 @@ __device__ bool merge_pool_short(const uint64_t* __restrict__ keys, int cnt, int
     s_t = 0ull;
     s_got = 0u;
   }
-  // heads: group maxima (every warp takes groups in turn), then sorted
-  // descending within each group of 32 heads; groups past the pool are 0
+  // heads: a team of `team` adjacent lanes (a power of two, as many as the
+  // block has threads per group) forms each group's maximum, lane `sub` of
+  // the team taking keys sub, sub + team, ... of the group; then the heads
+  // are sorted descending within each group of 32 heads; past the pool 0
   const int nhg = (ngr + 31) >> 5;
-  for (int g0 = warp; g0 < ngr; g0 += 4 * nwarps) {
-    uint64_t x[4];
+  int team = 1;
+  while (team < 32 && 2 * team * ngr <= (int)blockDim.x) team <<= 1;
+  for (int s0 = 0; s0 < ngr * team; s0 += blockDim.x) {  // block-uniform trip count
+    const int sl = s0 + threadIdx.x;
+    const int g = sl / team, sub = sl - g * team;
+    uint64_t m = 0ull;
+    for (int j0 = sub; j0 < 32; j0 += 8 * team) {
+      uint64_t x[8];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int i = (g0 + u * nwarps) * 32 + lane;
-      x[u] = i < cnt ? key_at(i) : 0ull;
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int g = g0 + u * nwarps;  // warp-uniform
-      if (g < ngr) {
-        const uint64_t m = warp_max64(x[u]);
-        if (lane == 0) s_heads[g] = m;
+      for (int u = 0; u < 8; ++u) {
+        const int j = j0 + u * team;
+        const int i = g + j * ngr;
+        x[u] = (g < ngr && j < 32 && i < cnt) ? key_at(i) : 0ull;
       }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) m = x[u] > m ? x[u] : m;
     }
+    for (int off = team >> 1; off > 0; off >>= 1) {
+      const uint64_t o = __shfl_xor_sync(0xffffffffu, m, off);
+      m = o > m ? o : m;
+    }
+    if (sub == 0 && g < ngr) s_heads[g] = m;
   }
   for (int g = ngr + threadIdx.x; g < nhg * 32; g += blockDim.x) s_heads[g] = 0ull;
   __syncthreads();
@@ -194,20 +200,36 @@ __device__ bool merge_pool_short(const uint64_t* __restrict__ keys, int cnt, int
     if (rank == k - 1) s_t = h;
   }
   __syncthreads();
+  // every key >= T, appended with one shared atomic per warp and load batch
   const uint64_t t = s_t;
-  for (int i0 = threadIdx.x; i0 < cnt; i0 += 4 * blockDim.x) {
-    uint64_t x[4];
+  for (int b0 = 0; b0 < cnt; b0 += 8 * (int)blockDim.x) {  // block-uniform trip count
+    uint64_t x[8];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int i = i0 + u * blockDim.x;
+    for (int u = 0; u < 8; ++u) {
+      const int i = b0 + u * (int)blockDim.x + (int)threadIdx.x;
       x[u] = i < cnt ? key_at(i) : 0ull;
     }
+    unsigned take = 0u;  // bit u: x[u] is a candidate
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const uint64_t c = x[u];
-      if (c != 0ull && c >= t) {
-        const unsigned p = atomicAdd(&s_got, 1u);
-        if (p < (unsigned)kPoolCand) cand[p] = c;
+    for (int u = 0; u < 8; ++u)
+      if (x[u] != 0ull && x[u] >= t) take |= 1u << u;
+    const unsigned mine = (unsigned)__popc(take);
+    unsigned incl = mine;  // inclusive prefix of the lanes' counts
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const unsigned o = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += o;
+    }
+    const unsigned total = __shfl_sync(0xffffffffu, incl, 31);
+    if (total == 0u) continue;  // warp-uniform
+    unsigned base = 0u;
+    if (lane == 31) base = atomicAdd(&s_got, total);
+    base = __shfl_sync(0xffffffffu, base, 31) + incl - mine;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if ((take >> u) & 1u) {
+        if (base < (unsigned)kPoolCand) cand[base] = x[u];
+        ++base;
       }
     }
   }
