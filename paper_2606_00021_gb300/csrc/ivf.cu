@@ -114,7 +114,11 @@ constexpr long long kBulkWaitCycles = 4000000000LL;
 // project_rows_kernel (lane l: its 4-column groups ascending; butterfly).
 // NORM: the blocks of a row are one cluster (gridDim.x <= 16); block 0
 // gathers the v outputs through distributed shared memory and writes the
-// row divided by its L2 norm, in the order of normalize_rows_kernel.  A
+// row divided by its L2 norm, in the order of normalize_rows_kernel.  With
+// s_row (a fused caller) every block does the same into its own s_row[v]
+// (block 0 still writes the row) and the function returns without the
+// closing cluster barrier: the caller must pass one before it exits, since
+// other blocks read this block's outputs.  A
 // copy that never lands (bounded wait) sets SENSE_DEVST_TIMEOUT; the row is
 // then left unwritten.
 template <bool NORM>
@@ -122,7 +126,7 @@ __device__ __forceinline__ void project_bulk_block(const uint16_t* __restrict__ 
                                                    const float* __restrict__ w, int v,
                                                    const float* __restrict__ mu,
                                                    float* __restrict__ out, uint32_t* status,
-                                                   int opb = 8) {
+                                                   int opb = 8, float* s_row = nullptr) {
   extern __shared__ __align__(128) uint8_t smb[];
   __shared__ __align__(8) uint64_t bar;
   __shared__ float s_out[8];
@@ -185,7 +189,7 @@ __device__ __forceinline__ void project_bulk_block(const uint16_t* __restrict__ 
     cg::cluster_group cl = cg::this_cluster();
     if (lane == 0) s_out[wid] = acc;
     cl.sync();  // every block's outputs and failure flag are written
-    if (blockIdx.x == 0 && wid == 0) {
+    if ((s_row || blockIdx.x == 0) && wid == 0) {
       bool any_fail = false;
       for (unsigned r = 0; r < gridDim.x; ++r) any_fail |= *cl.map_shared_rank(&s_fail, r) != 0;
       if (!any_fail) {
@@ -205,10 +209,20 @@ __device__ __forceinline__ void project_bulk_block(const uint16_t* __restrict__ 
         }
         const float nrm = __fsqrt_rn(ss);
 #pragma unroll
-        for (int t = 0; t < 4; ++t)
-          if (32 * t + lane < v)
-            out[row * v + 32 * t + lane] = nrm > 0.0f ? __fdiv_rn(part[t], nrm) : 0.0f;
+        for (int t = 0; t < 4; ++t) {
+          if (32 * t + lane < v) {
+            const float y = nrm > 0.0f ? __fdiv_rn(part[t], nrm) : 0.0f;
+            if (blockIdx.x == 0) out[row * v + 32 * t + lane] = y;
+            if (s_row) s_row[32 * t + lane] = y;
+          }
+        }
+      } else if (s_row) {
+        for (int t = lane; t < v; t += 32) s_row[t] = 0.0f;
       }
+    }
+    if (s_row) {
+      __syncthreads();  // s_row is complete
+      return;
     }
     cl.sync();  // the other blocks' shared memory stays alive until it is read
   }
@@ -510,16 +524,15 @@ project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __rest
                       int32_t* __restrict__ pcell, int keys_off, int opb, uint32_t* status) {
   pdl_wait();  // inputs written by the kernels before this one
   pdl_launch_dependents();
-  project_bulk_block<true>(x, d, w, D, mu, out, status, opb);  // ends on a cluster barrier
+  __shared__ float sqr[D];  // the normalised row, formed by every block
+  // the closing cluster barrier is the one before the cell selection below
+  project_bulk_block<true>(x, d, w, D, mu, out, status, opb, sqr);
   namespace cg = cooperative_groups;
   cg::cluster_group cl = cg::this_cluster();
   extern __shared__ __align__(128) uint8_t smd[];
   const int64_t row = blockIdx.y;
   if (blockIdx.x == 0 && threadIdx.x == 0) counts[row] = 0u;  // the list scan's pool is empty
-  const float* qrow = out + row * D;
   const int C = (int)gridDim.x, r = (int)blockIdx.x;
-  __shared__ float sqr[D];  // the normalised row
-  for (int j = threadIdx.x; j < D; j += blockDim.x) sqr[j] = qrow[j];
   // coarse keys: tiles of 256 cells staged in shared memory by coalesced
   // loads (row stride D + 1: conflict-free reads), each thread one cell's
   // in-order dot product (the ALL_IP arithmetic), the key stored straight
@@ -565,7 +578,7 @@ project_coarse_kernel(const uint16_t* __restrict__ x, int d, const float* __rest
   __shared__ float sq[128];
   for (int m = r; m < pq_m; m += C) {
     __syncthreads();
-    for (int j = threadIdx.x; j < dsub; j += blockDim.x) sq[j] = qrow[m * dsub + j];
+    for (int j = threadIdx.x; j < dsub; j += blockDim.x) sq[j] = sqr[m * dsub + j];
     __syncthreads();
     for (int cw = threadIdx.x; cw < 256; cw += blockDim.x) {
       const int e = m * 256 + cw;
