@@ -369,9 +369,12 @@ __device__ void merge_pool_block(const uint64_t* __restrict__ pool,
   int64_t cnt = (counts && !in_smem) ? (int64_t)counts[q] : pool_cap;  // else every slot is used
   if (cnt > pool_cap) cnt = pool_cap;
   // the short path (pool read where it is) needs a pruning threshold (k
-  // group heads) or a tiny pool
-  const bool short_ok =
-      cnt > 0 && cnt <= 32 * kPoolGroups && (cnt <= kPoolAll || (cnt + 31) / 32 >= (int64_t)k);
+  // group heads) or a tiny pool; past k = 128 it also wants 4 k groups, or
+  // the keys above the k-th head overflow its kPoolCand candidates (a
+  // 256-key shortlist of a 9,400-key pool did, every time)
+  const int64_t ngr = (cnt + 31) / 32;
+  const bool short_ok = cnt > 0 && cnt <= 32 * kPoolGroups &&
+                        (cnt <= kPoolAll || (ngr >= (int64_t)k && (k <= 128 || ngr >= 4 * (int64_t)k)));
   if (short_ok &&
       (in_smem ? merge_pool_short<true>(src, (int)cnt, k, pad_short, sel, out_scores + (int64_t)q * k,
                                         out_idx + (int64_t)q * k)
