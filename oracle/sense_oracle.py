@@ -175,8 +175,8 @@ def gather_drafts(spans: np.ndarray, idx: np.ndarray, anchor=None,
     (anchor match first, then retrieval rank, which is the similarity
     order), i.e. a stable partition of the retrieved list; the first n_keep
     rows are kept.  With ``force_anchor`` the first token of the first kept
-    row and of the last kept row are set to x~ (Alg. 2, "D[0,0] <- x~" and
-    "D[-1,0] <- x~").
+    row and of the last kept row are set to x~ (Alg. 2 forces the anchor
+    into the first token of the first and of the last candidate).
     """
     spans = np.asarray(spans)
     idx = np.atleast_2d(np.asarray(idx, dtype=np.int64))
