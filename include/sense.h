@@ -89,14 +89,18 @@ typedef enum sense_status {
 #define SENSE_MAX_WINDOW 64       /* gate lookahead window                    */
 #define SENSE_MAX_PROJ_DIM 128    /* projected key dimension                  */
 
+/* Library version, and the name of a status code (the paper has no
+ * counterpart; these describe the library itself). */
 int32_t sense_version(void);
 const char* sense_status_string(sense_status s);
-/* Message of the last error raised on the calling thread ("" if none). */
+/* Message of the last error raised on the calling thread ("" if none; the
+ * paper has no counterpart). */
 const char* sense_last_error(void);
 
 /*
- * Reads the status word of the current device, after synchronising
- * `stream`; if `clear` is non-zero the word is reset to 0 afterwards.
+ * Device-side failure reporting (the paper has no counterpart): reads the
+ * status word of the current device, after synchronising `stream`; if
+ * `clear` is non-zero the word is reset to 0 afterwards.
  * Returns SENSE_ERR_DEVICE_STATUS when any bit is set, else SENSE_OK.
  */
 sense_status sense_device_status(sense_stream_t stream, uint32_t* out_bits, int32_t clear);
@@ -155,8 +159,9 @@ sense_status sense_retrieve_topk(const sense_datastore* ds, const uint16_t* quer
                                  void* workspace, size_t workspace_bytes, sense_stream_t stream);
 
 /*
- * Same search as sense_retrieve_topk, for callers that cannot allocate
- * device memory and have no workspace to pass: for example a serving
+ * Sec. 3.2.2 Eq. 7's exact top-k, the same search as sense_retrieve_topk,
+ * for callers that cannot allocate device memory and have no workspace to
+ * pass: for example a serving
  * process whose device memory is all handed out in advance by another
  * allocator, or a plug-in whose host application exposes no device
  * allocator and forbids cudaMalloc (it can synchronise the device and fail
@@ -226,6 +231,7 @@ sense_status sense_retrieve_noalloc_selftest(sense_stream_t stream, int64_t limi
  */
 
 /*
+ * The key / query construction k = L2Norm(PCA(h)) of Alg. 2 and App. E:
  * y = (x - mean) W^T for bf16 rows x [n, d] and a basis W [v, d] f32 (rows =
  * principal axes); mean [d] f32 or NULL.  With SENSE_PROJECT_NORMALIZE each
  * row is then divided by its L2 norm (zero rows stay zero).  out [n, v] f32.
@@ -239,8 +245,8 @@ sense_status sense_project(const uint16_t* x, int64_t n, int32_t d, const float*
                            const float* mean, uint32_t flags, float* out, sense_stream_t stream);
 
 /*
- * Lloyd's k-means (training of the coarse quantizer and of the PQ
- * codebooks): `iters` rounds of assignment (SENSE_KMEANS_SPHERICAL: largest
+ * Lloyd's k-means, the training of App. E's IVF-PQ index (its coarse
+ * quantizer and its PQ codebooks, which the paper's FAISS trains): `iters` rounds of assignment (SENSE_KMEANS_SPHERICAL: largest
  * inner product, else smallest squared L2 distance; ties to the lowest
  * centroid) and update (member means accumulated as 2^-31 fixed-point
  * integers, divided in fp64, rounded to fp32; an empty cluster keeps its
@@ -258,8 +264,9 @@ sense_status sense_kmeans(const float* x, int64_t n, int32_t dim, int32_t ld, in
                           sense_stream_t stream);
 
 /*
- * Cell of each vector (largest inner product with a centroid, ties to the
- * lowest cell) and its residual r = x - c_cell, for training PQ codebooks.
+ * App. E's IVF-PQ encodes residuals: cell of each vector (largest inner
+ * product with a centroid, ties to the lowest cell) and its residual
+ * r = x - c_cell, for training PQ codebooks.
  * vecs [n, v] f32, centroids [nlist, v]; out_cell [n] int32,
  * out_residuals [n, v] f32.  v in {16, 32, 64, 128}, nlist <= 16384.
  */
@@ -268,8 +275,10 @@ sense_status sense_ivf_residuals(const float* vecs, int64_t n, int32_t v, const 
                                  sense_stream_t stream);
 
 /*
- * Builds an inverted-file index over unit vectors vecs [n, v] f32 (copied;
- * the index owns its memory, allocated here, freed by sense_ivf_destroy).
+ * The index of Sec. 3.2.2 Eq. 7's ANN search as App. E sets it up (IVF or
+ * IVF-PQ over L2-normalised PCA keys): builds an inverted-file index over
+ * unit vectors vecs [n, v] f32 (copied; the index owns its memory,
+ * allocated here, freed by sense_ivf_destroy).
  *  - cell of x = arg max_c <x, c> over centroids [nlist, v] (unit centroids:
  *    the nearest one);
  *  - lists in cell order, members in ascending key index;
@@ -286,7 +295,8 @@ sense_status sense_ivf_build(const float* vecs, int64_t n, int32_t v, const floa
 sense_status sense_ivf_destroy(sense_ivf* ix);
 
 /*
- * Read-only view of an index: out_info [5] = {n, v, nlist, pq_m, longest
+ * Read-only view of an index (inspection; the paper has no counterpart):
+ * out_info [5] = {n, v, nlist, pq_m, longest
  * list}; device pointers to the list offsets [nlist + 1] int64, the key
  * index of each slot [n] int32 and the payload (flat: vectors [n, v] f32;
  * PQ: codes [n, pq_m] uint8), in list order.  Any output may be NULL.
@@ -295,7 +305,8 @@ sense_status sense_ivf_arrays(const sense_ivf* ix, int64_t* out_info, const int6
                               const int32_t** out_ids, const void** out_payload);
 
 /*
- * Top-k of the approximate scores over the nprobe best cells, per query:
+ * Sec. 3.2.2 Eq. 7's ANN(k_t, C_db, N') with App. E's nprobe: top-k of the
+ * approximate scores over the nprobe best cells, per query:
  *  - coarse score <q, c> for every cell; the nprobe largest are probed
  *    (ties to the lower cell); out_probes [q, nprobe] int32 or NULL;
  *  - IVF-flat: score = <q, x>; IVF-PQ: score = <q, c_cell> +
@@ -424,12 +435,14 @@ sense_status sense_gather_drafts(const sense_datastore* ds, const int32_t* idx, 
  * (ties to the older position).
  */
 
-/* Creates an empty buffer (allocates capacity * (2 d + 4) bytes on the
+/* The dynamic context buffer C_d of Sec. 3.2.1 (Eq. 6) and Alg. 1:
+ * creates an empty buffer (allocates capacity * (2 d + 4) bytes on the
  * current device).  Limits: 1 <= m <= SENSE_MAX_M, m <= capacity <= 2^24,
  * d % 8 == 0. */
 sense_status sense_ctx_create(int32_t capacity, int32_t d, int32_t m, sense_ctx** out);
 sense_status sense_ctx_destroy(sense_ctx* ctx);
-/* The buffer's position counter lives on the device, so that appends whose
+/* C_d's bookkeeping (Alg. 1 appends to it; the paper gives no reset or
+ * count).  The buffer's position counter lives on the device, so that appends whose
  * length is only known there (sense_ctx_append_path) need no host round
  * trip.  sense_ctx_reset forgets every entry (asynchronous on `stream`);
  * sense_ctx_count synchronises `stream` and reads the number of positions
@@ -464,7 +477,8 @@ sense_status sense_ctx_append_path(sense_ctx* ctx, const uint16_t* root_hidden,
                                    sense_stream_t stream);
 
 /*
- * DynSearch: per query (queries [q, d] bf16, 16-byte aligned), the k
+ * Alg. 2's DynSearch over C_d (with the boost delta of its scores): per
+ * query (queries [q, d] bf16, 16-byte aligned), the k
  * searchable entries with the largest <q, key> (fp32 accumulation), order
  * (score desc, position asc).  out_scores [q, k] f32 = score + delta;
  * out_pos [q, k] int64 positions; out_spans [q, k, m] int32.  Slots past the
@@ -716,21 +730,25 @@ sense_status sense_selftest_timeout(sense_stream_t stream, int64_t limit_cycles)
 /* Launch profiling                                                         */
 /* ---------------------------------------------------------------------- */
 /*
- * When enabled, every kernel launch of the library is bracketed by two CUDA
- * events recorded on the launching stream.  sense_profile_enable(1) clears
+ * Instrumentation (the paper has no counterpart).  When enabled, every
+ * kernel launch of the library is bracketed by two CUDA events recorded on
+ * the launching stream.  sense_profile_enable(1) clears
  * earlier records.  sense_profile_query synchronises on the recorded events
  * and returns, for the kernel family `name` (see sense_profile_name), the
  * summed device time in milliseconds and the number of launches.
  */
 sense_status sense_profile_enable(int32_t on);
 /*
- * Restricts the bracketing to the comma-separated kernel families in
+ * Instrumentation, continued (no counterpart in the paper).  Restricts the
+ * bracketing to the comma-separated kernel families in
  * `names` (NULL or "" = every family) until the next sense_profile_enable,
  * which selects every family again.  Each bracketed launch adds two event
  * records to its stream; filtering keeps them off the launches that are not
  * being measured.  SENSE_ERR_INVALID_ARG for an unknown family name.
  */
 sense_status sense_profile_filter(const char* names);
+/* The kernel families (count, i-th name) and the summed time of one family
+ * (instrumentation; no counterpart in the paper). */
 int32_t sense_profile_count(void);
 const char* sense_profile_name(int32_t i);
 sense_status sense_profile_query(const char* name, double* total_ms, int64_t* launches);

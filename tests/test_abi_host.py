@@ -32,6 +32,23 @@ def test_every_declared_symbol_is_exported(lib):
     assert set(names) == set(_abi.SIGNATURES), "binding and header disagree"
 
 
+def test_every_declaration_cites_its_passage():
+    """Each entry point of the header is documented by the comment before it
+    (shared by a run of declarations): the paper's section, equation,
+    algorithm or appendix it implements, or that the paper has none."""
+    src = open(os.path.join(ROOT, "include", "sense.h")).read()
+    decl = re.compile(r"\n(?:sense_status|size_t|const char\*|int32_t|int|void)\s+(sense_\w+)\s*\(")
+    cite = re.compile(r"Sec\.|Eq\.|Alg\.|App\.|no\s+(?:\*\s+)?counterpart", re.S)
+    found = 0
+    for m in decl.finditer(src):
+        before = src[:m.start()]
+        end = before.rfind("*/")
+        start = before.rfind("/*", 0, end)
+        assert end > 0 and cite.search(before[start:end]), m.group(1)
+        found += 1
+    assert found >= 40
+
+
 def test_status_strings(lib):
     assert lib.sense_status_string(0) == b"SENSE_OK"
     assert lib.sense_status_string(1) == b"SENSE_ERR_INVALID_ARG"
